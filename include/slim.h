@@ -1,0 +1,170 @@
+/*
+ * libslim -- sliced causal linear (Performer) attention, forward and backward,
+ * on one NVIDIA GB300 (sm_103a).
+ *
+ * The operation is the causal linear self-attention of eq. 2 of "Sub-Linear
+ * Memory: How to Make Performers SLiM" (arXiv 2012.11346), for B*H
+ * independent chains (batch x head):
+ *
+ *     out_i = sum_{j<=i} (g(q_i).g(k_j)) v_j  /  sum_{j<=i} g(q_i).g(k_j)
+ *
+ * evaluated the way Algorithm 1 prescribes: the sequence is cut into
+ * N = ceil(L/C) slices of C rows (Sec. 3.2, the last slice may be shorter),
+ * and only the prefix state B^(n) = (S, z) is carried from slice to slice:
+ *
+ *     S = sum_j g(k_j) v_j^T   ([M, d], the transpose of the paper's R, eq. 3)
+ *     z = sum_j g(k_j)         ([M],    the paper's S, eq. 3)
+ *
+ * The backward pass walks the slices in reverse (Sec. 3.3): it recomputes
+ * each slice, rolls the state back by subtraction (eq. 17) and carries the
+ * state gradient G^(n) (eq. 18).  Memory beyond inputs and outputs is the
+ * caller-provided workspace, whose size grows with C, not with L.
+ *
+ * Feature maps g: R^d -> R_+^M (Omega is [M, d], shared by all chains):
+ *     SLIM_FEAT_EXP  : g(x)_m = exp(omega_m.x - |x|^2/2) / sqrt(M)   (FAVOR+)
+ *     SLIM_FEAT_RELU : g(x)_m = max(omega_m.x, 0) / sqrt(M), ReLU'(0) = 0
+ * A row whose denominator is exactly 0 (possible only with the ReLU map)
+ * gets output 0 and passes no gradient.
+ *
+ * Conventions for every entry point
+ *   - All tensor pointers are DEVICE pointers, contiguous, row-major, 16-byte
+ *     aligned.  q, k, v, out, dout, dq, dk, dv are [B, H, L, d] in `dtype`;
+ *     omega and domega are [M, d] fp32; S_state is [B, H, M, d] fp32 and
+ *     z_state is [B, H, M] fp32.
+ *   - The caller owns every buffer.  The library allocates no device or host
+ *     memory and never synchronises the device; all work is enqueued on
+ *     `stream` (a cudaStream_t passed as void*; NULL is the legacy default
+ *     stream).  Inputs must not be modified until that work completes.
+ *   - Arguments are validated before anything is enqueued.  On any error
+ *     nothing has been launched, except SLIM_ERR_CUDA (a launch failed part
+ *     way; outputs are then undefined).
+ *   - 1 <= C; C > L behaves as C = L.  L % C != 0 gives a shorter last slice.
+ *   - Outputs are written in `dtype` rounded to nearest even; accumulation and
+ *     the carried state are fp32 (the state as an fp32 value/error pair).
+ *   - Supported: d in {16, 32, 64, 128}; M a multiple of 16 in [16, 256];
+ *     dtype SLIM_F32 or SLIM_BF16; both feature maps.  Other combinations
+ *     return SLIM_ERR_UNSUPPORTED.
+ */
+#ifndef SLIM_H_
+#define SLIM_H_
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SLIM_OK = 0,
+  SLIM_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad size, C < 1 ... */
+  SLIM_ERR_UNSUPPORTED = 2,   /* valid but unsupported (d, M, dtype, feature) */
+  SLIM_ERR_WORKSPACE = 3,     /* workspace pointer null or too small          */
+  SLIM_ERR_CUDA = 4,          /* a CUDA launch or runtime call failed          */
+  SLIM_ERR_TIMEOUT = 5        /* a bounded device-side wait gave up            */
+} slim_status;
+
+typedef enum { SLIM_F32 = 0, SLIM_BF16 = 1 } slim_dtype;
+typedef enum { SLIM_FEAT_EXP = 0, SLIM_FEAT_RELU = 1 } slim_feature;
+
+/* Human-readable name of a status code (static storage, never NULL). */
+const char* slim_status_string(slim_status status);
+
+/* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
+int slim_version(void);
+
+/*
+ * Workspace bytes needed by slim_fwd / slim_bwd for this problem.  Pure host
+ * computation (no CUDA call).  The size grows linearly with min(C, L) and with
+ * B*H, and does not depend on L otherwise (Sec. 3.4: O(C) memory).
+ * Returns SLIM_ERR_INVALID_ARG / SLIM_ERR_UNSUPPORTED as the entry points
+ * would; *bytes is written only on SLIM_OK.
+ */
+slim_status slim_fwd_workspace_size(int B, int H, int L, int d, int M, int C,
+                                    slim_dtype dtype, slim_feature feature,
+                                    size_t* bytes);
+slim_status slim_bwd_workspace_size(int B, int H, int L, int d, int M, int C,
+                                    slim_dtype dtype, slim_feature feature,
+                                    size_t* bytes);
+
+/*
+ * Forward sweep of Algorithm 1 (Sec. 3.2, eqs. 14-16) for one causal
+ * linear-attention layer.
+ *   q, k, v   [B,H,L,d] dtype, read-only.
+ *   omega     [M,d] fp32, read-only; the random-feature matrix of g.
+ *   out       [B,H,L,d] dtype, written: eq. 2 for every row.
+ *   S_state   [B,H,M,d] fp32, written: final state S^(N) = sum_j g(k_j) v_j^T.
+ *   z_state   [B,H,M]   fp32, written: final state z^(N) = sum_j g(k_j).
+ *   workspace device scratch of at least slim_fwd_workspace_size() bytes,
+ *             256-byte aligned; contents on entry are ignored.
+ * L = 0 is valid and only zeroes S_state / z_state.
+ */
+slim_status slim_fwd(const void* q, const void* k, const void* v, const float* omega,
+                     int B, int H, int L, int d, int M, int C,
+                     slim_dtype dtype, slim_feature feature,
+                     void* out, float* S_state, float* z_state,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Backward sweep of Algorithm 1 (Sec. 3.3, eqs. 17-18): the vector-Jacobian
+ * product of eq. 2 for the upstream gradient dout, i.e. the gradients of
+ * <dout, out> with respect to q, k, v and omega.
+ *   q, k, v, omega  as for slim_fwd, read-only.
+ *   out        [B,H,L,d] dtype, read-only: the output slim_fwd returned.
+ *   dout       [B,H,L,d] dtype, read-only: upstream gradient.
+ *   S_state, z_state  read-only: the final state B^(N) slim_fwd returned; the
+ *              reverse walk starts from it and rolls it back slice by slice.
+ *              Not modified, so a second call gives the same result.
+ *   dq, dk, dv [B,H,L,d] dtype, written.
+ *   domega     [M,d] fp32, written (sum over all chains, queries and keys).
+ *   workspace  at least slim_bwd_workspace_size() bytes, 256-byte aligned.
+ * The same C as the forward is expected; any C gives the same result in exact
+ * arithmetic (Sec. 4.2), differing only by rounding.
+ */
+slim_status slim_bwd(const void* q, const void* k, const void* v, const float* omega,
+                     const void* out, const void* dout,
+                     const float* S_state, const float* z_state,
+                     int B, int H, int L, int d, int M, int C,
+                     slim_dtype dtype, slim_feature feature,
+                     void* dq, void* dk, void* dv, float* domega,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Reads the device error word that bounded waits in the kernels set when they
+ * give up, and clears it.  Copies 4 bytes from the workspace on `stream` and
+ * synchronises that stream (this call, unlike the others, blocks).
+ * Returns SLIM_OK, SLIM_ERR_TIMEOUT, or SLIM_ERR_CUDA.
+ */
+slim_status slim_check_device_error(void* workspace, void* stream);
+
+/*
+ * Launch accounting and per-kernel timing (a host-side runtime feature for
+ * benchmarking; no counterpart in the paper).  Process-global, not
+ * thread-safe.
+ *
+ * slim_launch_count: number of libslim kernel launches since load.
+ * slim_profiler_enable(1): from now on every libslim kernel launch is
+ *   bracketed by two CUDA events recorded on its stream; each launch site also
+ *   tallies the algorithmic FLOPs and HBM bytes of the launch.
+ * slim_profiler_read: waits for the recorded events, folds them into
+ *   per-kernel totals and writes up to `cap` entries (one per kernel that ran);
+ *   returns the number of entries, or -1 on a CUDA error.
+ * slim_profiler_reset: drops all records and totals.
+ */
+typedef struct {
+  char name[48];
+  unsigned long long launches;
+  double total_ms;  /* summed CUDA-event durations of the recorded launches */
+  double flops;     /* algorithmic floating-point operations of those launches */
+  double bytes;     /* algorithmic HBM bytes (reads + writes) of those launches */
+} slim_kernel_stats;
+
+unsigned long long slim_launch_count(void);
+void slim_profiler_enable(int on);
+void slim_profiler_reset(void);
+int slim_profiler_read(slim_kernel_stats* stats, int cap);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif  /* SLIM_H_ */

@@ -1,0 +1,680 @@
+// fp32-compute (SIMT) path of libslim: every supported (d, M, dtype, feature).
+//
+// One slice of Algorithm 1 at a time.  Inside a slice the rows are cut into
+// tiles of T rows and every step is a small batched contraction over
+// (chain, tile) -- App. B's "block" evaluation with the block's prefix sums
+// written as masked matrix products:
+//
+//   forward, slice n (Sec. 3.2, eqs. 14-16):
+//     phiQ, phiK = g(Q), g(K)                    (F, row-wise)
+//     Delta_t    = phiK_t^T [V_t | 1]            (the tile's sum of T_l)
+//     P_t        = B + sum_{t'<t} Delta_t'       (state before tile t)
+//     A_t        = tril(phiQ_t phiK_t^T)         (inclusive causal mask)
+//     [num|den]  = phiQ_t P_t + A_t [V_t | 1];  out = num / den   (eq. 4)
+//     B         += sum_t Delta_t
+//   backward, slice n (Sec. 3.3, eqs. 17-18), from B^(n), G^(n):
+//     B -= sum_t Delta_t                          (eq. 17), then P_t as above
+//     dnum = dout/den, dden = -<dout, out>/den,  W = [dnum | dden]
+//     dA_t   = tril(W_t [V_t | 1]^T)
+//     dphiQ  = W_t P_t^T + dA_t phiK_t
+//     Gd_t   = phiQ_t^T W_t;   G_t = G + sum_{t'>t} Gd_t'   (reversed prefix sum)
+//     dphiK  = dA_t^T phiQ_t + [V_t | 1] G_t^T
+//     dV     = A_t^T dnum + phiK_t G_t(S part)
+//     G     += sum_t Gd_t                           (eq. 18)
+//     feature VJP: dq, dk; dOmega += u^T x
+// The state B and its gradient G are carried as fp32 value/error pairs so the
+// rollback returns the forward's state to within the pair's precision.
+#include <math.h>
+
+#include "common.cuh"
+#include "profiler.h"
+#include "simt_path.h"
+
+namespace slim {
+namespace simt {
+
+constexpr int GT = 64;  // output tile of the contraction kernel
+constexpr int GK = 16;  // reduction chunk
+
+struct Mat {
+  const float* p;
+  long long b0, b1;  // batch strides (batch z = z0 * nb1 + z1)
+  long long rs, cs;  // element (i, k) at p + i*rs + k*cs
+};
+struct OutMat {
+  float* p;
+  long long b0, b1, rs, cs;
+};
+
+struct GemmP {
+  int m, n, k;
+  Mat a, b;
+  OutMat c;
+  int nb1;
+  int zoff;      // first batch index of this launch
+  float beta;    // C = A B + beta * C
+  int causal;    // C(i, j) = 0 for j > i
+  // optional epilogue C(i, j) -= X(i, j) * s(i)
+  const float* sx;
+  long long sx_b0, sx_rs;
+  const float* ss;
+  long long ss_b0;
+};
+
+// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z.  256 threads,
+// 64 x 64 outputs per CTA, 4 x 4 per thread, fp32 FMA.
+__global__ void __launch_bounds__(256) k_gemm(GemmP P) {
+  __shared__ __align__(16) float As[GK][GT + 4];
+  __shared__ __align__(16) float Bs[GK][GT + 4];
+  const int z = blockIdx.z + P.zoff;
+  const int z0 = z / P.nb1, z1 = z % P.nb1;
+  const float* A = P.a.p + z0 * P.a.b0 + z1 * P.a.b1;
+  const float* Bm = P.b.p + z0 * P.b.b0 + z1 * P.b.b1;
+  const int i0 = blockIdx.y * GT, j0 = blockIdx.x * GT;
+  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  float acc[4][4];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+
+  for (int k0 = 0; k0 < P.k; k0 += GK) {
+    if (P.a.cs == 1) {  // k contiguous
+      for (int e = tid; e < GT * GK; e += 256) {
+        int r = e / GK, kk = e % GK, gi = i0 + r, gk = k0 + kk;
+        As[kk][r] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk] : 0.f;
+      }
+    } else {            // rows contiguous
+      for (int e = tid; e < GT * GK; e += 256) {
+        int kk = e / GT, r = e % GT, gi = i0 + r, gk = k0 + kk;
+        As[kk][r] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
+      }
+    }
+    if (P.b.cs == 1) {  // columns contiguous
+      for (int e = tid; e < GT * GK; e += 256) {
+        int kk = e / GT, c = e % GT, gk = k0 + kk, gj = j0 + c;
+        Bs[kk][c] = (gk < P.k && gj < P.n) ? Bm[gk * P.b.rs + gj] : 0.f;
+      }
+    } else {            // k contiguous
+      for (int e = tid; e < GT * GK; e += 256) {
+        int c = e / GK, kk = e % GK, gk = k0 + kk, gj = j0 + c;
+        Bs[kk][c] = (gk < P.k && gj < P.n) ? Bm[gk * P.b.rs + gj * P.b.cs] : 0.f;
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < GK; ++kk) {
+      float4 a4 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
+      float4 b4 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+      float a[4] = {a4.x, a4.y, a4.z, a4.w};
+      float b[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
+    }
+    __syncthreads();
+  }
+
+  float* Cm = P.c.p + z0 * P.c.b0 + z1 * P.c.b1;
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int i = i0 + ty * 4 + r;
+    if (i >= P.m) continue;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int j = j0 + tx * 4 + c;
+      if (j >= P.n) continue;
+      float v = acc[r][c];
+      if (P.causal && j > i) v = 0.f;
+      if (P.sx) v -= P.sx[z0 * P.sx_b0 + i * P.sx_rs + j] * P.ss[z0 * P.ss_b0 + i];
+      float* dst = Cm + i * P.c.rs + j * P.c.cs;
+      if (P.beta != 0.f) v += P.beta * *dst;
+      *dst = v;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ per-slice staging
+// Loads rows [a, a+b) of every chain, converts to fp32, applies the feature
+// map.  Rows b..Cp-1 of the padded tile are zero everywhere (including the
+// ones column of [V | 1]), so they add nothing to any contraction.
+template <typename T>
+__global__ void __launch_bounds__(256) k_prep(
+    const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
+    const T* __restrict__ dout, const T* __restrict__ out, const float* __restrict__ omega,
+    int L, int d, int M, int a, int b, int Cp, int feature, float inv_sqrt_m,
+    float* Xq, float* Xk, float* Vx, float* phiQ, float* phiK, float* dout32, float* rowdot) {
+  extern __shared__ __align__(16) float sm[];
+  constexpr int R = 16;            // rows per CTA (q and k -> 32 vectors)
+  float* xs = sm;                  // [32][d]
+  float* xn2 = xs + 32 * d;        // [32]
+  float* omT = xn2 + 32;           // [d][64]
+  float* omn = omT + d * 64;       // [64]
+  const int c = blockIdx.y, r0 = blockIdx.x * R, tid = threadIdx.x;
+  const int dp = d + 1;
+  const size_t rowbase = (size_t)c * L + a;
+
+  for (int e = tid; e < R * d; e += 256) {
+    int rr = e / d, j = e % d, r = r0 + rr;
+    float xq = 0.f, xk = 0.f, xv = 0.f;
+    if (r < b) {
+      size_t g = (rowbase + r) * d + j;
+      xq = Io<T>::load(q, g);
+      xk = Io<T>::load(k, g);
+      xv = Io<T>::load(v, g);
+    }
+    xs[rr * d + j] = xq;
+    xs[(R + rr) * d + j] = xk;
+    size_t o = ((size_t)c * Cp + r) * d + j;
+    Xq[o] = xq;
+    Xk[o] = xk;
+    Vx[((size_t)c * Cp + r) * dp + j] = xv;
+    if (dout32) dout32[o] = (r < b) ? Io<T>::load(dout, (rowbase + r) * d + j) : 0.f;
+  }
+  for (int rr = tid; rr < R; rr += 256)
+    Vx[((size_t)c * Cp + r0 + rr) * dp + d] = (r0 + rr < b) ? 1.f : 0.f;
+  __syncthreads();
+
+  const int warp = tid / 32, lane = tid % 32;
+  for (int vec = warp; vec < 2 * R; vec += 8) {
+    float s = 0.f;
+    for (int j = lane; j < d; j += 32) s = fmaf(xs[vec * d + j], xs[vec * d + j], s);
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) xn2[vec] = s;
+  }
+  if (rowdot) {
+    for (int rr = warp; rr < R; rr += 8) {
+      const int r = r0 + rr;
+      float s = 0.f;
+      if (r < b)
+        for (int j = lane; j < d; j += 32) {
+          size_t g = (rowbase + r) * d + j;
+          s = fmaf(Io<T>::load(dout, g), Io<T>::load(out, g), s);
+        }
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      if (lane == 0) rowdot[(size_t)c * Cp + r] = s;
+    }
+  }
+
+  // error bound of an fp32 dot product of length d, times a safety factor 2
+  const float gamma = 2.f * (float)(d + 2) * 5.9604645e-08f;
+  for (int m0 = 0; m0 < M; m0 += 64) {
+    __syncthreads();
+    for (int e = tid; e < 64 * d; e += 256) {
+      int mm = e / d, j = e % d;
+      omT[j * 64 + mm] = (m0 + mm < M) ? omega[(size_t)(m0 + mm) * d + j] : 0.f;
+    }
+    __syncthreads();
+    if (tid < 64) {
+      float s = 0.f;
+      for (int j = 0; j < d; ++j) s = fmaf(omT[j * 64 + tid], omT[j * 64 + tid], s);
+      omn[tid] = sqrtf(s);
+    }
+    __syncthreads();
+    const int mm = tid % 64, grp = tid / 64, m = m0 + mm;
+    if (m < M) {
+      for (int vv = 0; vv < 8; ++vv) {
+        const int vec = grp * 8 + vv;
+        const int rr = vec % R, r = r0 + rr;
+        float dot = 0.f;
+        for (int j = 0; j < d; ++j) dot = fmaf(xs[vec * d + j], omT[j * 64 + mm], dot);
+        float phi = 0.f;
+        if (r < b) {
+          if (feature == SLIM_FEAT_EXP) {
+            phi = expf(dot - 0.5f * xn2[vec]) * inv_sqrt_m;
+          } else {
+            // The sign of omega.x decides ReLU's branch; near zero it is
+            // recomputed in fp64 so the decision is the exact one.
+            if (fabsf(dot) <= gamma * omn[mm] * sqrtf(xn2[vec])) {
+              double acc = 0.0;
+              for (int j = 0; j < d; ++j)
+                acc += (double)omega[(size_t)m * d + j] * (double)xs[vec * d + j];
+              phi = acc > 0.0 ? (float)acc * inv_sqrt_m : 0.f;
+            } else {
+              phi = dot > 0.f ? dot * inv_sqrt_m : 0.f;
+            }
+          }
+        }
+        float* dst = (vec < R) ? phiQ : phiK;
+        dst[((size_t)c * Cp + r) * M + m] = phi;
+      }
+    }
+  }
+}
+
+// State scans over the tiles of one slice, one thread per (chain, element).
+enum ScanMode { SCAN_FWD = 0, SCAN_ROLLBACK = 1, SCAN_GREV = 2 };
+
+__global__ void k_scan(float* buf, float* hi_p, float* lo_p, int chains, int nt, int E, int mode) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (long long)chains * E) return;
+  const int c = (int)(idx / E), e = (int)(idx % E);
+  float hi = hi_p[idx], lo = lo_p[idx];
+  float* col = buf + (size_t)c * nt * E + e;
+  if (mode == SCAN_GREV) {
+    // G_t = G + sum_{t' > t} Gd_t'  (reversed prefix sum), then G += all
+    for (int t = nt - 1; t >= 0; --t) {
+      float x = col[(size_t)t * E];
+      col[(size_t)t * E] = hi + lo;
+      pair_add(hi, lo, x);
+    }
+    hi_p[idx] = hi;
+    lo_p[idx] = lo;
+    return;
+  }
+  if (mode == SCAN_ROLLBACK) {
+    // eq. 17: B^(n-1) = B^(n) - sum_t Delta_t, undone in reverse order
+    for (int t = nt - 1; t >= 0; --t) pair_add(hi, lo, -col[(size_t)t * E]);
+    hi_p[idx] = hi;
+    lo_p[idx] = lo;
+  }
+  for (int t = 0; t < nt; ++t) {
+    float x = col[(size_t)t * E];
+    col[(size_t)t * E] = hi + lo;
+    pair_add(hi, lo, x);
+  }
+  if (mode == SCAN_FWD) {
+    hi_p[idx] = hi;
+    lo_p[idx] = lo;
+  }
+}
+
+template <typename T>
+__global__ void k_finalize_out(const float* numden, T* out, int L, int d, int a, int b, int Cp,
+                               int chains) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (long long)chains * b * d) return;
+  const int j = (int)(idx % d);
+  const long long rc = idx / d;
+  const int r = (int)(rc % b), c = (int)(rc / b);
+  const float* row = numden + ((size_t)c * Cp + r) * (d + 1);
+  const float den = row[d];
+  Io<T>::store(out, ((size_t)c * L + a + r) * d + j, den != 0.f ? row[j] / den : 0.f);
+}
+
+__global__ void k_dstat(const float* numden, const float* dout32, const float* rowdot, float* W,
+                        int d, int b, int Cp, int chains) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const int dp = d + 1;
+  if (idx >= (long long)chains * Cp * dp) return;
+  const int j = (int)(idx % dp);
+  const long long rc = idx / dp;
+  const int r = (int)(rc % Cp);
+  const float den = numden[rc * dp + d];
+  float w = 0.f;
+  if (r < b && den != 0.f) w = (j < d) ? dout32[rc * d + j] / den : -rowdot[rc] / den;
+  W[idx] = w;
+}
+
+// u = dphi * phi (exp) or dphi * 1[phi > 0] / sqrt(M) (ReLU), in place; row sums.
+__global__ void k_vjp_prep(float* dphi, const float* phi, float* usum, int M, int rows,
+                           int feature, float inv_sqrt_m) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) / 32, lane = threadIdx.x % 32;
+  if (warp >= rows) return;
+  float* u = dphi + (size_t)warp * M;
+  const float* p = phi + (size_t)warp * M;
+  float s = 0.f;
+  for (int m = lane; m < M; m += 32) {
+    float x = (feature == SLIM_FEAT_EXP) ? u[m] * p[m] : (p[m] > 0.f ? u[m] * inv_sqrt_m : 0.f);
+    u[m] = x;
+    s += x;
+  }
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) usum[warp] = s;
+}
+
+template <typename T>
+__global__ void k_store(const float* stage, T* dst, int L, int d, int a, int b, int Cp,
+                        int chains) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (long long)chains * b * d) return;
+  const int j = (int)(idx % d);
+  const long long rc = idx / d;
+  const int r = (int)(rc % b), c = (int)(rc / b);
+  Io<T>::store(dst, ((size_t)c * L + a + r) * d + j, stage[((size_t)c * Cp + r) * d + j]);
+}
+
+// dOmega += sum over chains of the slice's per-chain partials, fixed order.
+__global__ void k_reduce_domega(const float* part, float* domega, int chains, int MD) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= MD) return;
+  float s = 0.f;
+  for (int c = 0; c < chains; ++c) s += part[(size_t)c * MD + e];
+  domega[e] += s;
+}
+
+__global__ void k_state_out(const float* hi, const float* lo, float* S_state, float* z_state,
+                            int chains, int M, int d) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const int dp = d + 1;
+  if (idx >= (long long)chains * M * dp) return;
+  const int j = (int)(idx % dp);
+  const long long cm = idx / dp;
+  const float x = hi[idx] + lo[idx];
+  if (j < d) S_state[cm * d + j] = x;
+  else z_state[cm] = x;
+}
+
+__global__ void k_state_in(const float* S_state, const float* z_state, float* hi, float* lo,
+                           int chains, int M, int d) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const int dp = d + 1;
+  if (idx >= (long long)chains * M * dp) return;
+  const int j = (int)(idx % dp);
+  const long long cm = idx / dp;
+  hi[idx] = (j < d) ? S_state[cm * d + j] : z_state[cm];
+  lo[idx] = 0.f;
+}
+
+// ------------------------------------------------------------------ host side
+namespace {
+
+struct Geo {
+  int chains, d, dp, M, Cs, T, nt, Cp, N;
+};
+
+Geo geometry(const Problem& p) {
+  Geo g;
+  g.chains = p.chains();
+  g.d = p.d;
+  g.dp = p.d + 1;
+  g.M = p.M;
+  g.Cs = p.slice_len();
+  g.T = g.Cs >= 64 ? 64 : ((g.Cs + 15) / 16) * 16;
+  if (g.T < 16) g.T = 16;
+  g.nt = (g.Cs + g.T - 1) / g.T;
+  g.Cp = g.nt * g.T;
+  g.N = p.num_slices();
+  return g;
+}
+
+struct Ws {
+  int* err;
+  float *st_hi, *st_lo, *g_hi, *g_lo;
+  float *Xq, *Xk, *Vx, *phiQ, *phiK, *delta, *A, *numden;
+  float *dout32, *rowdot, *W, *dA, *dphiQ, *dphiK, *gdelta, *usum_q, *usum_k, *stage, *pOm;
+};
+
+Ws carve(Carver& cv, const Geo& g, bool bwd) {
+  Ws w{};
+  const size_t C = g.chains;
+  w.err = cv.take<int>(64);
+  w.st_hi = cv.take<float>(C * g.M * g.dp);
+  w.st_lo = cv.take<float>(C * g.M * g.dp);
+  w.Xq = cv.take<float>(C * g.Cp * g.d);
+  w.Xk = cv.take<float>(C * g.Cp * g.d);
+  w.Vx = cv.take<float>(C * g.Cp * g.dp);
+  w.phiQ = cv.take<float>(C * g.Cp * g.M);
+  w.phiK = cv.take<float>(C * g.Cp * g.M);
+  w.delta = cv.take<float>(C * g.nt * g.M * g.dp);
+  w.A = cv.take<float>(C * g.nt * g.T * g.T);
+  w.numden = cv.take<float>(C * g.Cp * g.dp);
+  if (bwd) {
+    w.g_hi = cv.take<float>(C * g.M * g.dp);
+    w.g_lo = cv.take<float>(C * g.M * g.dp);
+    w.dout32 = cv.take<float>(C * g.Cp * g.d);
+    w.rowdot = cv.take<float>(C * g.Cp);
+    w.W = cv.take<float>(C * g.Cp * g.dp);
+    w.dA = cv.take<float>(C * g.nt * g.T * g.T);
+    w.dphiQ = cv.take<float>(C * g.Cp * g.M);
+    w.dphiK = cv.take<float>(C * g.Cp * g.M);
+    w.gdelta = cv.take<float>(C * g.nt * g.M * g.dp);
+    w.usum_q = cv.take<float>(C * g.Cp);
+    w.usum_k = cv.take<float>(C * g.Cp);
+    w.stage = cv.take<float>(C * g.Cp * g.d);
+    w.pOm = cv.take<float>(C * g.M * g.d);
+  }
+  return w;
+}
+
+Mat mat(const float* p, long long b0, long long b1, long long rs, long long cs) {
+  return Mat{p, b0, b1, rs, cs};
+}
+OutMat omat(float* p, long long b0, long long b1, long long rs, long long cs) {
+  return OutMat{p, b0, b1, rs, cs};
+}
+
+cudaError_t gemm(cudaStream_t s, int m, int n, int k, Mat a, Mat b, OutMat c, int nb0, int nb1,
+                 float beta, int causal, const float* sx = nullptr, long long sx_b0 = 0,
+                 long long sx_rs = 0, const float* ss = nullptr, long long ss_b0 = 0) {
+  const int nz = nb0 * nb1;
+  for (int z = 0; z < nz; z += 65535) {
+    GemmP P{m, n, k, a, b, c, nb1, z, beta, causal, sx, sx_b0, sx_rs, ss, ss_b0};
+    const int zc = (nz - z < 65535) ? nz - z : 65535;
+    dim3 grid((n + GT - 1) / GT, (m + GT - 1) / GT, zc);
+    prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
+    k_gemm<<<grid, 256, 0, s>>>(P);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+unsigned blocks(long long n, int t = 256) { return (unsigned)((n + t - 1) / t); }
+
+#define SLIM_TRY(x)                                   \
+  do {                                                \
+    cudaError_t e_ = (x);                             \
+    if (e_ != cudaSuccess) return SLIM_ERR_CUDA;      \
+  } while (0)
+
+template <typename T>
+cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w,
+                        const void* q, const void* k, const void* v, const void* dout,
+                        const void* out, const float* omega, int a, int b, bool bwd) {
+  const size_t smem = (32 * g.d + 32 + g.d * 64 + 64) * sizeof(float);
+  static bool attr_set = false;  // one instantiation per dtype; set once
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_prep<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         64 * 1024);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid(g.Cp / 16, g.chains);
+  const float inv_sqrt_m = (float)(1.0 / sqrt((double)g.M));
+  const double rows = (double)g.chains * b;
+  prof::Scope ps(prof::K_PREP, s, 4.0 * rows * g.d * g.M,
+                 rows * g.d * sizeof(T) * (bwd ? 5.0 : 3.0));
+  k_prep<T><<<grid, 256, smem, s>>>(
+      (const T*)q, (const T*)k, (const T*)v, bwd ? (const T*)dout : nullptr,
+      bwd ? (const T*)out : nullptr, omega, p.L, g.d, g.M, a, b, g.Cp, (int)p.feature,
+      inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
+      bwd ? w.rowdot : nullptr);
+  return cudaGetLastError();
+}
+
+// Delta_t = phiK_t^T [V_t | 1]  (M x dp per tile)
+cudaError_t tile_deltas(cudaStream_t s, const Geo& g, const Ws& w) {
+  const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
+  return gemm(s, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
+              omat(w.delta, nt * M * dp, M * dp, dp, 1), g.chains, g.nt, 0.f, 0);
+}
+
+// A_t = tril(phiQ_t phiK_t^T); [num | den] = phiQ_t P_t + A_t [V_t | 1]
+cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w) {
+  const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
+  cudaError_t e = gemm(s, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+                       mat(w.phiK, Cp * M, T * M, 1, M), omat(w.A, nt * T * T, T * T, T, 1),
+                       g.chains, g.nt, 0.f, 1);
+  if (e != cudaSuccess) return e;
+  e = gemm(s, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+           mat(w.delta, nt * M * dp, M * dp, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
+           g.chains, g.nt, 0.f, 0);
+  if (e != cudaSuccess) return e;
+  return gemm(s, g.T, g.dp, g.T, mat(w.A, nt * T * T, T * T, T, 1),
+              mat(w.Vx, Cp * dp, T * dp, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
+              g.chains, g.nt, 1.f, 0);
+}
+
+cudaError_t scan(cudaStream_t s, const Geo& g, float* buf, float* hi, float* lo, int mode) {
+  const long long E = (long long)g.M * g.dp;
+  prof::Scope ps(prof::K_SCAN, s);
+  k_scan<<<blocks(g.chains * E), 256, 0, s>>>(buf, hi, lo, g.chains, g.nt, (int)E, mode);
+  return cudaGetLastError();
+}
+
+template <typename T>
+slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void* v,
+                     const float* omega, void* out, float* S_state, float* z_state,
+                     void* workspace, cudaStream_t s) {
+  const Geo g = geometry(p);
+  Carver cv(workspace);
+  const Ws w = carve(cv, g, false);
+  const size_t E = (size_t)g.chains * g.M * g.dp;
+  SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(cudaMemsetAsync(w.st_hi, 0, E * sizeof(float), s));
+  SLIM_TRY(cudaMemsetAsync(w.st_lo, 0, E * sizeof(float), s));
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(tile_deltas(s, g, w));
+    SLIM_TRY(scan(s, g, w.delta, w.st_hi, w.st_lo, SCAN_FWD));
+    SLIM_TRY(scores_and_readout(s, g, w));
+    { prof::Scope ps(prof::K_FINALIZE, s, 0.0, (double)g.chains * b * g.d * sizeof(T));
+    k_finalize_out<T><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(
+        w.numden, (T*)out, p.L, g.d, a, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+  }
+  {
+    prof::Scope ps(prof::K_STATE, s);
+    k_state_out<<<blocks((long long)E), 256, 0, s>>>(w.st_hi, w.st_lo, S_state, z_state,
+                                                     g.chains, g.M, g.d);
+  }
+  SLIM_TRY(cudaGetLastError());
+  return SLIM_OK;
+}
+
+template <typename IO>
+slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void* v,
+                     const float* omega, const void* out, const void* dout,
+                     const float* S_state, const float* z_state, void* dq, void* dk, void* dv,
+                     float* domega, void* workspace, cudaStream_t s) {
+  const Geo g = geometry(p);
+  Carver cv(workspace);
+  const Ws w = carve(cv, g, true);
+  const long long T = g.T, M = g.M, d = g.d, dp = g.dp, Cp = g.Cp, nt = g.nt;
+  const size_t E = (size_t)g.chains * g.M * g.dp;
+  SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
+  { prof::Scope ps(prof::K_STATE, s);
+  k_state_in<<<blocks((long long)E), 256, 0, s>>>(S_state, z_state, w.st_hi, w.st_lo, g.chains,
+                                                  g.M, g.d); }
+  SLIM_TRY(cudaGetLastError());
+  SLIM_TRY(cudaMemsetAsync(w.g_hi, 0, E * sizeof(float), s));
+  SLIM_TRY(cudaMemsetAsync(w.g_lo, 0, E * sizeof(float), s));
+  const float inv_sqrt_m = (float)(1.0 / sqrt((double)g.M));
+
+  for (int n = g.N - 1; n >= 0; --n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
+    SLIM_TRY(tile_deltas(s, g, w));
+    SLIM_TRY(scan(s, g, w.delta, w.st_hi, w.st_lo, SCAN_ROLLBACK));
+    SLIM_TRY(scores_and_readout(s, g, w));
+    { prof::Scope ps(prof::K_DSTAT, s);
+    k_dstat<<<blocks((long long)g.chains * Cp * dp), 256, 0, s>>>(w.numden, w.dout32, w.rowdot, w.W,
+                                                               g.d, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+    // dA_t = tril(W_t [V_t | 1]^T)
+    SLIM_TRY(gemm(s, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+                  mat(w.Vx, Cp * dp, T * dp, 1, dp), omat(w.dA, nt * T * T, T * T, T, 1),
+                  g.chains, g.nt, 0.f, 1));
+    // dphiQ = W_t P_t^T + dA_t phiK_t
+    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+                  mat(w.delta, nt * M * dp, M * dp, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
+                  g.chains, g.nt, 0.f, 0));
+    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
+                  mat(w.phiK, Cp * M, T * M, M, 1), omat(w.dphiQ, Cp * M, T * M, M, 1), g.chains,
+                  g.nt, 1.f, 0));
+    // Gd_t = phiQ_t^T W_t, then G_t = G + sum_{t' > t} Gd_t'
+    SLIM_TRY(gemm(s, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+                  mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
+                  g.chains, g.nt, 0.f, 0));
+    SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
+    // dphiK = dA_t^T phiQ_t + [V_t | 1] G_t^T
+    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
+                  mat(w.phiQ, Cp * M, T * M, M, 1), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
+                  g.nt, 0.f, 0));
+    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+                  mat(w.gdelta, nt * M * dp, M * dp, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1),
+                  g.chains, g.nt, 1.f, 0));
+    // dV = A_t^T dnum + phiK_t G_t(S)
+    SLIM_TRY(gemm(s, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
+                  mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
+                  g.nt, 0.f, 0));
+    SLIM_TRY(gemm(s, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+                  mat(w.gdelta, nt * M * dp, M * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1),
+                  g.chains, g.nt, 1.f, 0));
+    { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+    k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dv, p.L, g.d,
+                                                                      a, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+    // feature VJPs
+    const int rows = g.chains * g.Cp;
+    { prof::Scope ps(prof::K_VJP, s);
+    k_vjp_prep<<<blocks((long long)rows * 32), 256, 0, s>>>(w.dphiQ, w.phiQ, w.usum_q, g.M, rows,
+                                                            (int)p.feature, inv_sqrt_m); }
+    SLIM_TRY(cudaGetLastError());
+    { prof::Scope ps(prof::K_VJP, s);
+    k_vjp_prep<<<blocks((long long)rows * 32), 256, 0, s>>>(w.dphiK, w.phiK, w.usum_k, g.M, rows,
+                                                            (int)p.feature, inv_sqrt_m); }
+    SLIM_TRY(cudaGetLastError());
+    const bool ex = p.feature == SLIM_FEAT_EXP;
+    // dX = u Omega (- x sum u for the exp map)
+    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+                  omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xq : nullptr,
+                  Cp * d, d, w.usum_q, Cp));
+    { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+    k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dq, p.L, g.d,
+                                                                      a, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+                  omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xk : nullptr,
+                  Cp * d, d, w.usum_k, Cp));
+    { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+    k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dk, p.L, g.d,
+                                                                      a, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+    // dOmega partial per chain: u_q^T x_q + u_k^T x_k
+    SLIM_TRY(gemm(s, g.M, g.d, g.Cp, mat(w.dphiQ, Cp * M, 0, 1, M), mat(w.Xq, Cp * d, 0, d, 1),
+                  omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 0.f, 0));
+    SLIM_TRY(gemm(s, g.M, g.d, g.Cp, mat(w.dphiK, Cp * M, 0, 1, M), mat(w.Xk, Cp * d, 0, d, 1),
+                  omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 1.f, 0));
+    { prof::Scope ps(prof::K_REDUCE, s);
+    k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains,
+                                                             (int)(M * d)); }
+    SLIM_TRY(cudaGetLastError());
+  }
+  return SLIM_OK;
+}
+
+}  // namespace
+
+size_t workspace_bytes(const Problem& p, bool bwd) {
+  const Geo g = geometry(p);
+  Carver cv(nullptr);
+  carve(cv, g, bwd);
+  return cv.bytes();
+}
+
+slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
+                const float* omega, void* out, float* S_state, float* z_state, void* workspace,
+                cudaStream_t s) {
+  if (p.dtype == SLIM_BF16)
+    return fwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, S_state, z_state, workspace, s);
+  return fwd_impl<float>(p, q, k, v, omega, out, S_state, z_state, workspace, s);
+}
+
+slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
+                const float* omega, const void* out, const void* dout, const float* S_state,
+                const float* z_state, void* dq, void* dk, void* dv, float* domega,
+                void* workspace, cudaStream_t s) {
+  if (p.dtype == SLIM_BF16)
+    return bwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv,
+                                   domega, workspace, s);
+  return bwd_impl<float>(p, q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv, domega,
+                         workspace, s);
+}
+
+}  // namespace simt
+}  // namespace slim

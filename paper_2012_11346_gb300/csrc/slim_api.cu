@@ -1,0 +1,139 @@
+// C ABI of libslim: argument validation, workspace sizing, dispatch.
+// Declarations and the contract of every entry point: include/slim.h.
+#include <stdint.h>
+
+#include "common.cuh"
+#include "simt_path.h"
+
+using slim::Problem;
+
+namespace {
+
+constexpr int kVersion = 100;  // 0.1.0
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+slim_status check_problem(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                          slim_feature feature, Problem* out) {
+  if (B < 1 || H < 1 || L < 0 || C < 1) return SLIM_ERR_INVALID_ARG;
+  if (dtype != SLIM_F32 && dtype != SLIM_BF16) return SLIM_ERR_INVALID_ARG;
+  if (feature != SLIM_FEAT_EXP && feature != SLIM_FEAT_RELU) return SLIM_ERR_INVALID_ARG;
+  if (d < 1 || M < 1) return SLIM_ERR_INVALID_ARG;
+  // element counts must stay far inside 64-bit range, chains inside int
+  const long long chains = (long long)B * H;
+  if (chains > (1LL << 24)) return SLIM_ERR_INVALID_ARG;
+  if ((long long)L * d > (1LL << 40) / chains) return SLIM_ERR_INVALID_ARG;
+  if (!(d == 16 || d == 32 || d == 64 || d == 128)) return SLIM_ERR_UNSUPPORTED;
+  if (M % 16 != 0 || M > 256) return SLIM_ERR_UNSUPPORTED;
+  *out = Problem{B, H, L, d, M, C, dtype, feature};
+  return SLIM_OK;
+}
+
+size_t ws_bytes(const Problem& p, bool bwd) { return slim::simt::workspace_bytes(p, bwd); }
+
+slim_status check_workspace(const Problem& p, bool bwd, void* ws, size_t bytes) {
+  const size_t need = ws_bytes(p, bwd);
+  if (need == 0) return SLIM_OK;
+  if (ws == nullptr || bytes < need) return SLIM_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return SLIM_ERR_INVALID_ARG;
+  return SLIM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* slim_status_string(slim_status s) {
+  switch (s) {
+    case SLIM_OK: return "SLIM_OK";
+    case SLIM_ERR_INVALID_ARG: return "SLIM_ERR_INVALID_ARG: invalid argument";
+    case SLIM_ERR_UNSUPPORTED: return "SLIM_ERR_UNSUPPORTED: unsupported (d, M, dtype, feature)";
+    case SLIM_ERR_WORKSPACE: return "SLIM_ERR_WORKSPACE: workspace missing or too small";
+    case SLIM_ERR_CUDA: return "SLIM_ERR_CUDA: a CUDA launch or runtime call failed";
+    case SLIM_ERR_TIMEOUT: return "SLIM_ERR_TIMEOUT: a bounded device-side wait gave up";
+  }
+  return "unknown slim_status";
+}
+
+int slim_version(void) { return kVersion; }
+
+slim_status slim_fwd_workspace_size(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                                    slim_feature feature, size_t* bytes) {
+  if (!bytes) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  *bytes = ws_bytes(p, false);
+  return SLIM_OK;
+}
+
+slim_status slim_bwd_workspace_size(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                                    slim_feature feature, size_t* bytes) {
+  if (!bytes) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  *bytes = ws_bytes(p, true);
+  return SLIM_OK;
+}
+
+slim_status slim_fwd(const void* q, const void* k, const void* v, const float* omega, int B,
+                     int H, int L, int d, int M, int C, slim_dtype dtype, slim_feature feature,
+                     void* out, float* S_state, float* z_state, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  const void* ptrs[] = {q, k, v, omega, out, S_state, z_state};
+  for (const void* ptr : ptrs)
+    if (ptr == nullptr || !aligned16(ptr)) return SLIM_ERR_INVALID_ARG;
+  st = check_workspace(p, false, workspace, workspace_bytes);
+  if (st != SLIM_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (L == 0) {
+    const size_t n = (size_t)p.chains() * M;
+    if (cudaMemsetAsync(S_state, 0, n * d * sizeof(float), s) != cudaSuccess) return SLIM_ERR_CUDA;
+    if (cudaMemsetAsync(z_state, 0, n * sizeof(float), s) != cudaSuccess) return SLIM_ERR_CUDA;
+    return SLIM_OK;
+  }
+  return slim::simt::fwd(p, q, k, v, omega, out, S_state, z_state, workspace, s);
+}
+
+slim_status slim_bwd(const void* q, const void* k, const void* v, const float* omega,
+                     const void* out, const void* dout, const float* S_state,
+                     const float* z_state, int B, int H, int L, int d, int M, int C,
+                     slim_dtype dtype, slim_feature feature, void* dq, void* dk, void* dv,
+                     float* domega, void* workspace, size_t workspace_bytes, void* stream) {
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  const void* ptrs[] = {q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv, domega};
+  for (const void* ptr : ptrs)
+    if (ptr == nullptr || !aligned16(ptr)) return SLIM_ERR_INVALID_ARG;
+  st = check_workspace(p, true, workspace, workspace_bytes);
+  if (st != SLIM_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (L == 0) {
+    if (cudaMemsetAsync(domega, 0, (size_t)M * d * sizeof(float), s) != cudaSuccess)
+      return SLIM_ERR_CUDA;
+    return SLIM_OK;
+  }
+  return slim::simt::bwd(p, q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv, domega,
+                         workspace, s);
+}
+
+slim_status slim_check_device_error(void* workspace, void* stream) {
+  if (workspace == nullptr) return SLIM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int word = 0;
+  if (cudaMemcpyAsync(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return SLIM_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return SLIM_ERR_CUDA;
+  if (word != 0) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(int), s) != cudaSuccess) return SLIM_ERR_CUDA;
+    return SLIM_ERR_TIMEOUT;
+  }
+  return SLIM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,217 @@
+"""Python binding of libslim (ctypes): argument marshalling only.
+
+Every computation runs in the CUDA kernels behind the C ABI declared in
+include/slim.h.  PyTorch supplies device memory (outputs and workspace, so
+torch.cuda.max_memory_allocated sees all of it) and the current stream.  There
+is no CPU fallback: if libslim.so is missing or no GPU is present, the calls
+raise.
+"""
+import ctypes
+import os
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libslim.so")
+_lib = None
+
+DTYPES = {torch.float32: 0, torch.bfloat16: 1}
+FEATURES = {"exp": 0, "relu": 1}
+STATUS = {0: "SLIM_OK", 1: "SLIM_ERR_INVALID_ARG", 2: "SLIM_ERR_UNSUPPORTED",
+          3: "SLIM_ERR_WORKSPACE", 4: "SLIM_ERR_CUDA", 5: "SLIM_ERR_TIMEOUT"}
+
+_i, _p, _sz = ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t
+
+# (name, argtypes) for every symbol of include/slim.h
+SIGNATURES = {
+    "slim_status_string": ([_i], ctypes.c_char_p),
+    "slim_version": ([], _i),
+    "slim_fwd_workspace_size": ([_i] * 6 + [_i, _i, ctypes.POINTER(_sz)], _i),
+    "slim_bwd_workspace_size": ([_i] * 6 + [_i, _i, ctypes.POINTER(_sz)], _i),
+    "slim_fwd": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 3 + [_p, _sz, _p], _i),
+    "slim_bwd": ([_p] * 8 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
+    "slim_check_device_error": ([_p, _p], _i),
+    "slim_launch_count": ([], ctypes.c_ulonglong),
+    "slim_profiler_enable": ([_i], None),
+    "slim_profiler_reset": ([], None),
+    "slim_profiler_read": ([_p, _i], _i),
+}
+
+
+class KernelStats(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_ulonglong),
+                ("total_ms", ctypes.c_double), ("flops", ctypes.c_double),
+                ("bytes", ctypes.c_double)]
+
+
+class SlimError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)}")
+
+
+def library():
+    """Loads libslim.so (built by paper_2012_11346_gb300.build); raises if absent."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(f"libslim.so not built ({_LIB_PATH}); run "
+                               "python -m paper_2012_11346_gb300.build")
+        lib = ctypes.CDLL(_LIB_PATH)
+        for name, (args, res) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = lib
+    return _lib
+
+
+def status_string(status):
+    return library().slim_status_string(int(status)).decode()
+
+
+def _check(status, where):
+    if status != 0:
+        raise SlimError(status, where)
+
+
+def _dims(q, omega):
+    B, H, L, d = q.shape
+    M = omega.shape[0]
+    return B, H, L, d, M
+
+
+def workspace_size(B, H, L, d, M, C, dtype, feature, backward):
+    n = _sz(0)
+    fn = library().slim_bwd_workspace_size if backward else library().slim_fwd_workspace_size
+    _check(fn(B, H, L, d, M, C, DTYPES[dtype], FEATURES[feature], ctypes.byref(n)),
+           "workspace_size")
+    return n.value
+
+
+def _stream_handle(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _workspace(nbytes, device):
+    return torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+
+
+def _require_cuda(*ts):
+    for t in ts:
+        if not t.is_cuda:
+            raise RuntimeError("libslim runs on CUDA tensors only (no CPU fallback)")
+        if not t.is_contiguous():
+            raise RuntimeError("libslim needs contiguous tensors")
+
+
+def forward(q, k, v, omega, C, feature="exp", workspace=None, stream=None):
+    """slim_fwd: returns (out, S_state, z_state)."""
+    _require_cuda(q, k, v, omega)
+    B, H, L, d, M = _dims(q, omega)
+    out = torch.empty_like(q)
+    S_state = torch.empty(B, H, M, d, dtype=torch.float32, device=q.device)
+    z_state = torch.empty(B, H, M, dtype=torch.float32, device=q.device)
+    need = workspace_size(B, H, L, d, M, C, q.dtype, feature, False)
+    ws = workspace if workspace is not None else _workspace(need, q.device)
+    _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
+                              B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
+                              out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
+                              ws.data_ptr(), ws.numel(), _stream_handle(stream)), "slim_fwd")
+    return out, S_state, z_state
+
+
+def backward(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp", workspace=None,
+             stream=None):
+    """slim_bwd: returns (dq, dk, dv, domega)."""
+    _require_cuda(q, k, v, omega, out, dout, S_state, z_state)
+    B, H, L, d, M = _dims(q, omega)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    domega = torch.empty(M, d, dtype=torch.float32, device=q.device)
+    need = workspace_size(B, H, L, d, M, C, q.dtype, feature, True)
+    ws = workspace if workspace is not None else _workspace(need, q.device)
+    _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
+                              out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
+                              z_state.data_ptr(), B, H, L, d, M, C, DTYPES[q.dtype],
+                              FEATURES[feature], dq.data_ptr(), dk.data_ptr(), dv.data_ptr(),
+                              domega.data_ptr(), ws.data_ptr(), ws.numel(),
+                              _stream_handle(stream)), "slim_bwd")
+    return dq, dk, dv, domega
+
+
+def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None):
+    """slim_fwd into caller-allocated outputs and workspace (no allocation)."""
+    B, H, L, d, M = _dims(q, omega)
+    _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
+                              B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
+                              out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
+                              workspace.data_ptr(), workspace.numel(), _stream_handle(stream)),
+           "slim_fwd")
+
+
+def backward_into(q, k, v, omega, out, dout, S_state, z_state, C, feature, dq, dk, dv, domega,
+                  workspace, stream=None):
+    """slim_bwd into caller-allocated gradients and workspace (no allocation)."""
+    B, H, L, d, M = _dims(q, omega)
+    _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
+                              out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
+                              z_state.data_ptr(), B, H, L, d, M, C, DTYPES[q.dtype],
+                              FEATURES[feature], dq.data_ptr(), dk.data_ptr(), dv.data_ptr(),
+                              domega.data_ptr(), workspace.data_ptr(), workspace.numel(),
+                              _stream_handle(stream)), "slim_bwd")
+
+
+def check_device_error(workspace, stream=None):
+    """Raises SlimError(SLIM_ERR_TIMEOUT) if a bounded device wait gave up."""
+    _check(library().slim_check_device_error(workspace.data_ptr(), _stream_handle(stream)),
+           "slim_check_device_error")
+
+
+def launch_count():
+    """Number of libslim kernel launches since the library was loaded."""
+    return int(library().slim_launch_count())
+
+
+def profiler_enable(on=True):
+    library().slim_profiler_enable(1 if on else 0)
+
+
+def profiler_reset():
+    library().slim_profiler_reset()
+
+
+def profiler_read():
+    """Per-kernel totals since the last reset: list of dicts with name,
+    launches, total_ms (CUDA events), flops and bytes (algorithmic)."""
+    arr = (KernelStats * 64)()
+    n = library().slim_profiler_read(ctypes.cast(arr, ctypes.c_void_p), 64)
+    if n < 0:
+        raise SlimError(4, "slim_profiler_read")
+    return [{"name": arr[i].name.decode(), "launches": int(arr[i].launches),
+             "total_ms": arr[i].total_ms, "flops": arr[i].flops, "bytes": arr[i].bytes}
+            for i in range(min(n, 64))]
+
+
+class SlimAttention(torch.autograd.Function):
+    """Causal linear attention with the SLiM forward/backward (state carried
+    across slices of C rows; backward by rollback, no stored activations)."""
+
+    @staticmethod
+    def forward(ctx, q, k, v, omega, C, feature):
+        out, S_state, z_state = forward(q.contiguous(), k.contiguous(), v.contiguous(),
+                                        omega.contiguous(), C, feature)
+        ctx.save_for_backward(q, k, v, omega, out, S_state, z_state)
+        ctx.C, ctx.feature = C, feature
+        return out
+
+    @staticmethod
+    def backward(ctx, dout):
+        q, k, v, omega, out, S_state, z_state = ctx.saved_tensors
+        dq, dk, dv, domega = backward(q.contiguous(), k.contiguous(), v.contiguous(),
+                                      omega.contiguous(), out, dout.contiguous(), S_state,
+                                      z_state, ctx.C, ctx.feature)
+        return dq, dk, dv, domega, None, None
+
+
+def slim_attention(q, k, v, omega, C, feature="exp"):
+    return SlimAttention.apply(q, k, v, omega, C, feature)

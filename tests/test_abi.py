@@ -1,0 +1,137 @@
+"""Host-only checks of the C ABI: the library loads, exports every symbol that
+include/slim.h declares, sizes workspaces, and rejects bad arguments before
+anything is enqueued (these calls never reach a CUDA launch)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2012_11346_gb300 import slim
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = [os.path.join(ROOT, "include", f) for f in sorted(os.listdir(os.path.join(ROOT, "include")))
+           if f.endswith(".h")]
+
+OK, INVALID, UNSUPPORTED, WORKSPACE = 0, 1, 2, 3
+
+
+def declared_symbols():
+    names = set()
+    for h in HEADERS:
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        names.update(re.findall(r"\b(slim_[a-z0-9_]+)\s*\(", text))
+    return sorted(names)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(slim._LIB_PATH):
+        from paper_2012_11346_gb300 import build
+        build.build()
+    return slim.library()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_symbols()
+    assert "slim_fwd" in names and "slim_bwd" in names
+    for n in names:
+        assert hasattr(lib, n), n
+        assert n in slim.SIGNATURES, f"binding lacks {n}"
+
+
+def test_status_strings(lib):
+    for code, name in slim.STATUS.items():
+        assert slim.status_string(code).startswith(name)
+    assert lib.slim_version() >= 100
+
+
+def ws(B, H, L, d, M, C, dt=0, ft=0, bwd=False):
+    n = ctypes.c_size_t(0)
+    fn = slim.library().slim_bwd_workspace_size if bwd else slim.library().slim_fwd_workspace_size
+    st = fn(B, H, L, d, M, C, dt, ft, ctypes.byref(n))
+    return st, n.value
+
+
+def test_workspace_sizes_scale_with_C_not_L(lib):
+    for bwd in (False, True):
+        st, a = ws(2, 8, 32768, 64, 256, 64, 1, 0, bwd)
+        assert st == OK and a > 0
+        _, b = ws(2, 8, 32768, 64, 256, 4096, 1, 0, bwd)
+        _, c = ws(2, 8, 65536, 64, 256, 4096, 1, 0, bwd)
+        assert b > a and c == b                    # O(C), independent of L
+        _, big = ws(2, 8, 32768, 64, 256, 32768, 1, 0, bwd)
+        _, half = ws(2, 8, 32768, 64, 256, 16384, 1, 0, bwd)
+        assert 1.8 < big / half < 2.1              # linear in C
+        _, clamp = ws(2, 8, 1000, 64, 256, 5000, 1, 0, bwd)
+        _, same = ws(2, 8, 1000, 64, 256, 1000, 1, 0, bwd)
+        assert clamp == same                       # C > L behaves as C = L
+
+
+@pytest.mark.parametrize("args,code", [
+    ((0, 1, 8, 16, 32, 4), INVALID),     # B < 1
+    ((1, 0, 8, 16, 32, 4), INVALID),     # H < 1
+    ((1, 1, -1, 16, 32, 4), INVALID),    # L < 0
+    ((1, 1, 8, 16, 32, 0), INVALID),     # C < 1
+    ((1, 1, 8, 48, 32, 4), UNSUPPORTED),  # d not in {16, 32, 64, 128}
+    ((1, 1, 8, 16, 24, 4), UNSUPPORTED),  # M not a multiple of 16
+    ((1, 1, 8, 16, 272, 4), UNSUPPORTED),  # M > 256
+])
+def test_workspace_size_rejects(lib, args, code):
+    assert ws(*args)[0] == code
+    assert ws(*args, bwd=True)[0] == code
+
+
+def test_bad_enums_and_null_out(lib):
+    n = ctypes.c_size_t(0)
+    assert lib.slim_fwd_workspace_size(1, 1, 8, 16, 32, 4, 7, 0, ctypes.byref(n)) == INVALID
+    assert lib.slim_fwd_workspace_size(1, 1, 8, 16, 32, 4, 0, 9, ctypes.byref(n)) == INVALID
+    assert lib.slim_fwd_workspace_size(1, 1, 8, 16, 32, 4, 0, 0, None) == INVALID
+
+
+FAKE = 0x10000  # aligned, never dereferenced: every call below fails validation first
+
+
+def fwd_call(lib, ptrs=None, dims=(1, 1, 8, 16, 32, 4), dt=0, ft=0, wsp=FAKE, wsb=0):
+    p = ptrs or [FAKE] * 7
+    return lib.slim_fwd(p[0], p[1], p[2], p[3], *dims, dt, ft, p[4], p[5], p[6], wsp, wsb, None)
+
+
+def bwd_call(lib, ptrs=None, dims=(1, 1, 8, 16, 32, 4), wsp=FAKE, wsb=0):
+    p = ptrs or [FAKE] * 12
+    return lib.slim_bwd(*p[:8], *dims, 0, 0, *p[8:12], wsp, wsb, None)
+
+
+def test_fwd_rejects_before_launch(lib):
+    for i in range(7):
+        ptrs = [FAKE] * 7
+        ptrs[i] = None
+        assert fwd_call(lib, ptrs) == INVALID
+        ptrs[i] = FAKE + 8                      # not 16-byte aligned
+        assert fwd_call(lib, ptrs) == INVALID
+    assert fwd_call(lib, dims=(1, 1, 8, 16, 32, 0)) == INVALID
+    assert fwd_call(lib, dims=(1, 1, 8, 20, 32, 4)) == UNSUPPORTED
+    _, need = ws(1, 1, 8, 16, 32, 4)
+    assert fwd_call(lib, wsb=need - 1) == WORKSPACE
+    assert fwd_call(lib, wsp=None, wsb=need) == WORKSPACE
+    assert fwd_call(lib, wsp=FAKE + 16, wsb=need) == INVALID   # workspace not 256-aligned
+
+
+def test_bwd_rejects_before_launch(lib):
+    for i in range(12):
+        ptrs = [FAKE] * 12
+        ptrs[i] = None
+        assert bwd_call(lib, ptrs) == INVALID
+        ptrs[i] = FAKE + 4
+        assert bwd_call(lib, ptrs) == INVALID
+    _, need = ws(1, 1, 8, 16, 32, 4, bwd=True)
+    assert bwd_call(lib, wsb=need - 1) == WORKSPACE
+    assert bwd_call(lib, dims=(1, 1, 8, 16, 31, 4)) == UNSUPPORTED
+
+
+def test_binding_refuses_cpu_tensors():
+    import torch
+    x = torch.zeros(1, 1, 8, 16)
+    with pytest.raises(RuntimeError):
+        slim.forward(x, x, x, torch.zeros(32, 16), 4)

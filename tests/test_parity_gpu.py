@@ -1,0 +1,210 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Sizes: (1) the small workload exactly; (2) every workload's shape, dtype,
+feature map and distributions at a length the oracle finishes in seconds,
+spanning several tiles and slices with a ragged tail; (3) the full-size
+workloads in the launch configuration the benchmark times, checked on sampled
+chains, on prefixes (rows before L' depend only on rows before L'), and on
+properties that hold at any size.  Tolerances: rel-L2 <= 1e-5 (fp32 inputs)
+and <= 2e-2 (bf16 inputs, fp32 accumulation), per tensor.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import features
+from paper_2012_11346_gb300 import workloads as W
+
+from gpu_common import TOL, compare, cpu_inputs, gpu_run, oracle_run, to64
+
+pytestmark = pytest.mark.gpu
+
+
+def inputs(w, device):
+    return W.make_inputs(w, device=device)
+
+
+def test_tiny_f32_exact_workload(cuda_device):
+    w = W.WORKLOADS["tiny_f32"]
+    x = inputs(w, cuda_device)
+    compare(gpu_run(x, w.C, w.feature), oracle_run(cpu_inputs(x), w.C, w.feature), TOL[w.dtype],
+            where=w.name)
+
+
+SHRUNK = [
+    # name, overrides (several tiles, several slices, ragged last slice)
+    ("L4096_bf16", dict(B=2, H=2, L=2600)),
+    ("L32768_bf16", dict(B=1, H=2, L=4200, C=1024)),
+    ("L8192_relu_f32", dict(B=2, H=3, L=1500)),
+    ("L65536_C16_bf16", dict(B=1, H=2, L=700)),
+]
+
+
+@pytest.mark.parametrize("name,kw", SHRUNK, ids=[s[0] for s in SHRUNK])
+def test_shrunk_workloads(cuda_device, name, kw):
+    w = W.WORKLOADS[name].with_(**kw)
+    x = inputs(w, cuda_device)
+    compare(gpu_run(x, w.C, w.feature), oracle_run(cpu_inputs(x), w.C, w.feature), TOL[w.dtype],
+            where=w.name)
+
+
+@pytest.mark.parametrize("C", W.C_SWEEP)
+def test_c_sweep_shape(cuda_device, C):
+    """The L = 32768 workload's slice sweep, on a shorter sequence (one oracle
+    result, every C compared against it: the result does not depend on C)."""
+    w = W.WORKLOADS["L32768_bf16"].with_(B=1, H=2, L=4100)
+    x = inputs(w, cuda_device)
+    compare(gpu_run(x, C, w.feature), _oracle_cached(w, x), TOL[w.dtype], where=f"C={C}")
+
+
+_CACHE = {}
+
+
+def _oracle_cached(w, x):
+    if w not in _CACHE:
+        _CACHE[w] = oracle_run(cpu_inputs(x), w.C, w.feature)
+    return _CACHE[w]
+
+
+EDGE = [
+    # (d, M, L, C, dtype, feature)
+    (16, 32, 1, 1, "f32", "exp"),
+    (16, 32, 17, 1, "f32", "exp"),
+    (16, 32, 17, 7, "f32", "relu"),
+    (32, 48, 65, 64, "f32", "exp"),
+    (32, 48, 65, 65, "bf16", "exp"),
+    (64, 16, 130, 1000, "f32", "exp"),
+    (64, 128, 200, 33, "bf16", "relu"),
+    (128, 256, 70, 16, "f32", "exp"),
+    (128, 64, 129, 128, "bf16", "exp"),
+]
+
+
+@pytest.mark.parametrize("d,M,L,C,dtype,feature", EDGE)
+def test_edge_shapes(cuda_device, d, M, L, C, dtype, feature):
+    w = W.Workload("edge", 2, 1, L, d, M, C, dtype, feature,
+                   "uniform" if feature == "relu" else "normal", "iid", seed=5)
+    x = inputs(w, cuda_device)
+    compare(gpu_run(x, C, feature), oracle_run(cpu_inputs(x), C, feature), TOL[dtype],
+            where=f"d{d} M{M} L{L} C{C} {dtype} {feature}")
+
+
+def test_empty_sequence(cuda_device):
+    w = W.Workload("empty", 2, 2, 0, 16, 32, 4, "f32", "exp", "normal", "iid")
+    x = inputs(w, cuda_device)
+    g = gpu_run(x, 4, "exp")
+    assert torch.count_nonzero(g["S_state"]) == 0 and torch.count_nonzero(g["z_state"]) == 0
+    assert torch.count_nonzero(g["domega"]) == 0
+
+
+def test_deterministic_and_bwd_leaves_state(cuda_device):
+    w = W.WORKLOADS["L4096_bf16"].with_(B=1, H=4, L=1500, C=256)
+    x = inputs(w, cuda_device)
+    a = gpu_run(x, w.C, w.feature)
+    S0, z0 = a["S_state"].clone(), a["z_state"].clone()
+    b = gpu_run(x, w.C, w.feature)
+    for n in a:
+        assert torch.equal(a[n], b[n]), n
+    from paper_2012_11346_gb300 import slim
+    g2 = slim.backward(x["q"], x["k"], x["v"], x["omega"], a["out"], x["dout"], a["S_state"],
+                       a["z_state"], w.C, w.feature)
+    torch.cuda.synchronize()
+    assert torch.equal(a["S_state"], S0) and torch.equal(a["z_state"], z0)
+    for n, t in zip(("dq", "dk", "dv", "domega"), g2):
+        assert torch.equal(a[n], t), n
+
+
+def test_c_invariance_fp32(cuda_device):
+    """Sec. 4.2: gradients for different C agree up to rounding (the paper saw
+    1e-6..1e-5 in fp32)."""
+    w = W.WORKLOADS["L8192_relu_f32"].with_(B=1, H=2, L=1024)
+    x = inputs(w, cuda_device)
+    ref = gpu_run(x, 1024, w.feature)
+    for C in (1, 16, 100, 512):
+        g = gpu_run(x, C, w.feature)
+        for n in ("out", "dq", "dk", "dv", "domega"):
+            assert oracle.rel_l2(to64(g[n]), to64(ref[n])) < 1e-5, (C, n)
+
+
+def test_autograd_function(cuda_device):
+    from paper_2012_11346_gb300.slim import slim_attention
+    w = W.WORKLOADS["tiny_f32"].with_(B=2, H=2, L=100)
+    x = inputs(w, cuda_device)
+    leaves = {n: x[n].clone().requires_grad_(True) for n in ("q", "k", "v", "omega")}
+    out = slim_attention(leaves["q"], leaves["k"], leaves["v"], leaves["omega"], 16, "exp")
+    (out * x["dout"]).sum().backward()
+    ref = oracle_run(cpu_inputs(x), 16, "exp")
+    for n, r in (("q", "dq"), ("k", "dk"), ("v", "dv"), ("omega", "domega")):
+        assert oracle.rel_l2(to64(leaves[n].grad), ref[r]) < TOL["f32"], n
+
+
+# ----------------------------------------------------------------- full size
+
+def _chain_slice(xc, b, h):
+    return {n: (a[b:b + 1, h:h + 1] if a.ndim == 4 else a) for n, a in xc.items()}
+
+
+def _masked_dout(x, keep):
+    """dout zero outside the chains in `keep` (list of (b, h))."""
+    m = torch.zeros_like(x["dout"])
+    for b, h in keep:
+        m[b, h] = x["dout"][b, h]
+    return m
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["L4096_bf16", "L8192_relu_f32"])
+def test_full_size_sampled_chains(cuda_device, name):
+    """Full workload, benchmark launch configuration; the oracle recomputes two
+    chains.  dOmega (a sum over all chains) is checked on a second backward
+    whose dout is zero outside the sampled chains."""
+    w = W.WORKLOADS[name]
+    x = inputs(w, cuda_device)
+    g = gpu_run(x, w.C, w.feature)
+    xc = cpu_inputs(x)
+    keep = [(0, 0), (w.B - 1, w.H - 1)]
+    tol = TOL[w.dtype]
+    for b, h in keep:
+        ref = oracle_run(_chain_slice(xc, b, h), w.C, w.feature)
+        sub = {n: g[n][b:b + 1, h:h + 1] for n in ("out", "S_state", "z_state", "dq", "dk", "dv")}
+        compare(sub, ref, tol, names=tuple(sub), where=f"{name} chain ({b},{h})")
+    gm = gpu_run(x, w.C, w.feature, dout=_masked_dout(x, keep))
+    dom = sum(oracle_run(_chain_slice(xc, b, h), w.C, w.feature)["domega"] for b, h in keep)
+    assert oracle.rel_l2(to64(gm["domega"]), dom) <= tol
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name,Lp", [("L32768_bf16", 3000), ("L65536_C16_bf16", 1500)])
+def test_full_size_prefix_and_state(cuda_device, name, Lp):
+    """Long workloads at full size.  (a) Rows before L' depend only on rows
+    before L' (causal mask): they match the oracle on the prefix.  (b) The final
+    state is the closed form S = g(K)^T V, z = sum g(K) (eq. 3, last row).
+    (c) With dout zero from row L' on, all gradients equal those of the
+    prefix problem and rows from L' on get zero gradient."""
+    w = W.WORKLOADS[name]
+    x = inputs(w, cuda_device)
+    tol = TOL[w.dtype]
+    dmask = x["dout"].clone()
+    dmask[:, :, Lp:] = 0
+    g = gpu_run(x, w.C, w.feature, dout=dmask)
+    xc = cpu_inputs(x)
+    pre = {n: (a[:1, :1, :Lp] if a.ndim == 4 else a) for n, a in xc.items()}
+    ref = oracle_run(pre, w.C, w.feature)
+    sub = {n: g[n][:1, :1, :Lp] for n in ("out", "dq", "dk", "dv")}
+    compare(sub, ref, tol, names=tuple(sub), where=f"{name} prefix")
+    for n in ("dq", "dk", "dv"):
+        assert torch.count_nonzero(g[n][:, :, Lp:]) == 0, n
+    # dOmega: every chain's prefix contributes; the oracle sums chain 0 only, so
+    # compare chain-0-only dout
+    dm0 = torch.zeros_like(dmask)
+    dm0[0, 0] = dmask[0, 0]
+    g0 = gpu_run(x, w.C, w.feature, dout=dm0)
+    assert oracle.rel_l2(to64(g0["domega"]), ref["domega"]) <= tol
+    # closed-form final state, every chain
+    Kt = features.feature_map(xc["k"].reshape(-1, w.L, w.d), xc["omega"], w.feature)
+    V = xc["v"].reshape(-1, w.L, w.d)
+    S_cf = np.einsum("clm,cld->cmd", Kt, V).reshape(w.B, w.H, w.M, w.d)
+    z_cf = Kt.sum(axis=1).reshape(w.B, w.H, w.M)
+    assert oracle.rel_l2(to64(g["S_state"]), S_cf) <= tol
+    assert oracle.rel_l2(to64(g["z_state"]), z_cf) <= tol
