@@ -251,7 +251,7 @@ def _oracle_chain(args):
 
 
 def oracle_pool_size():
-    return max(1, min(len(os.sched_getaffinity(0)), 8))
+    return max(1, min(len(os.sched_getaffinity(0)), 16))
 
 
 def oracle_sample(w, overrides, pool, nchains):

@@ -28,7 +28,8 @@
  *
  * Conventions for every entry point
  *   - All tensor pointers are DEVICE pointers, contiguous, row-major, 16-byte
- *     aligned.  q, k, v, out, dout, dq, dk, dv are [B, H, L, d] in `dtype`;
+ *     aligned, and non-null -- except that when L = 0 the (empty) [B, H, L, d]
+ *     tensors may be null.  q, k, v, out, dout, dq, dk, dv are [B, H, L, d] in `dtype`;
  *     omega and domega are [M, d] fp32; S_state is [B, H, M, d] fp32 and
  *     z_state is [B, H, M] fp32.
  *   - The caller owns every buffer.  The library allocates no device or host
@@ -39,8 +40,10 @@
  *     nothing has been launched, except SLIM_ERR_CUDA (a launch failed part
  *     way; outputs are then undefined).
  *   - 1 <= C; C > L behaves as C = L.  L % C != 0 gives a shorter last slice.
- *   - Outputs are written in `dtype` rounded to nearest even; accumulation and
- *     the carried state are fp32 (the state as an fp32 value/error pair).
+ *   - Outputs are written in `dtype` rounded to nearest even; the carried
+ *     state is an fp32 value/error pair.  fp32 problems accumulate every
+ *     contraction in compensated fp32 (error-free products and sums); bf16
+ *     problems accumulate in fp32.
  *   - Supported: d in {16, 32, 64, 128}; M a multiple of 16 in [16, 256];
  *     dtype SLIM_F32 or SLIM_BF16; both feature maps.  Other combinations
  *     return SLIM_ERR_UNSUPPORTED.

@@ -62,7 +62,14 @@ struct GemmP {
 };
 
 // C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z.  256 threads,
-// 64 x 64 outputs per CTA, 4 x 4 per thread, fp32 FMA.
+// 64 x 64 outputs per CTA, 4 x 4 per thread.  PRECISE = false: fp32 FMA.
+// PRECISE = true (fp32 problems): every product and sum is error-free
+// transformed (FMA-based TwoProduct, Knuth TwoSum) and the errors are
+// accumulated beside the sum, so the result is as accurate as a sum computed
+// in twice the working precision and rounded once.  The backward pass needs
+// it: its contractions cancel (signed feature gradients summed against
+// Omega), which multiplies plain fp32 rounding error by 10-30.
+template <bool PRECISE>
 __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
   __shared__ __align__(16) float As[GK][GT + 4];
   __shared__ __align__(16) float Bs[GK][GT + 4];
@@ -72,11 +79,11 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
   const float* Bm = P.b.p + z0 * P.b.b0 + z1 * P.b.b1;
   const int i0 = blockIdx.y * GT, j0 = blockIdx.x * GT;
   const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
-  float acc[4][4];
+  float acc[4][4], err[4][4];
 #pragma unroll
   for (int r = 0; r < 4; ++r)
 #pragma unroll
-    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+    for (int c = 0; c < 4; ++c) acc[r][c] = err[r][c] = 0.f;
 
   for (int k0 = 0; k0 < P.k; k0 += GK) {
     if (P.a.cs == 1) {  // k contiguous
@@ -111,7 +118,18 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
 #pragma unroll
       for (int r = 0; r < 4; ++r)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
+        for (int c = 0; c < 4; ++c) {
+          if (PRECISE) {
+            const float p = __fmul_rn(a[r], b[c]);
+            const float ep = __fmaf_rn(a[r], b[c], -p);
+            float sum, es;
+            two_sum(acc[r][c], p, sum, es);
+            acc[r][c] = sum;
+            err[r][c] = __fadd_rn(err[r][c], __fadd_rn(es, ep));
+          } else {
+            acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
+          }
+        }
     }
     __syncthreads();
   }
@@ -125,7 +143,7 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
     for (int c = 0; c < 4; ++c) {
       const int j = j0 + tx * 4 + c;
       if (j >= P.n) continue;
-      float v = acc[r][c];
+      float v = PRECISE ? __fadd_rn(acc[r][c], err[r][c]) : acc[r][c];
       if (P.causal && j > i) v = 0.f;
       if (P.sx) v -= P.sx[z0 * P.sx_b0 + i * P.sx_rs + j] * P.ss[z0 * P.ss_b0 + i];
       float* dst = Cm + i * P.c.rs + j * P.c.cs;
@@ -372,6 +390,7 @@ namespace {
 
 struct Geo {
   int chains, d, dp, M, Cs, T, nt, Cp, N;
+  bool precise;  // fp32 problems: compensated contractions
 };
 
 Geo geometry(const Problem& p) {
@@ -386,6 +405,7 @@ Geo geometry(const Problem& p) {
   g.nt = (g.Cs + g.T - 1) / g.T;
   g.Cp = g.nt * g.T;
   g.N = p.num_slices();
+  g.precise = p.dtype == SLIM_F32;
   return g;
 }
 
@@ -435,7 +455,8 @@ OutMat omat(float* p, long long b0, long long b1, long long rs, long long cs) {
   return OutMat{p, b0, b1, rs, cs};
 }
 
-cudaError_t gemm(cudaStream_t s, int m, int n, int k, Mat a, Mat b, OutMat c, int nb0, int nb1,
+cudaError_t gemm(cudaStream_t s, bool precise, int m, int n, int k, Mat a, Mat b, OutMat c,
+                 int nb0, int nb1,
                  float beta, int causal, const float* sx = nullptr, long long sx_b0 = 0,
                  long long sx_rs = 0, const float* ss = nullptr, long long ss_b0 = 0) {
   const int nz = nb0 * nb1;
@@ -444,7 +465,10 @@ cudaError_t gemm(cudaStream_t s, int m, int n, int k, Mat a, Mat b, OutMat c, in
     const int zc = (nz - z < 65535) ? nz - z : 65535;
     dim3 grid((n + GT - 1) / GT, (m + GT - 1) / GT, zc);
     prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
-    k_gemm<<<grid, 256, 0, s>>>(P);
+    if (precise)
+      k_gemm<true><<<grid, 256, 0, s>>>(P);
+    else
+      k_gemm<false><<<grid, 256, 0, s>>>(P);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -487,22 +511,22 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
 // Delta_t = phiK_t^T [V_t | 1]  (M x dp per tile)
 cudaError_t tile_deltas(cudaStream_t s, const Geo& g, const Ws& w) {
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
-  return gemm(s, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
+  return gemm(s, g.precise, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
               omat(w.delta, nt * M * dp, M * dp, dp, 1), g.chains, g.nt, 0.f, 0);
 }
 
 // A_t = tril(phiQ_t phiK_t^T); [num | den] = phiQ_t P_t + A_t [V_t | 1]
 cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w) {
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
-  cudaError_t e = gemm(s, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+  cudaError_t e = gemm(s, g.precise, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                        mat(w.phiK, Cp * M, T * M, 1, M), omat(w.A, nt * T * T, T * T, T, 1),
                        g.chains, g.nt, 0.f, 1);
   if (e != cudaSuccess) return e;
-  e = gemm(s, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+  e = gemm(s, g.precise, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
            mat(w.delta, nt * M * dp, M * dp, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
            g.chains, g.nt, 0.f, 0);
   if (e != cudaSuccess) return e;
-  return gemm(s, g.T, g.dp, g.T, mat(w.A, nt * T * T, T * T, T, 1),
+  return gemm(s, g.precise, g.T, g.dp, g.T, mat(w.A, nt * T * T, T * T, T, 1),
               mat(w.Vx, Cp * dp, T * dp, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
               g.chains, g.nt, 1.f, 0);
 }
@@ -576,33 +600,33 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
                                                                g.d, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
     // dA_t = tril(W_t [V_t | 1]^T)
-    SLIM_TRY(gemm(s, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.Vx, Cp * dp, T * dp, 1, dp), omat(w.dA, nt * T * T, T * T, T, 1),
                   g.chains, g.nt, 0.f, 1));
     // dphiQ = W_t P_t^T + dA_t phiK_t
-    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.delta, nt * M * dp, M * dp, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
                   mat(w.phiK, Cp * M, T * M, M, 1), omat(w.dphiQ, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 1.f, 0));
     // Gd_t = phiQ_t^T W_t, then G_t = G + sum_{t' > t} Gd_t'
-    SLIM_TRY(gemm(s, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+    SLIM_TRY(gemm(s, g.precise, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
     // dphiK = dA_t^T phiQ_t + [V_t | 1] G_t^T
-    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
                   mat(w.phiQ, Cp * M, T * M, M, 1), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
                   mat(w.gdelta, nt * M * dp, M * dp, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 1.f, 0));
     // dV = A_t^T dnum + phiK_t G_t(S)
-    SLIM_TRY(gemm(s, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.precise, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
                   mat(w.gdelta, nt * M * dp, M * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1),
                   g.chains, g.nt, 1.f, 0));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
@@ -621,14 +645,14 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(cudaGetLastError());
     const bool ex = p.feature == SLIM_FEAT_EXP;
     // dX = u Omega (- x sum u for the exp map)
-    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    SLIM_TRY(gemm(s, g.precise, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
                   omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xq : nullptr,
                   Cp * d, d, w.usum_q, Cp));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
     k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dq, p.L, g.d,
                                                                       a, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
-    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    SLIM_TRY(gemm(s, g.precise, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
                   omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xk : nullptr,
                   Cp * d, d, w.usum_k, Cp));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
@@ -636,9 +660,9 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
                                                                       a, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
     // dOmega partial per chain: u_q^T x_q + u_k^T x_k
-    SLIM_TRY(gemm(s, g.M, g.d, g.Cp, mat(w.dphiQ, Cp * M, 0, 1, M), mat(w.Xq, Cp * d, 0, d, 1),
+    SLIM_TRY(gemm(s, g.precise, g.M, g.d, g.Cp, mat(w.dphiQ, Cp * M, 0, 1, M), mat(w.Xq, Cp * d, 0, d, 1),
                   omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 0.f, 0));
-    SLIM_TRY(gemm(s, g.M, g.d, g.Cp, mat(w.dphiK, Cp * M, 0, 1, M), mat(w.Xk, Cp * d, 0, d, 1),
+    SLIM_TRY(gemm(s, g.precise, g.M, g.d, g.Cp, mat(w.dphiK, Cp * M, 0, 1, M), mat(w.Xk, Cp * d, 0, d, 1),
                   omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 1.f, 0));
     { prof::Scope ps(prof::K_REDUCE, s);
     k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains,

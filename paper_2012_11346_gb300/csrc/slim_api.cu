@@ -13,6 +13,17 @@ constexpr int kVersion = 100;  // 0.1.0
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+bool pointers_ok(const void* const* ptrs, int n, bool null_allowed) {
+  for (int i = 0; i < n; ++i) {
+    if (ptrs[i] == nullptr) {
+      if (!null_allowed) return false;
+    } else if (!aligned16(ptrs[i])) {
+      return false;
+    }
+  }
+  return true;
+}
+
 slim_status check_problem(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
                           slim_feature feature, Problem* out) {
   if (B < 1 || H < 1 || L < 0 || C < 1) return SLIM_ERR_INVALID_ARG;
@@ -84,9 +95,10 @@ slim_status slim_fwd(const void* q, const void* k, const void* v, const float* o
   Problem p;
   slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
   if (st != SLIM_OK) return st;
-  const void* ptrs[] = {q, k, v, omega, out, S_state, z_state};
-  for (const void* ptr : ptrs)
-    if (ptr == nullptr || !aligned16(ptr)) return SLIM_ERR_INVALID_ARG;
+  // [B,H,L,d] tensors are empty when L = 0 and may then be null
+  const void* seq[] = {q, k, v, out};
+  const void* fixed[] = {omega, S_state, z_state};
+  if (!pointers_ok(seq, 4, L == 0) || !pointers_ok(fixed, 3, false)) return SLIM_ERR_INVALID_ARG;
   st = check_workspace(p, false, workspace, workspace_bytes);
   if (st != SLIM_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -107,9 +119,9 @@ slim_status slim_bwd(const void* q, const void* k, const void* v, const float* o
   Problem p;
   slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
   if (st != SLIM_OK) return st;
-  const void* ptrs[] = {q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv, domega};
-  for (const void* ptr : ptrs)
-    if (ptr == nullptr || !aligned16(ptr)) return SLIM_ERR_INVALID_ARG;
+  const void* seq[] = {q, k, v, out, dout, dq, dk, dv};
+  const void* fixed[] = {omega, S_state, z_state, domega};
+  if (!pointers_ok(seq, 8, L == 0) || !pointers_ok(fixed, 4, false)) return SLIM_ERR_INVALID_ARG;
   st = check_workspace(p, true, workspace, workspace_bytes);
   if (st != SLIM_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -1,0 +1,209 @@
+// Blackwell (sm_103a) tensor-core building blocks for libslim, in inline PTX:
+// mbarriers with bounded waits, tcgen05 TMEM allocation / MMA / commit / load,
+// 128-byte-swizzled shared-memory operand layouts and their descriptors.
+//
+// Operand tiles.  Every bf16 operand lives in shared memory as "row tiles":
+// a row-major [R][64] block, 128 bytes per row, 1024-byte aligned, with the
+// 16-byte chunk c of row r stored at chunk position c ^ (r % 8) (the 128B
+// swizzle).  A matrix with more than 64 columns is a sequence of such blocks
+// (columns 64b..64b+63 in block b, blocks R*128 bytes apart).  The same bytes
+// serve as
+//   * a K-major operand (rows = M or N index, columns = K), and
+//   * an MN-major operand (columns = M or N index, rows = K),
+// which only changes the descriptor:
+//   K-major : start + 32 B per 16-element K step inside a block, next block
+//             for the next 64 K; SBO = 1024 B (8 rows), LBO unused.
+//   MN-major: start + 2048 B per 16-element K step (16 rows); LBO = byte
+//             distance between 64-column blocks, SBO = 1024 B (8 K rows).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace slim {
+namespace tc {
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ------------------------------------------------------------------ mbarrier
+__device__ __forceinline__ void mbar_init(uint32_t addr, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(addr), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait: gives up after ~2^22 polls (well over a second with the
+// back-off), records the failure in *err and returns false.
+__device__ __forceinline__ bool mbar_wait(uint32_t addr, uint32_t parity, int* err) {
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    if (mbar_try_wait(addr, parity)) return true;
+    if (i > 16) __nanosleep(256);
+  }
+  if (err) atomicExch(err, 1);
+  return false;
+}
+
+// ------------------------------------------------------------------ proxies / fences
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// ------------------------------------------------------------------ TMEM
+// Executed by one whole warp.  Writes the TMEM base address to smem.
+__device__ __forceinline__ void tmem_alloc(uint32_t smem_dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_dst),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane (warp w reads lanes
+// 32w..32w+31; `taddr` carries the lane base in bits 31:16).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_ld1(uint32_t taddr, float& v) {
+  uint32_t r;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+  v = __uint_as_float(r);
+}
+
+// ------------------------------------------------------------------ MMA
+// Instruction descriptor, kind::f16 with bf16 A/B and fp32 accumulate.
+// a_mn / b_mn = 1 selects the MN-major (transposed) operand layout.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;  // descriptor version of tcgen05
+  d |= (uint64_t)2 << 61;  // 128-byte swizzle
+  return d;
+}
+// K-major operand stored as row tiles of `rows` rows: element (row, k0..k0+15).
+__device__ __forceinline__ uint64_t kmaj(uint32_t base, int rows, int k0) {
+  return sdesc(base + (uint32_t)((k0 >> 6) * rows * 128 + (k0 & 63) * 2), 16, 1024);
+}
+// MN-major operand stored as row tiles whose rows are K and columns MN:
+// K rows k0..k0+15, MN blocks `block_bytes` apart.
+__device__ __forceinline__ uint64_t mnmaj(uint32_t base, int k0, uint32_t block_bytes) {
+  return sdesc(base + (uint32_t)(k0 * 128), block_bytes, 1024);
+}
+
+// D[tmem] (+)= A * B, issued by a single thread.
+__device__ __forceinline__ void mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                    uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the mbarrier once every MMA issued so far by this thread is done.
+__device__ __forceinline__ void mma_commit(uint32_t mbar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar)
+      : "memory");
+}
+
+// ------------------------------------------------------------------ tile memory
+// Byte offset of element (r, c) inside a row tile with R rows (c may exceed 63).
+__device__ __forceinline__ uint32_t tile_off(int R, int r, int c) {
+  return (uint32_t)((c >> 6) * R * 128 + r * 128 + ((((c & 63) >> 3) ^ (r & 7)) << 4) +
+                    (c & 7) * 2);
+}
+// Stores 8 consecutive bf16 (one 16-byte chunk, c multiple of 8).
+__device__ __forceinline__ void st_chunk(uint8_t* tile, int R, int r, int c, uint4 v) {
+  *reinterpret_cast<uint4*>(tile + tile_off(R, r, c)) = v;
+}
+__device__ __forceinline__ uint4 ld_chunk(const uint8_t* tile, int R, int r, int c) {
+  return *reinterpret_cast<const uint4*>(tile + tile_off(R, r, c));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ void unpack_bf16(uint32_t u, float& lo, float& hi) {
+  __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&u);
+  lo = __low2float(h);
+  hi = __high2float(h);
+}
+
+// cp.async of one 16-byte chunk; src_bytes = 0 zero-fills the destination.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+// Loads rows [0, R) of a row-major [.][64] bf16 global matrix (row stride 64
+// elements) into a row tile; rows >= valid are zero.  All `nthreads` threads
+// of the CTA take part; completes with cp_async_wait_all().
+__device__ __forceinline__ void load_rows64(uint8_t* tile, int R, const __nv_bfloat16* g,
+                                            int valid, int tid, int nthreads) {
+  const uint32_t base = smem_u32(tile);
+  for (int e = tid; e < R * 8; e += nthreads) {
+    const int r = e >> 3, c = (e & 7) * 8;
+    const bool ok = r < valid;
+    const __nv_bfloat16* src = g + (size_t)(ok ? r : 0) * 64 + c;
+    cp_async16(base + tile_off(R, r, c), src, ok ? 16u : 0u);
+  }
+}
+
+// ex2 on the MUFU unit (approximate, ~2 ulp), used for the FAVOR+ features.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+}  // namespace tc
+}  // namespace slim

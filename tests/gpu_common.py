@@ -35,11 +35,20 @@ def oracle_run(xc, C, feature, dout=None):
             "extra": extra}
 
 
-def compare(gpu, ref, tol, names=NAMES, where=""):
+def compare(gpu, ref, tol, names=NAMES, where="", scale=None):
+    """rel-L2 per tensor.  A reference that vanishes identically (e.g. dq and
+    dk for L = 1, where out_1 = v_1 does not depend on q or k) has no relative
+    error; there the error is taken relative to `scale` (the gradient scale,
+    e.g. ||dout||) instead."""
     errs = {}
     for n in names:
         g = to64(gpu[n]) if torch.is_tensor(gpu[n]) else np.asarray(gpu[n])
-        errs[n] = oracle.rel_l2(g, ref[n])
+        r = np.asarray(ref[n], dtype=np.float64)
+        nr = np.linalg.norm(r.ravel())
+        if scale is not None and nr <= 1e-9 * scale:
+            errs[n] = float(np.linalg.norm((g - r).ravel()) / scale)
+        else:
+            errs[n] = oracle.rel_l2(g, r)
     bad = {n: e for n, e in errs.items() if not (e <= tol)}
     assert not bad, f"{where} rel-L2 above {tol}: {bad} (all: {errs})"
     return errs

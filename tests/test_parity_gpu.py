@@ -86,8 +86,10 @@ def test_edge_shapes(cuda_device, d, M, L, C, dtype, feature):
     w = W.Workload("edge", 2, 1, L, d, M, C, dtype, feature,
                    "uniform" if feature == "relu" else "normal", "iid", seed=5)
     x = inputs(w, cuda_device)
-    compare(gpu_run(x, C, feature), oracle_run(cpu_inputs(x), C, feature), TOL[dtype],
-            where=f"d{d} M{M} L{L} C{C} {dtype} {feature}")
+    xc = cpu_inputs(x)
+    compare(gpu_run(x, C, feature), oracle_run(xc, C, feature), TOL[dtype],
+            where=f"d{d} M{M} L{L} C{C} {dtype} {feature}",
+            scale=float(np.linalg.norm(xc["dout"].ravel())))
 
 
 def test_empty_sequence(cuda_device):
