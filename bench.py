@@ -286,6 +286,7 @@ def run_ours(args, rank, ws, local):
     out = torch.empty_like(q)
     S = torch.empty(B, H, M, d, dtype=torch.float32, device=dev)
     z = torch.empty(B, H, M, dtype=torch.float32, device=dev)
+    S_lo, z_lo = torch.empty_like(S), torch.empty_like(z)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dom = torch.empty(M, d, dtype=torch.float32, device=dev)
     wsf = torch.empty(max(256, slim.workspace_size(B, H, L, d, M, w.C, q.dtype, w.feature, False)),
@@ -294,8 +295,9 @@ def run_ours(args, rank, ws, local):
                       dtype=torch.uint8, device=dev)
 
     def step():
-        slim.forward_into(q, k, v, om, w.C, w.feature, out, S, z, wsf)
-        slim.backward_into(q, k, v, om, out, dout, S, z, w.C, w.feature, dq, dk, dv, dom, wsb)
+        slim.forward_into(q, k, v, om, w.C, w.feature, out, S, z, wsf, S_lo=S_lo, z_lo=z_lo)
+        slim.backward_into(q, k, v, om, out, dout, S, z, w.C, w.feature, dq, dk, dv, dom, wsb,
+                           S_lo=S_lo, z_lo=z_lo)
 
     for _ in range(args.warmup):
         step()
@@ -358,11 +360,11 @@ def run_ours(args, rank, ws, local):
     torch.cuda.synchronize()
     torch.cuda.reset_peak_memory_stats(dev)
     base = torch.cuda.memory_allocated(dev)
-    o2, S2, z2 = slim.forward(q, k, v, om, w.C, w.feature)
-    g2 = slim.backward(q, k, v, om, o2, dout, S2, z2, w.C, w.feature)
+    o2, S2, z2, S2l, z2l = slim.forward(q, k, v, om, w.C, w.feature, residuals=True)
+    g2 = slim.backward(q, k, v, om, o2, dout, S2, z2, w.C, w.feature, S_lo=S2l, z_lo=z2l)
     torch.cuda.synchronize()
     peak = torch.cuda.max_memory_allocated(dev)
-    del o2, S2, z2, g2
+    del o2, S2, z2, S2l, z2l, g2
 
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws,
@@ -453,8 +455,10 @@ def run_sweep(args, local):
         w = w0.with_(C=C)
 
         def step():
-            o, S, z = slim.forward(x["q"], x["k"], x["v"], x["omega"], C, w.feature)
-            slim.backward(x["q"], x["k"], x["v"], x["omega"], o, x["dout"], S, z, C, w.feature)
+            o, S, z, Sl, zl = slim.forward(x["q"], x["k"], x["v"], x["omega"], C, w.feature,
+                                           residuals=True)
+            slim.backward(x["q"], x["k"], x["v"], x["omega"], o, x["dout"], S, z, C, w.feature,
+                          S_lo=Sl, z_lo=zl)
 
         for _ in range(max(1, args.warmup)):
             step()

@@ -97,6 +97,12 @@ slim_status slim_bwd_workspace_size(int B, int H, int L, int d, int M, int C,
  *   out       [B,H,L,d] dtype, written: eq. 2 for every row.
  *   S_state   [B,H,M,d] fp32, written: final state S^(N) = sum_j g(k_j) v_j^T.
  *   z_state   [B,H,M]   fp32, written: final state z^(N) = sum_j g(k_j).
+ *   S_state_lo, z_state_lo  same shapes, written if non-NULL: the low-order
+ *             residual of the carried fp32 value/error pair (state = S_state +
+ *             S_state_lo to about 48 bits).  Passing them back to slim_bwd
+ *             lets the rollback of eq. 17 start from the unrounded state; an
+ *             fp32-rounded z^(N) alone perturbs the early rows' denominators,
+ *             which are small next to z^(N), by ~6e-8 * z^(N).
  *   workspace device scratch of at least slim_fwd_workspace_size() bytes,
  *             256-byte aligned; contents on entry are ignored.
  * L = 0 is valid and only zeroes S_state / z_state.
@@ -105,6 +111,7 @@ slim_status slim_fwd(const void* q, const void* k, const void* v, const float* o
                      int B, int H, int L, int d, int M, int C,
                      slim_dtype dtype, slim_feature feature,
                      void* out, float* S_state, float* z_state,
+                     float* S_state_lo, float* z_state_lo,
                      void* workspace, size_t workspace_bytes, void* stream);
 
 /*
@@ -117,6 +124,8 @@ slim_status slim_fwd(const void* q, const void* k, const void* v, const float* o
  *   S_state, z_state  read-only: the final state B^(N) slim_fwd returned; the
  *              reverse walk starts from it and rolls it back slice by slice.
  *              Not modified, so a second call gives the same result.
+ *   S_state_lo, z_state_lo  read-only, may be NULL (then taken as zero): the
+ *              residuals slim_fwd wrote.
  *   dq, dk, dv [B,H,L,d] dtype, written.
  *   domega     [M,d] fp32, written (sum over all chains, queries and keys).
  *   workspace  at least slim_bwd_workspace_size() bytes, 256-byte aligned.
@@ -126,10 +135,22 @@ slim_status slim_fwd(const void* q, const void* k, const void* v, const float* o
 slim_status slim_bwd(const void* q, const void* k, const void* v, const float* omega,
                      const void* out, const void* dout,
                      const float* S_state, const float* z_state,
+                     const float* S_state_lo, const float* z_state_lo,
                      int B, int H, int L, int d, int M, int C,
                      slim_dtype dtype, slim_feature feature,
                      void* dq, void* dk, void* dv, float* domega,
                      void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Which kernels serve this problem: *path = 1 for the tensor-core path
+ * (tcgen05 MMAs, bf16 operands, fp32 accumulation; bf16 inputs with d = 64,
+ * M in {128, 256} and slices of at least 64 rows), 0 for the fp32-compute
+ * path (every other supported problem).  Setting the environment variable
+ * SLIM_PATH=simt (read on every call) selects the fp32-compute path for every
+ * problem.  Pure host computation.
+ */
+slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                          slim_feature feature, int* path);
 
 /*
  * Reads the device error word that bounded waits in the kernels set when they
@@ -165,6 +186,18 @@ unsigned long long slim_launch_count(void);
 void slim_profiler_enable(int on);
 void slim_profiler_reset(void);
 int slim_profiler_read(slim_kernel_stats* stats, int cap);
+
+/*
+ * Diagnostic of the tensor-core building blocks (no counterpart in the
+ * paper): one CTA computes D = A x B with a single chain of tcgen05 MMAs,
+ * the operands staged in 128-byte-swizzled shared memory in K-major (0) or
+ * MN-major (1) layout, so a caller can compare D against a reference.
+ *   A  [128, K] bf16 row-major device; B [K, N] bf16 row-major device;
+ *   D  [128, N] fp32 row-major device (written); err: device int, set to 1 if
+ *   the MMA completion wait gave up.  K, N in {64, 128, 256}.
+ */
+slim_status slim_tc_selftest(int a_mn, int b_mn, int K, int N, const void* A, const void* B,
+                             float* D, int* err, void* stream);
 
 #ifdef __cplusplus
 }

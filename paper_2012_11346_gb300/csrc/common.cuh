@@ -70,4 +70,13 @@ struct Problem {
   int num_slices() const { int c = slice_len(); return L == 0 ? 0 : (L + c - 1) / c; }
 };
 
+// Final state handed from the forward to the backward: fp32 values plus the
+// optional low-order residuals of the carried value/error pair.
+struct StateOut {
+  float *S, *z, *S_lo, *z_lo;
+};
+struct StateIn {
+  const float *S, *z, *S_lo, *z_lo;
+};
+
 }  // namespace slim

@@ -23,6 +23,8 @@ enum Kid {
   K_TC_BWD_Q,
   K_TC_BWD_KV,
   K_TC_REDUCE,
+  K_TC_SELFTEST,
+  K_TC_PREP,
   K_COUNT
 };
 

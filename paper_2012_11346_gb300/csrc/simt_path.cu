@@ -28,6 +28,7 @@
 
 #include "common.cuh"
 #include "profiler.h"
+#include "scan.h"
 #include "simt_path.h"
 
 namespace slim {
@@ -261,43 +262,6 @@ __global__ void __launch_bounds__(256) k_prep(
   }
 }
 
-// State scans over the tiles of one slice, one thread per (chain, element).
-enum ScanMode { SCAN_FWD = 0, SCAN_ROLLBACK = 1, SCAN_GREV = 2 };
-
-__global__ void k_scan(float* buf, float* hi_p, float* lo_p, int chains, int nt, int E, int mode) {
-  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (long long)chains * E) return;
-  const int c = (int)(idx / E), e = (int)(idx % E);
-  float hi = hi_p[idx], lo = lo_p[idx];
-  float* col = buf + (size_t)c * nt * E + e;
-  if (mode == SCAN_GREV) {
-    // G_t = G + sum_{t' > t} Gd_t'  (reversed prefix sum), then G += all
-    for (int t = nt - 1; t >= 0; --t) {
-      float x = col[(size_t)t * E];
-      col[(size_t)t * E] = hi + lo;
-      pair_add(hi, lo, x);
-    }
-    hi_p[idx] = hi;
-    lo_p[idx] = lo;
-    return;
-  }
-  if (mode == SCAN_ROLLBACK) {
-    // eq. 17: B^(n-1) = B^(n) - sum_t Delta_t, undone in reverse order
-    for (int t = nt - 1; t >= 0; --t) pair_add(hi, lo, -col[(size_t)t * E]);
-    hi_p[idx] = hi;
-    lo_p[idx] = lo;
-  }
-  for (int t = 0; t < nt; ++t) {
-    float x = col[(size_t)t * E];
-    col[(size_t)t * E] = hi + lo;
-    pair_add(hi, lo, x);
-  }
-  if (mode == SCAN_FWD) {
-    hi_p[idx] = hi;
-    lo_p[idx] = lo;
-  }
-}
-
 template <typename T>
 __global__ void k_finalize_out(const float* numden, T* out, int L, int d, int a, int b, int Cp,
                                int chains) {
@@ -362,27 +326,37 @@ __global__ void k_reduce_domega(const float* part, float* domega, int chains, in
   domega[e] += s;
 }
 
-__global__ void k_state_out(const float* hi, const float* lo, float* S_state, float* z_state,
-                            int chains, int M, int d) {
+// The pair is kept normalised (|lo| <= ulp(hi)/2), so hi is the rounded state
+// and lo its residual.
+__global__ void k_state_out(const float* hi, const float* lo, StateOut st, int chains, int M,
+                            int d) {
   const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const int dp = d + 1;
   if (idx >= (long long)chains * M * dp) return;
   const int j = (int)(idx % dp);
   const long long cm = idx / dp;
-  const float x = hi[idx] + lo[idx];
-  if (j < d) S_state[cm * d + j] = x;
-  else z_state[cm] = x;
+  if (j < d) {
+    st.S[cm * d + j] = hi[idx];
+    if (st.S_lo) st.S_lo[cm * d + j] = lo[idx];
+  } else {
+    st.z[cm] = hi[idx];
+    if (st.z_lo) st.z_lo[cm] = lo[idx];
+  }
 }
 
-__global__ void k_state_in(const float* S_state, const float* z_state, float* hi, float* lo,
-                           int chains, int M, int d) {
+__global__ void k_state_in(StateIn st, float* hi, float* lo, int chains, int M, int d) {
   const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const int dp = d + 1;
   if (idx >= (long long)chains * M * dp) return;
   const int j = (int)(idx % dp);
   const long long cm = idx / dp;
-  hi[idx] = (j < d) ? S_state[cm * d + j] : z_state[cm];
-  lo[idx] = 0.f;
+  if (j < d) {
+    hi[idx] = st.S[cm * d + j];
+    lo[idx] = st.S_lo ? st.S_lo[cm * d + j] : 0.f;
+  } else {
+    hi[idx] = st.z[cm];
+    lo[idx] = st.z_lo ? st.z_lo[cm] : 0.f;
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -531,17 +505,14 @@ cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w) {
               g.chains, g.nt, 1.f, 0);
 }
 
-cudaError_t scan(cudaStream_t s, const Geo& g, float* buf, float* hi, float* lo, int mode) {
-  const long long E = (long long)g.M * g.dp;
-  prof::Scope ps(prof::K_SCAN, s);
-  k_scan<<<blocks(g.chains * E), 256, 0, s>>>(buf, hi, lo, g.chains, g.nt, (int)E, mode);
-  return cudaGetLastError();
+cudaError_t scan(cudaStream_t s, const Geo& g, float* buf, float* hi, float* lo, ScanMode mode) {
+  return launch_scan(s, buf, hi, lo, g.chains, g.nt, g.M * g.dp, mode, prof::K_SCAN);
 }
 
 template <typename T>
 slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void* v,
-                     const float* omega, void* out, float* S_state, float* z_state,
-                     void* workspace, cudaStream_t s) {
+                     const float* omega, void* out, const StateOut& st, void* workspace,
+                     cudaStream_t s) {
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, false);
@@ -562,7 +533,7 @@ slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void*
   }
   {
     prof::Scope ps(prof::K_STATE, s);
-    k_state_out<<<blocks((long long)E), 256, 0, s>>>(w.st_hi, w.st_lo, S_state, z_state,
+    k_state_out<<<blocks((long long)E), 256, 0, s>>>(w.st_hi, w.st_lo, st,
                                                      g.chains, g.M, g.d);
   }
   SLIM_TRY(cudaGetLastError());
@@ -572,7 +543,7 @@ slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void*
 template <typename IO>
 slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void* v,
                      const float* omega, const void* out, const void* dout,
-                     const float* S_state, const float* z_state, void* dq, void* dk, void* dv,
+                     const StateIn& st, void* dq, void* dk, void* dv,
                      float* domega, void* workspace, cudaStream_t s) {
   const Geo g = geometry(p);
   Carver cv(workspace);
@@ -582,7 +553,7 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
   SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
   { prof::Scope ps(prof::K_STATE, s);
-  k_state_in<<<blocks((long long)E), 256, 0, s>>>(S_state, z_state, w.st_hi, w.st_lo, g.chains,
+  k_state_in<<<blocks((long long)E), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains,
                                                   g.M, g.d); }
   SLIM_TRY(cudaGetLastError());
   SLIM_TRY(cudaMemsetAsync(w.g_hi, 0, E * sizeof(float), s));
@@ -682,21 +653,20 @@ size_t workspace_bytes(const Problem& p, bool bwd) {
 }
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, void* out, float* S_state, float* z_state, void* workspace,
+                const float* omega, void* out, const StateOut& st, void* workspace,
                 cudaStream_t s) {
   if (p.dtype == SLIM_BF16)
-    return fwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, S_state, z_state, workspace, s);
-  return fwd_impl<float>(p, q, k, v, omega, out, S_state, z_state, workspace, s);
+    return fwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, st, workspace, s);
+  return fwd_impl<float>(p, q, k, v, omega, out, st, workspace, s);
 }
 
 slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, const void* out, const void* dout, const float* S_state,
-                const float* z_state, void* dq, void* dk, void* dv, float* domega,
-                void* workspace, cudaStream_t s) {
+                const float* omega, const void* out, const void* dout, const StateIn& st,
+                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s) {
   if (p.dtype == SLIM_BF16)
-    return bwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv,
+    return bwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, dout, st, dq, dk, dv,
                                    domega, workspace, s);
-  return bwd_impl<float>(p, q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv, domega,
+  return bwd_impl<float>(p, q, k, v, omega, out, dout, st, dq, dk, dv, domega,
                          workspace, s);
 }
 

@@ -8,13 +8,12 @@ namespace simt {
 size_t workspace_bytes(const Problem& p, bool bwd);
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, void* out, float* S_state, float* z_state, void* workspace,
+                const float* omega, void* out, const StateOut& st, void* workspace,
                 cudaStream_t s);
 
 slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, const void* out, const void* dout, const float* S_state,
-                const float* z_state, void* dq, void* dk, void* dv, float* domega,
-                void* workspace, cudaStream_t s);
+                const float* omega, const void* out, const void* dout, const StateIn& st,
+                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s);
 
 }  // namespace simt
 }  // namespace slim

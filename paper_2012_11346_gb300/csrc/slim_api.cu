@@ -1,9 +1,12 @@
 // C ABI of libslim: argument validation, workspace sizing, dispatch.
 // Declarations and the contract of every entry point: include/slim.h.
 #include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include "common.cuh"
 #include "simt_path.h"
+#include "tc_path.h"
 
 using slim::Problem;
 
@@ -40,7 +43,18 @@ slim_status check_problem(int B, int H, int L, int d, int M, int C, slim_dtype d
   return SLIM_OK;
 }
 
-size_t ws_bytes(const Problem& p, bool bwd) { return slim::simt::workspace_bytes(p, bwd); }
+// Path selection: the tensor-core path where it applies, else the fp32-compute
+// path.  SLIM_PATH=simt in the environment (read on every call) forces the
+// fp32-compute path.
+bool use_tc(const Problem& p) {
+  const char* e = getenv("SLIM_PATH");
+  if (e && strcmp(e, "simt") == 0) return false;
+  return slim::tc::supports(p);
+}
+
+size_t ws_bytes(const Problem& p, bool bwd) {
+  return use_tc(p) ? slim::tc::workspace_bytes(p, bwd) : slim::simt::workspace_bytes(p, bwd);
+}
 
 slim_status check_workspace(const Problem& p, bool bwd, void* ws, size_t bytes) {
   const size_t need = ws_bytes(p, bwd);
@@ -90,15 +104,17 @@ slim_status slim_bwd_workspace_size(int B, int H, int L, int d, int M, int C, sl
 
 slim_status slim_fwd(const void* q, const void* k, const void* v, const float* omega, int B,
                      int H, int L, int d, int M, int C, slim_dtype dtype, slim_feature feature,
-                     void* out, float* S_state, float* z_state, void* workspace,
-                     size_t workspace_bytes, void* stream) {
+                     void* out, float* S_state, float* z_state, float* S_state_lo,
+                     float* z_state_lo, void* workspace, size_t workspace_bytes, void* stream) {
   Problem p;
   slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
   if (st != SLIM_OK) return st;
   // [B,H,L,d] tensors are empty when L = 0 and may then be null
   const void* seq[] = {q, k, v, out};
   const void* fixed[] = {omega, S_state, z_state};
-  if (!pointers_ok(seq, 4, L == 0) || !pointers_ok(fixed, 3, false)) return SLIM_ERR_INVALID_ARG;
+  const void* opt[] = {S_state_lo, z_state_lo};
+  if (!pointers_ok(seq, 4, L == 0) || !pointers_ok(fixed, 3, false) || !pointers_ok(opt, 2, true))
+    return SLIM_ERR_INVALID_ARG;
   st = check_workspace(p, false, workspace, workspace_bytes);
   if (st != SLIM_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -106,14 +122,21 @@ slim_status slim_fwd(const void* q, const void* k, const void* v, const float* o
     const size_t n = (size_t)p.chains() * M;
     if (cudaMemsetAsync(S_state, 0, n * d * sizeof(float), s) != cudaSuccess) return SLIM_ERR_CUDA;
     if (cudaMemsetAsync(z_state, 0, n * sizeof(float), s) != cudaSuccess) return SLIM_ERR_CUDA;
+    if (S_state_lo && cudaMemsetAsync(S_state_lo, 0, n * d * sizeof(float), s) != cudaSuccess)
+      return SLIM_ERR_CUDA;
+    if (z_state_lo && cudaMemsetAsync(z_state_lo, 0, n * sizeof(float), s) != cudaSuccess)
+      return SLIM_ERR_CUDA;
     return SLIM_OK;
   }
-  return slim::simt::fwd(p, q, k, v, omega, out, S_state, z_state, workspace, s);
+  const slim::StateOut so{S_state, z_state, S_state_lo, z_state_lo};
+  if (use_tc(p)) return slim::tc::fwd(p, q, k, v, omega, out, so, workspace, s);
+  return slim::simt::fwd(p, q, k, v, omega, out, so, workspace, s);
 }
 
 slim_status slim_bwd(const void* q, const void* k, const void* v, const float* omega,
                      const void* out, const void* dout, const float* S_state,
-                     const float* z_state, int B, int H, int L, int d, int M, int C,
+                     const float* z_state, const float* S_state_lo, const float* z_state_lo,
+                     int B, int H, int L, int d, int M, int C,
                      slim_dtype dtype, slim_feature feature, void* dq, void* dk, void* dv,
                      float* domega, void* workspace, size_t workspace_bytes, void* stream) {
   Problem p;
@@ -121,7 +144,9 @@ slim_status slim_bwd(const void* q, const void* k, const void* v, const float* o
   if (st != SLIM_OK) return st;
   const void* seq[] = {q, k, v, out, dout, dq, dk, dv};
   const void* fixed[] = {omega, S_state, z_state, domega};
-  if (!pointers_ok(seq, 8, L == 0) || !pointers_ok(fixed, 4, false)) return SLIM_ERR_INVALID_ARG;
+  const void* opt[] = {S_state_lo, z_state_lo};
+  if (!pointers_ok(seq, 8, L == 0) || !pointers_ok(fixed, 4, false) || !pointers_ok(opt, 2, true))
+    return SLIM_ERR_INVALID_ARG;
   st = check_workspace(p, true, workspace, workspace_bytes);
   if (st != SLIM_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -130,8 +155,20 @@ slim_status slim_bwd(const void* q, const void* k, const void* v, const float* o
       return SLIM_ERR_CUDA;
     return SLIM_OK;
   }
-  return slim::simt::bwd(p, q, k, v, omega, out, dout, S_state, z_state, dq, dk, dv, domega,
-                         workspace, s);
+  const slim::StateIn si{S_state, z_state, S_state_lo, z_state_lo};
+  if (use_tc(p))
+    return slim::tc::bwd(p, q, k, v, omega, out, dout, si, dq, dk, dv, domega, workspace, s);
+  return slim::simt::bwd(p, q, k, v, omega, out, dout, si, dq, dk, dv, domega, workspace, s);
+}
+
+slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                          slim_feature feature, int* path) {
+  if (!path) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  *path = use_tc(p) ? 1 : 0;
+  return SLIM_OK;
 }
 
 slim_status slim_check_device_error(void* workspace, void* stream) {

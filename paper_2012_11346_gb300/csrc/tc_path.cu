@@ -1,0 +1,1202 @@
+// Tensor-core (tcgen05) path of libslim: bf16 inputs, d = 64, M in {128, 256}.
+//
+// Same slice algorithm as the fp32 path (Algorithm 1, App. B block form with
+// masked tile products), with tiles of T = 128 rows, one CTA of 128 threads
+// per (tile, chain).  Every tile product is a chain of tcgen05 MMAs on
+// 128-byte-swizzled bf16 shared-memory operands with an fp32 accumulator in
+// tensor memory; thread r of the CTA owns row r (TMEM lane r) in the
+// epilogues.  Per slice:
+//
+//   forward   tc_delta : phiK = g(K_t), Delta_t = phiK^T [V_t | 1]
+//             scan     : P_t = B + sum_{t'<t} Delta_t', B += sum Delta_t
+//             tc_fwd   : phiQ, phiK, A = tril(phiQ phiK^T),
+//                        num = phiQ S_t + A V_t, den = phiQ z_t + rowsum A
+//   backward  tc_delta, scan(rollback, eq. 17)
+//             tc_bwd_q : den, dnum = dout/den, dden = -<dout,out>/den,
+//                        dA = tril(dnum V^T + dden), dphiQ = dnum S_t^T +
+//                        dden z_t + dA phiK, Gd_t = phiQ^T [dnum | dden],
+//                        dq = u Omega - q sum(u), dOmega partial u^T q
+//             scan     : G_t = G + sum_{t'>t} Gd_t' (eq. 18)
+//             tc_bwd_kv: dV = A^T dnum + phiK G_t(S), dphiK = dA^T phiQ +
+//                        V G_t(S)^T + g_t(z), dk = u Omega - k sum(u),
+//                        dOmega partial += u^T k
+//             reduce   : dOmega += sum of partials (fixed order)
+//
+// The state rows of the workspace hold [S (M x 64) | z (M)] per tile (E =
+// 65 M floats), exactly what the shared scan carries.
+#include <math.h>
+
+#include "common.cuh"
+#include "profiler.h"
+#include "scan.h"
+#include "tc_common.cuh"
+#include "tc_path.h"
+
+namespace slim {
+namespace tc {
+
+constexpr int T = 128;           // tile rows
+constexpr int D = 64;            // head width handled here
+constexpr int ROWT = T * 128;    // bytes of a [128][64] bf16 row tile
+constexpr float kLog2e = 1.4426950408889634f;
+
+template <int MF>
+struct Cfg {
+  static constexpr int MH = MF / 128;       // feature halves (MMA M = 128 each)
+  static constexpr int FEATB = T * MF * 2;  // [128][MF] bf16 feature tile
+  static constexpr int OMB = MF * 128;      // [MF][64] bf16 (Omega, state)
+  static constexpr int E = MF * 64 + MF;    // state floats per tile
+};
+
+// ------------------------------------------------------------------ helpers
+__device__ __forceinline__ float row_norm2(const uint8_t* tile, int r) {
+  float s = 0.f;
+#pragma unroll
+  for (int c = 0; c < 64; c += 8) {
+    uint4 v = ld_chunk(tile, T, r, c);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float a, b;
+      unpack_bf16(w[i], a, b);
+      s = fmaf(a, a, s);
+      s = fmaf(b, b, s);
+    }
+  }
+  return s;
+}
+
+// fp32 [R][64] global -> bf16 row tile (R rows), all 128 threads.
+__device__ __forceinline__ void load_f32_rows64(uint8_t* tile, int R, const float* g, int tid) {
+  for (int e = tid; e < R * 8; e += 128) {
+    const int r = e >> 3, c = (e & 7) * 8;
+    const float4 a = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c);
+    const float4 b = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c + 4);
+    st_chunk(tile, R, r, c, make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w),
+                                       pack_bf16(b.x, b.y), pack_bf16(b.z, b.w)));
+  }
+}
+
+// Reads the projection P = X Omega^T of this thread's row from TMEM, applies
+// the feature map and stores phi (bf16) into the [128][MF] feature tile.
+// Returns sum_m phi_m z_m when z != nullptr.
+template <int MF, int FEAT>
+__device__ __forceinline__ float feature_epilogue(uint32_t trow, uint8_t* phi, int r, float x2,
+                                                  bool valid, const float* z) {
+  // exp map: phi = 2^(p log2e - (|x|^2/2) log2e - log2 sqrt(M))
+  const float bias = -0.5f * x2 * kLog2e - 0.5f * log2f((float)MF);
+  const float relu_scale = rsqrtf((float)MF);
+  float acc = 0.f;
+#pragma unroll 1
+  for (int c0 = 0; c0 < MF; c0 += 32) {
+    float v[32];
+    tmem_ld32(trow + c0, v);
+    uint32_t pk[16];
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+      float a, b;
+      if (FEAT == SLIM_FEAT_EXP) {
+        a = ex2_approx(fmaf(v[i], kLog2e, bias));
+        b = ex2_approx(fmaf(v[i + 1], kLog2e, bias));
+      } else {
+        a = fmaxf(v[i], 0.f) * relu_scale;
+        b = fmaxf(v[i + 1], 0.f) * relu_scale;
+      }
+      if (!valid) a = b = 0.f;
+      if (z) acc = fmaf(a, z[c0 + i], fmaf(b, z[c0 + i + 1], acc));
+      pk[i / 2] = pack_bf16(a, b);
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      st_chunk(phi, T, r, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+  }
+  return acc;
+}
+
+// Loads 16 bf16 of a feature-tile row (columns c..c+15) as floats.
+__device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, float* f) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint4 v = ld_chunk(tile, T, r, c + 8 * h);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) unpack_bf16(w[i], f[8 * h + 2 * i], f[8 * h + 2 * i + 1]);
+  }
+}
+
+struct Sync {
+  uint32_t mbar;
+  uint32_t phase;
+  int* err;
+  __device__ bool wait() {
+    const bool ok = mbar_wait(mbar, phase, err);
+    phase ^= 1u;
+    tc_fence_after();
+    return ok;
+  }
+};
+
+// Make generic-proxy smem writes visible to the tensor core and order them
+// with the thread that issues the next MMAs.
+__device__ __forceinline__ void publish() {
+  fence_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+}
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+// Abort after a failed wait: every thread leaves through the teardown.
+#define TC_WAIT(sy)                  \
+  do {                               \
+    if (!(sy).wait()) abort_ = 1;    \
+    __syncthreads();                 \
+    if (abort_) goto teardown;       \
+  } while (0)
+
+// ================================================================== tc_delta
+template <int MF, int FEAT>
+__global__ void __launch_bounds__(128, 1)
+    k_tc_delta(const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
+               const __nv_bfloat16* __restrict__ om16, int L, int a, int b, int nt,
+               float* __restrict__ delta, int* err) {
+  using C = Cfg<MF>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = align1024(smem_raw);
+  uint8_t* sK = base;
+  uint8_t* sV = sK + ROWT;
+  uint8_t* sOm = sV + ROWT;
+  uint8_t* sPhi = sOm + C::OMB;
+  uint8_t* sOnes = sPhi + C::FEATB;  // [16][128] K-major, all ones
+  __shared__ __align__(8) uint64_t mbar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_;
+  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int row0 = a + t * T;
+  const int valid = min(T, b - t * T);
+  const size_t g0 = ((size_t)c * L + row0) * D;
+
+  if (tid == 0) {
+    abort_ = 0;
+    mbar_init(smem_u32(&mbar), 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
+  load_rows64(sK, T, K + g0, valid, tid, 128);
+  load_rows64(sV, T, V + g0, valid, tid, 128);
+  load_rows64(sOm, MF, om16, MF, tid, 128);
+  load_rows64(sPhi, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phi overwrites it
+  for (int e = tid; e < 4096 / 16; e += 128)
+    reinterpret_cast<uint4*>(sOnes)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+  cp_async_wait_all();
+  __syncthreads();  // rows were copied by other threads
+  {
+    const float x2 = row_norm2(sK, tid);
+    publish();
+    const uint32_t tmem = tmem_base;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    Sync sy{smem_u32(&mbar), 0u, err};
+    if (tid == 0) {
+      const uint32_t aK = smem_u32(sK), aOm = smem_u32(sOm), aOl = smem_u32(sPhi);
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        mma(tmem, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    feature_epilogue<MF, FEAT>(trow, sPhi, tid, x2, tid < valid, nullptr);
+    publish();
+    if (tid == 0) {
+      const uint32_t aPhi = smem_u32(sPhi), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
+      for (int h = 0; h < C::MH; ++h)
+        for (int k0 = 0; k0 < T; k0 += 16) {
+          const uint64_t ad = mnmaj(aPhi + h * 2 * ROWT, k0, ROWT);
+          mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+          mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
+        }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    float* dst = delta + ((size_t)c * nt + t) * C::E;
+    for (int h = 0; h < C::MH; ++h) {
+      const int m = 128 * h + tid;
+      float v[32];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        tmem_ld32(trow + 256 + 64 * h + 32 * q, v);
+        float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      }
+      float zz;
+      tmem_ld1(trow + 384 + 16 * h, zz);
+      dst[MF * 64 + m] = zz;
+    }
+  }
+teardown:
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem_base, 512);
+}
+
+// ================================================================== tc_fwd
+template <int MF, int FEAT>
+__global__ void __launch_bounds__(128, 1)
+    k_tc_fwd(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+             const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ om16,
+             const float* __restrict__ pfx, int L, int a, int b, int nt,
+             __nv_bfloat16* __restrict__ out, int* err) {
+  using C = Cfg<MF>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = align1024(smem_raw);
+  uint8_t* sPhiQ = base;
+  uint8_t* sPhiK = sPhiQ + C::FEATB;
+  uint8_t* sQ = sPhiK + C::FEATB;  // later: A tile (2 row tiles)
+  uint8_t* sK = sQ + ROWT;
+  uint8_t* sA = sQ;
+  uint8_t* sOm = sK + ROWT;        // later: S_t (bf16)
+  uint8_t* sS = sOm;
+  uint8_t* sV = sOm + C::OMB;
+  float* sZ = reinterpret_cast<float*>(sV + ROWT);
+  __shared__ __align__(8) uint64_t mbar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_;
+  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int row0 = a + t * T;
+  const int valid = min(T, b - t * T);
+  const size_t g0 = ((size_t)c * L + row0) * D;
+  const float* P = pfx + ((size_t)c * nt + t) * C::E;
+
+  if (tid == 0) {
+    abort_ = 0;
+    mbar_init(smem_u32(&mbar), 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
+  load_rows64(sQ, T, Q + g0, valid, tid, 128);
+  load_rows64(sK, T, K + g0, valid, tid, 128);
+  load_rows64(sV, T, V + g0, valid, tid, 128);
+  load_rows64(sOm, MF, om16, MF, tid, 128);
+  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phiQ overwrites it
+  for (int m = tid; m < MF; m += 128) sZ[m] = P[MF * 64 + m];
+  cp_async_wait_all();
+  __syncthreads();  // rows were copied by other threads
+  {
+    const float q2 = row_norm2(sQ, tid), k2 = row_norm2(sK, tid);
+    const bool rv = tid < valid;
+    publish();
+    const uint32_t tmem = tmem_base;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    Sync sy{smem_u32(&mbar), 0u, err};
+    if (tid == 0) {
+      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
+      const uint32_t aOl = smem_u32(sPhiQ);
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    load_f32_rows64(sS, MF, P, tid);  // Omega no longer needed: S_t takes its place
+    const float dz = feature_epilogue<MF, FEAT>(trow, sPhiQ, tid, q2, rv, sZ);
+    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, tid, k2, rv, nullptr);
+    publish();
+    if (tid == 0) {
+      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK), aS = smem_u32(sS);
+      for (int k0 = 0; k0 < MF; k0 += 16) {
+        mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+        mma(tmem + 128, kmaj(aPQ, T, k0), mnmaj(aS, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+      }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    // A row: inclusive causal mask, bf16, row sum of the rounded values
+    float rs = 0.f;
+#pragma unroll 1
+    for (int c0 = 0; c0 < T; c0 += 32) {
+      float v[32];
+      tmem_ld32(trow + c0, v);
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        const float x0 = (c0 + i <= tid) ? v[i] : 0.f;
+        const float x1 = (c0 + i + 1 <= tid) ? v[i + 1] : 0.f;
+        pk[i / 2] = pack_bf16(x0, x1);
+        float r0, r1;
+        unpack_bf16(pk[i / 2], r0, r1);
+        rs += r0 + r1;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_chunk(sA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+    }
+    publish();
+    if (tid == 0) {
+      const uint32_t aA = smem_u32(sA), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < T; k0 += 16)
+        mma(tmem + 128, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), 1);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    {
+      const float den = rs + dz;
+      const float inv = den != 0.f ? 1.f / den : 0.f;
+      __nv_bfloat16* o = out + g0 + (size_t)tid * D;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        float v[32];
+        tmem_ld32(trow + 128 + 32 * q, v);  // every lane loads (warp-aligned op)
+        if (rv) {
+          uint4* dst = reinterpret_cast<uint4*>(o + 32 * q);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            dst[i] = make_uint4(pack_bf16(v[8 * i] * inv, v[8 * i + 1] * inv),
+                                pack_bf16(v[8 * i + 2] * inv, v[8 * i + 3] * inv),
+                                pack_bf16(v[8 * i + 4] * inv, v[8 * i + 5] * inv),
+                                pack_bf16(v[8 * i + 6] * inv, v[8 * i + 7] * inv));
+        }
+      }
+    }
+  }
+teardown:
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem_base, 512);
+}
+
+// ================================================================== tc_bwd_q
+template <int MF, int FEAT>
+__global__ void __launch_bounds__(128, 1)
+    k_tc_bwd_q(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+               const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ Out,
+               const __nv_bfloat16* __restrict__ dOut, const __nv_bfloat16* __restrict__ om16,
+               const float* __restrict__ pfx, int L, int a, int b, int nt,
+               __nv_bfloat16* __restrict__ dq, float* __restrict__ gdelta,
+               float* __restrict__ rowstat, float* __restrict__ part, int* err) {
+  using C = Cfg<MF>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = align1024(smem_raw);
+  uint8_t* sPhiQ = base;
+  uint8_t* sPhiK = sPhiQ + C::FEATB;  // later: u
+  uint8_t* sU = sPhiK;
+  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [dA (2 tiles) | S_t] -> [Q | - | Omega]
+  uint8_t* sQ = sX;
+  uint8_t* sK = sX + ROWT;
+  uint8_t* sdA = sX;
+  uint8_t* sOm = sX + 2 * ROWT;
+  uint8_t* sS = sOm;
+  uint8_t* sV = sOm + C::OMB;         // later: dden as a K-major [16][128] operand
+  uint8_t* sDd = sV;
+  uint8_t* sDo = sV + ROWT;           // dout, then dnum in place
+  float* sZ = reinterpret_cast<float*>(sDo + ROWT);
+  __shared__ __align__(8) uint64_t mbar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_;
+  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int row0 = a + t * T;
+  const int valid = min(T, b - t * T);
+  const size_t g0 = ((size_t)c * L + row0) * D;
+  const float* P = pfx + ((size_t)c * nt + t) * C::E;
+
+  if (tid == 0) {
+    abort_ = 0;
+    mbar_init(smem_u32(&mbar), 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
+  load_rows64(sQ, T, Q + g0, valid, tid, 128);
+  load_rows64(sK, T, K + g0, valid, tid, 128);
+  load_rows64(sV, T, V + g0, valid, tid, 128);
+  load_rows64(sDo, T, dOut + g0, valid, tid, 128);
+  load_rows64(sOm, MF, om16, MF, tid, 128);
+  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phiQ overwrites it
+  for (int m = tid; m < MF; m += 128) sZ[m] = P[MF * 64 + m];
+  cp_async_wait_all();
+  __syncthreads();  // rows were copied by other threads
+  {
+    const bool rv = tid < valid;
+    const float q2 = row_norm2(sQ, tid), k2 = row_norm2(sK, tid);
+    // <dout_r, out_r>
+    float rowdot = 0.f;
+    if (rv) {
+      const __nv_bfloat16* orow = Out + g0 + (size_t)tid * D;
+#pragma unroll
+      for (int c8 = 0; c8 < 64; c8 += 8) {
+        const uint4 o = *reinterpret_cast<const uint4*>(orow + c8);
+        const uint4 g = ld_chunk(sDo, T, tid, c8);
+        const uint32_t ow[4] = {o.x, o.y, o.z, o.w}, gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          float o0, o1, g0f, g1f;
+          unpack_bf16(ow[i], o0, o1);
+          unpack_bf16(gw[i], g0f, g1f);
+          rowdot = fmaf(o0, g0f, fmaf(o1, g1f, rowdot));
+        }
+      }
+    }
+    publish();
+    const uint32_t tmem = tmem_base;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    Sync sy{smem_u32(&mbar), 0u, err};
+    if (tid == 0) {
+      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
+      const uint32_t aOl = smem_u32(sPhiQ);
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    load_f32_rows64(sS, MF, P, tid);
+    const float dz = feature_epilogue<MF, FEAT>(trow, sPhiQ, tid, q2, rv, sZ);
+    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, tid, k2, rv, nullptr);
+    publish();
+    if (tid == 0) {
+      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
+      const uint32_t aDo = smem_u32(sDo), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < MF; k0 += 16)
+        mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      for (int k0 = 0; k0 < D; k0 += 16)  // dout V^T (scaled by 1/den below)
+        mma(tmem + 128, kmaj(aDo, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    float rs = 0.f;
+#pragma unroll 1
+    for (int c0 = 0; c0 < T; c0 += 32) {
+      float v[32];
+      tmem_ld32(trow + c0, v);
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        const float x0 = (c0 + i <= tid) ? v[i] : 0.f;
+        const float x1 = (c0 + i + 1 <= tid) ? v[i + 1] : 0.f;
+        float r0, r1;
+        unpack_bf16(pack_bf16(x0, x1), r0, r1);
+        rs += r0 + r1;
+      }
+    }
+    const float den = rs + dz;
+    const bool live = rv && den != 0.f;
+    const float inv = live ? 1.f / den : 0.f;
+    const float dden = live ? -rowdot * inv : 0.f;
+    // dnum = dout / den, in place of dout
+#pragma unroll
+    for (int c8 = 0; c8 < 64; c8 += 8) {
+      const uint4 g = ld_chunk(sDo, T, tid, c8);
+      const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+      uint32_t pw[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float g0f, g1f;
+        unpack_bf16(gw[i], g0f, g1f);
+        pw[i] = pack_bf16(g0f * inv, g1f * inv);
+      }
+      st_chunk(sDo, T, tid, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
+    }
+    // dA = tril(dnum V^T + dden)
+#pragma unroll 1
+    for (int c0 = 0; c0 < T; c0 += 32) {
+      float v[32];
+      tmem_ld32(trow + 128 + c0, v);
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        const float x0 = (live && c0 + i <= tid) ? fmaf(v[i], inv, dden) : 0.f;
+        const float x1 = (live && c0 + i + 1 <= tid) ? fmaf(v[i + 1], inv, dden) : 0.f;
+        pk[i / 2] = pack_bf16(x0, x1);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_chunk(sdA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+    }
+    // dden as the first row of a K-major [16][128] operand (other rows zero)
+    {
+      const __nv_bfloat16 zb = __float2bfloat16_rn(0.f);
+      for (int n = 0; n < 16; ++n)
+        *reinterpret_cast<__nv_bfloat16*>(sDd + tile_off(16, n, tid)) =
+            n == 0 ? __float2bfloat16_rn(dden) : zb;
+    }
+    if (rv) {
+      float* rsw = rowstat + (((size_t)c * nt + t) * T + tid) * 2;
+      rsw[0] = den;
+      rsw[1] = dden;
+    }
+    publish();
+    if (tid == 0) {
+      const uint32_t aDn = smem_u32(sDo), aS = smem_u32(sS), adA = smem_u32(sdA);
+      const uint32_t aPK = smem_u32(sPhiK), aPQ = smem_u32(sPhiQ), aDd = smem_u32(sDd);
+      for (int k0 = 0; k0 < D; k0 += 16)  // dnum S_t^T
+        mma(tmem + 256, kmaj(aDn, T, k0), kmaj(aS, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+      for (int k0 = 0; k0 < T; k0 += 16)  // + dA phiK
+        mma(tmem + 256, kmaj(adA, T, k0), mnmaj(aPK, k0, ROWT), idesc_bf16(T, MF, 0, 1), 1);
+      for (int h = 0; h < C::MH; ++h)
+        for (int k0 = 0; k0 < T; k0 += 16) {  // Gd = phiQ^T [dnum | dden]
+          const uint64_t ad = mnmaj(aPQ + h * 2 * ROWT, k0, ROWT);
+          mma(tmem + 64 * h, ad, mnmaj(aDn, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+          mma(tmem + 128 + 16 * h, ad, kmaj(aDd, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
+        }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    {
+      float* dst = gdelta + ((size_t)c * nt + t) * C::E;
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + tid;
+        float v[32];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          tmem_ld32(trow + 64 * h + 32 * q, v);
+          float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+        float zz;
+        tmem_ld1(trow + 128 + 16 * h, zz);
+        dst[MF * 64 + m] = zz;
+      }
+    }
+    // dphiQ -> u (into the phiK tile)
+    float usum = 0.f;
+    const float rscale = rsqrtf((float)MF);
+#pragma unroll 1
+    for (int c0 = 0; c0 < MF; c0 += 32) {
+      float v[32];
+      tmem_ld32(trow + 256 + c0, v);
+      uint32_t pk[16];
+#pragma unroll
+      for (int s16 = 0; s16 < 32; s16 += 16) {
+        float f[16];
+        ld_feat16(sPhiQ, tid, c0 + s16, f);
+#pragma unroll
+        for (int i = 0; i < 16; i += 2) {
+          float u0 = fmaf(dden, sZ[c0 + s16 + i], v[s16 + i]);
+          float u1 = fmaf(dden, sZ[c0 + s16 + i + 1], v[s16 + i + 1]);
+          if (FEAT == SLIM_FEAT_EXP) {
+            u0 *= f[i];
+            u1 *= f[i + 1];
+          } else {
+            u0 = f[i] > 0.f ? u0 * rscale : 0.f;
+            u1 = f[i + 1] > 0.f ? u1 * rscale : 0.f;
+          }
+          if (!live) u0 = u1 = 0.f;
+          pk[(s16 + i) / 2] = pack_bf16(u0, u1);
+          float r0, r1;
+          unpack_bf16(pk[(s16 + i) / 2], r0, r1);
+          usum += r0 + r1;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_chunk(sU, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+    }
+    // Q and Omega again for dq = u Omega - q sum(u) and dOmega += u^T q
+    load_rows64(sQ, T, Q + g0, valid, tid, 128);
+    load_rows64(sOm, MF, om16, MF, tid, 128);
+    cp_async_wait_all();
+    publish();
+    if (tid == 0) {
+      const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aQ = smem_u32(sQ);
+      for (int k0 = 0; k0 < MF; k0 += 16)
+        mma(tmem, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+      for (int h = 0; h < C::MH; ++h)
+        for (int k0 = 0; k0 < T; k0 += 16)
+          mma(tmem + 64 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aQ, k0, ROWT),
+              idesc_bf16(T, 64, 1, 1), k0 > 0);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    {
+      float xq[64];
+#pragma unroll
+      for (int c8 = 0; c8 < 64; c8 += 8) {
+        const uint4 g = ld_chunk(sQ, T, tid, c8);
+        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) unpack_bf16(gw[i], xq[c8 + 2 * i], xq[c8 + 2 * i + 1]);
+      }
+      const float us = (FEAT == SLIM_FEAT_EXP) ? usum : 0.f;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        float v[32];
+        tmem_ld32(trow + 32 * q, v);
+        if (rv) {
+          uint4* dst = reinterpret_cast<uint4*>(dq + g0 + (size_t)tid * D + 32 * q);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int j = 32 * q + 8 * i;
+            dst[i] = make_uint4(pack_bf16(fmaf(-us, xq[j], v[8 * i]), fmaf(-us, xq[j + 1], v[8 * i + 1])),
+                                pack_bf16(fmaf(-us, xq[j + 2], v[8 * i + 2]), fmaf(-us, xq[j + 3], v[8 * i + 3])),
+                                pack_bf16(fmaf(-us, xq[j + 4], v[8 * i + 4]), fmaf(-us, xq[j + 5], v[8 * i + 5])),
+                                pack_bf16(fmaf(-us, xq[j + 6], v[8 * i + 6]), fmaf(-us, xq[j + 7], v[8 * i + 7])));
+          }
+        }
+      }
+      float* dst = part + ((size_t)c * nt + t) * (size_t)(MF * 64);
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + tid;
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          float v[32];
+          tmem_ld32(trow + 64 + 64 * h + 32 * q, v);
+          float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+      }
+    }
+  }
+teardown:
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem_base, 512);
+}
+
+// ================================================================== tc_bwd_kv
+template <int MF, int FEAT>
+__global__ void __launch_bounds__(128, 1)
+    k_tc_bwd_kv(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+                const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ dOut,
+                const __nv_bfloat16* __restrict__ om16, const float* __restrict__ gsfx,
+                const float* __restrict__ rowstat, int L, int a, int b, int nt,
+                __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv,
+                float* __restrict__ part, int* err) {
+  using C = Cfg<MF>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = align1024(smem_raw);
+  uint8_t* sPhiQ = base;               // later: u
+  uint8_t* sU = sPhiQ;
+  uint8_t* sPhiK = sPhiQ + C::FEATB;
+  uint8_t* sX = sPhiK + C::FEATB;      // [Q | K | Omega] -> [A | G_t] -> [dA | G_t] -> [K | - | Omega]
+  uint8_t* sQ = sX;
+  uint8_t* sK = sX + ROWT;
+  uint8_t* sA = sX;
+  uint8_t* sKr = sX;
+  uint8_t* sOm = sX + 2 * ROWT;
+  uint8_t* sG = sOm;
+  uint8_t* sV = sOm + C::OMB;
+  uint8_t* sDn = sV + ROWT;            // dout, then dnum in place
+  float* sGz = reinterpret_cast<float*>(sDn + ROWT);
+  __shared__ __align__(8) uint64_t mbar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_;
+  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int row0 = a + t * T;
+  const int valid = min(T, b - t * T);
+  const size_t g0 = ((size_t)c * L + row0) * D;
+  const float* G = gsfx + ((size_t)c * nt + t) * C::E;
+
+  if (tid == 0) {
+    abort_ = 0;
+    mbar_init(smem_u32(&mbar), 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
+  load_rows64(sQ, T, Q + g0, valid, tid, 128);
+  load_rows64(sK, T, K + g0, valid, tid, 128);
+  load_rows64(sV, T, V + g0, valid, tid, 128);
+  load_rows64(sDn, T, dOut + g0, valid, tid, 128);
+  load_rows64(sOm, MF, om16, MF, tid, 128);
+  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phiQ overwrites it
+  for (int m = tid; m < MF; m += 128) sGz[m] = G[MF * 64 + m];
+  float den = 0.f, dden = 0.f;
+  if (tid < valid) {
+    const float* rsr = rowstat + (((size_t)c * nt + t) * T + tid) * 2;
+    den = rsr[0];
+    dden = rsr[1];
+  }
+  cp_async_wait_all();
+  __syncthreads();  // rows were copied by other threads
+  {
+    const bool rv = tid < valid;
+    const bool live = rv && den != 0.f;
+    const float inv = live ? 1.f / den : 0.f;
+    if (!live) dden = 0.f;
+    const float q2 = row_norm2(sQ, tid), k2 = row_norm2(sK, tid);
+#pragma unroll
+    for (int c8 = 0; c8 < 64; c8 += 8) {  // dnum = dout / den, in place
+      const uint4 g = ld_chunk(sDn, T, tid, c8);
+      const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+      uint32_t pw[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float g0f, g1f;
+        unpack_bf16(gw[i], g0f, g1f);
+        pw[i] = pack_bf16(g0f * inv, g1f * inv);
+      }
+      st_chunk(sDn, T, tid, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
+    }
+    publish();
+    const uint32_t tmem = tmem_base;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    Sync sy{smem_u32(&mbar), 0u, err};
+    if (tid == 0) {
+      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
+      const uint32_t aOl = smem_u32(sPhiQ);
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    load_f32_rows64(sG, MF, G, tid);  // G_t(S) replaces Omega
+    feature_epilogue<MF, FEAT>(trow, sPhiQ, tid, q2, rv, nullptr);
+    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, tid, k2, rv, nullptr);
+    publish();
+    if (tid == 0) {
+      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
+      const uint32_t aDn = smem_u32(sDn), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < MF; k0 += 16)
+        mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      for (int k0 = 0; k0 < D; k0 += 16)  // dnum V^T
+        mma(tmem + 128, kmaj(aDn, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+#pragma unroll 1
+    for (int c0 = 0; c0 < T; c0 += 32) {  // A -> smem (masked, bf16)
+      float v[32];
+      tmem_ld32(trow + c0, v);
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2)
+        pk[i / 2] = pack_bf16((c0 + i <= tid) ? v[i] : 0.f, (c0 + i + 1 <= tid) ? v[i + 1] : 0.f);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_chunk(sA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+    }
+    publish();
+    if (tid == 0) {
+      const uint32_t aA = smem_u32(sA), aDn = smem_u32(sDn), aPK = smem_u32(sPhiK);
+      const uint32_t aG = smem_u32(sG), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < T; k0 += 16)  // dV = A^T dnum
+        mma(tmem, mnmaj(aA, k0, ROWT), mnmaj(aDn, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+      for (int k0 = 0; k0 < MF; k0 += 16)  // + phiK G_t(S)
+        mma(tmem, kmaj(aPK, T, k0), mnmaj(aG, k0, C::OMB), idesc_bf16(T, 64, 0, 1), 1);
+      for (int k0 = 0; k0 < D; k0 += 16)  // dphiK = V G_t(S)^T
+        mma(tmem + 256, kmaj(aV, T, k0), kmaj(aG, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {  // dv
+      float v[32];
+      tmem_ld32(trow + 32 * q, v);
+      if (rv) {
+        uint4* dst = reinterpret_cast<uint4*>(dv + g0 + (size_t)tid * D + 32 * q);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          dst[i] = make_uint4(pack_bf16(v[8 * i], v[8 * i + 1]), pack_bf16(v[8 * i + 2], v[8 * i + 3]),
+                              pack_bf16(v[8 * i + 4], v[8 * i + 5]), pack_bf16(v[8 * i + 6], v[8 * i + 7]));
+      }
+    }
+#pragma unroll 1
+    for (int c0 = 0; c0 < T; c0 += 32) {  // dA = tril(dnum V^T + dden) -> smem
+      float v[32];
+      tmem_ld32(trow + 128 + c0, v);
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        const float x0 = (live && c0 + i <= tid) ? v[i] + dden : 0.f;
+        const float x1 = (live && c0 + i + 1 <= tid) ? v[i + 1] + dden : 0.f;
+        pk[i / 2] = pack_bf16(x0, x1);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_chunk(sA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+    }
+    publish();
+    if (tid == 0) {
+      const uint32_t adA = smem_u32(sA), aPQ = smem_u32(sPhiQ);
+      for (int k0 = 0; k0 < T; k0 += 16)  // dphiK += dA^T phiQ
+        mma(tmem + 256, mnmaj(adA, k0, ROWT), mnmaj(aPQ, k0, ROWT), idesc_bf16(T, MF, 1, 1), 1);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    float usum = 0.f;
+    const float rscale = rsqrtf((float)MF);
+#pragma unroll 1
+    for (int c0 = 0; c0 < MF; c0 += 32) {  // dphiK (+ g_z) -> u (into the phiQ tile)
+      float v[32];
+      tmem_ld32(trow + 256 + c0, v);
+      uint32_t pk[16];
+#pragma unroll
+      for (int s16 = 0; s16 < 32; s16 += 16) {
+        float f[16];
+        ld_feat16(sPhiK, tid, c0 + s16, f);
+#pragma unroll
+        for (int i = 0; i < 16; i += 2) {
+          float u0 = v[s16 + i] + sGz[c0 + s16 + i];
+          float u1 = v[s16 + i + 1] + sGz[c0 + s16 + i + 1];
+          if (FEAT == SLIM_FEAT_EXP) {
+            u0 *= f[i];
+            u1 *= f[i + 1];
+          } else {
+            u0 = f[i] > 0.f ? u0 * rscale : 0.f;
+            u1 = f[i + 1] > 0.f ? u1 * rscale : 0.f;
+          }
+          if (!rv) u0 = u1 = 0.f;
+          pk[(s16 + i) / 2] = pack_bf16(u0, u1);
+          float r0, r1;
+          unpack_bf16(pk[(s16 + i) / 2], r0, r1);
+          usum += r0 + r1;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_chunk(sU, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+    }
+    load_rows64(sKr, T, K + g0, valid, tid, 128);
+    load_rows64(sOm, MF, om16, MF, tid, 128);
+    cp_async_wait_all();
+    publish();
+    if (tid == 0) {
+      const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aK = smem_u32(sKr);
+      for (int k0 = 0; k0 < MF; k0 += 16)
+        mma(tmem, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+      for (int h = 0; h < C::MH; ++h)
+        for (int k0 = 0; k0 < T; k0 += 16)
+          mma(tmem + 64 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aK, k0, ROWT),
+              idesc_bf16(T, 64, 1, 1), k0 > 0);
+      mma_commit(sy.mbar);
+    }
+    TC_WAIT(sy);
+    {
+      float xk[64];
+#pragma unroll
+      for (int c8 = 0; c8 < 64; c8 += 8) {
+        const uint4 g = ld_chunk(sKr, T, tid, c8);
+        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) unpack_bf16(gw[i], xk[c8 + 2 * i], xk[c8 + 2 * i + 1]);
+      }
+      const float us = (FEAT == SLIM_FEAT_EXP) ? usum : 0.f;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        float v[32];
+        tmem_ld32(trow + 32 * q, v);
+        if (rv) {
+          uint4* dst = reinterpret_cast<uint4*>(dk + g0 + (size_t)tid * D + 32 * q);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int j = 32 * q + 8 * i;
+            dst[i] = make_uint4(pack_bf16(fmaf(-us, xk[j], v[8 * i]), fmaf(-us, xk[j + 1], v[8 * i + 1])),
+                                pack_bf16(fmaf(-us, xk[j + 2], v[8 * i + 2]), fmaf(-us, xk[j + 3], v[8 * i + 3])),
+                                pack_bf16(fmaf(-us, xk[j + 4], v[8 * i + 4]), fmaf(-us, xk[j + 5], v[8 * i + 5])),
+                                pack_bf16(fmaf(-us, xk[j + 6], v[8 * i + 6]), fmaf(-us, xk[j + 7], v[8 * i + 7])));
+          }
+        }
+      }
+      float* dst = part + ((size_t)c * nt + t) * (size_t)(MF * 64);
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + tid;
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          float v[32];
+          tmem_ld32(trow + 64 + 64 * h + 32 * q, v);
+          float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            float4 x = o[i];
+            x.x += v[4 * i];
+            x.y += v[4 * i + 1];
+            x.z += v[4 * i + 2];
+            x.w += v[4 * i + 3];
+            o[i] = x;
+          }
+        }
+      }
+    }
+  }
+teardown:
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem_base, 512);
+}
+
+// ================================================================== small kernels
+// Omega as a bf16 pair: hi = bf16(Omega), lo = bf16(Omega - hi), so the
+// projections X Omega^T = X hi^T + X lo^T carry ~16 mantissa bits.
+__global__ void k_omega_bf16(const float* om, __nv_bfloat16* om16, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) {
+    const __nv_bfloat16 hi = __float2bfloat16_rn(om[i]);
+    om16[i] = hi;
+    om16[n + i] = __float2bfloat16_rn(om[i] - __bfloat162float(hi));
+  }
+}
+
+// state pair [chains][E] <-> S_state [chains][M][64], z_state [chains][M]
+// (the pair is normalised: hi is the rounded state, lo its residual)
+__global__ void k_tc_state_out(const float* hi, const float* lo, StateOut st, int chains, int MF) {
+  const long long E = (long long)MF * 65;
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= chains * E) return;
+  const long long c = i / E, e = i % E;
+  if (e < (long long)MF * 64) {
+    st.S[c * MF * 64 + e] = hi[i];
+    if (st.S_lo) st.S_lo[c * MF * 64 + e] = lo[i];
+  } else {
+    st.z[c * MF + (e - (long long)MF * 64)] = hi[i];
+    if (st.z_lo) st.z_lo[c * MF + (e - (long long)MF * 64)] = lo[i];
+  }
+}
+__global__ void k_tc_state_in(StateIn st, float* hi, float* lo, int chains, int MF) {
+  const long long E = (long long)MF * 65;
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= chains * E) return;
+  const long long c = i / E, e = i % E;
+  if (e < (long long)MF * 64) {
+    hi[i] = st.S[c * MF * 64 + e];
+    lo[i] = st.S_lo ? st.S_lo[c * MF * 64 + e] : 0.f;
+  } else {
+    hi[i] = st.z[c * MF + (e - (long long)MF * 64)];
+    lo[i] = st.z_lo ? st.z_lo[c * MF + (e - (long long)MF * 64)] : 0.f;
+  }
+}
+// dOmega[e] += sum over the slice's partials, fixed order
+__global__ void k_tc_reduce(const float* part, float* domega, int nparts, int n) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= n) return;
+  float s = 0.f;
+  for (int i = 0; i < nparts; ++i) s += part[(size_t)i * n + e];
+  domega[e] += s;
+}
+
+// ================================================================== host
+namespace {
+
+struct Geo {
+  int chains, MF, Cs, nt, N;
+  int E;
+};
+
+Geo geometry(const Problem& p) {
+  Geo g;
+  g.chains = p.chains();
+  g.MF = p.M;
+  g.Cs = p.slice_len();
+  g.nt = (g.Cs + T - 1) / T;
+  g.N = p.num_slices();
+  g.E = g.MF * 65;
+  return g;
+}
+
+struct Ws {
+  int* err;
+  __nv_bfloat16* om16;
+  float *st_hi, *st_lo, *delta;
+  float *g_hi, *g_lo, *gdelta, *rowstat, *part;
+};
+
+Ws carve(Carver& cv, const Geo& g, bool bwd) {
+  Ws w{};
+  const size_t C = g.chains;
+  w.err = cv.take<int>(64);
+  w.om16 = cv.take<__nv_bfloat16>((size_t)2 * g.MF * D);
+  w.st_hi = cv.take<float>(C * g.E);
+  w.st_lo = cv.take<float>(C * g.E);
+  w.delta = cv.take<float>(C * g.nt * g.E);
+  if (bwd) {
+    w.g_hi = cv.take<float>(C * g.E);
+    w.g_lo = cv.take<float>(C * g.E);
+    w.gdelta = cv.take<float>(C * g.nt * g.E);
+    w.rowstat = cv.take<float>(C * g.nt * T * 2);
+    w.part = cv.take<float>(C * g.nt * (size_t)g.MF * D);
+  }
+  return w;
+}
+
+// dynamic shared memory of each kernel (plus 1 KB for 1024-byte alignment)
+template <int MF>
+constexpr size_t smem_delta() { return 1024 + 2 * ROWT + Cfg<MF>::OMB + Cfg<MF>::FEATB + 4096; }
+template <int MF>
+constexpr size_t smem_fwd() { return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + MF * 4; }
+template <int MF>
+constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4; }
+
+template <typename F>
+cudaError_t set_smem(F* f, size_t bytes) {
+  return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+template <int MF, int FEAT>
+cudaError_t configure() {
+  static bool done = false;
+  if (done) return cudaSuccess;
+  cudaError_t e;
+  if ((e = set_smem(k_tc_delta<MF, FEAT>, smem_delta<MF>())) != cudaSuccess) return e;
+  if ((e = set_smem(k_tc_fwd<MF, FEAT>, smem_fwd<MF>())) != cudaSuccess) return e;
+  if ((e = set_smem(k_tc_bwd_q<MF, FEAT>, smem_bwd<MF>())) != cudaSuccess) return e;
+  if ((e = set_smem(k_tc_bwd_kv<MF, FEAT>, smem_bwd<MF>())) != cudaSuccess) return e;
+  done = true;
+  return cudaSuccess;
+}
+
+#define TC_TRY(x)                                  \
+  do {                                             \
+    cudaError_t e_ = (x);                          \
+    if (e_ != cudaSuccess) return SLIM_ERR_CUDA;   \
+  } while (0)
+
+unsigned nblk(long long n) { return (unsigned)((n + 255) / 256); }
+
+// Algorithmic work per tile launch, for the profiler.
+double tile_rows(const Geo& g, int b) { return (double)g.chains * b; }
+
+template <int MF, int FEAT>
+slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat16* k,
+                     const __nv_bfloat16* v, const float* omega, __nv_bfloat16* out,
+                     const StateOut& st, void* workspace, cudaStream_t s) {
+  TC_TRY((configure<MF, FEAT>()));
+  const Geo g = geometry(p);
+  Carver cv(workspace);
+  const Ws w = carve(cv, g, false);
+  const size_t SE = (size_t)g.chains * g.E;
+  TC_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  TC_TRY(cudaMemsetAsync(w.st_hi, 0, SE * sizeof(float), s));
+  TC_TRY(cudaMemsetAsync(w.st_lo, 0, SE * sizeof(float), s));
+  {
+    prof::Scope ps(prof::K_TC_PREP, s);
+    k_omega_bf16<<<nblk(MF * D), 256, 0, s>>>(omega, w.om16, MF * D);  // hi and lo
+    TC_TRY(cudaGetLastError());
+  }
+  const double MD = (double)MF * D;
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    const int ntn = (b + T - 1) / T;
+    const double rows = tile_rows(g, b);
+    {
+      // phiK (2dM) and Delta (2dM) per row
+      prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
+      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_delta<MF>(), s>>>(
+          k, v, w.om16, p.L, a, b, ntn, w.delta, w.err);
+      TC_TRY(cudaGetLastError());
+    }
+    TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_FWD, prof::K_TC_SCAN));
+    {
+      // phiQ, phiK (4dM), phiQ S (2dM) per row: the recurrent-form work
+      prof::Scope ps(prof::K_TC_FWD, s, rows * 6.0 * MD, rows * D * 2.0 * 4);
+      k_tc_fwd<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_fwd<MF>(), s>>>(
+          q, k, v, w.om16, w.delta, p.L, a, b, ntn, out, w.err);
+      TC_TRY(cudaGetLastError());
+    }
+  }
+  {
+    prof::Scope ps(prof::K_STATE, s);
+    k_tc_state_out<<<nblk((long long)SE), 256, 0, s>>>(w.st_hi, w.st_lo, st, g.chains, MF);
+    TC_TRY(cudaGetLastError());
+  }
+  return SLIM_OK;
+}
+
+template <int MF, int FEAT>
+slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat16* k,
+                     const __nv_bfloat16* v, const float* omega, const __nv_bfloat16* out,
+                     const __nv_bfloat16* dout, const StateIn& st,
+                     __nv_bfloat16* dq, __nv_bfloat16* dk, __nv_bfloat16* dv, float* domega,
+                     void* workspace, cudaStream_t s) {
+  TC_TRY((configure<MF, FEAT>()));
+  const Geo g = geometry(p);
+  Carver cv(workspace);
+  const Ws w = carve(cv, g, true);
+  const size_t SE = (size_t)g.chains * g.E;
+  TC_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  TC_TRY(cudaMemsetAsync(domega, 0, (size_t)MF * D * sizeof(float), s));
+  TC_TRY(cudaMemsetAsync(w.g_hi, 0, SE * sizeof(float), s));
+  TC_TRY(cudaMemsetAsync(w.g_lo, 0, SE * sizeof(float), s));
+  {
+    prof::Scope ps(prof::K_TC_PREP, s);
+    k_omega_bf16<<<nblk(MF * D), 256, 0, s>>>(omega, w.om16, MF * D);  // hi and lo
+    TC_TRY(cudaGetLastError());
+    k_tc_state_in<<<nblk((long long)SE), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains, MF);
+    TC_TRY(cudaGetLastError());
+  }
+  const double MD = (double)MF * D;
+  for (int n = g.N - 1; n >= 0; --n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    const int ntn = (b + T - 1) / T;
+    const double rows = tile_rows(g, b);
+    {
+      prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
+      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_delta<MF>(), s>>>(
+          k, v, w.om16, p.L, a, b, ntn, w.delta, w.err);
+      TC_TRY(cudaGetLastError());
+    }
+    TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_ROLLBACK, prof::K_TC_SCAN));
+    {
+      // phiQ, phiK (4dM), dphiQ state part (2dM), Gd (2dM), dq (2dM), dOmega_q (2dM)
+      prof::Scope ps(prof::K_TC_BWD_Q, s, rows * 12.0 * MD, rows * D * 2.0 * 6);
+      k_tc_bwd_q<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_bwd<MF>(), s>>>(
+          q, k, v, out, dout, w.om16, w.delta, p.L, a, b, ntn, dq, w.gdelta, w.rowstat, w.part,
+          w.err);
+      TC_TRY(cudaGetLastError());
+    }
+    TC_TRY(launch_scan(s, w.gdelta, w.g_hi, w.g_lo, g.chains, ntn, g.E, SCAN_GREV, prof::K_TC_SCAN));
+    {
+      // phiQ, phiK (4dM), dV state part (2dM), dphiK state part (2dM), dk (2dM), dOmega_k (2dM)
+      prof::Scope ps(prof::K_TC_BWD_KV, s, rows * 12.0 * MD, rows * D * 2.0 * 6);
+      k_tc_bwd_kv<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_bwd<MF>(), s>>>(
+          q, k, v, dout, w.om16, w.gdelta, w.rowstat, p.L, a, b, ntn, dk, dv, w.part, w.err);
+      TC_TRY(cudaGetLastError());
+    }
+    {
+      prof::Scope ps(prof::K_TC_REDUCE, s);
+      k_tc_reduce<<<nblk(MF * D), 256, 0, s>>>(w.part, domega, g.chains * ntn, MF * D);
+      TC_TRY(cudaGetLastError());
+    }
+  }
+  return SLIM_OK;
+}
+
+}  // namespace
+
+bool supports(const Problem& p) {
+  return p.dtype == SLIM_BF16 && p.d == D && (p.M == 128 || p.M == 256) && p.slice_len() >= 64;
+}
+
+size_t workspace_bytes(const Problem& p, bool bwd) {
+  Carver cv(nullptr);
+  carve(cv, geometry(p), bwd);
+  return cv.bytes();
+}
+
+#define TC_DISPATCH(FN, ...)                                                        \
+  do {                                                                              \
+    if (p.M == 256)                                                                 \
+      return p.feature == SLIM_FEAT_EXP ? FN<256, SLIM_FEAT_EXP>(__VA_ARGS__)       \
+                                        : FN<256, SLIM_FEAT_RELU>(__VA_ARGS__);     \
+    return p.feature == SLIM_FEAT_EXP ? FN<128, SLIM_FEAT_EXP>(__VA_ARGS__)         \
+                                      : FN<128, SLIM_FEAT_RELU>(__VA_ARGS__);       \
+  } while (0)
+
+slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
+                const float* omega, void* out, const StateOut& st, void* workspace,
+                cudaStream_t s) {
+  using B16 = __nv_bfloat16;
+  TC_DISPATCH(fwd_impl, p, (const B16*)q, (const B16*)k, (const B16*)v, omega, (B16*)out, st,
+              workspace, s);
+}
+
+slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
+                const float* omega, const void* out, const void* dout, const StateIn& st,
+                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s) {
+  using B16 = __nv_bfloat16;
+  TC_DISPATCH(bwd_impl, p, (const B16*)q, (const B16*)k, (const B16*)v, omega, (const B16*)out,
+              (const B16*)dout, st, (B16*)dq, (B16*)dk, (B16*)dv, domega, workspace, s);
+}
+
+}  // namespace tc
+}  // namespace slim

@@ -1,0 +1,21 @@
+// Tensor-core (tcgen05) path of libslim; see tc_path.cu.
+#pragma once
+#include "common.cuh"
+
+namespace slim {
+namespace tc {
+
+// bf16, d = 64, M in {128, 256}, slices of at least 64 rows.
+bool supports(const Problem& p);
+size_t workspace_bytes(const Problem& p, bool bwd);
+
+slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
+                const float* omega, void* out, const StateOut& st, void* workspace,
+                cudaStream_t s);
+
+slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
+                const float* omega, const void* out, const void* dout, const StateIn& st,
+                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s);
+
+}  // namespace tc
+}  // namespace slim

@@ -27,13 +27,15 @@ SIGNATURES = {
     "slim_version": ([], _i),
     "slim_fwd_workspace_size": ([_i] * 6 + [_i, _i, ctypes.POINTER(_sz)], _i),
     "slim_bwd_workspace_size": ([_i] * 6 + [_i, _i, ctypes.POINTER(_sz)], _i),
-    "slim_fwd": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 3 + [_p, _sz, _p], _i),
-    "slim_bwd": ([_p] * 8 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
+    "slim_fwd": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 5 + [_p, _sz, _p], _i),
+    "slim_bwd": ([_p] * 10 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
     "slim_check_device_error": ([_p, _p], _i),
     "slim_launch_count": ([], ctypes.c_ulonglong),
     "slim_profiler_enable": ([_i], None),
     "slim_profiler_reset": ([], None),
     "slim_profiler_read": ([_p, _i], _i),
+    "slim_tc_selftest": ([_i, _i, _i, _i, _p, _p, _p, _p, _p], _i),
+    "slim_path_for": ([_i] * 6 + [_i, _i, ctypes.POINTER(_i)], _i),
 }
 
 
@@ -88,6 +90,14 @@ def workspace_size(B, H, L, d, M, C, dtype, feature, backward):
     return n.value
 
 
+def path_for(B, H, L, d, M, C, dtype, feature):
+    """1 if the tensor-core kernels serve this problem, 0 for the fp32 path."""
+    r = _i(0)
+    _check(library().slim_path_for(B, H, L, d, M, C, DTYPES[dtype], FEATURES[feature],
+                                   ctypes.byref(r)), "slim_path_for")
+    return r.value
+
+
 def _stream_handle(stream):
     s = torch.cuda.current_stream() if stream is None else stream
     return ctypes.c_void_p(s.cuda_stream)
@@ -105,25 +115,37 @@ def _require_cuda(*ts):
             raise RuntimeError("libslim needs contiguous tensors")
 
 
-def forward(q, k, v, omega, C, feature="exp", workspace=None, stream=None):
-    """slim_fwd: returns (out, S_state, z_state)."""
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def forward(q, k, v, omega, C, feature="exp", workspace=None, stream=None, residuals=False):
+    """slim_fwd: returns (out, S_state, z_state), or with residuals=True
+    (out, S_state, z_state, S_state_lo, z_state_lo) -- the low-order parts of
+    the carried state, which slim_bwd uses to start its rollback exactly."""
     _require_cuda(q, k, v, omega)
     B, H, L, d, M = _dims(q, omega)
     out = torch.empty_like(q)
     S_state = torch.empty(B, H, M, d, dtype=torch.float32, device=q.device)
     z_state = torch.empty(B, H, M, dtype=torch.float32, device=q.device)
+    S_lo = torch.empty_like(S_state) if residuals else None
+    z_lo = torch.empty_like(z_state) if residuals else None
     need = workspace_size(B, H, L, d, M, C, q.dtype, feature, False)
     ws = workspace if workspace is not None else _workspace(need, q.device)
     _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
                               B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
                               out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
-                              ws.data_ptr(), ws.numel(), _stream_handle(stream)), "slim_fwd")
+                              _ptr(S_lo), _ptr(z_lo), ws.data_ptr(), ws.numel(),
+                              _stream_handle(stream)), "slim_fwd")
+    if residuals:
+        return out, S_state, z_state, S_lo, z_lo
     return out, S_state, z_state
 
 
 def backward(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp", workspace=None,
-             stream=None):
-    """slim_bwd: returns (dq, dk, dv, domega)."""
+             stream=None, S_lo=None, z_lo=None):
+    """slim_bwd: returns (dq, dk, dv, domega).  S_lo / z_lo: the residuals
+    from forward(..., residuals=True), or None."""
     _require_cuda(q, k, v, omega, out, dout, S_state, z_state)
     B, H, L, d, M = _dims(q, omega)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
@@ -132,33 +154,34 @@ def backward(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp", work
     ws = workspace if workspace is not None else _workspace(need, q.device)
     _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
                               out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
-                              z_state.data_ptr(), B, H, L, d, M, C, DTYPES[q.dtype],
-                              FEATURES[feature], dq.data_ptr(), dk.data_ptr(), dv.data_ptr(),
-                              domega.data_ptr(), ws.data_ptr(), ws.numel(),
+                              z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo), B, H, L, d, M, C,
+                              DTYPES[q.dtype], FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
+                              dv.data_ptr(), domega.data_ptr(), ws.data_ptr(), ws.numel(),
                               _stream_handle(stream)), "slim_bwd")
     return dq, dk, dv, domega
 
 
-def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None):
+def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None,
+                 S_lo=None, z_lo=None):
     """slim_fwd into caller-allocated outputs and workspace (no allocation)."""
     B, H, L, d, M = _dims(q, omega)
     _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
                               B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
                               out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
-                              workspace.data_ptr(), workspace.numel(), _stream_handle(stream)),
-           "slim_fwd")
+                              _ptr(S_lo), _ptr(z_lo), workspace.data_ptr(), workspace.numel(),
+                              _stream_handle(stream)), "slim_fwd")
 
 
 def backward_into(q, k, v, omega, out, dout, S_state, z_state, C, feature, dq, dk, dv, domega,
-                  workspace, stream=None):
+                  workspace, stream=None, S_lo=None, z_lo=None):
     """slim_bwd into caller-allocated gradients and workspace (no allocation)."""
     B, H, L, d, M = _dims(q, omega)
     _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
                               out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
-                              z_state.data_ptr(), B, H, L, d, M, C, DTYPES[q.dtype],
-                              FEATURES[feature], dq.data_ptr(), dk.data_ptr(), dv.data_ptr(),
-                              domega.data_ptr(), workspace.data_ptr(), workspace.numel(),
-                              _stream_handle(stream)), "slim_bwd")
+                              z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo), B, H, L, d, M, C,
+                              DTYPES[q.dtype], FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
+                              dv.data_ptr(), domega.data_ptr(), workspace.data_ptr(),
+                              workspace.numel(), _stream_handle(stream)), "slim_bwd")
 
 
 def check_device_error(workspace, stream=None):
@@ -192,24 +215,36 @@ def profiler_read():
             for i in range(min(n, 64))]
 
 
+def tc_selftest(A, B, a_mn, b_mn):
+    """D = A @ B through one chain of tcgen05 MMAs (diagnostic of the
+    tensor-core operand layouts); A [128, K], B [K, N] bf16 CUDA tensors."""
+    _require_cuda(A, B)
+    K, N = B.shape
+    D = torch.empty(A.shape[0], N, dtype=torch.float32, device=A.device)
+    err = torch.zeros(1, dtype=torch.int32, device=A.device)
+    _check(library().slim_tc_selftest(a_mn, b_mn, K, N, A.data_ptr(), B.data_ptr(), D.data_ptr(),
+                                      err.data_ptr(), _stream_handle(None)), "slim_tc_selftest")
+    return D, err
+
+
 class SlimAttention(torch.autograd.Function):
     """Causal linear attention with the SLiM forward/backward (state carried
     across slices of C rows; backward by rollback, no stored activations)."""
 
     @staticmethod
     def forward(ctx, q, k, v, omega, C, feature):
-        out, S_state, z_state = forward(q.contiguous(), k.contiguous(), v.contiguous(),
-                                        omega.contiguous(), C, feature)
-        ctx.save_for_backward(q, k, v, omega, out, S_state, z_state)
+        out, S, z, S_lo, z_lo = forward(q.contiguous(), k.contiguous(), v.contiguous(),
+                                        omega.contiguous(), C, feature, residuals=True)
+        ctx.save_for_backward(q, k, v, omega, out, S, z, S_lo, z_lo)
         ctx.C, ctx.feature = C, feature
         return out
 
     @staticmethod
     def backward(ctx, dout):
-        q, k, v, omega, out, S_state, z_state = ctx.saved_tensors
+        q, k, v, omega, out, S, z, S_lo, z_lo = ctx.saved_tensors
         dq, dk, dv, domega = backward(q.contiguous(), k.contiguous(), v.contiguous(),
-                                      omega.contiguous(), out, dout.contiguous(), S_state,
-                                      z_state, ctx.C, ctx.feature)
+                                      omega.contiguous(), out, dout.contiguous(), S, z, ctx.C,
+                                      ctx.feature, S_lo=S_lo, z_lo=z_lo)
         return dq, dk, dv, domega, None, None
 
 

@@ -18,11 +18,14 @@ def to64(t):
 
 def gpu_run(x, C, feature, dout=None):
     """x: dict of device tensors from workloads.make_inputs."""
-    out, S, z = slim.forward(x["q"], x["k"], x["v"], x["omega"], C, feature)
+    out, S, z, S_lo, z_lo = slim.forward(x["q"], x["k"], x["v"], x["omega"], C, feature,
+                                         residuals=True)
     dq, dk, dv, dom = slim.backward(x["q"], x["k"], x["v"], x["omega"], out,
-                                    x["dout"] if dout is None else dout, S, z, C, feature)
+                                    x["dout"] if dout is None else dout, S, z, C, feature,
+                                    S_lo=S_lo, z_lo=z_lo)
     torch.cuda.synchronize()
-    return {"out": out, "S_state": S, "z_state": z, "dq": dq, "dk": dk, "dv": dv, "domega": dom}
+    return {"out": out, "S_state": S, "z_state": z, "dq": dq, "dk": dk, "dv": dv, "domega": dom,
+            "S_lo": S_lo, "z_lo": z_lo}
 
 
 def oracle_run(xc, C, feature, dout=None):

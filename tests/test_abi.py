@@ -93,14 +93,15 @@ def test_bad_enums_and_null_out(lib):
 FAKE = 0x10000  # aligned, never dereferenced: every call below fails validation first
 
 
-def fwd_call(lib, ptrs=None, dims=(1, 1, 8, 16, 32, 4), dt=0, ft=0, wsp=FAKE, wsb=0):
+def fwd_call(lib, ptrs=None, dims=(1, 1, 8, 16, 32, 4), dt=0, ft=0, wsp=FAKE, wsb=0, lo=(None, None)):
     p = ptrs or [FAKE] * 7
-    return lib.slim_fwd(p[0], p[1], p[2], p[3], *dims, dt, ft, p[4], p[5], p[6], wsp, wsb, None)
+    return lib.slim_fwd(p[0], p[1], p[2], p[3], *dims, dt, ft, p[4], p[5], p[6], lo[0], lo[1],
+                        wsp, wsb, None)
 
 
-def bwd_call(lib, ptrs=None, dims=(1, 1, 8, 16, 32, 4), wsp=FAKE, wsb=0):
+def bwd_call(lib, ptrs=None, dims=(1, 1, 8, 16, 32, 4), wsp=FAKE, wsb=0, lo=(None, None)):
     p = ptrs or [FAKE] * 12
-    return lib.slim_bwd(*p[:8], *dims, 0, 0, *p[8:12], wsp, wsb, None)
+    return lib.slim_bwd(*p[:8], lo[0], lo[1], *dims, 0, 0, *p[8:12], wsp, wsb, None)
 
 
 def test_fwd_rejects_before_launch(lib):
@@ -116,6 +117,8 @@ def test_fwd_rejects_before_launch(lib):
     assert fwd_call(lib, wsb=need - 1) == WORKSPACE
     assert fwd_call(lib, wsp=None, wsb=need) == WORKSPACE
     assert fwd_call(lib, wsp=FAKE + 16, wsb=need) == INVALID   # workspace not 256-aligned
+    assert fwd_call(lib, lo=(FAKE + 4, None)) == INVALID         # misaligned residual
+    assert fwd_call(lib, lo=(None, FAKE + 8), wsb=need - 1) == INVALID
 
 
 def test_bwd_rejects_before_launch(lib):
@@ -128,6 +131,7 @@ def test_bwd_rejects_before_launch(lib):
     _, need = ws(1, 1, 8, 16, 32, 4, bwd=True)
     assert bwd_call(lib, wsb=need - 1) == WORKSPACE
     assert bwd_call(lib, dims=(1, 1, 8, 16, 31, 4)) == UNSUPPORTED
+    assert bwd_call(lib, lo=(FAKE, FAKE + 4)) == INVALID
 
 
 def test_binding_refuses_cpu_tensors():

@@ -110,7 +110,7 @@ def test_deterministic_and_bwd_leaves_state(cuda_device):
         assert torch.equal(a[n], b[n]), n
     from paper_2012_11346_gb300 import slim
     g2 = slim.backward(x["q"], x["k"], x["v"], x["omega"], a["out"], x["dout"], a["S_state"],
-                       a["z_state"], w.C, w.feature)
+                       a["z_state"], w.C, w.feature, S_lo=a["S_lo"], z_lo=a["z_lo"])
     torch.cuda.synchronize()
     assert torch.equal(a["S_state"], S0) and torch.equal(a["z_state"], z0)
     for n, t in zip(("dq", "dk", "dv", "domega"), g2):
