@@ -49,6 +49,12 @@ struct Cfg {
 };
 
 // ------------------------------------------------------------------ helpers
+// NG warps share each TMEM lane quarter: warp w serves rows 32(w%4)..+31 and
+// column group w/4 of every row-wise epilogue, so a row's element-wise work
+// is spread over NG threads.
+constexpr int NG = 4;
+constexpr int NTHR = 128 * NG;
+
 __device__ __forceinline__ float row_norm2(const uint8_t* tile, int r) {
   float s = 0.f;
 #pragma unroll
@@ -66,9 +72,27 @@ __device__ __forceinline__ float row_norm2(const uint8_t* tile, int r) {
   return s;
 }
 
-// fp32 [R][64] global -> bf16 row tile (R rows), all 128 threads.
+// sum_m phi[r][m] z[m] over the bf16 feature tile row (all MF columns).
+template <int MF>
+__device__ __forceinline__ float row_dot_z(const uint8_t* phi, int r, const float* z) {
+  float s = 0.f;
+#pragma unroll 4
+  for (int c = 0; c < MF; c += 8) {
+    uint4 v = ld_chunk(phi, T, r, c);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float a, b;
+      unpack_bf16(w[i], a, b);
+      s = fmaf(a, z[c + 2 * i], fmaf(b, z[c + 2 * i + 1], s));
+    }
+  }
+  return s;
+}
+
+// fp32 [R][64] global -> bf16 row tile (R rows), all NTHR threads.
 __device__ __forceinline__ void load_f32_rows64(uint8_t* tile, int R, const float* g, int tid) {
-  for (int e = tid; e < R * 8; e += 128) {
+  for (int e = tid; e < R * 8; e += NTHR) {
     const int r = e >> 3, c = (e & 7) * 8;
     const float4 a = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c);
     const float4 b = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c + 4);
@@ -77,18 +101,17 @@ __device__ __forceinline__ void load_f32_rows64(uint8_t* tile, int R, const floa
   }
 }
 
-// Reads the projection P = X Omega^T of this thread's row from TMEM, applies
-// the feature map and stores phi (bf16) into the [128][MF] feature tile.
-// Returns sum_m phi_m z_m when z != nullptr.
+// Reads this thread's column group of the projection P = X Omega^T from TMEM,
+// applies the feature map, stores phi (bf16) into the [128][MF] feature tile.
 template <int MF, int FEAT>
-__device__ __forceinline__ float feature_epilogue(uint32_t trow, uint8_t* phi, int r, float x2,
-                                                  bool valid, const float* z) {
+__device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
+                                                 float x2, bool valid) {
+  constexpr int W = MF / NG;
   // exp map: phi = 2^(p log2e - (|x|^2/2) log2e - log2 sqrt(M))
   const float bias = -0.5f * x2 * kLog2e - 0.5f * log2f((float)MF);
   const float relu_scale = rsqrtf((float)MF);
-  float acc = 0.f;
 #pragma unroll 1
-  for (int c0 = 0; c0 < MF; c0 += 32) {
+  for (int c0 = cg * W; c0 < (cg + 1) * W; c0 += 32) {
     float v[32];
     tmem_ld32(trow + c0, v);
     uint32_t pk[16];
@@ -103,14 +126,12 @@ __device__ __forceinline__ float feature_epilogue(uint32_t trow, uint8_t* phi, i
         b = fmaxf(v[i + 1], 0.f) * relu_scale;
       }
       if (!valid) a = b = 0.f;
-      if (z) acc = fmaf(a, z[c0 + i], fmaf(b, z[c0 + i + 1], acc));
       pk[i / 2] = pack_bf16(a, b);
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q)
       st_chunk(phi, T, r, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
   }
-  return acc;
 }
 
 // Loads 16 bf16 of a feature-tile row (columns c..c+15) as floats.
@@ -122,6 +143,20 @@ __device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, flo
 #pragma unroll
     for (int i = 0; i < 4; ++i) unpack_bf16(w[i], f[8 * h + 2 * i], f[8 * h + 2 * i + 1]);
   }
+}
+
+// 16 fp32 values -> 16 bf16 at global dst (32 bytes, 16-byte aligned).
+__device__ __forceinline__ void st_row16(__nv_bfloat16* dst, const float* v) {
+  uint4* d = reinterpret_cast<uint4*>(dst);
+  d[0] = make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
+                    pack_bf16(v[6], v[7]));
+  d[1] = make_uint4(pack_bf16(v[8], v[9]), pack_bf16(v[10], v[11]), pack_bf16(v[12], v[13]),
+                    pack_bf16(v[14], v[15]));
+}
+__device__ __forceinline__ void st_f32x16(float* dst, const float* v) {
+  float4* o = reinterpret_cast<float4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
 }
 
 struct Sync {
@@ -157,9 +192,27 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
     if (abort_) goto teardown;       \
   } while (0)
 
+#define TC_PROLOGUE()                                    \
+  const int tid = threadIdx.x, warp = tid >> 5;         \
+  const int row = 32 * (warp & 3) + (tid & 31);         \
+  const int cg = warp >> 2;                             \
+  (void)cg;                                             \
+  if (tid == 0) {                                       \
+    abort_ = 0;                                         \
+    mbar_init(smem_u32(&mbar), 1);                      \
+    mbar_fence_init();                                  \
+  }                                                     \
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512)
+
+#define TC_TEARDOWN()                                   \
+  teardown:                                             \
+  tc_fence_before();                                    \
+  __syncthreads();                                      \
+  if (warp == 0) tmem_dealloc(tmem_base, 512)
+
 // ================================================================== tc_delta
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(NTHR, 1)
     k_tc_delta(const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
                const __nv_bfloat16* __restrict__ om16, int L, int a, int b, int nt,
                float* __restrict__ delta, int* err) {
@@ -174,30 +227,24 @@ __global__ void __launch_bounds__(128, 1)
   __shared__ __align__(8) uint64_t mbar;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
-
-  if (tid == 0) {
-    abort_ = 0;
-    mbar_init(smem_u32(&mbar), 1);
-    mbar_fence_init();
-  }
-  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
-  load_rows64(sK, T, K + g0, valid, tid, 128);
-  load_rows64(sV, T, V + g0, valid, tid, 128);
-  load_rows64(sOm, MF, om16, MF, tid, 128);
-  load_rows64(sPhi, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phi overwrites it
-  for (int e = tid; e < 4096 / 16; e += 128)
+  TC_PROLOGUE();
+  load_rows64(sK, T, K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, V + g0, valid, tid, NTHR);
+  load_rows64(sOm, MF, om16, MF, tid, NTHR);
+  load_rows64(sPhi, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phi overwrites it
+  for (int e = tid; e < 4096 / 16; e += NTHR)
     reinterpret_cast<uint4*>(sOnes)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
-    const float x2 = row_norm2(sK, tid);
+    const float x2 = row_norm2(sK, row);
     publish();
     const uint32_t tmem = tmem_base;
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
       const uint32_t aK = smem_u32(sK), aOm = smem_u32(sOm), aOl = smem_u32(sPhi);
@@ -208,7 +255,7 @@ __global__ void __launch_bounds__(128, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-    feature_epilogue<MF, FEAT>(trow, sPhi, tid, x2, tid < valid, nullptr);
+    feature_epilogue<MF, FEAT>(trow, sPhi, row, cg, x2, row < valid);
     publish();
     if (tid == 0) {
       const uint32_t aPhi = smem_u32(sPhi), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
@@ -223,29 +270,23 @@ __global__ void __launch_bounds__(128, 1)
     TC_WAIT(sy);
     float* dst = delta + ((size_t)c * nt + t) * C::E;
     for (int h = 0; h < C::MH; ++h) {
-      const int m = 128 * h + tid;
-      float v[32];
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        tmem_ld32(trow + 256 + 64 * h + 32 * q, v);
-        float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      const int m = 128 * h + row;
+      float v[16];
+      tmem_ld16(trow + 256 + 64 * h + 16 * cg, v);
+      st_f32x16(dst + (size_t)m * 64 + 16 * cg, v);
+      if (cg == 0) {
+        float zz;
+        tmem_ld1(trow + 384 + 16 * h, zz);
+        dst[MF * 64 + m] = zz;
       }
-      float zz;
-      tmem_ld1(trow + 384 + 16 * h, zz);
-      dst[MF * 64 + m] = zz;
     }
   }
-teardown:
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem_base, 512);
+  TC_TEARDOWN();
 }
 
 // ================================================================== tc_fwd
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(NTHR, 1)
     k_tc_fwd(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
              const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ om16,
              const float* __restrict__ pfx, int L, int a, int b, int nt,
@@ -262,35 +303,30 @@ __global__ void __launch_bounds__(128, 1)
   uint8_t* sS = sOm;
   uint8_t* sV = sOm + C::OMB;
   float* sZ = reinterpret_cast<float*>(sV + ROWT);
+  float* red = sZ + MF;            // [NG][128] row-sum partials
   __shared__ __align__(8) uint64_t mbar;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
   const float* P = pfx + ((size_t)c * nt + t) * C::E;
-
-  if (tid == 0) {
-    abort_ = 0;
-    mbar_init(smem_u32(&mbar), 1);
-    mbar_fence_init();
-  }
-  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
-  load_rows64(sQ, T, Q + g0, valid, tid, 128);
-  load_rows64(sK, T, K + g0, valid, tid, 128);
-  load_rows64(sV, T, V + g0, valid, tid, 128);
-  load_rows64(sOm, MF, om16, MF, tid, 128);
-  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phiQ overwrites it
-  for (int m = tid; m < MF; m += 128) sZ[m] = P[MF * 64 + m];
+  TC_PROLOGUE();
+  load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
+  load_rows64(sK, T, K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, V + g0, valid, tid, NTHR);
+  load_rows64(sOm, MF, om16, MF, tid, NTHR);
+  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
+  for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
-    const float q2 = row_norm2(sQ, tid), k2 = row_norm2(sK, tid);
-    const bool rv = tid < valid;
+    const float q2 = row_norm2(sQ, row), k2 = row_norm2(sK, row);
+    const bool rv = row < valid;
     publish();
     const uint32_t tmem = tmem_base;
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -305,8 +341,8 @@ __global__ void __launch_bounds__(128, 1)
     }
     TC_WAIT(sy);
     load_f32_rows64(sS, MF, P, tid);  // Omega no longer needed: S_t takes its place
-    const float dz = feature_epilogue<MF, FEAT>(trow, sPhiQ, tid, q2, rv, sZ);
-    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, tid, k2, rv, nullptr);
+    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
       const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK), aS = smem_u32(sS);
@@ -316,18 +352,19 @@ __global__ void __launch_bounds__(128, 1)
       }
       mma_commit(sy.mbar);
     }
+    const float dz = row_dot_z<MF>(sPhiQ, row, sZ);  // phiQ z_t, overlapping the MMAs
     TC_WAIT(sy);
-    // A row: inclusive causal mask, bf16, row sum of the rounded values
-    float rs = 0.f;
-#pragma unroll 1
-    for (int c0 = 0; c0 < T; c0 += 32) {
+    {
+      // A: inclusive causal mask, bf16; row sum of the rounded values
       float v[32];
+      const int c0 = 32 * cg;
       tmem_ld32(trow + c0, v);
       uint32_t pk[16];
+      float rs = 0.f;
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
-        const float x0 = (c0 + i <= tid) ? v[i] : 0.f;
-        const float x1 = (c0 + i + 1 <= tid) ? v[i + 1] : 0.f;
+        const float x0 = (c0 + i <= row) ? v[i] : 0.f;
+        const float x1 = (c0 + i + 1 <= row) ? v[i + 1] : 0.f;
         pk[i / 2] = pack_bf16(x0, x1);
         float r0, r1;
         unpack_bf16(pk[i / 2], r0, r1);
@@ -335,7 +372,8 @@ __global__ void __launch_bounds__(128, 1)
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        st_chunk(sA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+        st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+      red[cg * T + row] = rs;
     }
     publish();
     if (tid == 0) {
@@ -344,36 +382,26 @@ __global__ void __launch_bounds__(128, 1)
         mma(tmem + 128, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), 1);
       mma_commit(sy.mbar);
     }
+    float rs = 0.f;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) rs += red[g * T + row];
     TC_WAIT(sy);
     {
       const float den = rs + dz;
       const float inv = den != 0.f ? 1.f / den : 0.f;
-      __nv_bfloat16* o = out + g0 + (size_t)tid * D;
+      float v[16];
+      tmem_ld16(trow + 128 + 16 * cg, v);  // every lane loads (warp-aligned op)
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        float v[32];
-        tmem_ld32(trow + 128 + 32 * q, v);  // every lane loads (warp-aligned op)
-        if (rv) {
-          uint4* dst = reinterpret_cast<uint4*>(o + 32 * q);
-#pragma unroll
-          for (int i = 0; i < 4; ++i)
-            dst[i] = make_uint4(pack_bf16(v[8 * i] * inv, v[8 * i + 1] * inv),
-                                pack_bf16(v[8 * i + 2] * inv, v[8 * i + 3] * inv),
-                                pack_bf16(v[8 * i + 4] * inv, v[8 * i + 5] * inv),
-                                pack_bf16(v[8 * i + 6] * inv, v[8 * i + 7] * inv));
-        }
-      }
+      for (int i = 0; i < 16; ++i) v[i] *= inv;
+      if (rv) st_row16(out + g0 + (size_t)row * D + 16 * cg, v);
     }
   }
-teardown:
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem_base, 512);
+  TC_TEARDOWN();
 }
 
 // ================================================================== tc_bwd_q
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(NTHR, 1)
     k_tc_bwd_q(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
                const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ Out,
                const __nv_bfloat16* __restrict__ dOut, const __nv_bfloat16* __restrict__ om16,
@@ -386,51 +414,46 @@ __global__ void __launch_bounds__(128, 1)
   uint8_t* sPhiQ = base;
   uint8_t* sPhiK = sPhiQ + C::FEATB;  // later: u
   uint8_t* sU = sPhiK;
-  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [dA (2 tiles) | S_t] -> [Q | - | Omega]
+  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [dA (2 tiles) | S_t] -> [Q | red | Omega]
   uint8_t* sQ = sX;
   uint8_t* sK = sX + ROWT;
   uint8_t* sdA = sX;
   uint8_t* sOm = sX + 2 * ROWT;
   uint8_t* sS = sOm;
-  uint8_t* sV = sOm + C::OMB;         // later: dden as a K-major [16][128] operand
+  float* redU = reinterpret_cast<float*>(sX + ROWT);  // [NG][128], phase 4
+  uint8_t* sV = sOm + C::OMB;         // later: dden as a K-major [16][128] operand + row sums
   uint8_t* sDd = sV;
+  float* redA = reinterpret_cast<float*>(sV + 8192);  // [NG][128], phase 2
   uint8_t* sDo = sV + ROWT;           // dout, then dnum in place
   float* sZ = reinterpret_cast<float*>(sDo + ROWT);
   __shared__ __align__(8) uint64_t mbar;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
   const float* P = pfx + ((size_t)c * nt + t) * C::E;
-
-  if (tid == 0) {
-    abort_ = 0;
-    mbar_init(smem_u32(&mbar), 1);
-    mbar_fence_init();
-  }
-  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
-  load_rows64(sQ, T, Q + g0, valid, tid, 128);
-  load_rows64(sK, T, K + g0, valid, tid, 128);
-  load_rows64(sV, T, V + g0, valid, tid, 128);
-  load_rows64(sDo, T, dOut + g0, valid, tid, 128);
-  load_rows64(sOm, MF, om16, MF, tid, 128);
-  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phiQ overwrites it
-  for (int m = tid; m < MF; m += 128) sZ[m] = P[MF * 64 + m];
+  TC_PROLOGUE();
+  load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
+  load_rows64(sK, T, K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, V + g0, valid, tid, NTHR);
+  load_rows64(sDo, T, dOut + g0, valid, tid, NTHR);
+  load_rows64(sOm, MF, om16, MF, tid, NTHR);
+  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
+  for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
-    const bool rv = tid < valid;
-    const float q2 = row_norm2(sQ, tid), k2 = row_norm2(sK, tid);
-    // <dout_r, out_r>
-    float rowdot = 0.f;
+    const bool rv = row < valid;
+    const float q2 = row_norm2(sQ, row), k2 = row_norm2(sK, row);
+    float rowdot = 0.f;  // <dout_r, out_r>
     if (rv) {
-      const __nv_bfloat16* orow = Out + g0 + (size_t)tid * D;
+      const __nv_bfloat16* orow = Out + g0 + (size_t)row * D;
 #pragma unroll
       for (int c8 = 0; c8 < 64; c8 += 8) {
         const uint4 o = *reinterpret_cast<const uint4*>(orow + c8);
-        const uint4 g = ld_chunk(sDo, T, tid, c8);
+        const uint4 g = ld_chunk(sDo, T, row, c8);
         const uint32_t ow[4] = {o.x, o.y, o.z, o.w}, gw[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -443,7 +466,7 @@ __global__ void __launch_bounds__(128, 1)
     }
     publish();
     const uint32_t tmem = tmem_base;
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -458,8 +481,8 @@ __global__ void __launch_bounds__(128, 1)
     }
     TC_WAIT(sy);
     load_f32_rows64(sS, MF, P, tid);
-    const float dz = feature_epilogue<MF, FEAT>(trow, sPhiQ, tid, q2, rv, sZ);
-    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, tid, k2, rv, nullptr);
+    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
       const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
@@ -470,29 +493,34 @@ __global__ void __launch_bounds__(128, 1)
         mma(tmem + 128, kmaj(aDo, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
       mma_commit(sy.mbar);
     }
+    const float dz = row_dot_z<MF>(sPhiQ, row, sZ);
     TC_WAIT(sy);
-    float rs = 0.f;
-#pragma unroll 1
-    for (int c0 = 0; c0 < T; c0 += 32) {
+    {
       float v[32];
-      tmem_ld32(trow + c0, v);
+      tmem_ld32(trow + 32 * cg, v);
+      float rs = 0.f;
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
-        const float x0 = (c0 + i <= tid) ? v[i] : 0.f;
-        const float x1 = (c0 + i + 1 <= tid) ? v[i + 1] : 0.f;
+        const float x0 = (32 * cg + i <= row) ? v[i] : 0.f;
+        const float x1 = (32 * cg + i + 1 <= row) ? v[i + 1] : 0.f;
         float r0, r1;
         unpack_bf16(pack_bf16(x0, x1), r0, r1);
         rs += r0 + r1;
       }
+      redA[cg * T + row] = rs;  // V is no longer read: its tile holds the partials
     }
+    __syncthreads();
+    float rs = 0.f;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) rs += redA[g * T + row];
     const float den = rs + dz;
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     const float dden = live ? -rowdot * inv : 0.f;
-    // dnum = dout / den, in place of dout
+    // dnum = dout / den, in place of dout (this thread's 16 columns)
 #pragma unroll
-    for (int c8 = 0; c8 < 64; c8 += 8) {
-      const uint4 g = ld_chunk(sDo, T, tid, c8);
+    for (int c8 = 16 * cg; c8 < 16 * cg + 16; c8 += 8) {
+      const uint4 g = ld_chunk(sDo, T, row, c8);
       const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
       uint32_t pw[4];
 #pragma unroll
@@ -501,33 +529,31 @@ __global__ void __launch_bounds__(128, 1)
         unpack_bf16(gw[i], g0f, g1f);
         pw[i] = pack_bf16(g0f * inv, g1f * inv);
       }
-      st_chunk(sDo, T, tid, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
+      st_chunk(sDo, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
     }
-    // dA = tril(dnum V^T + dden)
-#pragma unroll 1
-    for (int c0 = 0; c0 < T; c0 += 32) {
+    {
+      // dA = tril(dnum V^T + dden), this thread's 32 columns
       float v[32];
+      const int c0 = 32 * cg;
       tmem_ld32(trow + 128 + c0, v);
       uint32_t pk[16];
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
-        const float x0 = (live && c0 + i <= tid) ? fmaf(v[i], inv, dden) : 0.f;
-        const float x1 = (live && c0 + i + 1 <= tid) ? fmaf(v[i + 1], inv, dden) : 0.f;
+        const float x0 = (live && c0 + i <= row) ? fmaf(v[i], inv, dden) : 0.f;
+        const float x1 = (live && c0 + i + 1 <= row) ? fmaf(v[i + 1], inv, dden) : 0.f;
         pk[i / 2] = pack_bf16(x0, x1);
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        st_chunk(sdA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+        st_chunk(sdA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
     }
     // dden as the first row of a K-major [16][128] operand (other rows zero)
-    {
-      const __nv_bfloat16 zb = __float2bfloat16_rn(0.f);
-      for (int n = 0; n < 16; ++n)
-        *reinterpret_cast<__nv_bfloat16*>(sDd + tile_off(16, n, tid)) =
-            n == 0 ? __float2bfloat16_rn(dden) : zb;
-    }
-    if (rv) {
-      float* rsw = rowstat + (((size_t)c * nt + t) * T + tid) * 2;
+#pragma unroll
+    for (int n = 4 * cg; n < 4 * cg + 4; ++n)
+      *reinterpret_cast<__nv_bfloat16*>(sDd + tile_off(16, n, row)) =
+          __float2bfloat16_rn(n == 0 ? dden : 0.f);
+    if (rv && cg == 0) {
+      float* rsw = rowstat + (((size_t)c * nt + t) * T + row) * 2;
       rsw[0] = den;
       rsw[1] = dden;
     }
@@ -551,57 +577,58 @@ __global__ void __launch_bounds__(128, 1)
     {
       float* dst = gdelta + ((size_t)c * nt + t) * C::E;
       for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + tid;
-        float v[32];
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          tmem_ld32(trow + 64 * h + 32 * q, v);
-          float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        const int m = 128 * h + row;
+        float v[16];
+        tmem_ld16(trow + 64 * h + 16 * cg, v);
+        st_f32x16(dst + (size_t)m * 64 + 16 * cg, v);
+        if (cg == 0) {
+          float zz;
+          tmem_ld1(trow + 128 + 16 * h, zz);
+          dst[MF * 64 + m] = zz;
         }
-        float zz;
-        tmem_ld1(trow + 128 + 16 * h, zz);
-        dst[MF * 64 + m] = zz;
       }
     }
-    // dphiQ -> u (into the phiK tile)
-    float usum = 0.f;
-    const float rscale = rsqrtf((float)MF);
+    {
+      // dphiQ (+ dden z_t) -> u (into the phiK tile), this thread's columns
+      constexpr int W = MF / NG;
+      float usum = 0.f;
+      const float rscale = rsqrtf((float)MF);
 #pragma unroll 1
-    for (int c0 = 0; c0 < MF; c0 += 32) {
-      float v[32];
-      tmem_ld32(trow + 256 + c0, v);
-      uint32_t pk[16];
+      for (int c0 = cg * W; c0 < (cg + 1) * W; c0 += 32) {
+        float v[32];
+        tmem_ld32(trow + 256 + c0, v);
+        uint32_t pk[16];
 #pragma unroll
-      for (int s16 = 0; s16 < 32; s16 += 16) {
-        float f[16];
-        ld_feat16(sPhiQ, tid, c0 + s16, f);
+        for (int s16 = 0; s16 < 32; s16 += 16) {
+          float f[16];
+          ld_feat16(sPhiQ, row, c0 + s16, f);
 #pragma unroll
-        for (int i = 0; i < 16; i += 2) {
-          float u0 = fmaf(dden, sZ[c0 + s16 + i], v[s16 + i]);
-          float u1 = fmaf(dden, sZ[c0 + s16 + i + 1], v[s16 + i + 1]);
-          if (FEAT == SLIM_FEAT_EXP) {
-            u0 *= f[i];
-            u1 *= f[i + 1];
-          } else {
-            u0 = f[i] > 0.f ? u0 * rscale : 0.f;
-            u1 = f[i + 1] > 0.f ? u1 * rscale : 0.f;
+          for (int i = 0; i < 16; i += 2) {
+            float u0 = fmaf(dden, sZ[c0 + s16 + i], v[s16 + i]);
+            float u1 = fmaf(dden, sZ[c0 + s16 + i + 1], v[s16 + i + 1]);
+            if (FEAT == SLIM_FEAT_EXP) {
+              u0 *= f[i];
+              u1 *= f[i + 1];
+            } else {
+              u0 = f[i] > 0.f ? u0 * rscale : 0.f;
+              u1 = f[i + 1] > 0.f ? u1 * rscale : 0.f;
+            }
+            if (!live) u0 = u1 = 0.f;
+            pk[(s16 + i) / 2] = pack_bf16(u0, u1);
+            float r0, r1;
+            unpack_bf16(pk[(s16 + i) / 2], r0, r1);
+            usum += r0 + r1;
           }
-          if (!live) u0 = u1 = 0.f;
-          pk[(s16 + i) / 2] = pack_bf16(u0, u1);
-          float r0, r1;
-          unpack_bf16(pk[(s16 + i) / 2], r0, r1);
-          usum += r0 + r1;
         }
-      }
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        st_chunk(sU, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+        for (int q = 0; q < 4; ++q)
+          st_chunk(sU, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+      }
+      redU[cg * T + row] = usum;
     }
     // Q and Omega again for dq = u Omega - q sum(u) and dOmega += u^T q
-    load_rows64(sQ, T, Q + g0, valid, tid, 128);
-    load_rows64(sOm, MF, om16, MF, tid, 128);
+    load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
+    load_rows64(sOm, MF, om16, MF, tid, NTHR);
     cp_async_wait_all();
     publish();
     if (tid == 0) {
@@ -614,56 +641,34 @@ __global__ void __launch_bounds__(128, 1)
               idesc_bf16(T, 64, 1, 1), k0 > 0);
       mma_commit(sy.mbar);
     }
+    float us = 0.f;
+    if (FEAT == SLIM_FEAT_EXP) {
+#pragma unroll
+      for (int g = 0; g < NG; ++g) us += redU[g * T + row];
+    }
     TC_WAIT(sy);
     {
-      float xq[64];
+      float xq[16];
+      ld_feat16(sQ, row, 16 * cg, xq);
+      float v[16];
+      tmem_ld16(trow + 16 * cg, v);
 #pragma unroll
-      for (int c8 = 0; c8 < 64; c8 += 8) {
-        const uint4 g = ld_chunk(sQ, T, tid, c8);
-        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) unpack_bf16(gw[i], xq[c8 + 2 * i], xq[c8 + 2 * i + 1]);
-      }
-      const float us = (FEAT == SLIM_FEAT_EXP) ? usum : 0.f;
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        float v[32];
-        tmem_ld32(trow + 32 * q, v);
-        if (rv) {
-          uint4* dst = reinterpret_cast<uint4*>(dq + g0 + (size_t)tid * D + 32 * q);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int j = 32 * q + 8 * i;
-            dst[i] = make_uint4(pack_bf16(fmaf(-us, xq[j], v[8 * i]), fmaf(-us, xq[j + 1], v[8 * i + 1])),
-                                pack_bf16(fmaf(-us, xq[j + 2], v[8 * i + 2]), fmaf(-us, xq[j + 3], v[8 * i + 3])),
-                                pack_bf16(fmaf(-us, xq[j + 4], v[8 * i + 4]), fmaf(-us, xq[j + 5], v[8 * i + 5])),
-                                pack_bf16(fmaf(-us, xq[j + 6], v[8 * i + 6]), fmaf(-us, xq[j + 7], v[8 * i + 7])));
-          }
-        }
-      }
+      for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xq[i], v[i]);
+      if (rv) st_row16(dq + g0 + (size_t)row * D + 16 * cg, v);
       float* dst = part + ((size_t)c * nt + t) * (size_t)(MF * 64);
       for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + tid;
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          float v[32];
-          tmem_ld32(trow + 64 + 64 * h + 32 * q, v);
-          float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-        }
+        const int m = 128 * h + row;
+        tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
+        st_f32x16(dst + (size_t)m * 64 + 16 * cg, v);
       }
     }
   }
-teardown:
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem_base, 512);
+  TC_TEARDOWN();
 }
 
 // ================================================================== tc_bwd_kv
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(NTHR, 1)
     k_tc_bwd_kv(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
                 const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ dOut,
                 const __nv_bfloat16* __restrict__ om16, const float* __restrict__ gsfx,
@@ -676,11 +681,12 @@ __global__ void __launch_bounds__(128, 1)
   uint8_t* sPhiQ = base;               // later: u
   uint8_t* sU = sPhiQ;
   uint8_t* sPhiK = sPhiQ + C::FEATB;
-  uint8_t* sX = sPhiK + C::FEATB;      // [Q | K | Omega] -> [A | G_t] -> [dA | G_t] -> [K | - | Omega]
+  uint8_t* sX = sPhiK + C::FEATB;      // [Q | K | Omega] -> [A | G_t] -> [dA | G_t] -> [K | red | Omega]
   uint8_t* sQ = sX;
   uint8_t* sK = sX + ROWT;
   uint8_t* sA = sX;
   uint8_t* sKr = sX;
+  float* redU = reinterpret_cast<float*>(sX + ROWT);
   uint8_t* sOm = sX + 2 * ROWT;
   uint8_t* sG = sOm;
   uint8_t* sV = sOm + C::OMB;
@@ -689,42 +695,36 @@ __global__ void __launch_bounds__(128, 1)
   __shared__ __align__(8) uint64_t mbar;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, warp = tid >> 5;
+  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
   const float* G = gsfx + ((size_t)c * nt + t) * C::E;
-
-  if (tid == 0) {
-    abort_ = 0;
-    mbar_init(smem_u32(&mbar), 1);
-    mbar_fence_init();
-  }
-  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
-  load_rows64(sQ, T, Q + g0, valid, tid, 128);
-  load_rows64(sK, T, K + g0, valid, tid, 128);
-  load_rows64(sV, T, V + g0, valid, tid, 128);
-  load_rows64(sDn, T, dOut + g0, valid, tid, 128);
-  load_rows64(sOm, MF, om16, MF, tid, 128);
-  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, 128);  // Omega lo, until phiQ overwrites it
-  for (int m = tid; m < MF; m += 128) sGz[m] = G[MF * 64 + m];
+  TC_PROLOGUE();
+  load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
+  load_rows64(sK, T, K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, V + g0, valid, tid, NTHR);
+  load_rows64(sDn, T, dOut + g0, valid, tid, NTHR);
+  load_rows64(sOm, MF, om16, MF, tid, NTHR);
+  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
+  for (int m = tid; m < MF; m += NTHR) sGz[m] = G[MF * 64 + m];
   float den = 0.f, dden = 0.f;
-  if (tid < valid) {
-    const float* rsr = rowstat + (((size_t)c * nt + t) * T + tid) * 2;
+  if (row < valid) {
+    const float* rsr = rowstat + (((size_t)c * nt + t) * T + row) * 2;
     den = rsr[0];
     dden = rsr[1];
   }
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
-    const bool rv = tid < valid;
+    const bool rv = row < valid;
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     if (!live) dden = 0.f;
-    const float q2 = row_norm2(sQ, tid), k2 = row_norm2(sK, tid);
+    const float q2 = row_norm2(sQ, row), k2 = row_norm2(sK, row);
 #pragma unroll
-    for (int c8 = 0; c8 < 64; c8 += 8) {  // dnum = dout / den, in place
-      const uint4 g = ld_chunk(sDn, T, tid, c8);
+    for (int c8 = 16 * cg; c8 < 16 * cg + 16; c8 += 8) {  // dnum = dout / den, in place
+      const uint4 g = ld_chunk(sDn, T, row, c8);
       const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
       uint32_t pw[4];
 #pragma unroll
@@ -733,11 +733,11 @@ __global__ void __launch_bounds__(128, 1)
         unpack_bf16(gw[i], g0f, g1f);
         pw[i] = pack_bf16(g0f * inv, g1f * inv);
       }
-      st_chunk(sDn, T, tid, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
+      st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
     }
     publish();
     const uint32_t tmem = tmem_base;
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -752,8 +752,8 @@ __global__ void __launch_bounds__(128, 1)
     }
     TC_WAIT(sy);
     load_f32_rows64(sG, MF, G, tid);  // G_t(S) replaces Omega
-    feature_epilogue<MF, FEAT>(trow, sPhiQ, tid, q2, rv, nullptr);
-    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, tid, k2, rv, nullptr);
+    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
       const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
@@ -765,17 +765,17 @@ __global__ void __launch_bounds__(128, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-#pragma unroll 1
-    for (int c0 = 0; c0 < T; c0 += 32) {  // A -> smem (masked, bf16)
+    {  // A -> smem (masked, bf16), this thread's 32 columns
       float v[32];
+      const int c0 = 32 * cg;
       tmem_ld32(trow + c0, v);
       uint32_t pk[16];
 #pragma unroll
       for (int i = 0; i < 32; i += 2)
-        pk[i / 2] = pack_bf16((c0 + i <= tid) ? v[i] : 0.f, (c0 + i + 1 <= tid) ? v[i + 1] : 0.f);
+        pk[i / 2] = pack_bf16((c0 + i <= row) ? v[i] : 0.f, (c0 + i + 1 <= row) ? v[i + 1] : 0.f);
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        st_chunk(sA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+        st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
     }
     publish();
     if (tid == 0) {
@@ -790,32 +790,25 @@ __global__ void __launch_bounds__(128, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {  // dv
-      float v[32];
-      tmem_ld32(trow + 32 * q, v);
-      if (rv) {
-        uint4* dst = reinterpret_cast<uint4*>(dv + g0 + (size_t)tid * D + 32 * q);
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          dst[i] = make_uint4(pack_bf16(v[8 * i], v[8 * i + 1]), pack_bf16(v[8 * i + 2], v[8 * i + 3]),
-                              pack_bf16(v[8 * i + 4], v[8 * i + 5]), pack_bf16(v[8 * i + 6], v[8 * i + 7]));
-      }
+    {
+      float v[16];
+      tmem_ld16(trow + 16 * cg, v);  // dv
+      if (rv) st_row16(dv + g0 + (size_t)row * D + 16 * cg, v);
     }
-#pragma unroll 1
-    for (int c0 = 0; c0 < T; c0 += 32) {  // dA = tril(dnum V^T + dden) -> smem
+    {  // dA = tril(dnum V^T + dden) -> smem, this thread's 32 columns
       float v[32];
+      const int c0 = 32 * cg;
       tmem_ld32(trow + 128 + c0, v);
       uint32_t pk[16];
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
-        const float x0 = (live && c0 + i <= tid) ? v[i] + dden : 0.f;
-        const float x1 = (live && c0 + i + 1 <= tid) ? v[i + 1] + dden : 0.f;
+        const float x0 = (live && c0 + i <= row) ? v[i] + dden : 0.f;
+        const float x1 = (live && c0 + i + 1 <= row) ? v[i + 1] + dden : 0.f;
         pk[i / 2] = pack_bf16(x0, x1);
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        st_chunk(sA, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+        st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
     }
     publish();
     if (tid == 0) {
@@ -825,41 +818,46 @@ __global__ void __launch_bounds__(128, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-    float usum = 0.f;
-    const float rscale = rsqrtf((float)MF);
+    {
+      // dphiK (+ g_z) -> u (into the phiQ tile), this thread's columns
+      constexpr int W = MF / NG;
+      float usum = 0.f;
+      const float rscale = rsqrtf((float)MF);
 #pragma unroll 1
-    for (int c0 = 0; c0 < MF; c0 += 32) {  // dphiK (+ g_z) -> u (into the phiQ tile)
-      float v[32];
-      tmem_ld32(trow + 256 + c0, v);
-      uint32_t pk[16];
+      for (int c0 = cg * W; c0 < (cg + 1) * W; c0 += 32) {
+        float v[32];
+        tmem_ld32(trow + 256 + c0, v);
+        uint32_t pk[16];
 #pragma unroll
-      for (int s16 = 0; s16 < 32; s16 += 16) {
-        float f[16];
-        ld_feat16(sPhiK, tid, c0 + s16, f);
+        for (int s16 = 0; s16 < 32; s16 += 16) {
+          float f[16];
+          ld_feat16(sPhiK, row, c0 + s16, f);
 #pragma unroll
-        for (int i = 0; i < 16; i += 2) {
-          float u0 = v[s16 + i] + sGz[c0 + s16 + i];
-          float u1 = v[s16 + i + 1] + sGz[c0 + s16 + i + 1];
-          if (FEAT == SLIM_FEAT_EXP) {
-            u0 *= f[i];
-            u1 *= f[i + 1];
-          } else {
-            u0 = f[i] > 0.f ? u0 * rscale : 0.f;
-            u1 = f[i + 1] > 0.f ? u1 * rscale : 0.f;
+          for (int i = 0; i < 16; i += 2) {
+            float u0 = v[s16 + i] + sGz[c0 + s16 + i];
+            float u1 = v[s16 + i + 1] + sGz[c0 + s16 + i + 1];
+            if (FEAT == SLIM_FEAT_EXP) {
+              u0 *= f[i];
+              u1 *= f[i + 1];
+            } else {
+              u0 = f[i] > 0.f ? u0 * rscale : 0.f;
+              u1 = f[i + 1] > 0.f ? u1 * rscale : 0.f;
+            }
+            if (!rv) u0 = u1 = 0.f;
+            pk[(s16 + i) / 2] = pack_bf16(u0, u1);
+            float r0, r1;
+            unpack_bf16(pk[(s16 + i) / 2], r0, r1);
+            usum += r0 + r1;
           }
-          if (!rv) u0 = u1 = 0.f;
-          pk[(s16 + i) / 2] = pack_bf16(u0, u1);
-          float r0, r1;
-          unpack_bf16(pk[(s16 + i) / 2], r0, r1);
-          usum += r0 + r1;
         }
-      }
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        st_chunk(sU, T, tid, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+        for (int q = 0; q < 4; ++q)
+          st_chunk(sU, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+      }
+      redU[cg * T + row] = usum;
     }
-    load_rows64(sKr, T, K + g0, valid, tid, 128);
-    load_rows64(sOm, MF, om16, MF, tid, 128);
+    load_rows64(sKr, T, K + g0, valid, tid, NTHR);
+    load_rows64(sOm, MF, om16, MF, tid, NTHR);
     cp_async_wait_all();
     publish();
     if (tid == 0) {
@@ -872,58 +870,38 @@ __global__ void __launch_bounds__(128, 1)
               idesc_bf16(T, 64, 1, 1), k0 > 0);
       mma_commit(sy.mbar);
     }
+    float us = 0.f;
+    if (FEAT == SLIM_FEAT_EXP) {
+#pragma unroll
+      for (int g = 0; g < NG; ++g) us += redU[g * T + row];
+    }
     TC_WAIT(sy);
     {
-      float xk[64];
+      float xk[16];
+      ld_feat16(sKr, row, 16 * cg, xk);
+      float v[16];
+      tmem_ld16(trow + 16 * cg, v);
 #pragma unroll
-      for (int c8 = 0; c8 < 64; c8 += 8) {
-        const uint4 g = ld_chunk(sKr, T, tid, c8);
-        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) unpack_bf16(gw[i], xk[c8 + 2 * i], xk[c8 + 2 * i + 1]);
-      }
-      const float us = (FEAT == SLIM_FEAT_EXP) ? usum : 0.f;
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        float v[32];
-        tmem_ld32(trow + 32 * q, v);
-        if (rv) {
-          uint4* dst = reinterpret_cast<uint4*>(dk + g0 + (size_t)tid * D + 32 * q);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int j = 32 * q + 8 * i;
-            dst[i] = make_uint4(pack_bf16(fmaf(-us, xk[j], v[8 * i]), fmaf(-us, xk[j + 1], v[8 * i + 1])),
-                                pack_bf16(fmaf(-us, xk[j + 2], v[8 * i + 2]), fmaf(-us, xk[j + 3], v[8 * i + 3])),
-                                pack_bf16(fmaf(-us, xk[j + 4], v[8 * i + 4]), fmaf(-us, xk[j + 5], v[8 * i + 5])),
-                                pack_bf16(fmaf(-us, xk[j + 6], v[8 * i + 6]), fmaf(-us, xk[j + 7], v[8 * i + 7])));
-          }
-        }
-      }
+      for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xk[i], v[i]);
+      if (rv) st_row16(dk + g0 + (size_t)row * D + 16 * cg, v);
       float* dst = part + ((size_t)c * nt + t) * (size_t)(MF * 64);
       for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + tid;
+        const int m = 128 * h + row;
+        tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
+        float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 16 * cg);
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          float v[32];
-          tmem_ld32(trow + 64 + 64 * h + 32 * q, v);
-          float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 32 * q);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            float4 x = o[i];
-            x.x += v[4 * i];
-            x.y += v[4 * i + 1];
-            x.z += v[4 * i + 2];
-            x.w += v[4 * i + 3];
-            o[i] = x;
-          }
+        for (int i = 0; i < 4; ++i) {
+          float4 x = o[i];
+          x.x += v[4 * i];
+          x.y += v[4 * i + 1];
+          x.z += v[4 * i + 2];
+          x.w += v[4 * i + 3];
+          o[i] = x;
         }
       }
     }
   }
-teardown:
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem_base, 512);
+  TC_TEARDOWN();
 }
 
 // ================================================================== small kernels
@@ -966,12 +944,26 @@ __global__ void k_tc_state_in(StateIn st, float* hi, float* lo, int chains, int 
     lo[i] = st.z_lo ? st.z_lo[c * MF + (e - (long long)MF * 64)] : 0.f;
   }
 }
-// dOmega[e] += sum over the slice's partials, fixed order
-__global__ void k_tc_reduce(const float* part, float* domega, int nparts, int n) {
+// dOmega[e] += sum over the slice's partials, in a fixed order: each of
+// RSPLIT blocks sums a contiguous range of partials, then one pass adds the
+// RSPLIT sums in order.
+constexpr int RSPLIT = 16;
+__global__ void k_tc_reduce1(const float* part, float* sums, int nparts, int n) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= n) return;
+  const int per = (nparts + RSPLIT - 1) / RSPLIT;
+  const int i0 = blockIdx.y * per, i1 = min(nparts, i0 + per);
+  float s = 0.f;
+#pragma unroll 4
+  for (int i = i0; i < i1; ++i) s += part[(size_t)i * n + e];
+  sums[(size_t)blockIdx.y * n + e] = s;
+}
+__global__ void k_tc_reduce2(const float* sums, float* domega, int n) {
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= n) return;
   float s = 0.f;
-  for (int i = 0; i < nparts; ++i) s += part[(size_t)i * n + e];
+#pragma unroll
+  for (int i = 0; i < RSPLIT; ++i) s += sums[(size_t)i * n + e];
   domega[e] += s;
 }
 
@@ -998,7 +990,7 @@ struct Ws {
   int* err;
   __nv_bfloat16* om16;
   float *st_hi, *st_lo, *delta;
-  float *g_hi, *g_lo, *gdelta, *rowstat, *part;
+  float *g_hi, *g_lo, *gdelta, *rowstat, *part, *rsums;
 };
 
 Ws carve(Carver& cv, const Geo& g, bool bwd) {
@@ -1015,6 +1007,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
     w.gdelta = cv.take<float>(C * g.nt * g.E);
     w.rowstat = cv.take<float>(C * g.nt * T * 2);
     w.part = cv.take<float>(C * g.nt * (size_t)g.MF * D);
+    w.rsums = cv.take<float>((size_t)RSPLIT * g.MF * D);
   }
   return w;
 }
@@ -1023,7 +1016,9 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
 template <int MF>
 constexpr size_t smem_delta() { return 1024 + 2 * ROWT + Cfg<MF>::OMB + Cfg<MF>::FEATB + 4096; }
 template <int MF>
-constexpr size_t smem_fwd() { return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + MF * 4; }
+constexpr size_t smem_fwd() {
+  return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + MF * 4 + NG * T * 4;
+}
 template <int MF>
 constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4; }
 
@@ -1079,17 +1074,18 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
     const int ntn = (b + T - 1) / T;
     const double rows = tile_rows(g, b);
     {
-      // phiK (2dM) and Delta (2dM) per row
+      // algorithmic: phiK (2dM) + Delta (2dM) per row
       prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
-      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_delta<MF>(), s>>>(
+      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_delta<MF>(), s>>>(
           k, v, w.om16, p.L, a, b, ntn, w.delta, w.err);
       TC_TRY(cudaGetLastError());
     }
     TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_FWD, prof::K_TC_SCAN));
     {
-      // phiQ, phiK (4dM), phiQ S (2dM) per row: the recurrent-form work
-      prof::Scope ps(prof::K_TC_FWD, s, rows * 6.0 * MD, rows * D * 2.0 * 4);
-      k_tc_fwd<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_fwd<MF>(), s>>>(
+      // algorithmic: phiQ (2dM) + readout phiQ S (2dM) per row; the phiK
+      // recomputation and the 128 x 128 tile products are not counted
+      prof::Scope ps(prof::K_TC_FWD, s, rows * 4.0 * MD, rows * D * 2.0 * 4);
+      k_tc_fwd<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_fwd<MF>(), s>>>(
           q, k, v, w.om16, w.delta, p.L, a, b, ntn, out, w.err);
       TC_TRY(cudaGetLastError());
     }
@@ -1130,31 +1126,37 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
     const int ntn = (b + T - 1) / T;
     const double rows = tile_rows(g, b);
     {
+      // algorithmic: phiK recomputation (2dM) + rollback Delta (2dM) per row
       prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
-      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_delta<MF>(), s>>>(
+      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_delta<MF>(), s>>>(
           k, v, w.om16, p.L, a, b, ntn, w.delta, w.err);
       TC_TRY(cudaGetLastError());
     }
     TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_ROLLBACK, prof::K_TC_SCAN));
     {
-      // phiQ, phiK (4dM), dphiQ state part (2dM), Gd (2dM), dq (2dM), dOmega_q (2dM)
-      prof::Scope ps(prof::K_TC_BWD_Q, s, rows * 12.0 * MD, rows * D * 2.0 * 6);
-      k_tc_bwd_q<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_bwd<MF>(), s>>>(
+      // algorithmic: phiQ recomputation, dnum S^T, G_S update, dq VJP, dOmega_q
+      // (2dM each) per row
+      prof::Scope ps(prof::K_TC_BWD_Q, s, rows * 10.0 * MD, rows * D * 2.0 * 6);
+      k_tc_bwd_q<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_bwd<MF>(), s>>>(
           q, k, v, out, dout, w.om16, w.delta, p.L, a, b, ntn, dq, w.gdelta, w.rowstat, w.part,
           w.err);
       TC_TRY(cudaGetLastError());
     }
     TC_TRY(launch_scan(s, w.gdelta, w.g_hi, w.g_lo, g.chains, ntn, g.E, SCAN_GREV, prof::K_TC_SCAN));
     {
-      // phiQ, phiK (4dM), dV state part (2dM), dphiK state part (2dM), dk (2dM), dOmega_k (2dM)
-      prof::Scope ps(prof::K_TC_BWD_KV, s, rows * 12.0 * MD, rows * D * 2.0 * 6);
-      k_tc_bwd_kv<MF, FEAT><<<dim3(ntn, g.chains), 128, smem_bwd<MF>(), s>>>(
+      // algorithmic: dV state part, dphiK state part, dk VJP, dOmega_k (2dM
+      // each) per row
+      prof::Scope ps(prof::K_TC_BWD_KV, s, rows * 8.0 * MD, rows * D * 2.0 * 6);
+      k_tc_bwd_kv<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_bwd<MF>(), s>>>(
           q, k, v, dout, w.om16, w.gdelta, w.rowstat, p.L, a, b, ntn, dk, dv, w.part, w.err);
       TC_TRY(cudaGetLastError());
     }
     {
       prof::Scope ps(prof::K_TC_REDUCE, s);
-      k_tc_reduce<<<nblk(MF * D), 256, 0, s>>>(w.part, domega, g.chains * ntn, MF * D);
+      k_tc_reduce1<<<dim3(nblk(MF * D), RSPLIT), 256, 0, s>>>(w.part, w.rsums, g.chains * ntn,
+                                                              MF * D);
+      TC_TRY(cudaGetLastError());
+      k_tc_reduce2<<<nblk(MF * D), 256, 0, s>>>(w.rsums, domega, MF * D);
       TC_TRY(cudaGetLastError());
     }
   }
