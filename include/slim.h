@@ -199,6 +199,37 @@ int slim_profiler_read(slim_kernel_stats* stats, int cap);
 slim_status slim_tc_selftest(int a_mn, int b_mn, int K, int N, const void* A, const void* B,
                              float* D, int* err, void* stream);
 
+/*
+ * Allocation-free forward (the paper has no counterpart; this is for callers
+ * that cannot allocate device memory).  Some callers cannot call cudaMalloc or
+ * any allocating routine where they run the forward -- code inside an
+ * allocator or memory-pool callback, hosts that fix their device memory at
+ * start-up, plug-ins whose host owns every allocation.  slim_fwd_noalloc is
+ * slim_fwd with the workspace replaced by a scratch array that the library
+ * itself reserves in device memory: SLIM_NOALLOC_SCRATCH_BYTES (16 MiB) on
+ * every GPU that loads the library, held until the process exits.  The caller
+ * still passes every input and output (same arguments and rules as slim_fwd,
+ * minus the workspace).
+ *   - Allocates nothing: no cudaMalloc, cudaFree or other allocating call
+ *     (keep the launch profiler off, it creates CUDA events when on).
+ *   - Returns SLIM_ERR_WORKSPACE when the problem needs more scratch than
+ *     SLIM_NOALLOC_SCRATCH_BYTES (compare slim_fwd_workspace_size); use
+ *     slim_fwd with a caller workspace, or a smaller C or B*H, then.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture on the device.
+ *   - All calls share the one array and it keeps the last call's contents;
+ *     the call clears, on its stream, what must start at zero.  Calls that
+ *     overlap on the GPU (different streams, or several host threads) race
+ *     on the array and give wrong results: order them on one stream.
+ */
+#define SLIM_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+slim_status slim_fwd_noalloc(const void* q, const void* k, const void* v, const float* omega,
+                             int B, int H, int L, int d, int M, int C,
+                             slim_dtype dtype, slim_feature feature,
+                             void* out, float* S_state, float* z_state,
+                             float* S_state_lo, float* z_state_lo, void* stream);
+
 #ifdef __cplusplus
 }
 #endif
