@@ -27,6 +27,9 @@ __device__ __forceinline__ float4 neg4(const float4& x) { return make_float4(-x.
 constexpr int KB = 8;
 __global__ void k_scan(float4* buf, float4* hi_p, float4* lo_p, int chains, int nt, int E4,
                        int mode) {
+  // the tile totals come from the kernel just before (programmatic launch)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (long long)chains * E4) return;
   const int c = (int)(idx / E4), e = (int)(idx % E4);
@@ -88,10 +91,19 @@ cudaError_t launch_scan(cudaStream_t s, float* buf, float* hi, float* lo, int ch
   const long long n = (long long)chains * E4;
   // bytes: the tile totals read and rewritten, the pair read and written
   prof::Scope ps(kid, s, 0.0, (double)chains * E * 4.0 * (2.0 * nt + 4.0));
-  k_scan<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(
-      reinterpret_cast<float4*>(buf), reinterpret_cast<float4*>(hi), reinterpret_cast<float4*>(lo),
-      chains, nt, E4, (int)mode);
-  return cudaGetLastError();
+  // launched as a programmatic dependent of the previous kernel in the stream
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((n + 255) / 256));
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_scan, reinterpret_cast<float4*>(buf),
+                            reinterpret_cast<float4*>(hi), reinterpret_cast<float4*>(lo), chains, nt,
+                            E4, (int)mode);
 }
 
 }  // namespace slim

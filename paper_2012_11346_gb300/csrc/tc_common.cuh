@@ -211,6 +211,16 @@ __device__ __forceinline__ void load_rows64(uint8_t* tile, int R, const __nv_bfl
   }
 }
 
+// Programmatic dependent launch: wait until the previous kernel in the stream
+// has completed and its writes are visible (returns at once when the kernel
+// was not launched as a dependent), then let the next kernel start launching.
+// Work before grid_dependency_wait() may only touch data that no kernel of the
+// same call writes (the caller's input tensors).
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ex2 on the MUFU unit (approximate, ~2 ulp), used for the FAVOR+ features.
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;

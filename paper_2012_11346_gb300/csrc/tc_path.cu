@@ -55,41 +55,6 @@ struct Cfg {
 constexpr int NG = 4;
 constexpr int NTHR = 128 * NG;
 
-__device__ __forceinline__ float row_norm2(const uint8_t* tile, int r) {
-  float s = 0.f;
-#pragma unroll
-  for (int c = 0; c < 64; c += 8) {
-    uint4 v = ld_chunk(tile, T, r, c);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float a, b;
-      unpack_bf16(w[i], a, b);
-      s = fmaf(a, a, s);
-      s = fmaf(b, b, s);
-    }
-  }
-  return s;
-}
-
-// sum_m phi[r][m] z[m] over the bf16 feature tile row (all MF columns).
-template <int MF>
-__device__ __forceinline__ float row_dot_z(const uint8_t* phi, int r, const float* z) {
-  float s = 0.f;
-#pragma unroll 4
-  for (int c = 0; c < MF; c += 8) {
-    uint4 v = ld_chunk(phi, T, r, c);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float a, b;
-      unpack_bf16(w[i], a, b);
-      s = fmaf(a, z[c + 2 * i], fmaf(b, z[c + 2 * i + 1], s));
-    }
-  }
-  return s;
-}
-
 // fp32 [R][64] global -> bf16 row tile (R rows), all NTHR threads.
 __device__ __forceinline__ void load_f32_rows64(uint8_t* tile, int R, const float* g, int tid) {
   for (int e = tid; e < R * 8; e += NTHR) {
@@ -101,12 +66,25 @@ __device__ __forceinline__ void load_f32_rows64(uint8_t* tile, int R, const floa
   }
 }
 
+// Loads 16 bf16 of a feature-tile row (columns c..c+15) as floats.
+__device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, float* f) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint4 v = ld_chunk(tile, T, r, c + 8 * h);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) unpack_bf16(w[i], f[8 * h + 2 * i], f[8 * h + 2 * i + 1]);
+  }
+}
+
 // Reads this thread's column group of the projection P = X Omega^T from TMEM,
 // applies the feature map, stores phi (bf16) into the [128][MF] feature tile.
 template <int MF, int FEAT>
-__device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
-                                                 float x2, bool valid) {
+__device__ __forceinline__ float feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
+                                                  float x2, bool valid,
+                                                  const float* z = nullptr) {
   constexpr int W = MF / NG;
+  float dz = 0.f;  // sum over this thread's columns of bf16(phi) * z
   // exp map: phi = 2^(p log2e - (|x|^2/2) log2e - log2 sqrt(M))
   const float bias = -0.5f * x2 * kLog2e - 0.5f * log2f((float)MF);
   const float relu_scale = rsqrtf((float)MF);
@@ -127,22 +105,36 @@ __device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, in
       }
       if (!valid) a = b = 0.f;
       pk[i / 2] = pack_bf16(a, b);
+      if (z) {
+        float ra, rb;
+        unpack_bf16(pk[i / 2], ra, rb);
+        dz = fmaf(ra, z[c0 + i], fmaf(rb, z[c0 + i + 1], dz));
+      }
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q)
       st_chunk(phi, T, r, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
   }
+  return dz;
 }
 
-// Loads 16 bf16 of a feature-tile row (columns c..c+15) as floats.
-__device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, float* f) {
+// Squared norm of columns 16cg..16cg+15 of row r of a [128][64] row tile.
+__device__ __forceinline__ float row_norm2_part(const uint8_t* tile, int r, int cg) {
+  float f[16];
+  ld_feat16(tile, r, 16 * cg, f);
+  float s = 0.f;
 #pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    uint4 v = ld_chunk(tile, T, r, c + 8 * h);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  for (int i = 0; i < 16; ++i) s = fmaf(f[i], f[i], s);
+  return s;
+}
+
+// Sum of the NG column-group partials of each row, through shared scratch
+// red[NG][128] (the caller separates writes and reads with a barrier).
+__device__ __forceinline__ float group_total(const float* red, int row) {
+  float s = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) unpack_bf16(w[i], f[8 * h + 2 * i], f[8 * h + 2 * i + 1]);
-  }
+  for (int g = 0; g < NG; ++g) s += red[g * T + row];
+  return s;
 }
 
 // 16 fp32 values -> 16 bf16 at global dst (32 bytes, 16-byte aligned).
@@ -234,15 +226,16 @@ __global__ void __launch_bounds__(NTHR, 1)
   TC_PROLOGUE();
   load_rows64(sK, T, K + g0, valid, tid, NTHR);
   load_rows64(sV, T, V + g0, valid, tid, NTHR);
+  grid_dependency_wait();  // Omega (bf16) and the delta buffer belong to earlier kernels
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
   load_rows64(sPhi, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phi overwrites it
-  for (int e = tid; e < 4096 / 16; e += NTHR)
-    reinterpret_cast<uint4*>(sOnes)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
-    const float x2 = row_norm2(sK, row);
+    float* redN = reinterpret_cast<float*>(sOnes);  // scratch until the ones are written
+    redN[cg * T + row] = row_norm2_part(sK, row, cg);
     publish();
+    const float x2 = group_total(redN, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
@@ -255,6 +248,8 @@ __global__ void __launch_bounds__(NTHR, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
+    for (int e = tid; e < 4096 / 16; e += NTHR)
+      reinterpret_cast<uint4*>(sOnes)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
     feature_epilogue<MF, FEAT>(trow, sPhi, row, cg, x2, row < valid);
     publish();
     if (tid == 0) {
@@ -316,15 +311,19 @@ __global__ void __launch_bounds__(NTHR, 1)
   load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
   load_rows64(sK, T, K + g0, valid, tid, NTHR);
   load_rows64(sV, T, V + g0, valid, tid, NTHR);
+  grid_dependency_wait();  // the state prefixes come from the scan just before
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
   load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
   for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
-    const float q2 = row_norm2(sQ, row), k2 = row_norm2(sK, row);
     const bool rv = row < valid;
+    float* redN = reinterpret_cast<float*>(sPhiK);  // phiK is written only after phase 1
+    redN[cg * T + row] = row_norm2_part(sQ, row, cg);
+    redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
     publish();
+    const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
@@ -341,7 +340,8 @@ __global__ void __launch_bounds__(NTHR, 1)
     }
     TC_WAIT(sy);
     load_f32_rows64(sS, MF, P, tid);  // Omega no longer needed: S_t takes its place
-    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    float* redZ = reinterpret_cast<float*>(sQ);  // Q, K are dead; A is written after the next wait
+    redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
@@ -352,7 +352,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       }
       mma_commit(sy.mbar);
     }
-    const float dz = row_dot_z<MF>(sPhiQ, row, sZ);  // phiQ z_t, overlapping the MMAs
+    const float dz = group_total(redZ, row);  // phiQ z_t
     TC_WAIT(sy);
     {
       // A: inclusive causal mask, bf16; row sum of the rounded values
@@ -439,6 +439,14 @@ __global__ void __launch_bounds__(NTHR, 1)
   load_rows64(sK, T, K + g0, valid, tid, NTHR);
   load_rows64(sV, T, V + g0, valid, tid, NTHR);
   load_rows64(sDo, T, dOut + g0, valid, tid, NTHR);
+  // this thread's 16 columns of its out row, fetched while the tiles stream in
+  uint4 orow[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+  if (row < valid) {
+    const uint4* src = reinterpret_cast<const uint4*>(Out + g0 + (size_t)row * D + 16 * cg);
+    orow[0] = src[0];
+    orow[1] = src[1];
+  }
+  grid_dependency_wait();  // the state prefixes come from the scan just before
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
   load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
   for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
@@ -446,25 +454,29 @@ __global__ void __launch_bounds__(NTHR, 1)
   __syncthreads();  // rows were copied by other threads
   {
     const bool rv = row < valid;
-    const float q2 = row_norm2(sQ, row), k2 = row_norm2(sK, row);
-    float rowdot = 0.f;  // <dout_r, out_r>
-    if (rv) {
-      const __nv_bfloat16* orow = Out + g0 + (size_t)row * D;
+    float* redN = reinterpret_cast<float*>(sPhiK);  // phiK is written only after phase 1
+    {
+      float part = 0.f;  // <dout_r, out_r> over this thread's 16 columns
 #pragma unroll
-      for (int c8 = 0; c8 < 64; c8 += 8) {
-        const uint4 o = *reinterpret_cast<const uint4*>(orow + c8);
-        const uint4 g = ld_chunk(sDo, T, row, c8);
-        const uint32_t ow[4] = {o.x, o.y, o.z, o.w}, gw[4] = {g.x, g.y, g.z, g.w};
+      for (int h = 0; h < 2; ++h) {
+        const uint4 g = ld_chunk(sDo, T, row, 16 * cg + 8 * h);
+        const uint32_t ow[4] = {orow[h].x, orow[h].y, orow[h].z, orow[h].w};
+        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           float o0, o1, g0f, g1f;
           unpack_bf16(ow[i], o0, o1);
           unpack_bf16(gw[i], g0f, g1f);
-          rowdot = fmaf(o0, g0f, fmaf(o1, g1f, rowdot));
+          part = fmaf(o0, g0f, fmaf(o1, g1f, part));
         }
       }
+      redN[cg * T + row] = row_norm2_part(sQ, row, cg);
+      redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
+      redN[(2 * NG + cg) * T + row] = part;
     }
     publish();
+    const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
+    const float rowdot = group_total(redN + 2 * NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
@@ -481,7 +493,8 @@ __global__ void __launch_bounds__(NTHR, 1)
     }
     TC_WAIT(sy);
     load_f32_rows64(sS, MF, P, tid);
-    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    float* redZ = reinterpret_cast<float*>(sQ);  // Q, K are dead; dA is written after the next wait
+    redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
@@ -493,7 +506,7 @@ __global__ void __launch_bounds__(NTHR, 1)
         mma(tmem + 128, kmaj(aDo, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
       mma_commit(sy.mbar);
     }
-    const float dz = row_dot_z<MF>(sPhiQ, row, sZ);
+    const float dz = group_total(redZ, row);
     TC_WAIT(sy);
     {
       float v[32];
@@ -574,6 +587,10 @@ __global__ void __launch_bounds__(NTHR, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
+    // Q and Omega again (for dq = u Omega - q sum(u) and dOmega += u^T q); the
+    // copies overlap the epilogue below
+    load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
+    load_rows64(sOm, MF, om16, MF, tid, NTHR);
     {
       float* dst = gdelta + ((size_t)c * nt + t) * C::E;
       for (int h = 0; h < C::MH; ++h) {
@@ -626,9 +643,6 @@ __global__ void __launch_bounds__(NTHR, 1)
       }
       redU[cg * T + row] = usum;
     }
-    // Q and Omega again for dq = u Omega - q sum(u) and dOmega += u^T q
-    load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
-    load_rows64(sOm, MF, om16, MF, tid, NTHR);
     cp_async_wait_all();
     publish();
     if (tid == 0) {
@@ -705,6 +719,7 @@ __global__ void __launch_bounds__(NTHR, 1)
   load_rows64(sK, T, K + g0, valid, tid, NTHR);
   load_rows64(sV, T, V + g0, valid, tid, NTHR);
   load_rows64(sDn, T, dOut + g0, valid, tid, NTHR);
+  grid_dependency_wait();  // G suffixes (scan) and row statistics (tc_bwd_q) are earlier kernels'
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
   load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
   for (int m = tid; m < MF; m += NTHR) sGz[m] = G[MF * 64 + m];
@@ -721,7 +736,9 @@ __global__ void __launch_bounds__(NTHR, 1)
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     if (!live) dden = 0.f;
-    const float q2 = row_norm2(sQ, row), k2 = row_norm2(sK, row);
+    float* redN = reinterpret_cast<float*>(sPhiK);  // phiK is written only after phase 1
+    redN[cg * T + row] = row_norm2_part(sQ, row, cg);
+    redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
 #pragma unroll
     for (int c8 = 16 * cg; c8 < 16 * cg + 16; c8 += 8) {  // dnum = dout / den, in place
       const uint4 g = ld_chunk(sDn, T, row, c8);
@@ -736,6 +753,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
     }
     publish();
+    const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
@@ -818,6 +836,9 @@ __global__ void __launch_bounds__(NTHR, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
+    // K and Omega again (dk = u Omega - k sum(u), dOmega += u^T k), overlapping the epilogue
+    load_rows64(sKr, T, K + g0, valid, tid, NTHR);
+    load_rows64(sOm, MF, om16, MF, tid, NTHR);
     {
       // dphiK (+ g_z) -> u (into the phiQ tile), this thread's columns
       constexpr int W = MF / NG;
@@ -856,8 +877,6 @@ __global__ void __launch_bounds__(NTHR, 1)
       }
       redU[cg * T + row] = usum;
     }
-    load_rows64(sKr, T, K + g0, valid, tid, NTHR);
-    load_rows64(sOm, MF, om16, MF, tid, NTHR);
     cp_async_wait_all();
     publish();
     if (tid == 0) {
@@ -919,6 +938,7 @@ __global__ void k_omega_bf16(const float* om, __nv_bfloat16* om16, int n) {
 // state pair [chains][E] <-> S_state [chains][M][64], z_state [chains][M]
 // (the pair is normalised: hi is the rounded state, lo its residual)
 __global__ void k_tc_state_out(const float* hi, const float* lo, StateOut st, int chains, int MF) {
+  grid_dependency_wait();
   const long long E = (long long)MF * 65;
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= chains * E) return;
@@ -949,6 +969,7 @@ __global__ void k_tc_state_in(StateIn st, float* hi, float* lo, int chains, int 
 // RSPLIT sums in order.
 constexpr int RSPLIT = 16;
 __global__ void k_tc_reduce1(const float* part, float* sums, int nparts, int n) {
+  grid_dependency_wait();
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= n) return;
   const int per = (nparts + RSPLIT - 1) / RSPLIT;
@@ -959,6 +980,7 @@ __global__ void k_tc_reduce1(const float* part, float* sums, int nparts, int n) 
   sums[(size_t)blockIdx.y * n + e] = s;
 }
 __global__ void k_tc_reduce2(const float* sums, float* domega, int n) {
+  grid_dependency_wait();
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= n) return;
   float s = 0.f;
@@ -1048,6 +1070,25 @@ cudaError_t configure() {
 
 unsigned nblk(long long n) { return (unsigned)((n + 255) / 256); }
 
+// Launch as a programmatic dependent of the previous kernel in the stream:
+// the kernel may start while its predecessor drains and waits for it inside
+// (grid_dependency_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dep(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Algorithmic work per tile launch, for the profiler.
 double tile_rows(const Geo& g, int b) { return (double)g.chains * b; }
 
@@ -1076,24 +1117,22 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
     {
       // algorithmic: phiK (2dM) + Delta (2dM) per row
       prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
-      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_delta<MF>(), s>>>(
-          k, v, w.om16, p.L, a, b, ntn, w.delta, w.err);
-      TC_TRY(cudaGetLastError());
+      TC_TRY(launch_dep(k_tc_delta<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_delta<MF>(), s,
+                        k, v, w.om16, p.L, a, b, ntn, w.delta, w.err));
     }
     TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_FWD, prof::K_TC_SCAN));
     {
       // algorithmic: phiQ (2dM) + readout phiQ S (2dM) per row; the phiK
       // recomputation and the 128 x 128 tile products are not counted
       prof::Scope ps(prof::K_TC_FWD, s, rows * 4.0 * MD, rows * D * 2.0 * 4);
-      k_tc_fwd<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_fwd<MF>(), s>>>(
-          q, k, v, w.om16, w.delta, p.L, a, b, ntn, out, w.err);
-      TC_TRY(cudaGetLastError());
+      TC_TRY(launch_dep(k_tc_fwd<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_fwd<MF>(), s, q,
+                        k, v, w.om16, w.delta, p.L, a, b, ntn, out, w.err));
     }
   }
   {
     prof::Scope ps(prof::K_STATE, s);
-    k_tc_state_out<<<nblk((long long)SE), 256, 0, s>>>(w.st_hi, w.st_lo, st, g.chains, MF);
-    TC_TRY(cudaGetLastError());
+    TC_TRY(launch_dep(k_tc_state_out, dim3(nblk((long long)SE)), dim3(256), 0, s,
+                      (const float*)w.st_hi, (const float*)w.st_lo, st, g.chains, MF));
   }
   return SLIM_OK;
 }
@@ -1128,36 +1167,33 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
     {
       // algorithmic: phiK recomputation (2dM) + rollback Delta (2dM) per row
       prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
-      k_tc_delta<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_delta<MF>(), s>>>(
-          k, v, w.om16, p.L, a, b, ntn, w.delta, w.err);
-      TC_TRY(cudaGetLastError());
+      TC_TRY(launch_dep(k_tc_delta<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_delta<MF>(), s,
+                        k, v, w.om16, p.L, a, b, ntn, w.delta, w.err));
     }
     TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_ROLLBACK, prof::K_TC_SCAN));
     {
       // algorithmic: phiQ recomputation, dnum S^T, G_S update, dq VJP, dOmega_q
       // (2dM each) per row
       prof::Scope ps(prof::K_TC_BWD_Q, s, rows * 10.0 * MD, rows * D * 2.0 * 6);
-      k_tc_bwd_q<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_bwd<MF>(), s>>>(
-          q, k, v, out, dout, w.om16, w.delta, p.L, a, b, ntn, dq, w.gdelta, w.rowstat, w.part,
-          w.err);
-      TC_TRY(cudaGetLastError());
+      TC_TRY(launch_dep(k_tc_bwd_q<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_bwd<MF>(), s,
+                        q, k, v, out, dout, w.om16, w.delta, p.L, a, b, ntn, dq, w.gdelta,
+                        w.rowstat, w.part, w.err));
     }
     TC_TRY(launch_scan(s, w.gdelta, w.g_hi, w.g_lo, g.chains, ntn, g.E, SCAN_GREV, prof::K_TC_SCAN));
     {
       // algorithmic: dV state part, dphiK state part, dk VJP, dOmega_k (2dM
       // each) per row
       prof::Scope ps(prof::K_TC_BWD_KV, s, rows * 8.0 * MD, rows * D * 2.0 * 6);
-      k_tc_bwd_kv<MF, FEAT><<<dim3(ntn, g.chains), NTHR, smem_bwd<MF>(), s>>>(
-          q, k, v, dout, w.om16, w.gdelta, w.rowstat, p.L, a, b, ntn, dk, dv, w.part, w.err);
-      TC_TRY(cudaGetLastError());
+      TC_TRY(launch_dep(k_tc_bwd_kv<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_bwd<MF>(), s,
+                        q, k, v, dout, w.om16, w.gdelta, w.rowstat, p.L, a, b, ntn, dk, dv, w.part,
+                        w.err));
     }
     {
       prof::Scope ps(prof::K_TC_REDUCE, s);
-      k_tc_reduce1<<<dim3(nblk(MF * D), RSPLIT), 256, 0, s>>>(w.part, w.rsums, g.chains * ntn,
-                                                              MF * D);
-      TC_TRY(cudaGetLastError());
-      k_tc_reduce2<<<nblk(MF * D), 256, 0, s>>>(w.rsums, domega, MF * D);
-      TC_TRY(cudaGetLastError());
+      TC_TRY(launch_dep(k_tc_reduce1, dim3(nblk(MF * D), RSPLIT), dim3(256), 0, s,
+                        (const float*)w.part, w.rsums, g.chains * ntn, MF * D));
+      TC_TRY(launch_dep(k_tc_reduce2, dim3(nblk(MF * D)), dim3(256), 0, s, (const float*)w.rsums,
+                        domega, MF * D));
     }
   }
   return SLIM_OK;
