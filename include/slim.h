@@ -200,6 +200,16 @@ slim_status slim_tc_selftest(int a_mn, int b_mn, int K, int N, const void* A, co
                              float* D, int* err, void* stream);
 
 /*
+ * Diagnostic of the failure path (no counterpart in the paper): one warp
+ * waits on an mbarrier that nothing arrives at.  The wait gives up after its
+ * bounded number of polls (about a second), sets the error word at the start
+ * of `workspace` (a workspace as passed to slim_fwd/slim_bwd, at least 256
+ * bytes) and the kernel returns; slim_check_device_error then reports
+ * SLIM_ERR_TIMEOUT.  Nothing faults and the context stays usable.
+ */
+slim_status slim_diag_wait_timeout(void* workspace, void* stream);
+
+/*
  * Allocation-free forward (the paper has no counterpart; this is for callers
  * that cannot allocate device memory).  Some callers cannot call cudaMalloc or
  * any allocating routine where they run the forward -- code inside an

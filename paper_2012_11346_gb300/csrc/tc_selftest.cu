@@ -66,8 +66,29 @@ __global__ void __launch_bounds__(128) k_tc_selftest(const __nv_bfloat16* A, con
   if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
+// A bounded wait on an mbarrier that nothing arrives at: it gives up after
+// its iteration limit, records the failure in the error word and returns --
+// the same path every kernel takes when a wait gives up.
+__global__ void k_wait_timeout(int* err) {
+  __shared__ __align__(8) uint64_t mbar;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&mbar), 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  mbar_wait(smem_u32(&mbar), 0, err);
+}
+
 }  // namespace tc
 }  // namespace slim
+
+extern "C" slim_status slim_diag_wait_timeout(void* workspace, void* stream) {
+  if (!workspace) return SLIM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  slim::prof::Scope ps(slim::prof::K_TC_SELFTEST, s);
+  slim::tc::k_wait_timeout<<<1, 32, 0, s>>>(static_cast<int*>(workspace));
+  return cudaGetLastError() == cudaSuccess ? SLIM_OK : SLIM_ERR_CUDA;
+}
 
 extern "C" slim_status slim_tc_selftest(int a_mn, int b_mn, int K, int N, const void* A,
                                         const void* B, float* D, int* err, void* stream) {

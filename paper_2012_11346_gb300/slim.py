@@ -37,6 +37,7 @@ SIGNATURES = {
     "slim_tc_selftest": ([_i, _i, _i, _i, _p, _p, _p, _p, _p], _i),
     "slim_path_for": ([_i] * 6 + [_i, _i, ctypes.POINTER(_i)], _i),
     "slim_fwd_noalloc": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 5 + [_p], _i),
+    "slim_diag_wait_timeout": ([_p, _p], _i),
 }
 
 
