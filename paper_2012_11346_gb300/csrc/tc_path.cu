@@ -29,6 +29,7 @@
 #include "common.cuh"
 #include "profiler.h"
 #include "scan.h"
+#include "scan_dev.cuh"
 #include "tc_common.cuh"
 #include "tc_path.h"
 
@@ -55,14 +56,25 @@ struct Cfg {
 constexpr int NG = 4;
 constexpr int NTHR = 128 * NG;
 
-// fp32 [R][64] global -> bf16 row tile (R rows), all NTHR threads.
-__device__ __forceinline__ void load_f32_rows64(uint8_t* tile, int R, const float* g, int tid) {
-  for (int e = tid; e < R * 8; e += NTHR) {
-    const int r = e >> 3, c = (e & 7) * 8;
-    const float4 a = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c);
-    const float4 b = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c + 4);
-    st_chunk(tile, R, r, c, make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w),
-                                       pack_bf16(b.x, b.y), pack_bf16(b.z, b.w)));
+// fp32 [R][64] global -> bf16 row tile (R rows), all NTHR threads.  Every
+// thread issues all of its loads before converting, so they are in flight
+// together.
+template <int R>
+__device__ __forceinline__ void load_f32_rows64(uint8_t* tile, const float* g, int tid) {
+  constexpr int PER = R * 8 / NTHR;  // 16-byte bf16 chunks per thread
+  static_assert(R * 8 % NTHR == 0, "rows must split evenly over the CTA");
+  float4 a[PER], b[PER];
+#pragma unroll
+  for (int i = 0; i < PER; ++i) {
+    const int e = tid + i * NTHR, r = e >> 3, c = (e & 7) * 8;
+    a[i] = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c);
+    b[i] = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c + 4);
+  }
+#pragma unroll
+  for (int i = 0; i < PER; ++i) {
+    const int e = tid + i * NTHR, r = e >> 3, c = (e & 7) * 8;
+    st_chunk(tile, R, r, c, make_uint4(pack_bf16(a[i].x, a[i].y), pack_bf16(a[i].z, a[i].w),
+                                       pack_bf16(b[i].x, b[i].y), pack_bf16(b[i].z, b[i].w)));
   }
 }
 
@@ -204,22 +216,17 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 
 // ================================================================== tc_delta
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(NTHR, 1)
-    k_tc_delta(const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
+__device__ __forceinline__ void role_delta(const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
                const __nv_bfloat16* __restrict__ om16, int L, int a, int b, int nt,
-               float* __restrict__ delta, int* err) {
+               float* __restrict__ delta, int* err,
+    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
-  extern __shared__ uint8_t smem_raw[];
   uint8_t* base = align1024(smem_raw);
   uint8_t* sK = base;
   uint8_t* sV = sK + ROWT;
   uint8_t* sOm = sV + ROWT;
   uint8_t* sPhi = sOm + C::OMB;
   uint8_t* sOnes = sPhi + C::FEATB;  // [16][128] K-major, all ones
-  __shared__ __align__(8) uint64_t mbar;
-  __shared__ uint32_t tmem_base;
-  __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
@@ -281,13 +288,12 @@ __global__ void __launch_bounds__(NTHR, 1)
 
 // ================================================================== tc_fwd
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(NTHR, 1)
-    k_tc_fwd(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+__device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
              const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ om16,
              const float* __restrict__ pfx, int L, int a, int b, int nt,
-             __nv_bfloat16* __restrict__ out, int* err) {
+             __nv_bfloat16* __restrict__ out, int* err,
+    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
-  extern __shared__ uint8_t smem_raw[];
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;
   uint8_t* sPhiK = sPhiQ + C::FEATB;
@@ -299,10 +305,6 @@ __global__ void __launch_bounds__(NTHR, 1)
   uint8_t* sV = sOm + C::OMB;
   float* sZ = reinterpret_cast<float*>(sV + ROWT);
   float* red = sZ + MF;            // [NG][128] row-sum partials
-  __shared__ __align__(8) uint64_t mbar;
-  __shared__ uint32_t tmem_base;
-  __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
@@ -339,7 +341,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-    load_f32_rows64(sS, MF, P, tid);  // Omega no longer needed: S_t takes its place
+    load_f32_rows64<MF>(sS, P, tid);  // Omega no longer needed: S_t takes its place
     float* redZ = reinterpret_cast<float*>(sQ);  // Q, K are dead; A is written after the next wait
     redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
@@ -401,15 +403,14 @@ __global__ void __launch_bounds__(NTHR, 1)
 
 // ================================================================== tc_bwd_q
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(NTHR, 1)
-    k_tc_bwd_q(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+__device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
                const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ Out,
                const __nv_bfloat16* __restrict__ dOut, const __nv_bfloat16* __restrict__ om16,
                const float* __restrict__ pfx, int L, int a, int b, int nt,
                __nv_bfloat16* __restrict__ dq, float* __restrict__ gdelta,
-               float* __restrict__ rowstat, float* __restrict__ part, int* err) {
+               float* __restrict__ rowstat, float* __restrict__ part, int* err,
+    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
-  extern __shared__ uint8_t smem_raw[];
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;
   uint8_t* sPhiK = sPhiQ + C::FEATB;  // later: u
@@ -426,10 +427,6 @@ __global__ void __launch_bounds__(NTHR, 1)
   float* redA = reinterpret_cast<float*>(sV + 8192);  // [NG][128], phase 2
   uint8_t* sDo = sV + ROWT;           // dout, then dnum in place
   float* sZ = reinterpret_cast<float*>(sDo + ROWT);
-  __shared__ __align__(8) uint64_t mbar;
-  __shared__ uint32_t tmem_base;
-  __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
@@ -492,7 +489,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-    load_f32_rows64(sS, MF, P, tid);
+    load_f32_rows64<MF>(sS, P, tid);
     float* redZ = reinterpret_cast<float*>(sQ);  // Q, K are dead; dA is written after the next wait
     redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
@@ -682,15 +679,14 @@ __global__ void __launch_bounds__(NTHR, 1)
 
 // ================================================================== tc_bwd_kv
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(NTHR, 1)
-    k_tc_bwd_kv(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+__device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
                 const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ dOut,
                 const __nv_bfloat16* __restrict__ om16, const float* __restrict__ gsfx,
                 const float* __restrict__ rowstat, int L, int a, int b, int nt,
                 __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv,
-                float* __restrict__ part, int* err) {
+                float* __restrict__ part, int* err,
+    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
-  extern __shared__ uint8_t smem_raw[];
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;               // later: u
   uint8_t* sU = sPhiQ;
@@ -706,10 +702,6 @@ __global__ void __launch_bounds__(NTHR, 1)
   uint8_t* sV = sOm + C::OMB;
   uint8_t* sDn = sV + ROWT;            // dout, then dnum in place
   float* sGz = reinterpret_cast<float*>(sDn + ROWT);
-  __shared__ __align__(8) uint64_t mbar;
-  __shared__ uint32_t tmem_base;
-  __shared__ int abort_;
-  const int t = blockIdx.x, c = blockIdx.y;
   const int row0 = a + t * T;
   const int valid = min(T, b - t * T);
   const size_t g0 = ((size_t)c * L + row0) * D;
@@ -769,7 +761,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);
-    load_f32_rows64(sG, MF, G, tid);  // G_t(S) replaces Omega
+    load_f32_rows64<MF>(sG, G, tid);  // G_t(S) replaces Omega
     feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
@@ -923,6 +915,141 @@ __global__ void __launch_bounds__(NTHR, 1)
   TC_TEARDOWN();
 }
 
+// ================================================================== launches
+// One launch runs tiles of up to four roles (independent work of different
+// slices, longest role first so the short ones fill the last wave); CTA b of
+// a role handles tile b % nt of chain b / nt.
+struct DeltaJob {
+  const __nv_bfloat16 *K, *V, *om16;
+  int L, a, b, nt;
+  float* delta;
+  int* err;
+};
+struct FwdJob {
+  const __nv_bfloat16 *Q, *K, *V, *om16;
+  const float* pfx;
+  int L, a, b, nt;
+  __nv_bfloat16* out;
+  int* err;
+};
+struct BwdQJob {
+  const __nv_bfloat16 *Q, *K, *V, *Out, *dOut, *om16;
+  const float* pfx;
+  int L, a, b, nt;
+  __nv_bfloat16* dq;
+  float *gdelta, *rowstat, *part;
+  int* err;
+};
+struct BwdKVJob {
+  const __nv_bfloat16 *Q, *K, *V, *dOut, *om16;
+  const float *gsfx, *rowstat;
+  int L, a, b, nt;
+  __nv_bfloat16 *dk, *dv;
+  float* part;
+  int* err;
+};
+struct TileJobs {
+  int n_kv, n_q, n_fwd, n_delta;  // CTAs of each role, in dispatch order
+  BwdKVJob kv;
+  BwdQJob q;
+  FwdJob f;
+  DeltaJob d;
+};
+
+template <int MF, int FEAT>
+__global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ TileJobs J) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t mbar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_;
+  int b = blockIdx.x;
+  if (b < J.n_kv) {
+    const BwdKVJob& p = J.kv;
+    role_bwd_kv<MF, FEAT>(p.Q, p.K, p.V, p.dOut, p.om16, p.gsfx, p.rowstat, p.L, p.a, p.b, p.nt,
+                          p.dk, p.dv, p.part, p.err, b % p.nt, b / p.nt, smem_raw, mbar,
+                          tmem_base, abort_);
+    return;
+  }
+  b -= J.n_kv;
+  if (b < J.n_q) {
+    const BwdQJob& p = J.q;
+    role_bwd_q<MF, FEAT>(p.Q, p.K, p.V, p.Out, p.dOut, p.om16, p.pfx, p.L, p.a, p.b, p.nt, p.dq,
+                         p.gdelta, p.rowstat, p.part, p.err, b % p.nt, b / p.nt, smem_raw, mbar,
+                         tmem_base, abort_);
+    return;
+  }
+  b -= J.n_q;
+  if (b < J.n_fwd) {
+    const FwdJob& p = J.f;
+    role_fwd<MF, FEAT>(p.Q, p.K, p.V, p.om16, p.pfx, p.L, p.a, p.b, p.nt, p.out, p.err, b % p.nt,
+                       b / p.nt, smem_raw, mbar, tmem_base, abort_);
+    return;
+  }
+  b -= J.n_fwd;
+  if (b < J.n_delta) {
+    const DeltaJob& p = J.d;
+    role_delta<MF, FEAT>(p.K, p.V, p.om16, p.L, p.a, p.b, p.nt, p.delta, p.err, b % p.nt,
+                         b / p.nt, smem_raw, mbar, tmem_base, abort_);
+  }
+}
+
+// The small steps between tile launches: up to two state scans (the
+// forward/rollback carry of one slice and the state-gradient carry of
+// another), and the two stages of the dOmega reduction of earlier slices.
+constexpr int RSPLIT = 64;
+struct ScanJob {
+  float *buf, *hi, *lo;
+  int chains, nt, E4, mode, blocks;
+};
+struct SmallJobs {
+  ScanJob scan[2];
+  int nscan;
+  // stage 1: sums[split][e] = sum of partials of one range (blocks = r1_bx * RSPLIT)
+  const float* r1_part;
+  float* r1_sums;
+  int r1_nparts, r1_bx;
+  // stage 2: domega[e] += sum over the RSPLIT sums, in order
+  const float* r2_sums;
+  float* r2_domega;
+  int r2_blocks;
+  int n;  // M * 64
+};
+
+__global__ void __launch_bounds__(256) k_tc_small(const __grid_constant__ SmallJobs J) {
+  grid_dependency_wait();
+  int b = blockIdx.x;
+  for (int i = 0; i < J.nscan; ++i) {
+    const ScanJob& q = J.scan[i];
+    if (b < q.blocks) {
+      scan_thread(reinterpret_cast<float4*>(q.buf), reinterpret_cast<float4*>(q.hi),
+                  reinterpret_cast<float4*>(q.lo), q.chains, q.nt, q.E4, q.mode,
+                  (long long)b * 256 + threadIdx.x);
+      return;
+    }
+    b -= q.blocks;
+  }
+  if (b < J.r1_bx * RSPLIT) {
+    const int e = (b % J.r1_bx) * 256 + threadIdx.x, split = b / J.r1_bx;
+    if (e >= J.n) return;
+    const int per = (J.r1_nparts + RSPLIT - 1) / RSPLIT;
+    const int i0 = split * per, i1 = min(J.r1_nparts, i0 + per);
+    float s = 0.f;
+#pragma unroll 4
+    for (int i = i0; i < i1; ++i) s += J.r1_part[(size_t)i * J.n + e];
+    J.r1_sums[(size_t)split * J.n + e] = s;
+    return;
+  }
+  b -= J.r1_bx * RSPLIT;
+  if (b < J.r2_blocks) {
+    const int e = b * 256 + threadIdx.x;
+    if (e >= J.n) return;
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < RSPLIT; ++i) s += J.r2_sums[(size_t)i * J.n + e];
+    J.r2_domega[e] += s;
+  }
+}
+
 // ================================================================== small kernels
 // Omega as a bf16 pair: hi = bf16(Omega), lo = bf16(Omega - hi), so the
 // projections X Omega^T = X hi^T + X lo^T carry ~16 mantissa bits.
@@ -964,31 +1091,6 @@ __global__ void k_tc_state_in(StateIn st, float* hi, float* lo, int chains, int 
     lo[i] = st.z_lo ? st.z_lo[c * MF + (e - (long long)MF * 64)] : 0.f;
   }
 }
-// dOmega[e] += sum over the slice's partials, in a fixed order: each of
-// RSPLIT blocks sums a contiguous range of partials, then one pass adds the
-// RSPLIT sums in order.
-constexpr int RSPLIT = 16;
-__global__ void k_tc_reduce1(const float* part, float* sums, int nparts, int n) {
-  grid_dependency_wait();
-  const int e = blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= n) return;
-  const int per = (nparts + RSPLIT - 1) / RSPLIT;
-  const int i0 = blockIdx.y * per, i1 = min(nparts, i0 + per);
-  float s = 0.f;
-#pragma unroll 4
-  for (int i = i0; i < i1; ++i) s += part[(size_t)i * n + e];
-  sums[(size_t)blockIdx.y * n + e] = s;
-}
-__global__ void k_tc_reduce2(const float* sums, float* domega, int n) {
-  grid_dependency_wait();
-  const int e = blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= n) return;
-  float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < RSPLIT; ++i) s += sums[(size_t)i * n + e];
-  domega[e] += s;
-}
-
 // ================================================================== host
 namespace {
 
@@ -1008,11 +1110,15 @@ Geo geometry(const Problem& p) {
   return g;
 }
 
+// Every per-slice buffer has two slots (slice n uses slot n % 2), because
+// consecutive slices overlap in the pipelined launches.
 struct Ws {
   int* err;
   __nv_bfloat16* om16;
-  float *st_hi, *st_lo, *delta;
-  float *g_hi, *g_lo, *gdelta, *rowstat, *part, *rsums;
+  float *st_hi, *st_lo;
+  float* delta[2];
+  float *g_hi, *g_lo;
+  float *gdelta[2], *rowstat[2], *part[2], *rsums[2];
 };
 
 Ws carve(Carver& cv, const Geo& g, bool bwd) {
@@ -1022,19 +1128,21 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   w.om16 = cv.take<__nv_bfloat16>((size_t)2 * g.MF * D);
   w.st_hi = cv.take<float>(C * g.E);
   w.st_lo = cv.take<float>(C * g.E);
-  w.delta = cv.take<float>(C * g.nt * g.E);
+  for (int k = 0; k < 2; ++k) w.delta[k] = cv.take<float>(C * g.nt * g.E);
   if (bwd) {
     w.g_hi = cv.take<float>(C * g.E);
     w.g_lo = cv.take<float>(C * g.E);
-    w.gdelta = cv.take<float>(C * g.nt * g.E);
-    w.rowstat = cv.take<float>(C * g.nt * T * 2);
-    w.part = cv.take<float>(C * g.nt * (size_t)g.MF * D);
-    w.rsums = cv.take<float>((size_t)RSPLIT * g.MF * D);
+    for (int k = 0; k < 2; ++k) {
+      w.gdelta[k] = cv.take<float>(C * g.nt * g.E);
+      w.rowstat[k] = cv.take<float>(C * g.nt * T * 2);
+      w.part[k] = cv.take<float>(C * g.nt * (size_t)g.MF * D);
+      w.rsums[k] = cv.take<float>((size_t)RSPLIT * g.MF * D);
+    }
   }
   return w;
 }
 
-// dynamic shared memory of each kernel (plus 1 KB for 1024-byte alignment)
+// dynamic shared memory of each role (plus 1 KB for 1024-byte alignment)
 template <int MF>
 constexpr size_t smem_delta() { return 1024 + 2 * ROWT + Cfg<MF>::OMB + Cfg<MF>::FEATB + 4096; }
 template <int MF>
@@ -1043,21 +1151,19 @@ constexpr size_t smem_fwd() {
 }
 template <int MF>
 constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4; }
-
-template <typename F>
-cudaError_t set_smem(F* f, size_t bytes) {
-  return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+template <int MF>
+constexpr size_t smem_max() {
+  return smem_bwd<MF>() > smem_fwd<MF>() ? smem_bwd<MF>() : smem_fwd<MF>();
 }
 
 template <int MF, int FEAT>
 cudaError_t configure() {
   static bool done = false;
   if (done) return cudaSuccess;
-  cudaError_t e;
-  if ((e = set_smem(k_tc_delta<MF, FEAT>, smem_delta<MF>())) != cudaSuccess) return e;
-  if ((e = set_smem(k_tc_fwd<MF, FEAT>, smem_fwd<MF>())) != cudaSuccess) return e;
-  if ((e = set_smem(k_tc_bwd_q<MF, FEAT>, smem_bwd<MF>())) != cudaSuccess) return e;
-  if ((e = set_smem(k_tc_bwd_kv<MF, FEAT>, smem_bwd<MF>())) != cudaSuccess) return e;
+  cudaError_t e = cudaFuncSetAttribute(k_tc_tiles<MF, FEAT>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem_max<MF>());
+  if (e != cudaSuccess) return e;
   done = true;
   return cudaSuccess;
 }
@@ -1089,8 +1195,51 @@ cudaError_t launch_dep(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
-// Algorithmic work per tile launch, for the profiler.
-double tile_rows(const Geo& g, int b) { return (double)g.chains * b; }
+// Slice n: rows [a, a+b) and its tile count.
+struct Slice {
+  int a, b, nt;
+};
+Slice slice_of(const Problem& p, const Geo& g, int n) {
+  Slice r;
+  r.a = n * g.Cs;
+  r.b = (p.L - r.a < g.Cs) ? p.L - r.a : g.Cs;
+  r.nt = (r.b + T - 1) / T;
+  return r;
+}
+
+template <int MF, int FEAT>
+cudaError_t launch_tiles(cudaStream_t s, const TileJobs& J, double flops, double bytes,
+                         prof::Kid kid) {
+  const int n = J.n_kv + J.n_q + J.n_fwd + J.n_delta;
+  if (n == 0) return cudaSuccess;
+  size_t smem = 0;
+  if (J.n_kv || J.n_q) smem = smem_bwd<MF>();
+  if (J.n_fwd && smem_fwd<MF>() > smem) smem = smem_fwd<MF>();
+  if (J.n_delta && smem_delta<MF>() > smem) smem = smem_delta<MF>();
+  prof::Scope ps(kid, s, flops, bytes);
+  return launch_dep(k_tc_tiles<MF, FEAT>, dim3(n), dim3(NTHR), smem, s, J);
+}
+
+cudaError_t launch_small(cudaStream_t s, SmallJobs& J, prof::Kid kid) {
+  int blocks = J.r1_bx * RSPLIT + J.r2_blocks;
+  for (int i = 0; i < J.nscan; ++i) blocks += J.scan[i].blocks;
+  if (blocks == 0) return cudaSuccess;
+  prof::Scope ps(kid, s);
+  return launch_dep(k_tc_small, dim3(blocks), dim3(256), 0, s, J);
+}
+
+ScanJob scan_job(float* buf, float* hi, float* lo, int chains, int nt, int E, ScanMode mode) {
+  ScanJob j;
+  j.buf = buf;
+  j.hi = hi;
+  j.lo = lo;
+  j.chains = chains;
+  j.nt = nt;
+  j.E4 = E / 4;
+  j.mode = (int)mode;
+  j.blocks = (int)nblk((long long)chains * (E / 4));
+  return j;
+}
 
 template <int MF, int FEAT>
 slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat16* k,
@@ -1110,23 +1259,37 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
     TC_TRY(cudaGetLastError());
   }
   const double MD = (double)MF * D;
-  for (int n = 0; n < g.N; ++n) {
-    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    const int ntn = (b + T - 1) / T;
-    const double rows = tile_rows(g, b);
-    {
-      // algorithmic: phiK (2dM) + Delta (2dM) per row
-      prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
-      TC_TRY(launch_dep(k_tc_delta<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_delta<MF>(), s,
-                        k, v, w.om16, p.L, a, b, ntn, w.delta, w.err));
+  auto delta_job = [&](int n) {
+    const Slice sl = slice_of(p, g, n);
+    return DeltaJob{k, v, w.om16, p.L, sl.a, sl.b, sl.nt, w.delta[n & 1], w.err};
+  };
+  // Pipeline: the deltas of slice n+1 are computed in the launch that reads
+  // slice n's state prefixes.  Algorithmic work per row: delta 4dM (phiK,
+  // Delta), forward 4dM (phiQ, readout); phiK recomputation and the 128 x 128
+  // tile products are not counted.
+  for (int n = -1; n < g.N; ++n) {
+    TileJobs J{};
+    double rows = 0.0;
+    if (n >= 0) {
+      const Slice sl = slice_of(p, g, n);
+      J.f = FwdJob{q, k, v, w.om16, w.delta[n & 1], p.L, sl.a, sl.b, sl.nt, out, w.err};
+      J.n_fwd = sl.nt * g.chains;
+      rows += (double)g.chains * sl.b;
     }
-    TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_FWD, prof::K_TC_SCAN));
-    {
-      // algorithmic: phiQ (2dM) + readout phiQ S (2dM) per row; the phiK
-      // recomputation and the 128 x 128 tile products are not counted
-      prof::Scope ps(prof::K_TC_FWD, s, rows * 4.0 * MD, rows * D * 2.0 * 4);
-      TC_TRY(launch_dep(k_tc_fwd<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_fwd<MF>(), s, q,
-                        k, v, w.om16, w.delta, p.L, a, b, ntn, out, w.err));
+    if (n + 1 < g.N) {
+      const Slice sl = slice_of(p, g, n + 1);
+      J.d = delta_job(n + 1);
+      J.n_delta = sl.nt * g.chains;
+      rows += (double)g.chains * sl.b;
+    }
+    TC_TRY((launch_tiles<MF, FEAT>(s, J, rows * 4.0 * MD, rows * D * 2.0 * 3, prof::K_TC_FWD)));
+    if (n + 1 < g.N) {
+      SmallJobs S{};
+      S.scan[0] = scan_job(w.delta[(n + 1) & 1], w.st_hi, w.st_lo, g.chains,
+                           slice_of(p, g, n + 1).nt, g.E, SCAN_FWD);
+      S.nscan = 1;
+      S.n = MF * D;
+      TC_TRY(launch_small(s, S, prof::K_TC_SCAN));
     }
   }
   {
@@ -1148,53 +1311,86 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   Carver cv(workspace);
   const Ws w = carve(cv, g, true);
   const size_t SE = (size_t)g.chains * g.E;
+  const int N = g.N;
   TC_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
   TC_TRY(cudaMemsetAsync(domega, 0, (size_t)MF * D * sizeof(float), s));
   TC_TRY(cudaMemsetAsync(w.g_hi, 0, SE * sizeof(float), s));
   TC_TRY(cudaMemsetAsync(w.g_lo, 0, SE * sizeof(float), s));
   {
     prof::Scope ps(prof::K_TC_PREP, s);
-    k_omega_bf16<<<nblk(MF * D), 256, 0, s>>>(omega, w.om16, MF * D);  // hi and lo
+    k_omega_bf16<<<nblk(MF * D), 256, 0, s>>>(omega, w.om16, MF * D);
     TC_TRY(cudaGetLastError());
     k_tc_state_in<<<nblk((long long)SE), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains, MF);
     TC_TRY(cudaGetLastError());
   }
   const double MD = (double)MF * D;
-  for (int n = g.N - 1; n >= 0; --n) {
-    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    const int ntn = (b + T - 1) / T;
-    const double rows = tile_rows(g, b);
-    {
-      // algorithmic: phiK recomputation (2dM) + rollback Delta (2dM) per row
-      prof::Scope ps(prof::K_TC_DELTA, s, rows * 4.0 * MD, rows * D * 2.0 * 2);
-      TC_TRY(launch_dep(k_tc_delta<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_delta<MF>(), s,
-                        k, v, w.om16, p.L, a, b, ntn, w.delta, w.err));
+  const unsigned r_bx = nblk(MF * D);
+  auto valid = [&](int n) { return n >= 0 && n < N; };
+  // Stage j of the reverse walk (slices n = N-1 .. 0):
+  //   tiles j : dk/dv side of slice N-j, dq side of slice N-1-j, deltas of slice N-2-j
+  //   small j : rollback scan of slice N-2-j, state-gradient scan of slice N-1-j,
+  //             dOmega reduction stage 1 of slice N-j and stage 2 of slice N+1-j
+  // Algorithmic work per row: delta 4dM (phiK, rollback Delta), dq side 10dM,
+  // dk/dv side 8dM.
+  for (int j = -1; j <= N + 1; ++j) {
+    if (j >= 0) {
+      TileJobs J{};
+      double fl = 0.0, by = 0.0;
+      const int nkv = N - j, nq = N - 1 - j, nd = N - 2 - j;
+      if (j >= 1 && valid(nkv)) {
+        const Slice sl = slice_of(p, g, nkv);
+        J.kv = BwdKVJob{q, k, v, dout, w.om16, w.gdelta[nkv & 1], w.rowstat[nkv & 1], p.L, sl.a,
+                        sl.b, sl.nt, dk, dv, w.part[nkv & 1], w.err};
+        J.n_kv = sl.nt * g.chains;
+        fl += (double)g.chains * sl.b * 8.0 * MD;
+        by += (double)g.chains * sl.b * D * 2.0 * 6;
+      }
+      if (valid(nq)) {
+        const Slice sl = slice_of(p, g, nq);
+        J.q = BwdQJob{q, k, v, out, dout, w.om16, w.delta[nq & 1], p.L, sl.a, sl.b, sl.nt, dq,
+                      w.gdelta[nq & 1], w.rowstat[nq & 1], w.part[nq & 1], w.err};
+        J.n_q = sl.nt * g.chains;
+        fl += (double)g.chains * sl.b * 10.0 * MD;
+        by += (double)g.chains * sl.b * D * 2.0 * 6;
+      }
+      if (valid(nd)) {
+        const Slice sl = slice_of(p, g, nd);
+        J.d = DeltaJob{k, v, w.om16, p.L, sl.a, sl.b, sl.nt, w.delta[nd & 1], w.err};
+        J.n_delta = sl.nt * g.chains;
+        fl += (double)g.chains * sl.b * 4.0 * MD;
+        by += (double)g.chains * sl.b * D * 2.0 * 2;
+      }
+      TC_TRY((launch_tiles<MF, FEAT>(s, J, fl, by, prof::K_TC_BWD)));
+    } else {
+      // prologue: deltas of the last slice
+      const Slice sl = slice_of(p, g, N - 1);
+      TileJobs J{};
+      J.d = DeltaJob{k, v, w.om16, p.L, sl.a, sl.b, sl.nt, w.delta[(N - 1) & 1], w.err};
+      J.n_delta = sl.nt * g.chains;
+      TC_TRY((launch_tiles<MF, FEAT>(s, J, (double)g.chains * sl.b * 4.0 * MD,
+                                     (double)g.chains * sl.b * D * 2.0 * 2, prof::K_TC_BWD)));
     }
-    TC_TRY(launch_scan(s, w.delta, w.st_hi, w.st_lo, g.chains, ntn, g.E, SCAN_ROLLBACK, prof::K_TC_SCAN));
-    {
-      // algorithmic: phiQ recomputation, dnum S^T, G_S update, dq VJP, dOmega_q
-      // (2dM each) per row
-      prof::Scope ps(prof::K_TC_BWD_Q, s, rows * 10.0 * MD, rows * D * 2.0 * 6);
-      TC_TRY(launch_dep(k_tc_bwd_q<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_bwd<MF>(), s,
-                        q, k, v, out, dout, w.om16, w.delta, p.L, a, b, ntn, dq, w.gdelta,
-                        w.rowstat, w.part, w.err));
+    SmallJobs S{};
+    S.n = MF * D;
+    const int nr = N - 2 - j, ng = N - 1 - j, nx1 = N - j, nx2 = N + 1 - j;
+    if (valid(nr))
+      S.scan[S.nscan++] = scan_job(w.delta[nr & 1], w.st_hi, w.st_lo, g.chains,
+                                   slice_of(p, g, nr).nt, g.E, SCAN_ROLLBACK);
+    if (j >= 0 && valid(ng))
+      S.scan[S.nscan++] = scan_job(w.gdelta[ng & 1], w.g_hi, w.g_lo, g.chains,
+                                   slice_of(p, g, ng).nt, g.E, SCAN_GREV);
+    if (j >= 1 && valid(nx1)) {
+      S.r1_part = w.part[nx1 & 1];
+      S.r1_sums = w.rsums[nx1 & 1];
+      S.r1_nparts = g.chains * slice_of(p, g, nx1).nt;
+      S.r1_bx = (int)r_bx;
     }
-    TC_TRY(launch_scan(s, w.gdelta, w.g_hi, w.g_lo, g.chains, ntn, g.E, SCAN_GREV, prof::K_TC_SCAN));
-    {
-      // algorithmic: dV state part, dphiK state part, dk VJP, dOmega_k (2dM
-      // each) per row
-      prof::Scope ps(prof::K_TC_BWD_KV, s, rows * 8.0 * MD, rows * D * 2.0 * 6);
-      TC_TRY(launch_dep(k_tc_bwd_kv<MF, FEAT>, dim3(ntn, g.chains), dim3(NTHR), smem_bwd<MF>(), s,
-                        q, k, v, dout, w.om16, w.gdelta, w.rowstat, p.L, a, b, ntn, dk, dv, w.part,
-                        w.err));
+    if (j >= 2 && valid(nx2)) {
+      S.r2_sums = w.rsums[nx2 & 1];
+      S.r2_domega = domega;
+      S.r2_blocks = (int)r_bx;
     }
-    {
-      prof::Scope ps(prof::K_TC_REDUCE, s);
-      TC_TRY(launch_dep(k_tc_reduce1, dim3(nblk(MF * D), RSPLIT), dim3(256), 0, s,
-                        (const float*)w.part, w.rsums, g.chains * ntn, MF * D));
-      TC_TRY(launch_dep(k_tc_reduce2, dim3(nblk(MF * D)), dim3(256), 0, s, (const float*)w.rsums,
-                        domega, MF * D));
-    }
+    TC_TRY(launch_small(s, S, prof::K_TC_SCAN));
   }
   return SLIM_OK;
 }
