@@ -315,13 +315,13 @@ __device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, co
   load_rows64(sV, T, V + g0, valid, tid, NTHR);
   grid_dependency_wait();  // the state prefixes come from the scan just before
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
+  load_rows64(sPhiK, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
   for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
     const bool rv = row < valid;
-    float* redN = reinterpret_cast<float*>(sPhiK);  // phiK is written only after phase 1
+    float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
     redN[cg * T + row] = row_norm2_part(sQ, row, cg);
     redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
     publish();
@@ -330,20 +330,25 @@ __device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, co
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
+      // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
-      const uint32_t aOl = smem_u32(sPhiQ);
+      const uint32_t aOl = smem_u32(sPhiK);
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+      for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
       mma_commit(sy.mbar);
     }
-    TC_WAIT(sy);
-    load_f32_rows64<MF>(sS, P, tid);  // Omega no longer needed: S_t takes its place
-    float* redZ = reinterpret_cast<float*>(sQ);  // Q, K are dead; A is written after the next wait
+    TC_WAIT(sy);  // Q projection done
+    float* redZ = reinterpret_cast<float*>(sQ);  // Q is dead; A is written after the next waits
     redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
+    TC_WAIT(sy);  // K projection done: Omega is no longer needed, S_t takes its place
+    load_f32_rows64<MF>(sS, P, tid);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
@@ -445,13 +450,13 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
   }
   grid_dependency_wait();  // the state prefixes come from the scan just before
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
+  load_rows64(sPhiK, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
   for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
     const bool rv = row < valid;
-    float* redN = reinterpret_cast<float*>(sPhiK);  // phiK is written only after phase 1
+    float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
     {
       float part = 0.f;  // <dout_r, out_r> over this thread's 16 columns
 #pragma unroll
@@ -478,20 +483,25 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
+      // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
-      const uint32_t aOl = smem_u32(sPhiQ);
+      const uint32_t aOl = smem_u32(sPhiK);
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+      for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
       mma_commit(sy.mbar);
     }
-    TC_WAIT(sy);
-    load_f32_rows64<MF>(sS, P, tid);
-    float* redZ = reinterpret_cast<float*>(sQ);  // Q, K are dead; dA is written after the next wait
+    TC_WAIT(sy);  // Q projection done
+    float* redZ = reinterpret_cast<float*>(sQ);  // Q is dead; dA is written after the next waits
     redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
+    TC_WAIT(sy);  // K projection done: S_t replaces Omega
+    load_f32_rows64<MF>(sS, P, tid);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
@@ -713,7 +723,7 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
   load_rows64(sDn, T, dOut + g0, valid, tid, NTHR);
   grid_dependency_wait();  // G suffixes (scan) and row statistics (tc_bwd_q) are earlier kernels'
   load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhiQ, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiQ overwrites it
+  load_rows64(sPhiK, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
   for (int m = tid; m < MF; m += NTHR) sGz[m] = G[MF * 64 + m];
   float den = 0.f, dden = 0.f;
   if (row < valid) {
@@ -728,7 +738,7 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     if (!live) dden = 0.f;
-    float* redN = reinterpret_cast<float*>(sPhiK);  // phiK is written only after phase 1
+    float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
     redN[cg * T + row] = row_norm2_part(sQ, row, cg);
     redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
 #pragma unroll
@@ -750,19 +760,24 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{smem_u32(&mbar), 0u, err};
     if (tid == 0) {
+      // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
-      const uint32_t aOl = smem_u32(sPhiQ);
+      const uint32_t aOl = smem_u32(sPhiK);
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(sy.mbar);
+      for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
       mma_commit(sy.mbar);
     }
-    TC_WAIT(sy);
-    load_f32_rows64<MF>(sG, G, tid);  // G_t(S) replaces Omega
+    TC_WAIT(sy);  // Q projection done
     feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    TC_WAIT(sy);  // K projection done: G_t(S) replaces Omega
+    load_f32_rows64<MF>(sG, G, tid);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
