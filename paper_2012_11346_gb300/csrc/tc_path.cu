@@ -1,35 +1,36 @@
 // Tensor-core (tcgen05) path of libslim: bf16 inputs, d = 64, M in {128, 256}.
 //
-// Same slice algorithm as the fp32 path (Algorithm 1, App. B block form with
-// masked tile products), with tiles of T = 128 rows, one CTA of 128 threads
+// Same slice algorithm as the fp32 path (Algorithm 1; App. B block form with
+// masked tile products), on tiles of T = 128 rows with one CTA of 512 threads
 // per (tile, chain).  Every tile product is a chain of tcgen05 MMAs on
 // 128-byte-swizzled bf16 shared-memory operands with an fp32 accumulator in
-// tensor memory; thread r of the CTA owns row r (TMEM lane r) in the
-// epilogues.  Per slice:
+// tensor memory.  In the row-wise epilogues warp w serves TMEM lanes
+// 32(w%4)..32(w%4)+31 and column group w/4 of each row.
 //
-//   forward   tc_delta : phiK = g(K_t), Delta_t = phiK^T [V_t | 1]
-//             scan     : P_t = B + sum_{t'<t} Delta_t', B += sum Delta_t
-//             tc_fwd   : phiQ, phiK, A = tril(phiQ phiK^T),
-//                        num = phiQ S_t + A V_t, den = phiQ z_t + rowsum A
-//   backward  tc_delta, scan(rollback, eq. 17)
-//             tc_bwd_q : den, dnum = dout/den, dden = -<dout,out>/den,
-//                        dA = tril(dnum V^T + dden), dphiQ = dnum S_t^T +
-//                        dden z_t + dA phiK, Gd_t = phiQ^T [dnum | dden],
-//                        dq = u Omega - q sum(u), dOmega partial u^T q
-//             scan     : G_t = G + sum_{t'>t} Gd_t' (eq. 18)
-//             tc_bwd_kv: dV = A^T dnum + phiK G_t(S), dphiK = dA^T phiQ +
-//                        V G_t(S)^T + g_t(z), dk = u Omega - k sum(u),
-//                        dOmega partial += u^T k
-//             reduce   : dOmega += sum of partials (fixed order)
+// State prefixes are chained from tile to tile.  The CTA of a tile computes
+// its own delta Delta_t = phiK^T [V_t | 1], waits (bounded) for the prefix its
+// neighbour tile left in a workspace slot, and leaves its own there for the
+// next tile: inside a slice this is the prefix sum of eqs. 14-15, across a
+// slice boundary it is the slice carry B^(n) (eq. 16).
 //
-// The state rows of the workspace hold [S (M x 64) | z (M)] per tile (E =
-// 65 M floats), exactly what the shared scan carries.
+//   forward, one launch, tiles in sequence order:
+//     phiQ, phiK, Delta_t, A = tril(phiQ phiK^T);  S_t, z_t = prefix before
+//     tile t;  num = phiQ S_t + A V_t,  den = phiQ z_t + rowsum A,  out = num/den
+//   backward, slices in reverse (Algorithm 1's reverse sweep), one launch each:
+//     dq side of slice n, tiles in reverse order: phiQ, phiK, Delta_t, A;
+//       rollback P_t = P_{t+1} - Delta_t (eq. 17);  den, dnum = dout/den,
+//       dden = -<dout,out>/den, dA = tril(dnum V^T + dden);
+//       dphiQ = dnum S_t^T + dden z_t + dA phiK,  Gd_t = phiQ^T [dnum | dden];
+//       state-gradient chain G_t = G_{t+1} + Gd_{t+1} (eq. 18);
+//       dq = u Omega - q sum(u),  dOmega partial u^T q
+//     dk/dv side of slice n (in the launch of the dq side of slice n-1):
+//       dV = A^T dnum + phiK G_t(S),  dphiK = dA^T phiQ + V G_t(S)^T + g_t(z),
+//       dk = u Omega - k sum(u),  dOmega partial += u^T k
+//     reduce: dOmega += the partials, in a fixed order
 #include <math.h>
 
 #include "common.cuh"
 #include "profiler.h"
-#include "scan.h"
-#include "scan_dev.cuh"
 #include "tc_common.cuh"
 #include "tc_path.h"
 
@@ -56,28 +57,6 @@ struct Cfg {
 constexpr int NG = 4;
 constexpr int NTHR = 128 * NG;
 
-// fp32 [R][64] global -> bf16 row tile (R rows), all NTHR threads.  Every
-// thread issues all of its loads before converting, so they are in flight
-// together.
-template <int R>
-__device__ __forceinline__ void load_f32_rows64(uint8_t* tile, const float* g, int tid) {
-  constexpr int PER = R * 8 / NTHR;  // 16-byte bf16 chunks per thread
-  static_assert(R * 8 % NTHR == 0, "rows must split evenly over the CTA");
-  float4 a[PER], b[PER];
-#pragma unroll
-  for (int i = 0; i < PER; ++i) {
-    const int e = tid + i * NTHR, r = e >> 3, c = (e & 7) * 8;
-    a[i] = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c);
-    b[i] = *reinterpret_cast<const float4*>(g + (size_t)r * 64 + c + 4);
-  }
-#pragma unroll
-  for (int i = 0; i < PER; ++i) {
-    const int e = tid + i * NTHR, r = e >> 3, c = (e & 7) * 8;
-    st_chunk(tile, R, r, c, make_uint4(pack_bf16(a[i].x, a[i].y), pack_bf16(a[i].z, a[i].w),
-                                       pack_bf16(b[i].x, b[i].y), pack_bf16(b[i].z, b[i].w)));
-  }
-}
-
 // Loads 16 bf16 of a feature-tile row (columns c..c+15) as floats.
 __device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, float* f) {
 #pragma unroll
@@ -92,11 +71,9 @@ __device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, flo
 // Reads this thread's column group of the projection P = X Omega^T from TMEM,
 // applies the feature map, stores phi (bf16) into the [128][MF] feature tile.
 template <int MF, int FEAT>
-__device__ __forceinline__ float feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
-                                                  float x2, bool valid,
-                                                  const float* z = nullptr) {
+__device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
+                                                 float x2, bool valid) {
   constexpr int W = MF / NG;
-  float dz = 0.f;  // sum over this thread's columns of bf16(phi) * z
   // exp map: phi = 2^(p log2e - (|x|^2/2) log2e - log2 sqrt(M))
   const float bias = -0.5f * x2 * kLog2e - 0.5f * log2f((float)MF);
   const float relu_scale = rsqrtf((float)MF);
@@ -117,17 +94,11 @@ __device__ __forceinline__ float feature_epilogue(uint32_t trow, uint8_t* phi, i
       }
       if (!valid) a = b = 0.f;
       pk[i / 2] = pack_bf16(a, b);
-      if (z) {
-        float ra, rb;
-        unpack_bf16(pk[i / 2], ra, rb);
-        dz = fmaf(ra, z[c0 + i], fmaf(rb, z[c0 + i + 1], dz));
-      }
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q)
       st_chunk(phi, T, r, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
   }
-  return dz;
 }
 
 // Squared norm of columns 16cg..16cg+15 of row r of a [128][64] row tile.
@@ -210,89 +181,157 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 
 #define TC_TEARDOWN()                                   \
   teardown:                                             \
+  cp_async_wait_all();                                  \
   tc_fence_before();                                    \
   __syncthreads();                                      \
   if (warp == 0) tmem_dealloc(tmem_base, 512)
 
-// ================================================================== tc_delta
-template <int MF, int FEAT>
-__device__ __forceinline__ void role_delta(const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
-               const __nv_bfloat16* __restrict__ om16, int L, int a, int b, int nt,
-               float* __restrict__ delta, int* err,
-    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
-  using C = Cfg<MF>;
-  uint8_t* base = align1024(smem_raw);
-  uint8_t* sK = base;
-  uint8_t* sV = sK + ROWT;
-  uint8_t* sOm = sV + ROWT;
-  uint8_t* sPhi = sOm + C::OMB;
-  uint8_t* sOnes = sPhi + C::FEATB;  // [16][128] K-major, all ones
-  const int row0 = a + t * T;
-  const int valid = min(T, b - t * T);
-  const size_t g0 = ((size_t)c * L + row0) * D;
-  TC_PROLOGUE();
-  load_rows64(sK, T, K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, V + g0, valid, tid, NTHR);
-  grid_dependency_wait();  // Omega (bf16) and the delta buffer belong to earlier kernels
-  load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhi, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phi overwrites it
-  cp_async_wait_all();
-  __syncthreads();  // rows were copied by other threads
-  {
-    float* redN = reinterpret_cast<float*>(sOnes);  // scratch until the ones are written
-    redN[cg * T + row] = row_norm2_part(sK, row, cg);
-    publish();
-    const float x2 = group_total(redN, row);
-    const uint32_t tmem = tmem_base;
-    const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, err};
-    if (tid == 0) {
-      const uint32_t aK = smem_u32(sK), aOm = smem_u32(sOm), aOl = smem_u32(sPhi);
-      for (int k0 = 0; k0 < D; k0 += 16) {
-        mma(tmem, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-        mma(tmem, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
-      }
-      mma_commit(sy.mbar);
-    }
-    TC_WAIT(sy);
-    for (int e = tid; e < 4096 / 16; e += NTHR)
-      reinterpret_cast<uint4*>(sOnes)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
-    feature_epilogue<MF, FEAT>(trow, sPhi, row, cg, x2, row < valid);
-    publish();
-    if (tid == 0) {
-      const uint32_t aPhi = smem_u32(sPhi), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
-      for (int h = 0; h < C::MH; ++h)
-        for (int k0 = 0; k0 < T; k0 += 16) {
-          const uint64_t ad = mnmaj(aPhi + h * 2 * ROWT, k0, ROWT);
-          mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
-          mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
-        }
-      mma_commit(sy.mbar);
-    }
-    TC_WAIT(sy);
-    float* dst = delta + ((size_t)c * nt + t) * C::E;
-    for (int h = 0; h < C::MH; ++h) {
-      const int m = 128 * h + row;
-      float v[16];
-      tmem_ld16(trow + 256 + 64 * h + 16 * cg, v);
-      st_f32x16(dst + (size_t)m * 64 + 16 * cg, v);
-      if (cg == 0) {
-        float zz;
-        tmem_ld1(trow + 384 + 16 * h, zz);
-        dst[MF * 64 + m] = zz;
-      }
-    }
-  }
-  TC_TEARDOWN();
+// ------------------------------------------------------------------ chained tile prefixes
+// A slot holds one state (or state-gradient) prefix, [S (M x 64) | z (M)] in
+// fp32; its flag holds n + 1 once slice n's prefix is in the slot.  The CTA
+// that waits on a slot always has a higher block index than the CTA that
+// fills it, so the filling CTA was dispatched first and is running or done.
+__device__ __forceinline__ int ld_relaxed_gpu(const int* p) {
+  int v;
+  asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void fence_acq_rel_gpu() {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+__device__ __forceinline__ void st_release_gpu(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
-// ================================================================== tc_fwd
+// Flags sit 128 bytes apart, so the CTAs polling different flags do not
+// share a cache line.
+constexpr int FLAG_STRIDE = 32;
+
+// Thread 0 waits for *flag == want; every thread learns the outcome.  The
+// wait is bounded (2^22 polls, ~1 s with the back-off) and stops early once
+// another CTA has reported an error (checked every 64 polls, so that the
+// waiting CTAs do not all hammer the error word); a failed wait records
+// itself in *err.
+__device__ __forceinline__ bool chain_acquire(const int* flag, int want, int* err, int& abort_) {
+  if (threadIdx.x == 0) {
+    bool ok = false;
+    for (uint32_t i = 0; i < (1u << 22); ++i) {
+      if (ld_relaxed_gpu(flag) == want) {
+        fence_acq_rel_gpu();
+        ok = true;
+        break;
+      }
+      if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) break;
+      __nanosleep(i < 16 ? 32 : 256);
+    }
+    if (!ok) {
+      atomicExch(err, 1);
+      abort_ = 1;
+    }
+  }
+  __syncthreads();
+  return abort_ == 0;
+}
+
+// Publishes the slot under its flag.  The barrier orders every thread's slot
+// writes before thread 0's release store, which (being cumulative) makes them
+// visible at GPU scope before the flag.
+__device__ __forceinline__ void chain_release(int* flag, int val) {
+  __syncthreads();
+  if (threadIdx.x == 0) st_release_gpu(flag, val);
+}
+
+// Buffers exchanged between tile CTAs (prefix slots, dOmega partials, G_t)
+// are "lane-major": the 16 values a thread owns in an epilogue (row m = 128h +
+// row, columns 16cg..16cg+15 of an [M][64] matrix) are spread over four float4
+// at  q = ((h NG + cg) 4 + i) 128 + row,  so a warp's 32 rows are 512
+// contiguous bytes and every warp access is coalesced.
+__device__ __forceinline__ size_t lm4(int h, int cg, int i, int row) {
+  return (size_t)((h * NG + cg) * 4 + i) * 128 + row;
+}
+// 16 floats through L2 (the data is written by other CTAs of the same
+// kernel, so L1 must not serve stale lines).
+__device__ __forceinline__ void ld_lm16(const float* base, int h, int cg, int row, float* v) {
+  const float4* s = reinterpret_cast<const float4*>(base);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 x = __ldcg(s + lm4(h, cg, i, row));
+    v[4 * i] = x.x;
+    v[4 * i + 1] = x.y;
+    v[4 * i + 2] = x.z;
+    v[4 * i + 3] = x.w;
+  }
+}
+__device__ __forceinline__ void st_lm16(float* base, int h, int cg, int row, const float* v) {
+  float4* d = reinterpret_cast<float4*>(base);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    __stcg(d + lm4(h, cg, i, row), make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+}
+// Row-major [M][64] (the caller's state tensors): 16 floats at p.
+__device__ __forceinline__ void ld_row16f(const float* p, float* v) {
+  const float4* s = reinterpret_cast<const float4*>(p);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 x = __ldcg(s + i);
+    v[4 * i] = x.x;
+    v[4 * i + 1] = x.y;
+    v[4 * i + 2] = x.z;
+    v[4 * i + 3] = x.w;
+  }
+}
+// bf16 lane-major: 16-byte chunk k = ((h NG + cg) 2 + half) 128 + row holds
+// row 128h + row, columns 16cg + 8 half .. +7.
+__device__ __forceinline__ void st_lm16_bf16(__nv_bfloat16* base, int h, int cg, int row, const float* v) {
+  uint4* d = reinterpret_cast<uint4*>(base);
+#pragma unroll
+  for (int hf = 0; hf < 2; ++hf)
+    d[(size_t)((h * NG + cg) * 2 + hf) * 128 + row] =
+        make_uint4(pack_bf16(v[8 * hf], v[8 * hf + 1]), pack_bf16(v[8 * hf + 2], v[8 * hf + 3]),
+                   pack_bf16(v[8 * hf + 4], v[8 * hf + 5]), pack_bf16(v[8 * hf + 6], v[8 * hf + 7]));
+}
+// Copies an [MF][64] bf16 lane-major matrix into an [MF][64] row tile
+// (cp.async, coalesced reads; completes with cp_async_wait_all()).
+__device__ __forceinline__ void load_lm_bf16(uint8_t* tile, int MF, const __nv_bfloat16* g, int tid) {
+  const uint32_t base = smem_u32(tile);
+  for (int k = tid; k < MF * 8; k += NTHR) {
+    const int row = k & 127, rest = k >> 7, hf = rest & 1, cg = (rest >> 1) % NG, h = rest / (2 * NG);
+    cp_async16(base + tile_off(MF, 128 * h + row, 16 * cg + 8 * hf), g + (size_t)k * 8, 16u);
+  }
+}
+// 16 floats as bf16 into columns c..c+15 of row r of a [R][64] row tile.
+__device__ __forceinline__ void st_tile16(uint8_t* tile, int R, int r, int c, const float* v) {
+  st_chunk(tile, R, r, c, make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]),
+                                     pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7])));
+  st_chunk(tile, R, r, c + 8, make_uint4(pack_bf16(v[8], v[9]), pack_bf16(v[10], v[11]),
+                                         pack_bf16(v[12], v[13]), pack_bf16(v[14], v[15])));
+}
+
+// One side of a chain link: where a prefix lives.  S rows are 64 floats
+// apart; lo (optional) adds a low-order residual to every value.
+struct StateRef {
+  const float *S, *z, *S_lo, *z_lo;
+};
+
+__device__ __forceinline__ void fill_ones(uint8_t* tile, int tid) {
+  for (int e = tid; e < 4096 / 16; e += NTHR)
+    reinterpret_cast<uint4*>(tile)[e] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+}
+
+// ================================================================== forward
+struct FwdJob {
+  const __nv_bfloat16 *Q, *K, *V, *om16;
+  int L, Cs, N, nt, P, chains;  // slice length, slices, tiles of a full slice, tile positions
+  float* slot;                  // [chains][nt][E] inclusive prefixes
+  int* flag;                    // [chains][nt], FLAG_STRIDE ints apart
+  __nv_bfloat16* out;
+  StateOut st;                  // B^(N), written by the last tile of each chain
+  int* err;
+};
+
 template <int MF, int FEAT>
-__device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
-             const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ om16,
-             const float* __restrict__ pfx, int L, int a, int b, int nt,
-             __nv_bfloat16* __restrict__ out, int* err,
-    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
+__device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_t* smem_raw,
+                                         uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;
@@ -303,20 +342,31 @@ __device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, co
   uint8_t* sOm = sK + ROWT;        // later: S_t (bf16)
   uint8_t* sS = sOm;
   uint8_t* sV = sOm + C::OMB;
-  float* sZ = reinterpret_cast<float*>(sV + ROWT);
-  float* red = sZ + MF;            // [NG][128] row-sum partials
+  uint8_t* sOnes = sV + ROWT;      // [16][128] K-major, all ones
+  float* sZ = reinterpret_cast<float*>(sOnes + 4096);
+  float* red = sZ + MF;            // [NG][128] row partials of den
+  // tile t of slice n
+  const int n = min(pos / J.nt, J.N - 1), t = pos - n * J.nt;
+  const int a = n * J.Cs, slen = min(J.Cs, J.L - a);
   const int row0 = a + t * T;
-  const int valid = min(T, b - t * T);
-  const size_t g0 = ((size_t)c * L + row0) * D;
-  const float* P = pfx + ((size_t)c * nt + t) * C::E;
+  const int valid = min(T, slen - t * T);
+  const size_t g0 = ((size_t)c * J.L + row0) * D;
+  // the tile before in sequence order (none for the first) and this tile's slot
+  const int tp = t > 0 ? t - 1 : J.nt - 1;
+  const float* pred = pos > 0 ? J.slot + ((size_t)c * J.nt + tp) * C::E : nullptr;
+  const int* pflag = J.flag + ((size_t)c * J.nt + tp) * FLAG_STRIDE;
+  const int pwant = (t > 0 ? n : n - 1) + 1;
+  float* own = J.slot + ((size_t)c * J.nt + t) * C::E;
+  int* oflag = J.flag + ((size_t)c * J.nt + t) * FLAG_STRIDE;
+  const bool last = pos == J.P - 1;
   TC_PROLOGUE();
-  load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
-  load_rows64(sK, T, K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, V + g0, valid, tid, NTHR);
-  grid_dependency_wait();  // the state prefixes come from the scan just before
-  load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhiK, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
-  for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
+  load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
+  load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
+  fill_ones(sOnes, tid);
+  grid_dependency_wait();  // Omega (bf16) and the slots belong to earlier kernels
+  load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
+  load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
@@ -328,7 +378,7 @@ __device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, co
     const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, err};
+    Sync sy{smem_u32(&mbar), 0u, J.err};
     if (tid == 0) {
       // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -345,29 +395,31 @@ __device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, co
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);  // Q projection done
-    float* redZ = reinterpret_cast<float*>(sQ);  // Q is dead; A is written after the next waits
-    redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
-    TC_WAIT(sy);  // K projection done: Omega is no longer needed, S_t takes its place
-    load_f32_rows64<MF>(sS, P, tid);
+    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    TC_WAIT(sy);  // K projection done: Omega is dead, phiK takes Omega lo's place
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
-      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK), aS = smem_u32(sS);
-      for (int k0 = 0; k0 < MF; k0 += 16) {
+      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
+      const uint32_t aV = smem_u32(sV), aOnes = smem_u32(sOnes);
+      for (int h = 0; h < C::MH; ++h)  // Delta_t = phiK^T [V | 1]
+        for (int k0 = 0; k0 < T; k0 += 16) {
+          const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
+          mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+          mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
+        }
+      for (int k0 = 0; k0 < MF; k0 += 16)  // A = phiQ phiK^T
         mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
-        mma(tmem + 128, kmaj(aPQ, T, k0), mnmaj(aS, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
-      }
       mma_commit(sy.mbar);
     }
-    const float dz = group_total(redZ, row);  // phiQ z_t
     TC_WAIT(sy);
+    float rs = 0.f;  // sum of this thread's rounded, masked A values
     {
-      // A: inclusive causal mask, bf16; row sum of the rounded values
+      // A: inclusive causal mask, bf16 (independent of the chain: done first)
       float v[32];
       const int c0 = 32 * cg;
       tmem_ld32(trow + c0, v);
       uint32_t pk[16];
-      float rs = 0.f;
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
         const float x0 = (c0 + i <= row) ? v[i] : 0.f;
@@ -380,78 +432,176 @@ __device__ __forceinline__ void role_fwd(const __nv_bfloat16* __restrict__ Q, co
 #pragma unroll
       for (int q = 0; q < 4; ++q)
         st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
-      red[cg * T + row] = rs;
+    }
+    // ---- chain: S_t, z_t = the predecessor's inclusive prefix (zero for the
+    // first tile); this tile's inclusive prefix S_t + Delta_t goes to its slot.
+    {
+      if (pred && !chain_acquire(pflag, pwant, J.err, abort_)) goto teardown;
+      // every load of the predecessor's prefix before any store: one L2 trip
+      float pv[C::MH][16], pz[C::MH];
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + row;
+        if (pred) {
+          ld_lm16(pred, h, cg, row, pv[h]);
+          pz[h] = cg == 0 ? __ldcg(pred + MF * 64 + m) : 0.f;
+        } else {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) pv[h][i] = 0.f;
+          pz[h] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + row;
+        float inc[16];
+        tmem_ld16(trow + 256 + 64 * h + 16 * cg, inc);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) inc[i] += pv[h][i];
+        st_lm16(own, h, cg, row, inc);
+        st_tile16(sS, MF, m, 16 * cg, pv[h]);
+        if (last) {
+          st_f32x16(J.st.S + ((size_t)c * MF + m) * 64 + 16 * cg, inc);
+          if (J.st.S_lo) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) inc[i] = 0.f;
+            st_f32x16(J.st.S_lo + ((size_t)c * MF + m) * 64 + 16 * cg, inc);
+          }
+        }
+      }
+      if (cg == 0) {
+#pragma unroll
+        for (int h = 0; h < C::MH; ++h) {
+          const int m = 128 * h + row;
+          float dz;
+          tmem_ld1(trow + 384 + 16 * h, dz);
+          __stcg(own + MF * 64 + m, pz[h] + dz);
+          sZ[m] = pz[h];
+          if (last) {
+            J.st.z[(size_t)c * MF + m] = pz[h] + dz;
+            if (J.st.z_lo) J.st.z_lo[(size_t)c * MF + m] = 0.f;
+          }
+        }
+      }
+      chain_release(oflag, n + 1);
+    }
+    {
+      // the row's den partial: rs plus phiQ . z_t over this thread's features
+      constexpr int W = MF / NG;
+      float zd = 0.f;
+#pragma unroll
+      for (int f0 = cg * W; f0 < (cg + 1) * W; f0 += 16) {
+        float f[16];
+        ld_feat16(sPhiQ, row, f0, f);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) zd = fmaf(f[i], sZ[f0 + i], zd);
+      }
+      red[cg * T + row] = rs + zd;
     }
     publish();
     if (tid == 0) {
+      const uint32_t aPQ = smem_u32(sPhiQ), aS = smem_u32(sS);
       const uint32_t aA = smem_u32(sA), aV = smem_u32(sV);
-      for (int k0 = 0; k0 < T; k0 += 16)
+      for (int k0 = 0; k0 < MF; k0 += 16)  // num = phiQ S_t
+        mma(tmem + 128, kmaj(aPQ, T, k0), mnmaj(aS, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+      for (int k0 = 0; k0 < T; k0 += 16)  // + A V
         mma(tmem + 128, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), 1);
       mma_commit(sy.mbar);
     }
-    float rs = 0.f;
-#pragma unroll
-    for (int g = 0; g < NG; ++g) rs += red[g * T + row];
+    const float den = group_total(red, row);
     TC_WAIT(sy);
     {
-      const float den = rs + dz;
       const float inv = den != 0.f ? 1.f / den : 0.f;
       float v[16];
       tmem_ld16(trow + 128 + 16 * cg, v);  // every lane loads (warp-aligned op)
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] *= inv;
-      if (rv) st_row16(out + g0 + (size_t)row * D + 16 * cg, v);
+      if (rv) st_row16(J.out + g0 + (size_t)row * D + 16 * cg, v);
     }
   }
   TC_TEARDOWN();
 }
 
-// ================================================================== tc_bwd_q
+// ================================================================== backward, dq side
+struct BwdQJob {
+  const __nv_bfloat16 *Q, *K, *V, *Out, *dOut, *om16;
+  StateIn fin;            // B^(N), the state the forward returned
+  int L, a, b, ntn, n, N, nt, chains;  // slice n = rows [a, a+b), ntn tiles; nt: full slice
+  float *slot1, *slot2;   // [chains][nt][E]: state prefixes, state-gradient prefixes
+  int *flag1, *flag2;     // [chains][nt], FLAG_STRIDE ints apart
+  __nv_bfloat16* gS;      // [chains][ntn][MF][64] G_t(S) for the dk/dv side
+  float* gz;              // [chains][ntn][MF]     g_t(z)
+  float *rowstat, *part;  // [chains][ntn][T][2] (den, dden), [chains][ntn][MF][64]
+  __nv_bfloat16* dq;
+  int* err;
+};
+
 template <int MF, int FEAT>
-__device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
-               const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ Out,
-               const __nv_bfloat16* __restrict__ dOut, const __nv_bfloat16* __restrict__ om16,
-               const float* __restrict__ pfx, int L, int a, int b, int nt,
-               __nv_bfloat16* __restrict__ dq, float* __restrict__ gdelta,
-               float* __restrict__ rowstat, float* __restrict__ part, int* err,
-    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
+__device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* smem_raw,
+                                           uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;
   uint8_t* sPhiK = sPhiQ + C::FEATB;  // later: u
   uint8_t* sU = sPhiK;
-  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [dA (2 tiles) | S_t] -> [Q | red | Omega]
+  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [ones | . | S_t] -> [dA | S_t] -> [Q | red | Omega]
   uint8_t* sQ = sX;
   uint8_t* sK = sX + ROWT;
+  uint8_t* sOnes = sX;
   uint8_t* sdA = sX;
   uint8_t* sOm = sX + 2 * ROWT;
   uint8_t* sS = sOm;
-  float* redU = reinterpret_cast<float*>(sX + ROWT);  // [NG][128], phase 4
+  float* redU = reinterpret_cast<float*>(sX + ROWT);  // [NG][128], late phase
   uint8_t* sV = sOm + C::OMB;         // later: dden as a K-major [16][128] operand + row sums
   uint8_t* sDd = sV;
-  float* redA = reinterpret_cast<float*>(sV + 8192);  // [NG][128], phase 2
+  float* redA = reinterpret_cast<float*>(sV + 8192);  // [NG][128]
   uint8_t* sDo = sV + ROWT;           // dout, then dnum in place
   float* sZ = reinterpret_cast<float*>(sDo + ROWT);
-  const int row0 = a + t * T;
-  const int valid = min(T, b - t * T);
-  const size_t g0 = ((size_t)c * L + row0) * D;
-  const float* P = pfx + ((size_t)c * nt + t) * C::E;
+  // tiles in reverse order: CTA b takes tile ntn-1-b/chains of chain b%chains
+  const int c = b % J.chains, t = J.ntn - 1 - b / J.chains, n = J.n;
+  const int row0 = J.a + t * T;
+  const int valid = min(T, J.b - t * T);
+  const size_t g0 = ((size_t)c * J.L + row0) * D;
+  const size_t ti = (size_t)c * J.ntn + t;  // this slice's per-tile buffers
+  // The prefixes after this tile: the next tile's slots, the first tile of
+  // slice n+1, or (at the end of the sequence) B^(N) and G = 0.
+  const bool inner = t + 1 < J.ntn, next_slice = n + 1 < J.N;
+  const int snext = inner ? t + 1 : 0;
+  const int wnext = inner ? n + 1 : n + 2;
+  const bool linked = inner || next_slice;
+  StateRef s1, s2;
+  if (linked) {
+    const float* p1 = J.slot1 + ((size_t)c * J.nt + snext) * C::E;
+    const float* p2 = J.slot2 + ((size_t)c * J.nt + snext) * C::E;
+    s1 = StateRef{p1, p1 + MF * 64, nullptr, nullptr};
+    s2 = StateRef{p2, p2 + MF * 64, nullptr, nullptr};
+  } else {
+    s1 = StateRef{J.fin.S + (size_t)c * MF * 64, J.fin.z + (size_t)c * MF,
+                  J.fin.S_lo ? J.fin.S_lo + (size_t)c * MF * 64 : nullptr,
+                  J.fin.z_lo ? J.fin.z_lo + (size_t)c * MF : nullptr};
+    s2 = StateRef{nullptr, nullptr, nullptr, nullptr};
+  }
+  const int* f1 = J.flag1 + ((size_t)c * J.nt + snext) * FLAG_STRIDE;
+  const int* f2 = J.flag2 + ((size_t)c * J.nt + snext) * FLAG_STRIDE;
+  float* own1 = J.slot1 + ((size_t)c * J.nt + t) * C::E;
+  float* own2 = J.slot2 + ((size_t)c * J.nt + t) * C::E;
+  int* of1 = J.flag1 + ((size_t)c * J.nt + t) * FLAG_STRIDE;
+  int* of2 = J.flag2 + ((size_t)c * J.nt + t) * FLAG_STRIDE;
   TC_PROLOGUE();
-  load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
-  load_rows64(sK, T, K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, V + g0, valid, tid, NTHR);
-  load_rows64(sDo, T, dOut + g0, valid, tid, NTHR);
+  load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
+  load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
+  load_rows64(sDo, T, J.dOut + g0, valid, tid, NTHR);
   // this thread's 16 columns of its out row, fetched while the tiles stream in
   uint4 orow[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
   if (row < valid) {
-    const uint4* src = reinterpret_cast<const uint4*>(Out + g0 + (size_t)row * D + 16 * cg);
+    const uint4* src = reinterpret_cast<const uint4*>(J.Out + g0 + (size_t)row * D + 16 * cg);
     orow[0] = src[0];
     orow[1] = src[1];
   }
-  grid_dependency_wait();  // the state prefixes come from the scan just before
-  load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhiK, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
-  for (int m = tid; m < MF; m += NTHR) sZ[m] = P[MF * 64 + m];
+  grid_dependency_wait();  // Omega (bf16), slots and buffers belong to earlier kernels
+  load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
+  load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
@@ -481,7 +631,7 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
     const float rowdot = group_total(redN + 2 * NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, err};
+    Sync sy{smem_u32(&mbar), 0u, J.err};
     if (tid == 0) {
       // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -498,27 +648,31 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
       mma_commit(sy.mbar);
     }
     TC_WAIT(sy);  // Q projection done
-    float* redZ = reinterpret_cast<float*>(sQ);  // Q is dead; dA is written after the next waits
-    redZ[cg * T + row] = feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv, sZ);
-    TC_WAIT(sy);  // K projection done: S_t replaces Omega
-    load_f32_rows64<MF>(sS, P, tid);
+    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    TC_WAIT(sy);  // K projection done: Q, K and Omega are dead
+    fill_ones(sOnes, tid);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
       const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
-      const uint32_t aDo = smem_u32(sDo), aV = smem_u32(sV);
-      for (int k0 = 0; k0 < MF; k0 += 16)
+      const uint32_t aDo = smem_u32(sDo), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
+      for (int k0 = 0; k0 < MF; k0 += 16)  // A = phiQ phiK^T
         mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
       for (int k0 = 0; k0 < D; k0 += 16)  // dout V^T (scaled by 1/den below)
         mma(tmem + 128, kmaj(aDo, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      for (int h = 0; h < C::MH; ++h)  // Delta_t = phiK^T [V | 1]
+        for (int k0 = 0; k0 < T; k0 += 16) {
+          const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
+          mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+          mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
+        }
       mma_commit(sy.mbar);
     }
-    const float dz = group_total(redZ, row);
     TC_WAIT(sy);
+    float rs = 0.f;  // den partial: the rounded masked A values of this thread's columns
     {
       float v[32];
       tmem_ld32(trow + 32 * cg, v);
-      float rs = 0.f;
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
         const float x0 = (32 * cg + i <= row) ? v[i] : 0.f;
@@ -527,13 +681,73 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
         unpack_bf16(pack_bf16(x0, x1), r0, r1);
         rs += r0 + r1;
       }
+    }
+    // ---- chain 1, the rollback (eq. 17 per tile): the state before this tile
+    // is the state after it minus Delta_t.
+    {
+      if (linked && !chain_acquire(f1, wnext, J.err, abort_)) goto teardown;
+      // every load of the prefix after this tile before any store: one L2 trip
+      float sv[C::MH][16], sz[C::MH];
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + row;
+        if (linked)
+          ld_lm16(s1.S, h, cg, row, sv[h]);
+        else
+          ld_row16f(s1.S + (size_t)m * 64 + 16 * cg, sv[h]);
+        sz[h] = cg == 0 ? __ldcg(s1.z + m) : 0.f;
+      }
+      if (s1.S_lo) {
+#pragma unroll
+        for (int h = 0; h < C::MH; ++h) {
+          const int m = 128 * h + row;
+          float lo[16];
+          ld_row16f(s1.S_lo + (size_t)m * 64 + 16 * cg, lo);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sv[h][i] += lo[i];
+        }
+      }
+      if (cg == 0 && s1.z_lo) {
+#pragma unroll
+        for (int h = 0; h < C::MH; ++h) sz[h] += __ldcg(s1.z_lo + 128 * h + row);
+      }
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + row;
+        float d[16];
+        tmem_ld16(trow + 256 + 64 * h + 16 * cg, d);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sv[h][i] -= d[i];
+        st_lm16(own1, h, cg, row, sv[h]);
+        st_tile16(sS, MF, m, 16 * cg, sv[h]);
+      }
+      if (cg == 0) {
+#pragma unroll
+        for (int h = 0; h < C::MH; ++h) {
+          const int m = 128 * h + row;
+          float dz;
+          tmem_ld1(trow + 384 + 16 * h, dz);
+          const float z = sz[h] - dz;
+          __stcg(own1 + MF * 64 + m, z);
+          sZ[m] = z;
+        }
+      }
+      chain_release(of1, n + 1);
+    }
+    {
+      // + phiQ . z_t over this thread's feature columns
+      constexpr int W = MF / NG;
+#pragma unroll
+      for (int f0 = cg * W; f0 < (cg + 1) * W; f0 += 16) {
+        float f[16];
+        ld_feat16(sPhiQ, row, f0, f);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rs = fmaf(f[i], sZ[f0 + i], rs);
+      }
       redA[cg * T + row] = rs;  // V is no longer read: its tile holds the partials
     }
     __syncthreads();
-    float rs = 0.f;
-#pragma unroll
-    for (int g = 0; g < NG; ++g) rs += redA[g * T + row];
-    const float den = rs + dz;
+    const float den = group_total(redA, row);
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     const float dden = live ? -rowdot * inv : 0.f;
@@ -569,11 +783,11 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
     }
     // dden as the first row of a K-major [16][128] operand (other rows zero)
 #pragma unroll
-    for (int n = 4 * cg; n < 4 * cg + 4; ++n)
-      *reinterpret_cast<__nv_bfloat16*>(sDd + tile_off(16, n, row)) =
-          __float2bfloat16_rn(n == 0 ? dden : 0.f);
+    for (int r16 = 4 * cg; r16 < 4 * cg + 4; ++r16)
+      *reinterpret_cast<__nv_bfloat16*>(sDd + tile_off(16, r16, row)) =
+          __float2bfloat16_rn(r16 == 0 ? dden : 0.f);
     if (rv && cg == 0) {
-      float* rsw = rowstat + (((size_t)c * nt + t) * T + row) * 2;
+      float* rsw = J.rowstat + (ti * T + row) * 2;
       rsw[0] = den;
       rsw[1] = dden;
     }
@@ -595,23 +809,9 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
     }
     TC_WAIT(sy);
     // Q and Omega again (for dq = u Omega - q sum(u) and dOmega += u^T q); the
-    // copies overlap the epilogue below
-    load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
-    load_rows64(sOm, MF, om16, MF, tid, NTHR);
-    {
-      float* dst = gdelta + ((size_t)c * nt + t) * C::E;
-      for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + row;
-        float v[16];
-        tmem_ld16(trow + 64 * h + 16 * cg, v);
-        st_f32x16(dst + (size_t)m * 64 + 16 * cg, v);
-        if (cg == 0) {
-          float zz;
-          tmem_ld1(trow + 128 + 16 * h, zz);
-          dst[MF * 64 + m] = zz;
-        }
-      }
-    }
+    // copies overlap the chain and the epilogue below
+    load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
+    load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
     {
       // dphiQ (+ dden z_t) -> u (into the phiK tile), this thread's columns
       constexpr int W = MF / NG;
@@ -653,14 +853,59 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
     cp_async_wait_all();
     publish();
     if (tid == 0) {
+      // dq and the dOmega partial go to the columns dphiQ held, so Gd stays
+      // readable for the chain below
       const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aQ = smem_u32(sQ);
       for (int k0 = 0; k0 < MF; k0 += 16)
-        mma(tmem, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+        mma(tmem + 256, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
       for (int h = 0; h < C::MH; ++h)
         for (int k0 = 0; k0 < T; k0 += 16)
-          mma(tmem + 64 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aQ, k0, ROWT),
+          mma(tmem + 320 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aQ, k0, ROWT),
               idesc_bf16(T, 64, 1, 1), k0 > 0);
       mma_commit(sy.mbar);
+    }
+    // ---- chain 2, the state gradient (eq. 18): G_t = the prefix after this
+    // tile (zero at the end of the sequence); G_t + Gd_t goes on to tile t-1.
+    // It runs while the tensor core computes dq.
+    {
+      if (linked && !chain_acquire(f2, wnext, J.err, abort_)) {
+        sy.wait();  // the dq products are in flight; let them land first
+        goto teardown;
+      }
+      float gs[C::MH][16], gzs[C::MH];
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + row;
+        if (s2.S) {
+          ld_lm16(s2.S, h, cg, row, gs[h]);
+          gzs[h] = cg == 0 ? __ldcg(s2.z + m) : 0.f;
+        } else {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) gs[h][i] = 0.f;
+          gzs[h] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        const int m = 128 * h + row;
+        st_lm16_bf16(J.gS + ti * MF * 64, h, cg, row, gs[h]);  // G_t(S) for the dk/dv side
+        float gd[16];
+        tmem_ld16(trow + 64 * h + 16 * cg, gd);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) gs[h][i] += gd[i];
+        st_lm16(own2, h, cg, row, gs[h]);
+      }
+      if (cg == 0) {
+#pragma unroll
+        for (int h = 0; h < C::MH; ++h) {
+          const int m = 128 * h + row;
+          float gdz;
+          tmem_ld1(trow + 128 + 16 * h, gdz);
+          J.gz[ti * MF + m] = gzs[h];
+          __stcg(own2 + MF * 64 + m, gzs[h] + gdz);
+        }
+      }
+      chain_release(of2, n + 1);
     }
     float us = 0.f;
     if (FEAT == SLIM_FEAT_EXP) {
@@ -672,30 +917,34 @@ __device__ __forceinline__ void role_bwd_q(const __nv_bfloat16* __restrict__ Q, 
       float xq[16];
       ld_feat16(sQ, row, 16 * cg, xq);
       float v[16];
-      tmem_ld16(trow + 16 * cg, v);
+      tmem_ld16(trow + 256 + 16 * cg, v);
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xq[i], v[i]);
-      if (rv) st_row16(dq + g0 + (size_t)row * D + 16 * cg, v);
-      float* dst = part + ((size_t)c * nt + t) * (size_t)(MF * 64);
+      if (rv) st_row16(J.dq + g0 + (size_t)row * D + 16 * cg, v);
+      float* dst = J.part + ti * (size_t)(MF * 64);
       for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + row;
-        tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
-        st_f32x16(dst + (size_t)m * 64 + 16 * cg, v);
+        tmem_ld16(trow + 320 + 64 * h + 16 * cg, v);
+        st_lm16(dst, h, cg, row, v);
       }
     }
   }
   TC_TEARDOWN();
 }
 
-// ================================================================== tc_bwd_kv
+// ================================================================== backward, dk/dv side
+struct BwdKVJob {
+  const __nv_bfloat16 *Q, *K, *V, *dOut, *om16;
+  const __nv_bfloat16* gS;  // [chains][nt][MF][64] G_t(S), from the dq side
+  const float *gz, *rowstat;
+  int L, a, b, nt;           // slice rows [a, a+b), nt tiles
+  __nv_bfloat16 *dk, *dv;
+  float* part;
+  int* err;
+};
+
 template <int MF, int FEAT>
-__device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
-                const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ dOut,
-                const __nv_bfloat16* __restrict__ om16, const float* __restrict__ gsfx,
-                const float* __restrict__ rowstat, int L, int a, int b, int nt,
-                __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv,
-                float* __restrict__ part, int* err,
-    int t, int c, uint8_t* smem_raw, uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
+__device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uint8_t* smem_raw,
+                                            uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;               // later: u
@@ -712,22 +961,22 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
   uint8_t* sV = sOm + C::OMB;
   uint8_t* sDn = sV + ROWT;            // dout, then dnum in place
   float* sGz = reinterpret_cast<float*>(sDn + ROWT);
-  const int row0 = a + t * T;
-  const int valid = min(T, b - t * T);
-  const size_t g0 = ((size_t)c * L + row0) * D;
-  const float* G = gsfx + ((size_t)c * nt + t) * C::E;
+  const int row0 = J.a + t * T;
+  const int valid = min(T, J.b - t * T);
+  const size_t g0 = ((size_t)c * J.L + row0) * D;
+  const size_t ti = (size_t)c * J.nt + t;
   TC_PROLOGUE();
-  load_rows64(sQ, T, Q + g0, valid, tid, NTHR);
-  load_rows64(sK, T, K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, V + g0, valid, tid, NTHR);
-  load_rows64(sDn, T, dOut + g0, valid, tid, NTHR);
-  grid_dependency_wait();  // G suffixes (scan) and row statistics (tc_bwd_q) are earlier kernels'
-  load_rows64(sOm, MF, om16, MF, tid, NTHR);
-  load_rows64(sPhiK, MF, om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
-  for (int m = tid; m < MF; m += NTHR) sGz[m] = G[MF * 64 + m];
+  load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
+  load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
+  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
+  load_rows64(sDn, T, J.dOut + g0, valid, tid, NTHR);
+  grid_dependency_wait();  // G_t and the row statistics come from the dq side, an earlier kernel
+  load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
+  load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
+  for (int m = tid; m < MF; m += NTHR) sGz[m] = J.gz[ti * MF + m];
   float den = 0.f, dden = 0.f;
   if (row < valid) {
-    const float* rsr = rowstat + (((size_t)c * nt + t) * T + row) * 2;
+    const float* rsr = J.rowstat + (ti * T + row) * 2;
     den = rsr[0];
     dden = rsr[1];
   }
@@ -758,7 +1007,7 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
     const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, err};
+    Sync sy{smem_u32(&mbar), 0u, J.err};
     if (tid == 0) {
       // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -776,8 +1025,8 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
     }
     TC_WAIT(sy);  // Q projection done
     feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
-    TC_WAIT(sy);  // K projection done: G_t(S) replaces Omega
-    load_f32_rows64<MF>(sG, G, tid);
+    TC_WAIT(sy);  // K projection done: G_t(S) replaces Omega (awaited before the dV products)
+    load_lm_bf16(sG, MF, J.gS + ti * MF * 64, tid);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
@@ -802,6 +1051,7 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
       for (int q = 0; q < 4; ++q)
         st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
     }
+    cp_async_wait_all();  // G_t(S)
     publish();
     if (tid == 0) {
       const uint32_t aA = smem_u32(sA), aDn = smem_u32(sDn), aPK = smem_u32(sPhiK);
@@ -818,7 +1068,7 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
     {
       float v[16];
       tmem_ld16(trow + 16 * cg, v);  // dv
-      if (rv) st_row16(dv + g0 + (size_t)row * D + 16 * cg, v);
+      if (rv) st_row16(J.dv + g0 + (size_t)row * D + 16 * cg, v);
     }
     {  // dA = tril(dnum V^T + dden) -> smem, this thread's 32 columns
       float v[32];
@@ -844,8 +1094,8 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
     }
     TC_WAIT(sy);
     // K and Omega again (dk = u Omega - k sum(u), dOmega += u^T k), overlapping the epilogue
-    load_rows64(sKr, T, K + g0, valid, tid, NTHR);
-    load_rows64(sOm, MF, om16, MF, tid, NTHR);
+    load_rows64(sKr, T, J.K + g0, valid, tid, NTHR);
+    load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
     {
       // dphiK (+ g_z) -> u (into the phiQ tile), this thread's columns
       constexpr int W = MF / NG;
@@ -909,21 +1159,15 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
       tmem_ld16(trow + 16 * cg, v);
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xk[i], v[i]);
-      if (rv) st_row16(dk + g0 + (size_t)row * D + 16 * cg, v);
-      float* dst = part + ((size_t)c * nt + t) * (size_t)(MF * 64);
+      if (rv) st_row16(J.dk + g0 + (size_t)row * D + 16 * cg, v);
+      float* dst = J.part + ti * (size_t)(MF * 64);
       for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + row;
+        float w[16];
+        ld_lm16(dst, h, cg, row, w);  // the dq side's partial of this tile
         tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
-        float4* o = reinterpret_cast<float4*>(dst + (size_t)m * 64 + 16 * cg);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          float4 x = o[i];
-          x.x += v[4 * i];
-          x.y += v[4 * i + 1];
-          x.z += v[4 * i + 2];
-          x.w += v[4 * i + 3];
-          o[i] = x;
-        }
+        for (int i = 0; i < 16; ++i) w[i] += v[i];
+        st_lm16(dst, h, cg, row, w);
       }
     }
   }
@@ -931,44 +1175,14 @@ __device__ __forceinline__ void role_bwd_kv(const __nv_bfloat16* __restrict__ Q,
 }
 
 // ================================================================== launches
-// One launch runs tiles of up to four roles (independent work of different
-// slices, longest role first so the short ones fill the last wave); CTA b of
-// a role handles tile b % nt of chain b / nt.
-struct DeltaJob {
-  const __nv_bfloat16 *K, *V, *om16;
-  int L, a, b, nt;
-  float* delta;
-  int* err;
-};
-struct FwdJob {
-  const __nv_bfloat16 *Q, *K, *V, *om16;
-  const float* pfx;
-  int L, a, b, nt;
-  __nv_bfloat16* out;
-  int* err;
-};
-struct BwdQJob {
-  const __nv_bfloat16 *Q, *K, *V, *Out, *dOut, *om16;
-  const float* pfx;
-  int L, a, b, nt;
-  __nv_bfloat16* dq;
-  float *gdelta, *rowstat, *part;
-  int* err;
-};
-struct BwdKVJob {
-  const __nv_bfloat16 *Q, *K, *V, *dOut, *om16;
-  const float *gsfx, *rowstat;
-  int L, a, b, nt;
-  __nv_bfloat16 *dk, *dv;
-  float* part;
-  int* err;
-};
+// One launch runs tiles of up to three roles; the roles with chain waits
+// (forward, dq side) come after the dk/dv side, and inside a role every tile
+// waits only on tiles with lower block indices.
 struct TileJobs {
-  int n_kv, n_q, n_fwd, n_delta;  // CTAs of each role, in dispatch order
+  int n_kv, n_q, n_fwd;  // CTAs of each role, in dispatch order
   BwdKVJob kv;
   BwdQJob q;
   FwdJob f;
-  DeltaJob d;
 };
 
 template <int MF, int FEAT>
@@ -979,70 +1193,37 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ Ti
   __shared__ int abort_;
   int b = blockIdx.x;
   if (b < J.n_kv) {
-    const BwdKVJob& p = J.kv;
-    role_bwd_kv<MF, FEAT>(p.Q, p.K, p.V, p.dOut, p.om16, p.gsfx, p.rowstat, p.L, p.a, p.b, p.nt,
-                          p.dk, p.dv, p.part, p.err, b % p.nt, b / p.nt, smem_raw, mbar,
-                          tmem_base, abort_);
+    role_bwd_kv<MF, FEAT>(J.kv, b % J.kv.nt, b / J.kv.nt, smem_raw, mbar, tmem_base, abort_);
     return;
   }
   b -= J.n_kv;
   if (b < J.n_q) {
-    const BwdQJob& p = J.q;
-    role_bwd_q<MF, FEAT>(p.Q, p.K, p.V, p.Out, p.dOut, p.om16, p.pfx, p.L, p.a, p.b, p.nt, p.dq,
-                         p.gdelta, p.rowstat, p.part, p.err, b % p.nt, b / p.nt, smem_raw, mbar,
-                         tmem_base, abort_);
+    role_bwd_q<MF, FEAT>(J.q, b, smem_raw, mbar, tmem_base, abort_);
     return;
   }
   b -= J.n_q;
-  if (b < J.n_fwd) {
-    const FwdJob& p = J.f;
-    role_fwd<MF, FEAT>(p.Q, p.K, p.V, p.om16, p.pfx, p.L, p.a, p.b, p.nt, p.out, p.err, b % p.nt,
-                       b / p.nt, smem_raw, mbar, tmem_base, abort_);
-    return;
-  }
-  b -= J.n_fwd;
-  if (b < J.n_delta) {
-    const DeltaJob& p = J.d;
-    role_delta<MF, FEAT>(p.K, p.V, p.om16, p.L, p.a, p.b, p.nt, p.delta, p.err, b % p.nt,
-                         b / p.nt, smem_raw, mbar, tmem_base, abort_);
-  }
+  if (b < J.n_fwd)
+    role_fwd<MF, FEAT>(J.f, b / J.f.chains, b % J.f.chains, smem_raw, mbar, tmem_base, abort_);
 }
 
-// The small steps between tile launches: up to two state scans (the
-// forward/rollback carry of one slice and the state-gradient carry of
-// another), and the two stages of the dOmega reduction of earlier slices.
+// dOmega reduction of one slice's per-tile partials (lane-major), in two
+// stages that run in the small launches between tile launches:
+//   stage 1: sums[split][e] = sum of the partials of one fixed range
+//   stage 2: domega[e] += sum over the RSPLIT sums, in order
 constexpr int RSPLIT = 64;
-struct ScanJob {
-  float *buf, *hi, *lo;
-  int chains, nt, E4, mode, blocks;
-};
-struct SmallJobs {
-  ScanJob scan[2];
-  int nscan;
-  // stage 1: sums[split][e] = sum of partials of one range (blocks = r1_bx * RSPLIT)
+struct ReduceJobs {
   const float* r1_part;
   float* r1_sums;
   int r1_nparts, r1_bx;
-  // stage 2: domega[e] += sum over the RSPLIT sums, in order
   const float* r2_sums;
   float* r2_domega;
   int r2_blocks;
   int n;  // M * 64
 };
 
-__global__ void __launch_bounds__(256) k_tc_small(const __grid_constant__ SmallJobs J) {
+__global__ void __launch_bounds__(256) k_tc_reduce(const __grid_constant__ ReduceJobs J) {
   grid_dependency_wait();
   int b = blockIdx.x;
-  for (int i = 0; i < J.nscan; ++i) {
-    const ScanJob& q = J.scan[i];
-    if (b < q.blocks) {
-      scan_thread(reinterpret_cast<float4*>(q.buf), reinterpret_cast<float4*>(q.hi),
-                  reinterpret_cast<float4*>(q.lo), q.chains, q.nt, q.E4, q.mode,
-                  (long long)b * 256 + threadIdx.x);
-      return;
-    }
-    b -= q.blocks;
-  }
   if (b < J.r1_bx * RSPLIT) {
     const int e = (b % J.r1_bx) * 256 + threadIdx.x, split = b / J.r1_bx;
     if (e >= J.n) return;
@@ -1061,7 +1242,11 @@ __global__ void __launch_bounds__(256) k_tc_small(const __grid_constant__ SmallJ
     float s = 0.f;
 #pragma unroll
     for (int i = 0; i < RSPLIT; ++i) s += J.r2_sums[(size_t)i * J.n + e];
-    J.r2_domega[e] += s;
+    // e is a lane-major index: float4 q = e / 4 holds row 128h + row,
+    // columns 16cg + 4i .. +3
+    const int q = e >> 2, row = q & 127, rest = q >> 7, i = rest & 3;
+    const int cg = (rest >> 2) % NG, h = rest / (4 * NG);
+    J.r2_domega[(128 * h + row) * 64 + 16 * cg + 4 * i + (e & 3)] += s;
   }
 }
 
@@ -1077,35 +1262,6 @@ __global__ void k_omega_bf16(const float* om, __nv_bfloat16* om16, int n) {
   }
 }
 
-// state pair [chains][E] <-> S_state [chains][M][64], z_state [chains][M]
-// (the pair is normalised: hi is the rounded state, lo its residual)
-__global__ void k_tc_state_out(const float* hi, const float* lo, StateOut st, int chains, int MF) {
-  grid_dependency_wait();
-  const long long E = (long long)MF * 65;
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= chains * E) return;
-  const long long c = i / E, e = i % E;
-  if (e < (long long)MF * 64) {
-    st.S[c * MF * 64 + e] = hi[i];
-    if (st.S_lo) st.S_lo[c * MF * 64 + e] = lo[i];
-  } else {
-    st.z[c * MF + (e - (long long)MF * 64)] = hi[i];
-    if (st.z_lo) st.z_lo[c * MF + (e - (long long)MF * 64)] = lo[i];
-  }
-}
-__global__ void k_tc_state_in(StateIn st, float* hi, float* lo, int chains, int MF) {
-  const long long E = (long long)MF * 65;
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= chains * E) return;
-  const long long c = i / E, e = i % E;
-  if (e < (long long)MF * 64) {
-    hi[i] = st.S[c * MF * 64 + e];
-    lo[i] = st.S_lo ? st.S_lo[c * MF * 64 + e] : 0.f;
-  } else {
-    hi[i] = st.z[c * MF + (e - (long long)MF * 64)];
-    lo[i] = st.z_lo ? st.z_lo[c * MF + (e - (long long)MF * 64)] : 0.f;
-  }
-}
 // ================================================================== host
 namespace {
 
@@ -1125,32 +1281,33 @@ Geo geometry(const Problem& p) {
   return g;
 }
 
-// Every per-slice buffer has two slots (slice n uses slot n % 2), because
-// consecutive slices overlap in the pipelined launches.
+// The chain slots hold one prefix per (chain, tile of a slice): a slice's
+// tiles overwrite the previous slice's only after reading them.  The buffers
+// the dq side hands to the dk/dv side have two slots (slice n uses n % 2),
+// because the dq side of slice n-1 runs beside the dk/dv side of slice n.
 struct Ws {
   int* err;
+  int* flags;  // [2][chains][nt], FLAG_STRIDE ints each
   __nv_bfloat16* om16;
-  float *st_hi, *st_lo;
-  float* delta[2];
-  float *g_hi, *g_lo;
-  float *gdelta[2], *rowstat[2], *part[2], *rsums[2];
+  float *slot1, *slot2;
+  __nv_bfloat16* gS[2];
+  float *gz[2], *rowstat[2], *part[2], *rsums[2];
 };
 
 Ws carve(Carver& cv, const Geo& g, bool bwd) {
   Ws w{};
-  const size_t C = g.chains;
+  const size_t C = g.chains, tiles = C * g.nt;
   w.err = cv.take<int>(64);
+  w.flags = cv.take<int>(2 * tiles * FLAG_STRIDE);
   w.om16 = cv.take<__nv_bfloat16>((size_t)2 * g.MF * D);
-  w.st_hi = cv.take<float>(C * g.E);
-  w.st_lo = cv.take<float>(C * g.E);
-  for (int k = 0; k < 2; ++k) w.delta[k] = cv.take<float>(C * g.nt * g.E);
+  w.slot1 = cv.take<float>(tiles * g.E);
   if (bwd) {
-    w.g_hi = cv.take<float>(C * g.E);
-    w.g_lo = cv.take<float>(C * g.E);
+    w.slot2 = cv.take<float>(tiles * g.E);
     for (int k = 0; k < 2; ++k) {
-      w.gdelta[k] = cv.take<float>(C * g.nt * g.E);
-      w.rowstat[k] = cv.take<float>(C * g.nt * T * 2);
-      w.part[k] = cv.take<float>(C * g.nt * (size_t)g.MF * D);
+      w.gS[k] = cv.take<__nv_bfloat16>(tiles * g.MF * D);
+      w.gz[k] = cv.take<float>(tiles * g.MF);
+      w.rowstat[k] = cv.take<float>(tiles * T * 2);
+      w.part[k] = cv.take<float>(tiles * (size_t)g.MF * D);
       w.rsums[k] = cv.take<float>((size_t)RSPLIT * g.MF * D);
     }
   }
@@ -1159,10 +1316,8 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
 
 // dynamic shared memory of each role (plus 1 KB for 1024-byte alignment)
 template <int MF>
-constexpr size_t smem_delta() { return 1024 + 2 * ROWT + Cfg<MF>::OMB + Cfg<MF>::FEATB + 4096; }
-template <int MF>
 constexpr size_t smem_fwd() {
-  return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + MF * 4 + NG * T * 4;
+  return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + 4096 + MF * 4 + NG * T * 4;
 }
 template <int MF>
 constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4; }
@@ -1170,6 +1325,7 @@ template <int MF>
 constexpr size_t smem_max() {
   return smem_bwd<MF>() > smem_fwd<MF>() ? smem_bwd<MF>() : smem_fwd<MF>();
 }
+static_assert(smem_max<256>() <= 232448, "a tile CTA must fit in 227 KB of shared memory");
 
 template <int MF, int FEAT>
 cudaError_t configure() {
@@ -1225,35 +1381,28 @@ Slice slice_of(const Problem& p, const Geo& g, int n) {
 template <int MF, int FEAT>
 cudaError_t launch_tiles(cudaStream_t s, const TileJobs& J, double flops, double bytes,
                          prof::Kid kid) {
-  const int n = J.n_kv + J.n_q + J.n_fwd + J.n_delta;
+  const int n = J.n_kv + J.n_q + J.n_fwd;
   if (n == 0) return cudaSuccess;
-  size_t smem = 0;
-  if (J.n_kv || J.n_q) smem = smem_bwd<MF>();
-  if (J.n_fwd && smem_fwd<MF>() > smem) smem = smem_fwd<MF>();
-  if (J.n_delta && smem_delta<MF>() > smem) smem = smem_delta<MF>();
+  const size_t smem = (J.n_kv || J.n_q) ? smem_bwd<MF>() : smem_fwd<MF>();
   prof::Scope ps(kid, s, flops, bytes);
   return launch_dep(k_tc_tiles<MF, FEAT>, dim3(n), dim3(NTHR), smem, s, J);
 }
 
-cudaError_t launch_small(cudaStream_t s, SmallJobs& J, prof::Kid kid) {
-  int blocks = J.r1_bx * RSPLIT + J.r2_blocks;
-  for (int i = 0; i < J.nscan; ++i) blocks += J.scan[i].blocks;
+cudaError_t launch_reduce(cudaStream_t s, const ReduceJobs& J) {
+  const int blocks = J.r1_bx * RSPLIT + J.r2_blocks;
   if (blocks == 0) return cudaSuccess;
-  prof::Scope ps(kid, s);
-  return launch_dep(k_tc_small, dim3(blocks), dim3(256), 0, s, J);
+  prof::Scope ps(prof::K_TC_REDUCE, s);
+  return launch_dep(k_tc_reduce, dim3(blocks), dim3(256), 0, s, J);
 }
 
-ScanJob scan_job(float* buf, float* hi, float* lo, int chains, int nt, int E, ScanMode mode) {
-  ScanJob j;
-  j.buf = buf;
-  j.hi = hi;
-  j.lo = lo;
-  j.chains = chains;
-  j.nt = nt;
-  j.E4 = E / 4;
-  j.mode = (int)mode;
-  j.blocks = (int)nblk((long long)chains * (E / 4));
-  return j;
+cudaError_t prepare(const Ws& w, const Geo& g, const float* omega, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(w.flags, 0, (size_t)2 * g.chains * g.nt * FLAG_STRIDE * sizeof(int), s);
+  if (e != cudaSuccess) return e;
+  prof::Scope ps(prof::K_TC_PREP, s);
+  k_omega_bf16<<<nblk(g.MF * D), 256, 0, s>>>(omega, w.om16, g.MF * D);  // hi and lo
+  return cudaGetLastError();
 }
 
 template <int MF, int FEAT>
@@ -1264,54 +1413,15 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, false);
-  const size_t SE = (size_t)g.chains * g.E;
-  TC_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
-  TC_TRY(cudaMemsetAsync(w.st_hi, 0, SE * sizeof(float), s));
-  TC_TRY(cudaMemsetAsync(w.st_lo, 0, SE * sizeof(float), s));
-  {
-    prof::Scope ps(prof::K_TC_PREP, s);
-    k_omega_bf16<<<nblk(MF * D), 256, 0, s>>>(omega, w.om16, MF * D);  // hi and lo
-    TC_TRY(cudaGetLastError());
-  }
-  const double MD = (double)MF * D;
-  auto delta_job = [&](int n) {
-    const Slice sl = slice_of(p, g, n);
-    return DeltaJob{k, v, w.om16, p.L, sl.a, sl.b, sl.nt, w.delta[n & 1], w.err};
-  };
-  // Pipeline: the deltas of slice n+1 are computed in the launch that reads
-  // slice n's state prefixes.  Algorithmic work per row: delta 4dM (phiK,
-  // Delta), forward 4dM (phiQ, readout); phiK recomputation and the 128 x 128
-  // tile products are not counted.
-  for (int n = -1; n < g.N; ++n) {
-    TileJobs J{};
-    double rows = 0.0;
-    if (n >= 0) {
-      const Slice sl = slice_of(p, g, n);
-      J.f = FwdJob{q, k, v, w.om16, w.delta[n & 1], p.L, sl.a, sl.b, sl.nt, out, w.err};
-      J.n_fwd = sl.nt * g.chains;
-      rows += (double)g.chains * sl.b;
-    }
-    if (n + 1 < g.N) {
-      const Slice sl = slice_of(p, g, n + 1);
-      J.d = delta_job(n + 1);
-      J.n_delta = sl.nt * g.chains;
-      rows += (double)g.chains * sl.b;
-    }
-    TC_TRY((launch_tiles<MF, FEAT>(s, J, rows * 4.0 * MD, rows * D * 2.0 * 3, prof::K_TC_FWD)));
-    if (n + 1 < g.N) {
-      SmallJobs S{};
-      S.scan[0] = scan_job(w.delta[(n + 1) & 1], w.st_hi, w.st_lo, g.chains,
-                           slice_of(p, g, n + 1).nt, g.E, SCAN_FWD);
-      S.nscan = 1;
-      S.n = MF * D;
-      TC_TRY(launch_small(s, S, prof::K_TC_SCAN));
-    }
-  }
-  {
-    prof::Scope ps(prof::K_STATE, s);
-    TC_TRY(launch_dep(k_tc_state_out, dim3(nblk((long long)SE)), dim3(256), 0, s,
-                      (const float*)w.st_hi, (const float*)w.st_lo, st, g.chains, MF));
-  }
+  TC_TRY(prepare(w, g, omega, s));
+  // every tile of every slice in one launch, in sequence order, chains inside
+  // a tile position.  Algorithmic work per row: 8dM (phiQ, phiK, Delta, readout).
+  TileJobs J{};
+  const int P = (g.N - 1) * g.nt + slice_of(p, g, g.N - 1).nt;
+  J.f = FwdJob{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flags, out, st, w.err};
+  J.n_fwd = P * g.chains;
+  const double rows = (double)g.chains * p.L, MD = (double)MF * D;
+  TC_TRY((launch_tiles<MF, FEAT>(s, J, rows * 8.0 * MD, rows * D * 2.0 * 4, prof::K_TC_FWD)));
   return SLIM_OK;
 }
 
@@ -1325,87 +1435,58 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, true);
-  const size_t SE = (size_t)g.chains * g.E;
   const int N = g.N;
-  TC_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
   TC_TRY(cudaMemsetAsync(domega, 0, (size_t)MF * D * sizeof(float), s));
-  TC_TRY(cudaMemsetAsync(w.g_hi, 0, SE * sizeof(float), s));
-  TC_TRY(cudaMemsetAsync(w.g_lo, 0, SE * sizeof(float), s));
-  {
-    prof::Scope ps(prof::K_TC_PREP, s);
-    k_omega_bf16<<<nblk(MF * D), 256, 0, s>>>(omega, w.om16, MF * D);
-    TC_TRY(cudaGetLastError());
-    k_tc_state_in<<<nblk((long long)SE), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains, MF);
-    TC_TRY(cudaGetLastError());
-  }
+  TC_TRY(prepare(w, g, omega, s));
   const double MD = (double)MF * D;
   const unsigned r_bx = nblk(MF * D);
+  int* flag1 = w.flags;
+  int* flag2 = w.flags + (size_t)g.chains * g.nt * FLAG_STRIDE;
   auto valid = [&](int n) { return n >= 0 && n < N; };
-  // Stage j of the reverse walk (slices n = N-1 .. 0):
-  //   tiles j : dk/dv side of slice N-j, dq side of slice N-1-j, deltas of slice N-2-j
-  //   small j : rollback scan of slice N-2-j, state-gradient scan of slice N-1-j,
-  //             dOmega reduction stage 1 of slice N-j and stage 2 of slice N+1-j
-  // Algorithmic work per row: delta 4dM (phiK, rollback Delta), dq side 10dM,
-  // dk/dv side 8dM.
-  for (int j = -1; j <= N + 1; ++j) {
-    if (j >= 0) {
-      TileJobs J{};
-      double fl = 0.0, by = 0.0;
-      const int nkv = N - j, nq = N - 1 - j, nd = N - 2 - j;
-      if (j >= 1 && valid(nkv)) {
-        const Slice sl = slice_of(p, g, nkv);
-        J.kv = BwdKVJob{q, k, v, dout, w.om16, w.gdelta[nkv & 1], w.rowstat[nkv & 1], p.L, sl.a,
-                        sl.b, sl.nt, dk, dv, w.part[nkv & 1], w.err};
-        J.n_kv = sl.nt * g.chains;
-        fl += (double)g.chains * sl.b * 8.0 * MD;
-        by += (double)g.chains * sl.b * D * 2.0 * 6;
-      }
-      if (valid(nq)) {
-        const Slice sl = slice_of(p, g, nq);
-        J.q = BwdQJob{q, k, v, out, dout, w.om16, w.delta[nq & 1], p.L, sl.a, sl.b, sl.nt, dq,
-                      w.gdelta[nq & 1], w.rowstat[nq & 1], w.part[nq & 1], w.err};
-        J.n_q = sl.nt * g.chains;
-        fl += (double)g.chains * sl.b * 10.0 * MD;
-        by += (double)g.chains * sl.b * D * 2.0 * 6;
-      }
-      if (valid(nd)) {
-        const Slice sl = slice_of(p, g, nd);
-        J.d = DeltaJob{k, v, w.om16, p.L, sl.a, sl.b, sl.nt, w.delta[nd & 1], w.err};
-        J.n_delta = sl.nt * g.chains;
-        fl += (double)g.chains * sl.b * 4.0 * MD;
-        by += (double)g.chains * sl.b * D * 2.0 * 2;
-      }
-      TC_TRY((launch_tiles<MF, FEAT>(s, J, fl, by, prof::K_TC_BWD)));
-    } else {
-      // prologue: deltas of the last slice
-      const Slice sl = slice_of(p, g, N - 1);
-      TileJobs J{};
-      J.d = DeltaJob{k, v, w.om16, p.L, sl.a, sl.b, sl.nt, w.delta[(N - 1) & 1], w.err};
-      J.n_delta = sl.nt * g.chains;
-      TC_TRY((launch_tiles<MF, FEAT>(s, J, (double)g.chains * sl.b * 4.0 * MD,
-                                     (double)g.chains * sl.b * D * 2.0 * 2, prof::K_TC_BWD)));
+  // Stage j of the reverse walk:
+  //   tiles j  : dk/dv side of slice N-j, dq side of slice N-1-j
+  //   reduce j : dOmega stage 1 of slice N-j, stage 2 of slice N+1-j
+  // Algorithmic work per row: dq side 14dM (phiQ, phiK, rollback Delta, dphiQ,
+  // G, dq, dOmega), dk/dv side 8dM (dV, dphiK, dk, dOmega).
+  for (int j = 0; j <= N + 1; ++j) {
+    TileJobs J{};
+    double fl = 0.0, by = 0.0;
+    const int nkv = N - j, nq = N - 1 - j;
+    if (j >= 1 && valid(nkv)) {
+      const Slice sl = slice_of(p, g, nkv);
+      const int x = nkv & 1;
+      J.kv = BwdKVJob{q, k, v, dout, w.om16, w.gS[x], w.gz[x], w.rowstat[x], p.L, sl.a, sl.b,
+                      sl.nt, dk, dv, w.part[x], w.err};
+      J.n_kv = sl.nt * g.chains;
+      fl += (double)g.chains * sl.b * 8.0 * MD;
+      by += (double)g.chains * sl.b * D * 2.0 * 6;
     }
-    SmallJobs S{};
-    S.n = MF * D;
-    const int nr = N - 2 - j, ng = N - 1 - j, nx1 = N - j, nx2 = N + 1 - j;
-    if (valid(nr))
-      S.scan[S.nscan++] = scan_job(w.delta[nr & 1], w.st_hi, w.st_lo, g.chains,
-                                   slice_of(p, g, nr).nt, g.E, SCAN_ROLLBACK);
-    if (j >= 0 && valid(ng))
-      S.scan[S.nscan++] = scan_job(w.gdelta[ng & 1], w.g_hi, w.g_lo, g.chains,
-                                   slice_of(p, g, ng).nt, g.E, SCAN_GREV);
+    if (valid(nq)) {
+      const Slice sl = slice_of(p, g, nq);
+      const int x = nq & 1;
+      J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, sl.a, sl.b, sl.nt, nq, N, g.nt,
+                    g.chains, w.slot1, w.slot2, flag1, flag2, w.gS[x], w.gz[x], w.rowstat[x],
+                    w.part[x], dq, w.err};
+      J.n_q = sl.nt * g.chains;
+      fl += (double)g.chains * sl.b * 14.0 * MD;
+      by += (double)g.chains * sl.b * D * 2.0 * 6;
+    }
+    TC_TRY((launch_tiles<MF, FEAT>(s, J, fl, by, prof::K_TC_BWD)));
+    ReduceJobs R{};
+    R.n = MF * D;
+    const int nx1 = N - j, nx2 = N + 1 - j;
     if (j >= 1 && valid(nx1)) {
-      S.r1_part = w.part[nx1 & 1];
-      S.r1_sums = w.rsums[nx1 & 1];
-      S.r1_nparts = g.chains * slice_of(p, g, nx1).nt;
-      S.r1_bx = (int)r_bx;
+      R.r1_part = w.part[nx1 & 1];
+      R.r1_sums = w.rsums[nx1 & 1];
+      R.r1_nparts = g.chains * slice_of(p, g, nx1).nt;
+      R.r1_bx = (int)r_bx;
     }
     if (j >= 2 && valid(nx2)) {
-      S.r2_sums = w.rsums[nx2 & 1];
-      S.r2_domega = domega;
-      S.r2_blocks = (int)r_bx;
+      R.r2_sums = w.rsums[nx2 & 1];
+      R.r2_domega = domega;
+      R.r2_blocks = (int)r_bx;
     }
-    TC_TRY(launch_small(s, S, prof::K_TC_SCAN));
+    TC_TRY(launch_reduce(s, R));
   }
   return SLIM_OK;
 }
