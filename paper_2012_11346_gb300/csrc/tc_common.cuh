@@ -137,14 +137,19 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo_bytes, ui
   d |= (uint64_t)2 << 61;  // 128-byte swizzle
   return d;
 }
+// The start-address field holds address >> 4 in the low 14 bits, and shared
+// memory offsets stay below 256 KB, so the descriptor of a later position in
+// the same operand is the base descriptor plus (byte offset >> 4).  Every
+// offset below is a multiple of 16 bytes, and the base descriptor is loop
+// invariant, so an MMA loop pays one 64-bit add per operand.
 // K-major operand stored as row tiles of `rows` rows: element (row, k0..k0+15).
 __device__ __forceinline__ uint64_t kmaj(uint32_t base, int rows, int k0) {
-  return sdesc(base + (uint32_t)((k0 >> 6) * rows * 128 + (k0 & 63) * 2), 16, 1024);
+  return sdesc(base, 16, 1024) + (uint64_t)((k0 >> 6) * rows * 8 + (k0 & 63) / 8);
 }
 // MN-major operand stored as row tiles whose rows are K and columns MN:
 // K rows k0..k0+15, MN blocks `block_bytes` apart.
 __device__ __forceinline__ uint64_t mnmaj(uint32_t base, int k0, uint32_t block_bytes) {
-  return sdesc(base + (uint32_t)(k0 * 128), block_bytes, 1024);
+  return sdesc(base, block_bytes, 1024) + (uint64_t)(k0 * 8);
 }
 
 // D[tmem] (+)= A * B, issued by a single thread.

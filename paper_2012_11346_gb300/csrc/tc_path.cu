@@ -70,15 +70,15 @@ __device__ __forceinline__ void ld_feat16(const uint8_t* tile, int r, int c, flo
 
 // Reads this thread's column group of the projection P = X Omega^T from TMEM,
 // applies the feature map, stores phi (bf16) into the [128][MF] feature tile.
+// Columns c0 = first, first + step, ... below last, 32 at a time.
 template <int MF, int FEAT>
-__device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
-                                                 float x2, bool valid) {
-  constexpr int W = MF / NG;
+__device__ __forceinline__ void feature_cols(uint32_t trow, uint8_t* phi, int r, int first,
+                                             int last, int step, float x2, bool valid) {
   // exp map: phi = 2^(p log2e - (|x|^2/2) log2e - log2 sqrt(M))
   const float bias = -0.5f * x2 * kLog2e - 0.5f * log2f((float)MF);
   const float relu_scale = rsqrtf((float)MF);
 #pragma unroll 1
-  for (int c0 = cg * W; c0 < (cg + 1) * W; c0 += 32) {
+  for (int c0 = first; c0 < last; c0 += step) {
     float v[32];
     tmem_ld32(trow + c0, v);
     uint32_t pk[16];
@@ -99,6 +99,13 @@ __device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, in
     for (int q = 0; q < 4; ++q)
       st_chunk(phi, T, r, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
   }
+}
+// This thread's column group cg (MF/NG contiguous columns).
+template <int MF, int FEAT>
+__device__ __forceinline__ void feature_epilogue(uint32_t trow, uint8_t* phi, int r, int cg,
+                                                 float x2, bool valid) {
+  constexpr int W = MF / NG;
+  feature_cols<MF, FEAT>(trow, phi, r, cg * W, (cg + 1) * W, 32, x2, valid);
 }
 
 // Squared norm of columns 16cg..16cg+15 of row r of a [128][64] row tile.
@@ -329,9 +336,39 @@ struct FwdJob {
   int* err;
 };
 
+// The forward splits its warps after the g(K) epilogue: warps 0-7 (column
+// groups 0, 1) compute g(Q), A and the A epilogue, while warps 8-15 (column
+// groups 2, 3) take the chain hop, which needs only Delta_t.  Each MMA
+// completion has its own single-use mbarrier, so the two groups wait on
+// different events without sharing a phase.
+constexpr int GRP = NTHR / 2;
+__device__ __forceinline__ void group_bar(int id) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(GRP) : "memory");
+}
+// publish() for one warp group.
+__device__ __forceinline__ void group_publish(int id) {
+  fence_async_smem();
+  tc_fence_before();
+  group_bar(id);
+  tc_fence_after();
+}
+// Bounded poll of a chain flag by one thread (see chain_acquire).
+__device__ __forceinline__ bool flag_poll(const int* flag, int want, int* err) {
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    if (ld_relaxed_gpu(flag) == want) {
+      fence_acq_rel_gpu();
+      return true;
+    }
+    if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) return false;
+    __nanosleep(i < 16 ? 32 : 256);
+  }
+  atomicExch(err, 1);
+  return false;
+}
+
 template <int MF, int FEAT>
 __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_t* smem_raw,
-                                         uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
+                                         uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;
@@ -342,9 +379,10 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
   uint8_t* sOm = sK + ROWT;        // later: S_t (bf16)
   uint8_t* sS = sOm;
   uint8_t* sV = sOm + C::OMB;
-  uint8_t* sOnes = sV + ROWT;      // [16][128] K-major, all ones
-  float* sZ = reinterpret_cast<float*>(sOnes + 4096);
-  float* red = sZ + MF;            // [NG][128] row partials of den
+  uint8_t* sOnes = sV + ROWT;      // [16][128] K-major, all ones (8 KB region)
+  uint8_t* sZt = sOnes;            // later: [16][MF] K-major, rows z_hi, z_lo, then zeros
+  float* redA = reinterpret_cast<float*>(sOnes + 8192);  // [2][128] row sums of A
+  int* gfail = reinterpret_cast<int*>(redA + 2 * T);    // [2] per-group failure flags
   // tile t of slice n
   const int n = min(pos / J.nt, J.N - 1), t = pos - n * J.nt;
   const int a = n * J.Cs, slen = min(J.Cs, J.L - a);
@@ -359,11 +397,20 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
   float* own = J.slot + ((size_t)c * J.nt + t) * C::E;
   int* oflag = J.flag + ((size_t)c * J.nt + t) * FLAG_STRIDE;
   const bool last = pos == J.P - 1;
-  TC_PROLOGUE();
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int row = 32 * (warp & 3) + (tid & 31);
+  const int cg = warp >> 2;
+  if (tid == 0) {
+    abort_ = 0;
+    for (int i = 0; i < 5; ++i) mbar_init(smem_u32(&mb[i]), 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
   load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
   load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
   load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
   fill_ones(sOnes, tid);
+  if (tid < 2) gfail[tid] = 0;
   grid_dependency_wait();  // Omega (bf16) and the slots belong to earlier kernels
   load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
   load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
@@ -378,139 +425,175 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, J.err};
     if (tid == 0) {
-      // two commits: the phiQ epilogue runs while the K projection is computed
+      // K first: the chain needs only Delta_t
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
       const uint32_t aOl = smem_u32(sPhiK);
-      for (int k0 = 0; k0 < D; k0 += 16) {
-        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
-      }
-      mma_commit(sy.mbar);
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
-      mma_commit(sy.mbar);
+      mma_commit(smem_u32(&mb[0]));
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(smem_u32(&mb[1]));
     }
-    TC_WAIT(sy);  // Q projection done
-    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
-    TC_WAIT(sy);  // K projection done: Omega is dead, phiK takes Omega lo's place
+    if (!mbar_wait(smem_u32(&mb[0]), 0, J.err)) abort_ = 1;
+    tc_fence_after();
+    __syncthreads();
+    if (abort_) goto teardown;
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
-      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
-      const uint32_t aV = smem_u32(sV), aOnes = smem_u32(sOnes);
+      const uint32_t aPK = smem_u32(sPhiK), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
       for (int h = 0; h < C::MH; ++h)  // Delta_t = phiK^T [V | 1]
         for (int k0 = 0; k0 < T; k0 += 16) {
           const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
           mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
           mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
         }
-      for (int k0 = 0; k0 < MF; k0 += 16)  // A = phiQ phiK^T
-        mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
-      mma_commit(sy.mbar);
+      mma_commit(smem_u32(&mb[2]));
     }
-    TC_WAIT(sy);
-    float rs = 0.f;  // sum of this thread's rounded, masked A values
-    {
-      // A: inclusive causal mask, bf16 (independent of the chain: done first)
-      float v[32];
-      const int c0 = 32 * cg;
-      tmem_ld32(trow + c0, v);
-      uint32_t pk[16];
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        const float x0 = (c0 + i <= row) ? v[i] : 0.f;
-        const float x1 = (c0 + i + 1 <= row) ? v[i + 1] : 0.f;
-        pk[i / 2] = pack_bf16(x0, x1);
-        float r0, r1;
-        unpack_bf16(pk[i / 2], r0, r1);
-        rs += r0 + r1;
+    if (warp < 8) {
+      // ---- compute group: g(Q), A = tril(g(Q) g(K)^T), A's bf16 tile and row sums
+      if (!mbar_wait(smem_u32(&mb[1]), 0, J.err)) gfail[0] = 1;
+      tc_fence_after();
+      group_bar(1);
+      if (gfail[0]) goto join;
+      feature_cols<MF, FEAT>(trow, sPhiQ, row, 32 * cg, MF, 64, q2, rv);
+      group_publish(1);
+      if (tid == 0) {
+        const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
+        for (int k0 = 0; k0 < MF; k0 += 16)
+          mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+        mma_commit(smem_u32(&mb[3]));
       }
+      if (!mbar_wait(smem_u32(&mb[3]), 0, J.err)) gfail[0] = 1;
+      tc_fence_after();
+      group_bar(1);
+      if (gfail[0]) goto join;
+      float rs = 0.f;
+#pragma unroll 1
+      for (int c0 = 32 * cg; c0 < T; c0 += 64) {
+        float v[32];
+        tmem_ld32(trow + c0, v);
+        uint32_t pk[16];
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
-    }
-    // ---- chain: S_t, z_t = the predecessor's inclusive prefix (zero for the
-    // first tile); this tile's inclusive prefix S_t + Delta_t goes to its slot.
-    {
-      if (pred && !chain_acquire(pflag, pwant, J.err, abort_)) goto teardown;
-      // every load of the predecessor's prefix before any store: one L2 trip
-      float pv[C::MH][16], pz[C::MH];
-#pragma unroll
-      for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + row;
-        if (pred) {
-          ld_lm16(pred, h, cg, row, pv[h]);
-          pz[h] = cg == 0 ? __ldcg(pred + MF * 64 + m) : 0.f;
-        } else {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) pv[h][i] = 0.f;
-          pz[h] = 0.f;
+        for (int i = 0; i < 32; i += 2) {
+          const float x0 = (c0 + i <= row) ? v[i] : 0.f;
+          const float x1 = (c0 + i + 1 <= row) ? v[i + 1] : 0.f;
+          pk[i / 2] = pack_bf16(x0, x1);
+          float r0, r1;
+          unpack_bf16(pk[i / 2], r0, r1);
+          rs += r0 + r1;
         }
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
+      }
+      redA[cg * T + row] = rs;
+    } else {
+      // ---- chain group: S_t, z_t = the predecessor's inclusive prefix (zero
+      // for the first tile); S_t + Delta_t goes to this tile's slot.  Thread
+      // (row, cg) handles column groups 2(cg-2) and 2(cg-2)+1.
+      const int gl = tid - GRP;  // 0..255
+      if (!mbar_wait(smem_u32(&mb[2]), 0, J.err)) gfail[1] = 1;
+      tc_fence_after();
+      if (pred && gl == 0 && !gfail[1] && !flag_poll(pflag, pwant, J.err)) gfail[1] = 1;
+      group_bar(2);
+      if (gfail[1]) goto join;
+      const int cq = 2 * (cg - 2);
+      float pv[C::MH][2][16], pz[C::MH];
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          if (pred) {
+            ld_lm16(pred, h, cq + j, row, pv[h][j]);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) pv[h][j][i] = 0.f;
+          }
+        }
+        pz[h] = (pred && cq == 0) ? __ldcg(pred + MF * 64 + 128 * h + row) : 0.f;
       }
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         const int m = 128 * h + row;
-        float inc[16];
-        tmem_ld16(trow + 256 + 64 * h + 16 * cg, inc);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) inc[i] += pv[h][i];
-        st_lm16(own, h, cg, row, inc);
-        st_tile16(sS, MF, m, 16 * cg, pv[h]);
-        if (last) {
-          st_f32x16(J.st.S + ((size_t)c * MF + m) * 64 + 16 * cg, inc);
-          if (J.st.S_lo) {
+        for (int j = 0; j < 2; ++j) {
+          float inc[16];
+          tmem_ld16(trow + 256 + 64 * h + 16 * (cq + j), inc);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) inc[i] = 0.f;
-            st_f32x16(J.st.S_lo + ((size_t)c * MF + m) * 64 + 16 * cg, inc);
+          for (int i = 0; i < 16; ++i) inc[i] += pv[h][j][i];
+          st_lm16(own, h, cq + j, row, inc);
+          st_tile16(sS, MF, m, 16 * (cq + j), pv[h][j]);
+          if (last) {
+            st_f32x16(J.st.S + ((size_t)c * MF + m) * 64 + 16 * (cq + j), inc);
+            if (J.st.S_lo) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) inc[i] = 0.f;
+              st_f32x16(J.st.S_lo + ((size_t)c * MF + m) * 64 + 16 * (cq + j), inc);
+            }
           }
         }
       }
-      if (cg == 0) {
+      // z_t as the first two rows (hi, lo in bf16) of a K-major [16][MF]
+      // operand, so that g(Q) z_t is a tensor-core product with ~16-bit z
+      if (cq == 0) {
 #pragma unroll
         for (int h = 0; h < C::MH; ++h) {
           const int m = 128 * h + row;
           float dz;
           tmem_ld1(trow + 384 + 16 * h, dz);
           __stcg(own + MF * 64 + m, pz[h] + dz);
-          sZ[m] = pz[h];
+          const __nv_bfloat16 zh = __float2bfloat16_rn(pz[h]);
+          *reinterpret_cast<__nv_bfloat16*>(sZt + tile_off(16, 0, m)) = zh;
+          *reinterpret_cast<__nv_bfloat16*>(sZt + tile_off(16, 1, m)) =
+              __float2bfloat16_rn(pz[h] - __bfloat162float(zh));
           if (last) {
             J.st.z[(size_t)c * MF + m] = pz[h] + dz;
             if (J.st.z_lo) J.st.z_lo[(size_t)c * MF + m] = 0.f;
           }
         }
+      } else {
+        // rows 2..15 of the z operand are zero (the ones tile was there)
+        for (int e = gl - 128; e < 14 * MF / 8; e += 128) {
+          const int r16 = 2 + e / (MF / 8), k = (e % (MF / 8)) * 8;
+          st_chunk(sZt, 16, r16, k, make_uint4(0u, 0u, 0u, 0u));
+        }
       }
-      chain_release(oflag, n + 1);
+      group_bar(2);  // every slot write of the group is issued
+      if (gl == 0) st_release_gpu(oflag, n + 1);
     }
-    {
-      // the row's den partial: rs plus phiQ . z_t over this thread's features
-      constexpr int W = MF / NG;
-      float zd = 0.f;
-#pragma unroll
-      for (int f0 = cg * W; f0 < (cg + 1) * W; f0 += 16) {
-        float f[16];
-        ld_feat16(sPhiQ, row, f0, f);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) zd = fmaf(f[i], sZ[f0 + i], zd);
-      }
-      red[cg * T + row] = rs + zd;
-    }
+  join:
+    __syncthreads();
+    if (gfail[0] | gfail[1]) goto teardown;
     publish();
     if (tid == 0) {
-      const uint32_t aPQ = smem_u32(sPhiQ), aS = smem_u32(sS);
+      const uint32_t aPQ = smem_u32(sPhiQ), aS = smem_u32(sS), aZ = smem_u32(sZt);
       const uint32_t aA = smem_u32(sA), aV = smem_u32(sV);
-      for (int k0 = 0; k0 < MF; k0 += 16)  // num = phiQ S_t
+      for (int k0 = 0; k0 < MF; k0 += 16) {
+        // num = phiQ S_t;  phiQ [z_hi | z_lo]
         mma(tmem + 128, kmaj(aPQ, T, k0), mnmaj(aS, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
-      for (int k0 = 0; k0 < T; k0 += 16)  // + A V
+        mma(tmem + 192, kmaj(aPQ, T, k0), kmaj(aZ, 16, k0), idesc_bf16(T, 16, 0, 0), k0 > 0);
+      }
+      for (int k0 = 0; k0 < T; k0 += 16)  // num += A V
         mma(tmem + 128, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), 1);
-      mma_commit(sy.mbar);
+      mma_commit(smem_u32(&mb[4]));
     }
-    const float den = group_total(red, row);
-    TC_WAIT(sy);
+    const float rsA = redA[row] + redA[T + row];
+    if (!mbar_wait(smem_u32(&mb[4]), 0, J.err)) abort_ = 1;
+    tc_fence_after();
+    __syncthreads();
+    if (abort_) goto teardown;
     {
+      float zh, zl;
+      tmem_ld1(trow + 192, zh);
+      tmem_ld1(trow + 193, zl);
+      const float den = rsA + (zh + zl);
       const float inv = den != 0.f ? 1.f / den : 0.f;
       float v[16];
       tmem_ld16(trow + 128 + 16 * cg, v);  // every lane loads (warp-aligned op)
@@ -1175,35 +1258,36 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
 }
 
 // ================================================================== launches
-// One launch runs tiles of up to three roles; the roles with chain waits
-// (forward, dq side) come after the dk/dv side, and inside a role every tile
-// waits only on tiles with lower block indices.
+// One launch runs tiles of up to three roles.  The chained roles (dq side,
+// forward) come first so their chains start early; the independent dk/dv
+// tiles follow and fill the launch's tail.  Inside a role every tile waits
+// only on tiles with lower block indices.
 struct TileJobs {
-  int n_kv, n_q, n_fwd;  // CTAs of each role, in dispatch order
-  BwdKVJob kv;
+  int n_q, n_fwd, n_kv;  // CTAs of each role, in dispatch order
   BwdQJob q;
   FwdJob f;
+  BwdKVJob kv;
 };
 
 template <int MF, int FEAT>
 __global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ TileJobs J) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t mbar;
+  __shared__ __align__(8) uint64_t mbar[5];
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
   int b = blockIdx.x;
-  if (b < J.n_kv) {
-    role_bwd_kv<MF, FEAT>(J.kv, b % J.kv.nt, b / J.kv.nt, smem_raw, mbar, tmem_base, abort_);
-    return;
-  }
-  b -= J.n_kv;
   if (b < J.n_q) {
-    role_bwd_q<MF, FEAT>(J.q, b, smem_raw, mbar, tmem_base, abort_);
+    role_bwd_q<MF, FEAT>(J.q, b, smem_raw, mbar[0], tmem_base, abort_);
     return;
   }
   b -= J.n_q;
-  if (b < J.n_fwd)
+  if (b < J.n_fwd) {
     role_fwd<MF, FEAT>(J.f, b / J.f.chains, b % J.f.chains, smem_raw, mbar, tmem_base, abort_);
+    return;
+  }
+  b -= J.n_fwd;
+  if (b < J.n_kv)
+    role_bwd_kv<MF, FEAT>(J.kv, b % J.kv.nt, b / J.kv.nt, smem_raw, mbar[0], tmem_base, abort_);
 }
 
 // dOmega reduction of one slice's per-tile partials (lane-major), in two
@@ -1317,7 +1401,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
 // dynamic shared memory of each role (plus 1 KB for 1024-byte alignment)
 template <int MF>
 constexpr size_t smem_fwd() {
-  return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + 4096 + MF * 4 + NG * T * 4;
+  return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + 8192 + 2 * T * 4 + 16;
 }
 template <int MF>
 constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4; }
