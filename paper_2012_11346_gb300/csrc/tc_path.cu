@@ -413,12 +413,16 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
   if (tid < 2) gfail[tid] = 0;
   grid_dependency_wait();  // Omega (bf16) and the slots belong to earlier kernels
   load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
-  load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
+  // Omega lo in the upper half of the phiQ tile: that half is written only
+  // by the g(Q) epilogue, after the Q projection (the last reader) is done,
+  // while the phiK tile is overwritten as soon as the K projection is done
+  uint8_t* sOl = sPhiQ + C::OMB;
+  load_rows64(sOl, MF, J.om16 + MF * D, MF, tid, NTHR);
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
     const bool rv = row < valid;
-    float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
+    float* redN = reinterpret_cast<float*>(sPhiQ);  // 4 KB scratch below Omega lo
     redN[cg * T + row] = row_norm2_part(sQ, row, cg);
     redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
     publish();
@@ -428,7 +432,7 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     if (tid == 0) {
       // K first: the chain needs only Delta_t
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
-      const uint32_t aOl = smem_u32(sPhiK);
+      const uint32_t aOl = smem_u32(sOl);
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
@@ -619,27 +623,34 @@ struct BwdQJob {
   int* err;
 };
 
+// The dq side splits its warps twice, as the forward does: after the g(K)
+// epilogue, warps 0-7 compute g(Q), A and dout V^T while warps 8-15 run the
+// rollback chain (which needs only Delta_t); after dphiQ, warps 0-7 compute u
+// and issue dq while warps 8-15 run the state-gradient chain.
 template <int MF, int FEAT>
 __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* smem_raw,
-                                           uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
+                                           uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
-  uint8_t* sPhiQ = base;
+  uint8_t* sPhiQ = base;              // first: norm scratch | Omega lo (upper half)
+  uint8_t* sOl = sPhiQ + C::OMB;
   uint8_t* sPhiK = sPhiQ + C::FEATB;  // later: u
   uint8_t* sU = sPhiK;
-  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [ones | . | S_t] -> [dA | S_t] -> [Q | red | Omega]
+  uint8_t* sX = sPhiK + C::FEATB;     // [Q | K | Omega] -> [Q | ones | S_t] -> [dA | S_t] -> [Q | red | Omega]
   uint8_t* sQ = sX;
   uint8_t* sK = sX + ROWT;
-  uint8_t* sOnes = sX;
+  uint8_t* sOnes = sK;                // written once the K projection is done
   uint8_t* sdA = sX;
   uint8_t* sOm = sX + 2 * ROWT;
   uint8_t* sS = sOm;
-  float* redU = reinterpret_cast<float*>(sX + ROWT);  // [NG][128], late phase
-  uint8_t* sV = sOm + C::OMB;         // later: dden as a K-major [16][128] operand + row sums
+  float* redU = reinterpret_cast<float*>(sX + ROWT);  // [2][128], late phase
+  uint8_t* sV = sOm + C::OMB;         // later: dden as a K-major [16][128] operand + row partials
   uint8_t* sDd = sV;
-  float* redA = reinterpret_cast<float*>(sV + 8192);  // [NG][128]
+  float* redA = reinterpret_cast<float*>(sV + 8192);  // [2][128] row sums of A
+  float* redZ = redA + 2 * T;                          // [NG][128] g(Q) . z_t partials
   uint8_t* sDo = sV + ROWT;           // dout, then dnum in place
   float* sZ = reinterpret_cast<float*>(sDo + ROWT);
+  int* gfail = reinterpret_cast<int*>(sZ + MF);       // [2] per-group failure flags
   // tiles in reverse order: CTA b takes tile ntn-1-b/chains of chain b%chains
   const int c = b % J.chains, t = J.ntn - 1 - b / J.chains, n = J.n;
   const int row0 = J.a + t * T;
@@ -670,7 +681,17 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   float* own2 = J.slot2 + ((size_t)c * J.nt + t) * C::E;
   int* of1 = J.flag1 + ((size_t)c * J.nt + t) * FLAG_STRIDE;
   int* of2 = J.flag2 + ((size_t)c * J.nt + t) * FLAG_STRIDE;
-  TC_PROLOGUE();
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int row = 32 * (warp & 3) + (tid & 31);
+  const int cg = warp >> 2;
+  const int gl = tid - GRP;     // index inside the chain group (warps 8-15)
+  const int cq = 2 * (cg - 2);  // chain group: column groups cq, cq + 1
+  if (tid == 0) {
+    abort_ = 0;
+    for (int i = 0; i < 6; ++i) mbar_init(smem_u32(&mb[i]), 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
   load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
   load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
   load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
@@ -682,14 +703,15 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     orow[0] = src[0];
     orow[1] = src[1];
   }
+  if (tid < 2) gfail[tid] = 0;
   grid_dependency_wait();  // Omega (bf16), slots and buffers belong to earlier kernels
   load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
-  load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
+  load_rows64(sOl, MF, J.om16 + MF * D, MF, tid, NTHR);
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
     const bool rv = row < valid;
-    float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
+    float* redN = reinterpret_cast<float*>(sPhiQ);  // 6 KB scratch below Omega lo
     {
       float part = 0.f;  // <dout_r, out_r> over this thread's 16 columns
 #pragma unroll
@@ -714,97 +736,125 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     const float rowdot = group_total(redN + 2 * NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, J.err};
     if (tid == 0) {
-      // two commits: the phiQ epilogue runs while the K projection is computed
+      // K first: the rollback chain needs only Delta_t
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
-      const uint32_t aOl = smem_u32(sPhiK);
-      for (int k0 = 0; k0 < D; k0 += 16) {
-        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
-      }
-      mma_commit(sy.mbar);
+      const uint32_t aOl = smem_u32(sOl);
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
-      mma_commit(sy.mbar);
+      mma_commit(smem_u32(&mb[0]));
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
+      }
+      mma_commit(smem_u32(&mb[1]));
     }
-    TC_WAIT(sy);  // Q projection done
-    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
-    TC_WAIT(sy);  // K projection done: Q, K and Omega are dead
-    fill_ones(sOnes, tid);
+    if (!mbar_wait(smem_u32(&mb[0]), 0, J.err)) abort_ = 1;
+    tc_fence_after();
+    __syncthreads();
+    if (abort_) goto teardown;
+    fill_ones(sOnes, tid);  // the K tile is no longer read
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
-      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
-      const uint32_t aDo = smem_u32(sDo), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
-      for (int k0 = 0; k0 < MF; k0 += 16)  // A = phiQ phiK^T
-        mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
-      for (int k0 = 0; k0 < D; k0 += 16)  // dout V^T (scaled by 1/den below)
-        mma(tmem + 128, kmaj(aDo, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      const uint32_t aPK = smem_u32(sPhiK), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
       for (int h = 0; h < C::MH; ++h)  // Delta_t = phiK^T [V | 1]
         for (int k0 = 0; k0 < T; k0 += 16) {
           const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
           mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
           mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
         }
-      mma_commit(sy.mbar);
+      mma_commit(smem_u32(&mb[2]));
     }
-    TC_WAIT(sy);
-    float rs = 0.f;  // den partial: the rounded masked A values of this thread's columns
-    {
-      float v[32];
-      tmem_ld32(trow + 32 * cg, v);
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        const float x0 = (32 * cg + i <= row) ? v[i] : 0.f;
-        const float x1 = (32 * cg + i + 1 <= row) ? v[i + 1] : 0.f;
-        float r0, r1;
-        unpack_bf16(pack_bf16(x0, x1), r0, r1);
-        rs += r0 + r1;
+    if (warp < 8) {
+      // ---- compute group: g(Q), then A and dout V^T, and A's row sums
+      if (!mbar_wait(smem_u32(&mb[1]), 0, J.err)) gfail[0] = 1;
+      tc_fence_after();
+      group_bar(1);
+      if (gfail[0]) goto join1;
+      feature_cols<MF, FEAT>(trow, sPhiQ, row, 32 * cg, MF, 64, q2, rv);
+      group_publish(1);
+      if (tid == 0) {
+        const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
+        const uint32_t aDo = smem_u32(sDo), aV = smem_u32(sV);
+        for (int k0 = 0; k0 < MF; k0 += 16)  // A = phiQ phiK^T
+          mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+        for (int k0 = 0; k0 < D; k0 += 16)  // dout V^T (scaled by 1/den below)
+          mma(tmem + 128, kmaj(aDo, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+        mma_commit(smem_u32(&mb[3]));
       }
-    }
-    // ---- chain 1, the rollback (eq. 17 per tile): the state before this tile
-    // is the state after it minus Delta_t.
-    {
-      if (linked && !chain_acquire(f1, wnext, J.err, abort_)) goto teardown;
+      if (!mbar_wait(smem_u32(&mb[3]), 0, J.err)) gfail[0] = 1;
+      tc_fence_after();
+      group_bar(1);
+      if (gfail[0]) goto join1;
+      float rs = 0.f;  // the rounded masked A values of this thread's columns
+#pragma unroll 1
+      for (int c0 = 32 * cg; c0 < T; c0 += 64) {
+        float v[32];
+        tmem_ld32(trow + c0, v);
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const float x0 = (c0 + i <= row) ? v[i] : 0.f;
+          const float x1 = (c0 + i + 1 <= row) ? v[i + 1] : 0.f;
+          float r0, r1;
+          unpack_bf16(pack_bf16(x0, x1), r0, r1);
+          rs += r0 + r1;
+        }
+      }
+      redA[cg * T + row] = rs;  // V is no longer read: its tile holds the partials
+    } else {
+      // ---- chain group, rollback (eq. 17 per tile): the state before this
+      // tile is the state after it minus Delta_t
+      if (!mbar_wait(smem_u32(&mb[2]), 0, J.err)) gfail[1] = 1;
+      tc_fence_after();
+      if (linked && gl == 0 && !gfail[1] && !flag_poll(f1, wnext, J.err)) gfail[1] = 1;
+      group_bar(2);
+      if (gfail[1]) goto join1;
       // every load of the prefix after this tile before any store: one L2 trip
-      float sv[C::MH][16], sz[C::MH];
+      float sv[C::MH][2][16], sz[C::MH];
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         const int m = 128 * h + row;
-        if (linked)
-          ld_lm16(s1.S, h, cg, row, sv[h]);
-        else
-          ld_row16f(s1.S + (size_t)m * 64 + 16 * cg, sv[h]);
-        sz[h] = cg == 0 ? __ldcg(s1.z + m) : 0.f;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          if (linked)
+            ld_lm16(s1.S, h, cq + j, row, sv[h][j]);
+          else
+            ld_row16f(s1.S + (size_t)m * 64 + 16 * (cq + j), sv[h][j]);
+        }
+        sz[h] = cq == 0 ? __ldcg(s1.z + m) : 0.f;
       }
       if (s1.S_lo) {
 #pragma unroll
-        for (int h = 0; h < C::MH; ++h) {
-          const int m = 128 * h + row;
-          float lo[16];
-          ld_row16f(s1.S_lo + (size_t)m * 64 + 16 * cg, lo);
+        for (int h = 0; h < C::MH; ++h)
 #pragma unroll
-          for (int i = 0; i < 16; ++i) sv[h][i] += lo[i];
-        }
+          for (int j = 0; j < 2; ++j) {
+            float lo[16];
+            ld_row16f(s1.S_lo + (size_t)(128 * h + row) * 64 + 16 * (cq + j), lo);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) sv[h][j][i] += lo[i];
+          }
       }
-      if (cg == 0 && s1.z_lo) {
+      if (cq == 0 && s1.z_lo) {
 #pragma unroll
         for (int h = 0; h < C::MH; ++h) sz[h] += __ldcg(s1.z_lo + 128 * h + row);
       }
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         const int m = 128 * h + row;
-        float d[16];
-        tmem_ld16(trow + 256 + 64 * h + 16 * cg, d);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) sv[h][i] -= d[i];
-        st_lm16(own1, h, cg, row, sv[h]);
-        st_tile16(sS, MF, m, 16 * cg, sv[h]);
+        for (int j = 0; j < 2; ++j) {
+          float d[16];
+          tmem_ld16(trow + 256 + 64 * h + 16 * (cq + j), d);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sv[h][j][i] -= d[i];
+          st_lm16(own1, h, cq + j, row, sv[h][j]);
+          st_tile16(sS, MF, m, 16 * (cq + j), sv[h][j]);
+        }
       }
-      if (cg == 0) {
+      if (cq == 0) {
 #pragma unroll
         for (int h = 0; h < C::MH; ++h) {
           const int m = 128 * h + row;
@@ -815,22 +865,27 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           sZ[m] = z;
         }
       }
-      chain_release(of1, n + 1);
+      group_bar(2);  // every slot write of the group is issued
+      if (gl == 0) st_release_gpu(of1, n + 1);
     }
+  join1:
+    __syncthreads();
+    if (gfail[0] | gfail[1]) goto teardown;
     {
-      // + phiQ . z_t over this thread's feature columns
+      // g(Q) . z_t over this thread's feature columns
       constexpr int W = MF / NG;
+      float zd = 0.f;
 #pragma unroll
       for (int f0 = cg * W; f0 < (cg + 1) * W; f0 += 16) {
         float f[16];
         ld_feat16(sPhiQ, row, f0, f);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) rs = fmaf(f[i], sZ[f0 + i], rs);
+        for (int i = 0; i < 16; ++i) zd = fmaf(f[i], sZ[f0 + i], zd);
       }
-      redA[cg * T + row] = rs;  // V is no longer read: its tile holds the partials
+      redZ[cg * T + row] = zd;
     }
     __syncthreads();
-    const float den = group_total(redA, row);
+    const float den = redA[row] + redA[T + row] + group_total(redZ, row);
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     const float dden = live ? -rowdot * inv : 0.f;
@@ -888,20 +943,21 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           mma(tmem + 64 * h, ad, mnmaj(aDn, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
           mma(tmem + 128 + 16 * h, ad, kmaj(aDd, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
         }
-      mma_commit(sy.mbar);
+      mma_commit(smem_u32(&mb[4]));
     }
-    TC_WAIT(sy);
-    // Q and Omega again (for dq = u Omega - q sum(u) and dOmega += u^T q); the
-    // copies overlap the chain and the epilogue below
-    load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
-    load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
-    {
-      // dphiQ (+ dden z_t) -> u (into the phiK tile), this thread's columns
-      constexpr int W = MF / NG;
+    if (!mbar_wait(smem_u32(&mb[4]), 0, J.err)) abort_ = 1;
+    tc_fence_after();
+    __syncthreads();
+    if (abort_) goto teardown;
+    if (warp < 8) {
+      // ---- compute group: Q and Omega again (dq = u Omega - q sum(u),
+      // dOmega += u^T q), u = (dphiQ + dden z_t) (.) g'(Q), then the products
+      load_rows64(sQ, T, J.Q + g0, valid, tid, GRP);
+      load_rows64(sOm, MF, J.om16, MF, tid, GRP);
       float usum = 0.f;
       const float rscale = rsqrtf((float)MF);
 #pragma unroll 1
-      for (int c0 = cg * W; c0 < (cg + 1) * W; c0 += 32) {
+      for (int c0 = 32 * cg; c0 < MF; c0 += 64) {
         float v[32];
         tmem_ld32(trow + 256 + c0, v);
         uint32_t pk[16];
@@ -932,53 +988,53 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           st_chunk(sU, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
       }
       redU[cg * T + row] = usum;
-    }
-    cp_async_wait_all();
-    publish();
-    if (tid == 0) {
-      // dq and the dOmega partial go to the columns dphiQ held, so Gd stays
-      // readable for the chain below
-      const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aQ = smem_u32(sQ);
-      for (int k0 = 0; k0 < MF; k0 += 16)
-        mma(tmem + 256, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
-      for (int h = 0; h < C::MH; ++h)
-        for (int k0 = 0; k0 < T; k0 += 16)
-          mma(tmem + 320 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aQ, k0, ROWT),
-              idesc_bf16(T, 64, 1, 1), k0 > 0);
-      mma_commit(sy.mbar);
-    }
-    // ---- chain 2, the state gradient (eq. 18): G_t = the prefix after this
-    // tile (zero at the end of the sequence); G_t + Gd_t goes on to tile t-1.
-    // It runs while the tensor core computes dq.
-    {
-      if (linked && !chain_acquire(f2, wnext, J.err, abort_)) {
-        sy.wait();  // the dq products are in flight; let them land first
-        goto teardown;
+      cp_async_wait_all();
+      group_publish(1);
+      if (tid == 0) {
+        // dq and the dOmega partial go to the columns dphiQ held, so Gd stays
+        // readable for the chain group
+        const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aQ = smem_u32(sQ);
+        for (int k0 = 0; k0 < MF; k0 += 16)
+          mma(tmem + 256, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+        for (int h = 0; h < C::MH; ++h)
+          for (int k0 = 0; k0 < T; k0 += 16)
+            mma(tmem + 320 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aQ, k0, ROWT),
+                idesc_bf16(T, 64, 1, 1), k0 > 0);
+        mma_commit(smem_u32(&mb[5]));
       }
-      float gs[C::MH][16], gzs[C::MH];
+    } else {
+      // ---- chain group, state gradient (eq. 18): G_t = the prefix after this
+      // tile (zero at the end of the sequence); G_t + Gd_t goes on to tile t-1
+      if (linked && gl == 0 && !flag_poll(f2, wnext, J.err)) gfail[1] = 1;
+      group_bar(2);
+      if (gfail[1]) goto join2;
+      float gs[C::MH][2][16], gzs[C::MH];
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + row;
-        if (s2.S) {
-          ld_lm16(s2.S, h, cg, row, gs[h]);
-          gzs[h] = cg == 0 ? __ldcg(s2.z + m) : 0.f;
-        } else {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) gs[h][i] = 0.f;
-          gzs[h] = 0.f;
+        for (int j = 0; j < 2; ++j) {
+          if (s2.S) {
+            ld_lm16(s2.S, h, cq + j, row, gs[h][j]);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) gs[h][j][i] = 0.f;
+          }
+        }
+        gzs[h] = (s2.z && cq == 0) ? __ldcg(s2.z + 128 * h + row) : 0.f;
+      }
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          st_lm16_bf16(J.gS + ti * MF * 64, h, cq + j, row, gs[h][j]);  // G_t(S), dk/dv side
+          float gd[16];
+          tmem_ld16(trow + 64 * h + 16 * (cq + j), gd);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) gs[h][j][i] += gd[i];
+          st_lm16(own2, h, cq + j, row, gs[h][j]);
         }
       }
-#pragma unroll
-      for (int h = 0; h < C::MH; ++h) {
-        const int m = 128 * h + row;
-        st_lm16_bf16(J.gS + ti * MF * 64, h, cg, row, gs[h]);  // G_t(S) for the dk/dv side
-        float gd[16];
-        tmem_ld16(trow + 64 * h + 16 * cg, gd);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) gs[h][i] += gd[i];
-        st_lm16(own2, h, cg, row, gs[h]);
-      }
-      if (cg == 0) {
+      if (cq == 0) {
 #pragma unroll
         for (int h = 0; h < C::MH; ++h) {
           const int m = 128 * h + row;
@@ -988,15 +1044,19 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           __stcg(own2 + MF * 64 + m, gzs[h] + gdz);
         }
       }
-      chain_release(of2, n + 1);
+      group_bar(2);  // every slot write of the group is issued
+      if (gl == 0) st_release_gpu(of2, n + 1);
     }
-    float us = 0.f;
-    if (FEAT == SLIM_FEAT_EXP) {
-#pragma unroll
-      for (int g = 0; g < NG; ++g) us += redU[g * T + row];
-    }
-    TC_WAIT(sy);
+  join2:
+    __syncthreads();
     {
+      float us = 0.f;
+      if (FEAT == SLIM_FEAT_EXP) us = redU[row] + redU[T + row];
+      // the dq products were issued in every case: let them land
+      if (!mbar_wait(smem_u32(&mb[5]), 0, J.err)) abort_ = 1;
+      tc_fence_after();
+      __syncthreads();
+      if (abort_ | gfail[1]) goto teardown;
       float xq[16];
       ld_feat16(sQ, row, 16 * cg, xq);
       float v[16];
@@ -1272,12 +1332,12 @@ struct TileJobs {
 template <int MF, int FEAT>
 __global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ TileJobs J) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t mbar[5];
+  __shared__ __align__(8) uint64_t mbar[6];
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
   int b = blockIdx.x;
   if (b < J.n_q) {
-    role_bwd_q<MF, FEAT>(J.q, b, smem_raw, mbar[0], tmem_base, abort_);
+    role_bwd_q<MF, FEAT>(J.q, b, smem_raw, mbar, tmem_base, abort_);
     return;
   }
   b -= J.n_q;
@@ -1404,7 +1464,7 @@ constexpr size_t smem_fwd() {
   return 1024 + 2 * Cfg<MF>::FEATB + 3 * ROWT + Cfg<MF>::OMB + 8192 + 2 * T * 4 + 16;
 }
 template <int MF>
-constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4; }
+constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4 + 16; }
 template <int MF>
 constexpr size_t smem_max() {
   return smem_bwd<MF>() > smem_fwd<MF>() ? smem_bwd<MF>() : smem_fwd<MF>();
