@@ -58,6 +58,9 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--C", type=int, default=None)
+    # shape overrides, for profiling a smaller case of a workload (ncu captures)
+    ap.add_argument("--B", type=int, default=None)
+    ap.add_argument("--H", type=int, default=None)
     ap.add_argument("--sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -254,6 +257,26 @@ def oracle_pool_size():
     return max(1, min(len(os.sched_getaffinity(0)), 16))
 
 
+def _pool_warm(_):
+    """Imports what the oracle workers need, then holds the worker briefly so
+    that the other workers take the remaining items."""
+    os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
+    os.environ.setdefault("OMP_NUM_THREADS", "1")
+    import oracle  # noqa: F401
+    from paper_2012_11346_gb300 import workloads  # noqa: F401
+    time.sleep(0.2)
+    return os.getpid()
+
+
+def start_oracle_pool(n):
+    """A spawned pool whose workers have finished starting up and importing,
+    so that no worker start-up competes with the GPU timing for host cores."""
+    import multiprocessing as mp
+    pool = mp.get_context("spawn").Pool(n)
+    pool.map(_pool_warm, range(n), chunksize=1)
+    return pool
+
+
 def oracle_sample(w, overrides, pool, nchains):
     """Runs nchains chains of the workload through the oracle in parallel;
     returns (tokens, wall seconds)."""
@@ -269,17 +292,16 @@ def run_ours(args, rank, ws, local):
     from paper_2012_11346_gb300 import slim
     from paper_2012_11346_gb300 import workloads as W
 
-    # Oracle pool first (spawned before any GPU work).
-    pool = None
-    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        import multiprocessing as mp
-        pool = mp.get_context("spawn").Pool(oracle_pool_size())
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     w = W.WORKLOADS[args.workload]
     if args.C:
         w = w.with_(C=args.C)
+    if args.B:
+        w = w.with_(B=args.B)
+    if args.H:
+        w = w.with_(H=args.H)
     x = W.make_inputs(w, device=dev)
     q, k, v, om, dout = x["q"], x["k"], x["v"], x["omega"], x["dout"]
     B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
@@ -398,8 +420,13 @@ def run_ours(args, rank, ws, local):
         "kernels": [{k_: (round(v_, 4) if isinstance(v_, float) else v_) for k_, v_ in s.items()}
                     for s in stats],
     }
-    if pool is not None:
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        # The oracle pool starts only after every GPU measurement: with an
+        # idle pool alive during the GPU passes, the end-to-end pass was
+        # measured ~400x slower on a 16-core host.  Spawned workers do not
+        # inherit the parent's CUDA context.
         n = oracle_pool_size()
+        pool = start_oracle_pool(n)
         tok, sec = oracle_sample(w, {"C": w.C}, pool, n)
         line["cpu_baseline"] = {"value": round(tok / sec, 2), "unit": "tokens/s", "cores": n,
                                 "kind": "oracle",
@@ -426,6 +453,10 @@ def run_reference(args, rank, ws):
     w = W.WORKLOADS[args.workload]
     if args.C:
         w = w.with_(C=args.C)
+    if args.B:
+        w = w.with_(B=args.B)
+    if args.H:
+        w = w.with_(H=args.H)
     n = oracle_pool_size()
     with mp.get_context("spawn").Pool(n) as pool:
         for _ in range(args.warmup):
