@@ -342,6 +342,7 @@ def run_ours(args, rank, ws, local):
     barrier(ws)
     launches = slim.launch_count() - launches0
     clocks = sampler.stop()
+    slim.check_device_error(wsf)
     slim.check_device_error(wsb)
     ms = max_over_ranks(e0.elapsed_time(e1), ws)
     tokens = sum_over_ranks(B * L * args.steps, ws)
@@ -359,6 +360,17 @@ def run_ours(args, rank, ws, local):
     slim.profiler_enable(False)
     ms_profiled = e0.elapsed_time(e1)
     stats = slim.profiler_read()
+    # a bounded device wait that gave up would make the timings meaningless
+    slim.check_device_error(wsf)
+    slim.check_device_error(wsb)
+
+    # untimed validation pass: every call clears the device error word at its
+    # start, so check it after each step; a bounded wait that gave up during
+    # the measurement would make the numbers above meaningless
+    for _ in range(args.steps):
+        step()
+        slim.check_device_error(wsf)
+        slim.check_device_error(wsb)
 
     # end to end through the public API: pinned host inputs in, results out
     hq, hk, hv, hdo = (t.cpu().pin_memory() for t in (q, k, v, dout))

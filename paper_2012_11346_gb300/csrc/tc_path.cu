@@ -141,17 +141,23 @@ __device__ __forceinline__ void st_f32x16(float* dst, const float* v) {
   for (int i = 0; i < 4; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
 }
 
+// One single-use mbarrier per MMA commit, each waited on with parity 0.  A
+// barrier reused across commits would let a warp that reaches its wait after
+// two completions see the parity of a later, unfinished phase and wait for
+// it; with one barrier per event a late warp simply finds its phase done.
 struct Sync {
-  uint32_t mbar;
-  uint32_t phase;
+  uint64_t* mb;
+  int next;  // barrier of the next wait()
   int* err;
+  __device__ uint32_t bar(int i) const { return smem_u32(&mb[i]); }
   __device__ bool wait() {
-    const bool ok = mbar_wait(mbar, phase, err);
-    phase ^= 1u;
+    const bool ok = mbar_wait(smem_u32(&mb[next]), 0, err);
+    ++next;
     tc_fence_after();
     return ok;
   }
 };
+constexpr int NBAR = 6;  // mbarriers per tile CTA
 
 // Make generic-proxy smem writes visible to the tensor core and order them
 // with the thread that issues the next MMAs.
@@ -181,7 +187,7 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   (void)cg;                                             \
   if (tid == 0) {                                       \
     abort_ = 0;                                         \
-    mbar_init(smem_u32(&mbar), 1);                      \
+    for (int i_ = 0; i_ < NBAR; ++i_) mbar_init(smem_u32(&mb[i_]), 1); \
     mbar_fence_init();                                  \
   }                                                     \
   if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512)
@@ -331,6 +337,7 @@ struct FwdJob {
   int L, Cs, N, nt, P, chains;  // slice length, slices, tiles of a full slice, tile positions
   float* slot;                  // [chains][nt][E] inclusive prefixes
   int* flag;                    // [chains][nt], FLAG_STRIDE ints apart
+  int* ticket;                  // tile counter of this launch (starts at 0)
   __nv_bfloat16* out;
   StateOut st;                  // B^(N), written by the last tile of each chain
   int* err;
@@ -616,6 +623,7 @@ struct BwdQJob {
   int L, a, b, ntn, n, N, nt, chains;  // slice n = rows [a, a+b), ntn tiles; nt: full slice
   float *slot1, *slot2;   // [chains][nt][E]: state prefixes, state-gradient prefixes
   int *flag1, *flag2;     // [chains][nt], FLAG_STRIDE ints apart
+  int* ticket;            // tile counter of this launch (starts at 0)
   __nv_bfloat16* gS;      // [chains][ntn][MF][64] G_t(S) for the dk/dv side
   float* gz;              // [chains][ntn][MF]     g_t(z)
   float *rowstat, *part;  // [chains][ntn][T][2] (den, dden), [chains][ntn][MF][64]
@@ -1087,7 +1095,7 @@ struct BwdKVJob {
 
 template <int MF, int FEAT>
 __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uint8_t* smem_raw,
-                                            uint64_t& mbar, uint32_t& tmem_base, int& abort_) {
+                                            uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;               // later: u
@@ -1150,7 +1158,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    Sync sy{smem_u32(&mbar), 0u, J.err};
+    Sync sy{mb, 0, J.err};
     if (tid == 0) {
       // two commits: the phiQ epilogue runs while the K projection is computed
       const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
@@ -1159,12 +1167,12 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
-      mma_commit(sy.mbar);
+      mma_commit(sy.bar(0));
       for (int k0 = 0; k0 < D; k0 += 16) {
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
         mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
       }
-      mma_commit(sy.mbar);
+      mma_commit(sy.bar(1));
     }
     TC_WAIT(sy);  // Q projection done
     feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
@@ -1179,7 +1187,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
         mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
       for (int k0 = 0; k0 < D; k0 += 16)  // dnum V^T
         mma(tmem + 128, kmaj(aDn, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
-      mma_commit(sy.mbar);
+      mma_commit(sy.bar(2));
     }
     TC_WAIT(sy);
     {  // A -> smem (masked, bf16), this thread's 32 columns
@@ -1205,7 +1213,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
         mma(tmem, kmaj(aPK, T, k0), mnmaj(aG, k0, C::OMB), idesc_bf16(T, 64, 0, 1), 1);
       for (int k0 = 0; k0 < D; k0 += 16)  // dphiK = V G_t(S)^T
         mma(tmem + 256, kmaj(aV, T, k0), kmaj(aG, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-      mma_commit(sy.mbar);
+      mma_commit(sy.bar(3));
     }
     TC_WAIT(sy);
     {
@@ -1233,7 +1241,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       const uint32_t adA = smem_u32(sA), aPQ = smem_u32(sPhiQ);
       for (int k0 = 0; k0 < T; k0 += 16)  // dphiK += dA^T phiQ
         mma(tmem + 256, mnmaj(adA, k0, ROWT), mnmaj(aPQ, k0, ROWT), idesc_bf16(T, MF, 1, 1), 1);
-      mma_commit(sy.mbar);
+      mma_commit(sy.bar(4));
     }
     TC_WAIT(sy);
     // K and Omega again (dk = u Omega - k sum(u), dOmega += u^T k), overlapping the epilogue
@@ -1287,7 +1295,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
         for (int k0 = 0; k0 < T; k0 += 16)
           mma(tmem + 64 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aK, k0, ROWT),
               idesc_bf16(T, 64, 1, 1), k0 > 0);
-      mma_commit(sy.mbar);
+      mma_commit(sy.bar(5));
     }
     float us = 0.f;
     if (FEAT == SLIM_FEAT_EXP) {
@@ -1303,14 +1311,10 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xk[i], v[i]);
       if (rv) st_row16(J.dk + g0 + (size_t)row * D + 16 * cg, v);
-      float* dst = J.part + ti * (size_t)(MF * 64);
+      float* dst = J.part + ti * (size_t)(MF * 64);  // this side's own partial
       for (int h = 0; h < C::MH; ++h) {
-        float w[16];
-        ld_lm16(dst, h, cg, row, w);  // the dq side's partial of this tile
         tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) w[i] += v[i];
-        st_lm16(dst, h, cg, row, w);
+        st_lm16(dst, h, cg, row, v);
       }
     }
   }
@@ -1318,80 +1322,138 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
 }
 
 // ================================================================== launches
-// One launch runs tiles of up to three roles.  The chained roles (dq side,
-// forward) come first so their chains start early; the independent dk/dv
-// tiles follow and fill the launch's tail.  Inside a role every tile waits
-// only on tiles with lower block indices.
+// dOmega reduction of one slice's per-tile partials (both sides, lane-major),
+// in two stages with fixed ranges and orders, so dOmega is reproducible:
+//   stage 1, CTA r < RS1: sums[r] = partials [r*per, (r+1)*per) summed in order
+//   stage 2, CTA s < RS2: dOmega += sums[0] + ... + sums[RS1-1] over one
+//            RS2-th of the elements (another slice's sums)
+constexpr int RS1 = 128, RS2 = 16;
+struct RedJob {
+  const float* part;  // stage 1: [nparts][M*64] lane-major partials
+  int nparts;
+  float* sums;        // stage 1 out: [RS1][M*64]
+  const float* sums2; // stage 2 in: [RS1][M*64]
+  float* domega;      // [M][64], accumulated into
+  int n;              // M * 64
+};
+
+__device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
+  const int per = (J.nparts + RS1 - 1) / RS1;
+  const int i0 = min(J.nparts, r * per), i1 = min(J.nparts, i0 + per);
+  const int n4 = J.n / 4, tid = threadIdx.x;
+  constexpr int QMAX = 256 * 64 / 4 / NTHR;  // float4 per thread at M = 256
+  float4 acc[QMAX];
+#pragma unroll
+  for (int k = 0; k < QMAX; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i = i0; i < i1; ++i) {
+    const float4* src = reinterpret_cast<const float4*>(J.part + (size_t)i * J.n);
+#pragma unroll
+    for (int k = 0; k < QMAX; ++k) {
+      const int q = tid + k * NTHR;
+      if (q < n4) {
+        const float4 x = __ldcg(src + q);
+        acc[k].x += x.x;
+        acc[k].y += x.y;
+        acc[k].z += x.z;
+        acc[k].w += x.w;
+      }
+    }
+  }
+  float4* dst = reinterpret_cast<float4*>(J.sums + (size_t)r * J.n);
+#pragma unroll
+  for (int k = 0; k < QMAX; ++k) {
+    const int q = tid + k * NTHR;
+    if (q < n4) dst[q] = acc[k];
+  }
+}
+
+__device__ __forceinline__ void reduce_stage2(const RedJob& J, int s) {
+  const int n4 = J.n / 4, share = (n4 + RS2 - 1) / RS2;
+  const int q1 = min(n4, (s + 1) * share);
+  for (int q = s * share + (int)threadIdx.x; q < q1; q += NTHR) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r = 0; r < RS1; ++r) {
+      const float4 x = __ldcg(reinterpret_cast<const float4*>(J.sums2 + (size_t)r * J.n) + q);
+      acc.x += x.x;
+      acc.y += x.y;
+      acc.z += x.z;
+      acc.w += x.w;
+    }
+    // lane-major float4 q holds row 128h + row, columns 16cg + 4i .. +3
+    const int row = q & 127, rest = q >> 7, i = rest & 3;
+    const int cg = (rest >> 2) % NG, h = rest / (4 * NG);
+    float* o = J.domega + (128 * h + row) * 64 + 16 * cg + 4 * i;
+    o[0] += acc.x;
+    o[1] += acc.y;
+    o[2] += acc.z;
+    o[3] += acc.w;
+  }
+}
+
+// One launch runs tiles of up to three roles, then the dOmega reduction of
+// earlier slices.  The chained roles (dq side, forward) come first so their
+// chains start early; the independent dk/dv tiles follow, and the reduction
+// CTAs fill the launch's tail.  Inside a role every tile waits only on tiles
+// with lower block indices.
 struct TileJobs {
-  int n_q, n_fwd, n_kv;  // CTAs of each role, in dispatch order
+  int n_q, n_fwd, n_kv, n_red1, n_red2;  // CTAs of each role, in dispatch order
   BwdQJob q;
   FwdJob f;
   BwdKVJob kv;
+  RedJob red;
 };
 
 template <int MF, int FEAT>
 __global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ TileJobs J) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t mbar[6];
+  __shared__ __align__(8) uint64_t mbar[NBAR];
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
+  __shared__ int ticket;
+  // A chained tile waits only on tiles earlier in its chain.  The chained
+  // roles take their tile from a counter rather than from blockIdx: the
+  // tiles handed out so far always belong to CTAs that are running, so every
+  // awaited tile is in progress whatever order the CTAs are dispatched in.
+  // (The counter is zeroed by the call's memset, long before this launch.)
   int b = blockIdx.x;
   if (b < J.n_q) {
-    role_bwd_q<MF, FEAT>(J.q, b, smem_raw, mbar, tmem_base, abort_);
+    if (threadIdx.x == 0) ticket = atomicAdd(J.q.ticket, 1);
+    __syncthreads();
+    role_bwd_q<MF, FEAT>(J.q, ticket, smem_raw, mbar, tmem_base, abort_);
     return;
   }
   b -= J.n_q;
   if (b < J.n_fwd) {
-    role_fwd<MF, FEAT>(J.f, b / J.f.chains, b % J.f.chains, smem_raw, mbar, tmem_base, abort_);
+    if (threadIdx.x == 0) ticket = atomicAdd(J.f.ticket, 1);
+    __syncthreads();
+    role_fwd<MF, FEAT>(J.f, ticket / J.f.chains, ticket % J.f.chains, smem_raw, mbar, tmem_base,
+                       abort_);
     return;
   }
   b -= J.n_fwd;
-  if (b < J.n_kv)
-    role_bwd_kv<MF, FEAT>(J.kv, b % J.kv.nt, b / J.kv.nt, smem_raw, mbar[0], tmem_base, abort_);
-}
-
-// dOmega reduction of one slice's per-tile partials (lane-major), in two
-// stages that run in the small launches between tile launches:
-//   stage 1: sums[split][e] = sum of the partials of one fixed range
-//   stage 2: domega[e] += sum over the RSPLIT sums, in order
-constexpr int RSPLIT = 64;
-struct ReduceJobs {
-  const float* r1_part;
-  float* r1_sums;
-  int r1_nparts, r1_bx;
-  const float* r2_sums;
-  float* r2_domega;
-  int r2_blocks;
-  int n;  // M * 64
-};
-
-__global__ void __launch_bounds__(256) k_tc_reduce(const __grid_constant__ ReduceJobs J) {
-  grid_dependency_wait();
-  int b = blockIdx.x;
-  if (b < J.r1_bx * RSPLIT) {
-    const int e = (b % J.r1_bx) * 256 + threadIdx.x, split = b / J.r1_bx;
-    if (e >= J.n) return;
-    const int per = (J.r1_nparts + RSPLIT - 1) / RSPLIT;
-    const int i0 = split * per, i1 = min(J.r1_nparts, i0 + per);
-    float s = 0.f;
-#pragma unroll 4
-    for (int i = i0; i < i1; ++i) s += J.r1_part[(size_t)i * J.n + e];
-    J.r1_sums[(size_t)split * J.n + e] = s;
+  if (b < J.n_kv) {
+    role_bwd_kv<MF, FEAT>(J.kv, b % J.kv.nt, b / J.kv.nt, smem_raw, mbar, tmem_base, abort_);
     return;
   }
-  b -= J.r1_bx * RSPLIT;
-  if (b < J.r2_blocks) {
-    const int e = b * 256 + threadIdx.x;
-    if (e >= J.n) return;
-    float s = 0.f;
-#pragma unroll
-    for (int i = 0; i < RSPLIT; ++i) s += J.r2_sums[(size_t)i * J.n + e];
-    // e is a lane-major index: float4 q = e / 4 holds row 128h + row,
-    // columns 16cg + 4i .. +3
-    const int q = e >> 2, row = q & 127, rest = q >> 7, i = rest & 3;
-    const int cg = (rest >> 2) % NG, h = rest / (4 * NG);
-    J.r2_domega[(128 * h + row) * 64 + 16 * cg + 4 * i + (e & 3)] += s;
+  b -= J.n_kv;
+  grid_dependency_wait();  // partials and sums of earlier launches
+  if (b < J.n_red1) {
+    reduce_stage1(J.red, b);
+    return;
   }
+  b -= J.n_red1;
+  if (b < J.n_red2) reduce_stage2(J.red, b);
+}
+
+// The reduction stages that have no tile launch left to ride in.
+__global__ void __launch_bounds__(NTHR) k_tc_reduce(const __grid_constant__ RedJob J, int n_red1,
+                                                    int n_red2) {
+  grid_dependency_wait();
+  const int b = blockIdx.x;
+  if (b < n_red1)
+    reduce_stage1(J, b);
+  else if (b - n_red1 < n_red2)
+    reduce_stage2(J, b - n_red1);
 }
 
 // ================================================================== small kernels
@@ -1429,13 +1491,17 @@ Geo geometry(const Problem& p) {
 // tiles overwrite the previous slice's only after reading them.  The buffers
 // the dq side hands to the dk/dv side have two slots (slice n uses n % 2),
 // because the dq side of slice n-1 runs beside the dk/dv side of slice n.
+// The dOmega partials of slice n are reduced in the launch after its dk/dv
+// side, beside the dq side of slice n-2: they take three slots.
 struct Ws {
   int* err;
-  int* flags;  // [2][chains][nt], FLAG_STRIDE ints each
+  int* flags;    // [2][chains][nt], FLAG_STRIDE ints each
+  int* tickets;  // one tile counter per launch of the call
   __nv_bfloat16* om16;
   float *slot1, *slot2;
   __nv_bfloat16* gS[2];
-  float *gz[2], *rowstat[2], *part[2], *rsums[2];
+  float *gz[2], *rowstat[2], *rsums[2];
+  float* part[3];  // [2 sides][chains][nt][M*64]; slice n uses n % 3
 };
 
 Ws carve(Carver& cv, const Geo& g, bool bwd) {
@@ -1443,6 +1509,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   const size_t C = g.chains, tiles = C * g.nt;
   w.err = cv.take<int>(64);
   w.flags = cv.take<int>(2 * tiles * FLAG_STRIDE);
+  w.tickets = cv.take<int>((size_t)g.N + 3);
   w.om16 = cv.take<__nv_bfloat16>((size_t)2 * g.MF * D);
   w.slot1 = cv.take<float>(tiles * g.E);
   if (bwd) {
@@ -1451,9 +1518,9 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
       w.gS[k] = cv.take<__nv_bfloat16>(tiles * g.MF * D);
       w.gz[k] = cv.take<float>(tiles * g.MF);
       w.rowstat[k] = cv.take<float>(tiles * T * 2);
-      w.part[k] = cv.take<float>(tiles * (size_t)g.MF * D);
-      w.rsums[k] = cv.take<float>((size_t)RSPLIT * g.MF * D);
+      w.rsums[k] = cv.take<float>((size_t)RS1 * g.MF * D);
     }
+    for (int k = 0; k < 3; ++k) w.part[k] = cv.take<float>(2 * tiles * (size_t)g.MF * D);
   }
   return w;
 }
@@ -1525,24 +1592,24 @@ Slice slice_of(const Problem& p, const Geo& g, int n) {
 template <int MF, int FEAT>
 cudaError_t launch_tiles(cudaStream_t s, const TileJobs& J, double flops, double bytes,
                          prof::Kid kid) {
-  const int n = J.n_kv + J.n_q + J.n_fwd;
+  const int n = J.n_kv + J.n_q + J.n_fwd + J.n_red1 + J.n_red2;
   if (n == 0) return cudaSuccess;
   const size_t smem = (J.n_kv || J.n_q) ? smem_bwd<MF>() : smem_fwd<MF>();
   prof::Scope ps(kid, s, flops, bytes);
   return launch_dep(k_tc_tiles<MF, FEAT>, dim3(n), dim3(NTHR), smem, s, J);
 }
 
-cudaError_t launch_reduce(cudaStream_t s, const ReduceJobs& J) {
-  const int blocks = J.r1_bx * RSPLIT + J.r2_blocks;
-  if (blocks == 0) return cudaSuccess;
+cudaError_t launch_reduce(cudaStream_t s, const RedJob& J, int n_red1, int n_red2) {
+  if (n_red1 + n_red2 == 0) return cudaSuccess;
   prof::Scope ps(prof::K_TC_REDUCE, s);
-  return launch_dep(k_tc_reduce, dim3(blocks), dim3(256), 0, s, J);
+  return launch_dep(k_tc_reduce, dim3(n_red1 + n_red2), dim3(NTHR), 0, s, J, n_red1, n_red2);
 }
 
 cudaError_t prepare(const Ws& w, const Geo& g, const float* omega, cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(w.flags, 0, (size_t)2 * g.chains * g.nt * FLAG_STRIDE * sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w.tickets, 0, ((size_t)g.N + 3) * sizeof(int), s);
   if (e != cudaSuccess) return e;
   prof::Scope ps(prof::K_TC_PREP, s);
   k_omega_bf16<<<nblk(g.MF * D), 256, 0, s>>>(omega, w.om16, g.MF * D);  // hi and lo
@@ -1562,7 +1629,8 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // a tile position.  Algorithmic work per row: 8dM (phiQ, phiK, Delta, readout).
   TileJobs J{};
   const int P = (g.N - 1) * g.nt + slice_of(p, g, g.N - 1).nt;
-  J.f = FwdJob{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flags, out, st, w.err};
+  J.f = FwdJob{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flags, w.tickets,
+               out, st, w.err};
   J.n_fwd = P * g.chains;
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
   TC_TRY((launch_tiles<MF, FEAT>(s, J, rows * 8.0 * MD, rows * D * 2.0 * 4, prof::K_TC_FWD)));
@@ -1583,54 +1651,55 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   TC_TRY(cudaMemsetAsync(domega, 0, (size_t)MF * D * sizeof(float), s));
   TC_TRY(prepare(w, g, omega, s));
   const double MD = (double)MF * D;
-  const unsigned r_bx = nblk(MF * D);
+  const size_t MD64 = (size_t)MF * D;
   int* flag1 = w.flags;
   int* flag2 = w.flags + (size_t)g.chains * g.nt * FLAG_STRIDE;
   auto valid = [&](int n) { return n >= 0 && n < N; };
+  auto tiles_of = [&](int n) { return (size_t)g.chains * slice_of(p, g, n).nt; };
   // Stage j of the reverse walk:
-  //   tiles j  : dk/dv side of slice N-j, dq side of slice N-1-j
-  //   reduce j : dOmega stage 1 of slice N-j, stage 2 of slice N+1-j
+  //   dq side of slice N-1-j, dk/dv side of slice N-j, dOmega stage 1 of
+  //   slice N+1-j and stage 2 of slice N+2-j.
   // Algorithmic work per row: dq side 14dM (phiQ, phiK, rollback Delta, dphiQ,
   // G, dq, dOmega), dk/dv side 8dM (dV, dphiK, dk, dOmega).
-  for (int j = 0; j <= N + 1; ++j) {
+  for (int j = 0; j <= N + 2; ++j) {
     TileJobs J{};
     double fl = 0.0, by = 0.0;
-    const int nkv = N - j, nq = N - 1 - j;
-    if (j >= 1 && valid(nkv)) {
-      const Slice sl = slice_of(p, g, nkv);
-      const int x = nkv & 1;
-      J.kv = BwdKVJob{q, k, v, dout, w.om16, w.gS[x], w.gz[x], w.rowstat[x], p.L, sl.a, sl.b,
-                      sl.nt, dk, dv, w.part[x], w.err};
-      J.n_kv = sl.nt * g.chains;
-      fl += (double)g.chains * sl.b * 8.0 * MD;
-      by += (double)g.chains * sl.b * D * 2.0 * 6;
-    }
+    const int nq = N - 1 - j, nkv = N - j, nr1 = N + 1 - j, nr2 = N + 2 - j;
     if (valid(nq)) {
       const Slice sl = slice_of(p, g, nq);
       const int x = nq & 1;
       J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, sl.a, sl.b, sl.nt, nq, N, g.nt,
-                    g.chains, w.slot1, w.slot2, flag1, flag2, w.gS[x], w.gz[x], w.rowstat[x],
-                    w.part[x], dq, w.err};
+                    g.chains, w.slot1, w.slot2, flag1, flag2, w.tickets + j, w.gS[x], w.gz[x],
+                    w.rowstat[x], w.part[nq % 3], dq, w.err};
       J.n_q = sl.nt * g.chains;
       fl += (double)g.chains * sl.b * 14.0 * MD;
       by += (double)g.chains * sl.b * D * 2.0 * 6;
     }
-    TC_TRY((launch_tiles<MF, FEAT>(s, J, fl, by, prof::K_TC_BWD)));
-    ReduceJobs R{};
-    R.n = MF * D;
-    const int nx1 = N - j, nx2 = N + 1 - j;
-    if (j >= 1 && valid(nx1)) {
-      R.r1_part = w.part[nx1 & 1];
-      R.r1_sums = w.rsums[nx1 & 1];
-      R.r1_nparts = g.chains * slice_of(p, g, nx1).nt;
-      R.r1_bx = (int)r_bx;
+    if (j >= 1 && valid(nkv)) {
+      const Slice sl = slice_of(p, g, nkv);
+      const int x = nkv & 1;
+      J.kv = BwdKVJob{q, k, v, dout, w.om16, w.gS[x], w.gz[x], w.rowstat[x], p.L, sl.a, sl.b,
+                      sl.nt, dk, dv, w.part[nkv % 3] + tiles_of(nkv) * MD64, w.err};
+      J.n_kv = sl.nt * g.chains;
+      fl += (double)g.chains * sl.b * 8.0 * MD;
+      by += (double)g.chains * sl.b * D * 2.0 * 6;
     }
-    if (j >= 2 && valid(nx2)) {
-      R.r2_sums = w.rsums[nx2 & 1];
-      R.r2_domega = domega;
-      R.r2_blocks = (int)r_bx;
+    J.red.n = MF * D;
+    if (j >= 2 && valid(nr1)) {
+      J.red.part = w.part[nr1 % 3];
+      J.red.nparts = (int)(2 * tiles_of(nr1));
+      J.red.sums = w.rsums[nr1 & 1];
+      J.n_red1 = RS1;
     }
-    TC_TRY(launch_reduce(s, R));
+    if (j >= 3 && valid(nr2)) {
+      J.red.sums2 = w.rsums[nr2 & 1];
+      J.red.domega = domega;
+      J.n_red2 = RS2;
+    }
+    if (J.n_q + J.n_kv > 0)
+      TC_TRY((launch_tiles<MF, FEAT>(s, J, fl, by, prof::K_TC_BWD)));
+    else
+      TC_TRY(launch_reduce(s, J.red, J.n_red1, J.n_red2));
   }
   return SLIM_OK;
 }
