@@ -27,6 +27,8 @@ CASES = [
     (128, 640, 512, "exp"),
     (128, 300, 64, "relu"),      # 64-row slices (half-filled tiles)
     (256, 513, 4096, "exp"),     # C > L
+    (256, 1000, 200, "exp"),     # slices of 128 + 72 rows: a ragged tile in every slice
+    (128, 700, 320, "relu"),     # 3-tile slices (128 + 128 + 64), ragged last slice
 ]
 
 
@@ -52,3 +54,46 @@ def test_tc_matches_fp32_path(cuda_device, monkeypatch):
     import oracle
     for n in ("out", "S_state", "z_state", "dq", "dk", "dv", "domega"):
         assert oracle.rel_l2(to64(a[n]), to64(b[n])) <= TOL["bf16"], n
+
+
+def _run_case(cuda_device, B, H, L, C, seed=3):
+    w = W.Workload("tc", B, H, L, 64, 256, C, "bf16", "exp", "normal", "orthogonal", seed=seed)
+    assert slim.path_for(B, H, L, 64, 256, C, torch.bfloat16, "exp") == 1
+    x = W.make_inputs(w, device=cuda_device)
+    compare(gpu_run(x, C, "exp"), oracle_run(cpu_inputs(x), C, "exp"), TOL["bf16"],
+            where=f"tc B{B} H{H} L{L} C{C}")
+
+
+def test_tc_single_long_chain(cuda_device):
+    """One chain of 64 tiles (8 slices of 8): every prefix is handed along a
+    single chain, in the forward and in both backward chains."""
+    _run_case(cuda_device, 1, 1, 8192, 1024)
+
+
+def test_tc_many_short_chains(cuda_device):
+    """256 chains of 2 tiles, one tile per slice: hand-offs across slice
+    boundaries only."""
+    _run_case(cuda_device, 16, 16, 256, 128)
+
+
+def test_tc_workspace_reuse(cuda_device):
+    """Back-to-back calls on one workspace give identical results: the chain
+    flags and tile counters start afresh in every call."""
+    w = W.Workload("tc", 2, 4, 1536, 64, 256, 512, "bf16", "exp", "normal", "orthogonal", seed=9)
+    x = W.make_inputs(w, device=cuda_device)
+    q, k, v, om, dout = x["q"], x["k"], x["v"], x["omega"], x["dout"]
+    B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
+    wsf = torch.empty(slim.workspace_size(B, H, L, d, M, w.C, q.dtype, "exp", False),
+                      dtype=torch.uint8, device=cuda_device)
+    wsb = torch.empty(slim.workspace_size(B, H, L, d, M, w.C, q.dtype, "exp", True),
+                      dtype=torch.uint8, device=cuda_device)
+    runs = []
+    for _ in range(3):
+        out, S, z = slim.forward(q, k, v, om, w.C, "exp", workspace=wsf)
+        g = slim.backward(q, k, v, om, out, dout, S, z, w.C, "exp", workspace=wsb)
+        torch.cuda.synchronize()
+        slim.check_device_error(wsf)
+        slim.check_device_error(wsb)
+        runs.append([out, S, z, *g])
+    for a, b in zip(runs[0], runs[2]):
+        assert torch.equal(a, b)
