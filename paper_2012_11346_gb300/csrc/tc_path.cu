@@ -157,7 +157,7 @@ struct Sync {
     return ok;
   }
 };
-constexpr int NBAR = 6;  // mbarriers per tile CTA
+constexpr int NBAR = 9;  // mbarriers per tile CTA
 
 // Make generic-proxy smem writes visible to the tensor core and order them
 // with the thread that issues the next MMAs.
@@ -409,7 +409,7 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
   const int cg = warp >> 2;
   if (tid == 0) {
     abort_ = 0;
-    for (int i = 0; i < 5; ++i) mbar_init(smem_u32(&mb[i]), 1);
+    for (int i = 0; i < NBAR; ++i) mbar_init(smem_u32(&mb[i]), 1);
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
@@ -457,15 +457,17 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     if (abort_) goto teardown;
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
-    if (tid == 0) {
+    if (tid == 0 || (C::MH > 1 && tid == 32)) {
+      // Delta_t = phiK^T [V | 1], one feature half per issuing thread: two
+      // issuers keep the tensor pipe fed with these narrow products
+      const int h = tid == 0 ? 0 : 1;
       const uint32_t aPK = smem_u32(sPhiK), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
-      for (int h = 0; h < C::MH; ++h)  // Delta_t = phiK^T [V | 1]
-        for (int k0 = 0; k0 < T; k0 += 16) {
-          const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
-          mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
-          mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
-        }
-      mma_commit(smem_u32(&mb[2]));
+      for (int k0 = 0; k0 < T; k0 += 16) {
+        const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
+        mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+        mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
+      }
+      mma_commit(smem_u32(&mb[h == 0 ? 2 : 5]));
     }
     if (warp < 8) {
       // ---- compute group: g(Q), A = tril(g(Q) g(K)^T), A's bf16 tile and row sums
@@ -511,6 +513,7 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
       // (row, cg) handles column groups 2(cg-2) and 2(cg-2)+1.
       const int gl = tid - GRP;  // 0..255
       if (!mbar_wait(smem_u32(&mb[2]), 0, J.err)) gfail[1] = 1;
+      if (C::MH > 1 && !mbar_wait(smem_u32(&mb[5]), 0, J.err)) gfail[1] = 1;
       tc_fence_after();
       if (pred && gl == 0 && !gfail[1] && !flag_poll(pflag, pwant, J.err)) gfail[1] = 1;
       group_bar(2);
@@ -584,19 +587,23 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     if (gfail[0] | gfail[1]) goto teardown;
     publish();
     if (tid == 0) {
-      const uint32_t aPQ = smem_u32(sPhiQ), aS = smem_u32(sS), aZ = smem_u32(sZt);
+      const uint32_t aPQ = smem_u32(sPhiQ), aS = smem_u32(sS);
       const uint32_t aA = smem_u32(sA), aV = smem_u32(sV);
-      for (int k0 = 0; k0 < MF; k0 += 16) {
-        // num = phiQ S_t;  phiQ [z_hi | z_lo]
+      for (int k0 = 0; k0 < MF; k0 += 16)  // num = phiQ S_t
         mma(tmem + 128, kmaj(aPQ, T, k0), mnmaj(aS, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
-        mma(tmem + 192, kmaj(aPQ, T, k0), kmaj(aZ, 16, k0), idesc_bf16(T, 16, 0, 0), k0 > 0);
-      }
       for (int k0 = 0; k0 < T; k0 += 16)  // num += A V
         mma(tmem + 128, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), 1);
       mma_commit(smem_u32(&mb[4]));
+    } else if (tid == 32) {
+      // phiQ [z_hi | z_lo], from a second issuing thread
+      const uint32_t aPQ = smem_u32(sPhiQ), aZ = smem_u32(sZt);
+      for (int k0 = 0; k0 < MF; k0 += 16)
+        mma(tmem + 192, kmaj(aPQ, T, k0), kmaj(aZ, 16, k0), idesc_bf16(T, 16, 0, 0), k0 > 0);
+      mma_commit(smem_u32(&mb[6]));
     }
     const float rsA = redA[row] + redA[T + row];
     if (!mbar_wait(smem_u32(&mb[4]), 0, J.err)) abort_ = 1;
+    if (!mbar_wait(smem_u32(&mb[6]), 0, J.err)) abort_ = 1;
     tc_fence_after();
     __syncthreads();
     if (abort_) goto teardown;
@@ -696,7 +703,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   const int cq = 2 * (cg - 2);  // chain group: column groups cq, cq + 1
   if (tid == 0) {
     abort_ = 0;
-    for (int i = 0; i < 6; ++i) mbar_init(smem_u32(&mb[i]), 1);
+    for (int i = 0; i < NBAR; ++i) mbar_init(smem_u32(&mb[i]), 1);
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
@@ -766,15 +773,16 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     fill_ones(sOnes, tid);  // the K tile is no longer read
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
-    if (tid == 0) {
+    if (tid == 0 || (C::MH > 1 && tid == 32)) {
+      // Delta_t = phiK^T [V | 1], one feature half per issuing thread
+      const int h = tid == 0 ? 0 : 1;
       const uint32_t aPK = smem_u32(sPhiK), aV = smem_u32(sV), aOnes = smem_u32(sOnes);
-      for (int h = 0; h < C::MH; ++h)  // Delta_t = phiK^T [V | 1]
-        for (int k0 = 0; k0 < T; k0 += 16) {
-          const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
-          mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
-          mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
-        }
-      mma_commit(smem_u32(&mb[2]));
+      for (int k0 = 0; k0 < T; k0 += 16) {
+        const uint64_t ad = mnmaj(aPK + h * 2 * ROWT, k0, ROWT);
+        mma(tmem + 256 + 64 * h, ad, mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
+        mma(tmem + 384 + 16 * h, ad, kmaj(aOnes, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
+      }
+      mma_commit(smem_u32(&mb[h == 0 ? 2 : 6]));
     }
     if (warp < 8) {
       // ---- compute group: g(Q), then A and dout V^T, and A's row sums
@@ -816,6 +824,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       // ---- chain group, rollback (eq. 17 per tile): the state before this
       // tile is the state after it minus Delta_t
       if (!mbar_wait(smem_u32(&mb[2]), 0, J.err)) gfail[1] = 1;
+      if (C::MH > 1 && !mbar_wait(smem_u32(&mb[6]), 0, J.err)) gfail[1] = 1;
       tc_fence_after();
       if (linked && gl == 0 && !gfail[1] && !flag_poll(f1, wnext, J.err)) gfail[1] = 1;
       group_bar(2);
@@ -940,20 +949,25 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     publish();
     if (tid == 0) {
       const uint32_t aDn = smem_u32(sDo), aS = smem_u32(sS), adA = smem_u32(sdA);
-      const uint32_t aPK = smem_u32(sPhiK), aPQ = smem_u32(sPhiQ), aDd = smem_u32(sDd);
+      const uint32_t aPK = smem_u32(sPhiK);
       for (int k0 = 0; k0 < D; k0 += 16)  // dnum S_t^T
         mma(tmem + 256, kmaj(aDn, T, k0), kmaj(aS, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
       for (int k0 = 0; k0 < T; k0 += 16)  // + dA phiK
         mma(tmem + 256, kmaj(adA, T, k0), mnmaj(aPK, k0, ROWT), idesc_bf16(T, MF, 0, 1), 1);
+      mma_commit(smem_u32(&mb[4]));
+    } else if (tid == 32) {
+      // Gd = phiQ^T [dnum | dden], from a second issuing thread
+      const uint32_t aDn = smem_u32(sDo), aPQ = smem_u32(sPhiQ), aDd = smem_u32(sDd);
       for (int h = 0; h < C::MH; ++h)
-        for (int k0 = 0; k0 < T; k0 += 16) {  // Gd = phiQ^T [dnum | dden]
+        for (int k0 = 0; k0 < T; k0 += 16) {
           const uint64_t ad = mnmaj(aPQ + h * 2 * ROWT, k0, ROWT);
           mma(tmem + 64 * h, ad, mnmaj(aDn, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
           mma(tmem + 128 + 16 * h, ad, kmaj(aDd, 16, k0), idesc_bf16(T, 16, 1, 0), k0 > 0);
         }
-      mma_commit(smem_u32(&mb[4]));
+      mma_commit(smem_u32(&mb[7]));
     }
     if (!mbar_wait(smem_u32(&mb[4]), 0, J.err)) abort_ = 1;
+    if (!mbar_wait(smem_u32(&mb[7]), 0, J.err)) abort_ = 1;
     tc_fence_after();
     __syncthreads();
     if (abort_) goto teardown;
@@ -998,17 +1012,20 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       redU[cg * T + row] = usum;
       cp_async_wait_all();
       group_publish(1);
+      // dq and the dOmega partial go to the columns dphiQ held, so Gd stays
+      // readable for the chain group; one issuing thread each
       if (tid == 0) {
-        // dq and the dOmega partial go to the columns dphiQ held, so Gd stays
-        // readable for the chain group
-        const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aQ = smem_u32(sQ);
+        const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm);
         for (int k0 = 0; k0 < MF; k0 += 16)
           mma(tmem + 256, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+        mma_commit(smem_u32(&mb[5]));
+      } else if (tid == 32) {
+        const uint32_t aU = smem_u32(sU), aQ = smem_u32(sQ);
         for (int h = 0; h < C::MH; ++h)
           for (int k0 = 0; k0 < T; k0 += 16)
             mma(tmem + 320 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aQ, k0, ROWT),
                 idesc_bf16(T, 64, 1, 1), k0 > 0);
-        mma_commit(smem_u32(&mb[5]));
+        mma_commit(smem_u32(&mb[8]));
       }
     } else {
       // ---- chain group, state gradient (eq. 18): G_t = the prefix after this
@@ -1062,6 +1079,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       if (FEAT == SLIM_FEAT_EXP) us = redU[row] + redU[T + row];
       // the dq products were issued in every case: let them land
       if (!mbar_wait(smem_u32(&mb[5]), 0, J.err)) abort_ = 1;
+      if (!mbar_wait(smem_u32(&mb[8]), 0, J.err)) abort_ = 1;
       tc_fence_after();
       __syncthreads();
       if (abort_ | gfail[1]) goto teardown;
@@ -1206,15 +1224,20 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     publish();
     if (tid == 0) {
       const uint32_t aA = smem_u32(sA), aDn = smem_u32(sDn), aPK = smem_u32(sPhiK);
-      const uint32_t aG = smem_u32(sG), aV = smem_u32(sV);
+      const uint32_t aG = smem_u32(sG);
       for (int k0 = 0; k0 < T; k0 += 16)  // dV = A^T dnum
         mma(tmem, mnmaj(aA, k0, ROWT), mnmaj(aDn, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
       for (int k0 = 0; k0 < MF; k0 += 16)  // + phiK G_t(S)
         mma(tmem, kmaj(aPK, T, k0), mnmaj(aG, k0, C::OMB), idesc_bf16(T, 64, 0, 1), 1);
-      for (int k0 = 0; k0 < D; k0 += 16)  // dphiK = V G_t(S)^T
-        mma(tmem + 256, kmaj(aV, T, k0), kmaj(aG, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
       mma_commit(sy.bar(3));
+    } else if (tid == 32) {
+      // dphiK = V G_t(S)^T, from a second issuing thread
+      const uint32_t aG = smem_u32(sG), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < D; k0 += 16)
+        mma(tmem + 256, kmaj(aV, T, k0), kmaj(aG, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
+      mma_commit(sy.bar(4));
     }
+    TC_WAIT(sy);
     TC_WAIT(sy);
     {
       float v[16];
@@ -1241,7 +1264,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       const uint32_t adA = smem_u32(sA), aPQ = smem_u32(sPhiQ);
       for (int k0 = 0; k0 < T; k0 += 16)  // dphiK += dA^T phiQ
         mma(tmem + 256, mnmaj(adA, k0, ROWT), mnmaj(aPQ, k0, ROWT), idesc_bf16(T, MF, 1, 1), 1);
-      mma_commit(sy.bar(4));
+      mma_commit(sy.bar(5));
     }
     TC_WAIT(sy);
     // K and Omega again (dk = u Omega - k sum(u), dOmega += u^T k), overlapping the epilogue
@@ -1288,20 +1311,25 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     cp_async_wait_all();
     publish();
     if (tid == 0) {
-      const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm), aK = smem_u32(sKr);
+      const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm);
       for (int k0 = 0; k0 < MF; k0 += 16)
         mma(tmem, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
+      mma_commit(sy.bar(6));
+    } else if (tid == 32) {
+      // the dOmega partial, from a second issuing thread
+      const uint32_t aU = smem_u32(sU), aK = smem_u32(sKr);
       for (int h = 0; h < C::MH; ++h)
         for (int k0 = 0; k0 < T; k0 += 16)
           mma(tmem + 64 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aK, k0, ROWT),
               idesc_bf16(T, 64, 1, 1), k0 > 0);
-      mma_commit(sy.bar(5));
+      mma_commit(sy.bar(7));
     }
     float us = 0.f;
     if (FEAT == SLIM_FEAT_EXP) {
 #pragma unroll
       for (int g = 0; g < NG; ++g) us += redU[g * T + row];
     }
+    TC_WAIT(sy);
     TC_WAIT(sy);
     {
       float xk[16];
