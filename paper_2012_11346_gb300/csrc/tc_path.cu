@@ -1355,7 +1355,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
 //   stage 1, CTA r < RS1: sums[r] = partials [r*per, (r+1)*per) summed in order
 //   stage 2, CTA s < RS2: dOmega += sums[0] + ... + sums[RS1-1] over one
 //            RS2-th of the elements (another slice's sums)
-constexpr int RS1 = 128, RS2 = 16;
+constexpr int RS1 = 128, RS2 = 32;
 struct RedJob {
   const float* part;  // stage 1: [nparts][M*64] lane-major partials
   int nparts;
@@ -1373,13 +1373,33 @@ __device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
   float4 acc[QMAX];
 #pragma unroll
   for (int k = 0; k < QMAX; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int i = i0; i < i1; ++i) {
-    const float4* src = reinterpret_cast<const float4*>(J.part + (size_t)i * J.n);
+  // partials in order; two at a time so that 2 * QMAX loads are in flight
+  int i = i0;
+  for (; i + 1 < i1; i += 2) {
+    const float4* s0 = reinterpret_cast<const float4*>(J.part + (size_t)i * J.n);
+    const float4* s1 = reinterpret_cast<const float4*>(J.part + (size_t)(i + 1) * J.n);
+    float4 x0[QMAX], x1[QMAX];
+#pragma unroll
+    for (int k = 0; k < QMAX; ++k) {
+      const int q = tid + k * NTHR;
+      x0[k] = q < n4 ? __ldcg(s0 + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+      x1[k] = q < n4 ? __ldcg(s1 + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < QMAX; ++k) {
+      acc[k].x = (acc[k].x + x0[k].x) + x1[k].x;
+      acc[k].y = (acc[k].y + x0[k].y) + x1[k].y;
+      acc[k].z = (acc[k].z + x0[k].z) + x1[k].z;
+      acc[k].w = (acc[k].w + x0[k].w) + x1[k].w;
+    }
+  }
+  if (i < i1) {
+    const float4* s0 = reinterpret_cast<const float4*>(J.part + (size_t)i * J.n);
 #pragma unroll
     for (int k = 0; k < QMAX; ++k) {
       const int q = tid + k * NTHR;
       if (q < n4) {
-        const float4 x = __ldcg(src + q);
+        const float4 x = __ldcg(s0 + q);
         acc[k].x += x.x;
         acc[k].y += x.y;
         acc[k].z += x.z;
@@ -1395,26 +1415,53 @@ __device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
   }
 }
 
-__device__ __forceinline__ void reduce_stage2(const RedJob& J, int s) {
+// Stage 2: CTA s owns float4 indices [s*share, (s+1)*share); thread (q, part)
+// sums the range sums [part*RS1/4, (part+1)*RS1/4) of float4 q, and the four
+// parts are then added in order through shared scratch red4[NTHR].
+__device__ __forceinline__ void reduce_stage2(const RedJob& J, int s, float4* red4) {
   const int n4 = J.n / 4, share = (n4 + RS2 - 1) / RS2;
-  const int q1 = min(n4, (s + 1) * share);
-  for (int q = s * share + (int)threadIdx.x; q < q1; q += NTHR) {
+  static_assert(NTHR % 4 == 0 && RS1 % 4 == 0, "stage 2 splits the ranges in four");
+  constexpr int QPER = NTHR / 4;  // float4 per round
+  const int tid = threadIdx.x, ql = tid % QPER, part = tid / QPER;
+  for (int q0 = s * share; q0 < min(n4, (s + 1) * share); q0 += QPER) {
+    const int q = q0 + ql;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int r = 0; r < RS1; ++r) {
-      const float4 x = __ldcg(reinterpret_cast<const float4*>(J.sums2 + (size_t)r * J.n) + q);
-      acc.x += x.x;
-      acc.y += x.y;
-      acc.z += x.z;
-      acc.w += x.w;
+    if (q < min(n4, (s + 1) * share)) {
+      constexpr int R4 = RS1 / 4;
+      float4 x[R4];
+#pragma unroll
+      for (int r = 0; r < R4; ++r)
+        x[r] = __ldcg(reinterpret_cast<const float4*>(J.sums2 + (size_t)(part * R4 + r) * J.n) + q);
+#pragma unroll
+      for (int r = 0; r < R4; ++r) {
+        acc.x += x[r].x;
+        acc.y += x[r].y;
+        acc.z += x[r].z;
+        acc.w += x[r].w;
+      }
     }
-    // lane-major float4 q holds row 128h + row, columns 16cg + 4i .. +3
-    const int row = q & 127, rest = q >> 7, i = rest & 3;
-    const int cg = (rest >> 2) % NG, h = rest / (4 * NG);
-    float* o = J.domega + (128 * h + row) * 64 + 16 * cg + 4 * i;
-    o[0] += acc.x;
-    o[1] += acc.y;
-    o[2] += acc.z;
-    o[3] += acc.w;
+    red4[tid] = acc;
+    __syncthreads();
+    if (part == 0 && q < min(n4, (s + 1) * share)) {
+      float4 t = red4[ql];
+#pragma unroll
+      for (int k = 1; k < 4; ++k) {
+        const float4 u = red4[k * QPER + ql];
+        t.x += u.x;
+        t.y += u.y;
+        t.z += u.z;
+        t.w += u.w;
+      }
+      // lane-major float4 q holds row 128h + row, columns 16cg + 4i .. +3
+      const int row = q & 127, rest = q >> 7, i = rest & 3;
+      const int cg = (rest >> 2) % NG, h = rest / (4 * NG);
+      float* o = J.domega + (128 * h + row) * 64 + 16 * cg + 4 * i;
+      o[0] += t.x;
+      o[1] += t.y;
+      o[2] += t.z;
+      o[3] += t.w;
+    }
+    __syncthreads();
   }
 }
 
@@ -1470,18 +1517,19 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ Ti
     return;
   }
   b -= J.n_red1;
-  if (b < J.n_red2) reduce_stage2(J.red, b);
+  if (b < J.n_red2) reduce_stage2(J.red, b, reinterpret_cast<float4*>(align1024(smem_raw)));
 }
 
 // The reduction stages that have no tile launch left to ride in.
 __global__ void __launch_bounds__(NTHR) k_tc_reduce(const __grid_constant__ RedJob J, int n_red1,
                                                     int n_red2) {
+  __shared__ float4 red4[NTHR];
   grid_dependency_wait();
   const int b = blockIdx.x;
   if (b < n_red1)
     reduce_stage1(J, b);
   else if (b - n_red1 < n_red2)
-    reduce_stage2(J, b - n_red1);
+    reduce_stage2(J, b - n_red1, red4);
 }
 
 // ================================================================== small kernels
