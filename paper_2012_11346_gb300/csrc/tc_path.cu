@@ -16,17 +16,19 @@
 //   forward, one launch, tiles in sequence order:
 //     phiQ, phiK, Delta_t, A = tril(phiQ phiK^T);  S_t, z_t = prefix before
 //     tile t;  num = phiQ S_t + A V_t,  den = phiQ z_t + rowsum A,  out = num/den
-//   backward, slices in reverse (Algorithm 1's reverse sweep), one launch each:
+//   backward, one launch, slices in reverse (Algorithm 1's reverse sweep):
 //     dq side of slice n, tiles in reverse order: phiQ, phiK, Delta_t, A;
 //       rollback P_t = P_{t+1} - Delta_t (eq. 17);  den, dnum = dout/den,
 //       dden = -<dout,out>/den, dA = tril(dnum V^T + dden);
 //       dphiQ = dnum S_t^T + dden z_t + dA phiK,  Gd_t = phiQ^T [dnum | dden];
 //       state-gradient chain G_t = G_{t+1} + Gd_{t+1} (eq. 18);
 //       dq = u Omega - q sum(u),  dOmega partial u^T q
-//     dk/dv side of slice n (in the launch of the dq side of slice n-1):
+//     dk/dv side of slice n (beside the dq side of slice n-1):
 //       dV = A^T dnum + phiK G_t(S),  dphiK = dA^T phiQ + V G_t(S)^T + g_t(z),
-//       dk = u Omega - k sum(u),  dOmega partial += u^T k
-//     reduce: dOmega += the partials, in a fixed order
+//       dk = u Omega - k sum(u),  dOmega partial u^T k
+//     each side adds its dOmega partials to one running sum per tile position
+//     (slices in order N-1 .. 0), and the sums are reduced once, in a fixed
+//     order, at the end of the launch
 #include <math.h>
 
 #include "common.cuh"
@@ -215,6 +217,9 @@ __device__ __forceinline__ void fence_acq_rel_gpu() {
 __device__ __forceinline__ void st_release_gpu(int* p, int v) {
   asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+__device__ __forceinline__ void red_release_gpu(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
 
 // Flags sit 128 bytes apart, so the CTAs polling different flags do not
 // share a cache line.
@@ -280,6 +285,16 @@ __device__ __forceinline__ void st_lm16(float* base, int h, int cg, int row, con
 #pragma unroll
   for (int i = 0; i < 4; ++i)
     __stcg(d + lm4(h, cg, i, row), make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+}
+// Adds 16 floats to a lane-major buffer in L2 (one vector reduction per
+// float4; the adds of one element are ordered by the flags around them).
+__device__ __forceinline__ void red_lm16(float* base, int h, int cg, int row, const float* v) {
+  float4* d = reinterpret_cast<float4*>(base);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(d + lm4(h, cg, i, row)),
+                 "f"(v[4 * i]), "f"(v[4 * i + 1]), "f"(v[4 * i + 2]), "f"(v[4 * i + 3])
+                 : "memory");
 }
 // Row-major [M][64] (the caller's state tensors): 16 floats at p.
 __device__ __forceinline__ void ld_row16f(const float* p, float* v) {
@@ -363,6 +378,39 @@ __device__ __forceinline__ void group_publish(int id) {
 __device__ __forceinline__ bool flag_poll(const int* flag, int want, int* err) {
   for (uint32_t i = 0; i < (1u << 22); ++i) {
     if (ld_relaxed_gpu(flag) == want) {
+      fence_acq_rel_gpu();
+      return true;
+    }
+    if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) return false;
+    __nanosleep(i < 16 ? 32 : 256);
+  }
+  atomicExch(err, 1);
+  return false;
+}
+// Bounded wait by one thread for up to two flags at once (a null flag is not
+// waited on): both are read in every round, so a satisfied pair costs one trip.
+__device__ __forceinline__ bool flag_poll2(const int* f1, int w1, const int* f2, int w2, int* err) {
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    const int v1 = f1 ? ld_relaxed_gpu(f1) : w1;
+    const int v2 = f2 ? ld_relaxed_gpu(f2) : w2;
+    if (v1 == w1 && v2 == w2) {
+      fence_acq_rel_gpu();
+      return true;
+    }
+    if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) return false;
+    __nanosleep(i < 16 ? 32 : 256);
+  }
+  atomicExch(err, 1);
+  return false;
+}
+// The thread that polls the flags a tile needs from other tiles: lane 0 of
+// the last warp, which takes no part in the tile loads, so its fence waits on
+// no copies of its own.
+constexpr int POLL = NTHR - 32, LDT = NTHR - 32;
+// Bounded wait by one thread for a counter to reach at least want.
+__device__ __forceinline__ bool counter_poll(const int* ctr, int want, int* err) {
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    if (ld_relaxed_gpu(ctr) - want >= 0) {
       fence_acq_rel_gpu();
       return true;
     }
@@ -630,10 +678,19 @@ struct BwdQJob {
   int L, a, b, ntn, n, N, nt, chains;  // slice n = rows [a, a+b), ntn tiles; nt: full slice
   float *slot1, *slot2;   // [chains][nt][E]: state prefixes, state-gradient prefixes
   int *flag1, *flag2;     // [chains][nt], FLAG_STRIDE ints apart
-  int* ticket;            // tile counter of this launch (starts at 0)
-  __nv_bfloat16* gS;      // [chains][ntn][MF][64] G_t(S) for the dk/dv side
-  float* gz;              // [chains][ntn][MF]     g_t(z)
-  float *rowstat, *part;  // [chains][ntn][T][2] (den, dden), [chains][ntn][MF][64]
+  // Hand-off to the dk/dv side of the same slice, through buffers of parity
+  // n % 2 indexed by (chain, tile) of a full slice:
+  __nv_bfloat16* gS;      // [chains][nt][MF][64] G_t(S)
+  float* gz;              // [chains][nt][MF]     g_t(z)
+  float* rowstat;         // [chains][nt][T][2]   (den, dden)
+  int* gflag;             // [chains][nt]: n + 1 once the three above are written
+  const int* kvread;      // [chains][nt]: n + 3 once slice n+2's dk/dv side has read them
+  int n2tiles;            // tiles of slice n+2 per chain (0: no such slice)
+  // dOmega: this side's per-position sums over slices N-1 .. n
+  float* acc;             // [chains][nt][MF][64] lane-major
+  int* accflag;           // [chains][nt]: n + 1 once slice n has added its partial
+  int n1tiles;            // tiles of slice n+1 per chain (0: no such slice)
+  int* sums_done;         // slice 0 only: counter of final sums written
   __nv_bfloat16* dq;
   int* err;
 };
@@ -671,7 +728,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   const int row0 = J.a + t * T;
   const int valid = min(T, J.b - t * T);
   const size_t g0 = ((size_t)c * J.L + row0) * D;
-  const size_t ti = (size_t)c * J.ntn + t;  // this slice's per-tile buffers
+  const size_t tf = (size_t)c * J.nt + t;   // hand-off buffers, flags, dOmega sums
+  // the first slice (from the end) with a tile at this position starts its sum
+  const bool acc_first = t >= J.n1tiles;
   // The prefixes after this tile: the next tile's slots, the first tile of
   // slice n+1, or (at the end of the sequence) B^(N) and G = 0.
   const bool inner = t + 1 < J.ntn, next_slice = n + 1 < J.N;
@@ -707,10 +766,20 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
-  load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
-  load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
-  load_rows64(sDo, T, J.dOut + g0, valid, tid, NTHR);
+  if (tid == POLL) {
+    // while the tiles stream in: the hand-off buffers of parity n % 2 are
+    // free once slice n+2's dk/dv side has read them (rowstat is written
+    // after join1, G_t after chain 2), and slice n+1's dOmega sum at this
+    // position is complete (this tile adds to it at the end)
+    const bool ok = flag_poll2(t < J.n2tiles ? J.kvread + tf * FLAG_STRIDE : nullptr, n + 3,
+                               acc_first ? nullptr : J.accflag + tf * FLAG_STRIDE, n + 2, J.err);
+    gfail[1] = ok ? 0 : 1;
+  } else if (tid < LDT) {
+    load_rows64(sQ, T, J.Q + g0, valid, tid, LDT);
+    load_rows64(sK, T, J.K + g0, valid, tid, LDT);
+    load_rows64(sV, T, J.V + g0, valid, tid, LDT);
+    load_rows64(sDo, T, J.dOut + g0, valid, tid, LDT);
+  }
   // this thread's 16 columns of its out row, fetched while the tiles stream in
   uint4 orow[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
   if (row < valid) {
@@ -718,10 +787,12 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     orow[0] = src[0];
     orow[1] = src[1];
   }
-  if (tid < 2) gfail[tid] = 0;
+  if (tid == 0) gfail[0] = 0;
   grid_dependency_wait();  // Omega (bf16), slots and buffers belong to earlier kernels
-  load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
-  load_rows64(sOl, MF, J.om16 + MF * D, MF, tid, NTHR);
+  if (tid < LDT) {
+    load_rows64(sOm, MF, J.om16, MF, tid, LDT);
+    load_rows64(sOl, MF, J.om16 + MF * D, MF, tid, LDT);
+  }
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   {
@@ -942,7 +1013,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       *reinterpret_cast<__nv_bfloat16*>(sDd + tile_off(16, r16, row)) =
           __float2bfloat16_rn(r16 == 0 ? dden : 0.f);
     if (rv && cg == 0) {
-      float* rsw = J.rowstat + (ti * T + row) * 2;
+      float* rsw = J.rowstat + (tf * T + row) * 2;
       rsw[0] = den;
       rsw[1] = dden;
     }
@@ -1051,7 +1122,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       for (int h = 0; h < C::MH; ++h) {
 #pragma unroll
         for (int j = 0; j < 2; ++j) {
-          st_lm16_bf16(J.gS + ti * MF * 64, h, cq + j, row, gs[h][j]);  // G_t(S), dk/dv side
+          st_lm16_bf16(J.gS + tf * MF * 64, h, cq + j, row, gs[h][j]);  // G_t(S), dk/dv side
           float gd[16];
           tmem_ld16(trow + 64 * h + 16 * (cq + j), gd);
 #pragma unroll
@@ -1065,12 +1136,15 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           const int m = 128 * h + row;
           float gdz;
           tmem_ld1(trow + 128 + 16 * h, gdz);
-          J.gz[ti * MF + m] = gzs[h];
+          J.gz[tf * MF + m] = gzs[h];
           __stcg(own2 + MF * 64 + m, gzs[h] + gdz);
         }
       }
       group_bar(2);  // every slot write of the group is issued
-      if (gl == 0) st_release_gpu(of2, n + 1);
+      if (gl == 0) {
+        st_release_gpu(of2, n + 1);
+        st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);  // G_t, g_t(z), rowstat
+      }
     }
   join2:
     __syncthreads();
@@ -1083,18 +1157,29 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       tc_fence_after();
       __syncthreads();
       if (abort_ | gfail[1]) goto teardown;
+      // the partial goes onto the running dOmega sum at this position (or
+      // starts it): one add per slice, in slice order
+      float* accp = J.acc + tf * (size_t)(MF * 64);
+      float v[16];
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        tmem_ld16(trow + 320 + 64 * h + 16 * cg, v);
+        if (acc_first)
+          st_lm16(accp, h, cg, row, v);
+        else
+          red_lm16(accp, h, cg, row, v);
+      }
+      __syncthreads();
+      if (tid == 0) {  // warp 0 waits for the release while the others store dq
+        st_release_gpu(J.accflag + tf * FLAG_STRIDE, n + 1);
+        if (J.sums_done) red_release_gpu(J.sums_done, 1);
+      }
       float xq[16];
       ld_feat16(sQ, row, 16 * cg, xq);
-      float v[16];
       tmem_ld16(trow + 256 + 16 * cg, v);
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xq[i], v[i]);
       if (rv) st_row16(J.dq + g0 + (size_t)row * D + 16 * cg, v);
-      float* dst = J.part + ti * (size_t)(MF * 64);
-      for (int h = 0; h < C::MH; ++h) {
-        tmem_ld16(trow + 320 + 64 * h + 16 * cg, v);
-        st_lm16(dst, h, cg, row, v);
-      }
     }
   }
   TC_TEARDOWN();
@@ -1103,11 +1188,17 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
 // ================================================================== backward, dk/dv side
 struct BwdKVJob {
   const __nv_bfloat16 *Q, *K, *V, *dOut, *om16;
-  const __nv_bfloat16* gS;  // [chains][nt][MF][64] G_t(S), from the dq side
+  // from the dq side of the same slice, indexed by (chain, tile) of a full slice
+  const __nv_bfloat16* gS;   // [chains][ntf][MF][64] G_t(S)
   const float *gz, *rowstat;
-  int L, a, b, nt;           // slice rows [a, a+b), nt tiles
+  const int* gflag;          // n + 1 once they are written
+  int* kvread;               // set to n + 1 once this side has read them
+  int L, a, b, ntn, ntf, n;  // slice n = rows [a, a+b), ntn tiles; ntf: full slice
   __nv_bfloat16 *dk, *dv;
-  float* part;
+  float* acc;                // as for the dq side: this side's dOmega sums
+  int* accflag;
+  int n1tiles;
+  int* sums_done;
   int* err;
 };
 
@@ -1133,45 +1224,42 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   const int row0 = J.a + t * T;
   const int valid = min(T, J.b - t * T);
   const size_t g0 = ((size_t)c * J.L + row0) * D;
-  const size_t ti = (size_t)c * J.nt + t;
-  TC_PROLOGUE();
-  load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
-  load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
-  load_rows64(sDn, T, J.dOut + g0, valid, tid, NTHR);
-  grid_dependency_wait();  // G_t and the row statistics come from the dq side, an earlier kernel
-  load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
-  load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, NTHR);  // Omega lo, until phiK overwrites it
-  for (int m = tid; m < MF; m += NTHR) sGz[m] = J.gz[ti * MF + m];
+  const size_t tf = (size_t)c * J.ntf + t;  // hand-off buffers, flags, dOmega sums
+  const bool acc_first = t >= J.n1tiles;
   float den = 0.f, dden = 0.f;
-  if (row < valid) {
-    const float* rsr = J.rowstat + (ti * T + row) * 2;
-    den = rsr[0];
-    dden = rsr[1];
+  __shared__ int poll_ok;  // written by the polling thread only
+  TC_PROLOGUE();
+  if (tid == POLL) {
+    // while the tiles stream in: G_t, g_t(z) and the row statistics come from
+    // the dq side of this tile, and the dOmega sum at this position from
+    // slice n+1
+    poll_ok = flag_poll2(J.gflag + tf * FLAG_STRIDE, J.n + 1,
+                         acc_first ? nullptr : J.accflag + tf * FLAG_STRIDE, J.n + 2, J.err);
+  } else if (tid < LDT) {
+    load_rows64(sQ, T, J.Q + g0, valid, tid, LDT);
+    load_rows64(sK, T, J.K + g0, valid, tid, LDT);
+    load_rows64(sV, T, J.V + g0, valid, tid, LDT);
+    load_rows64(sDn, T, J.dOut + g0, valid, tid, LDT);
+  }
+  grid_dependency_wait();  // Omega (bf16) comes from an earlier kernel
+  if (tid < LDT) {
+    load_rows64(sOm, MF, J.om16, MF, tid, LDT);
+    load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, LDT);  // Omega lo, until phiK overwrites it
   }
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
+  if (!poll_ok) goto teardown;
+  for (int m = tid; m < MF; m += NTHR) sGz[m] = __ldcg(J.gz + tf * MF + m);
+  if (row < valid) {
+    const float* rsr = J.rowstat + (tf * T + row) * 2;
+    den = __ldcg(rsr);
+    dden = __ldcg(rsr + 1);
+  }
   {
     const bool rv = row < valid;
-    const bool live = rv && den != 0.f;
-    const float inv = live ? 1.f / den : 0.f;
-    if (!live) dden = 0.f;
     float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
     redN[cg * T + row] = row_norm2_part(sQ, row, cg);
     redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
-#pragma unroll
-    for (int c8 = 16 * cg; c8 < 16 * cg + 16; c8 += 8) {  // dnum = dout / den, in place
-      const uint4 g = ld_chunk(sDn, T, row, c8);
-      const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
-      uint32_t pw[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        float g0f, g1f;
-        unpack_bf16(gw[i], g0f, g1f);
-        pw[i] = pack_bf16(g0f * inv, g1f * inv);
-      }
-      st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
-    }
     publish();
     const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
@@ -1194,8 +1282,24 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     }
     TC_WAIT(sy);  // Q projection done
     feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
+    const bool live = rv && den != 0.f;
+    const float inv = live ? 1.f / den : 0.f;
+    if (!live) dden = 0.f;
+#pragma unroll
+    for (int c8 = 16 * cg; c8 < 16 * cg + 16; c8 += 8) {  // dnum = dout / den, in place
+      const uint4 g = ld_chunk(sDn, T, row, c8);
+      const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+      uint32_t pw[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float g0f, g1f;
+        unpack_bf16(gw[i], g0f, g1f);
+        pw[i] = pack_bf16(g0f * inv, g1f * inv);
+      }
+      st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
+    }
     TC_WAIT(sy);  // K projection done: G_t(S) replaces Omega (awaited before the dV products)
-    load_lm_bf16(sG, MF, J.gS + ti * MF * 64, tid);
+    load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
     if (tid == 0) {
@@ -1222,6 +1326,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     }
     cp_async_wait_all();  // G_t(S)
     publish();
+    if (tid == POLL) st_release_gpu(J.kvread + tf * FLAG_STRIDE, J.n + 1);  // hand-off buffers read
     if (tid == 0) {
       const uint32_t aA = smem_u32(sA), aDn = smem_u32(sDn), aPK = smem_u32(sPhiK);
       const uint32_t aG = smem_u32(sG);
@@ -1332,41 +1437,53 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     TC_WAIT(sy);
     TC_WAIT(sy);
     {
+      // the partial goes onto the running dOmega sum at this position (or
+      // starts it): one add per slice, in slice order
+      float* accp = J.acc + tf * (size_t)(MF * 64);
+      float v[16];
+#pragma unroll
+      for (int h = 0; h < C::MH; ++h) {
+        tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
+        if (acc_first)
+          st_lm16(accp, h, cg, row, v);
+        else
+          red_lm16(accp, h, cg, row, v);
+      }
+      __syncthreads();
+      if (tid == 0) {  // warp 0 waits for the release while the others store dk
+        st_release_gpu(J.accflag + tf * FLAG_STRIDE, J.n + 1);
+        if (J.sums_done) red_release_gpu(J.sums_done, 1);
+      }
       float xk[16];
       ld_feat16(sKr, row, 16 * cg, xk);
-      float v[16];
       tmem_ld16(trow + 16 * cg, v);
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xk[i], v[i]);
       if (rv) st_row16(J.dk + g0 + (size_t)row * D + 16 * cg, v);
-      float* dst = J.part + ti * (size_t)(MF * 64);  // this side's own partial
-      for (int h = 0; h < C::MH; ++h) {
-        tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
-        st_lm16(dst, h, cg, row, v);
-      }
     }
   }
   TC_TEARDOWN();
 }
 
 // ================================================================== launches
-// dOmega reduction of one slice's per-tile partials (both sides, lane-major),
+// Final dOmega reduction of the per-position sums (both sides, lane-major),
 // in two stages with fixed ranges and orders, so dOmega is reproducible:
-//   stage 1, CTA r < RS1: sums[r] = partials [r*per, (r+1)*per) summed in order
-//   stage 2, CTA s < RS2: dOmega += sums[0] + ... + sums[RS1-1] over one
-//            RS2-th of the elements (another slice's sums)
-constexpr int RS1 = 128, RS2 = 32;
+//   stage 1, CTA r < nsums: sums[r] = positions [r*per, (r+1)*per) summed in order
+//   stage 2, CTA s: dOmega = sums[0] + ... + sums[nsums-1] over its share of
+//            the elements
+constexpr int RS1 = 128, RS2 = 32;  // most CTAs of stages 1 and 2
 struct RedJob {
-  const float* part;  // stage 1: [nparts][M*64] lane-major partials
+  const float* part;  // stage 1: [nparts][M*64] lane-major per-position sums
   int nparts;
-  float* sums;        // stage 1 out: [RS1][M*64]
-  const float* sums2; // stage 2 in: [RS1][M*64]
-  float* domega;      // [M][64], accumulated into
+  float* sums;        // [nsums][M*64]: stage 1 out, stage 2 in
+  int nsums;          // stage-1 CTAs, a multiple of 4
+  int nsplit;         // stage-2 CTAs
+  float* domega;      // [M][64]
   int n;              // M * 64
 };
 
 __device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
-  const int per = (J.nparts + RS1 - 1) / RS1;
+  const int per = (J.nparts + J.nsums - 1) / J.nsums;
   const int i0 = min(J.nparts, r * per), i1 = min(J.nparts, i0 + per);
   const int n4 = J.n / 4, tid = threadIdx.x;
   constexpr int QMAX = 256 * 64 / 4 / NTHR;  // float4 per thread at M = 256
@@ -1411,38 +1528,43 @@ __device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
 #pragma unroll
   for (int k = 0; k < QMAX; ++k) {
     const int q = tid + k * NTHR;
-    if (q < n4) dst[q] = acc[k];
+    if (q < n4) __stcg(dst + q, acc[k]);
   }
 }
 
 // Stage 2: CTA s owns float4 indices [s*share, (s+1)*share); thread (q, part)
-// sums the range sums [part*RS1/4, (part+1)*RS1/4) of float4 q, and the four
-// parts are then added in order through shared scratch red4[NTHR].
+// sums the range sums [part*nsums/4, (part+1)*nsums/4) of float4 q in order,
+// and the four parts are then added in order through shared scratch red4[NTHR].
 __device__ __forceinline__ void reduce_stage2(const RedJob& J, int s, float4* red4) {
-  const int n4 = J.n / 4, share = (n4 + RS2 - 1) / RS2;
-  static_assert(NTHR % 4 == 0 && RS1 % 4 == 0, "stage 2 splits the ranges in four");
+  const int n4 = J.n / 4, share = (n4 + J.nsplit - 1) / J.nsplit;
+  static_assert(NTHR % 4 == 0, "stage 2 splits the ranges in four");
   constexpr int QPER = NTHR / 4;  // float4 per round
+  constexpr int BATCH = 16;       // loads in flight per thread
   const int tid = threadIdx.x, ql = tid % QPER, part = tid / QPER;
-  for (int q0 = s * share; q0 < min(n4, (s + 1) * share); q0 += QPER) {
+  const int R4 = J.nsums / 4, end = min(n4, (s + 1) * share);
+  for (int q0 = s * share; q0 < end; q0 += QPER) {
     const int q = q0 + ql;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (q < min(n4, (s + 1) * share)) {
-      constexpr int R4 = RS1 / 4;
-      float4 x[R4];
+    if (q < end) {
+      for (int r0 = 0; r0 < R4; r0 += BATCH) {
+        float4 x[BATCH];
 #pragma unroll
-      for (int r = 0; r < R4; ++r)
-        x[r] = __ldcg(reinterpret_cast<const float4*>(J.sums2 + (size_t)(part * R4 + r) * J.n) + q);
+        for (int r = 0; r < BATCH; ++r)
+          if (r0 + r < R4)
+            x[r] = __ldcg(reinterpret_cast<const float4*>(J.sums + (size_t)(part * R4 + r0 + r) * J.n) + q);
 #pragma unroll
-      for (int r = 0; r < R4; ++r) {
-        acc.x += x[r].x;
-        acc.y += x[r].y;
-        acc.z += x[r].z;
-        acc.w += x[r].w;
+        for (int r = 0; r < BATCH; ++r)
+          if (r0 + r < R4) {
+            acc.x += x[r].x;
+            acc.y += x[r].y;
+            acc.z += x[r].z;
+            acc.w += x[r].w;
+          }
       }
     }
     red4[tid] = acc;
     __syncthreads();
-    if (part == 0 && q < min(n4, (s + 1) * share)) {
+    if (part == 0 && q < end) {
       float4 t = red4[ql];
 #pragma unroll
       for (int k = 1; k < 4; ++k) {
@@ -1456,80 +1578,203 @@ __device__ __forceinline__ void reduce_stage2(const RedJob& J, int s, float4* re
       const int row = q & 127, rest = q >> 7, i = rest & 3;
       const int cg = (rest >> 2) % NG, h = rest / (4 * NG);
       float* o = J.domega + (128 * h + row) * 64 + 16 * cg + 4 * i;
-      o[0] += t.x;
-      o[1] += t.y;
-      o[2] += t.z;
-      o[3] += t.w;
+      o[0] = t.x;
+      o[1] = t.y;
+      o[2] = t.z;
+      o[3] = t.w;
     }
     __syncthreads();
   }
 }
 
-// One launch runs tiles of up to three roles, then the dOmega reduction of
-// earlier slices.  The chained roles (dq side, forward) come first so their
-// chains start early; the independent dk/dv tiles follow, and the reduction
-// CTAs fill the launch's tail.  Inside a role every tile waits only on tiles
-// with lower block indices.
-struct TileJobs {
-  int n_q, n_fwd, n_kv, n_red1, n_red2;  // CTAs of each role, in dispatch order
-  BwdQJob q;
-  FwdJob f;
-  BwdKVJob kv;
-  RedJob red;
-};
-
+// ------------------------------------------------------------------ forward launch
+// Every tile of every slice in one launch.  A tile waits only on tiles earlier
+// in its chain; the CTAs take their tile from a counter rather than from
+// blockIdx, so the tiles handed out so far always belong to CTAs that are
+// running and every awaited tile is in progress whatever order the CTAs are
+// dispatched in.  (The counter is zeroed by the call's memset.)
 template <int MF, int FEAT>
-__global__ void __launch_bounds__(NTHR, 1) k_tc_tiles(const __grid_constant__ TileJobs J) {
+__global__ void __launch_bounds__(NTHR, 1) k_tc_fwd(const __grid_constant__ FwdJob J) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t mbar[NBAR];
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
   __shared__ int ticket;
-  // A chained tile waits only on tiles earlier in its chain.  The chained
-  // roles take their tile from a counter rather than from blockIdx: the
-  // tiles handed out so far always belong to CTAs that are running, so every
-  // awaited tile is in progress whatever order the CTAs are dispatched in.
-  // (The counter is zeroed by the call's memset, long before this launch.)
-  int b = blockIdx.x;
-  if (b < J.n_q) {
-    if (threadIdx.x == 0) ticket = atomicAdd(J.q.ticket, 1);
-    __syncthreads();
-    role_bwd_q<MF, FEAT>(J.q, ticket, smem_raw, mbar, tmem_base, abort_);
-    return;
-  }
-  b -= J.n_q;
-  if (b < J.n_fwd) {
-    if (threadIdx.x == 0) ticket = atomicAdd(J.f.ticket, 1);
-    __syncthreads();
-    role_fwd<MF, FEAT>(J.f, ticket / J.f.chains, ticket % J.f.chains, smem_raw, mbar, tmem_base,
-                       abort_);
-    return;
-  }
-  b -= J.n_fwd;
-  if (b < J.n_kv) {
-    role_bwd_kv<MF, FEAT>(J.kv, b % J.kv.nt, b / J.kv.nt, smem_raw, mbar, tmem_base, abort_);
-    return;
-  }
-  b -= J.n_kv;
-  grid_dependency_wait();  // partials and sums of earlier launches
-  if (b < J.n_red1) {
-    reduce_stage1(J.red, b);
-    return;
-  }
-  b -= J.n_red1;
-  if (b < J.n_red2) reduce_stage2(J.red, b, reinterpret_cast<float4*>(align1024(smem_raw)));
+  if (threadIdx.x == 0) ticket = atomicAdd(J.ticket, 1);
+  __syncthreads();
+  role_fwd<MF, FEAT>(J, ticket / J.chains, ticket % J.chains, smem_raw, mbar, tmem_base, abort_);
 }
 
-// The reduction stages that have no tile launch left to ride in.
-__global__ void __launch_bounds__(NTHR) k_tc_reduce(const __grid_constant__ RedJob J, int n_red1,
-                                                    int n_red2) {
-  __shared__ float4 red4[NTHR];
-  grid_dependency_wait();
-  const int b = blockIdx.x;
-  if (b < n_red1)
-    reduce_stage1(J, b);
-  else if (b - n_red1 < n_red2)
-    reduce_stage2(J, b - n_red1, red4);
+// ------------------------------------------------------------------ backward launch
+// The backward is one launch too.  Its items (tiles of either side, dOmega
+// reduction CTAs) are handed out by the same kind of counter, in stage order:
+// stage j = 0 .. N holds the dq-side tiles of slice N-1-j and the dk/dv-side
+// tiles of slice N-j (those that exist), and the final dOmega reduction
+// (stage 1, then stage 2) comes last.  Every wait of an item is on items of
+// earlier stages or on earlier tiles of its own chain, which hold lower
+// tickets:
+//   dq side of slice n    <- its chain (slice n's later tiles, slice n+1's first),
+//                            slice n+2's dk/dv side (hand-off buffers of parity
+//                            n%2), slice n+1's dq side at its position (dOmega sum)
+//   dk/dv side of slice n <- the dq side of the same tile; slice n+1's dk/dv side
+//                            at its position (dOmega sum)
+//   reduction stage 1     <- every tile of slice 0 (the last to add to a sum)
+//   reduction stage 2     <- stage 1
+// so the lowest unfinished item never waits and the launch always progresses.
+// Both sides take a slice's tiles in the same order (last tile first, chains
+// inside a tile position), and the two sides of a stage alternate by rows of
+// `chains` tiles: the dq-side tiles of one chain are further apart than in
+// one block per side, and a dk/dv tile comes a full stage after its dq tile.
+struct BwdSched {
+  int N, chains, nt, ntl;  // slices, chains, tiles of a full slice and of the last
+  int r1n, r2n;            // final dOmega stage-1 and stage-2 CTAs
+};
+enum { IT_Q = 0, IT_KV = 1, IT_R1 = 2, IT_R2 = 3 };
+struct BwdItem {
+  int kind, n, idx;  // role, slice, index among the role's items of the slice
+};
+
+__host__ __device__ inline int sched_tiles(const BwdSched& s, int n) {
+  return s.chains * (n == s.N - 1 ? s.ntl : s.nt);
+}
+__host__ __device__ inline void sched_stage(const BwdSched& s, int j, int& q, int& kv) {
+  const int nq = s.N - 1 - j, nkv = s.N - j;
+  q = (nq >= 0 && nq < s.N) ? sched_tiles(s, nq) : 0;
+  kv = (nkv >= 0 && nkv < s.N) ? sched_tiles(s, nkv) : 0;
+}
+__host__ __device__ inline long long sched_items(const BwdSched& s) {
+  long long n = s.r1n + s.r2n;
+  for (int k = 0; k < s.N; ++k) n += 2LL * sched_tiles(s, k);
+  return n;
+}
+// Item of ticket x.  Stages 2 .. N-1 all have the same size and are skipped
+// arithmetically.
+__host__ __device__ inline BwdItem sched_locate(const BwdSched& s, int x) {
+  int j = 0;
+  for (;;) {
+    if (j == 2 && s.N >= 3) {
+      const int cnt = s.N - 2, sz = 2 * s.chains * s.nt;
+      const int k = x / sz;
+      if (k < cnt) {
+        j = 2 + k;
+        x -= k * sz;
+        break;
+      }
+      x -= cnt * sz;
+      j = s.N;
+    }
+    if (j > s.N) break;
+    int q, kv;
+    sched_stage(s, j, q, kv);
+    if (x < q + kv) break;
+    x -= q + kv;
+    ++j;
+  }
+  if (j > s.N) {  // the final reduction
+    if (x < s.r1n) return BwdItem{IT_R1, 0, x};
+    return BwdItem{IT_R2, 0, x - s.r1n};
+  }
+  int q, kv;
+  sched_stage(s, j, q, kv);
+  bool isq = x < q;
+  int idx = isq ? x : x - q;
+  if (q > 0 && kv > 0) {
+    const int ch = s.chains, m = (q < kv ? q : kv) / ch;  // row pairs
+    if (x < 2 * m * ch) {
+      const int p = x / (2 * ch), w = x % (2 * ch);
+      isq = w < ch;
+      idx = p * ch + (isq ? w : w - ch);
+    } else {
+      isq = q > kv;
+      idx = m * ch + (x - 2 * m * ch);
+    }
+  }
+  return isq ? BwdItem{IT_Q, s.N - 1 - j, idx} : BwdItem{IT_KV, s.N - j, idx};
+}
+
+struct BwdJob {
+  BwdSched s;
+  BwdQJob q;   // slice fields set per item
+  BwdKVJob kv;
+  RedJob red;
+  int L, Cs;
+  int* ticket;
+  __nv_bfloat16* gS[2];
+  float *gz[2], *rowstat[2];
+  int *gflag[2], *kvread[2];
+  float* acc;       // [2 sides][chains][nt][M*64] per-position dOmega sums
+  int* accflag[2];  // [chains][nt] per side
+  int *sums_done, *r1done;  // slice-0 tiles done, final stage-1 CTAs done
+};
+
+template <int MF, int FEAT>
+__global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJob J) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t mbar[NBAR];
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_;
+  __shared__ int ticket;
+  if (threadIdx.x == 0) ticket = atomicAdd(J.ticket, 1);
+  __syncthreads();
+  const BwdItem it = sched_locate(J.s, ticket);
+  const int n = it.n, N = J.s.N;
+  if (it.kind <= IT_KV) {
+    const int a = n * J.Cs, b = min(J.Cs, J.L - a), ntn = (b + T - 1) / T;
+    const int n1 = n + 1 < N ? (n + 1 == N - 1 ? J.s.ntl : J.s.nt) : 0;
+    const size_t side = (size_t)J.s.chains * J.s.nt * MF * D;
+    if (it.kind == IT_Q) {
+      BwdQJob q = J.q;
+      q.a = a;
+      q.b = b;
+      q.ntn = ntn;
+      q.n = n;
+      q.gS = J.gS[n & 1];
+      q.gz = J.gz[n & 1];
+      q.rowstat = J.rowstat[n & 1];
+      q.gflag = J.gflag[n & 1];
+      q.kvread = J.kvread[n & 1];
+      q.n2tiles = n + 2 < N ? (n + 2 == N - 1 ? J.s.ntl : J.s.nt) : 0;
+      q.acc = J.acc;
+      q.accflag = J.accflag[0];
+      q.n1tiles = n1;
+      q.sums_done = n == 0 ? J.sums_done : nullptr;
+      role_bwd_q<MF, FEAT>(q, it.idx, smem_raw, mbar, tmem_base, abort_);
+    } else {
+      BwdKVJob kv = J.kv;
+      kv.a = a;
+      kv.b = b;
+      kv.ntn = ntn;
+      kv.n = n;
+      kv.gS = J.gS[n & 1];
+      kv.gz = J.gz[n & 1];
+      kv.rowstat = J.rowstat[n & 1];
+      kv.gflag = J.gflag[n & 1];
+      kv.kvread = J.kvread[n & 1];
+      kv.acc = J.acc + side;
+      kv.accflag = J.accflag[1];
+      kv.n1tiles = n1;
+      kv.sums_done = n == 0 ? J.sums_done : nullptr;
+      // the dq side's order: last tile first, chains inside a position
+      role_bwd_kv<MF, FEAT>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains, smem_raw, mbar,
+                            tmem_base, abort_);
+    }
+    return;
+  }
+  // final dOmega reduction over every position of both sides
+  if (threadIdx.x == 0) {
+    abort_ = 0;
+    const int want = it.kind == IT_R1 ? J.red.nparts : J.s.r1n;
+    if (!counter_poll(it.kind == IT_R1 ? J.sums_done : J.r1done, want, J.q.err)) abort_ = 1;
+  }
+  __syncthreads();
+  if (abort_) return;
+  if (it.kind == IT_R1) {
+    reduce_stage1(J.red, it.idx);
+    __syncthreads();
+    if (threadIdx.x == 0) red_release_gpu(J.r1done, 1);
+  } else {
+    reduce_stage2(J.red, it.idx, reinterpret_cast<float4*>(align1024(smem_raw)));
+  }
 }
 
 // ================================================================== small kernels
@@ -1567,25 +1812,50 @@ Geo geometry(const Problem& p) {
 // tiles overwrite the previous slice's only after reading them.  The buffers
 // the dq side hands to the dk/dv side have two slots (slice n uses n % 2),
 // because the dq side of slice n-1 runs beside the dk/dv side of slice n.
-// The dOmega partials of slice n are reduced in the launch after its dk/dv
-// side, beside the dq side of slice n-2: they take three slots.
+// dOmega is summed per (side, chain, tile position) over the slices and
+// reduced once at the end.
 struct Ws {
   int* err;
-  int* flags;    // [2][chains][nt], FLAG_STRIDE ints each
-  int* tickets;  // one tile counter per launch of the call
+  int* flags;  // every flag and counter of the call, zeroed together
+  int nflags;
+  int *flag1, *flag2;         // [chains][nt] chain flags, FLAG_STRIDE ints each
+  int *gflag[2], *kvread[2];  // [chains][nt] hand-off flags (backward)
+  int* accflag[2];            // [chains][nt] per side: dOmega sums (backward)
+  int *sums_done, *r1done;    // final reduction counters (backward)
+  int* ticket;
   __nv_bfloat16* om16;
   float *slot1, *slot2;
   __nv_bfloat16* gS[2];
-  float *gz[2], *rowstat[2], *rsums[2];
-  float* part[3];  // [2 sides][chains][nt][M*64]; slice n uses n % 3
+  float *gz[2], *rowstat[2];
+  float* acc;    // [2 sides][chains][nt][M*64]
+  float* rsums;  // [RS1][M*64]
 };
 
 Ws carve(Carver& cv, const Geo& g, bool bwd) {
   Ws w{};
-  const size_t C = g.chains, tiles = C * g.nt;
+  const size_t C = g.chains, tiles = C * g.nt, FS = FLAG_STRIDE;
   w.err = cv.take<int>(64);
-  w.flags = cv.take<int>(2 * tiles * FLAG_STRIDE);
-  w.tickets = cv.take<int>((size_t)g.N + 3);
+  w.nflags = (int)((bwd ? 8 * tiles + 2 : 2 * tiles) * FS + FS);
+  w.flags = cv.take<int>(w.nflags);
+  int* f = w.flags;
+  w.flag1 = f;
+  w.flag2 = f + tiles * FS;
+  f += 2 * tiles * FS;
+  if (bwd) {
+    for (int k = 0; k < 2; ++k) {
+      w.gflag[k] = f;
+      w.kvread[k] = f + tiles * FS;
+      f += 2 * tiles * FS;
+    }
+    for (int k = 0; k < 2; ++k) {
+      w.accflag[k] = f;
+      f += tiles * FS;
+    }
+    w.sums_done = f;
+    w.r1done = f + FS;
+    f += 2 * FS;
+  }
+  w.ticket = f;
   w.om16 = cv.take<__nv_bfloat16>((size_t)2 * g.MF * D);
   w.slot1 = cv.take<float>(tiles * g.E);
   if (bwd) {
@@ -1594,9 +1864,9 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
       w.gS[k] = cv.take<__nv_bfloat16>(tiles * g.MF * D);
       w.gz[k] = cv.take<float>(tiles * g.MF);
       w.rowstat[k] = cv.take<float>(tiles * T * 2);
-      w.rsums[k] = cv.take<float>((size_t)RS1 * g.MF * D);
     }
-    for (int k = 0; k < 3; ++k) w.part[k] = cv.take<float>(2 * tiles * (size_t)g.MF * D);
+    w.acc = cv.take<float>(2 * tiles * (size_t)g.MF * D);
+    w.rsums = cv.take<float>((size_t)RS1 * g.MF * D);
   }
   return w;
 }
@@ -1608,19 +1878,20 @@ constexpr size_t smem_fwd() {
 }
 template <int MF>
 constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<MF>::OMB + MF * 4 + 16; }
-template <int MF>
-constexpr size_t smem_max() {
-  return smem_bwd<MF>() > smem_fwd<MF>() ? smem_bwd<MF>() : smem_fwd<MF>();
-}
-static_assert(smem_max<256>() <= 232448, "a tile CTA must fit in 227 KB of shared memory");
+static_assert(smem_fwd<256>() <= 232448 && smem_bwd<256>() <= 232448,
+              "a tile CTA must fit in 227 KB of shared memory");
+static_assert(NTHR * sizeof(float4) <= smem_bwd<128>() - 1024, "stage-2 scratch fits");
 
 template <int MF, int FEAT>
 cudaError_t configure() {
   static bool done = false;
   if (done) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(k_tc_tiles<MF, FEAT>,
+  cudaError_t e = cudaFuncSetAttribute(k_tc_fwd<MF, FEAT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem_max<MF>());
+                                       (int)smem_fwd<MF>());
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem_bwd<MF>());
   if (e != cudaSuccess) return e;
   done = true;
   return cudaSuccess;
@@ -1665,27 +1936,9 @@ Slice slice_of(const Problem& p, const Geo& g, int n) {
   return r;
 }
 
-template <int MF, int FEAT>
-cudaError_t launch_tiles(cudaStream_t s, const TileJobs& J, double flops, double bytes,
-                         prof::Kid kid) {
-  const int n = J.n_kv + J.n_q + J.n_fwd + J.n_red1 + J.n_red2;
-  if (n == 0) return cudaSuccess;
-  const size_t smem = (J.n_kv || J.n_q) ? smem_bwd<MF>() : smem_fwd<MF>();
-  prof::Scope ps(kid, s, flops, bytes);
-  return launch_dep(k_tc_tiles<MF, FEAT>, dim3(n), dim3(NTHR), smem, s, J);
-}
-
-cudaError_t launch_reduce(cudaStream_t s, const RedJob& J, int n_red1, int n_red2) {
-  if (n_red1 + n_red2 == 0) return cudaSuccess;
-  prof::Scope ps(prof::K_TC_REDUCE, s);
-  return launch_dep(k_tc_reduce, dim3(n_red1 + n_red2), dim3(NTHR), 0, s, J, n_red1, n_red2);
-}
-
 cudaError_t prepare(const Ws& w, const Geo& g, const float* omega, cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
-  if (e == cudaSuccess)
-    e = cudaMemsetAsync(w.flags, 0, (size_t)2 * g.chains * g.nt * FLAG_STRIDE * sizeof(int), s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(w.tickets, 0, ((size_t)g.N + 3) * sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w.flags, 0, (size_t)w.nflags * sizeof(int), s);
   if (e != cudaSuccess) return e;
   prof::Scope ps(prof::K_TC_PREP, s);
   k_omega_bf16<<<nblk(g.MF * D), 256, 0, s>>>(omega, w.om16, g.MF * D);  // hi and lo
@@ -1703,14 +1956,23 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   TC_TRY(prepare(w, g, omega, s));
   // every tile of every slice in one launch, in sequence order, chains inside
   // a tile position.  Algorithmic work per row: 8dM (phiQ, phiK, Delta, readout).
-  TileJobs J{};
   const int P = (g.N - 1) * g.nt + slice_of(p, g, g.N - 1).nt;
-  J.f = FwdJob{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flags, w.tickets,
-               out, st, w.err};
-  J.n_fwd = P * g.chains;
+  const FwdJob J{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flag1, w.ticket,
+                 out, st, w.err};
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
-  TC_TRY((launch_tiles<MF, FEAT>(s, J, rows * 8.0 * MD, rows * D * 2.0 * 4, prof::K_TC_FWD)));
+  prof::Scope ps(prof::K_TC_FWD, s, rows * 8.0 * MD, rows * D * 2.0 * 4);
+  TC_TRY(launch_dep(k_tc_fwd<MF, FEAT>, dim3(P * g.chains), dim3(NTHR), smem_fwd<MF>(), s, J));
   return SLIM_OK;
+}
+
+// Final reduction: stage-1 CTAs each sum at least 8 positions, at most RS1
+// CTAs, a multiple of 4; stage 2 takes a quarter as many (at least 4).
+void reduction_split(const Geo& g, int& r1n, int& r2n) {
+  const int nparts = 2 * g.chains * g.nt;
+  r1n = nparts / 8;
+  r1n = r1n < 4 ? 4 : (r1n > RS1 ? RS1 : r1n);
+  r1n -= r1n % 4;
+  r2n = r1n / 4 < 4 ? 4 : (r1n / 4 > RS2 ? RS2 : r1n / 4);
 }
 
 template <int MF, int FEAT>
@@ -1724,59 +1986,42 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   Carver cv(workspace);
   const Ws w = carve(cv, g, true);
   const int N = g.N;
-  TC_TRY(cudaMemsetAsync(domega, 0, (size_t)MF * D * sizeof(float), s));
   TC_TRY(prepare(w, g, omega, s));
-  const double MD = (double)MF * D;
-  const size_t MD64 = (size_t)MF * D;
-  int* flag1 = w.flags;
-  int* flag2 = w.flags + (size_t)g.chains * g.nt * FLAG_STRIDE;
-  auto valid = [&](int n) { return n >= 0 && n < N; };
-  auto tiles_of = [&](int n) { return (size_t)g.chains * slice_of(p, g, n).nt; };
-  // Stage j of the reverse walk:
-  //   dq side of slice N-1-j, dk/dv side of slice N-j, dOmega stage 1 of
-  //   slice N+1-j and stage 2 of slice N+2-j.
-  // Algorithmic work per row: dq side 14dM (phiQ, phiK, rollback Delta, dphiQ,
-  // G, dq, dOmega), dk/dv side 8dM (dV, dphiK, dk, dOmega).
-  for (int j = 0; j <= N + 2; ++j) {
-    TileJobs J{};
-    double fl = 0.0, by = 0.0;
-    const int nq = N - 1 - j, nkv = N - j, nr1 = N + 1 - j, nr2 = N + 2 - j;
-    if (valid(nq)) {
-      const Slice sl = slice_of(p, g, nq);
-      const int x = nq & 1;
-      J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, sl.a, sl.b, sl.nt, nq, N, g.nt,
-                    g.chains, w.slot1, w.slot2, flag1, flag2, w.tickets + j, w.gS[x], w.gz[x],
-                    w.rowstat[x], w.part[nq % 3], dq, w.err};
-      J.n_q = sl.nt * g.chains;
-      fl += (double)g.chains * sl.b * 14.0 * MD;
-      by += (double)g.chains * sl.b * D * 2.0 * 6;
-    }
-    if (j >= 1 && valid(nkv)) {
-      const Slice sl = slice_of(p, g, nkv);
-      const int x = nkv & 1;
-      J.kv = BwdKVJob{q, k, v, dout, w.om16, w.gS[x], w.gz[x], w.rowstat[x], p.L, sl.a, sl.b,
-                      sl.nt, dk, dv, w.part[nkv % 3] + tiles_of(nkv) * MD64, w.err};
-      J.n_kv = sl.nt * g.chains;
-      fl += (double)g.chains * sl.b * 8.0 * MD;
-      by += (double)g.chains * sl.b * D * 2.0 * 6;
-    }
-    J.red.n = MF * D;
-    if (j >= 2 && valid(nr1)) {
-      J.red.part = w.part[nr1 % 3];
-      J.red.nparts = (int)(2 * tiles_of(nr1));
-      J.red.sums = w.rsums[nr1 & 1];
-      J.n_red1 = RS1;
-    }
-    if (j >= 3 && valid(nr2)) {
-      J.red.sums2 = w.rsums[nr2 & 1];
-      J.red.domega = domega;
-      J.n_red2 = RS2;
-    }
-    if (J.n_q + J.n_kv > 0)
-      TC_TRY((launch_tiles<MF, FEAT>(s, J, fl, by, prof::K_TC_BWD)));
-    else
-      TC_TRY(launch_reduce(s, J.red, J.n_red1, J.n_red2));
+  BwdJob J{};
+  J.s.N = N;
+  J.s.chains = g.chains;
+  J.s.nt = g.nt;
+  J.s.ntl = slice_of(p, g, N - 1).nt;
+  reduction_split(g, J.s.r1n, J.s.r2n);
+  // slice 0 (C rows, or all L rows) has a tile at every position, so its
+  // tiles close every dOmega sum
+  // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
+  J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
+                w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
+                nullptr, nullptr, 0, nullptr, dq, w.err};
+  J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, p.L, 0, 0,
+                  0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
+  J.red = RedJob{w.acc, 2 * g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
+  J.L = p.L;
+  J.Cs = g.Cs;
+  J.ticket = w.ticket;
+  for (int x = 0; x < 2; ++x) {
+    J.gS[x] = w.gS[x];
+    J.gz[x] = w.gz[x];
+    J.rowstat[x] = w.rowstat[x];
+    J.gflag[x] = w.gflag[x];
+    J.kvread[x] = w.kvread[x];
+    J.accflag[x] = w.accflag[x];
   }
+  J.acc = w.acc;
+  J.sums_done = w.sums_done;
+  J.r1done = w.r1done;
+  // Algorithmic work per row: dq side 14dM (phiQ, phiK, rollback Delta,
+  // dphiQ, G, dq, dOmega), dk/dv side 8dM (dV, dphiK, dk, dOmega).
+  const double rows = (double)g.chains * p.L, MD = (double)MF * D;
+  const long long items = sched_items(J.s);
+  prof::Scope ps(prof::K_TC_BWD, s, rows * 22.0 * MD, rows * D * 2.0 * 12);
+  TC_TRY(launch_dep(k_tc_bwd<MF, FEAT>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(), s, J));
   return SLIM_OK;
 }
 
