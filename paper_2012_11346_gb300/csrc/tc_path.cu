@@ -197,6 +197,7 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 #define TC_TEARDOWN()                                   \
   teardown:                                             \
   cp_async_wait_all();                                  \
+  bulk_wait_read();                                     \
   tc_fence_before();                                    \
   __syncthreads();                                      \
   if (warp == 0) tmem_dealloc(tmem_base, 512)
@@ -683,7 +684,11 @@ struct BwdQJob {
   __nv_bfloat16* gS;      // [chains][nt][MF][64] G_t(S)
   float* gz;              // [chains][nt][MF]     g_t(z)
   float* rowstat;         // [chains][nt][T][2]   (den, dden)
-  int* gflag;             // [chains][nt]: n + 1 once the three above are written
+  uint8_t* img;           // [chains][nt][2 FEATB + 32 KB]: phiQ and phiK as shared-
+                          //   memory tile images (bf16, 128-byte swizzle), then tril(A)
+                          //   in bf16, lane-major (chunk of 8 columns c/8, row r at
+                          //   16-byte unit (c/8) 128 + r)
+  int* gflag;             // [chains][nt]: n + 1 once the four above are written
   const int* kvread;      // [chains][nt]: n + 3 once slice n+2's dk/dv side has read them
   int n2tiles;            // tiles of slice n+2 per chain (0: no such slice)
   // dOmega: this side's per-position sums over slices N-1 .. n
@@ -844,6 +849,8 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     fill_ones(sOnes, tid);  // the K tile is no longer read
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
+    // the dk/dv side of this tile takes phiK, phiQ and tril(A) from here
+    uint8_t* img = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT);
     if (tid == 0 || (C::MH > 1 && tid == 32)) {
       // Delta_t = phiK^T [V | 1], one feature half per issuing thread
       const int h = tid == 0 ? 0 : 1;
@@ -877,18 +884,25 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       group_bar(1);
       if (gfail[0]) goto join1;
       float rs = 0.f;  // the rounded masked A values of this thread's columns
+      uint8_t* imgA = img + 2 * C::FEATB;
 #pragma unroll 1
       for (int c0 = 32 * cg; c0 < T; c0 += 64) {
         float v[32];
         tmem_ld32(trow + c0, v);
+        uint32_t pk[16];
 #pragma unroll
         for (int i = 0; i < 32; i += 2) {
           const float x0 = (c0 + i <= row) ? v[i] : 0.f;
           const float x1 = (c0 + i + 1 <= row) ? v[i + 1] : 0.f;
+          pk[i / 2] = pack_bf16(x0, x1);
           float r0, r1;
-          unpack_bf16(pack_bf16(x0, x1), r0, r1);
+          unpack_bf16(pk[i / 2], r0, r1);
           rs += r0 + r1;
         }
+#pragma unroll
+        for (int q = 0; q < 4; ++q)  // tril(A) for the dk/dv side: a warp writes 512 bytes
+          reinterpret_cast<uint4*>(imgA)[((c0 >> 3) + q) * T + row] =
+              make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
       }
       redA[cg * T + row] = rs;  // V is no longer read: its tile holds the partials
     } else {
@@ -959,6 +973,12 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   join1:
     __syncthreads();
     if (gfail[0] | gfail[1]) goto teardown;
+    // the two feature tiles' images, while the MMAs of the next phases run
+    // (phiK's tile is overwritten by u once they have landed)
+    if (tid == GRP) {
+      bulk_store(img, smem_u32(sPhiQ), C::FEATB);
+      bulk_store(img + C::FEATB, smem_u32(sPhiK), C::FEATB);
+    }
     {
       // g(Q) . z_t over this thread's feature columns
       constexpr int W = MF / NG;
@@ -1039,6 +1059,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     }
     if (!mbar_wait(smem_u32(&mb[4]), 0, J.err)) abort_ = 1;
     if (!mbar_wait(smem_u32(&mb[7]), 0, J.err)) abort_ = 1;
+    if (tid == GRP) bulk_wait_read();  // u goes to phiK's tile next
     tc_fence_after();
     __syncthreads();
     if (abort_) goto teardown;
@@ -1143,7 +1164,8 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       group_bar(2);  // every slot write of the group is issued
       if (gl == 0) {
         st_release_gpu(of2, n + 1);
-        st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);  // G_t, g_t(z), rowstat
+        bulk_wait_done();  // phiQ's and phiK's images
+        st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);  // G_t, g_t(z), rowstat, images
       }
     }
   join2:
@@ -1191,6 +1213,7 @@ struct BwdKVJob {
   // from the dq side of the same slice, indexed by (chain, tile) of a full slice
   const __nv_bfloat16* gS;   // [chains][ntf][MF][64] G_t(S)
   const float *gz, *rowstat;
+  const uint8_t* img;        // [chains][ntf][...] phiQ, phiK tile images, tril(A) lane-major
   const int* gflag;          // n + 1 once they are written
   int* kvread;               // set to n + 1 once this side has read them
   int L, a, b, ntn, ntf, n;  // slice n = rows [a, a+b), ntn tiles; ntf: full slice
@@ -1210,9 +1233,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   uint8_t* sPhiQ = base;               // later: u
   uint8_t* sU = sPhiQ;
   uint8_t* sPhiK = sPhiQ + C::FEATB;
-  uint8_t* sX = sPhiK + C::FEATB;      // [Q | K | Omega] -> [A | G_t] -> [dA | G_t] -> [K | red | Omega]
-  uint8_t* sQ = sX;
-  uint8_t* sK = sX + ROWT;
+  uint8_t* sX = sPhiK + C::FEATB;      // [A | G_t] -> [dA | G_t] -> [K | red | Omega]
   uint8_t* sA = sX;
   uint8_t* sKr = sX;
   float* redU = reinterpret_cast<float*>(sX + ROWT);
@@ -1227,25 +1248,31 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   const size_t tf = (size_t)c * J.ntf + t;  // hand-off buffers, flags, dOmega sums
   const bool acc_first = t >= J.n1tiles;
   float den = 0.f, dden = 0.f;
-  __shared__ int poll_ok;  // written by the polling thread only
+  __shared__ int poll_ok;              // written by the polling thread only
+  __shared__ __align__(8) uint64_t mb_img;  // the two feature tiles, initialised by that thread
   TC_PROLOGUE();
   if (tid == POLL) {
-    // while the tiles stream in: G_t, g_t(z) and the row statistics come from
-    // the dq side of this tile, and the dOmega sum at this position from
-    // slice n+1
+    // while V and dout stream in: phiQ, phiK, tril(A), G_t, g_t(z) and the
+    // row statistics come from the dq side of this tile, and the dOmega sum
+    // at this position from slice n+1; then the two feature tiles, by bulk
+    // copies completing on mb_img
     poll_ok = flag_poll2(J.gflag + tf * FLAG_STRIDE, J.n + 1,
                          acc_first ? nullptr : J.accflag + tf * FLAG_STRIDE, J.n + 2, J.err);
+    if (poll_ok) {
+      const uint8_t* img = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT);
+      const uint32_t bar = smem_u32(&mb_img);
+      mbar_init(bar, 1);
+      mbar_fence_init();
+      fence_proxy_async_global();
+      mbar_expect_tx(bar, 2 * C::FEATB);
+      bulk_load(smem_u32(sPhiQ), img, C::FEATB, bar);
+      bulk_load(smem_u32(sPhiK), img + C::FEATB, C::FEATB, bar);
+    }
   } else if (tid < LDT) {
-    load_rows64(sQ, T, J.Q + g0, valid, tid, LDT);
-    load_rows64(sK, T, J.K + g0, valid, tid, LDT);
     load_rows64(sV, T, J.V + g0, valid, tid, LDT);
     load_rows64(sDn, T, J.dOut + g0, valid, tid, LDT);
   }
-  grid_dependency_wait();  // Omega (bf16) comes from an earlier kernel
-  if (tid < LDT) {
-    load_rows64(sOm, MF, J.om16, MF, tid, LDT);
-    load_rows64(sPhiK, MF, J.om16 + MF * D, MF, tid, LDT);  // Omega lo, until phiK overwrites it
-  }
+  grid_dependency_wait();
   cp_async_wait_all();
   __syncthreads();  // rows were copied by other threads
   if (!poll_ok) goto teardown;
@@ -1255,33 +1282,18 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     den = __ldcg(rsr);
     dden = __ldcg(rsr + 1);
   }
+  load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);  // G_t(S), awaited before the dV products
+  {
+    // tril(A) into its tile (lane-major in global memory: coalesced reads)
+    const uint8_t* imgA = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT) + 2 * C::FEATB;
+    for (int k = tid; k < T * T / 8; k += NTHR)
+      cp_async16(smem_u32(sA) + tile_off(T, k % T, 8 * (k / T)), imgA + (size_t)k * 16, 16u);
+  }
   {
     const bool rv = row < valid;
-    float* redN = reinterpret_cast<float*>(sPhiQ);  // phiQ is written only after phase 1
-    redN[cg * T + row] = row_norm2_part(sQ, row, cg);
-    redN[(NG + cg) * T + row] = row_norm2_part(sK, row, cg);
-    publish();
-    const float q2 = group_total(redN, row), k2 = group_total(redN + NG * T, row);
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{mb, 0, J.err};
-    if (tid == 0) {
-      // two commits: the phiQ epilogue runs while the K projection is computed
-      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aOm = smem_u32(sOm);
-      const uint32_t aOl = smem_u32(sPhiK);
-      for (int k0 = 0; k0 < D; k0 += 16) {
-        mma(tmem, kmaj(aQ, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-        mma(tmem, kmaj(aQ, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
-      }
-      mma_commit(sy.bar(0));
-      for (int k0 = 0; k0 < D; k0 += 16) {
-        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOm, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-        mma(tmem + 256, kmaj(aK, T, k0), kmaj(aOl, MF, k0), idesc_bf16(T, MF, 0, 0), 1);
-      }
-      mma_commit(sy.bar(1));
-    }
-    TC_WAIT(sy);  // Q projection done
-    feature_epilogue<MF, FEAT>(trow, sPhiQ, row, cg, q2, rv);
     const bool live = rv && den != 0.f;
     const float inv = live ? 1.f / den : 0.f;
     if (!live) dden = 0.f;
@@ -1298,50 +1310,31 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       }
       st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
     }
-    TC_WAIT(sy);  // K projection done: G_t(S) replaces Omega (awaited before the dV products)
-    load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);
-    feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
+    if (!mbar_wait(smem_u32(&mb_img), 0, J.err)) abort_ = 1;  // the two feature tiles
+    cp_async_wait_all();  // G_t(S), tril(A)
     publish();
-    if (tid == 0) {
-      const uint32_t aPQ = smem_u32(sPhiQ), aPK = smem_u32(sPhiK);
-      const uint32_t aDn = smem_u32(sDn), aV = smem_u32(sV);
-      for (int k0 = 0; k0 < MF; k0 += 16)
-        mma(tmem, kmaj(aPQ, T, k0), kmaj(aPK, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
-      for (int k0 = 0; k0 < D; k0 += 16)  // dnum V^T
-        mma(tmem + 128, kmaj(aDn, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
-      mma_commit(sy.bar(2));
-    }
-    TC_WAIT(sy);
-    {  // A -> smem (masked, bf16), this thread's 32 columns
-      float v[32];
-      const int c0 = 32 * cg;
-      tmem_ld32(trow + c0, v);
-      uint32_t pk[16];
-#pragma unroll
-      for (int i = 0; i < 32; i += 2)
-        pk[i / 2] = pack_bf16((c0 + i <= row) ? v[i] : 0.f, (c0 + i + 1 <= row) ? v[i + 1] : 0.f);
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        st_chunk(sA, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
-    }
-    cp_async_wait_all();  // G_t(S)
-    publish();
+    if (abort_) goto teardown;
     if (tid == POLL) st_release_gpu(J.kvread + tf * FLAG_STRIDE, J.n + 1);  // hand-off buffers read
     if (tid == 0) {
-      const uint32_t aA = smem_u32(sA), aDn = smem_u32(sDn), aPK = smem_u32(sPhiK);
+      const uint32_t aDn = smem_u32(sDn), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < D; k0 += 16)  // dnum V^T
+        mma(tmem + 128, kmaj(aDn, T, k0), kmaj(aV, T, k0), idesc_bf16(T, T, 0, 0), k0 > 0);
+      mma_commit(sy.bar(0));
+      const uint32_t aA = smem_u32(sA), aPK = smem_u32(sPhiK);
       const uint32_t aG = smem_u32(sG);
       for (int k0 = 0; k0 < T; k0 += 16)  // dV = A^T dnum
         mma(tmem, mnmaj(aA, k0, ROWT), mnmaj(aDn, k0, ROWT), idesc_bf16(T, 64, 1, 1), k0 > 0);
       for (int k0 = 0; k0 < MF; k0 += 16)  // + phiK G_t(S)
         mma(tmem, kmaj(aPK, T, k0), mnmaj(aG, k0, C::OMB), idesc_bf16(T, 64, 0, 1), 1);
-      mma_commit(sy.bar(3));
+      mma_commit(sy.bar(1));
     } else if (tid == 32) {
       // dphiK = V G_t(S)^T, from a second issuing thread
       const uint32_t aG = smem_u32(sG), aV = smem_u32(sV);
       for (int k0 = 0; k0 < D; k0 += 16)
         mma(tmem + 256, kmaj(aV, T, k0), kmaj(aG, MF, k0), idesc_bf16(T, MF, 0, 0), k0 > 0);
-      mma_commit(sy.bar(4));
+      mma_commit(sy.bar(2));
     }
+    TC_WAIT(sy);
     TC_WAIT(sy);
     TC_WAIT(sy);
     {
@@ -1369,7 +1362,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       const uint32_t adA = smem_u32(sA), aPQ = smem_u32(sPhiQ);
       for (int k0 = 0; k0 < T; k0 += 16)  // dphiK += dA^T phiQ
         mma(tmem + 256, mnmaj(adA, k0, ROWT), mnmaj(aPQ, k0, ROWT), idesc_bf16(T, MF, 1, 1), 1);
-      mma_commit(sy.bar(5));
+      mma_commit(sy.bar(3));
     }
     TC_WAIT(sy);
     // K and Omega again (dk = u Omega - k sum(u), dOmega += u^T k), overlapping the epilogue
@@ -1419,7 +1412,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm);
       for (int k0 = 0; k0 < MF; k0 += 16)
         mma(tmem, kmaj(aU, T, k0), mnmaj(aOm, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
-      mma_commit(sy.bar(6));
+      mma_commit(sy.bar(4));
     } else if (tid == 32) {
       // the dOmega partial, from a second issuing thread
       const uint32_t aU = smem_u32(sU), aK = smem_u32(sKr);
@@ -1427,7 +1420,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
         for (int k0 = 0; k0 < T; k0 += 16)
           mma(tmem + 64 + 64 * h, mnmaj(aU + h * 2 * ROWT, k0, ROWT), mnmaj(aK, k0, ROWT),
               idesc_bf16(T, 64, 1, 1), k0 > 0);
-      mma_commit(sy.bar(7));
+      mma_commit(sy.bar(5));
     }
     float us = 0.f;
     if (FEAT == SLIM_FEAT_EXP) {
@@ -1701,6 +1694,7 @@ struct BwdJob {
   int* ticket;
   __nv_bfloat16* gS[2];
   float *gz[2], *rowstat[2];
+  uint8_t* img[2];
   int *gflag[2], *kvread[2];
   float* acc;       // [2 sides][chains][nt][M*64] per-position dOmega sums
   int* accflag[2];  // [chains][nt] per side
@@ -1732,6 +1726,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
       q.gz = J.gz[n & 1];
       q.rowstat = J.rowstat[n & 1];
       q.gflag = J.gflag[n & 1];
+      q.img = J.img[n & 1];
       q.kvread = J.kvread[n & 1];
       q.n2tiles = n + 2 < N ? (n + 2 == N - 1 ? J.s.ntl : J.s.nt) : 0;
       q.acc = J.acc;
@@ -1749,6 +1744,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
       kv.gz = J.gz[n & 1];
       kv.rowstat = J.rowstat[n & 1];
       kv.gflag = J.gflag[n & 1];
+      kv.img = J.img[n & 1];
       kv.kvread = J.kvread[n & 1];
       kv.acc = J.acc + side;
       kv.accflag = J.accflag[1];
@@ -1827,6 +1823,7 @@ struct Ws {
   float *slot1, *slot2;
   __nv_bfloat16* gS[2];
   float *gz[2], *rowstat[2];
+  uint8_t* img[2];  // [chains][nt]: phiQ, phiK (T x M bf16 each) and tril(A) (T x T bf16)
   float* acc;    // [2 sides][chains][nt][M*64]
   float* rsums;  // [RS1][M*64]
 };
@@ -1864,6 +1861,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
       w.gS[k] = cv.take<__nv_bfloat16>(tiles * g.MF * D);
       w.gz[k] = cv.take<float>(tiles * g.MF);
       w.rowstat[k] = cv.take<float>(tiles * T * 2);
+      w.img[k] = cv.take<uint8_t>(tiles * ((size_t)4 * T * g.MF + 2 * T * T));
     }
     w.acc = cv.take<float>(2 * tiles * (size_t)g.MF * D);
     w.rsums = cv.take<float>((size_t)RS1 * g.MF * D);
@@ -1997,10 +1995,10 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // tiles close every dOmega sum
   // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
   J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
-                w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
-                nullptr, nullptr, 0, nullptr, dq, w.err};
-  J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, p.L, 0, 0,
-                  0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
+                w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
+                0, nullptr, nullptr, 0, nullptr, dq, w.err};
+  J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
+                  p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
   J.red = RedJob{w.acc, 2 * g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
   J.L = p.L;
   J.Cs = g.Cs;
@@ -2010,6 +2008,7 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
     J.gz[x] = w.gz[x];
     J.rowstat[x] = w.rowstat[x];
     J.gflag[x] = w.gflag[x];
+    J.img[x] = w.img[x];
     J.kvread[x] = w.kvread[x];
     J.accflag[x] = w.accflag[x];
   }
