@@ -635,14 +635,17 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     __syncthreads();
     if (gfail[0] | gfail[1]) goto teardown;
     publish();
+    // three issuing threads: the narrow products are issue-bound
     if (tid == 0) {
       const uint32_t aPQ = smem_u32(sPhiQ), aS = smem_u32(sS);
-      const uint32_t aA = smem_u32(sA), aV = smem_u32(sV);
       for (int k0 = 0; k0 < MF; k0 += 16)  // num = phiQ S_t
         mma(tmem + 128, kmaj(aPQ, T, k0), mnmaj(aS, k0, C::OMB), idesc_bf16(T, 64, 0, 1), k0 > 0);
-      for (int k0 = 0; k0 < T; k0 += 16)  // num += A V
-        mma(tmem + 128, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), 1);
       mma_commit(smem_u32(&mb[4]));
+    } else if (tid == 64) {
+      const uint32_t aA = smem_u32(sA), aV = smem_u32(sV);
+      for (int k0 = 0; k0 < T; k0 += 16)  // + A V, in a second accumulator
+        mma(tmem + 256, kmaj(aA, T, k0), mnmaj(aV, k0, ROWT), idesc_bf16(T, 64, 0, 1), k0 > 0);
+      mma_commit(smem_u32(&mb[7]));
     } else if (tid == 32) {
       // phiQ [z_hi | z_lo], from a second issuing thread
       const uint32_t aPQ = smem_u32(sPhiQ), aZ = smem_u32(sZt);
@@ -653,6 +656,7 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     const float rsA = redA[row] + redA[T + row];
     if (!mbar_wait(smem_u32(&mb[4]), 0, J.err)) abort_ = 1;
     if (!mbar_wait(smem_u32(&mb[6]), 0, J.err)) abort_ = 1;
+    if (!mbar_wait(smem_u32(&mb[7]), 0, J.err)) abort_ = 1;
     tc_fence_after();
     __syncthreads();
     if (abort_) goto teardown;
@@ -662,10 +666,11 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
       tmem_ld1(trow + 193, zl);
       const float den = rsA + (zh + zl);
       const float inv = den != 0.f ? 1.f / den : 0.f;
-      float v[16];
+      float v[16], w[16];
       tmem_ld16(trow + 128 + 16 * cg, v);  // every lane loads (warp-aligned op)
+      tmem_ld16(trow + 256 + 16 * cg, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] *= inv;
+      for (int i = 0; i < 16; ++i) v[i] = (v[i] + w[i]) * inv;
       if (rv) st_row16(J.out + g0 + (size_t)row * D + 16 * cg, v);
     }
   }
@@ -1162,11 +1167,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
         }
       }
       group_bar(2);  // every slot write of the group is issued
-      if (gl == 0) {
-        st_release_gpu(of2, n + 1);
-        bulk_wait_done();  // phiQ's and phiK's images
-        st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);  // G_t, g_t(z), rowstat, images
-      }
+      if (gl == 0) st_release_gpu(of2, n + 1);
     }
   join2:
     __syncthreads();
@@ -1195,6 +1196,11 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       if (tid == 0) {  // warp 0 waits for the release while the others store dq
         st_release_gpu(J.accflag + tf * FLAG_STRIDE, n + 1);
         if (J.sums_done) red_release_gpu(J.sums_done, 1);
+      } else if (tid == GRP) {
+        // the hand-off to the dk/dv side (a stage later): G_t, g_t(z), rowstat,
+        // tril(A) and, once its bulk copies are done, the feature tiles
+        bulk_wait_done();
+        st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);
       }
       float xq[16];
       ld_feat16(sQ, row, 16 * cg, xq);
@@ -1525,6 +1531,63 @@ __device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
   }
 }
 
+// Stage 1 streaming its positions through shared memory: NSLOT slots of one
+// position each, filled by bulk copies (one thread, mbarrier per slot), so
+// NSLOT positions are in flight; the sum is taken in the same order.
+constexpr int NSLOT = 3;
+__device__ __forceinline__ void reduce_stage1_bulk(const RedJob& J, int r, uint8_t* smem,
+                                                   uint64_t* mb, int* err) {
+  const int per = (J.nparts + J.nsums - 1) / J.nsums;
+  const int i0 = min(J.nparts, r * per), cnt = min(J.nparts, i0 + per) - i0;
+  const int n4 = J.n / 4, tid = threadIdx.x;
+  const uint32_t bytes = (uint32_t)J.n * 4;
+  constexpr int QMAX = 256 * 64 / 4 / NTHR;
+  float4 acc[QMAX];
+#pragma unroll
+  for (int k = 0; k < QMAX; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (tid == 0) {
+    for (int sl = 0; sl < NSLOT; ++sl) mbar_init(smem_u32(&mb[sl]), 1);
+    mbar_fence_init();
+    fence_proxy_async_global();  // the sums were acquired by this thread
+    for (int sl = 0; sl < NSLOT && sl < cnt; ++sl) {
+      mbar_expect_tx(smem_u32(&mb[sl]), bytes);
+      bulk_load(smem_u32(smem + (size_t)sl * bytes), J.part + (size_t)(i0 + sl) * J.n, bytes,
+                smem_u32(&mb[sl]));
+    }
+  }
+  __syncthreads();
+  bool ok = true;
+  for (int k = 0; k < cnt; ++k) {
+    const int sl = k % NSLOT;
+    if (!mbar_wait(smem_u32(&mb[sl]), (uint32_t)((k / NSLOT) & 1), err)) ok = false;
+    const float4* src = reinterpret_cast<const float4*>(smem + (size_t)sl * bytes);
+#pragma unroll
+    for (int q = 0; q < QMAX; ++q) {
+      const int e = tid + q * NTHR;
+      if (e < n4) {
+        const float4 x = src[e];
+        acc[q].x += x.x;
+        acc[q].y += x.y;
+        acc[q].z += x.z;
+        acc[q].w += x.w;
+      }
+    }
+    __syncthreads();  // the slot is read by every thread
+    if (tid == 0 && ok && k + NSLOT < cnt) {
+      fence_async_smem();
+      mbar_expect_tx(smem_u32(&mb[sl]), bytes);
+      bulk_load(smem_u32(smem + (size_t)sl * bytes), J.part + (size_t)(i0 + k + NSLOT) * J.n, bytes,
+                smem_u32(&mb[sl]));
+    }
+  }
+  float4* dst = reinterpret_cast<float4*>(J.sums + (size_t)r * J.n);
+#pragma unroll
+  for (int q = 0; q < QMAX; ++q) {
+    const int e = tid + q * NTHR;
+    if (e < n4) __stcg(dst + e, acc[q]);
+  }
+}
+
 // Stage 2: CTA s owns float4 indices [s*share, (s+1)*share); thread (q, part)
 // sums the range sums [part*nsums/4, (part+1)*nsums/4) of float4 q in order,
 // and the four parts are then added in order through shared scratch red4[NTHR].
@@ -1765,7 +1828,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
   __syncthreads();
   if (abort_) return;
   if (it.kind == IT_R1) {
-    reduce_stage1(J.red, it.idx);
+    reduce_stage1_bulk(J.red, it.idx, align1024(smem_raw), mbar, J.q.err);
     __syncthreads();
     if (threadIdx.x == 0) red_release_gpu(J.r1done, 1);
   } else {
@@ -1879,6 +1942,9 @@ constexpr size_t smem_bwd() { return 1024 + 2 * Cfg<MF>::FEATB + 4 * ROWT + Cfg<
 static_assert(smem_fwd<256>() <= 232448 && smem_bwd<256>() <= 232448,
               "a tile CTA must fit in 227 KB of shared memory");
 static_assert(NTHR * sizeof(float4) <= smem_bwd<128>() - 1024, "stage-2 scratch fits");
+static_assert(NSLOT * 128 * 64 * 4 <= smem_bwd<128>() - 1024 &&
+                  NSLOT * 256 * 64 * 4 <= smem_bwd<256>() - 1024,
+              "stage-1 slots fit");
 
 template <int MF, int FEAT>
 cudaError_t configure() {
