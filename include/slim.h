@@ -153,6 +153,24 @@ slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype d
                           slim_feature feature, int* path);
 
 /*
+ * The order in which the tensor-core backward (one launch, Algorithm 1's
+ * reverse sweep) hands out its work items; a pure host computation, for
+ * inspecting and testing that order (no counterpart in the paper).  Ticket x
+ * names item (role, slice, index), written to items[3x], items[3x+1],
+ * items[3x+2] for x < min(*count, cap):
+ *   role 0: dq side of tile index of the slice (tiles last first, chains
+ *           inside a position: tile ntn-1-index/(B*H) of chain index%(B*H)),
+ *   role 1: dk/dv side of the same tile numbering,
+ *   role 2: final dOmega reduction, stage 1 CTA index (slice 0),
+ *   role 3: final dOmega reduction, stage 2 CTA index (slice 0).
+ * *count receives the number of items.  items may be null when cap is 0.
+ * Returns SLIM_ERR_UNSUPPORTED for problems the tensor-core path does not
+ * take (see slim_path_for) and for L = 0.
+ */
+slim_status slim_bwd_schedule(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                              slim_feature feature, int* items, int cap, int* count);
+
+/*
  * Reads the device error word that bounded waits in the kernels set when they
  * give up, and clears it.  Copies 4 bytes from the workspace on `stream` and
  * synchronises that stream (this call, unlike the others, blocks).

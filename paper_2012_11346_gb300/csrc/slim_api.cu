@@ -171,6 +171,17 @@ slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype d
   return SLIM_OK;
 }
 
+slim_status slim_bwd_schedule(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                              slim_feature feature, int* items, int cap, int* count) {
+  if (!count || cap < 0 || (cap > 0 && !items)) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  if (!use_tc(p) || L == 0) return SLIM_ERR_UNSUPPORTED;
+  *count = slim::tc::bwd_schedule(p, items, cap);
+  return SLIM_OK;
+}
+
 slim_status slim_check_device_error(void* workspace, void* stream) {
   if (workspace == nullptr) return SLIM_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -2102,6 +2102,24 @@ size_t workspace_bytes(const Problem& p, bool bwd) {
   return cv.bytes();
 }
 
+int bwd_schedule(const Problem& p, int* items, int cap) {
+  const Geo g = geometry(p);
+  BwdSched sc{};
+  sc.N = g.N;
+  sc.chains = g.chains;
+  sc.nt = g.nt;
+  sc.ntl = slice_of(p, g, g.N - 1).nt;
+  reduction_split(g, sc.r1n, sc.r2n);
+  const long long n = sched_items(sc);
+  for (long long x = 0; x < n && x < cap; ++x) {
+    const BwdItem it = sched_locate(sc, (int)x);
+    items[3 * x] = it.kind;
+    items[3 * x + 1] = it.n;
+    items[3 * x + 2] = it.idx;
+  }
+  return (int)n;
+}
+
 #define TC_DISPATCH(FN, ...)                                                        \
   do {                                                                              \
     if (p.M == 256)                                                                 \

@@ -8,6 +8,9 @@ namespace tc {
 // bf16, d = 64, M in {128, 256}, slices of at least 64 rows.
 bool supports(const Problem& p);
 size_t workspace_bytes(const Problem& p, bool bwd);
+// The backward launch's item order: items[3 x] = (role, slice, index) of
+// ticket x, for x < min(count, cap).  Returns the item count.
+int bwd_schedule(const Problem& p, int* items, int cap);
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
                 const float* omega, void* out, const StateOut& st, void* workspace,
