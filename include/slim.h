@@ -164,11 +164,15 @@ slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype d
  *   role 2: final dOmega reduction, stage 1 CTA index (slice 0),
  *   role 3: final dOmega reduction, stage 2 CTA index (slice 0).
  * *count receives the number of items.  items may be null when cap is 0.
+ * *ring (when ring is not null) receives R, the slots of the ring through
+ * which the dq side of slice n hands its tiles to the dk/dv side (slot n % R;
+ * the dq side of slice n-R waits until slice n's dk/dv side has read it).
  * Returns SLIM_ERR_UNSUPPORTED for problems the tensor-core path does not
  * take (see slim_path_for) and for L = 0.
  */
 slim_status slim_bwd_schedule(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
-                              slim_feature feature, int* items, int cap, int* count);
+                              slim_feature feature, int* items, int cap, int* count,
+                              int* ring);
 
 /*
  * Reads the device error word that bounded waits in the kernels set when they

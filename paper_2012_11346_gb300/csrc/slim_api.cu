@@ -172,13 +172,14 @@ slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype d
 }
 
 slim_status slim_bwd_schedule(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
-                              slim_feature feature, int* items, int cap, int* count) {
+                              slim_feature feature, int* items, int cap, int* count,
+                              int* ring) {
   if (!count || cap < 0 || (cap > 0 && !items)) return SLIM_ERR_INVALID_ARG;
   Problem p;
   slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
   if (st != SLIM_OK) return st;
   if (!use_tc(p) || L == 0) return SLIM_ERR_UNSUPPORTED;
-  *count = slim::tc::bwd_schedule(p, items, cap);
+  *count = slim::tc::bwd_schedule(p, items, cap, ring);
   return SLIM_OK;
 }
 

@@ -684,8 +684,8 @@ struct BwdQJob {
   int L, a, b, ntn, n, N, nt, chains;  // slice n = rows [a, a+b), ntn tiles; nt: full slice
   float *slot1, *slot2;   // [chains][nt][E]: state prefixes, state-gradient prefixes
   int *flag1, *flag2;     // [chains][nt], FLAG_STRIDE ints apart
-  // Hand-off to the dk/dv side of the same slice, through buffers of parity
-  // n % 2 indexed by (chain, tile) of a full slice:
+  // Hand-off to the dk/dv side of the same slice, through the buffers of ring
+  // slot n % R indexed by (chain, tile) of a full slice:
   __nv_bfloat16* gS;      // [chains][nt][MF][64] G_t(S)
   float* gz;              // [chains][nt][MF]     g_t(z)
   float* rowstat;         // [chains][nt][T][2]   (den, dden)
@@ -694,8 +694,9 @@ struct BwdQJob {
                           //   in bf16, lane-major (chunk of 8 columns c/8, row r at
                           //   16-byte unit (c/8) 128 + r)
   int* gflag;             // [chains][nt]: n + 1 once the four above are written
-  const int* kvread;      // [chains][nt]: n + 3 once slice n+2's dk/dv side has read them
-  int n2tiles;            // tiles of slice n+2 per chain (0: no such slice)
+  const int* kvread;      // [chains][nt]: n + R + 1 once slice n+R's dk/dv side has read them
+  int ring;               // R, slots of the hand-off ring
+  int nRtiles;            // tiles of slice n+R per chain (0: no such slice)
   // dOmega: this side's per-position sums over slices N-1 .. n
   float* acc;             // [chains][nt][MF][64] lane-major
   int* accflag;           // [chains][nt]: n + 1 once slice n has added its partial
@@ -709,7 +710,7 @@ struct BwdQJob {
 // epilogue, warps 0-7 compute g(Q), A and dout V^T while warps 8-15 run the
 // rollback chain (which needs only Delta_t); after dphiQ, warps 0-7 compute u
 // and issue dq while warps 8-15 run the state-gradient chain.
-template <int MF, int FEAT>
+template <int MF, int FEAT, bool EARLY>
 __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* smem_raw,
                                            uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
@@ -777,12 +778,13 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   }
   if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
   if (tid == POLL) {
-    // while the tiles stream in: the hand-off buffers of parity n % 2 are
-    // free once slice n+2's dk/dv side has read them (rowstat is written
-    // after join1, G_t after chain 2), and slice n+1's dOmega sum at this
-    // position is complete (this tile adds to it at the end)
-    const bool ok = flag_poll2(t < J.n2tiles ? J.kvread + tf * FLAG_STRIDE : nullptr, n + 3,
-                               acc_first ? nullptr : J.accflag + tf * FLAG_STRIDE, n + 2, J.err);
+    // while the tiles stream in: the hand-off buffers of ring slot n % R are
+    // free once slice n+R's dk/dv side has read them (tril(A) is written in
+    // the A row-sum loop, the rest after join1)
+    const bool ok = flag_poll2(t < J.nRtiles ? J.kvread + tf * FLAG_STRIDE : nullptr,
+                               n + J.ring + 1,
+                               EARLY && !acc_first ? J.accflag + tf * FLAG_STRIDE : nullptr,
+                               n + 2, J.err);
     gfail[1] = ok ? 0 : 1;
   } else if (tid < LDT) {
     load_rows64(sQ, T, J.Q + g0, valid, tid, LDT);
@@ -1167,7 +1169,17 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
         }
       }
       group_bar(2);  // every slot write of the group is issued
-      if (gl == 0) st_release_gpu(of2, n + 1);
+      if (gl == 0) {
+        st_release_gpu(of2, n + 1);
+        if (!EARLY) {
+          // the hand-off to the dk/dv side: G_t, g_t(z), rowstat, tril(A) and,
+          // once its bulk copies are done, the feature tiles
+          bulk_wait_done();
+          st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);
+          // slice n+1's dOmega sum at this position (added to after join2)
+          if (!acc_first && !flag_poll(J.accflag + tf * FLAG_STRIDE, n + 2, J.err)) gfail[1] = 1;
+        }
+      }
     }
   join2:
     __syncthreads();
@@ -1196,9 +1208,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       if (tid == 0) {  // warp 0 waits for the release while the others store dq
         st_release_gpu(J.accflag + tf * FLAG_STRIDE, n + 1);
         if (J.sums_done) red_release_gpu(J.sums_done, 1);
-      } else if (tid == GRP) {
-        // the hand-off to the dk/dv side (a stage later): G_t, g_t(z), rowstat,
-        // tril(A) and, once its bulk copies are done, the feature tiles
+      } else if (tid == GRP && EARLY) {
+        // long stages: the hand-off (its dk/dv side is a stage away), off the
+        // G chain's path
         bulk_wait_done();
         st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);
       }
@@ -1231,7 +1243,7 @@ struct BwdKVJob {
   int* err;
 };
 
-template <int MF, int FEAT>
+template <int MF, int FEAT, bool EARLY>
 __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uint8_t* smem_raw,
                                             uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
@@ -1259,11 +1271,11 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   TC_PROLOGUE();
   if (tid == POLL) {
     // while V and dout stream in: phiQ, phiK, tril(A), G_t, g_t(z) and the
-    // row statistics come from the dq side of this tile, and the dOmega sum
-    // at this position from slice n+1; then the two feature tiles, by bulk
-    // copies completing on mb_img
+    // row statistics come from the dq side of this tile; then the two feature
+    // tiles, by bulk copies completing on mb_img
     poll_ok = flag_poll2(J.gflag + tf * FLAG_STRIDE, J.n + 1,
-                         acc_first ? nullptr : J.accflag + tf * FLAG_STRIDE, J.n + 2, J.err);
+                         EARLY && !acc_first ? J.accflag + tf * FLAG_STRIDE : nullptr, J.n + 2,
+                         J.err);
     if (poll_ok) {
       const uint8_t* img = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT);
       const uint32_t bar = smem_u32(&mb_img);
@@ -1433,6 +1445,10 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
 #pragma unroll
       for (int g = 0; g < NG; ++g) us += redU[g * T + row];
     }
+    // slice n+1's dOmega sum at this position, added to after the next waits
+    if (tid == POLL && !EARLY && !acc_first &&
+        !flag_poll(J.accflag + tf * FLAG_STRIDE, J.n + 2, J.err))
+      abort_ = 1;
     TC_WAIT(sy);
     TC_WAIT(sy);
     {
@@ -1755,16 +1771,26 @@ struct BwdJob {
   RedJob red;
   int L, Cs;
   int* ticket;
-  __nv_bfloat16* gS[2];
-  float *gz[2], *rowstat[2];
-  uint8_t* img[2];
-  int *gflag[2], *kvread[2];
+  // hand-off ring: slot k (slice n uses n % ring) holds, at hand + k hand_slot,
+  // G_t(S) bf16 [chains][nt][M][64], then g_t(z), the row statistics and the
+  // tile images at the given offsets; its two flag arrays (gflag, kvread) are
+  // hflag + (2k, 2k+1) * chains * nt * FLAG_STRIDE
+  uint8_t* hand;
+  size_t hand_slot, off_gz, off_rs, off_img;
+  int ring;
+  int* hflag;
   float* acc;       // [2 sides][chains][nt][M*64] per-position dOmega sums
   int* accflag[2];  // [chains][nt] per side
   int *sums_done, *r1done;  // slice-0 tiles done, final stage-1 CTAs done
 };
 
-template <int MF, int FEAT>
+// EARLY (stages of at least EARLY_STAGE items): the flags a tile waits on were
+// set long before it starts, so it polls them up front, and the dq side
+// releases the hand-off once it is done, off the G chain's path.  With shorter
+// stages, tiles of neighbouring slices run at the same time: the running-sum
+// flags are then polled just before the adds and the hand-off is released in
+// the G chain, so that no tile waits for another one to finish.
+template <int MF, int FEAT, bool EARLY>
 __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJob J) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t mbar[NBAR];
@@ -1779,42 +1805,47 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
     const int a = n * J.Cs, b = min(J.Cs, J.L - a), ntn = (b + T - 1) / T;
     const int n1 = n + 1 < N ? (n + 1 == N - 1 ? J.s.ntl : J.s.nt) : 0;
     const size_t side = (size_t)J.s.chains * J.s.nt * MF * D;
+    const size_t tiles = (size_t)J.s.chains * J.s.nt;
+    const int slot = n % J.ring;
+    uint8_t* hs = J.hand + slot * J.hand_slot;
+    int* hf = J.hflag + (size_t)(2 * slot) * tiles * FLAG_STRIDE;
     if (it.kind == IT_Q) {
       BwdQJob q = J.q;
       q.a = a;
       q.b = b;
       q.ntn = ntn;
       q.n = n;
-      q.gS = J.gS[n & 1];
-      q.gz = J.gz[n & 1];
-      q.rowstat = J.rowstat[n & 1];
-      q.gflag = J.gflag[n & 1];
-      q.img = J.img[n & 1];
-      q.kvread = J.kvread[n & 1];
-      q.n2tiles = n + 2 < N ? (n + 2 == N - 1 ? J.s.ntl : J.s.nt) : 0;
+      q.gS = reinterpret_cast<__nv_bfloat16*>(hs);
+      q.gz = reinterpret_cast<float*>(hs + J.off_gz);
+      q.rowstat = reinterpret_cast<float*>(hs + J.off_rs);
+      q.img = hs + J.off_img;
+      q.gflag = hf;
+      q.kvread = hf + tiles * FLAG_STRIDE;
+      q.ring = J.ring;
+      q.nRtiles = n + J.ring < N ? (n + J.ring == N - 1 ? J.s.ntl : J.s.nt) : 0;
       q.acc = J.acc;
       q.accflag = J.accflag[0];
       q.n1tiles = n1;
       q.sums_done = n == 0 ? J.sums_done : nullptr;
-      role_bwd_q<MF, FEAT>(q, it.idx, smem_raw, mbar, tmem_base, abort_);
+      role_bwd_q<MF, FEAT, EARLY>(q, it.idx, smem_raw, mbar, tmem_base, abort_);
     } else {
       BwdKVJob kv = J.kv;
       kv.a = a;
       kv.b = b;
       kv.ntn = ntn;
       kv.n = n;
-      kv.gS = J.gS[n & 1];
-      kv.gz = J.gz[n & 1];
-      kv.rowstat = J.rowstat[n & 1];
-      kv.gflag = J.gflag[n & 1];
-      kv.img = J.img[n & 1];
-      kv.kvread = J.kvread[n & 1];
+      kv.gS = reinterpret_cast<const __nv_bfloat16*>(hs);
+      kv.gz = reinterpret_cast<const float*>(hs + J.off_gz);
+      kv.rowstat = reinterpret_cast<const float*>(hs + J.off_rs);
+      kv.img = hs + J.off_img;
+      kv.gflag = hf;
+      kv.kvread = hf + tiles * FLAG_STRIDE;
       kv.acc = J.acc + side;
       kv.accflag = J.accflag[1];
       kv.n1tiles = n1;
       kv.sums_done = n == 0 ? J.sums_done : nullptr;
       // the dq side's order: last tile first, chains inside a position
-      role_bwd_kv<MF, FEAT>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains, smem_raw, mbar,
+      role_bwd_kv<MF, FEAT, EARLY>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains, smem_raw, mbar,
                             tmem_base, abort_);
     }
     return;
@@ -1869,24 +1900,37 @@ Geo geometry(const Problem& p) {
 
 // The chain slots hold one prefix per (chain, tile of a slice): a slice's
 // tiles overwrite the previous slice's only after reading them.  The buffers
-// the dq side hands to the dk/dv side have two slots (slice n uses n % 2),
-// because the dq side of slice n-1 runs beside the dk/dv side of slice n.
+// the dq side hands to the dk/dv side form a ring of R slots (slice n uses
+// n % R): the dq side of slice n-R reuses a slot once slice n's dk/dv side has
+// read it.  R is at least 2 (the dq side of slice n-1 runs beside the dk/dv
+// side of slice n) and large enough that those two items are KV_LEAD tickets
+// apart, so that the wait is almost never taken even when slices are short.
 // dOmega is summed per (side, chain, tile position) over the slices and
 // reduced once at the end.
+constexpr int KV_LEAD = 320;  // about two waves of tile CTAs
+constexpr int MAX_RING = 16;
+constexpr int EARLY_STAGE = 128;  // see k_tc_bwd
+int handoff_ring(const Geo& g) {
+  const int stage = 2 * g.chains * g.nt;  // items of a full stage
+  const int r = 1 + (KV_LEAD + stage - 1) / stage;
+  return r < 2 ? 2 : (r > MAX_RING ? MAX_RING : r);
+}
 struct Ws {
   int* err;
   int* flags;  // every flag and counter of the call, zeroed together
   int nflags;
   int *flag1, *flag2;         // [chains][nt] chain flags, FLAG_STRIDE ints each
-  int *gflag[2], *kvread[2];  // [chains][nt] hand-off flags (backward)
+  int* hflag;                 // [ring][2][chains][nt] hand-off flags (backward)
   int* accflag[2];            // [chains][nt] per side: dOmega sums (backward)
   int *sums_done, *r1done;    // final reduction counters (backward)
   int* ticket;
   __nv_bfloat16* om16;
   float *slot1, *slot2;
-  __nv_bfloat16* gS[2];
-  float *gz[2], *rowstat[2];
-  uint8_t* img[2];  // [chains][nt]: phiQ, phiK (T x M bf16 each) and tril(A) (T x T bf16)
+  // hand-off ring (see BwdJob): per slot G_t(S), g_t(z), the row statistics
+  // and per tile phiQ, phiK (T x M bf16 each) and tril(A) (T x T bf16)
+  uint8_t* hand;
+  size_t hand_slot, off_gz, off_rs, off_img;
+  int ring;
   float* acc;    // [2 sides][chains][nt][M*64]
   float* rsums;  // [RS1][M*64]
 };
@@ -1895,18 +1939,16 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   Ws w{};
   const size_t C = g.chains, tiles = C * g.nt, FS = FLAG_STRIDE;
   w.err = cv.take<int>(64);
-  w.nflags = (int)((bwd ? 8 * tiles + 2 : 2 * tiles) * FS + FS);
+  w.ring = bwd ? handoff_ring(g) : 0;
+  w.nflags = (int)((bwd ? (4 + 2 * (size_t)w.ring) * tiles + 2 : 2 * tiles) * FS + FS);
   w.flags = cv.take<int>(w.nflags);
   int* f = w.flags;
   w.flag1 = f;
   w.flag2 = f + tiles * FS;
   f += 2 * tiles * FS;
   if (bwd) {
-    for (int k = 0; k < 2; ++k) {
-      w.gflag[k] = f;
-      w.kvread[k] = f + tiles * FS;
-      f += 2 * tiles * FS;
-    }
+    w.hflag = f;
+    f += 2 * (size_t)w.ring * tiles * FS;
     for (int k = 0; k < 2; ++k) {
       w.accflag[k] = f;
       f += tiles * FS;
@@ -1920,12 +1962,12 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   w.slot1 = cv.take<float>(tiles * g.E);
   if (bwd) {
     w.slot2 = cv.take<float>(tiles * g.E);
-    for (int k = 0; k < 2; ++k) {
-      w.gS[k] = cv.take<__nv_bfloat16>(tiles * g.MF * D);
-      w.gz[k] = cv.take<float>(tiles * g.MF);
-      w.rowstat[k] = cv.take<float>(tiles * T * 2);
-      w.img[k] = cv.take<uint8_t>(tiles * ((size_t)4 * T * g.MF + 2 * T * T));
-    }
+    // byte offsets inside a slot (all multiples of 16)
+    w.off_gz = tiles * g.MF * D * 2;
+    w.off_rs = w.off_gz + tiles * g.MF * 4;
+    w.off_img = w.off_rs + tiles * T * 2 * 4;
+    w.hand_slot = (w.off_img + tiles * ((size_t)4 * T * g.MF + 2 * T * T) + 255) & ~size_t(255);
+    w.hand = cv.take<uint8_t>(w.ring * w.hand_slot);
     w.acc = cv.take<float>(2 * tiles * (size_t)g.MF * D);
     w.rsums = cv.take<float>((size_t)RS1 * g.MF * D);
   }
@@ -1954,7 +1996,10 @@ cudaError_t configure() {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem_fwd<MF>());
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem_bwd<MF>());
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem_bwd<MF>());
   if (e != cudaSuccess) return e;
   done = true;
@@ -2062,22 +2107,21 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
   J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
                 w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
-                0, nullptr, nullptr, 0, nullptr, dq, w.err};
+                0, 0, nullptr, nullptr, 0, nullptr, dq, w.err};
   J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                   p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
   J.red = RedJob{w.acc, 2 * g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
   J.L = p.L;
   J.Cs = g.Cs;
   J.ticket = w.ticket;
-  for (int x = 0; x < 2; ++x) {
-    J.gS[x] = w.gS[x];
-    J.gz[x] = w.gz[x];
-    J.rowstat[x] = w.rowstat[x];
-    J.gflag[x] = w.gflag[x];
-    J.img[x] = w.img[x];
-    J.kvread[x] = w.kvread[x];
-    J.accflag[x] = w.accflag[x];
-  }
+  J.hand = w.hand;
+  J.hand_slot = w.hand_slot;
+  J.off_gz = w.off_gz;
+  J.off_rs = w.off_rs;
+  J.off_img = w.off_img;
+  J.ring = w.ring;
+  J.hflag = w.hflag;
+  for (int x = 0; x < 2; ++x) J.accflag[x] = w.accflag[x];
   J.acc = w.acc;
   J.sums_done = w.sums_done;
   J.r1done = w.r1done;
@@ -2086,7 +2130,12 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
   const long long items = sched_items(J.s);
   prof::Scope ps(prof::K_TC_BWD, s, rows * 22.0 * MD, rows * D * 2.0 * 12);
-  TC_TRY(launch_dep(k_tc_bwd<MF, FEAT>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(), s, J));
+  if (2 * g.chains * g.nt >= EARLY_STAGE)
+    TC_TRY(launch_dep(k_tc_bwd<MF, FEAT, true>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(), s,
+                      J));
+  else
+    TC_TRY(launch_dep(k_tc_bwd<MF, FEAT, false>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(),
+                      s, J));
   return SLIM_OK;
 }
 
@@ -2102,8 +2151,9 @@ size_t workspace_bytes(const Problem& p, bool bwd) {
   return cv.bytes();
 }
 
-int bwd_schedule(const Problem& p, int* items, int cap) {
+int bwd_schedule(const Problem& p, int* items, int cap, int* ring) {
   const Geo g = geometry(p);
+  if (ring) *ring = handoff_ring(g);
   BwdSched sc{};
   sc.N = g.N;
   sc.chains = g.chains;

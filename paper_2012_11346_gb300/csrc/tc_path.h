@@ -9,8 +9,9 @@ namespace tc {
 bool supports(const Problem& p);
 size_t workspace_bytes(const Problem& p, bool bwd);
 // The backward launch's item order: items[3 x] = (role, slice, index) of
-// ticket x, for x < min(count, cap).  Returns the item count.
-int bwd_schedule(const Problem& p, int* items, int cap);
+// ticket x, for x < min(count, cap), and (if ring is not null) the number of
+// hand-off ring slots.  Returns the item count.
+int bwd_schedule(const Problem& p, int* items, int cap, int* ring);
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
                 const float* omega, void* out, const StateOut& st, void* workspace,

@@ -36,7 +36,8 @@ SIGNATURES = {
     "slim_profiler_read": ([_p, _i], _i),
     "slim_tc_selftest": ([_i, _i, _i, _i, _p, _p, _p, _p, _p], _i),
     "slim_path_for": ([_i] * 6 + [_i, _i, ctypes.POINTER(_i)], _i),
-    "slim_bwd_schedule": ([_i] * 6 + [_i, _i, _p, _i, ctypes.POINTER(_i)], _i),
+    "slim_bwd_schedule": ([_i] * 6 + [_i, _i, _p, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)],
+                          _i),
     "slim_fwd_noalloc": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 5 + [_p], _i),
     "slim_diag_wait_timeout": ([_p, _p], _i),
 }
@@ -102,16 +103,16 @@ def path_for(B, H, L, d, M, C, dtype, feature):
 
 
 def bwd_schedule(B, H, L, d, M, C, dtype, feature):
-    """The tensor-core backward's item order: a list of (role, slice, index)
-    per ticket (roles 0 dq side, 1 dk/dv side, 2 and 3 the final dOmega
-    reduction stages)."""
-    lib, n = library(), _i(0)
+    """The tensor-core backward's item order and hand-off ring depth R: a list
+    of (role, slice, index) per ticket (roles 0 dq side, 1 dk/dv side, 2 and 3
+    the final dOmega reduction stages), and R."""
+    lib, n, ring = library(), _i(0), _i(0)
     _check(lib.slim_bwd_schedule(B, H, L, d, M, C, DTYPES[dtype], FEATURES[feature], None, 0,
-                                 ctypes.byref(n)), "slim_bwd_schedule")
+                                 ctypes.byref(n), None), "slim_bwd_schedule")
     buf = (_i * (3 * n.value))()
     _check(lib.slim_bwd_schedule(B, H, L, d, M, C, DTYPES[dtype], FEATURES[feature], buf, n.value,
-                                 ctypes.byref(n)), "slim_bwd_schedule")
-    return [tuple(buf[3 * x:3 * x + 3]) for x in range(n.value)]
+                                 ctypes.byref(n), ctypes.byref(ring)), "slim_bwd_schedule")
+    return [tuple(buf[3 * x:3 * x + 3]) for x in range(n.value)], ring.value
 
 
 def _stream_handle(stream):

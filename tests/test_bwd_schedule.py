@@ -24,7 +24,11 @@ SHAPES = [(8, 8, 4096, 1024), (2, 2, 1000, 320), (2, 3, 700, 64), (1, 1, 8192, 1
 
 
 def schedule(B, H, L, C, M=256):
-    return slim.bwd_schedule(B, H, L, 64, M, C, torch.bfloat16, "exp")
+    return slim.bwd_schedule(B, H, L, 64, M, C, torch.bfloat16, "exp")[0]
+
+
+def ring(B, H, L, C, M=256):
+    return slim.bwd_schedule(B, H, L, 64, M, C, torch.bfloat16, "exp")[1]
 
 
 def geometry(B, H, L, C):
@@ -42,6 +46,7 @@ def tile_item(ntn, ch, n, t, c):
 def dependencies(B, H, L, C, items):
     """For every ticket, the tickets of the items its waits stand for."""
     ch, N, ntn = geometry(B, H, L, C)
+    R = ring(B, H, L, C)
     ticket = {it: x for x, it in enumerate(items)}
     r1n = sum(1 for it in items if it[0] == R1)
     deps = []
@@ -54,8 +59,8 @@ def dependencies(B, H, L, C, items):
                     d.append(ticket[(Q, n, tile_item(ntn, ch, n, t + 1, c))])
                 elif n + 1 < N:
                     d.append(ticket[(Q, n + 1, tile_item(ntn, ch, n + 1, 0, c))])
-                if n + 2 < N and t < ntn[n + 2]:  # hand-off buffers of parity n % 2
-                    d.append(ticket[(KV, n + 2, tile_item(ntn, ch, n + 2, t, c))])
+                if n + R < N and t < ntn[n + R]:  # hand-off ring slot n % R
+                    d.append(ticket[(KV, n + R, tile_item(ntn, ch, n + R, t, c))])
             else:
                 d.append(ticket[(Q, n, tile_item(ntn, ch, n, t, c))])  # its dq side
             if n + 1 < N and t < ntn[n + 1]:  # the dOmega sum at this position
@@ -94,6 +99,19 @@ def test_waits_are_on_lower_tickets(shape):
         assert all(y < x for y in d), (x, items[x])
 
 
+@pytest.mark.parametrize("shape", SHAPES)
+def test_ring_keeps_the_reuse_wait_far_back(shape):
+    # the dq side of slice n-R waits on slice n's dk/dv side: at least 320
+    # tickets apart (about two waves of tile CTAs), R in [2, 16]
+    B, H, L, C = shape
+    ch, N, ntn = geometry(B, H, L, C)
+    R = ring(B, H, L, C)
+    assert 2 <= R <= 16
+    stage = 2 * ch * ntn[0]
+    assert (R - 1) * stage >= 320 or R == 16
+    assert R == 2 or (R - 2) * stage < 320
+
+
 def test_stage_order():
     # stage j: dq side of slice N-1-j and dk/dv side of slice N-j, alternating by
     # rows of B*H tiles (dq first); a dk/dv tile comes a stage after its dq tile
@@ -116,9 +134,10 @@ def progress(shape, resident, seed):
     nt = ntn[0]
     items = schedule(B, H, L, C)
     deps = dependencies(B, H, L, C, items)
+    R = ring(B, H, L, C)
     r1n = sum(1 for it in items if it[0] == R1)
     flag1, flag2 = {}, {}
-    gflag, kvread, accflag = [{}, {}], [{}, {}], [{}, {}]
+    gflag, kvread, accflag = [{} for _ in range(R)], [{} for _ in range(R)], [{}, {}]
     sums_done = r1done = 0
     done = [False] * len(items)
 
@@ -132,10 +151,10 @@ def progress(shape, resident, seed):
                 if inner or n + 1 < N:
                     snext, want = (t + 1, n + 1) if inner else (0, n + 2)
                     ok &= flag1.get((c, snext), 0) == want and flag2.get((c, snext), 0) == want
-                if n + 2 < N and t < ntn[n + 2]:
-                    ok &= kvread[n % 2].get((c, t), 0) == n + 3
+                if n + R < N and t < ntn[n + R]:
+                    ok &= kvread[n % R].get((c, t), 0) == n + R + 1
             else:
-                ok &= gflag[n % 2].get((c, t), 0) == n + 1
+                ok &= gflag[n % R].get((c, t), 0) == n + 1
             if n + 1 < N and t < ntn[n + 1]:
                 ok &= accflag[kind].get((c, t), 0) == n + 2
             return ok
@@ -157,9 +176,9 @@ def progress(shape, resident, seed):
         if kind in (Q, KV):
             c, t = idx % ch, ntn[n] - 1 - idx // ch
             if kind == Q:
-                flag1[(c, t)] = flag2[(c, t)] = gflag[n % 2][(c, t)] = n + 1
+                flag1[(c, t)] = flag2[(c, t)] = gflag[n % R][(c, t)] = n + 1
             else:
-                kvread[n % 2][(c, t)] = n + 1
+                kvread[n % R][(c, t)] = n + 1
             accflag[kind][(c, t)] = n + 1
             sums_done += n == 0
         elif kind == R1:
