@@ -226,40 +226,6 @@ __device__ __forceinline__ void red_release_gpu(int* p, int v) {
 // share a cache line.
 constexpr int FLAG_STRIDE = 32;
 
-// Thread 0 waits for *flag == want; every thread learns the outcome.  The
-// wait is bounded (2^22 polls, ~1 s with the back-off) and stops early once
-// another CTA has reported an error (checked every 64 polls, so that the
-// waiting CTAs do not all hammer the error word); a failed wait records
-// itself in *err.
-__device__ __forceinline__ bool chain_acquire(const int* flag, int want, int* err, int& abort_) {
-  if (threadIdx.x == 0) {
-    bool ok = false;
-    for (uint32_t i = 0; i < (1u << 22); ++i) {
-      if (ld_relaxed_gpu(flag) == want) {
-        fence_acq_rel_gpu();
-        ok = true;
-        break;
-      }
-      if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) break;
-      __nanosleep(i < 16 ? 32 : 256);
-    }
-    if (!ok) {
-      atomicExch(err, 1);
-      abort_ = 1;
-    }
-  }
-  __syncthreads();
-  return abort_ == 0;
-}
-
-// Publishes the slot under its flag.  The barrier orders every thread's slot
-// writes before thread 0's release store, which (being cumulative) makes them
-// visible at GPU scope before the flag.
-__device__ __forceinline__ void chain_release(int* flag, int val) {
-  __syncthreads();
-  if (threadIdx.x == 0) st_release_gpu(flag, val);
-}
-
 // Buffers exchanged between tile CTAs (prefix slots, dOmega partials, G_t)
 // are "lane-major": the 16 values a thread owns in an epilogue (row m = 128h +
 // row, columns 16cg..16cg+15 of an [M][64] matrix) are spread over four float4
@@ -375,7 +341,11 @@ __device__ __forceinline__ void group_publish(int id) {
   group_bar(id);
   tc_fence_after();
 }
-// Bounded poll of a chain flag by one thread (see chain_acquire).
+// Bounded poll of a flag by one thread: returns once *flag == want (then an
+// acquire fence).  It gives up after 2^22 polls (~1 s with the back-off), or
+// early once another CTA has reported an error (checked every 64 polls, so
+// that waiting CTAs do not all hammer the error word); a wait that gives up
+// records itself in *err.
 __device__ __forceinline__ bool flag_poll(const int* flag, int want, int* err) {
   for (uint32_t i = 0; i < (1u << 22); ++i) {
     if (ld_relaxed_gpu(flag) == want) {
@@ -1496,56 +1466,6 @@ struct RedJob {
   float* domega;      // [M][64]
   int n;              // M * 64
 };
-
-__device__ __forceinline__ void reduce_stage1(const RedJob& J, int r) {
-  const int per = (J.nparts + J.nsums - 1) / J.nsums;
-  const int i0 = min(J.nparts, r * per), i1 = min(J.nparts, i0 + per);
-  const int n4 = J.n / 4, tid = threadIdx.x;
-  constexpr int QMAX = 256 * 64 / 4 / NTHR;  // float4 per thread at M = 256
-  float4 acc[QMAX];
-#pragma unroll
-  for (int k = 0; k < QMAX; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-  // partials in order; two at a time so that 2 * QMAX loads are in flight
-  int i = i0;
-  for (; i + 1 < i1; i += 2) {
-    const float4* s0 = reinterpret_cast<const float4*>(J.part + (size_t)i * J.n);
-    const float4* s1 = reinterpret_cast<const float4*>(J.part + (size_t)(i + 1) * J.n);
-    float4 x0[QMAX], x1[QMAX];
-#pragma unroll
-    for (int k = 0; k < QMAX; ++k) {
-      const int q = tid + k * NTHR;
-      x0[k] = q < n4 ? __ldcg(s0 + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-      x1[k] = q < n4 ? __ldcg(s1 + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll
-    for (int k = 0; k < QMAX; ++k) {
-      acc[k].x = (acc[k].x + x0[k].x) + x1[k].x;
-      acc[k].y = (acc[k].y + x0[k].y) + x1[k].y;
-      acc[k].z = (acc[k].z + x0[k].z) + x1[k].z;
-      acc[k].w = (acc[k].w + x0[k].w) + x1[k].w;
-    }
-  }
-  if (i < i1) {
-    const float4* s0 = reinterpret_cast<const float4*>(J.part + (size_t)i * J.n);
-#pragma unroll
-    for (int k = 0; k < QMAX; ++k) {
-      const int q = tid + k * NTHR;
-      if (q < n4) {
-        const float4 x = __ldcg(s0 + q);
-        acc[k].x += x.x;
-        acc[k].y += x.y;
-        acc[k].z += x.z;
-        acc[k].w += x.w;
-      }
-    }
-  }
-  float4* dst = reinterpret_cast<float4*>(J.sums + (size_t)r * J.n);
-#pragma unroll
-  for (int k = 0; k < QMAX; ++k) {
-    const int q = tid + k * NTHR;
-    if (q < n4) __stcg(dst + q, acc[k]);
-  }
-}
 
 // Stage 1 streaming its positions through shared memory: NSLOT slots of one
 // position each, filled by bulk copies (one thread, mbarrier per slot), so

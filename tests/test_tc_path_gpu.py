@@ -56,9 +56,9 @@ def test_tc_matches_fp32_path(cuda_device, monkeypatch):
         assert oracle.rel_l2(to64(a[n]), to64(b[n])) <= TOL["bf16"], n
 
 
-def _run_case(cuda_device, B, H, L, C, seed=3):
-    w = W.Workload("tc", B, H, L, 64, 256, C, "bf16", "exp", "normal", "orthogonal", seed=seed)
-    assert slim.path_for(B, H, L, 64, 256, C, torch.bfloat16, "exp") == 1
+def _run_case(cuda_device, B, H, L, C, seed=3, M=256):
+    w = W.Workload("tc", B, H, L, 64, M, C, "bf16", "exp", "normal", "orthogonal", seed=seed)
+    assert slim.path_for(B, H, L, 64, M, C, torch.bfloat16, "exp") == 1
     x = W.make_inputs(w, device=cuda_device)
     compare(gpu_run(x, C, "exp"), oracle_run(cpu_inputs(x), C, "exp"), TOL["bf16"],
             where=f"tc B{B} H{H} L{L} C{C}")
@@ -74,6 +74,27 @@ def test_tc_many_short_chains(cuda_device):
     """256 chains of 2 tiles, one tile per slice: hand-offs across slice
     boundaries only."""
     _run_case(cuda_device, 16, 16, 256, 128)
+
+
+def _ring(B, H, L, C, M):
+    return slim.bwd_schedule(B, H, L, 64, M, C, torch.bfloat16, "exp")[1]
+
+
+def test_tc_handoff_ring_wraps_short_stages(cuda_device):
+    """Two chains of one-tile slices: stages of 4 items, so the running-sum
+    flags are polled just before the adds, and the 16-slot hand-off ring is
+    reused over 32 slices (each dq tile of slice n waits for slice n+16's
+    dk/dv tile to have read its slot)."""
+    assert _ring(1, 2, 4096, 128, 256) == 16
+    _run_case(cuda_device, 1, 2, 4096, 128)
+
+
+def test_tc_handoff_ring_wraps_long_stages(cuda_device):
+    """64 chains of one-tile slices of 64 rows: stages of 128 items, so the
+    flags are polled up front and the hand-off is released after the last
+    join, and the 4-slot ring is reused (5 slices)."""
+    assert _ring(4, 16, 320, 64, 128) == 4
+    _run_case(cuda_device, 4, 16, 320, 64, M=128)
 
 
 def test_tc_workspace_reuse(cuda_device):
