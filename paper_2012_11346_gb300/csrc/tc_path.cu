@@ -130,12 +130,17 @@ __device__ __forceinline__ float group_total(const float* red, int row) {
 }
 
 // 16 fp32 values -> 16 bf16 at global dst (32 bytes, 16-byte aligned).
+// 16 values of an output row (out, dq, dk, dv: never read back here), so
+// evict-first in L2.
 __device__ __forceinline__ void st_row16(__nv_bfloat16* dst, const float* v) {
-  uint4* d = reinterpret_cast<uint4*>(dst);
-  d[0] = make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
-                    pack_bf16(v[6], v[7]));
-  d[1] = make_uint4(pack_bf16(v[8], v[9]), pack_bf16(v[10], v[11]), pack_bf16(v[12], v[13]),
-                    pack_bf16(v[14], v[15]));
+  const uint64_t pol = l2_evict_first();
+#pragma unroll
+  for (int h = 0; h < 2; ++h)
+    asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(dst + 8 * h),
+                 "r"(pack_bf16(v[8 * h], v[8 * h + 1])), "r"(pack_bf16(v[8 * h + 2], v[8 * h + 3])),
+                 "r"(pack_bf16(v[8 * h + 4], v[8 * h + 5])), "r"(pack_bf16(v[8 * h + 6], v[8 * h + 7])),
+                 "l"(pol)
+                 : "memory");
 }
 __device__ __forceinline__ void st_f32x16(float* dst, const float* v) {
   float4* o = reinterpret_cast<float4*>(dst);
@@ -234,18 +239,18 @@ constexpr int FLAG_STRIDE = 32;
 __device__ __forceinline__ size_t lm4(int h, int cg, int i, int row) {
   return (size_t)((h * NG + cg) * 4 + i) * 128 + row;
 }
-// 16 floats through L2 (the data is written by other CTAs of the same
-// kernel, so L1 must not serve stale lines).
+// 16 floats of a chain prefix through L2 (the data is written by other CTAs
+// of the same kernel, so L1 must not serve stale lines).  A prefix is read
+// once, by the next tile of its chain: evict-first in L2.
 __device__ __forceinline__ void ld_lm16(const float* base, int h, int cg, int row, float* v) {
   const float4* s = reinterpret_cast<const float4*>(base);
+  const uint64_t pol = l2_evict_first();
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float4 x = __ldcg(s + lm4(h, cg, i, row));
-    v[4 * i] = x.x;
-    v[4 * i + 1] = x.y;
-    v[4 * i + 2] = x.z;
-    v[4 * i + 3] = x.w;
-  }
+  for (int i = 0; i < 4; ++i)
+    asm volatile("ld.global.cg.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=f"(v[4 * i]), "=f"(v[4 * i + 1]), "=f"(v[4 * i + 2]), "=f"(v[4 * i + 3])
+                 : "l"(s + lm4(h, cg, i, row)), "l"(pol)
+                 : "memory");
 }
 __device__ __forceinline__ void st_lm16(float* base, int h, int cg, int row, const float* v) {
   float4* d = reinterpret_cast<float4*>(base);
