@@ -37,6 +37,10 @@ L2_BYTES = 129 * 1024 * 1024
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # FP32 FMA issue rate: 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz (maximum SM clock)
 FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+# MUFU exponentials: ex2.approx.f32 measured on this machine's GB300 with 8
+# independent chains per thread over 1216 CTAs of 256 threads: 9.5e12 per
+# second, 30 per clock per SM at 2070 MHz
+MUFU_EX2_PER_S = 9.5e12
 
 # roofline bound of each kernel: (bound, which algorithmic quantity)
 KERNEL_BOUND = {
@@ -236,6 +240,31 @@ def roofline(stats, steps):
             "share_of_kernel_time": round(top["total_ms"] / total_ms, 4) if total_ms else None}
 
 
+def step_ceilings(w, B, H, L, ms_per_step):
+    """The three floors of one fwd+bwd step from its algorithmic work per
+    token-head: 30dM FLOPs (on the tensor pipe for bf16, the FP32 FMA pipe
+    otherwise), 12ds HBM bytes (s = element size) and 4M exponentials (exp
+    features; none for ReLU), against the measured peaks."""
+    peaks, which = measured_peaks()
+    th = B * H * L
+    flops = 30.0 * w.d * w.M * th
+    s = 2 if w.dtype == "bf16" else 4
+    hbm_bytes = 12.0 * w.d * s * th
+    exps = 4.0 * w.M * th if w.feature == "exp" else 0.0
+    if w.dtype == "bf16":
+        compute_us, compute = flops / (peaks["bf16_tflops"] * 1e12) * 1e6, "tensor"
+    else:
+        compute_us, compute = flops / (FP32_ALU_TFLOPS * 1e12) * 1e6, "fp32 alu"
+    floors = {compute: compute_us, "hbm": hbm_bytes / (peaks["hbm_gbs"] * 1e9) * 1e6,
+              "mufu": exps / MUFU_EX2_PER_S * 1e6}
+    bound = max(floors, key=floors.get)
+    return {"floors_us": {k: round(v, 2) for k, v in floors.items()}, "bound": bound,
+            "t_star_us": round(floors[bound], 2),
+            "frac_of_step": round(floors[bound] / (ms_per_step * 1e3), 4),
+            "flops": flops, "hbm_bytes": hbm_bytes, "exps": exps,
+            "peak_source": f"{which} peaks; mufu {MUFU_EX2_PER_S:.2e}/s measured"}
+
+
 # ------------------------------------------------------------------ CPU oracle
 def _oracle_chain(args):
     """One chain's fp64 oracle fwd+bwd (runs in a spawned worker)."""
@@ -425,6 +454,7 @@ def run_ours(args, rank, ws, local):
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": int(launches),
         "roofline": roofline(stats, args.steps),
+        "ceilings": step_ceilings(w, B, H, L, ms / args.steps),
         "profiled_ms_per_step": round(ms_profiled / args.steps, 4),
         "clocks": clocks,
         "peak_mem": {"bytes": peak, "above_inputs_bytes": peak - base,
