@@ -139,3 +139,25 @@ def test_binding_refuses_cpu_tensors():
     x = torch.zeros(1, 1, 8, 16)
     with pytest.raises(RuntimeError):
         slim.forward(x, x, x, torch.zeros(32, 16), 4)
+
+
+def test_bwd_schedule_arguments(lib):
+    n, ring = ctypes.c_int(-1), ctypes.c_int(-1)
+    # count only (no buffer), then the tensor-core problems it serves
+    assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, None, 0, ctypes.byref(n),
+                                 ctypes.byref(ring)) == OK
+    assert n.value == 4 * 2 * 64 * 8 + 128 + 32 and ring.value == 2
+    buf = (ctypes.c_int * 6)()
+    assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, buf, 2, ctypes.byref(n),
+                                 None) == OK
+    assert list(buf) == [0, 3, 0, 0, 3, 1]  # the first two tickets: dq side of the last slice
+    # argument errors before anything else
+    assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, None, 0, None, None) == INVALID
+    assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, None, 4, ctypes.byref(n),
+                                 None) == INVALID
+    assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 0, 1, 0, None, 0, ctypes.byref(n),
+                                 None) == INVALID
+    # problems the tensor-core kernels do not take: fp32, d = 128, slices under 64 rows
+    for args in ((4, 12, 8192, 64, 128, 512, 0, 1), (1, 4, 65536, 128, 256, 16, 1, 0),
+                 (2, 8, 32768, 64, 256, 16, 1, 0)):
+        assert lib.slim_bwd_schedule(*args, None, 0, ctypes.byref(n), None) == UNSUPPORTED
