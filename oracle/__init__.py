@@ -6,7 +6,7 @@ calls it and shares no code with it; there is no CPU fallback through here.
 
 Modules
   features   -- the feature maps g (FAVOR+ exp, generalized ReLU) and VJPs
-  brute      -- eq. 2 written out row by row (O(L^2)); eq. 1 for comparison
+  brute      -- eq. 2 written out row by row (O(L^2))
   sliced     -- Algorithm 1 / Algorithm 2 for one layer: forward sweep, and
                 backward sweep with rollback (eq. 17) and G carry (eq. 18)
   iterative  -- the token-by-token recurrence of App. B (C = 1)
@@ -49,10 +49,12 @@ def oracle_fwd(q, k, v, omega, C, feature, S0=None, z0=None):
             S.reshape(B, H, M))
 
 
-def oracle_bwd(q, k, v, omega, dout, S_state, z_state, C, feature):
-    """Backward sweep from B^(N) = (S_state, z_state).  Returns dq, dk, dv
-    ([B,H,L,d]), domega ([M,d]) and a dict with the rolled-back state B^(0)
-    and the state gradient G^(0) (same layout as S_state / z_state)."""
+def oracle_bwd(q, k, v, omega, dout, S_state, z_state, C, feature, G_S=None, g_z=None):
+    """Backward sweep from B^(N) = (S_state, z_state), with the state gradient
+    G^(N) = (G_S, g_z) handed in by a later segment (zero if None; Sec. 3.3).
+    Returns dq, dk, dv ([B,H,L,d]), domega ([M,d]) and a dict with the
+    rolled-back state B^(0) and the state gradient G^(0) (same layout as
+    S_state / z_state)."""
     Q, (B, H) = _chains(q)
     K, _ = _chains(k)
     V, _ = _chains(v)
@@ -62,8 +64,10 @@ def oracle_bwd(q, k, v, omega, dout, S_state, z_state, C, feature):
     L, d = Q.shape[1], Q.shape[2]
     R_N = np.swapaxes(np.asarray(S_state, np.float64).reshape(B * H, M, d), 1, 2)
     S_N = np.asarray(z_state, np.float64).reshape(B * H, M)
+    G_R_N = None if G_S is None else np.swapaxes(np.asarray(G_S, np.float64).reshape(B * H, M, d), 1, 2)
+    G_S_N = None if g_z is None else np.asarray(g_z, np.float64).reshape(B * H, M)
     dQ, dK, dV, dOmega, (R0, S0), (G_R, G_S) = sliced.backward(
-        Q, K, V, Omega, dY, C, feature, R_N, S_N)
+        Q, K, V, Omega, dY, C, feature, R_N, S_N, G_R_N, G_S_N)
     extra = {
         "S0": np.swapaxes(R0, 1, 2).reshape(B, H, M, d),
         "z0": S0.reshape(B, H, M),

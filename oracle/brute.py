@@ -1,12 +1,10 @@
-"""Quadratic-time definitions (eqs. 1 and 2), fp64, for tiny inputs.
+"""Quadratic-time definition of eq. 2, fp64, for tiny inputs.
 
 ORACLE -- test infrastructure only; see oracle/__init__.py.
 
 att_lin_quadratic is the first form of eq. 2 written out row by row: for every
 position l, a weighted average of the values V_{l'} with l' <= l (inclusive
 causal mask, Sec. 2.1), the weight of l' being g(K_{l'})^T g(Q_l).
-att_exp_quadratic is eq. 1 (exponential self-attention); it is not the method,
-it only serves the FAVOR+ unbiasedness check.
 
 Shapes: Q, K, V are (chains, L, d); Omega is (M, d).
 """
@@ -30,14 +28,3 @@ def att_lin_quadratic(Q, K, V, Omega, feature):
                 Y[c, l] = (w[:, None] * V[c, : l + 1]).sum(axis=0) / den
     return Y
 
-
-def att_exp_quadratic(Q, K, V):
-    """Eq. 1: causal exponential (softmax) self-attention, for reference only."""
-    chains, L, d = V.shape
-    Y = np.zeros((chains, L, d))
-    for c in range(chains):
-        for l in range(L):
-            s = K[c, : l + 1] @ Q[c, l]
-            w = np.exp(s - s.max())
-            Y[c, l] = (w[:, None] * V[c, : l + 1]).sum(axis=0) / w.sum()
-    return Y

@@ -13,6 +13,11 @@ entries, M features per d-dimensional input.  Two instances are used here:
 * generalized ReLU random features:
       g(x)_m = max(omega_m . x, 0) / sqrt(M)
   with ReLU'(0) = 0.
+* the elementwise quadratic map of the paper's experiments (Sec. 4, with
+  M = d, and Sec. 2.1's remark that g can be elementwise):
+      g(x)_i = x_i^2,   i = 1..d
+  It has no random features: Omega is not used (only its shape, M = d, is
+  checked) and its gradient is zero.
 
 Omega is M x d and shared by every (batch, head) chain; its gradient is the sum
 over all chains and over both the query and the key side.
@@ -21,7 +26,7 @@ Arrays are float64.  X has shape (..., L, d), g(X) has shape (..., L, M).
 """
 import numpy as np
 
-FEATURES = ("exp", "relu")
+FEATURES = ("exp", "relu", "square")
 
 
 def projection(X, Omega):
@@ -42,11 +47,20 @@ def g_relu(X, Omega):
     return np.maximum(projection(X, Omega), 0.0) / np.sqrt(M)
 
 
+def g_square(X, Omega):
+    """Elementwise quadratic map (x_1^2, ..., x_d^2); M = d."""
+    if Omega.shape[0] != X.shape[-1]:
+        raise ValueError("the quadratic map has M = d features")
+    return X * X
+
+
 def feature_map(X, Omega, feature):
     if feature == "exp":
         return g_exp(X, Omega)
     if feature == "relu":
         return g_relu(X, Omega)
+    if feature == "square":
+        return g_square(X, Omega)
     raise ValueError(f"unknown feature map {feature!r}")
 
 
@@ -58,8 +72,13 @@ def feature_vjp(X, Omega, dG, feature):
     relu: dg_m/dx = 1[omega_m.x > 0] omega_m / sqrt(M)
                                               -> u = dG*1[.>0]/sqrt(M),
           dX = u Omega,                dOmega = sum_rows u^T x
+    square: dg_i/dx_i = 2 x_i (and 0 off the diagonal)
+                                              -> dX = 2 x * dG,  dOmega = 0
     dOmega is summed over every leading axis (all chains, all rows).
     """
+    if feature == "square":
+        g_square(X, Omega)  # shape check
+        return 2.0 * X * dG, np.zeros_like(Omega, dtype=np.float64)
     M = Omega.shape[0]
     if feature == "exp":
         u = dG * g_exp(X, Omega)

@@ -70,6 +70,20 @@ def _drop_key_normaliser_share(orig, R, S, G_R, G_S, Qt, Kt, V, dY):
     return dQt, dKt - dT_S, dV, R0, S0, G_R2, G_S2
 
 
+def _square_vjp_missing_two(X, Omega, dG, feature):
+    # mistake: quadratic map's derivative taken as x instead of 2x
+    if feature != "square":
+        return _orig_vjp(X, Omega, dG, feature)
+    return X * dG, np.zeros_like(Omega)
+
+
+def _g_abs(X, Omega):
+    # mistake: |x| in place of x^2 for the quadratic map
+    return np.abs(X)
+
+
+_orig_vjp = features.feature_vjp
+
 MUTATIONS = {
     "exclusive_mask": (lambda mp: mp.setattr(sliced, "_forward_rows", _exclusive_forward_rows),
                        lambda: P.pin_brute_vs_sliced("exp"), 1e-6),
@@ -88,6 +102,11 @@ MUTATIONS = {
     "key_grad_missing_normaliser": (
         lambda mp: mp.setattr(sliced, "_backward_rows", _wrap_backward_rows(_drop_key_normaliser_share)),
         lambda: P.pin_finite_differences("exp"), 1e-3),
+    "square_vjp_missing_factor_two": (
+        lambda mp: mp.setattr(sliced, "feature_vjp", _square_vjp_missing_two),
+        lambda: P.pin_finite_differences("square"), 1e-3),
+    "square_map_is_abs": (lambda mp: mp.setattr(features, "g_square", _g_abs),
+                          lambda: P.pin_golden(), 1e-6),
 }
 
 

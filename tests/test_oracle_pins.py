@@ -24,7 +24,9 @@ def small_case(seed, chains=2, L=40, d=4, M=None, feature="exp", scale=None):
     """Random fp64 inputs.  The ReLU map gets more features so that no row has
     an all-zero weight vector (eq. 2 needs a positive denominator)."""
     rng = np.random.default_rng(seed)
-    if M is None:
+    if feature == "square":
+        M = d            # the elementwise map has one feature per input coordinate
+    elif M is None:
         M = 6 if feature == "exp" else 24
     s = d ** -0.25 if scale is None else scale
     if feature == "relu":
@@ -230,6 +232,8 @@ def pin_autograd_brute(feature):
     tQ, tK, tV, tO = (torch.tensor(a, requires_grad=True) for a in (Q, K, V, Omega))
 
     def g(X):
+        if feature == "square":
+            return X * X
         p = X @ tO.T
         if feature == "exp":
             return torch.exp(p - 0.5 * (X * X).sum(-1, keepdim=True)) / math.sqrt(tO.shape[0])
@@ -240,13 +244,17 @@ def pin_autograd_brute(feature):
     (Y * torch.tensor(dY)).sum().backward()
     _, R, S = sliced.forward(Q, K, V, Omega, 6, feature)
     dQ, dK, dV, dO, _, _ = sliced.backward(Q, K, V, Omega, dY, 6, feature, R, S)
+    gO = tO.grad.numpy() if tO.grad is not None else np.zeros_like(Omega)
+    if feature == "square":  # Omega is not used: its gradient is zero
+        return max(rel(dQ, tQ.grad.numpy()), rel(dK, tK.grad.numpy()),
+                   rel(dV, tV.grad.numpy()), float(np.abs(dO).max()), float(np.abs(gO).max()))
     return max(rel(dQ, tQ.grad.numpy()), rel(dK, tK.grad.numpy()),
-               rel(dV, tV.grad.numpy()), rel(dO, tO.grad.numpy()))
+               rel(dV, tV.grad.numpy()), rel(dO, gO))
 
 
 # ----------------------------------------------------------------------------- tests
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_brute_vs_sliced(feature):
     assert pin_brute_vs_sliced(feature) < 1e-12
 
@@ -255,27 +263,27 @@ def test_zero_omega_closed_form():
     assert pin_zero_omega_closed_form() < 1e-13
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_final_state_closed_form(feature):
     assert pin_final_state_closed_form(feature) < 1e-13
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_recurrence_forward(feature):
     assert pin_recurrence_forward(feature) < 1e-12
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_recurrence_backward(feature):
     assert pin_recurrence_backward(feature) < 1e-11
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_finite_differences(feature):
     assert pin_finite_differences(feature) < 1e-6
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_rollback_closes(feature):
     assert pin_rollback_closes(feature) < 1e-12
 
@@ -284,7 +292,7 @@ def test_initial_state_gradient():
     assert pin_initial_state_gradient() < 1e-7
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_streaming_continuation(feature):
     assert pin_streaming_continuation(feature) < 1e-12
 
@@ -297,7 +305,7 @@ def test_relu_arccos_kernel():
     assert pin_relu_arccos() < 0.03
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_block_equals_whole(feature):
     assert pin_block_equals_whole(feature) < 1e-12
 
@@ -306,7 +314,7 @@ def test_golden_hand_examples():
     assert pin_golden() < 1e-12
 
 
-@pytest.mark.parametrize("feature", ["exp", "relu"])
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_autograd_cross_check(feature):
     assert pin_autograd_brute(feature) < 1e-10
 
@@ -344,3 +352,51 @@ def test_relu_zero_denominator_rows():
     assert np.all(Y[0, 3] == 0.0)
     dQ, dK, dV, dO, _, _ = sliced.backward(Q, K, V, Omega, dY, 2, "relu", R, S)
     assert np.all(np.isfinite(dQ)) and np.all(dQ[0, 3] == 0.0)
+
+
+def pin_square_map_closed_form():
+    """The quadratic map (Sec. 4): g(q).g(k) = sum_i q_i^2 k_i^2, so with every
+    key equal to e_1 (g(k) = e_1) each weight is q_{l,1}^2 and the output is the
+    plain causal mean of the values; and dOmega = 0 (no random features)."""
+    rng = np.random.default_rng(17)
+    L, d = 9, 3
+    Q = rng.standard_normal((1, L, d)) + 2.0
+    K = np.zeros((1, L, d))
+    K[..., 0] = 1.0
+    V = rng.standard_normal((1, L, d))
+    Y, _, _ = sliced.forward(Q, K, V, np.zeros((d, d)), 4, "square")
+    mean = np.cumsum(V[0], axis=0) / np.arange(1, L + 1)[:, None]
+    return rel(Y[0], mean)
+
+
+def test_square_map_closed_form():
+    assert pin_square_map_closed_form() < 1e-13
+
+
+def pin_streaming_backward(feature):
+    """Two segments: the backward of the later segment hands its G^(0) to the
+    backward of the earlier one as G^(N) (Sec. 3.3: G^(n) is the gradient with
+    respect to the state a segment starts from).  Gradients of the two calls
+    together equal the gradients of one call over the whole sequence."""
+    Q, K, V, Omega, dY = small_case(18, feature=feature)
+    rng = np.random.default_rng(19)
+    a, C = 23, 6
+    q, k, v, do = (x[:, None] for x in (Q, K, V, dY))     # [B, H=1, L, d]
+    o, S, z = oracle.oracle_fwd(q, k, v, Omega, C, feature)
+    full = oracle.oracle_bwd(q, k, v, Omega, do, S, z, C, feature)
+    _, S1, z1 = oracle.oracle_fwd(q[:, :, :a], k[:, :, :a], v[:, :, :a], Omega, C, feature)
+    _, S2, z2 = oracle.oracle_fwd(q[:, :, a:], k[:, :, a:], v[:, :, a:], Omega, C, feature, S1, z1)
+    late = oracle.oracle_bwd(q[:, :, a:], k[:, :, a:], v[:, :, a:], Omega, do[:, :, a:], S2, z2,
+                             C, feature)
+    early = oracle.oracle_bwd(q[:, :, :a], k[:, :, :a], v[:, :, :a], Omega, do[:, :, :a], S1, z1,
+                              C, feature, late[4]["G_S"], late[4]["g_z"])
+    errs = [rel(np.concatenate([early[i], late[i]], axis=2), full[i]) for i in range(3)]
+    errs.append(float(np.abs(early[3] + late[3] - full[3]).max()
+                      / max(np.abs(full[3]).max(), 1e-300)))
+    errs.append(rel(early[4]["G_S"], full[4]["G_S"]))
+    return max(errs)
+
+
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
+def test_streaming_backward(feature):
+    assert pin_streaming_backward(feature) < 1e-12
