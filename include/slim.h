@@ -21,10 +21,14 @@
  * caller-provided workspace, whose size grows with C, not with L.
  *
  * Feature maps g: R^d -> R_+^M (Omega is [M, d], shared by all chains):
- *     SLIM_FEAT_EXP  : g(x)_m = exp(omega_m.x - |x|^2/2) / sqrt(M)   (FAVOR+)
- *     SLIM_FEAT_RELU : g(x)_m = max(omega_m.x, 0) / sqrt(M), ReLU'(0) = 0
- * A row whose denominator is exactly 0 (possible only with the ReLU map)
- * gets output 0 and passes no gradient.
+ *     SLIM_FEAT_EXP    : g(x)_m = exp(omega_m.x - |x|^2/2) / sqrt(M)   (FAVOR+)
+ *     SLIM_FEAT_RELU   : g(x)_m = max(omega_m.x, 0) / sqrt(M), ReLU'(0) = 0
+ *     SLIM_FEAT_SQUARE : g(x)_i = x_i^2, M = d -- the elementwise map of the
+ *                        paper's experiments (Sec. 4).  Omega is not used (it
+ *                        may be NULL) and dOmega is zero (domega may be NULL).
+ * A row whose denominator is exactly 0 (possible with the ReLU map, and with
+ * the quadratic map for all-zero inputs) gets output 0 and passes no
+ * gradient.
  *
  * Conventions for every entry point
  *   - All tensor pointers are DEVICE pointers, contiguous, row-major, 16-byte
@@ -32,20 +36,36 @@
  *     tensors may be null.  q, k, v, out, dout, dq, dk, dv are [B, H, L, d] in `dtype`;
  *     omega and domega are [M, d] fp32; S_state is [B, H, M, d] fp32 and
  *     z_state is [B, H, M] fp32.
- *   - The caller owns every buffer.  The library allocates no device or host
- *     memory and never synchronises the device; all work is enqueued on
+ *   - The caller owns every buffer, and the library allocates no device
+ *     memory.  It never synchronises the device; all work is enqueued on
  *     `stream` (a cudaStream_t passed as void*; NULL is the legacy default
- *     stream).  Inputs must not be modified until that work completes.
+ *     stream).  Inputs must not be modified until that work completes, and a
+ *     workspace serves one call at a time.
  *   - Arguments are validated before anything is enqueued.  On any error
  *     nothing has been launched, except SLIM_ERR_CUDA (a launch failed part
  *     way; outputs are then undefined).
+ *   - Device-side waits (only the tensor-core kernels have any) are bounded
+ *     (about a second).  A wait that gives up makes its call leave early
+ *     (outputs undefined) and is reported as SLIM_ERR_TIMEOUT by the next
+ *     slim_fwd / slim_bwd / *_from call on the same workspace once the failed
+ *     work has finished, without blocking: that call then launches nothing.
+ *     For this the library pins and maps, on the first tensor-core call in a
+ *     process, one 4 KB page of its own static host memory
+ *     (cudaHostRegister), where the kernels count such failures; the call's
+ *     first kernel stores the counter's address in the workspace, so the
+ *     report adds no copy and no launch.  slim_check_device_error reads the
+ *     same failure by blocking instead.
  *   - 1 <= C; C > L behaves as C = L.  L % C != 0 gives a shorter last slice.
- *   - Outputs are written in `dtype` rounded to nearest even; the carried
- *     state is an fp32 value/error pair.  fp32 problems accumulate every
- *     contraction in compensated fp32 (error-free products and sums); bf16
- *     problems accumulate in fp32.
+ *   - Outputs are written in `dtype` rounded to nearest even.  The state
+ *     carried between slices depends on the kernels serving the problem (see
+ *     slim_path_for).  The fp32-compute kernels carry it as an fp32
+ *     value/error pair (TwoSum) and accumulate every contraction of fp32
+ *     problems in compensated fp32 (error-free products and sums); their
+ *     residual outputs (S_state_lo, z_state_lo) hold the pair's low part.
+ *     The tensor-core kernels (bf16) chain plain fp32 prefixes from tile to
+ *     tile, accumulate in fp32, and write zero residuals.
  *   - Supported: d in {16, 32, 64, 128}; M a multiple of 16 in [16, 256];
- *     dtype SLIM_F32 or SLIM_BF16; both feature maps.  Other combinations
+ *     dtype SLIM_F32 or SLIM_BF16; every feature map.  Other combinations
  *     return SLIM_ERR_UNSUPPORTED.
  */
 #ifndef SLIM_H_
@@ -67,7 +87,7 @@ typedef enum {
 } slim_status;
 
 typedef enum { SLIM_F32 = 0, SLIM_BF16 = 1 } slim_dtype;
-typedef enum { SLIM_FEAT_EXP = 0, SLIM_FEAT_RELU = 1 } slim_feature;
+typedef enum { SLIM_FEAT_EXP = 0, SLIM_FEAT_RELU = 1, SLIM_FEAT_SQUARE = 2 } slim_feature;
 
 /* Human-readable name of a status code (static storage, never NULL). */
 const char* slim_status_string(slim_status status);
@@ -99,10 +119,13 @@ slim_status slim_bwd_workspace_size(int B, int H, int L, int d, int M, int C,
  *   z_state   [B,H,M]   fp32, written: final state z^(N) = sum_j g(k_j).
  *   S_state_lo, z_state_lo  same shapes, written if non-NULL: the low-order
  *             residual of the carried fp32 value/error pair (state = S_state +
- *             S_state_lo to about 48 bits).  Passing them back to slim_bwd
- *             lets the rollback of eq. 17 start from the unrounded state; an
- *             fp32-rounded z^(N) alone perturbs the early rows' denominators,
- *             which are small next to z^(N), by ~6e-8 * z^(N).
+ *             S_state_lo to about 48 bits; zero from the tensor-core kernels).
+ *             Passing them back to slim_bwd lets the rollback of eq. 17 start
+ *             from the unrounded state.  For fp32 problems they are part of
+ *             the 1e-5 accuracy: an fp32-rounded z^(N) alone perturbs the
+ *             early rows' denominators, which are small next to z^(N), by
+ *             ~6e-8 * z^(N), and on long sequences that moves dq by about
+ *             2e-5 (rel-L2; B4 H12 L8192 d64 M128, ReLU map).
  *   workspace device scratch of at least slim_fwd_workspace_size() bytes,
  *             256-byte aligned; contents on entry are ignored.
  * L = 0 is valid and only zeroes S_state / z_state.
@@ -142,6 +165,55 @@ slim_status slim_bwd(const void* q, const void* k, const void* v, const float* o
                      void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * A sequence cut into segments, one call per segment (streaming).  The slice
+ * recurrence of Sec. 3.2 carries B^(n-1) into slice n (eq. 16), and the
+ * reverse sweep of Sec. 3.3 carries the state gradient G^(n) back into slice
+ * n (eq. 18, G^(N) = 0 only at the true end of the sequence).  These two
+ * entry points expose both carries at the ends of a call, so that calls on
+ * consecutive segments give the result of one call on the whole sequence:
+ *
+ *   slim_fwd_from: slim_fwd starting from the state B^(0) = (S_init, z_init)
+ *     instead of zero -- typically the S_state / z_state (and residuals) an
+ *     earlier segment's forward returned.  S_init [B,H,M,d] and z_init
+ *     [B,H,M] fp32, read-only, both NULL (zero state) or both given;
+ *     S_init_lo / z_init_lo optional residuals (NULL: zero), only with
+ *     S_init.  The outputs may alias the inputs (S_state == S_init updates a
+ *     running state in place).  The S_state it returns is the state after
+ *     the segment, including B^(0).
+ *
+ *   slim_bwd_from: slim_bwd with the incoming state gradient G^(N) =
+ *     (G_S_in [B,H,M,d], g_z_in [B,H,M] fp32, read-only; both NULL for zero)
+ *     -- the gradient of the later segments' loss with respect to this
+ *     segment's final state, i.e. the G_S_out / g_z_out of the later
+ *     segment's slim_bwd_from -- and returning G^(0) in G_S_out / g_z_out
+ *     (written if non-NULL, both or neither): the gradient with respect to
+ *     the state this segment started from, to hand to the previous segment.
+ *     S_state / z_state are this segment's final state as its slim_fwd_from
+ *     returned it; the rollback ends at this segment's B^(0).  The dOmega of
+ *     the segments add up to the whole sequence's.
+ *
+ * With all the extra pointers NULL they are slim_fwd and slim_bwd.
+ */
+slim_status slim_fwd_from(const void* q, const void* k, const void* v, const float* omega,
+                          int B, int H, int L, int d, int M, int C,
+                          slim_dtype dtype, slim_feature feature,
+                          const float* S_init, const float* z_init,
+                          const float* S_init_lo, const float* z_init_lo,
+                          void* out, float* S_state, float* z_state,
+                          float* S_state_lo, float* z_state_lo,
+                          void* workspace, size_t workspace_bytes, void* stream);
+slim_status slim_bwd_from(const void* q, const void* k, const void* v, const float* omega,
+                          const void* out, const void* dout,
+                          const float* S_state, const float* z_state,
+                          const float* S_state_lo, const float* z_state_lo,
+                          const float* G_S_in, const float* g_z_in,
+                          int B, int H, int L, int d, int M, int C,
+                          slim_dtype dtype, slim_feature feature,
+                          void* dq, void* dk, void* dv, float* domega,
+                          float* G_S_out, float* g_z_out,
+                          void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Which kernels serve this problem: *path = 1 for the tensor-core path
  * (tcgen05 MMAs, bf16 operands, fp32 accumulation; bf16 inputs with d = 64,
  * M in {128, 256} and slices of at least 64 rows), 0 for the fp32-compute
@@ -177,7 +249,8 @@ slim_status slim_bwd_schedule(int B, int H, int L, int d, int M, int C, slim_dty
 /*
  * Reads the device error word that bounded waits in the kernels set when they
  * give up, and clears it.  Copies 4 bytes from the workspace on `stream` and
- * synchronises that stream (this call, unlike the others, blocks).
+ * synchronises that stream (this call, unlike the others, blocks).  A failure
+ * it reports is not reported again by the next call on the workspace.
  * Returns SLIM_OK, SLIM_ERR_TIMEOUT, or SLIM_ERR_CUDA.
  */
 slim_status slim_check_device_error(void* workspace, void* stream);
@@ -224,10 +297,13 @@ slim_status slim_tc_selftest(int a_mn, int b_mn, int K, int N, const void* A, co
 /*
  * Diagnostic of the failure path (no counterpart in the paper): one warp
  * waits on an mbarrier that nothing arrives at.  The wait gives up after its
- * bounded number of polls (about a second), sets the error word at the start
- * of `workspace` (a workspace as passed to slim_fwd/slim_bwd, at least 256
- * bytes) and the kernel returns; slim_check_device_error then reports
- * SLIM_ERR_TIMEOUT.  Nothing faults and the context stays usable.
+ * time limit (about a second), sets the error word at the start of
+ * `workspace` (a workspace as passed to slim_fwd/slim_bwd, at least 256
+ * bytes) and the kernel returns.  Like slim_fwd/slim_bwd it takes part in the
+ * non-blocking report: once the kernel has finished, the next slim_fwd /
+ * slim_bwd on the same workspace returns SLIM_ERR_TIMEOUT (and launches
+ * nothing), or slim_check_device_error reports it by blocking.  Nothing
+ * faults and the context stays usable.
  */
 slim_status slim_diag_wait_timeout(void* workspace, void* stream);
 
@@ -243,13 +319,18 @@ slim_status slim_diag_wait_timeout(void* workspace, void* stream);
  * still passes every input and output (same arguments and rules as slim_fwd,
  * minus the workspace).
  *   - Allocates nothing: no cudaMalloc, cudaFree or other allocating call
- *     (keep the launch profiler off, it creates CUDA events when on).
+ *     (keep the launch profiler off, it creates CUDA events when on), and it
+ *     does not take part in the non-blocking timeout report (which pins a
+ *     host page on first use).
+ *   - CUDA loads a library's device code on a device lazily, and that load
+ *     reserves the array: the first libslim call that reaches a device does
+ *     it.  Make a first call on each device at start-up, outside any context
+ *     that must not allocate (and before any stream capture on the device).
  *   - Returns SLIM_ERR_WORKSPACE when the problem needs more scratch than
  *     SLIM_NOALLOC_SCRATCH_BYTES (compare slim_fwd_workspace_size); use
  *     slim_fwd with a caller workspace, or a smaller C or B*H, then.
  *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture on the device.
+ *     (cudaGetSymbolAddress) with that device current.
  *   - All calls share the one array and it keeps the last call's contents;
  *     the call clears, on its stream, what must start at zero.  Calls that
  *     overlap on the GPU (different streams, or several host threads) race

@@ -61,6 +61,16 @@ struct Carver {
   size_t bytes() const { return (off + 255) & ~size_t(255); }
 };
 
+// One-time, per-device set-up (kernel attributes such as the dynamic
+// shared-memory limit belong to the device that was current when they were
+// set).  Returns the current device's flag, or null when it cannot be told.
+constexpr int kMaxDevices = 64;
+inline bool* device_flag(bool (&flags)[kMaxDevices]) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  return &flags[dev];
+}
+
 struct Problem {
   int B, H, L, d, M, C;
   slim_dtype dtype;
@@ -77,6 +87,17 @@ struct StateOut {
 };
 struct StateIn {
   const float *S, *z, *S_lo, *z_lo;
+};
+// The state a forward sweep starts from, B^(0) (all null: zero), and the
+// state gradient a backward sweep starts from, G^(N) (null: zero), and
+// returns, G^(0) (null: not returned) -- the values a sequence cut into
+// segments hands from one call to the next (Sec. 3.2, eq. 16; Sec. 3.3, eq. 18).
+struct StateInit {
+  const float *S, *z, *S_lo, *z_lo;
+};
+struct GradIO {
+  const float *S_in, *z_in;
+  float *S_out, *z_out;
 };
 
 }  // namespace slim

@@ -216,6 +216,16 @@ __global__ void __launch_bounds__(256) k_prep(
     }
   }
 
+  if (feature == SLIM_FEAT_SQUARE) {
+    // elementwise quadratic map g(x)_i = x_i^2, M = d (Sec. 4): no Omega
+    for (int e = tid; e < 2 * R * d; e += 256) {
+      const int vec = e / d, m = e % d, r = r0 + vec % R;
+      const float x = xs[vec * d + m];
+      float* dst = (vec < R) ? phiQ : phiK;
+      dst[((size_t)c * Cp + r) * M + m] = (r < b) ? x * x : 0.f;
+    }
+    return;
+  }
   // error bound of an fp32 dot product of length d, times a safety factor 2
   const float gamma = 2.f * (float)(d + 2) * 5.9604645e-08f;
   for (int m0 = 0; m0 < M; m0 += 64) {
@@ -304,6 +314,12 @@ __global__ void k_vjp_prep(float* dphi, const float* phi, float* usum, int M, in
   }
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if (lane == 0) usum[warp] = s;
+}
+
+// Quadratic map: dX = 2 x (.) dphi (M = d, so both are [rows][d]).
+__global__ void k_vjp_square(const float* dphi, const float* X, float* stage, long long n) {
+  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx < n) stage[idx] = 2.f * X[idx] * dphi[idx];
 }
 
 template <typename T>
@@ -462,12 +478,14 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
                         const void* q, const void* k, const void* v, const void* dout,
                         const void* out, const float* omega, int a, int b, bool bwd) {
   const size_t smem = (32 * g.d + 32 + g.d * 64 + 64) * sizeof(float);
-  static bool attr_set = false;  // one instantiation per dtype; set once
-  if (!attr_set) {
+  static bool attr_set[kMaxDevices] = {};  // per dtype instantiation and device
+  bool* set = device_flag(attr_set);
+  if (set == nullptr) return cudaErrorInvalidDevice;
+  if (!*set) {
     cudaError_t e = cudaFuncSetAttribute(k_prep<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          64 * 1024);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    *set = true;
   }
   dim3 grid(g.Cp / 16, g.chains);
   const float inv_sqrt_m = (float)(1.0 / sqrt((double)g.M));
@@ -511,15 +529,23 @@ cudaError_t scan(cudaStream_t s, const Geo& g, float* buf, float* hi, float* lo,
 
 template <typename T>
 slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void* v,
-                     const float* omega, void* out, const StateOut& st, void* workspace,
-                     cudaStream_t s) {
+                     const float* omega, void* out, const StateOut& st, const StateInit& init,
+                     void* workspace, cudaStream_t s) {
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, false);
   const size_t E = (size_t)g.chains * g.M * g.dp;
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
-  SLIM_TRY(cudaMemsetAsync(w.st_hi, 0, E * sizeof(float), s));
-  SLIM_TRY(cudaMemsetAsync(w.st_lo, 0, E * sizeof(float), s));
+  if (init.S) {
+    // B^(0) from an earlier segment (eq. 16 with n - 1 = 0 carried in)
+    prof::Scope ps(prof::K_STATE, s);
+    k_state_in<<<blocks((long long)E), 256, 0, s>>>(StateIn{init.S, init.z, init.S_lo, init.z_lo},
+                                                    w.st_hi, w.st_lo, g.chains, g.M, g.d);
+    SLIM_TRY(cudaGetLastError());
+  } else {
+    SLIM_TRY(cudaMemsetAsync(w.st_hi, 0, E * sizeof(float), s));
+    SLIM_TRY(cudaMemsetAsync(w.st_lo, 0, E * sizeof(float), s));
+  }
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
@@ -543,7 +569,7 @@ slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void*
 template <typename IO>
 slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void* v,
                      const float* omega, const void* out, const void* dout,
-                     const StateIn& st, void* dq, void* dk, void* dv,
+                     const StateIn& st, const GradIO& gio, void* dq, void* dk, void* dv,
                      float* domega, void* workspace, cudaStream_t s) {
   const Geo g = geometry(p);
   Carver cv(workspace);
@@ -551,13 +577,22 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
   const long long T = g.T, M = g.M, d = g.d, dp = g.dp, Cp = g.Cp, nt = g.nt;
   const size_t E = (size_t)g.chains * g.M * g.dp;
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
-  SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
+  if (domega) SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
+  const bool square = p.feature == SLIM_FEAT_SQUARE;
   { prof::Scope ps(prof::K_STATE, s);
   k_state_in<<<blocks((long long)E), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains,
                                                   g.M, g.d); }
   SLIM_TRY(cudaGetLastError());
-  SLIM_TRY(cudaMemsetAsync(w.g_hi, 0, E * sizeof(float), s));
-  SLIM_TRY(cudaMemsetAsync(w.g_lo, 0, E * sizeof(float), s));
+  if (gio.S_in) {
+    // G^(N) handed in by the backward of a later segment (eq. 18)
+    prof::Scope ps(prof::K_STATE, s);
+    k_state_in<<<blocks((long long)E), 256, 0, s>>>(StateIn{gio.S_in, gio.z_in, nullptr, nullptr},
+                                                    w.g_hi, w.g_lo, g.chains, g.M, g.d);
+    SLIM_TRY(cudaGetLastError());
+  } else {
+    SLIM_TRY(cudaMemsetAsync(w.g_hi, 0, E * sizeof(float), s));
+    SLIM_TRY(cudaMemsetAsync(w.g_lo, 0, E * sizeof(float), s));
+  }
   const float inv_sqrt_m = (float)(1.0 / sqrt((double)g.M));
 
   for (int n = g.N - 1; n >= 0; --n) {
@@ -606,6 +641,25 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(cudaGetLastError());
     // feature VJPs
     const int rows = g.chains * g.Cp;
+    if (square) {
+      // dX = 2 x (.) dphi; no Omega, so no dOmega
+      const long long n = (long long)rows * g.d;
+      { prof::Scope ps(prof::K_VJP, s);
+      k_vjp_square<<<blocks(n), 256, 0, s>>>(w.dphiQ, w.Xq, w.stage, n); }
+      SLIM_TRY(cudaGetLastError());
+      { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+      k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dq, p.L, g.d,
+                                                                        a, b, g.Cp, g.chains); }
+      SLIM_TRY(cudaGetLastError());
+      { prof::Scope ps(prof::K_VJP, s);
+      k_vjp_square<<<blocks(n), 256, 0, s>>>(w.dphiK, w.Xk, w.stage, n); }
+      SLIM_TRY(cudaGetLastError());
+      { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+      k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dk, p.L, g.d,
+                                                                        a, b, g.Cp, g.chains); }
+      SLIM_TRY(cudaGetLastError());
+      continue;
+    }
     { prof::Scope ps(prof::K_VJP, s);
     k_vjp_prep<<<blocks((long long)rows * 32), 256, 0, s>>>(w.dphiQ, w.phiQ, w.usum_q, g.M, rows,
                                                             (int)p.feature, inv_sqrt_m); }
@@ -640,6 +694,14 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
                                                              (int)(M * d)); }
     SLIM_TRY(cudaGetLastError());
   }
+  if (gio.S_out) {
+    // G^(0): the gradient with respect to the state this segment started from
+    prof::Scope ps(prof::K_STATE, s);
+    k_state_out<<<blocks((long long)E), 256, 0, s>>>(w.g_hi, w.g_lo,
+                                                     StateOut{gio.S_out, gio.z_out, nullptr, nullptr},
+                                                     g.chains, g.M, g.d);
+    SLIM_TRY(cudaGetLastError());
+  }
   return SLIM_OK;
 }
 
@@ -653,20 +715,21 @@ size_t workspace_bytes(const Problem& p, bool bwd) {
 }
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, void* out, const StateOut& st, void* workspace,
-                cudaStream_t s) {
+                const float* omega, void* out, const StateOut& st, const StateInit& init,
+                void* workspace, cudaStream_t s) {
   if (p.dtype == SLIM_BF16)
-    return fwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, st, workspace, s);
-  return fwd_impl<float>(p, q, k, v, omega, out, st, workspace, s);
+    return fwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, st, init, workspace, s);
+  return fwd_impl<float>(p, q, k, v, omega, out, st, init, workspace, s);
 }
 
 slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
                 const float* omega, const void* out, const void* dout, const StateIn& st,
-                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s) {
+                const GradIO& gio, void* dq, void* dk, void* dv, float* domega, void* workspace,
+                cudaStream_t s) {
   if (p.dtype == SLIM_BF16)
-    return bwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, dout, st, dq, dk, dv,
+    return bwd_impl<__nv_bfloat16>(p, q, k, v, omega, out, dout, st, gio, dq, dk, dv,
                                    domega, workspace, s);
-  return bwd_impl<float>(p, q, k, v, omega, out, dout, st, dq, dk, dv, domega,
+  return bwd_impl<float>(p, q, k, v, omega, out, dout, st, gio, dq, dk, dv, domega,
                          workspace, s);
 }
 

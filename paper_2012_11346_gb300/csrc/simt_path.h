@@ -8,12 +8,13 @@ namespace simt {
 size_t workspace_bytes(const Problem& p, bool bwd);
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, void* out, const StateOut& st, void* workspace,
-                cudaStream_t s);
+                const float* omega, void* out, const StateOut& st, const StateInit& init,
+                void* workspace, cudaStream_t s);
 
 slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
                 const float* omega, const void* out, const void* dout, const StateIn& st,
-                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s);
+                const GradIO& gio, void* dq, void* dk, void* dv, float* domega, void* workspace,
+                cudaStream_t s);
 
 }  // namespace simt
 }  // namespace slim

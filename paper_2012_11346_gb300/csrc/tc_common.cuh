@@ -46,14 +46,53 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait: gives up after ~2^22 polls (well over a second with the
-// back-off), records the failure in *err and returns false.
-__device__ __forceinline__ bool mbar_wait(uint32_t addr, uint32_t parity, int* err) {
-  for (uint32_t i = 0; i < (1u << 22); ++i) {
+// ------------------------------------------------------------------ bounded waits
+// Every wait of a kernel is bounded by time: after kWaitLimitNs of the global
+// timer (and, as a second bound, a fixed number of polls) it gives up.
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+constexpr uint32_t kWaitMaxPolls = 1u << 24;
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// The error word of a call sits at the start of its workspace.  Word 0 is set
+// by a wait that gives up; the other CTAs of the call poll it and leave early.
+// Bytes 8..15 hold the address of a host-visible report counter (or zero),
+// stored by the call's first kernel, which a wait that gives up also
+// increments, so that the next call on the workspace learns of it without
+// synchronising the device.  The grid-dependency wait first makes that
+// kernel's store visible (it returns at once where there is nothing to wait
+// for, and a wait gives up only after a second anyway).
+__device__ __forceinline__ void give_up(int* err) {
+  atomicExch(err, 1);
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  unsigned* rep = reinterpret_cast<unsigned* const volatile*>(err)[1];
+  if (rep) atomicAdd_system(rep, 1u);
+}
+// Stores a call's report-counter address beside its error word (thread 0 of
+// the call's first kernel).
+__device__ __forceinline__ void set_report(int* err, unsigned* rep) {
+  reinterpret_cast<unsigned**>(err)[1] = rep;
+}
+// Bounded mbarrier wait: records a failure and returns false when it gives up.
+// err is a workspace error word (see give_up), or, with workspace_word false,
+// a plain int that is only set.
+__device__ __forceinline__ bool mbar_wait(uint32_t addr, uint32_t parity, int* err,
+                                          bool workspace_word = true) {
+  if (mbar_try_wait(addr, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 0; i < kWaitMaxPolls; ++i) {
     if (mbar_try_wait(addr, parity)) return true;
     if (i > 16) __nanosleep(256);
+    if ((i & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
   }
-  if (err) atomicExch(err, 1);
+  if (err) {
+    if (workspace_word)
+      give_up(err);
+    else
+      atomicExch(err, 1);
+  }
   return false;
 }
 

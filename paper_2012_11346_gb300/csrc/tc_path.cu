@@ -327,6 +327,7 @@ struct FwdJob {
   int* ticket;                  // tile counter of this launch (starts at 0)
   __nv_bfloat16* out;
   StateOut st;                  // B^(N), written by the last tile of each chain
+  StateInit init;               // B^(0), read by the first tile of each chain (null: zero)
   int* err;
 };
 
@@ -347,36 +348,46 @@ __device__ __forceinline__ void group_publish(int id) {
   tc_fence_after();
 }
 // Bounded poll of a flag by one thread: returns once *flag == want (then an
-// acquire fence).  It gives up after 2^22 polls (~1 s with the back-off), or
+// acquire fence).  It gives up after kWaitLimitNs (or kWaitMaxPolls polls), or
 // early once another CTA has reported an error (checked every 64 polls, so
 // that waiting CTAs do not all hammer the error word); a wait that gives up
-// records itself in *err.
+// records itself through give_up(err).
 __device__ __forceinline__ bool flag_poll(const int* flag, int want, int* err) {
-  for (uint32_t i = 0; i < (1u << 22); ++i) {
+  uint64_t t0 = 0;
+  for (uint32_t i = 0; i < kWaitMaxPolls; ++i) {
     if (ld_relaxed_gpu(flag) == want) {
       fence_acq_rel_gpu();
       return true;
     }
-    if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) return false;
+    if ((i & 63) == 63) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
+      if (i == 63) t0 = globaltimer_ns();
+      else if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    }
     __nanosleep(i < 16 ? 32 : 256);
   }
-  atomicExch(err, 1);
+  give_up(err);
   return false;
 }
 // Bounded wait by one thread for up to two flags at once (a null flag is not
 // waited on): both are read in every round, so a satisfied pair costs one trip.
 __device__ __forceinline__ bool flag_poll2(const int* f1, int w1, const int* f2, int w2, int* err) {
-  for (uint32_t i = 0; i < (1u << 22); ++i) {
+  uint64_t t0 = 0;
+  for (uint32_t i = 0; i < kWaitMaxPolls; ++i) {
     const int v1 = f1 ? ld_relaxed_gpu(f1) : w1;
     const int v2 = f2 ? ld_relaxed_gpu(f2) : w2;
     if (v1 == w1 && v2 == w2) {
       fence_acq_rel_gpu();
       return true;
     }
-    if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) return false;
+    if ((i & 63) == 63) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
+      if (i == 63) t0 = globaltimer_ns();
+      else if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    }
     __nanosleep(i < 16 ? 32 : 256);
   }
-  atomicExch(err, 1);
+  give_up(err);
   return false;
 }
 // The thread that polls the flags a tile needs from other tiles: lane 0 of
@@ -385,15 +396,20 @@ __device__ __forceinline__ bool flag_poll2(const int* f1, int w1, const int* f2,
 constexpr int POLL = NTHR - 32, LDT = NTHR - 32;
 // Bounded wait by one thread for a counter to reach at least want.
 __device__ __forceinline__ bool counter_poll(const int* ctr, int want, int* err) {
-  for (uint32_t i = 0; i < (1u << 22); ++i) {
+  uint64_t t0 = 0;
+  for (uint32_t i = 0; i < kWaitMaxPolls; ++i) {
     if (ld_relaxed_gpu(ctr) - want >= 0) {
       fence_acq_rel_gpu();
       return true;
     }
-    if ((i & 63) == 63 && *reinterpret_cast<volatile int*>(err) != 0) return false;
+    if ((i & 63) == 63) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
+      if (i == 63) t0 = globaltimer_ns();
+      else if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    }
     __nanosleep(i < 16 ? 32 : 256);
   }
-  atomicExch(err, 1);
+  give_up(err);
   return false;
 }
 
@@ -550,12 +566,29 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
         for (int j = 0; j < 2; ++j) {
           if (pred) {
             ld_lm16(pred, h, cq + j, row, pv[h][j]);
+          } else if (J.init.S) {
+            // the first tile of the sequence starts from the caller's B^(0)
+            const size_t e = ((size_t)c * MF + 128 * h + row) * 64 + 16 * (cq + j);
+            ld_row16f(J.init.S + e, pv[h][j]);
+            if (J.init.S_lo) {
+              float lo[16];
+              ld_row16f(J.init.S_lo + e, lo);
+#pragma unroll
+              for (int i = 0; i < 16; ++i) pv[h][j][i] += lo[i];
+            }
           } else {
 #pragma unroll
             for (int i = 0; i < 16; ++i) pv[h][j][i] = 0.f;
           }
         }
-        pz[h] = (pred && cq == 0) ? __ldcg(pred + MF * 64 + 128 * h + row) : 0.f;
+        pz[h] = 0.f;
+        if (cq == 0) {
+          const size_t e = (size_t)c * MF + 128 * h + row;
+          if (pred)
+            pz[h] = __ldcg(pred + MF * 64 + 128 * h + row);
+          else if (J.init.z)
+            pz[h] = __ldcg(J.init.z + e) + (J.init.z_lo ? __ldcg(J.init.z_lo + e) : 0.f);
+        }
       }
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
@@ -679,6 +712,7 @@ struct BwdQJob {
   int* sums_done;         // slice 0 only: counter of final sums written
   __nv_bfloat16* dq;
   int* err;
+  GradIO gio;             // G^(N) in (null: zero), G^(0) out (null: not returned)
 };
 
 // The dq side splits its warps twice, as the forward does: after the g(K)
@@ -724,6 +758,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   const int wnext = inner ? n + 1 : n + 2;
   const bool linked = inner || next_slice;
   StateRef s1, s2;
+  bool s2_rowmajor = false;  // the caller's G^(N) is row-major, the slots lane-major
   if (linked) {
     const float* p1 = J.slot1 + ((size_t)c * J.nt + snext) * C::E;
     const float* p2 = J.slot2 + ((size_t)c * J.nt + snext) * C::E;
@@ -733,8 +768,18 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     s1 = StateRef{J.fin.S + (size_t)c * MF * 64, J.fin.z + (size_t)c * MF,
                   J.fin.S_lo ? J.fin.S_lo + (size_t)c * MF * 64 : nullptr,
                   J.fin.z_lo ? J.fin.z_lo + (size_t)c * MF : nullptr};
-    s2 = StateRef{nullptr, nullptr, nullptr, nullptr};
+    // G^(N): zero at the true end of a sequence, or handed in by the backward
+    // of a later segment (eq. 18)
+    if (J.gio.S_in) {
+      s2 = StateRef{J.gio.S_in + (size_t)c * MF * 64, J.gio.z_in + (size_t)c * MF, nullptr, nullptr};
+      s2_rowmajor = true;
+    } else {
+      s2 = StateRef{nullptr, nullptr, nullptr, nullptr};
+    }
   }
+  // the first tile of the sequence hands on G^(0), the gradient with respect
+  // to the state the sequence started from
+  const bool seq_first = n == 0 && t == 0 && J.gio.S_out != nullptr;
   const int* f1 = J.flag1 + ((size_t)c * J.nt + snext) * FLAG_STRIDE;
   const int* f2 = J.flag2 + ((size_t)c * J.nt + snext) * FLAG_STRIDE;
   float* own1 = J.slot1 + ((size_t)c * J.nt + t) * C::E;
@@ -1112,7 +1157,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       for (int h = 0; h < C::MH; ++h) {
 #pragma unroll
         for (int j = 0; j < 2; ++j) {
-          if (s2.S) {
+          if (s2.S && s2_rowmajor) {
+            ld_row16f(s2.S + (size_t)(128 * h + row) * 64 + 16 * (cq + j), gs[h][j]);
+          } else if (s2.S) {
             ld_lm16(s2.S, h, cq + j, row, gs[h][j]);
           } else {
 #pragma unroll
@@ -1131,6 +1178,8 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
 #pragma unroll
           for (int i = 0; i < 16; ++i) gs[h][j][i] += gd[i];
           st_lm16(own2, h, cq + j, row, gs[h][j]);
+          if (seq_first)
+            st_f32x16(J.gio.S_out + ((size_t)c * MF + 128 * h + row) * 64 + 16 * (cq + j), gs[h][j]);
         }
       }
       if (cq == 0) {
@@ -1141,6 +1190,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           tmem_ld1(trow + 128 + 16 * h, gdz);
           J.gz[tf * MF + m] = gzs[h];
           __stcg(own2 + MF * 64 + m, gzs[h] + gdz);
+          if (seq_first) J.gio.z_out[(size_t)c * MF + m] = gzs[h] + gdz;
         }
       }
       group_bar(2);  // every slot write of the group is issued
@@ -1611,8 +1661,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_fwd(const __grid_constant__ FwdJ
 // earlier stages or on earlier tiles of its own chain, which hold lower
 // tickets:
 //   dq side of slice n    <- its chain (slice n's later tiles, slice n+1's first),
-//                            slice n+2's dk/dv side (hand-off buffers of parity
-//                            n%2), slice n+1's dq side at its position (dOmega sum)
+//                            slice n+R's dk/dv side (hand-off buffers of ring
+//                            slot n % R, R >= 2), slice n+1's dq side at its
+//                            position (dOmega sum)
 //   dk/dv side of slice n <- the dq side of the same tile; slice n+1's dk/dv side
 //                            at its position (dOmega sum)
 //   reduction stage 1     <- every tile of slice 0 (the last to add to a sum)
@@ -1795,8 +1846,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
 // ================================================================== small kernels
 // Omega as a bf16 pair: hi = bf16(Omega), lo = bf16(Omega - hi), so the
 // projections X Omega^T = X hi^T + X lo^T carry ~16 mantissa bits.
-__global__ void k_omega_bf16(const float* om, __nv_bfloat16* om16, int n) {
+// Thread 0 also stores the call's report-counter address (see give_up).
+__global__ void k_omega_bf16(const float* om, __nv_bfloat16* om16, int n, int* err,
+                             unsigned* rep) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i == 0) set_report(err, rep);
   if (i < n) {
     const __nv_bfloat16 hi = __float2bfloat16_rn(om[i]);
     om16[i] = hi;
@@ -1915,8 +1969,10 @@ static_assert(NSLOT * 128 * 64 * 4 <= smem_bwd<128>() - 1024 &&
 
 template <int MF, int FEAT>
 cudaError_t configure() {
-  static bool done = false;
-  if (done) return cudaSuccess;
+  static bool configured[kMaxDevices] = {};
+  bool* done = device_flag(configured);
+  if (done == nullptr) return cudaErrorInvalidDevice;
+  if (*done) return cudaSuccess;
   cudaError_t e = cudaFuncSetAttribute(k_tc_fwd<MF, FEAT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem_fwd<MF>());
@@ -1927,7 +1983,7 @@ cudaError_t configure() {
     e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem_bwd<MF>());
   if (e != cudaSuccess) return e;
-  done = true;
+  *done = true;
   return cudaSuccess;
 }
 
@@ -1970,29 +2026,31 @@ Slice slice_of(const Problem& p, const Geo& g, int n) {
   return r;
 }
 
-cudaError_t prepare(const Ws& w, const Geo& g, const float* omega, cudaStream_t s) {
+cudaError_t prepare(const Ws& w, const Geo& g, const float* omega, unsigned* rep,
+                    cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(w.flags, 0, (size_t)w.nflags * sizeof(int), s);
   if (e != cudaSuccess) return e;
   prof::Scope ps(prof::K_TC_PREP, s);
-  k_omega_bf16<<<nblk(g.MF * D), 256, 0, s>>>(omega, w.om16, g.MF * D);  // hi and lo
+  k_omega_bf16<<<nblk(g.MF * D), 256, 0, s>>>(omega, w.om16, g.MF * D, w.err, rep);  // hi and lo
   return cudaGetLastError();
 }
 
 template <int MF, int FEAT>
 slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat16* k,
                      const __nv_bfloat16* v, const float* omega, __nv_bfloat16* out,
-                     const StateOut& st, void* workspace, cudaStream_t s) {
+                     const StateOut& st, const StateInit& init, unsigned* rep, void* workspace,
+                     cudaStream_t s) {
   TC_TRY((configure<MF, FEAT>()));
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, false);
-  TC_TRY(prepare(w, g, omega, s));
+  TC_TRY(prepare(w, g, omega, rep, s));
   // every tile of every slice in one launch, in sequence order, chains inside
   // a tile position.  Algorithmic work per row: 8dM (phiQ, phiK, Delta, readout).
   const int P = (g.N - 1) * g.nt + slice_of(p, g, g.N - 1).nt;
   const FwdJob J{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flag1, w.ticket,
-                 out, st, w.err};
+                 out, st, init, w.err};
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
   prof::Scope ps(prof::K_TC_FWD, s, rows * 8.0 * MD, rows * D * 2.0 * 4);
   TC_TRY(launch_dep(k_tc_fwd<MF, FEAT>, dim3(P * g.chains), dim3(NTHR), smem_fwd<MF>(), s, J));
@@ -2012,15 +2070,15 @@ void reduction_split(const Geo& g, int& r1n, int& r2n) {
 template <int MF, int FEAT>
 slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat16* k,
                      const __nv_bfloat16* v, const float* omega, const __nv_bfloat16* out,
-                     const __nv_bfloat16* dout, const StateIn& st,
+                     const __nv_bfloat16* dout, const StateIn& st, const GradIO& gio,
                      __nv_bfloat16* dq, __nv_bfloat16* dk, __nv_bfloat16* dv, float* domega,
-                     void* workspace, cudaStream_t s) {
+                     unsigned* rep, void* workspace, cudaStream_t s) {
   TC_TRY((configure<MF, FEAT>()));
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, true);
   const int N = g.N;
-  TC_TRY(prepare(w, g, omega, s));
+  TC_TRY(prepare(w, g, omega, rep, s));
   BwdJob J{};
   J.s.N = N;
   J.s.chains = g.chains;
@@ -2032,7 +2090,7 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
   J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
                 w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
-                0, 0, nullptr, nullptr, 0, nullptr, dq, w.err};
+                0, 0, nullptr, nullptr, 0, nullptr, dq, w.err, gio};
   J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                   p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
   J.red = RedJob{w.acc, 2 * g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
@@ -2067,7 +2125,8 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
 }  // namespace
 
 bool supports(const Problem& p) {
-  return p.dtype == SLIM_BF16 && p.d == D && (p.M == 128 || p.M == 256) && p.slice_len() >= 64;
+  return p.dtype == SLIM_BF16 && p.d == D && (p.M == 128 || p.M == 256) &&
+         p.feature != SLIM_FEAT_SQUARE && p.slice_len() >= 64;
 }
 
 size_t workspace_bytes(const Problem& p, bool bwd) {
@@ -2105,19 +2164,21 @@ int bwd_schedule(const Problem& p, int* items, int cap, int* ring) {
   } while (0)
 
 slim_status fwd(const Problem& p, const void* q, const void* k, const void* v,
-                const float* omega, void* out, const StateOut& st, void* workspace,
-                cudaStream_t s) {
+                const float* omega, void* out, const StateOut& st, const StateInit& init,
+                unsigned* report, void* workspace, cudaStream_t s) {
   using B16 = __nv_bfloat16;
   TC_DISPATCH(fwd_impl, p, (const B16*)q, (const B16*)k, (const B16*)v, omega, (B16*)out, st,
-              workspace, s);
+              init, report, workspace, s);
 }
 
 slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
                 const float* omega, const void* out, const void* dout, const StateIn& st,
-                void* dq, void* dk, void* dv, float* domega, void* workspace, cudaStream_t s) {
+                const GradIO& gio, void* dq, void* dk, void* dv, float* domega,
+                unsigned* report, void* workspace, cudaStream_t s) {
   using B16 = __nv_bfloat16;
   TC_DISPATCH(bwd_impl, p, (const B16*)q, (const B16*)k, (const B16*)v, omega, (const B16*)out,
-              (const B16*)dout, st, (B16*)dq, (B16*)dk, (B16*)dv, domega, workspace, s);
+              (const B16*)dout, st, gio, (B16*)dq, (B16*)dk, (B16*)dv, domega, report, workspace,
+              s);
 }
 
 }  // namespace tc

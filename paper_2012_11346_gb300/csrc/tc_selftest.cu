@@ -4,6 +4,7 @@
 #include "../../include/slim.h"
 #include "common.cuh"
 #include "profiler.h"
+#include "report.h"
 #include "tc_common.cuh"
 
 namespace slim {
@@ -51,7 +52,7 @@ __global__ void __launch_bounds__(128) k_tc_selftest(const __nv_bfloat16* A, con
     }
     mma_commit(smem_u32(&mbar));
   }
-  const bool ok = mbar_wait(smem_u32(&mbar), 0, err);
+  const bool ok = mbar_wait(smem_u32(&mbar), 0, err, false);  // err: a plain int
   tc_fence_after();
   if (ok) {
     const int row = tid;
@@ -69,9 +70,11 @@ __global__ void __launch_bounds__(128) k_tc_selftest(const __nv_bfloat16* A, con
 // A bounded wait on an mbarrier that nothing arrives at: it gives up after
 // its iteration limit, records the failure in the error word and returns --
 // the same path every kernel takes when a wait gives up.
-__global__ void k_wait_timeout(int* err) {
+__global__ void k_wait_timeout(int* err, unsigned* rep) {
   __shared__ __align__(8) uint64_t mbar;
   if (threadIdx.x == 0) {
+    *err = 0;
+    set_report(err, rep);
     mbar_init(smem_u32(&mbar), 1);
     mbar_fence_init();
   }
@@ -85,8 +88,12 @@ __global__ void k_wait_timeout(int* err) {
 extern "C" slim_status slim_diag_wait_timeout(void* workspace, void* stream) {
   if (!workspace) return SLIM_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the same error word and report counter as the tensor-core calls
+  unsigned* counter = nullptr;
+  const slim_status st = slim::report::begin(workspace, true, &counter);
+  if (st != SLIM_OK) return st;
   slim::prof::Scope ps(slim::prof::K_TC_SELFTEST, s);
-  slim::tc::k_wait_timeout<<<1, 32, 0, s>>>(static_cast<int*>(workspace));
+  slim::tc::k_wait_timeout<<<1, 32, 0, s>>>(static_cast<int*>(workspace), counter);
   return cudaGetLastError() == cudaSuccess ? SLIM_OK : SLIM_ERR_CUDA;
 }
 

@@ -15,7 +15,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libslim.so
 _lib = None
 
 DTYPES = {torch.float32: 0, torch.bfloat16: 1}
-FEATURES = {"exp": 0, "relu": 1}
+FEATURES = {"exp": 0, "relu": 1, "square": 2}
 STATUS = {0: "SLIM_OK", 1: "SLIM_ERR_INVALID_ARG", 2: "SLIM_ERR_UNSUPPORTED",
           3: "SLIM_ERR_WORKSPACE", 4: "SLIM_ERR_CUDA", 5: "SLIM_ERR_TIMEOUT"}
 
@@ -29,6 +29,8 @@ SIGNATURES = {
     "slim_bwd_workspace_size": ([_i] * 6 + [_i, _i, ctypes.POINTER(_sz)], _i),
     "slim_fwd": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 5 + [_p, _sz, _p], _i),
     "slim_bwd": ([_p] * 10 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
+    "slim_fwd_from": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p] * 5 + [_p, _sz, _p], _i),
+    "slim_bwd_from": ([_p] * 12 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p] * 2 + [_p, _sz, _p], _i),
     "slim_check_device_error": ([_p, _p], _i),
     "slim_launch_count": ([], ctypes.c_ulonglong),
     "slim_profiler_enable": ([_i], None),
@@ -82,7 +84,7 @@ def _check(status, where):
 
 def _dims(q, omega):
     B, H, L, d = q.shape
-    M = omega.shape[0]
+    M = omega.shape[0] if omega is not None else d
     return B, H, L, d, M
 
 
@@ -136,12 +138,24 @@ def _ptr(t):
     return None if t is None else t.data_ptr()
 
 
-def forward(q, k, v, omega, C, feature="exp", workspace=None, stream=None, residuals=False):
-    """slim_fwd: returns (out, S_state, z_state), or with residuals=True
-    (out, S_state, z_state, S_state_lo, z_state_lo) -- the low-order parts of
-    the carried state, which slim_bwd uses to start its rollback exactly."""
-    _require_cuda(q, k, v, omega)
-    B, H, L, d, M = _dims(q, omega)
+def _opt_ptr(t):
+    if t is None:
+        return None
+    _require_cuda(t)
+    return t.data_ptr()
+
+
+def forward(q, k, v, omega, C, feature="exp", workspace=None, stream=None, residuals=False,
+            S_init=None, z_init=None, S_init_lo=None, z_init_lo=None):
+    """slim_fwd (slim_fwd_from when an initial state is given): returns
+    (out, S_state, z_state), or with residuals=True (out, S_state, z_state,
+    S_state_lo, z_state_lo) -- the low-order parts of the carried state, which
+    slim_bwd uses to start its rollback exactly.  S_init / z_init (and their
+    residuals): the state B^(0) the sequence starts from, e.g. the state an
+    earlier segment returned.  omega may be None for the quadratic map."""
+    _require_cuda(q, k, v)
+    B, H, L, d = q.shape
+    M = omega.shape[0] if omega is not None else d
     out = torch.empty_like(q)
     S_state = torch.empty(B, H, M, d, dtype=torch.float32, device=q.device)
     z_state = torch.empty(B, H, M, dtype=torch.float32, device=q.device)
@@ -149,32 +163,53 @@ def forward(q, k, v, omega, C, feature="exp", workspace=None, stream=None, resid
     z_lo = torch.empty_like(z_state) if residuals else None
     need = workspace_size(B, H, L, d, M, C, q.dtype, feature, False)
     ws = workspace if workspace is not None else _workspace(need, q.device)
-    _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
-                              B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
-                              out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
-                              _ptr(S_lo), _ptr(z_lo), ws.data_ptr(), ws.numel(),
-                              _stream_handle(stream)), "slim_fwd")
+    args = (q.data_ptr(), k.data_ptr(), v.data_ptr(), _opt_ptr(omega), B, H, L, d, M, C,
+            DTYPES[q.dtype], FEATURES[feature])
+    tail = (out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo),
+            ws.data_ptr(), ws.numel(), _stream_handle(stream))
+    if S_init is None and z_init is None:
+        _check(library().slim_fwd(*args, *tail), "slim_fwd")
+    else:
+        _check(library().slim_fwd_from(*args, _opt_ptr(S_init), _opt_ptr(z_init),
+                                       _opt_ptr(S_init_lo), _opt_ptr(z_init_lo), *tail),
+               "slim_fwd_from")
     if residuals:
         return out, S_state, z_state, S_lo, z_lo
     return out, S_state, z_state
 
 
 def backward(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp", workspace=None,
-             stream=None, S_lo=None, z_lo=None):
-    """slim_bwd: returns (dq, dk, dv, domega).  S_lo / z_lo: the residuals
-    from forward(..., residuals=True), or None."""
-    _require_cuda(q, k, v, omega, out, dout, S_state, z_state)
-    B, H, L, d, M = _dims(q, omega)
+             stream=None, S_lo=None, z_lo=None, G_S_in=None, g_z_in=None, return_state_grad=False):
+    """slim_bwd (slim_bwd_from when a state gradient is handed in or asked
+    for): returns (dq, dk, dv, domega), and with return_state_grad=True also
+    (G_S, g_z) = G^(0), the gradient with respect to the state the sequence
+    started from.  S_lo / z_lo: the residuals from forward(..., residuals=True),
+    or None.  G_S_in / g_z_in: G^(N) from the backward of a later segment.
+    For the quadratic map omega may be None; domega is then None."""
+    _require_cuda(q, k, v, out, dout, S_state, z_state)
+    B, H, L, d = q.shape
+    M = omega.shape[0] if omega is not None else d
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
-    domega = torch.empty(M, d, dtype=torch.float32, device=q.device)
+    domega = (torch.empty(M, d, dtype=torch.float32, device=q.device)
+              if omega is not None else None)
     need = workspace_size(B, H, L, d, M, C, q.dtype, feature, True)
     ws = workspace if workspace is not None else _workspace(need, q.device)
-    _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
-                              out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
-                              z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo), B, H, L, d, M, C,
-                              DTYPES[q.dtype], FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
-                              dv.data_ptr(), domega.data_ptr(), ws.data_ptr(), ws.numel(),
-                              _stream_handle(stream)), "slim_bwd")
+    G_S = g_z = None
+    head = (q.data_ptr(), k.data_ptr(), v.data_ptr(), _opt_ptr(omega), out.data_ptr(),
+            dout.data_ptr(), S_state.data_ptr(), z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo))
+    dims = (B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature])
+    grads = (dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), _ptr(domega))
+    tail = (ws.data_ptr(), ws.numel(), _stream_handle(stream))
+    if G_S_in is None and g_z_in is None and not return_state_grad:
+        _check(library().slim_bwd(*head, *dims, *grads, *tail), "slim_bwd")
+    else:
+        if return_state_grad:
+            G_S = torch.empty(B, H, M, d, dtype=torch.float32, device=q.device)
+            g_z = torch.empty(B, H, M, dtype=torch.float32, device=q.device)
+        _check(library().slim_bwd_from(*head, _opt_ptr(G_S_in), _opt_ptr(g_z_in), *dims, *grads,
+                                       _ptr(G_S), _ptr(g_z), *tail), "slim_bwd_from")
+    if return_state_grad:
+        return dq, dk, dv, domega, G_S, g_z
     return dq, dk, dv, domega
 
 
@@ -182,7 +217,7 @@ def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, s
                  S_lo=None, z_lo=None):
     """slim_fwd into caller-allocated outputs and workspace (no allocation)."""
     B, H, L, d, M = _dims(q, omega)
-    _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
+    _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega),
                               B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
                               out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
                               _ptr(S_lo), _ptr(z_lo), workspace.data_ptr(), workspace.numel(),
@@ -193,11 +228,11 @@ def backward_into(q, k, v, omega, out, dout, S_state, z_state, C, feature, dq, d
                   workspace, stream=None, S_lo=None, z_lo=None):
     """slim_bwd into caller-allocated gradients and workspace (no allocation)."""
     B, H, L, d, M = _dims(q, omega)
-    _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), omega.data_ptr(),
+    _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega),
                               out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
                               z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo), B, H, L, d, M, C,
                               DTYPES[q.dtype], FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
-                              dv.data_ptr(), domega.data_ptr(), workspace.data_ptr(),
+                              dv.data_ptr(), _ptr(domega), workspace.data_ptr(),
                               workspace.numel(), _stream_handle(stream)), "slim_bwd")
 
 

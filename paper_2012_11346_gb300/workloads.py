@@ -50,13 +50,16 @@ class Workload:
         return replace(self, **kw)
 
 
-# The five workloads of the benchmark plan.
+# The five workloads of the benchmark plan, and the quadratic-map workload.
 WORKLOADS = {
     "tiny_f32": Workload("tiny_f32", 1, 1, 256, 16, 32, 64, "f32", "exp", "normal", "iid"),
     "L4096_bf16": Workload("L4096_bf16", 8, 8, 4096, 64, 256, 1024, "bf16", "exp", "normal", "orthogonal"),
     "L32768_bf16": Workload("L32768_bf16", 2, 8, 32768, 64, 256, 1024, "bf16", "exp", "normal", "orthogonal"),
     "L8192_relu_f32": Workload("L8192_relu_f32", 4, 12, 8192, 64, 128, 512, "f32", "relu", "uniform", "iid"),
     "L65536_C16_bf16": Workload("L65536_C16_bf16", 1, 4, 65536, 128, 256, 16, "bf16", "exp", "normal", "orthogonal"),
+    # the paper's own experimental feature map (Sec. 4: g(x) = x^2 elementwise,
+    # M = d = 64 per head) on the bench shape; Omega is drawn but not used
+    "L4096_square_bf16": Workload("L4096_square_bf16", 8, 8, 4096, 64, 64, 1024, "bf16", "square", "normal", "iid"),
 }
 
 # Slice sizes swept on the L = 32768 workload (time and peak memory vs C).

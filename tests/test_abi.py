@@ -161,3 +161,55 @@ def test_bwd_schedule_arguments(lib):
     for args in ((4, 12, 8192, 64, 128, 512, 0, 1), (1, 4, 65536, 128, 256, 16, 1, 0),
                  (2, 8, 32768, 64, 256, 16, 1, 0)):
         assert lib.slim_bwd_schedule(*args, None, 0, ctypes.byref(n), None) == UNSUPPORTED
+
+
+SQUARE = 2
+
+
+def test_square_map_needs_M_equal_d(lib):
+    assert ws(1, 1, 8, 16, 16, 4, 0, SQUARE)[0] == OK
+    assert ws(1, 1, 8, 16, 32, 4, 0, SQUARE)[0] == INVALID      # g(x)_i = x_i^2 has M = d
+    assert ws(1, 1, 8, 64, 64, 4, 1, SQUARE, bwd=True)[0] == OK
+    n = ctypes.c_int(-1)
+    # the quadratic map runs on the fp32-compute kernels
+    assert lib.slim_path_for(8, 8, 4096, 64, 64, 1024, 1, SQUARE, ctypes.byref(n)) == OK
+    assert n.value == 0
+
+
+def test_omega_optional_only_for_square(lib):
+    _, need = ws(1, 1, 8, 16, 16, 4, 0, SQUARE)
+    p = [FAKE] * 7
+    p[3] = None                                                   # no Omega
+    assert fwd_call(lib, p, dims=(1, 1, 8, 16, 32, 4), ft=0) == INVALID
+    # with the quadratic map a null Omega passes validation; a too-small
+    # workspace is then the first error
+    assert fwd_call(lib, p, dims=(1, 1, 8, 16, 16, 4), ft=SQUARE, wsb=need - 1) == WORKSPACE
+
+
+def fwd_from_call(lib, init, dims=(1, 1, 8, 16, 32, 4), wsb=0):
+    p = [FAKE] * 7
+    return lib.slim_fwd_from(p[0], p[1], p[2], p[3], *dims, 0, 0, *init, p[4], p[5], p[6], None,
+                             None, FAKE, wsb, None)
+
+
+def bwd_from_call(lib, gin, gout, dims=(1, 1, 8, 16, 32, 4), wsb=0):
+    p = [FAKE] * 12
+    return lib.slim_bwd_from(*p[:8], None, None, gin[0], gin[1], *dims, 0, 0, *p[8:12], gout[0],
+                             gout[1], FAKE, wsb, None)
+
+
+def test_streaming_arguments_rejected_before_launch(lib):
+    _, nf = ws(1, 1, 8, 16, 32, 4)
+    _, nb = ws(1, 1, 8, 16, 32, 4, bwd=True)
+    # B^(0): value and normaliser together, residuals only with them, aligned
+    assert fwd_from_call(lib, (FAKE, None, None, None)) == INVALID
+    assert fwd_from_call(lib, (None, FAKE, None, None)) == INVALID
+    assert fwd_from_call(lib, (None, None, FAKE, None)) == INVALID
+    assert fwd_from_call(lib, (FAKE + 4, FAKE, None, None)) == INVALID
+    assert fwd_from_call(lib, (FAKE, FAKE, FAKE, None), wsb=nf - 1) == WORKSPACE
+    assert fwd_from_call(lib, (None, None, None, None), wsb=nf - 1) == WORKSPACE
+    # G^(N) in and G^(0) out: pairs, aligned
+    assert bwd_from_call(lib, (FAKE, None), (None, None)) == INVALID
+    assert bwd_from_call(lib, (None, None), (None, FAKE)) == INVALID
+    assert bwd_from_call(lib, (FAKE, FAKE), (FAKE + 8, FAKE)) == INVALID
+    assert bwd_from_call(lib, (FAKE, FAKE), (FAKE, FAKE), wsb=nb - 1) == WORKSPACE

@@ -29,7 +29,7 @@ def test_tiny_f32_exact_workload(cuda_device):
     w = W.WORKLOADS["tiny_f32"]
     x = inputs(w, cuda_device)
     compare(gpu_run(x, w.C, w.feature), oracle_run(cpu_inputs(x), w.C, w.feature), TOL[w.dtype],
-            where=w.name)
+            where=w.name, C=w.C)
 
 
 SHRUNK = [
@@ -38,6 +38,7 @@ SHRUNK = [
     ("L32768_bf16", dict(B=1, H=2, L=4200, C=1024)),
     ("L8192_relu_f32", dict(B=2, H=3, L=1500)),
     ("L65536_C16_bf16", dict(B=1, H=2, L=700)),
+    ("L4096_square_bf16", dict(B=2, H=2, L=2600)),
 ]
 
 
@@ -46,7 +47,7 @@ def test_shrunk_workloads(cuda_device, name, kw):
     w = W.WORKLOADS[name].with_(**kw)
     x = inputs(w, cuda_device)
     compare(gpu_run(x, w.C, w.feature), oracle_run(cpu_inputs(x), w.C, w.feature), TOL[w.dtype],
-            where=w.name)
+            where=w.name, C=w.C)
 
 
 @pytest.mark.parametrize("C", W.C_SWEEP)
@@ -55,7 +56,8 @@ def test_c_sweep_shape(cuda_device, C):
     result, every C compared against it: the result does not depend on C)."""
     w = W.WORKLOADS["L32768_bf16"].with_(B=1, H=2, L=4100)
     x = inputs(w, cuda_device)
-    compare(gpu_run(x, C, w.feature), _oracle_cached(w, x), TOL[w.dtype], where=f"C={C}")
+    compare(gpu_run(x, C, w.feature), _oracle_cached(w, x), TOL[w.dtype], where=f"C={C}",
+            C=C)
 
 
 _CACHE = {}
@@ -78,6 +80,8 @@ EDGE = [
     (64, 128, 200, 33, "bf16", "relu"),
     (128, 256, 70, 16, "f32", "exp"),
     (128, 64, 129, 128, "bf16", "exp"),
+    (32, 32, 150, 40, "f32", "square"),
+    (128, 128, 90, 64, "f32", "square"),
 ]
 
 
@@ -89,7 +93,7 @@ def test_edge_shapes(cuda_device, d, M, L, C, dtype, feature):
     xc = cpu_inputs(x)
     compare(gpu_run(x, C, feature), oracle_run(xc, C, feature), TOL[dtype],
             where=f"d{d} M{M} L{L} C{C} {dtype} {feature}",
-            scale=float(np.linalg.norm(xc["dout"].ravel())))
+            scale=float(np.linalg.norm(xc["dout"].ravel())), C=C)
 
 
 def test_empty_sequence(cuda_device):

@@ -39,7 +39,7 @@ def test_tc_parity(cuda_device, M, L, C, feature):
     assert slim.path_for(w.B, w.H, L, 64, M, C, torch.bfloat16, feature) == 1
     x = W.make_inputs(w, device=cuda_device)
     compare(gpu_run(x, C, feature), oracle_run(cpu_inputs(x), C, feature), TOL["bf16"],
-            where=f"tc M{M} L{L} C{C} {feature}")
+            where=f"tc M{M} L{L} C{C} {feature}", C=C)
 
 
 def test_tc_matches_fp32_path(cuda_device, monkeypatch):
