@@ -11,6 +11,7 @@ Modules
                 backward sweep with rollback (eq. 17) and G carry (eq. 18)
   iterative  -- the token-by-token recurrence of App. B (C = 1)
   fd         -- central finite differences of <dY, Y>
+  bidir      -- the non-causal form (no mask, one global state), two sweeps
 
 Library-facing wrappers below use the layout of the C ABI: q, k, v, dout are
 [B, H, L, d]; omega is [M, d]; the state is S_state = R^T ([B, H, M, d], the
@@ -24,7 +25,7 @@ function here is "parity unpinned".
 """
 import numpy as np
 
-from . import brute, features, fd, iterative, sliced  # noqa: F401
+from . import bidir, brute, features, fd, iterative, sliced  # noqa: F401
 
 
 def _chains(x):
@@ -76,6 +77,34 @@ def oracle_bwd(q, k, v, omega, dout, S_state, z_state, C, feature, G_S=None, g_z
     }
     return (dQ.reshape(B, H, L, d), dK.reshape(B, H, L, d), dV.reshape(B, H, L, d),
             dOmega, extra)
+
+
+def oracle_bidir_fwd(q, k, v, omega, C, feature):
+    """Non-causal forward.  Returns out [B,H,L,d], S_state [B,H,M,d], z_state
+    [B,H,M] (the global state)."""
+    Q, (B, H) = _chains(q)
+    K, _ = _chains(k)
+    V, _ = _chains(v)
+    Omega = np.asarray(omega, dtype=np.float64)
+    M = Omega.shape[0]
+    L, d = Q.shape[1], Q.shape[2]
+    Y, R, S = bidir.forward(Q, K, V, Omega, C, feature)
+    return (Y.reshape(B, H, L, d), np.swapaxes(R, 1, 2).reshape(B, H, M, d), S.reshape(B, H, M))
+
+
+def oracle_bidir_bwd(q, k, v, omega, dout, S_state, z_state, C, feature):
+    """Non-causal backward from the global state.  Returns dq, dk, dv, domega."""
+    Q, (B, H) = _chains(q)
+    K, _ = _chains(k)
+    V, _ = _chains(v)
+    dY, _ = _chains(dout)
+    Omega = np.asarray(omega, dtype=np.float64)
+    M = Omega.shape[0]
+    L, d = Q.shape[1], Q.shape[2]
+    R = np.swapaxes(np.asarray(S_state, np.float64).reshape(B * H, M, d), 1, 2)
+    S = np.asarray(z_state, np.float64).reshape(B * H, M)
+    dQ, dK, dV, dOmega, _ = bidir.backward(Q, K, V, Omega, dY, C, feature, R, S)
+    return (dQ.reshape(B, H, L, d), dK.reshape(B, H, L, d), dV.reshape(B, H, L, d), dOmega)
 
 
 def rel_l2(a, b):

@@ -10,12 +10,13 @@ import numpy as np
 from .brute import att_lin_quadratic
 
 
-def _objective(Q, K, V, Omega, dY, feature):
-    return float(np.sum(dY * att_lin_quadratic(Q, K, V, Omega, feature)))
+def _objective(Q, K, V, Omega, dY, feature, fn=att_lin_quadratic):
+    return float(np.sum(dY * fn(Q, K, V, Omega, feature)))
 
 
-def central_differences(Q, K, V, Omega, dY, feature, h=1e-6):
-    """Returns (dQ, dK, dV, dOmega) by (f(x+h e_i) - f(x-h e_i)) / 2h."""
+def central_differences(Q, K, V, Omega, dY, feature, h=1e-6, fn=att_lin_quadratic):
+    """Returns (dQ, dK, dV, dOmega) by (f(x+h e_i) - f(x-h e_i)) / 2h, f the
+    scalar <dY, fn(Q, K, V, Omega)> (eq. 2 by default)."""
     args = [np.array(a, dtype=np.float64) for a in (Q, K, V, Omega)]
     grads = []
     for which in range(4):
@@ -26,9 +27,9 @@ def central_differences(Q, K, V, Omega, dY, feature, h=1e-6):
             idx = it.multi_index
             keep = x[idx]
             x[idx] = keep + h
-            fp = _objective(*args, dY, feature)
+            fp = _objective(*args, dY, feature, fn)
             x[idx] = keep - h
-            fm = _objective(*args, dY, feature)
+            fm = _objective(*args, dY, feature, fn)
             x[idx] = keep
             g[idx] = (fp - fm) / (2.0 * h)
         grads.append(g)

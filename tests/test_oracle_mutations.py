@@ -84,6 +84,20 @@ def _g_abs(X, Omega):
 
 _orig_vjp = features.feature_vjp
 
+
+def _bidir_backward_drop_key_normaliser(Q, K, V, Omega, dY, C, feature, R, S):
+    # mistake: the non-causal key gradient without the normaliser's share G_S
+    from oracle import bidir
+    orig = _BIDIR_BACKWARD
+    dQ, dK, dV, dO, (G_R, G_S) = orig(Q, K, V, Omega, dY, C, feature, R, S)
+    Kt = features.feature_map(K, Omega, feature)
+    bad, _ = features.feature_vjp(K, Omega, np.broadcast_to(G_S[:, None, :], Kt.shape), feature)
+    return dQ, dK - bad, dV, dO, (G_R, G_S)
+
+
+from oracle import bidir as _bidir  # noqa: E402
+_BIDIR_BACKWARD = _bidir.backward
+
 MUTATIONS = {
     "exclusive_mask": (lambda mp: mp.setattr(sliced, "_forward_rows", _exclusive_forward_rows),
                        lambda: P.pin_brute_vs_sliced("exp"), 1e-6),
@@ -107,6 +121,9 @@ MUTATIONS = {
         lambda: P.pin_finite_differences("square"), 1e-3),
     "square_map_is_abs": (lambda mp: mp.setattr(features, "g_square", _g_abs),
                           lambda: P.pin_golden(), 1e-6),
+    "bidir_key_grad_missing_normaliser": (
+        lambda mp: mp.setattr(_bidir, "backward", _bidir_backward_drop_key_normaliser),
+        lambda: P.pin_bidir_finite_differences("exp"), 1e-3),
 }
 
 

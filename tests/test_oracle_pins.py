@@ -400,3 +400,64 @@ def pin_streaming_backward(feature):
 @pytest.mark.parametrize("feature", ["exp", "relu", "square"])
 def test_streaming_backward(feature):
     assert pin_streaming_backward(feature) < 1e-12
+
+
+# ----------------------------------------------------------------------------- non-causal form
+
+from oracle import bidir  # noqa: E402
+
+
+def pin_bidir_quadratic_vs_sweeps(feature, Cs=(1, 3, 16, 40, 64)):
+    """The non-causal definition row by row against the two slice sweeps, for
+    several slice sizes (the result does not depend on C)."""
+    Q, K, V, Omega, _ = small_case(20, feature=feature)
+    Yq = bidir.quadratic(Q, K, V, Omega, feature)
+    return max(rel(bidir.forward(Q, K, V, Omega, C, feature)[0], Yq) for C in Cs)
+
+
+def pin_bidir_zero_omega_closed_form():
+    """Omega = 0 with the exp map: every weight is w_j = exp(-|k_j|^2/2)/M,
+    independent of the query, so every row is the same global weighted mean."""
+    Q, K, V, _, _ = small_case(21, chains=1, L=30)
+    Y, _, _ = bidir.forward(Q, K, V, np.zeros((5, Q.shape[-1])), 7, "exp")
+    w = np.exp(-0.5 * np.sum(K[0] ** 2, axis=1))
+    mean = (w[:, None] * V[0]).sum(axis=0) / w.sum()
+    return rel(Y[0], np.broadcast_to(mean, Y[0].shape))
+
+
+def pin_bidir_finite_differences(feature, C=3):
+    """Central differences of <dY, Y> on the row-by-row definition against the
+    two backward sweeps."""
+    Q, K, V, Omega, dY = small_case(22, chains=1, L=7, d=3, M=5, feature=feature)
+    _, R, S = bidir.forward(Q, K, V, Omega, C, feature)
+    dQ, dK, dV, dO, _ = bidir.backward(Q, K, V, Omega, dY, C, feature, R, S)
+    fQ, fK, fV, fO = fd.central_differences(Q, K, V, Omega, dY, feature, fn=bidir.quadratic)
+    return max(rel(dQ, fQ), rel(dK, fK), rel(dV, fV), rel(dO, fO))
+
+
+def pin_bidir_last_row_is_causal():
+    """The last row reads every key in both forms: there the non-causal output
+    equals the causal one (eq. 2 at l = L), and the global state equals the
+    causal final state."""
+    Q, K, V, Omega, _ = small_case(23, feature="exp")
+    Yb, Rb, Sb = bidir.forward(Q, K, V, Omega, 8, "exp")
+    Yc, Rc, Sc = sliced.forward(Q, K, V, Omega, 8, "exp")
+    return max(rel(Yb[:, -1], Yc[:, -1]), rel(Rb, Rc), rel(Sb, Sc))
+
+
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
+def test_bidir_quadratic_vs_sweeps(feature):
+    assert pin_bidir_quadratic_vs_sweeps(feature) < 1e-12
+
+
+def test_bidir_zero_omega_closed_form():
+    assert pin_bidir_zero_omega_closed_form() < 1e-13
+
+
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
+def test_bidir_finite_differences(feature):
+    assert pin_bidir_finite_differences(feature) < 1e-6
+
+
+def test_bidir_last_row_is_causal():
+    assert pin_bidir_last_row_is_causal() < 1e-12
