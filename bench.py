@@ -1,11 +1,16 @@
 """Benchmark: fwd+bwd tokens/s of sliced causal Performer attention on GB300.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload NAME] [--C C] [--sweep]
+                    [--workload NAME] [--C C] [--mode causal|bidir|segments]
+                    [--segments S] [--sweep]
 
 A step is one slim_fwd + slim_bwd over the whole workload (every chain, every
 slice).  The default workload is B=8 H=8 L=4096 d=64 M=256, bf16 inputs, fp32
-accumulation, FAVOR+ features, slice C=1024.  Rank 0 prints ONE JSON line.
+accumulation, FAVOR+ features, slice C=1024.  Rank 0 prints ONE JSON line; on
+the default workload it carries `mem_vs_C`, the time and peak memory of the
+B2 H8 L32768 workload for each slice size C.  --mode bidir times the
+non-causal form instead, --mode segments the causal sweeps over S chained
+segment calls (slim_fwd_from / slim_bwd_from).
 
 Under torchrun (N > 1) every rank runs an independent replica of the workload
 on its own GPU (the chains are independent; there is no data-path
@@ -67,6 +72,11 @@ def parse():
     ap.add_argument("--H", type=int, default=None)
     ap.add_argument("--sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-mem-curve", action="store_true")
+    # what one step runs: the causal sweeps (default), the non-causal form, or
+    # the causal sweeps over --segments chained calls (streaming)
+    ap.add_argument("--mode", choices=["causal", "bidir", "segments"], default="causal")
+    ap.add_argument("--segments", type=int, default=4)
     return ap.parse_args()
 
 
@@ -267,8 +277,9 @@ def step_ceilings(w, B, H, L, ms_per_step):
 
 # ------------------------------------------------------------------ CPU oracle
 def _oracle_chain(args):
-    """One chain's fp64 oracle fwd+bwd (runs in a spawned worker)."""
-    name, overrides, b, h = args
+    """One chain's fp64 oracle fwd+bwd (runs in a spawned worker); the
+    non-causal form for mode bidir, the causal sweeps otherwise."""
+    name, overrides, b, h, mode = args
     os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
     os.environ.setdefault("OMP_NUM_THREADS", "1")
     import oracle
@@ -277,8 +288,13 @@ def _oracle_chain(args):
     x = W.make_inputs(w)
     c = {n: W.as_float64_numpy(t[b:b + 1, h:h + 1] if t.dim() == 4 else t) for n, t in x.items()}
     t0 = time.perf_counter()
-    o, S, z = oracle.oracle_fwd(c["q"], c["k"], c["v"], c["omega"], w.C, w.feature)
-    oracle.oracle_bwd(c["q"], c["k"], c["v"], c["omega"], c["dout"], S, z, w.C, w.feature)
+    if mode == "bidir":
+        o, S, z = oracle.oracle_bidir_fwd(c["q"], c["k"], c["v"], c["omega"], w.C, w.feature)
+        oracle.oracle_bidir_bwd(c["q"], c["k"], c["v"], c["omega"], c["dout"], S, z, w.C,
+                                w.feature)
+    else:
+        o, S, z = oracle.oracle_fwd(c["q"], c["k"], c["v"], c["omega"], w.C, w.feature)
+        oracle.oracle_bwd(c["q"], c["k"], c["v"], c["omega"], c["dout"], S, z, w.C, w.feature)
     return time.perf_counter() - t0
 
 
@@ -306,21 +322,231 @@ def start_oracle_pool(n):
     return pool
 
 
-def oracle_sample(w, overrides, pool, nchains):
+def oracle_sample(w, overrides, pool, nchains, mode="causal"):
     """Runs nchains chains of the workload through the oracle in parallel;
     returns (tokens, wall seconds)."""
-    jobs = [(w.name, overrides, (i // w.H) % w.B, i % w.H) for i in range(nchains)]
+    jobs = [(w.name, overrides, (i // w.H) % w.B, i % w.H, mode) for i in range(nchains)]
     secs = pool.map(_oracle_chain, jobs)
     # the chains run side by side; input generation is outside each worker's clock
     return nchains * w.L, max(secs)
 
 
 # ------------------------------------------------------------------ our arm
+class StepSet:
+    """Device buffers of one step and the calls that make it.  mode causal:
+    slim_fwd + slim_bwd (with the forward's residuals); bidir: the non-causal
+    pair; segments: the sequence cut into `segments` contiguous segments, the
+    forwards chained through slim_fwd_from and the backwards, last segment
+    first, through slim_bwd_from (each hands G^(0) to the one before)."""
+
+    def __init__(self, w, dev, mode, segments, x=None):
+        import torch
+        from paper_2012_11346_gb300 import slim
+        from paper_2012_11346_gb300 import workloads as W
+        self.w, self.mode, self.slim = w, mode, slim
+        self.x = x if x is not None else W.make_inputs(w, device=dev)
+        B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
+        q = self.x["q"]
+        f32 = torch.float32
+        self.om = None if w.feature == "square" else self.x["omega"]
+        if mode == "segments":
+            cuts = [round(i * L / segments) for i in range(segments + 1)]
+            self.segs = []
+            for a, b in zip(cuts[:-1], cuts[1:]):
+                sg = {n: self.x[n][:, :, a:b].contiguous() for n in ("q", "k", "v", "dout")}
+                sg.update(out=torch.empty_like(sg["q"]), dq=torch.empty_like(sg["q"]),
+                          dk=torch.empty_like(sg["q"]), dv=torch.empty_like(sg["q"]),
+                          S=torch.empty(B, H, M, d, dtype=f32, device=dev),
+                          z=torch.empty(B, H, M, dtype=f32, device=dev),
+                          S_lo=torch.empty(B, H, M, d, dtype=f32, device=dev),
+                          z_lo=torch.empty(B, H, M, dtype=f32, device=dev),
+                          G=torch.empty(B, H, M, d, dtype=f32, device=dev),
+                          gz=torch.empty(B, H, M, dtype=f32, device=dev),
+                          dom=torch.empty(M, d, dtype=f32, device=dev))
+                self.segs.append(sg)
+            Lmax = max(b - a for a, b in zip(cuts[:-1], cuts[1:]))
+            self.ws_f = self._ws(slim.workspace_size(B, H, Lmax, d, M, w.C, q.dtype, w.feature,
+                                                     False), dev)
+            self.ws_b = self._ws(slim.workspace_size(B, H, Lmax, d, M, w.C, q.dtype, w.feature,
+                                                     True), dev)
+            self.outputs = [t for sg in self.segs for t in (sg["out"], sg["dq"], sg["dk"],
+                                                            sg["dv"], sg["dom"])]
+            self.inputs = [t for sg in self.segs for t in (sg["q"], sg["k"], sg["v"],
+                                                           sg["dout"])] + [self.x["omega"]]
+            return
+        self.out = torch.empty_like(q)
+        self.S = torch.empty(B, H, M, d, dtype=f32, device=dev)
+        self.z = torch.empty(B, H, M, dtype=f32, device=dev)
+        self.S_lo, self.z_lo = torch.empty_like(self.S), torch.empty_like(self.z)
+        self.dq, self.dk, self.dv = (torch.empty_like(q) for _ in range(3))
+        self.dom = torch.empty(M, d, dtype=f32, device=dev)
+        if mode == "bidir":
+            size = slim.bidir_workspace_size
+            self.ws_f = self._ws(size(B, H, L, d, M, w.C, q.dtype, w.feature, False), dev)
+            self.ws_b = self._ws(size(B, H, L, d, M, w.C, q.dtype, w.feature, True), dev)
+        else:
+            size = slim.workspace_size
+            self.ws_f = self._ws(size(B, H, L, d, M, w.C, q.dtype, w.feature, False), dev)
+            self.ws_b = self._ws(size(B, H, L, d, M, w.C, q.dtype, w.feature, True), dev)
+        self.outputs = [self.out, self.dq, self.dk, self.dv, self.dom]
+        self.inputs = [self.x[n] for n in ("q", "k", "v", "dout", "omega")]
+
+    @staticmethod
+    def _ws(n, dev):
+        import torch
+        return torch.empty(max(256, n), dtype=torch.uint8, device=dev)
+
+    def run(self, stream=None):
+        sl, w, x, om = self.slim, self.w, self.x, self.om
+        C, f = w.C, w.feature
+        if self.mode == "causal":
+            sl.forward_into(x["q"], x["k"], x["v"], om, C, f, self.out, self.S, self.z, self.ws_f,
+                            stream, S_lo=self.S_lo, z_lo=self.z_lo)
+            sl.backward_into(x["q"], x["k"], x["v"], om, self.out, x["dout"], self.S, self.z, C, f,
+                             self.dq, self.dk, self.dv, self.dom, self.ws_b, stream,
+                             S_lo=self.S_lo, z_lo=self.z_lo)
+        elif self.mode == "bidir":
+            sl.forward_bidir_into(x["q"], x["k"], x["v"], om, C, f, self.out, self.S, self.z,
+                                  self.ws_f, stream)
+            sl.backward_bidir_into(x["q"], x["k"], x["v"], om, self.out, x["dout"], self.S,
+                                   self.z, C, f, self.dq, self.dk, self.dv, self.dom, self.ws_b,
+                                   stream)
+        else:
+            prev = None
+            for sg in self.segs:
+                sl.forward_into(sg["q"], sg["k"], sg["v"], om, C, f, sg["out"], sg["S"], sg["z"],
+                                self.ws_f, stream, S_lo=sg["S_lo"], z_lo=sg["z_lo"],
+                                S_init=None if prev is None else prev["S"],
+                                z_init=None if prev is None else prev["z"],
+                                S_init_lo=None if prev is None else prev["S_lo"],
+                                z_init_lo=None if prev is None else prev["z_lo"])
+                prev = sg
+            nxt = None
+            for sg in reversed(self.segs):
+                sl.backward_into(sg["q"], sg["k"], sg["v"], om, sg["out"], sg["dout"], sg["S"],
+                                 sg["z"], C, f, sg["dq"], sg["dk"], sg["dv"], sg["dom"],
+                                 self.ws_b, stream, S_lo=sg["S_lo"], z_lo=sg["z_lo"],
+                                 G_S_in=None if nxt is None else nxt["G"],
+                                 g_z_in=None if nxt is None else nxt["gz"],
+                                 G_S_out=sg["G"], g_z_out=sg["gz"])
+                nxt = sg
+
+    def check(self):
+        self.slim.check_device_error(self.ws_f)
+        self.slim.check_device_error(self.ws_b)
+
+
+def e2e_pipelined(sets, host_in, host_out, steps, warmup):
+    """End to end through the public API: every step copies its inputs in from
+    pinned host memory and its results (out, dq, dk, dv, dOmega) back.  Two
+    buffer sets alternate, so step i's copy in runs during step i-1's compute
+    and its copy out during step i+1's compute, on two copy streams; each step
+    still moves its own bytes.  Returns ms for `steps` steps."""
+    import torch
+    cin, comp, cout = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev = {k: [torch.cuda.Event() for _ in range(2)] for k in ("in", "comp", "out")}
+    used = [False, False]
+
+    def issue(i):
+        b = i % 2
+        st = sets[b]
+        with torch.cuda.stream(cin):
+            if used[b]:
+                cin.wait_event(ev["comp"][b])         # step i-2 has read these inputs
+            for dst, src in zip(st.inputs, host_in[b]):
+                dst.copy_(src, non_blocking=True)
+            ev["in"][b].record(cin)
+        comp.wait_event(ev["in"][b])
+        if used[b]:
+            comp.wait_event(ev["out"][b])             # step i-2's results have left
+        st.run(comp)
+        ev["comp"][b].record(comp)
+        with torch.cuda.stream(cout):
+            cout.wait_event(ev["comp"][b])
+            for dst, src in zip(host_out[b], st.outputs):
+                dst.copy_(src, non_blocking=True)
+            ev["out"][b].record(cout)
+        used[b] = True
+
+    for i in range(warmup):
+        issue(i)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(cin)
+    for i in range(warmup, warmup + steps):
+        issue(i)
+    cout.wait_stream(cin)
+    cout.wait_stream(comp)
+    t1.record(cout)
+    torch.cuda.synchronize()
+    return t0.elapsed_time(t1)
+
+
+def mem_vs_C(dev, steps):
+    """Peak device memory and tokens/s for each slice size C of the B2 H8
+    L32768 d64 M256 bf16 workload (Sec. 4.1's time/memory-vs-C protocol, Fig. 2):
+    workspace bytes, the measured peak above the inputs and outputs (IO floor),
+    and the same method on an input of length C alone (the length-C point)."""
+    import torch
+    from paper_2012_11346_gb300 import slim
+    from paper_2012_11346_gb300 import workloads as W
+    w0 = W.WORKLOADS["L32768_bf16"]
+    x = W.make_inputs(w0, device=dev)
+    floor = sum(t.numel() * t.element_size() for t in x.values()) + \
+        4 * x["q"].numel() * x["q"].element_size()   # + out, dq, dk, dv
+    rows = []
+    for C in W.C_SWEEP:
+        w = w0.with_(C=C)
+
+        def step():
+            o, S, z, Sl, zl = slim.forward(x["q"], x["k"], x["v"], x["omega"], C, w.feature,
+                                           residuals=True)
+            slim.backward(x["q"], x["k"], x["v"], x["omega"], o, x["dout"], S, z, C, w.feature,
+                          S_lo=Sl, z_lo=zl)
+
+        step()
+        torch.cuda.synchronize()
+        torch.cuda.reset_peak_memory_stats(dev)
+        base = torch.cuda.memory_allocated(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(steps):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / steps
+        peak = torch.cuda.max_memory_allocated(dev)
+        outs = 4 * x["q"].numel() * x["q"].element_size()      # out, dq, dk, dv
+        xl = {n: (t[:, :, :C].contiguous() if t.dim() == 4 else t) for n, t in x.items()}
+        torch.cuda.synchronize()
+        torch.cuda.reset_peak_memory_stats(dev)
+        base_lb = torch.cuda.memory_allocated(dev)
+        o, S, z, Sl, zl = slim.forward(xl["q"], xl["k"], xl["v"], xl["omega"], C, w.feature,
+                                       residuals=True)
+        slim.backward(xl["q"], xl["k"], xl["v"], xl["omega"], o, xl["dout"], S, z, C, w.feature,
+                      S_lo=Sl, z_lo=zl)
+        torch.cuda.synchronize()
+        lb_above = torch.cuda.max_memory_allocated(dev) - base_lb
+        del xl, o, S, z, Sl, zl
+        rows.append({"C": C, "tokens_per_s": round(w.B * w.L / (ms / 1e3), 1),
+                     "ms_per_step": round(ms, 3),
+                     "workspace_bytes": slim.workspace_size(w.B, w.H, w.L, w.d, w.M, C,
+                                                            x["q"].dtype, w.feature, False)
+                     + slim.workspace_size(w.B, w.H, w.L, w.d, w.M, C, x["q"].dtype,
+                                           w.feature, True),
+                     "peak_above_inputs_bytes": peak - base,
+                     "peak_above_io_floor_bytes": peak - base - outs,
+                     "length_C_input_above_inputs_bytes": lb_above})
+    del x
+    torch.cuda.empty_cache()
+    return {"workload": "B2 H8 L32768 d64 M256 bf16 exp", "io_floor_bytes": floor,
+            "steps_per_C": steps, "rows": rows}
+
+
 def run_ours(args, rank, ws, local):
     import torch
     from paper_2012_11346_gb300 import slim
     from paper_2012_11346_gb300 import workloads as W
-
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
@@ -331,24 +557,9 @@ def run_ours(args, rank, ws, local):
         w = w.with_(B=args.B)
     if args.H:
         w = w.with_(H=args.H)
-    x = W.make_inputs(w, device=dev)
-    q, k, v, om, dout = x["q"], x["k"], x["v"], x["omega"], x["dout"]
     B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
-    out = torch.empty_like(q)
-    S = torch.empty(B, H, M, d, dtype=torch.float32, device=dev)
-    z = torch.empty(B, H, M, dtype=torch.float32, device=dev)
-    S_lo, z_lo = torch.empty_like(S), torch.empty_like(z)
-    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
-    dom = torch.empty(M, d, dtype=torch.float32, device=dev)
-    wsf = torch.empty(max(256, slim.workspace_size(B, H, L, d, M, w.C, q.dtype, w.feature, False)),
-                      dtype=torch.uint8, device=dev)
-    wsb = torch.empty(max(256, slim.workspace_size(B, H, L, d, M, w.C, q.dtype, w.feature, True)),
-                      dtype=torch.uint8, device=dev)
-
-    def step():
-        slim.forward_into(q, k, v, om, w.C, w.feature, out, S, z, wsf, S_lo=S_lo, z_lo=z_lo)
-        slim.backward_into(q, k, v, om, out, dout, S, z, w.C, w.feature, dq, dk, dv, dom, wsb,
-                           S_lo=S_lo, z_lo=z_lo)
+    main = StepSet(w, dev, args.mode, args.segments)
+    step = main.run
 
     for _ in range(args.warmup):
         step()
@@ -371,8 +582,7 @@ def run_ours(args, rank, ws, local):
     barrier(ws)
     launches = slim.launch_count() - launches0
     clocks = sampler.stop()
-    slim.check_device_error(wsf)
-    slim.check_device_error(wsb)
+    main.check()
     ms = max_over_ranks(e0.elapsed_time(e1), ws)
     tokens = sum_over_ranks(B * L * args.steps, ws)
     value = tokens / (ms / 1e3)
@@ -390,55 +600,44 @@ def run_ours(args, rank, ws, local):
     ms_profiled = e0.elapsed_time(e1)
     stats = slim.profiler_read()
     # a bounded device wait that gave up would make the timings meaningless
-    slim.check_device_error(wsf)
-    slim.check_device_error(wsb)
+    main.check()
 
     # untimed validation pass: every call clears the device error word at its
     # start, so check it after each step; a bounded wait that gave up during
     # the measurement would make the numbers above meaningless
     for _ in range(args.steps):
         step()
-        slim.check_device_error(wsf)
-        slim.check_device_error(wsb)
+        main.check()
 
-    # end to end through the public API: pinned host inputs in, results out
-    hq, hk, hv, hdo = (t.cpu().pin_memory() for t in (q, k, v, dout))
-    hom = om.cpu().pin_memory()
-    hout, hdq, hdk, hdv = (torch.empty(q.shape, dtype=q.dtype).pin_memory() for _ in range(4))
-    hdom = torch.empty(M, d, dtype=torch.float32).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hdo, hom))
-    d2h = sum(t.numel() * t.element_size() for t in (hout, hdq, hdk, hdv, hdom))
-
-    def e2e_step():
-        for dst, src in ((q, hq), (k, hk), (v, hv), (dout, hdo), (om, hom)):
-            dst.copy_(src, non_blocking=True)
-        step()
-        for dst, src in ((hout, out), (hdq, dq), (hdk, dk), (hdv, dv), (hdom, dom)):
-            dst.copy_(src, non_blocking=True)
-
-    for _ in range(args.warmup):
-        e2e_step()
+    # end to end through the public API: pinned host inputs in, results out,
+    # copies overlapped with the neighbouring steps' compute (two buffer sets)
+    second = StepSet(w, dev, args.mode, args.segments, x=None)
+    sets = [main, second]
+    host_in = [[t.cpu().pin_memory() for t in st.inputs] for st in sets]
+    host_out = [[torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in st.outputs]
+                for st in sets]
+    h2d = sum(t.numel() * t.element_size() for t in main.inputs)
+    d2h = sum(t.numel() * t.element_size() for t in main.outputs)
     barrier(ws)
-    torch.cuda.synchronize()
-    e0.record(stream)
-    for _ in range(args.steps):
-        e2e_step()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier(ws)
-    ms_e2e = max_over_ranks(e0.elapsed_time(e1), ws)
+    ms_e2e = max_over_ranks(e2e_pipelined(sets, host_in, host_out, args.steps, args.warmup), ws)
     e2e_value = tokens / (ms_e2e / 1e3)
+    del second, sets, host_in, host_out
+    torch.cuda.empty_cache()
 
     # peak device memory of one fwd+bwd through the allocating API
-    del hq, hk, hv, hdo
-    torch.cuda.synchronize()
-    torch.cuda.reset_peak_memory_stats(dev)
-    base = torch.cuda.memory_allocated(dev)
-    o2, S2, z2, S2l, z2l = slim.forward(q, k, v, om, w.C, w.feature, residuals=True)
-    g2 = slim.backward(q, k, v, om, o2, dout, S2, z2, w.C, w.feature, S_lo=S2l, z_lo=z2l)
-    torch.cuda.synchronize()
-    peak = torch.cuda.max_memory_allocated(dev)
-    del o2, S2, z2, S2l, z2l, g2
+    peak, base = None, None
+    if args.mode == "causal":
+        x = main.x
+        torch.cuda.synchronize()
+        torch.cuda.reset_peak_memory_stats(dev)
+        base = torch.cuda.memory_allocated(dev)
+        o2, S2, z2, S2l, z2l = slim.forward(x["q"], x["k"], x["v"], main.om, w.C, w.feature,
+                                            residuals=True)
+        g2 = slim.backward(x["q"], x["k"], x["v"], main.om, o2, x["dout"], S2, z2, w.C,
+                           w.feature, S_lo=S2l, z_lo=z2l)
+        torch.cuda.synchronize()
+        peak = torch.cuda.max_memory_allocated(dev)
+        del o2, S2, z2, S2l, z2l, g2
 
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws,
@@ -446,22 +645,30 @@ def run_ours(args, rank, ws, local):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": path_dtype(stats, w), "data": "synthetic",
         "config": {"workload": w.name, "B": B, "H": H, "L": L, "d": d, "M": M, "C": w.C,
-                   "feature": w.feature, "input_dtype": w.dtype,
+                   "feature": w.feature, "input_dtype": w.dtype, "mode": args.mode,
+                   **({"segments": args.segments} if args.mode == "segments" else {}),
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
                    "l2": "no flush; per-step working set (q,k,v,dout,out,dq,dk,dv) "
-                         f"{8 * q.numel() * q.element_size() / 2**20:.0f} MiB > L2 129 MiB"},
+                         f"{8 * main.x['q'].numel() * main.x['q'].element_size() / 2**20:.0f} MiB "
+                         "> L2 129 MiB"},
         "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
+                "d2h_bytes_per_step": d2h,
+                "overlap": "copies of step i overlap compute of steps i-1 and i+1"},
         "gpu_launches": int(launches),
         "roofline": roofline(stats, args.steps),
         "ceilings": step_ceilings(w, B, H, L, ms / args.steps),
         "profiled_ms_per_step": round(ms_profiled / args.steps, 4),
         "clocks": clocks,
-        "peak_mem": {"bytes": peak, "above_inputs_bytes": peak - base,
-                     "workspace_bytes": wsb.numel()},
+        "peak_mem": ({"bytes": peak, "above_inputs_bytes": peak - base,
+                      "workspace_bytes": main.ws_b.numel()} if peak is not None else None),
         "kernels": [{k_: (round(v_, 4) if isinstance(v_, float) else v_) for k_, v_ in s.items()}
                     for s in stats],
     }
+    del main
+    torch.cuda.empty_cache()
+    if (rank == 0 and ws == 1 and not args.no_mem_curve and args.mode == "causal"
+            and args.workload == DEFAULT_WORKLOAD and not (args.B or args.H or args.C)):
+        line["mem_vs_C"] = mem_vs_C(dev, 3)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         # The oracle pool starts only after every GPU measurement: with an
         # idle pool alive during the GPU passes, the end-to-end pass was
@@ -469,7 +676,7 @@ def run_ours(args, rank, ws, local):
         # inherit the parent's CUDA context.
         n = oracle_pool_size()
         pool = start_oracle_pool(n)
-        tok, sec = oracle_sample(w, {"C": w.C}, pool, n)
+        tok, sec = oracle_sample(w, {"C": w.C}, pool, n, args.mode)
         line["cpu_baseline"] = {"value": round(tok / sec, 2), "unit": "tokens/s", "cores": n,
                                 "kind": "oracle",
                                 "sample": f"{n} chains x L={L} of this workload, fp64 NumPy, "
@@ -502,10 +709,10 @@ def run_reference(args, rank, ws):
     n = oracle_pool_size()
     with mp.get_context("spawn").Pool(n) as pool:
         for _ in range(args.warmup):
-            oracle_sample(w, {"C": w.C}, pool, n)
+            oracle_sample(w, {"C": w.C}, pool, n, args.mode)
         tok, sec = 0, 0.0
         for _ in range(args.steps):
-            t, s = oracle_sample(w, {"C": w.C}, pool, n)
+            t, s = oracle_sample(w, {"C": w.C}, pool, n, args.mode)
             tok += t
             sec += s
     value = tok / sec

@@ -214,6 +214,40 @@ slim_status slim_bwd_from(const void* q, const void* k, const void* v, const flo
                           void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * The non-causal (bidirectional) form: eq. 2 without the causal mask, every
+ * row reading every key,
+ *     out_i = sum_j (g(q_i).g(k_j)) v_j / sum_j g(q_i).g(k_j),   j = 1..L,
+ * so that one global state B = (S, z) (eq. 3 at the last row) serves every
+ * row.  The paper treats the causal form; this is the same computation with
+ * the prefix sums replaced by the full sum, with memory kept O(C) the same
+ * way: the forward reads the slices twice (accumulate B, then read it out)
+ * and the backward reads them twice (query side, accumulating the state
+ * gradient G, then key/value side, reading G).  It runs on the fp32-compute
+ * kernels for every supported problem.
+ *   slim_bidir_workspace_size: workspace bytes (backward != 0: the backward's).
+ *   slim_fwd_bidir: out and the global state S_state / z_state (written).
+ *   slim_bwd_bidir: gradients of <dout, out>; S_state / z_state as
+ *     slim_fwd_bidir returned them (read-only).
+ * Arguments, layouts and errors as for slim_fwd / slim_bwd (the quadratic map
+ * again needs no omega and writes no domega).  No device-side waits.
+ */
+slim_status slim_bidir_workspace_size(int B, int H, int L, int d, int M, int C,
+                                      slim_dtype dtype, slim_feature feature, int backward,
+                                      size_t* bytes);
+slim_status slim_fwd_bidir(const void* q, const void* k, const void* v, const float* omega,
+                           int B, int H, int L, int d, int M, int C,
+                           slim_dtype dtype, slim_feature feature,
+                           void* out, float* S_state, float* z_state,
+                           void* workspace, size_t workspace_bytes, void* stream);
+slim_status slim_bwd_bidir(const void* q, const void* k, const void* v, const float* omega,
+                           const void* out, const void* dout,
+                           const float* S_state, const float* z_state,
+                           int B, int H, int L, int d, int M, int C,
+                           slim_dtype dtype, slim_feature feature,
+                           void* dq, void* dk, void* dv, float* domega,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Which kernels serve this problem: *path = 1 for the tensor-core path
  * (tcgen05 MMAs, bf16 operands, fp32 accumulation; bf16 inputs with d = 64,
  * M in {128, 256} and slices of at least 64 rows), 0 for the fp32-compute

@@ -705,6 +705,144 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
   return SLIM_OK;
 }
 
+// ------------------------------------------------------------------ non-causal form
+// Eq. 2 without the mask: one global state B = sum over all rows (eq. 3 at
+// l = L) serves every row.  Memory stays O(C): the forward reads the slices
+// twice (accumulate B, then read it out), the backward twice as well (query
+// side, which also accumulates G = grad_B, then key/value side, which reads G).
+
+// Feature-map VJP of one side of a slice: u = dphi * g'(x) in place, dX stored
+// to rows [a, a+b) of dst, and the side's dOmega partial added to domega.
+template <typename IO>
+cudaError_t side_vjp(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w, float* dphi,
+                     const float* phi, const float* X, float* usum, const float* omega, void* dst,
+                     float* domega, int a, int b) {
+  const long long M = g.M, d = g.d, Cp = g.Cp;
+  const int rows = g.chains * g.Cp;
+  cudaError_t e;
+  if (p.feature == SLIM_FEAT_SQUARE) {
+    const long long n = (long long)rows * g.d;
+    { prof::Scope ps(prof::K_VJP, s);
+    k_vjp_square<<<blocks(n), 256, 0, s>>>(dphi, X, w.stage, n); }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  } else {
+    { prof::Scope ps(prof::K_VJP, s);
+    k_vjp_prep<<<blocks((long long)rows * 32), 256, 0, s>>>(dphi, phi, usum, g.M, rows,
+                                                            (int)p.feature,
+                                                            (float)(1.0 / sqrt((double)g.M))); }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const bool ex = p.feature == SLIM_FEAT_EXP;
+    e = gemm(s, g.precise, g.Cp, g.d, g.M, mat(dphi, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+             omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? X : nullptr, Cp * d, d,
+             usum, Cp);
+    if (e != cudaSuccess) return e;
+    e = gemm(s, g.precise, g.M, g.d, g.Cp, mat(dphi, Cp * M, 0, 1, M), mat(X, Cp * d, 0, d, 1),
+             omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 0.f, 0);
+    if (e != cudaSuccess) return e;
+    { prof::Scope ps(prof::K_REDUCE, s);
+    k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains,
+                                                             (int)(M * d)); }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+  k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dst, p.L, g.d,
+                                                                    a, b, g.Cp, g.chains); }
+  return cudaGetLastError();
+}
+
+template <typename T>
+slim_status fwd_bidir_impl(const Problem& p, const void* q, const void* k, const void* v,
+                           const float* omega, void* out, const StateOut& st, void* workspace,
+                           cudaStream_t s) {
+  const Geo g = geometry(p);
+  Carver cv(workspace);
+  const Ws w = carve(cv, g, false);
+  const long long TT = g.T, M = g.M, dp = g.dp, Cp = g.Cp;
+  const size_t E = (size_t)g.chains * g.M * g.dp;
+  SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(cudaMemsetAsync(w.st_hi, 0, E * sizeof(float), s));
+  SLIM_TRY(cudaMemsetAsync(w.st_lo, 0, E * sizeof(float), s));
+  // sweep 1: B = sum over every tile of every slice of g(K)^T [V | 1]
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(tile_deltas(s, g, w));
+    SLIM_TRY(scan(s, g, w.delta, w.st_hi, w.st_lo, SCAN_FWD));
+  }
+  { prof::Scope ps(prof::K_STATE, s);
+  k_state_out<<<blocks((long long)E), 256, 0, s>>>(w.st_hi, w.st_lo, st, g.chains, g.M, g.d); }
+  SLIM_TRY(cudaGetLastError());
+  // sweep 2: [num | den] = g(Q) B, out = num / den
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(gemm(s, g.precise, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, TT * M, M, 1),
+                  mat(w.st_hi, M * dp, 0, dp, 1), omat(w.numden, Cp * dp, TT * dp, dp, 1),
+                  g.chains, g.nt, 0.f, 0));
+    { prof::Scope ps(prof::K_FINALIZE, s, 0.0, (double)g.chains * b * g.d * sizeof(T));
+    k_finalize_out<T><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(
+        w.numden, (T*)out, p.L, g.d, a, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+  }
+  return SLIM_OK;
+}
+
+template <typename IO>
+slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const void* v,
+                           const float* omega, const void* out, const void* dout,
+                           const StateIn& st, void* dq, void* dk, void* dv, float* domega,
+                           void* workspace, cudaStream_t s) {
+  const Geo g = geometry(p);
+  Carver cv(workspace);
+  const Ws w = carve(cv, g, true);
+  const long long T = g.T, M = g.M, d = g.d, dp = g.dp, Cp = g.Cp, nt = g.nt;
+  const size_t E = (size_t)g.chains * g.M * g.dp;
+  SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  if (domega) SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
+  { prof::Scope ps(prof::K_STATE, s);
+  k_state_in<<<blocks((long long)E), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains, g.M, g.d); }
+  SLIM_TRY(cudaGetLastError());
+  SLIM_TRY(cudaMemsetAsync(w.g_hi, 0, E * sizeof(float), s));
+  SLIM_TRY(cudaMemsetAsync(w.g_lo, 0, E * sizeof(float), s));
+  // sweep 1, query side: W = [dnum | dden], dphiQ = W B^T, G += g(Q)^T W
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
+    SLIM_TRY(gemm(s, g.precise, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+                  mat(w.st_hi, M * dp, 0, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
+                  g.chains, g.nt, 0.f, 0));
+    { prof::Scope ps(prof::K_DSTAT, s);
+    k_dstat<<<blocks((long long)g.chains * Cp * dp), 256, 0, s>>>(w.numden, w.dout32, w.rowdot,
+                                                                  w.W, g.d, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+                  mat(w.st_hi, M * dp, 0, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
+                  g.chains, g.nt, 0.f, 0));
+    SLIM_TRY(gemm(s, g.precise, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+                  mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
+                  g.chains, g.nt, 0.f, 0));
+    SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
+    SLIM_TRY(side_vjp<IO>(s, p, g, w, w.dphiQ, w.phiQ, w.Xq, w.usum_q, omega, dq, domega, a, b));
+  }
+  // sweep 2, key/value side: dphiK = [V | 1] G^T, dV = g(K) G_S
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+                  mat(w.g_hi, M * dp, 0, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
+                  g.nt, 0.f, 0));
+    SLIM_TRY(gemm(s, g.precise, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+                  mat(w.g_hi, M * dp, 0, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
+                  g.nt, 0.f, 0));
+    { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
+    k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dv, p.L, g.d,
+                                                                      a, b, g.Cp, g.chains); }
+    SLIM_TRY(cudaGetLastError());
+    SLIM_TRY(side_vjp<IO>(s, p, g, w, w.dphiK, w.phiK, w.Xk, w.usum_k, omega, dk, domega, a, b));
+  }
+  return SLIM_OK;
+}
+
 }  // namespace
 
 size_t workspace_bytes(const Problem& p, bool bwd) {
@@ -731,6 +869,31 @@ slim_status bwd(const Problem& p, const void* q, const void* k, const void* v,
                                    domega, workspace, s);
   return bwd_impl<float>(p, q, k, v, omega, out, dout, st, gio, dq, dk, dv, domega,
                          workspace, s);
+}
+
+}  // namespace simt
+}  // namespace slim
+
+namespace slim {
+namespace simt {
+
+slim_status fwd_bidir(const Problem& p, const void* q, const void* k, const void* v,
+                      const float* omega, void* out, const StateOut& st, void* workspace,
+                      cudaStream_t s) {
+  if (p.dtype == SLIM_BF16)
+    return fwd_bidir_impl<__nv_bfloat16>(p, q, k, v, omega, out, st, workspace, s);
+  return fwd_bidir_impl<float>(p, q, k, v, omega, out, st, workspace, s);
+}
+
+slim_status bwd_bidir(const Problem& p, const void* q, const void* k, const void* v,
+                      const float* omega, const void* out, const void* dout, const StateIn& st,
+                      void* dq, void* dk, void* dv, float* domega, void* workspace,
+                      cudaStream_t s) {
+  if (p.dtype == SLIM_BF16)
+    return bwd_bidir_impl<__nv_bfloat16>(p, q, k, v, omega, out, dout, st, dq, dk, dv, domega,
+                                         workspace, s);
+  return bwd_bidir_impl<float>(p, q, k, v, omega, out, dout, st, dq, dk, dv, domega, workspace,
+                               s);
 }
 
 }  // namespace simt

@@ -260,6 +260,76 @@ slim_status slim_bwd_from(const void* q, const void* k, const void* v, const flo
                   workspace, workspace_bytes, static_cast<cudaStream_t>(stream));
 }
 
+slim_status slim_bidir_workspace_size(int B, int H, int L, int d, int M, int C,
+                                      slim_dtype dtype, slim_feature feature, int backward,
+                                      size_t* bytes) {
+  if (!bytes) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  *bytes = slim::simt::workspace_bytes(p, backward != 0);
+  return SLIM_OK;
+}
+
+slim_status slim_fwd_bidir(const void* q, const void* k, const void* v, const float* omega,
+                           int B, int H, int L, int d, int M, int C, slim_dtype dtype,
+                           slim_feature feature, void* out, float* S_state, float* z_state,
+                           void* workspace, size_t workspace_bytes, void* stream) {
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  const void* seq[] = {q, k, v, out};
+  const void* fixed[] = {S_state, z_state};
+  const void* opt[] = {omega};
+  if (!pointers_ok(seq, 4, L == 0) || !pointers_ok(fixed, 2, false) || !pointers_ok(opt, 1, true))
+    return SLIM_ERR_INVALID_ARG;
+  if (omega == nullptr && feature != SLIM_FEAT_SQUARE) return SLIM_ERR_INVALID_ARG;
+  const size_t need = slim::simt::workspace_bytes(p, false);
+  if (workspace == nullptr || workspace_bytes < need) return SLIM_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SLIM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (L == 0) {
+    const size_t n = (size_t)p.chains() * M;
+    if (cudaMemsetAsync(S_state, 0, n * d * sizeof(float), s) != cudaSuccess ||
+        cudaMemsetAsync(z_state, 0, n * sizeof(float), s) != cudaSuccess)
+      return SLIM_ERR_CUDA;
+    return SLIM_OK;
+  }
+  return slim::simt::fwd_bidir(p, q, k, v, omega, out, slim::StateOut{S_state, z_state, nullptr,
+                                                                       nullptr},
+                               workspace, s);
+}
+
+slim_status slim_bwd_bidir(const void* q, const void* k, const void* v, const float* omega,
+                           const void* out, const void* dout, const float* S_state,
+                           const float* z_state, int B, int H, int L, int d, int M, int C,
+                           slim_dtype dtype, slim_feature feature, void* dq, void* dk, void* dv,
+                           float* domega, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  const void* seq[] = {q, k, v, out, dout, dq, dk, dv};
+  const void* fixed[] = {S_state, z_state};
+  const void* opt[] = {omega, domega};
+  if (!pointers_ok(seq, 8, L == 0) || !pointers_ok(fixed, 2, false) || !pointers_ok(opt, 2, true))
+    return SLIM_ERR_INVALID_ARG;
+  if ((omega == nullptr || domega == nullptr) && feature != SLIM_FEAT_SQUARE)
+    return SLIM_ERR_INVALID_ARG;
+  const size_t need = slim::simt::workspace_bytes(p, true);
+  if (workspace == nullptr || workspace_bytes < need) return SLIM_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SLIM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (L == 0) {
+    if (domega && cudaMemsetAsync(domega, 0, (size_t)M * d * sizeof(float), s) != cudaSuccess)
+      return SLIM_ERR_CUDA;
+    return SLIM_OK;
+  }
+  return slim::simt::bwd_bidir(p, q, k, v, omega, out, dout,
+                               slim::StateIn{S_state, z_state, nullptr, nullptr}, dq, dk, dv,
+                               domega, workspace, s);
+}
+
 slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype dtype,
                           slim_feature feature, int* path) {
   if (!path) return SLIM_ERR_INVALID_ARG;

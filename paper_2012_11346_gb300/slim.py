@@ -31,6 +31,9 @@ SIGNATURES = {
     "slim_bwd": ([_p] * 10 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
     "slim_fwd_from": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p] * 5 + [_p, _sz, _p], _i),
     "slim_bwd_from": ([_p] * 12 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p] * 2 + [_p, _sz, _p], _i),
+    "slim_bidir_workspace_size": ([_i] * 6 + [_i, _i, _i, ctypes.POINTER(_sz)], _i),
+    "slim_fwd_bidir": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 3 + [_p, _sz, _p], _i),
+    "slim_bwd_bidir": ([_p] * 8 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
     "slim_check_device_error": ([_p, _p], _i),
     "slim_launch_count": ([], ctypes.c_ulonglong),
     "slim_profiler_enable": ([_i], None),
@@ -213,27 +216,105 @@ def backward(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp", work
     return dq, dk, dv, domega
 
 
-def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None,
-                 S_lo=None, z_lo=None):
-    """slim_fwd into caller-allocated outputs and workspace (no allocation)."""
+def bidir_workspace_size(B, H, L, d, M, C, dtype, feature, backward):
+    n = _sz(0)
+    _check(library().slim_bidir_workspace_size(B, H, L, d, M, C, DTYPES[dtype],
+                                               FEATURES[feature], 1 if backward else 0,
+                                               ctypes.byref(n)), "slim_bidir_workspace_size")
+    return n.value
+
+
+def forward_bidir(q, k, v, omega, C, feature="exp", workspace=None, stream=None):
+    """slim_fwd_bidir (non-causal): returns (out, S_state, z_state), the state
+    being the global sum over all rows."""
+    _require_cuda(q, k, v)
     B, H, L, d, M = _dims(q, omega)
-    _check(library().slim_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega),
-                              B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
-                              out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
-                              _ptr(S_lo), _ptr(z_lo), workspace.data_ptr(), workspace.numel(),
-                              _stream_handle(stream)), "slim_fwd")
+    out = torch.empty_like(q)
+    S_state = torch.empty(B, H, M, d, dtype=torch.float32, device=q.device)
+    z_state = torch.empty(B, H, M, dtype=torch.float32, device=q.device)
+    ws = workspace if workspace is not None else _workspace(
+        bidir_workspace_size(B, H, L, d, M, C, q.dtype, feature, False), q.device)
+    _check(library().slim_fwd_bidir(q.data_ptr(), k.data_ptr(), v.data_ptr(), _opt_ptr(omega),
+                                    B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
+                                    out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
+                                    ws.data_ptr(), ws.numel(), _stream_handle(stream)),
+           "slim_fwd_bidir")
+    return out, S_state, z_state
+
+
+def backward_bidir(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp", workspace=None,
+                   stream=None):
+    """slim_bwd_bidir (non-causal): returns (dq, dk, dv, domega)."""
+    _require_cuda(q, k, v, out, dout, S_state, z_state)
+    B, H, L, d, M = _dims(q, omega)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    domega = (torch.empty(M, d, dtype=torch.float32, device=q.device)
+              if omega is not None else None)
+    ws = workspace if workspace is not None else _workspace(
+        bidir_workspace_size(B, H, L, d, M, C, q.dtype, feature, True), q.device)
+    _check(library().slim_bwd_bidir(q.data_ptr(), k.data_ptr(), v.data_ptr(), _opt_ptr(omega),
+                                    out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
+                                    z_state.data_ptr(), B, H, L, d, M, C, DTYPES[q.dtype],
+                                    FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
+                                    dv.data_ptr(), _ptr(domega), ws.data_ptr(), ws.numel(),
+                                    _stream_handle(stream)), "slim_bwd_bidir")
+    return dq, dk, dv, domega
+
+
+def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None,
+                 S_lo=None, z_lo=None, S_init=None, z_init=None, S_init_lo=None, z_init_lo=None):
+    """slim_fwd (slim_fwd_from with an initial state) into caller-allocated
+    outputs and workspace (no allocation)."""
+    B, H, L, d, M = _dims(q, omega)
+    args = (q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega), B, H, L, d, M, C,
+            DTYPES[q.dtype], FEATURES[feature])
+    tail = (out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo),
+            workspace.data_ptr(), workspace.numel(), _stream_handle(stream))
+    if S_init is None:
+        _check(library().slim_fwd(*args, *tail), "slim_fwd")
+    else:
+        _check(library().slim_fwd_from(*args, _ptr(S_init), _ptr(z_init), _ptr(S_init_lo),
+                                       _ptr(z_init_lo), *tail), "slim_fwd_from")
 
 
 def backward_into(q, k, v, omega, out, dout, S_state, z_state, C, feature, dq, dk, dv, domega,
-                  workspace, stream=None, S_lo=None, z_lo=None):
-    """slim_bwd into caller-allocated gradients and workspace (no allocation)."""
+                  workspace, stream=None, S_lo=None, z_lo=None, G_S_in=None, g_z_in=None,
+                  G_S_out=None, g_z_out=None):
+    """slim_bwd (slim_bwd_from with state gradients in or out) into
+    caller-allocated gradients and workspace (no allocation)."""
     B, H, L, d, M = _dims(q, omega)
-    _check(library().slim_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega),
-                              out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
-                              z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo), B, H, L, d, M, C,
-                              DTYPES[q.dtype], FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
-                              dv.data_ptr(), _ptr(domega), workspace.data_ptr(),
-                              workspace.numel(), _stream_handle(stream)), "slim_bwd")
+    head = (q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega), out.data_ptr(),
+            dout.data_ptr(), S_state.data_ptr(), z_state.data_ptr(), _ptr(S_lo), _ptr(z_lo))
+    dims = (B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature])
+    grads = (dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), _ptr(domega))
+    tail = (workspace.data_ptr(), workspace.numel(), _stream_handle(stream))
+    if G_S_in is None and G_S_out is None:
+        _check(library().slim_bwd(*head, *dims, *grads, *tail), "slim_bwd")
+    else:
+        _check(library().slim_bwd_from(*head, _ptr(G_S_in), _ptr(g_z_in), *dims, *grads,
+                                       _ptr(G_S_out), _ptr(g_z_out), *tail), "slim_bwd_from")
+
+
+def forward_bidir_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None):
+    """slim_fwd_bidir into caller-allocated outputs and workspace."""
+    B, H, L, d, M = _dims(q, omega)
+    _check(library().slim_fwd_bidir(q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega),
+                                    B, H, L, d, M, C, DTYPES[q.dtype], FEATURES[feature],
+                                    out.data_ptr(), S_state.data_ptr(), z_state.data_ptr(),
+                                    workspace.data_ptr(), workspace.numel(),
+                                    _stream_handle(stream)), "slim_fwd_bidir")
+
+
+def backward_bidir_into(q, k, v, omega, out, dout, S_state, z_state, C, feature, dq, dk, dv,
+                        domega, workspace, stream=None):
+    """slim_bwd_bidir into caller-allocated gradients and workspace."""
+    B, H, L, d, M = _dims(q, omega)
+    _check(library().slim_bwd_bidir(q.data_ptr(), k.data_ptr(), v.data_ptr(), _ptr(omega),
+                                    out.data_ptr(), dout.data_ptr(), S_state.data_ptr(),
+                                    z_state.data_ptr(), B, H, L, d, M, C, DTYPES[q.dtype],
+                                    FEATURES[feature], dq.data_ptr(), dk.data_ptr(),
+                                    dv.data_ptr(), _ptr(domega), workspace.data_ptr(),
+                                    workspace.numel(), _stream_handle(stream)), "slim_bwd_bidir")
 
 
 def check_device_error(workspace, stream=None):

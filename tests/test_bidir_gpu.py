@@ -1,0 +1,73 @@
+"""Parity of the non-causal form (no mask, one global state) with the oracle,
+through the C ABI: every feature map, both dtypes, several slices with a ragged
+last one, and C-invariance."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2012_11346_gb300 import slim
+from paper_2012_11346_gb300 import workloads as W
+
+from gpu_common import TOL, compare, cpu_inputs, to64
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_bidir(x, C, feature):
+    om = None if feature == "square" else x["omega"]
+    out, S, z = slim.forward_bidir(x["q"], x["k"], x["v"], om, C, feature)
+    dq, dk, dv, dom = slim.backward_bidir(x["q"], x["k"], x["v"], om, out, x["dout"], S, z, C,
+                                          feature)
+    torch.cuda.synchronize()
+    r = {"out": out, "S_state": S, "z_state": z, "dq": dq, "dk": dk, "dv": dv}
+    if dom is not None:
+        r["domega"] = dom
+    return r
+
+
+def oracle_bidir(xc, C, feature):
+    out, S, z = oracle.oracle_bidir_fwd(xc["q"], xc["k"], xc["v"], xc["omega"], C, feature)
+    dq, dk, dv, dom = oracle.oracle_bidir_bwd(xc["q"], xc["k"], xc["v"], xc["omega"], xc["dout"],
+                                              S, z, C, feature)
+    return {"out": out, "S_state": S, "z_state": z, "dq": dq, "dk": dk, "dv": dv, "domega": dom}
+
+
+CASES = [
+    W.WORKLOADS["tiny_f32"],
+    W.WORKLOADS["L4096_bf16"].with_(B=2, H=2, L=1500, C=512),
+    W.WORKLOADS["L8192_relu_f32"].with_(B=2, H=2, L=700, C=256),
+    W.WORKLOADS["L4096_square_bf16"].with_(B=1, H=3, L=900, C=200),
+    W.Workload("bidir", 2, 1, 333, 128, 128, 100, "f32", "square", "normal", "iid", seed=6),
+    W.Workload("bidir", 1, 2, 1, 32, 48, 4, "f32", "exp", "normal", "iid", seed=7),
+]
+
+
+@pytest.mark.parametrize("w", CASES, ids=[f"{w.name}-{w.dtype}-{w.feature}-L{w.L}" for w in CASES])
+def test_bidir_parity(cuda_device, w):
+    x = W.make_inputs(w, device=cuda_device)
+    g = gpu_bidir(x, w.C, w.feature)
+    ref = oracle_bidir(cpu_inputs(x), w.C, w.feature)
+    compare(g, ref, TOL[w.dtype], names=tuple(g), where=f"bidir {w.name}", C=w.C,
+            scale=float(np.linalg.norm(cpu_inputs(x)["dout"].ravel())))
+
+
+def test_bidir_c_invariance_fp32(cuda_device):
+    w = W.WORKLOADS["L8192_relu_f32"].with_(B=1, H=2, L=1000)
+    x = W.make_inputs(w, device=cuda_device)
+    ref = gpu_bidir(x, 1000, w.feature)
+    for C in (1, 64, 333):
+        g = gpu_bidir(x, C, w.feature)
+        for n in ref:
+            assert oracle.rel_l2(to64(g[n]), to64(ref[n])) < 1e-5, (C, n)
+
+
+def test_bidir_last_row_matches_causal(cuda_device):
+    """The last row reads every key in both forms."""
+    w = W.WORKLOADS["L4096_bf16"].with_(B=1, H=2, L=777, C=256)
+    x = W.make_inputs(w, device=cuda_device)
+    ob, Sb, zb = slim.forward_bidir(x["q"], x["k"], x["v"], x["omega"], w.C, w.feature)
+    oc, Sc, zc = slim.forward(x["q"], x["k"], x["v"], x["omega"], w.C, w.feature)
+    torch.cuda.synchronize()
+    assert oracle.rel_l2(to64(ob[:, :, -1]), to64(oc[:, :, -1])) < TOL["bf16"]
+    assert oracle.rel_l2(to64(Sb), to64(Sc)) < TOL["bf16"]
