@@ -264,15 +264,15 @@ slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype d
  * inspecting and testing that order (no counterpart in the paper).  Ticket x
  * names item (role, slice, index), written to items[3x], items[3x+1],
  * items[3x+2] for x < min(*count, cap):
- *   role 0: dq side of tile index of the slice (tiles last first, chains
- *           inside a position: tile ntn-1-index/(B*H) of chain index%(B*H)),
- *   role 1: dk/dv side of the same tile numbering,
+ *   role 0: tile index of the slice, dq part then dk/dv part in one CTA
+ *           (tiles last first, chains inside a position: tile
+ *           ntn-1-index/(B*H) of chain index%(B*H)),
  *   role 2: final dOmega reduction, stage 1 CTA index (slice 0),
  *   role 3: final dOmega reduction, stage 2 CTA index (slice 0).
  * *count receives the number of items.  items may be null when cap is 0.
  * *ring (when ring is not null) receives R, the slots of the ring through
- * which the dq side of slice n hands its tiles to the dk/dv side (slot n % R;
- * the dq side of slice n-R waits until slice n's dk/dv side has read it).
+ * which a tile's dq part hands its results to its dk/dv part (slot n % R;
+ * slice n-R's tile at the same position waits until slice n's has read it).
  * Returns SLIM_ERR_UNSUPPORTED for problems the tensor-core path does not
  * take (see slim_path_for) and for L = 0.
  */

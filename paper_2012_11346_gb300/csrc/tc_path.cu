@@ -16,17 +16,18 @@
 //   forward, one launch, tiles in sequence order:
 //     phiQ, phiK, Delta_t, A = tril(phiQ phiK^T);  S_t, z_t = prefix before
 //     tile t;  num = phiQ S_t + A V_t,  den = phiQ z_t + rowsum A,  out = num/den
-//   backward, one launch, slices in reverse (Algorithm 1's reverse sweep):
-//     dq side of slice n, tiles in reverse order: phiQ, phiK, Delta_t, A;
+//   backward, one launch, slices in reverse (Algorithm 1's reverse sweep); one
+//   CTA per tile runs the tile's dq part and then its dk/dv part:
+//     dq part, tiles in reverse order: phiQ, phiK, Delta_t, A;
 //       rollback P_t = P_{t+1} - Delta_t (eq. 17);  den, dnum = dout/den,
 //       dden = -<dout,out>/den, dA = tril(dnum V^T + dden);
 //       dphiQ = dnum S_t^T + dden z_t + dA phiK,  Gd_t = phiQ^T [dnum | dden];
 //       state-gradient chain G_t = G_{t+1} + Gd_{t+1} (eq. 18);
 //       dq = u Omega - q sum(u),  dOmega partial u^T q
-//     dk/dv side of slice n (beside the dq side of slice n-1):
+//     dk/dv part of the same tile (phiQ still in shared memory):
 //       dV = A^T dnum + phiK G_t(S),  dphiK = dA^T phiQ + V G_t(S)^T + g_t(z),
-//       dk = u Omega - k sum(u),  dOmega partial u^T k
-//     each side adds its dOmega partials to one running sum per tile position
+//       dk = u Omega - k sum(u),  dOmega partial u^T k (+ the dq part's u^T q)
+//     the tile's dOmega partial goes onto one running sum per tile position
 //     (slices in order N-1 .. 0), and the sums are reduced once, in a fixed
 //     order, at the end of the launch
 #include <math.h>
@@ -207,6 +208,14 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   __syncthreads();                                      \
   if (warp == 0) tmem_dealloc(tmem_base, 512)
 
+// The same, for a role that runs on TMEM its caller allocated and frees.
+#define TC_TEARDOWN_KEEP()                              \
+  teardown:                                             \
+  cp_async_wait_all();                                  \
+  bulk_wait_read();                                     \
+  tc_fence_before();                                    \
+  __syncthreads()
+
 // ------------------------------------------------------------------ chained tile prefixes
 // A slot holds one state (or state-gradient) prefix, [S (M x 64) | z (M)] in
 // fp32; its flag holds n + 1 once slice n's prefix is in the slot.  The CTA
@@ -225,6 +234,17 @@ __device__ __forceinline__ void st_release_gpu(int* p, int v) {
 }
 __device__ __forceinline__ void red_release_gpu(int* p, int v) {
   asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Drops the L2 lines of a buffer that nobody reads again before it is next
+// written (discard.global.L2: the lines become undefined and are not written
+// back to DRAM).  A discard is a weak write, so it is ordered before a later
+// release like the thread's other writes.  p and bytes are multiples of 128;
+// `nthr` threads share the lines.
+__device__ __forceinline__ void discard_l2(const void* p, size_t bytes, int i, int nthr) {
+  const char* b = static_cast<const char*>(p);
+  for (size_t off = (size_t)i * 128; off < bytes; off += (size_t)nthr * 128)
+    asm volatile("discard.global.L2 [%0], 128;" ::"l"(b + off) : "memory");
 }
 
 // Flags sit 128 bytes apart, so the CTAs polling different flags do not
@@ -692,34 +712,32 @@ struct BwdQJob {
   int L, a, b, ntn, n, N, nt, chains;  // slice n = rows [a, a+b), ntn tiles; nt: full slice
   float *slot1, *slot2;   // [chains][nt][E]: state prefixes, state-gradient prefixes
   int *flag1, *flag2;     // [chains][nt], FLAG_STRIDE ints apart
-  // Hand-off to the dk/dv side of the same slice, through the buffers of ring
-  // slot n % R indexed by (chain, tile) of a full slice:
+  // Hand-off to the tile's dk/dv part, through the buffers of ring slot
+  // n % R indexed by (chain, tile) of a full slice (written by this CTA and read
+  // back by it, so they stay in L2; the dk/dv part discards them):
   __nv_bfloat16* gS;      // [chains][nt][MF][64] G_t(S)
   float* gz;              // [chains][nt][MF]     g_t(z)
   float* rowstat;         // [chains][nt][T][2]   (den, dden)
-  uint8_t* img;           // [chains][nt][2 FEATB + 32 KB]: phiQ and phiK as shared-
-                          //   memory tile images (bf16, 128-byte swizzle), then tril(A)
-                          //   in bf16, lane-major (chunk of 8 columns c/8, row r at
-                          //   16-byte unit (c/8) 128 + r)
-  int* gflag;             // [chains][nt]: n + 1 once the four above are written
-  const int* kvread;      // [chains][nt]: n + R + 1 once slice n+R's dk/dv side has read them
+  float* domq;            // [chains][nt][MF][64] lane-major: the dOmega partial u^T q
+  uint8_t* img;           // [chains][nt][FEATB + 32 KB]: phiK as its shared-memory tile
+                          //   image (bf16, 128-byte swizzle), then tril(A) in bf16,
+                          //   lane-major (chunk of 8 columns c/8, row r at 16-byte
+                          //   unit (c/8) 128 + r)
+  int* gflag;             // [chains][nt]: n + 1 once the five above are written
+  const int* kvread;      // [chains][nt]: n + R + 1 once slice n+R's dk/dv part has read them
   int ring;               // R, slots of the hand-off ring
   int nRtiles;            // tiles of slice n+R per chain (0: no such slice)
-  // dOmega: this side's per-position sums over slices N-1 .. n
-  float* acc;             // [chains][nt][MF][64] lane-major
-  int* accflag;           // [chains][nt]: n + 1 once slice n has added its partial
-  int n1tiles;            // tiles of slice n+1 per chain (0: no such slice)
-  int* sums_done;         // slice 0 only: counter of final sums written
   __nv_bfloat16* dq;
   int* err;
   GradIO gio;             // G^(N) in (null: zero), G^(0) out (null: not returned)
 };
 
-// The dq side splits its warps twice, as the forward does: after the g(K)
+// The dq part splits its warps twice, as the forward does: after the g(K)
 // epilogue, warps 0-7 compute g(Q), A and dout V^T while warps 8-15 run the
 // rollback chain (which needs only Delta_t); after dphiQ, warps 0-7 compute u
-// and issue dq while warps 8-15 run the state-gradient chain.
-template <int MF, int FEAT, bool EARLY>
+// and issue dq while warps 8-15 run the state-gradient chain.  The TMEM
+// columns (all 512) are allocated by the caller for both parts of the tile.
+template <int MF, int FEAT>
 __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* smem_raw,
                                            uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
@@ -748,9 +766,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   const int row0 = J.a + t * T;
   const int valid = min(T, J.b - t * T);
   const size_t g0 = ((size_t)c * J.L + row0) * D;
-  const size_t tf = (size_t)c * J.nt + t;   // hand-off buffers, flags, dOmega sums
-  // the first slice (from the end) with a tile at this position starts its sum
-  const bool acc_first = t >= J.n1tiles;
+  const size_t tf = (size_t)c * J.nt + t;   // hand-off buffers, flags
   // The prefixes after this tile: the next tile's slots, the first tile of
   // slice n+1, or (at the end of the sequence) B^(N) and G = 0.
   const bool inner = t + 1 < J.ntn, next_slice = n + 1 < J.N;
@@ -796,15 +812,12 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     for (int i = 0; i < NBAR; ++i) mbar_init(smem_u32(&mb[i]), 1);
     mbar_fence_init();
   }
-  if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
   if (tid == POLL) {
     // while the tiles stream in: the hand-off buffers of ring slot n % R are
-    // free once slice n+R's dk/dv side has read them (tril(A) is written in
+    // free once slice n+R's dk/dv part has read them (tril(A) is written in
     // the A row-sum loop, the rest after join1)
     const bool ok = flag_poll2(t < J.nRtiles ? J.kvread + tf * FLAG_STRIDE : nullptr,
-                               n + J.ring + 1,
-                               EARLY && !acc_first ? J.accflag + tf * FLAG_STRIDE : nullptr,
-                               n + 2, J.err);
+                               n + J.ring + 1, nullptr, 0, J.err);
     gfail[1] = ok ? 0 : 1;
   } else if (tid < LDT) {
     load_rows64(sQ, T, J.Q + g0, valid, tid, LDT);
@@ -876,8 +889,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     fill_ones(sOnes, tid);  // the K tile is no longer read
     feature_epilogue<MF, FEAT>(trow + 256, sPhiK, row, cg, k2, rv);
     publish();
-    // the dk/dv side of this tile takes phiK, phiQ and tril(A) from here
-    uint8_t* img = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT);
+    // the dk/dv part of this tile takes phiK and tril(A) from here (phiQ stays
+    // in shared memory)
+    uint8_t* img = J.img + tf * ((size_t)C::FEATB + 2 * ROWT);
     if (tid == 0 || (C::MH > 1 && tid == 32)) {
       // Delta_t = phiK^T [V | 1], one feature half per issuing thread
       const int h = tid == 0 ? 0 : 1;
@@ -911,7 +925,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       group_bar(1);
       if (gfail[0]) goto join1;
       float rs = 0.f;  // the rounded masked A values of this thread's columns
-      uint8_t* imgA = img + 2 * C::FEATB;
+      uint8_t* imgA = img + C::FEATB;
 #pragma unroll 1
       for (int c0 = 32 * cg; c0 < T; c0 += 64) {
         float v[32];
@@ -994,18 +1008,19 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           sZ[m] = z;
         }
       }
+      // the prefix after this tile is read only here: drop it from L2 (before
+      // the release, so that it comes before the slot's next writer), unless it
+      // sits in this tile's own slot (one-tile slices), just rewritten
+      if (linked && snext != t) discard_l2(s1.S, (size_t)C::E * 4, gl, GRP);
       group_bar(2);  // every slot write of the group is issued
       if (gl == 0) st_release_gpu(of1, n + 1);
     }
   join1:
     __syncthreads();
     if (gfail[0] | gfail[1]) goto teardown;
-    // the two feature tiles' images, while the MMAs of the next phases run
-    // (phiK's tile is overwritten by u once they have landed)
-    if (tid == GRP) {
-      bulk_store(img, smem_u32(sPhiQ), C::FEATB);
-      bulk_store(img + C::FEATB, smem_u32(sPhiK), C::FEATB);
-    }
+    // phiK's tile image, while the MMAs of the next phases run (the tile is
+    // overwritten by u once the copy has read it)
+    if (tid == GRP) bulk_store(img, smem_u32(sPhiK), C::FEATB);
     {
       // g(Q) . z_t over this thread's feature columns
       constexpr int W = MF / NG;
@@ -1193,18 +1208,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           if (seq_first) J.gio.z_out[(size_t)c * MF + m] = gzs[h] + gdz;
         }
       }
+      if (linked && snext != t) discard_l2(s2.S, (size_t)C::E * 4, gl, GRP);
       group_bar(2);  // every slot write of the group is issued
-      if (gl == 0) {
-        st_release_gpu(of2, n + 1);
-        if (!EARLY) {
-          // the hand-off to the dk/dv side: G_t, g_t(z), rowstat, tril(A) and,
-          // once its bulk copies are done, the feature tiles
-          bulk_wait_done();
-          st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);
-          // slice n+1's dOmega sum at this position (added to after join2)
-          if (!acc_first && !flag_poll(J.accflag + tf * FLAG_STRIDE, n + 2, J.err)) gfail[1] = 1;
-        }
-      }
+      if (gl == 0) st_release_gpu(of2, n + 1);
     }
   join2:
     __syncthreads();
@@ -1217,25 +1223,18 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       tc_fence_after();
       __syncthreads();
       if (abort_ | gfail[1]) goto teardown;
-      // the partial goes onto the running dOmega sum at this position (or
-      // starts it): one add per slice, in slice order
-      float* accp = J.acc + tf * (size_t)(MF * 64);
+      // the partial joins the key side's in the dk/dv part (through L2)
+      float* dqp = J.domq + tf * (size_t)(MF * 64);
       float v[16];
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         tmem_ld16(trow + 320 + 64 * h + 16 * cg, v);
-        if (acc_first)
-          st_lm16(accp, h, cg, row, v);
-        else
-          red_lm16(accp, h, cg, row, v);
+        st_lm16(dqp, h, cg, row, v);
       }
       __syncthreads();
-      if (tid == 0) {  // warp 0 waits for the release while the others store dq
-        st_release_gpu(J.accflag + tf * FLAG_STRIDE, n + 1);
-        if (J.sums_done) red_release_gpu(J.sums_done, 1);
-      } else if (tid == GRP && EARLY) {
-        // long stages: the hand-off (its dk/dv side is a stage away), off the
-        // G chain's path
+      if (tid == GRP) {
+        // the hand-off to the dk/dv part: G_t, g_t(z), rowstat, tril(A), the
+        // dOmega partial and, once its bulk copy is done, phiK's image
         bulk_wait_done();
         st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);
       }
@@ -1247,27 +1246,32 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       if (rv) st_row16(J.dq + g0 + (size_t)row * D + 16 * cg, v);
     }
   }
-  TC_TEARDOWN();
+  TC_TEARDOWN_KEEP();
 }
 
 // ================================================================== backward, dk/dv side
 struct BwdKVJob {
   const __nv_bfloat16 *Q, *K, *V, *dOut, *om16;
-  // from the dq side of the same slice, indexed by (chain, tile) of a full slice
+  // from the dq part of the same tile, indexed by (chain, tile) of a full slice
   const __nv_bfloat16* gS;   // [chains][ntf][MF][64] G_t(S)
   const float *gz, *rowstat;
-  const uint8_t* img;        // [chains][ntf][...] phiQ, phiK tile images, tril(A) lane-major
+  const float* domq;         // [chains][ntf][MF][64] lane-major: the dq part's u^T q
+  const uint8_t* img;        // [chains][ntf][...] phiK's tile image, tril(A) lane-major
   const int* gflag;          // n + 1 once they are written
-  int* kvread;               // set to n + 1 once this side has read them
+  int* kvread;               // set to n + 1 once this part has read them
   int L, a, b, ntn, ntf, n;  // slice n = rows [a, a+b), ntn tiles; ntf: full slice
   __nv_bfloat16 *dk, *dv;
-  float* acc;                // as for the dq side: this side's dOmega sums
-  int* accflag;
-  int n1tiles;
-  int* sums_done;
+  // dOmega: per-position sums over slices N-1 .. n of the tiles' partials
+  float* acc;                // [chains][ntf][MF][64] lane-major
+  int* accflag;              // [chains][ntf]: n + 1 once slice n has added its partial
+  int n1tiles;               // tiles of slice n+1 per chain (0: no such slice)
+  int* sums_done;            // slice 0 only: counter of final sums written
   int* err;
 };
 
+// The dk/dv part of a tile, run by the CTA that ran its dq part: phiQ is still
+// in shared memory, and the rest of the hand-off was written by this CTA and
+// is read back from L2.  The TMEM columns are the caller's.
 template <int MF, int FEAT, bool EARLY>
 __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uint8_t* smem_raw,
                                             uint64_t* mb, uint32_t& tmem_base, int& abort_) {
@@ -1292,24 +1296,30 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   const bool acc_first = t >= J.n1tiles;
   float den = 0.f, dden = 0.f;
   __shared__ int poll_ok;              // written by the polling thread only
-  __shared__ __align__(8) uint64_t mb_img;  // the two feature tiles, initialised by that thread
-  TC_PROLOGUE();
+  __shared__ __align__(8) uint64_t mb_img;  // phiK's tile, initialised by that thread
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int row = 32 * (warp & 3) + (tid & 31);
+  const int cg = warp >> 2;
+  if (tid == 0) {
+    abort_ = 0;
+    for (int i_ = 0; i_ < NBAR; ++i_) mbar_init(smem_u32(&mb[i_]), 1);
+    mbar_fence_init();
+  }
+  uint8_t* const img = const_cast<uint8_t*>(J.img) + tf * ((size_t)C::FEATB + 2 * ROWT);
   if (tid == POLL) {
-    // while V and dout stream in: phiQ, phiK, tril(A), G_t, g_t(z) and the
-    // row statistics come from the dq side of this tile; then the two feature
-    // tiles, by bulk copies completing on mb_img
+    // while V and dout stream in: phiK, tril(A), G_t, g_t(z), the row
+    // statistics and the dOmega partial come from the dq part of this tile;
+    // phiK's tile by a bulk copy completing on mb_img
     poll_ok = flag_poll2(J.gflag + tf * FLAG_STRIDE, J.n + 1,
                          EARLY && !acc_first ? J.accflag + tf * FLAG_STRIDE : nullptr, J.n + 2,
                          J.err);
     if (poll_ok) {
-      const uint8_t* img = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT);
       const uint32_t bar = smem_u32(&mb_img);
       mbar_init(bar, 1);
       mbar_fence_init();
       fence_proxy_async_global();
-      mbar_expect_tx(bar, 2 * C::FEATB);
-      bulk_load(smem_u32(sPhiQ), img, C::FEATB, bar);
-      bulk_load(smem_u32(sPhiK), img + C::FEATB, C::FEATB, bar);
+      mbar_expect_tx(bar, C::FEATB);
+      bulk_load(smem_u32(sPhiK), img, C::FEATB, bar);
     }
   } else if (tid < LDT) {
     load_rows64(sV, T, J.V + g0, valid, tid, LDT);
@@ -1328,7 +1338,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);  // G_t(S), awaited before the dV products
   {
     // tril(A) into its tile (lane-major in global memory: coalesced reads)
-    const uint8_t* imgA = J.img + tf * (2 * (size_t)C::FEATB + 2 * ROWT) + 2 * C::FEATB;
+    const uint8_t* imgA = img + C::FEATB;
     for (int k = tid; k < T * T / 8; k += NTHR)
       cp_async16(smem_u32(sA) + tile_off(T, k % T, 8 * (k / T)), imgA + (size_t)k * 16, 16u);
   }
@@ -1353,11 +1363,16 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       }
       st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
     }
-    if (!mbar_wait(smem_u32(&mb_img), 0, J.err)) abort_ = 1;  // the two feature tiles
+    if (!mbar_wait(smem_u32(&mb_img), 0, J.err)) abort_ = 1;  // phiK's tile
     cp_async_wait_all();  // G_t(S), tril(A)
     publish();
     if (abort_) goto teardown;
-    if (tid == POLL) st_release_gpu(J.kvread + tf * FLAG_STRIDE, J.n + 1);  // hand-off buffers read
+    // every thread has what it needs of the hand-off but the dOmega partial
+    // (read at the end): drop it from L2, it is not read again
+    discard_l2(img, (size_t)C::FEATB + 2 * ROWT, tid, NTHR);
+    discard_l2(J.gS + tf * MF * 64, (size_t)MF * 64 * 2, tid, NTHR);
+    discard_l2(J.gz + tf * MF, (size_t)MF * 4, tid, NTHR);
+    discard_l2(J.rowstat + tf * T * 2, (size_t)T * 2 * 4, tid, NTHR);
     if (tid == 0) {
       const uint32_t aDn = smem_u32(sDn), aV = smem_u32(sV);
       for (int k0 = 0; k0 < D; k0 += 16)  // dnum V^T
@@ -1477,22 +1492,30 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     TC_WAIT(sy);
     TC_WAIT(sy);
     {
-      // the partial goes onto the running dOmega sum at this position (or
-      // starts it): one add per slice, in slice order
+      // the tile's partial (key side + the dq part's query side) goes onto the
+      // running dOmega sum at this position (or starts it): one add per
+      // slice, in slice order
       float* accp = J.acc + tf * (size_t)(MF * 64);
-      float v[16];
+      const float* dqp = J.domq + tf * (size_t)(MF * 64);
+      float v[16], w[16];
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
+        ld_lm16(dqp, h, cg, row, w);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] += w[i];
         if (acc_first)
           st_lm16(accp, h, cg, row, v);
         else
           red_lm16(accp, h, cg, row, v);
       }
       __syncthreads();
-      if (tid == 0) {  // warp 0 waits for the release while the others store dk
+      discard_l2(dqp, (size_t)MF * 64 * 4, tid, NTHR);
+      __syncthreads();  // every discard of the hand-off comes before the release
+      if (tid == 0) {  // warp 0 waits for the releases while the others store dk
         st_release_gpu(J.accflag + tf * FLAG_STRIDE, J.n + 1);
         if (J.sums_done) red_release_gpu(J.sums_done, 1);
+        st_release_gpu(J.kvread + tf * FLAG_STRIDE, J.n + 1);  // hand-off buffers read
       }
       float xk[16];
       ld_feat16(sKr, row, 16 * cg, xk);
@@ -1502,7 +1525,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       if (rv) st_row16(J.dk + g0 + (size_t)row * D + 16 * cg, v);
     }
   }
-  TC_TEARDOWN();
+  TC_TEARDOWN_KEEP();
 }
 
 // ================================================================== launches
@@ -1653,31 +1676,25 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_fwd(const __grid_constant__ FwdJ
 }
 
 // ------------------------------------------------------------------ backward launch
-// The backward is one launch too.  Its items (tiles of either side, dOmega
-// reduction CTAs) are handed out by the same kind of counter, in stage order:
-// stage j = 0 .. N holds the dq-side tiles of slice N-1-j and the dk/dv-side
-// tiles of slice N-j (those that exist), and the final dOmega reduction
-// (stage 1, then stage 2) comes last.  Every wait of an item is on items of
-// earlier stages or on earlier tiles of its own chain, which hold lower
-// tickets:
-//   dq side of slice n    <- its chain (slice n's later tiles, slice n+1's first),
-//                            slice n+R's dk/dv side (hand-off buffers of ring
-//                            slot n % R, R >= 2), slice n+1's dq side at its
+// The backward is one launch too.  Its items (one per tile, running the
+// tile's dq part and then its dk/dv part, and the final dOmega reduction
+// CTAs) are handed out by the same kind of counter, in stage order: stage j =
+// 0 .. N-1 holds the tiles of slice N-1-j, last tile first, chains inside a
+// tile position, and the final dOmega reduction (stage 1, then stage 2) comes
+// last.  Every wait of an item is on items of earlier stages or on earlier
+// tiles of its own chain, which hold lower tickets:
+//   tile of slice n       <- its chain (slice n's later tiles, slice n+1's first),
+//                            slice n+R's tile at its position (hand-off buffers
+//                            of ring slot n % R, R >= 2), slice n+1's tile at its
 //                            position (dOmega sum)
-//   dk/dv side of slice n <- the dq side of the same tile; slice n+1's dk/dv side
-//                            at its position (dOmega sum)
 //   reduction stage 1     <- every tile of slice 0 (the last to add to a sum)
 //   reduction stage 2     <- stage 1
 // so the lowest unfinished item never waits and the launch always progresses.
-// Both sides take a slice's tiles in the same order (last tile first, chains
-// inside a tile position), and the two sides of a stage alternate by rows of
-// `chains` tiles: the dq-side tiles of one chain are further apart than in
-// one block per side, and a dk/dv tile comes a full stage after its dq tile.
 struct BwdSched {
   int N, chains, nt, ntl;  // slices, chains, tiles of a full slice and of the last
   int r1n, r2n;            // final dOmega stage-1 and stage-2 CTAs
 };
-enum { IT_Q = 0, IT_KV = 1, IT_R1 = 2, IT_R2 = 3 };
+enum { IT_TILE = 0, IT_R1 = 2, IT_R2 = 3 };
 struct BwdItem {
   int kind, n, idx;  // role, slice, index among the role's items of the slice
 };
@@ -1685,59 +1702,23 @@ struct BwdItem {
 __host__ __device__ inline int sched_tiles(const BwdSched& s, int n) {
   return s.chains * (n == s.N - 1 ? s.ntl : s.nt);
 }
-__host__ __device__ inline void sched_stage(const BwdSched& s, int j, int& q, int& kv) {
-  const int nq = s.N - 1 - j, nkv = s.N - j;
-  q = (nq >= 0 && nq < s.N) ? sched_tiles(s, nq) : 0;
-  kv = (nkv >= 0 && nkv < s.N) ? sched_tiles(s, nkv) : 0;
-}
 __host__ __device__ inline long long sched_items(const BwdSched& s) {
   long long n = s.r1n + s.r2n;
-  for (int k = 0; k < s.N; ++k) n += 2LL * sched_tiles(s, k);
+  for (int k = 0; k < s.N; ++k) n += sched_tiles(s, k);
   return n;
 }
-// Item of ticket x.  Stages 2 .. N-1 all have the same size and are skipped
-// arithmetically.
+// Item of ticket x: stage 0 is the last slice (possibly shorter), stages 1 ..
+// N-1 all have chains * nt items.
 __host__ __device__ inline BwdItem sched_locate(const BwdSched& s, int x) {
-  int j = 0;
-  for (;;) {
-    if (j == 2 && s.N >= 3) {
-      const int cnt = s.N - 2, sz = 2 * s.chains * s.nt;
-      const int k = x / sz;
-      if (k < cnt) {
-        j = 2 + k;
-        x -= k * sz;
-        break;
-      }
-      x -= cnt * sz;
-      j = s.N;
-    }
-    if (j > s.N) break;
-    int q, kv;
-    sched_stage(s, j, q, kv);
-    if (x < q + kv) break;
-    x -= q + kv;
-    ++j;
-  }
-  if (j > s.N) {  // the final reduction
-    if (x < s.r1n) return BwdItem{IT_R1, 0, x};
-    return BwdItem{IT_R2, 0, x - s.r1n};
-  }
-  int q, kv;
-  sched_stage(s, j, q, kv);
-  bool isq = x < q;
-  int idx = isq ? x : x - q;
-  if (q > 0 && kv > 0) {
-    const int ch = s.chains, m = (q < kv ? q : kv) / ch;  // row pairs
-    if (x < 2 * m * ch) {
-      const int p = x / (2 * ch), w = x % (2 * ch);
-      isq = w < ch;
-      idx = p * ch + (isq ? w : w - ch);
-    } else {
-      isq = q > kv;
-      idx = m * ch + (x - 2 * m * ch);
-    }
-  }
-  return isq ? BwdItem{IT_Q, s.N - 1 - j, idx} : BwdItem{IT_KV, s.N - j, idx};
+  const int first = sched_tiles(s, s.N - 1);
+  if (x < first) return BwdItem{IT_TILE, s.N - 1, x};
+  x -= first;
+  const int full = s.chains * s.nt;
+  const int k = x / full;
+  if (k < s.N - 1) return BwdItem{IT_TILE, s.N - 2 - k, x - k * full};
+  x -= (s.N - 1) * full;
+  if (x < s.r1n) return BwdItem{IT_R1, 0, x};
+  return BwdItem{IT_R2, 0, x - s.r1n};
 }
 
 struct BwdJob {
@@ -1748,28 +1729,27 @@ struct BwdJob {
   int L, Cs;
   int* ticket;
   // hand-off ring: slot k (slice n uses n % ring) holds, at hand + k hand_slot,
-  // G_t(S) bf16 [chains][nt][M][64], then g_t(z), the row statistics and the
-  // tile images at the given offsets; its two flag arrays (gflag, kvread) are
-  // hflag + (2k, 2k+1) * chains * nt * FLAG_STRIDE
+  // G_t(S) bf16 [chains][nt][M][64], then g_t(z), the row statistics, the dq
+  // part's dOmega partials and the tile images at the given offsets; its two
+  // flag arrays (gflag, kvread) are hflag + (2k, 2k+1) * chains * nt * FLAG_STRIDE
   uint8_t* hand;
-  size_t hand_slot, off_gz, off_rs, off_img;
+  size_t hand_slot, off_gz, off_rs, off_dq, off_img;
   int ring;
   int* hflag;
-  float* acc;       // [2 sides][chains][nt][M*64] per-position dOmega sums
-  int* accflag[2];  // [chains][nt] per side
+  float* acc;       // [chains][nt][M*64] per-position dOmega sums
+  int* accflag;     // [chains][nt]
   int *sums_done, *r1done;  // slice-0 tiles done, final stage-1 CTAs done
 };
 
-// EARLY (stages of at least EARLY_STAGE items): the flags a tile waits on were
-// set long before it starts, so it polls them up front, and the dq side
-// releases the hand-off once it is done, off the G chain's path.  With shorter
-// stages, tiles of neighbouring slices run at the same time: the running-sum
-// flags are then polled just before the adds and the hand-off is released in
-// the G chain, so that no tile waits for another one to finish.
+// EARLY (stages of at least EARLY_STAGE items): the dOmega-sum flag a tile
+// waits on was set long before it starts, so the dk/dv part polls it up
+// front.  With shorter stages, tiles of neighbouring slices run at the same
+// time, and it is polled just before the adds, so that no tile waits for
+// another one to finish.
 template <int MF, int FEAT, bool EARLY>
 __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJob J) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t mbar[NBAR];
+  __shared__ __align__(8) uint64_t mbar[2 * NBAR];  // the dq part's, then the dk/dv part's
   __shared__ uint32_t tmem_base;
   __shared__ int abort_;
   __shared__ int ticket;
@@ -1777,56 +1757,62 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
   __syncthreads();
   const BwdItem it = sched_locate(J.s, ticket);
   const int n = it.n, N = J.s.N;
-  if (it.kind <= IT_KV) {
+  if (it.kind == IT_TILE) {
     const int a = n * J.Cs, b = min(J.Cs, J.L - a), ntn = (b + T - 1) / T;
     const int n1 = n + 1 < N ? (n + 1 == N - 1 ? J.s.ntl : J.s.nt) : 0;
-    const size_t side = (size_t)J.s.chains * J.s.nt * MF * D;
     const size_t tiles = (size_t)J.s.chains * J.s.nt;
     const int slot = n % J.ring;
     uint8_t* hs = J.hand + slot * J.hand_slot;
     int* hf = J.hflag + (size_t)(2 * slot) * tiles * FLAG_STRIDE;
-    if (it.kind == IT_Q) {
-      BwdQJob q = J.q;
-      q.a = a;
-      q.b = b;
-      q.ntn = ntn;
-      q.n = n;
-      q.gS = reinterpret_cast<__nv_bfloat16*>(hs);
-      q.gz = reinterpret_cast<float*>(hs + J.off_gz);
-      q.rowstat = reinterpret_cast<float*>(hs + J.off_rs);
-      q.img = hs + J.off_img;
-      q.gflag = hf;
-      q.kvread = hf + tiles * FLAG_STRIDE;
-      q.ring = J.ring;
-      q.nRtiles = n + J.ring < N ? (n + J.ring == N - 1 ? J.s.ntl : J.s.nt) : 0;
-      q.acc = J.acc;
-      q.accflag = J.accflag[0];
-      q.n1tiles = n1;
-      q.sums_done = n == 0 ? J.sums_done : nullptr;
-      role_bwd_q<MF, FEAT, EARLY>(q, it.idx, smem_raw, mbar, tmem_base, abort_);
-    } else {
-      BwdKVJob kv = J.kv;
-      kv.a = a;
-      kv.b = b;
-      kv.ntn = ntn;
-      kv.n = n;
-      kv.gS = reinterpret_cast<const __nv_bfloat16*>(hs);
-      kv.gz = reinterpret_cast<const float*>(hs + J.off_gz);
-      kv.rowstat = reinterpret_cast<const float*>(hs + J.off_rs);
-      kv.img = hs + J.off_img;
-      kv.gflag = hf;
-      kv.kvread = hf + tiles * FLAG_STRIDE;
-      kv.acc = J.acc + side;
-      kv.accflag = J.accflag[1];
-      kv.n1tiles = n1;
-      kv.sums_done = n == 0 ? J.sums_done : nullptr;
-      // the dq side's order: last tile first, chains inside a position
-      role_bwd_kv<MF, FEAT, EARLY>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains, smem_raw, mbar,
-                            tmem_base, abort_);
+    BwdQJob q = J.q;
+    q.a = a;
+    q.b = b;
+    q.ntn = ntn;
+    q.n = n;
+    q.gS = reinterpret_cast<__nv_bfloat16*>(hs);
+    q.gz = reinterpret_cast<float*>(hs + J.off_gz);
+    q.rowstat = reinterpret_cast<float*>(hs + J.off_rs);
+    q.domq = reinterpret_cast<float*>(hs + J.off_dq);
+    q.img = hs + J.off_img;
+    q.gflag = hf;
+    q.kvread = hf + tiles * FLAG_STRIDE;
+    q.ring = J.ring;
+    q.nRtiles = n + J.ring < N ? (n + J.ring == N - 1 ? J.s.ntl : J.s.nt) : 0;
+    BwdKVJob kv = J.kv;
+    kv.a = a;
+    kv.b = b;
+    kv.ntn = ntn;
+    kv.n = n;
+    kv.gS = q.gS;
+    kv.gz = q.gz;
+    kv.rowstat = q.rowstat;
+    kv.domq = q.domq;
+    kv.img = q.img;
+    kv.gflag = hf;
+    kv.kvread = hf + tiles * FLAG_STRIDE;
+    kv.acc = J.acc;
+    kv.accflag = J.accflag;
+    kv.n1tiles = n1;
+    kv.sums_done = n == 0 ? J.sums_done : nullptr;
+    // one TMEM allocation (all 512 columns) serves both parts of the tile
+    if (threadIdx.x < 32) tmem_alloc(smem_u32(&tmem_base), 512);
+    role_bwd_q<MF, FEAT>(q, it.idx, smem_raw, mbar, tmem_base, abort_);
+    __syncthreads();
+    // a wait of the dq part that gave up (or saw another CTA's failure) has set
+    // the error word: the dk/dv part would only wait on what never comes
+    const bool failed = *reinterpret_cast<volatile int*>(J.q.err) != 0;
+    if (!failed) {
+      tc_fence_after();
+      // the dq part's order: last tile first, chains inside a position
+      role_bwd_kv<MF, FEAT, EARLY>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains,
+                                   smem_raw, mbar + NBAR, tmem_base, abort_);
     }
+    tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x < 32) tmem_dealloc(tmem_base, 512);
     return;
   }
-  // final dOmega reduction over every position of both sides
+  // final dOmega reduction over every position
   if (threadIdx.x == 0) {
     abort_ = 0;
     const int want = it.kind == IT_R1 ? J.red.nparts : J.s.r1n;
@@ -1879,18 +1865,17 @@ Geo geometry(const Problem& p) {
 
 // The chain slots hold one prefix per (chain, tile of a slice): a slice's
 // tiles overwrite the previous slice's only after reading them.  The buffers
-// the dq side hands to the dk/dv side form a ring of R slots (slice n uses
-// n % R): the dq side of slice n-R reuses a slot once slice n's dk/dv side has
-// read it.  R is at least 2 (the dq side of slice n-1 runs beside the dk/dv
-// side of slice n) and large enough that those two items are KV_LEAD tickets
+// a tile's dq part hands to its dk/dv part form a ring of R slots (slice n
+// uses n % R): slice n-R's tile reuses a slot once slice n's tile has read it.
+// R is at least 2 and large enough that those two items are KV_LEAD tickets
 // apart, so that the wait is almost never taken even when slices are short.
-// dOmega is summed per (side, chain, tile position) over the slices and
-// reduced once at the end.
+// dOmega is summed per (chain, tile position) over the slices and reduced
+// once at the end.
 constexpr int KV_LEAD = 320;  // about two waves of tile CTAs
 constexpr int MAX_RING = 16;
 constexpr int EARLY_STAGE = 128;  // see k_tc_bwd
 int handoff_ring(const Geo& g) {
-  const int stage = 2 * g.chains * g.nt;  // items of a full stage
+  const int stage = g.chains * g.nt;  // items of a full stage
   const int r = 1 + (KV_LEAD + stage - 1) / stage;
   return r < 2 ? 2 : (r > MAX_RING ? MAX_RING : r);
 }
@@ -1900,17 +1885,18 @@ struct Ws {
   int nflags;
   int *flag1, *flag2;         // [chains][nt] chain flags, FLAG_STRIDE ints each
   int* hflag;                 // [ring][2][chains][nt] hand-off flags (backward)
-  int* accflag[2];            // [chains][nt] per side: dOmega sums (backward)
+  int* accflag;               // [chains][nt]: dOmega sums (backward)
   int *sums_done, *r1done;    // final reduction counters (backward)
   int* ticket;
   __nv_bfloat16* om16;
   float *slot1, *slot2;
-  // hand-off ring (see BwdJob): per slot G_t(S), g_t(z), the row statistics
-  // and per tile phiQ, phiK (T x M bf16 each) and tril(A) (T x T bf16)
+  // hand-off ring (see BwdJob): per slot G_t(S), g_t(z), the row statistics,
+  // the dq parts' dOmega partials and per tile phiK (T x M bf16) and tril(A)
+  // (T x T bf16)
   uint8_t* hand;
-  size_t hand_slot, off_gz, off_rs, off_img;
+  size_t hand_slot, off_gz, off_rs, off_dq, off_img;
   int ring;
-  float* acc;    // [2 sides][chains][nt][M*64]
+  float* acc;    // [chains][nt][M*64]
   float* rsums;  // [RS1][M*64]
 };
 
@@ -1919,7 +1905,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   const size_t C = g.chains, tiles = C * g.nt, FS = FLAG_STRIDE;
   w.err = cv.take<int>(64);
   w.ring = bwd ? handoff_ring(g) : 0;
-  w.nflags = (int)((bwd ? (4 + 2 * (size_t)w.ring) * tiles + 2 : 2 * tiles) * FS + FS);
+  w.nflags = (int)((bwd ? (3 + 2 * (size_t)w.ring) * tiles + 2 : 2 * tiles) * FS + FS);
   w.flags = cv.take<int>(w.nflags);
   int* f = w.flags;
   w.flag1 = f;
@@ -1928,10 +1914,8 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   if (bwd) {
     w.hflag = f;
     f += 2 * (size_t)w.ring * tiles * FS;
-    for (int k = 0; k < 2; ++k) {
-      w.accflag[k] = f;
-      f += tiles * FS;
-    }
+    w.accflag = f;
+    f += tiles * FS;
     w.sums_done = f;
     w.r1done = f + FS;
     f += 2 * FS;
@@ -1944,10 +1928,11 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
     // byte offsets inside a slot (all multiples of 16)
     w.off_gz = tiles * g.MF * D * 2;
     w.off_rs = w.off_gz + tiles * g.MF * 4;
-    w.off_img = w.off_rs + tiles * T * 2 * 4;
-    w.hand_slot = (w.off_img + tiles * ((size_t)4 * T * g.MF + 2 * T * T) + 255) & ~size_t(255);
+    w.off_dq = w.off_rs + tiles * T * 2 * 4;
+    w.off_img = w.off_dq + tiles * g.MF * D * 4;
+    w.hand_slot = (w.off_img + tiles * ((size_t)2 * T * g.MF + 2 * T * T) + 255) & ~size_t(255);
     w.hand = cv.take<uint8_t>(w.ring * w.hand_slot);
-    w.acc = cv.take<float>(2 * tiles * (size_t)g.MF * D);
+    w.acc = cv.take<float>(tiles * (size_t)g.MF * D);
     w.rsums = cv.take<float>((size_t)RS1 * g.MF * D);
   }
   return w;
@@ -2060,7 +2045,7 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
 // Final reduction: stage-1 CTAs each sum at least 8 positions, at most RS1
 // CTAs, a multiple of 4; stage 2 takes a quarter as many (at least 4).
 void reduction_split(const Geo& g, int& r1n, int& r2n) {
-  const int nparts = 2 * g.chains * g.nt;
+  const int nparts = g.chains * g.nt;
   r1n = nparts / 8;
   r1n = r1n < 4 ? 4 : (r1n > RS1 ? RS1 : r1n);
   r1n -= r1n % 4;
@@ -2090,10 +2075,10 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
   J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
                 w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
-                0, 0, nullptr, nullptr, 0, nullptr, dq, w.err, gio};
+                nullptr, 0, 0, dq, w.err, gio};
   J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
-                  p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
-  J.red = RedJob{w.acc, 2 * g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
+                  nullptr, p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
+  J.red = RedJob{w.acc, g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
   J.L = p.L;
   J.Cs = g.Cs;
   J.ticket = w.ticket;
@@ -2101,19 +2086,20 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   J.hand_slot = w.hand_slot;
   J.off_gz = w.off_gz;
   J.off_rs = w.off_rs;
+  J.off_dq = w.off_dq;
   J.off_img = w.off_img;
   J.ring = w.ring;
   J.hflag = w.hflag;
-  for (int x = 0; x < 2; ++x) J.accflag[x] = w.accflag[x];
+  J.accflag = w.accflag;
   J.acc = w.acc;
   J.sums_done = w.sums_done;
   J.r1done = w.r1done;
-  // Algorithmic work per row: dq side 14dM (phiQ, phiK, rollback Delta,
-  // dphiQ, G, dq, dOmega), dk/dv side 8dM (dV, dphiK, dk, dOmega).
+  // Algorithmic work per row: dq part 14dM (phiQ, phiK, rollback Delta,
+  // dphiQ, G, dq, dOmega), dk/dv part 8dM (dV, dphiK, dk, dOmega).
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
   const long long items = sched_items(J.s);
   prof::Scope ps(prof::K_TC_BWD, s, rows * 22.0 * MD, rows * D * 2.0 * 12);
-  if (2 * g.chains * g.nt >= EARLY_STAGE)
+  if (g.chains * g.nt >= EARLY_STAGE)
     TC_TRY(launch_dep(k_tc_bwd<MF, FEAT, true>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(), s,
                       J));
   else

@@ -146,11 +146,11 @@ def test_bwd_schedule_arguments(lib):
     # count only (no buffer), then the tensor-core problems it serves
     assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, None, 0, ctypes.byref(n),
                                  ctypes.byref(ring)) == OK
-    assert n.value == 4 * 2 * 64 * 8 + 128 + 32 and ring.value == 2
+    assert n.value == 4 * 64 * 8 + 64 + 16 and ring.value == 2
     buf = (ctypes.c_int * 6)()
     assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, buf, 2, ctypes.byref(n),
                                  None) == OK
-    assert list(buf) == [0, 3, 0, 0, 3, 1]  # the first two tickets: dq side of the last slice
+    assert list(buf) == [0, 3, 0, 0, 3, 1]  # the first two tickets: tiles of the last slice
     # argument errors before anything else
     assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, None, 0, None, None) == INVALID
     assert lib.slim_bwd_schedule(8, 8, 4096, 64, 256, 1024, 1, 0, None, 4, ctypes.byref(n),

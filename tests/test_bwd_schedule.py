@@ -14,7 +14,7 @@ import torch
 
 from paper_2012_11346_gb300 import slim
 
-Q, KV, R1, R2 = 0, 1, 2, 3
+TILE, R1, R2 = 0, 2, 3
 T = 128
 
 # (B, H, L, C): full slices, a ragged last slice with fewer tiles, one-tile
@@ -39,12 +39,13 @@ def geometry(B, H, L, C):
 
 
 def tile_item(ntn, ch, n, t, c):
-    # both sides: last tile first, chains inside a tile position
+    # last tile first, chains inside a tile position
     return (ntn[n] - 1 - t) * ch + c
 
 
 def dependencies(B, H, L, C, items):
-    """For every ticket, the tickets of the items its waits stand for."""
+    """For every ticket, the tickets of the items its waits stand for.  A tile
+    item runs the tile's dq part and then its dk/dv part."""
     ch, N, ntn = geometry(B, H, L, C)
     R = ring(B, H, L, C)
     ticket = {it: x for x, it in enumerate(items)}
@@ -52,21 +53,18 @@ def dependencies(B, H, L, C, items):
     deps = []
     for kind, n, idx in items:
         d = []
-        if kind in (Q, KV):
+        if kind == TILE:
             c, t = idx % ch, ntn[n] - 1 - idx // ch
-            if kind == Q:
-                if t + 1 < ntn[n]:  # rollback and state-gradient chains
-                    d.append(ticket[(Q, n, tile_item(ntn, ch, n, t + 1, c))])
-                elif n + 1 < N:
-                    d.append(ticket[(Q, n + 1, tile_item(ntn, ch, n + 1, 0, c))])
-                if n + R < N and t < ntn[n + R]:  # hand-off ring slot n % R
-                    d.append(ticket[(KV, n + R, tile_item(ntn, ch, n + R, t, c))])
-            else:
-                d.append(ticket[(Q, n, tile_item(ntn, ch, n, t, c))])  # its dq side
+            if t + 1 < ntn[n]:  # rollback and state-gradient chains
+                d.append(ticket[(TILE, n, tile_item(ntn, ch, n, t + 1, c))])
+            elif n + 1 < N:
+                d.append(ticket[(TILE, n + 1, tile_item(ntn, ch, n + 1, 0, c))])
+            if n + R < N and t < ntn[n + R]:  # hand-off ring slot n % R
+                d.append(ticket[(TILE, n + R, tile_item(ntn, ch, n + R, t, c))])
             if n + 1 < N and t < ntn[n + 1]:  # the dOmega sum at this position
-                d.append(ticket[(kind, n + 1, tile_item(ntn, ch, n + 1, t, c))])
+                d.append(ticket[(TILE, n + 1, tile_item(ntn, ch, n + 1, t, c))])
         elif kind == R1:
-            d += [ticket[(k, 0, i)] for k in (Q, KV) for i in range(ch * ntn[0])]
+            d += [ticket[(TILE, 0, i)] for i in range(ch * ntn[0])]
         else:
             d += [ticket[(R1, 0, r)] for r in range(r1n)]
         deps.append(d)
@@ -79,10 +77,9 @@ def test_every_item_once(shape):
     ch, N, ntn = geometry(B, H, L, C)
     items = schedule(B, H, L, C)
     assert len(set(items)) == len(items)
-    for kind in (Q, KV):
-        for n in range(N):
-            got = sorted(i for k, s, i in items if k == kind and s == n)
-            assert got == list(range(ch * ntn[n])), (kind, n)
+    for n in range(N):
+        got = sorted(i for k, s, i in items if k == TILE and s == n)
+        assert got == list(range(ch * ntn[n])), n
     r1 = sorted(i for k, s, i in items if k == R1)
     r2 = sorted(i for k, s, i in items if k == R2)
     assert r1 == list(range(len(r1))) and r2 == list(range(len(r2)))
@@ -101,29 +98,29 @@ def test_waits_are_on_lower_tickets(shape):
 
 @pytest.mark.parametrize("shape", SHAPES)
 def test_ring_keeps_the_reuse_wait_far_back(shape):
-    # the dq side of slice n-R waits on slice n's dk/dv side: at least 320
-    # tickets apart (about two waves of tile CTAs), R in [2, 16]
+    # slice n-R's tile waits on slice n's tile at its position to have read the
+    # hand-off: at least 320 tickets apart (about two waves of tile CTAs), R in
+    # [2, 16]
     B, H, L, C = shape
     ch, N, ntn = geometry(B, H, L, C)
     R = ring(B, H, L, C)
     assert 2 <= R <= 16
-    stage = 2 * ch * ntn[0]
+    stage = ch * ntn[0]
     assert (R - 1) * stage >= 320 or R == 16
     assert R == 2 or (R - 2) * stage < 320
 
 
 def test_stage_order():
-    # stage j: dq side of slice N-1-j and dk/dv side of slice N-j, alternating by
-    # rows of B*H tiles (dq first); a dk/dv tile comes a stage after its dq tile
+    # stage j: the tiles of slice N-1-j, last tile first, chains inside a tile
+    # position
     B, H, L, C = 8, 8, 4096, 1024
     ch, N, ntn = geometry(B, H, L, C)
     items = schedule(B, H, L, C)
-    assert items[:ch] == [(Q, N - 1, i) for i in range(ch)]
-    stage1 = items[ch * ntn[N - 1]:ch * ntn[N - 1] + 2 * ch]
-    assert stage1 == [(Q, N - 2, i) for i in range(ch)] + [(KV, N - 1, i) for i in range(ch)]
-    first = {it: x for x, it in enumerate(items)}
-    gap = min(first[(KV, n, i)] - first[(Q, n, i)] for n in range(N) for i in range(ch * ntn[n]))
-    assert gap >= ch * min(ntn)
+    off = 0
+    for j in range(N):
+        n = N - 1 - j
+        assert items[off:off + ch * ntn[n]] == [(TILE, n, i) for i in range(ch * ntn[n])]
+        off += ch * ntn[n]
 
 
 def progress(shape, resident, seed):
@@ -136,30 +133,27 @@ def progress(shape, resident, seed):
     deps = dependencies(B, H, L, C, items)
     R = ring(B, H, L, C)
     r1n = sum(1 for it in items if it[0] == R1)
-    flag1, flag2 = {}, {}
-    gflag, kvread, accflag = [{} for _ in range(R)], [{} for _ in range(R)], [{}, {}]
+    flag1, flag2, accflag = {}, {}, {}
+    kvread = [{} for _ in range(R)]
     sums_done = r1done = 0
     done = [False] * len(items)
 
     def ready(x):
         kind, n, idx = items[x]
-        if kind in (Q, KV):
+        if kind == TILE:
             c, t = idx % ch, ntn[n] - 1 - idx // ch
             ok = True
-            if kind == Q:
-                inner = t + 1 < ntn[n]
-                if inner or n + 1 < N:
-                    snext, want = (t + 1, n + 1) if inner else (0, n + 2)
-                    ok &= flag1.get((c, snext), 0) == want and flag2.get((c, snext), 0) == want
-                if n + R < N and t < ntn[n + R]:
-                    ok &= kvread[n % R].get((c, t), 0) == n + R + 1
-            else:
-                ok &= gflag[n % R].get((c, t), 0) == n + 1
+            inner = t + 1 < ntn[n]
+            if inner or n + 1 < N:
+                snext, want = (t + 1, n + 1) if inner else (0, n + 2)
+                ok &= flag1.get((c, snext), 0) == want and flag2.get((c, snext), 0) == want
+            if n + R < N and t < ntn[n + R]:
+                ok &= kvread[n % R].get((c, t), 0) == n + R + 1
             if n + 1 < N and t < ntn[n + 1]:
-                ok &= accflag[kind].get((c, t), 0) == n + 2
+                ok &= accflag.get((c, t), 0) == n + 2
             return ok
         if kind == R1:
-            return sums_done >= 2 * ch * nt
+            return sums_done >= ch * nt
         return r1done >= r1n
 
     rng = random.Random(seed)
@@ -173,13 +167,11 @@ def progress(shape, resident, seed):
         x = rng.choice(can)
         assert all(done[y] for y in deps[x]), f"ticket {x} {items[x]} ran early"
         kind, n, idx = items[x]
-        if kind in (Q, KV):
+        if kind == TILE:
             c, t = idx % ch, ntn[n] - 1 - idx // ch
-            if kind == Q:
-                flag1[(c, t)] = flag2[(c, t)] = gflag[n % R][(c, t)] = n + 1
-            else:
-                kvread[n % R][(c, t)] = n + 1
-            accflag[kind][(c, t)] = n + 1
+            flag1[(c, t)] = flag2[(c, t)] = n + 1
+            kvread[n % R][(c, t)] = n + 1
+            accflag[(c, t)] = n + 1
             sums_done += n == 0
         elif kind == R1:
             r1done += 1

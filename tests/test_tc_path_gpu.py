@@ -81,20 +81,20 @@ def _ring(B, H, L, C, M):
 
 
 def test_tc_handoff_ring_wraps_short_stages(cuda_device):
-    """Two chains of one-tile slices: stages of 4 items, so the running-sum
-    flags are polled just before the adds, and the 16-slot hand-off ring is
-    reused over 32 slices (each dq tile of slice n waits for slice n+16's
-    dk/dv tile to have read its slot)."""
+    """Two chains of one-tile slices: stages of 2 items, so the running-sum
+    flag is polled just before the adds, and the 16-slot hand-off ring is
+    reused over 32 slices (each tile of slice n waits for slice n+16's tile at
+    its position to have read its slot)."""
     assert _ring(1, 2, 4096, 128, 256) == 16
     _run_case(cuda_device, 1, 2, 4096, 128)
 
 
 def test_tc_handoff_ring_wraps_long_stages(cuda_device):
-    """64 chains of one-tile slices of 64 rows: stages of 128 items, so the
-    flags are polled up front and the hand-off is released after the last
-    join, and the 4-slot ring is reused (5 slices)."""
-    assert _ring(4, 16, 320, 64, 128) == 4
-    _run_case(cuda_device, 4, 16, 320, 64, M=128)
+    """128 chains of one-tile slices of 64 rows: stages of 128 items, so the
+    running-sum flag is polled up front, and the 4-slot ring is reused (5
+    slices)."""
+    assert _ring(4, 32, 320, 64, 128) == 4
+    _run_case(cuda_device, 4, 32, 320, 64, M=128)
 
 
 def test_tc_workspace_reuse(cuda_device):
