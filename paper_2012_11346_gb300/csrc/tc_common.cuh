@@ -113,6 +113,11 @@ __device__ __forceinline__ uint64_t l2_evict_first() {
   asm("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// Brings `bytes` (a multiple of 16, 16-byte aligned) of global memory into L2
+// ahead of a later load.
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 // The source is read for the last time (evict-first in L2).
 __device__ __forceinline__ void bulk_load(uint32_t sdst, const void* gsrc, uint32_t bytes,
                                           uint32_t mbar) {

@@ -723,7 +723,6 @@ struct BwdQJob {
                           //   image (bf16, 128-byte swizzle), then tril(A) in bf16,
                           //   lane-major (chunk of 8 columns c/8, row r at 16-byte
                           //   unit (c/8) 128 + r)
-  int* gflag;             // [chains][nt]: n + 1 once the five above are written
   const int* kvread;      // [chains][nt]: n + R + 1 once slice n+R's dk/dv part has read them
   int ring;               // R, slots of the hand-off ring
   int nRtiles;            // tiles of slice n+R per chain (0: no such slice)
@@ -739,7 +738,8 @@ struct BwdQJob {
 // columns (all 512) are allocated by the caller for both parts of the tile.
 template <int MF, int FEAT>
 __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* smem_raw,
-                                           uint64_t* mb, uint32_t& tmem_base, int& abort_) {
+                                           uint64_t* mb, uint32_t& tmem_base, int& abort_,
+                                           int& done_) {
   using C = Cfg<MF>;
   uint8_t* base = align1024(smem_raw);
   uint8_t* sPhiQ = base;              // first: norm scratch | Omega lo (upper half)
@@ -1019,8 +1019,10 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     __syncthreads();
     if (gfail[0] | gfail[1]) goto teardown;
     // phiK's tile image, while the MMAs of the next phases run (the tile is
-    // overwritten by u once the copy has read it)
+    // overwritten by u once the copy has read it); Q, read again after them,
+    // back into L2
     if (tid == GRP) bulk_store(img, smem_u32(sPhiK), C::FEATB);
+    if (tid == GRP + 32) prefetch_l2(J.Q + g0, (uint32_t)valid * 128u);
     {
       // g(Q) . z_t over this thread's feature columns
       constexpr int W = MF / NG;
@@ -1214,6 +1216,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     }
   join2:
     __syncthreads();
+    // K and V, which the dk/dv part reads next, back into L2
+    if (tid == GRP) prefetch_l2(J.K + g0, (uint32_t)valid * 128u);
+    if (tid == GRP + 32) prefetch_l2(J.V + g0, (uint32_t)valid * 128u);
     {
       float us = 0.f;
       if (FEAT == SLIM_FEAT_EXP) us = redU[row] + redU[T + row];
@@ -1231,13 +1236,9 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
         tmem_ld16(trow + 320 + 64 * h + 16 * cg, v);
         st_lm16(dqp, h, cg, row, v);
       }
-      __syncthreads();
-      if (tid == GRP) {
-        // the hand-off to the dk/dv part: G_t, g_t(z), rowstat, tril(A), the
-        // dOmega partial and, once its bulk copy is done, phiK's image
-        bulk_wait_done();
-        st_release_gpu(J.gflag + tf * FLAG_STRIDE, n + 1);
-      }
+      // the hand-off to the dk/dv part is complete once phiK's bulk copy is:
+      // the part follows in this CTA, after a barrier
+      if (tid == GRP) bulk_wait_done();
       float xq[16];
       ld_feat16(sQ, row, 16 * cg, xq);
       tmem_ld16(trow + 256 + 16 * cg, v);
@@ -1245,6 +1246,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       for (int i = 0; i < 16; ++i) v[i] = fmaf(-us, xq[i], v[i]);
       if (rv) st_row16(J.dq + g0 + (size_t)row * D + 16 * cg, v);
     }
+    if (tid == 0) done_ = 1;  // reached only when no wait gave up
   }
   TC_TEARDOWN_KEEP();
 }
@@ -1257,7 +1259,6 @@ struct BwdKVJob {
   const float *gz, *rowstat;
   const float* domq;         // [chains][ntf][MF][64] lane-major: the dq part's u^T q
   const uint8_t* img;        // [chains][ntf][...] phiK's tile image, tril(A) lane-major
-  const int* gflag;          // n + 1 once they are written
   int* kvread;               // set to n + 1 once this part has read them
   int L, a, b, ntn, ntf, n;  // slice n = rows [a, a+b), ntn tiles; ntf: full slice
   __nv_bfloat16 *dk, *dv;
@@ -1272,7 +1273,7 @@ struct BwdKVJob {
 // The dk/dv part of a tile, run by the CTA that ran its dq part: phiQ is still
 // in shared memory, and the rest of the hand-off was written by this CTA and
 // is read back from L2.  The TMEM columns are the caller's.
-template <int MF, int FEAT, bool EARLY>
+template <int MF, int FEAT>
 __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uint8_t* smem_raw,
                                             uint64_t* mb, uint32_t& tmem_base, int& abort_) {
   using C = Cfg<MF>;
@@ -1287,7 +1288,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   uint8_t* sOm = sX + 2 * ROWT;
   uint8_t* sG = sOm;
   uint8_t* sV = sOm + C::OMB;
-  uint8_t* sDn = sV + ROWT;            // dout, then dnum in place
+  uint8_t* sDn = sV + ROWT;            // dnum, as the dq part left it (its sDo)
   float* sGz = reinterpret_cast<float*>(sDn + ROWT);
   const int row0 = J.a + t * T;
   const int valid = min(T, J.b - t * T);
@@ -1295,8 +1296,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   const size_t tf = (size_t)c * J.ntf + t;  // hand-off buffers, flags, dOmega sums
   const bool acc_first = t >= J.n1tiles;
   float den = 0.f, dden = 0.f;
-  __shared__ int poll_ok;              // written by the polling thread only
-  __shared__ __align__(8) uint64_t mb_img;  // phiK's tile, initialised by that thread
+  __shared__ __align__(8) uint64_t mb_img;  // phiK's tile, initialised by one thread
   const int tid = threadIdx.x, warp = tid >> 5;
   const int row = 32 * (warp & 3) + (tid & 31);
   const int cg = warp >> 2;
@@ -1307,64 +1307,43 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
   }
   uint8_t* const img = const_cast<uint8_t*>(J.img) + tf * ((size_t)C::FEATB + 2 * ROWT);
   if (tid == POLL) {
-    // while V and dout stream in: phiK, tril(A), G_t, g_t(z), the row
-    // statistics and the dOmega partial come from the dq part of this tile;
-    // phiK's tile by a bulk copy completing on mb_img
-    poll_ok = flag_poll2(J.gflag + tf * FLAG_STRIDE, J.n + 1,
-                         EARLY && !acc_first ? J.accflag + tf * FLAG_STRIDE : nullptr, J.n + 2,
-                         J.err);
-    if (poll_ok) {
-      const uint32_t bar = smem_u32(&mb_img);
-      mbar_init(bar, 1);
-      mbar_fence_init();
-      fence_proxy_async_global();
-      mbar_expect_tx(bar, C::FEATB);
-      bulk_load(smem_u32(sPhiK), img, C::FEATB, bar);
-    }
-  } else if (tid < LDT) {
-    load_rows64(sV, T, J.V + g0, valid, tid, LDT);
-    load_rows64(sDn, T, J.dOut + g0, valid, tid, LDT);
+    // phiK, tril(A), G_t, g_t(z), the row statistics and the dOmega partial
+    // come from the dq part of this tile, which this CTA ran before a barrier
+    // (its bulk copy waited for and fenced); phiK's tile by a bulk copy
+    // completing on mb_img
+    const uint32_t bar = smem_u32(&mb_img);
+    mbar_init(bar, 1);
+    mbar_fence_init();
+    fence_proxy_async_global();
+    mbar_expect_tx(bar, C::FEATB);
+    bulk_load(smem_u32(sPhiK), img, C::FEATB, bar);
   }
-  grid_dependency_wait();
-  cp_async_wait_all();
-  __syncthreads();  // rows were copied by other threads
-  if (!poll_ok) goto teardown;
-  for (int m = tid; m < MF; m += NTHR) sGz[m] = __ldcg(J.gz + tf * MF + m);
+  // every other load at once: V, dout, G_t (lane-major -> its tile), tril(A)
+  // (lane-major -> its tile), the row statistics and g_t(z)
   if (row < valid) {
     const float* rsr = J.rowstat + (tf * T + row) * 2;
     den = __ldcg(rsr);
     dden = __ldcg(rsr + 1);
   }
-  load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);  // G_t(S), awaited before the dV products
+  // (dnum = dout / den is still in its tile: the dq part left it there)
+  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
+  load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);
   {
-    // tril(A) into its tile (lane-major in global memory: coalesced reads)
     const uint8_t* imgA = img + C::FEATB;
     for (int k = tid; k < T * T / 8; k += NTHR)
       cp_async16(smem_u32(sA) + tile_off(T, k % T, 8 * (k / T)), imgA + (size_t)k * 16, 16u);
   }
+  for (int m = tid; m < MF; m += NTHR) sGz[m] = __ldcg(J.gz + tf * MF + m);
+  cp_async_wait_all();
+  __syncthreads();  // rows were copied by other threads
   {
     const bool rv = row < valid;
     const uint32_t tmem = tmem_base;
     const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
     Sync sy{mb, 0, J.err};
     const bool live = rv && den != 0.f;
-    const float inv = live ? 1.f / den : 0.f;
     if (!live) dden = 0.f;
-#pragma unroll
-    for (int c8 = 16 * cg; c8 < 16 * cg + 16; c8 += 8) {  // dnum = dout / den, in place
-      const uint4 g = ld_chunk(sDn, T, row, c8);
-      const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
-      uint32_t pw[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        float g0f, g1f;
-        unpack_bf16(gw[i], g0f, g1f);
-        pw[i] = pack_bf16(g0f * inv, g1f * inv);
-      }
-      st_chunk(sDn, T, row, c8, make_uint4(pw[0], pw[1], pw[2], pw[3]));
-    }
     if (!mbar_wait(smem_u32(&mb_img), 0, J.err)) abort_ = 1;  // phiK's tile
-    cp_async_wait_all();  // G_t(S), tril(A)
     publish();
     if (abort_) goto teardown;
     // every thread has what it needs of the hand-off but the dOmega partial
@@ -1485,8 +1464,13 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
 #pragma unroll
       for (int g = 0; g < NG; ++g) us += redU[g * T + row];
     }
+    // the dq part's dOmega partial, fetched while the last products run
+    const float* dqp = J.domq + tf * (size_t)(MF * 64);
+    float wq[C::MH][16];
+#pragma unroll
+    for (int h = 0; h < C::MH; ++h) ld_lm16(dqp, h, cg, row, wq[h]);
     // slice n+1's dOmega sum at this position, added to after the next waits
-    if (tid == POLL && !EARLY && !acc_first &&
+    if (tid == POLL && !acc_first &&
         !flag_poll(J.accflag + tf * FLAG_STRIDE, J.n + 2, J.err))
       abort_ = 1;
     TC_WAIT(sy);
@@ -1496,14 +1480,12 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       // running dOmega sum at this position (or starts it): one add per
       // slice, in slice order
       float* accp = J.acc + tf * (size_t)(MF * 64);
-      const float* dqp = J.domq + tf * (size_t)(MF * 64);
-      float v[16], w[16];
+      float v[16];
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         tmem_ld16(trow + 64 + 64 * h + 16 * cg, v);
-        ld_lm16(dqp, h, cg, row, w);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] += w[i];
+        for (int i = 0; i < 16; ++i) v[i] += wq[h][i];
         if (acc_first)
           st_lm16(accp, h, cg, row, v);
         else
@@ -1730,8 +1712,8 @@ struct BwdJob {
   int* ticket;
   // hand-off ring: slot k (slice n uses n % ring) holds, at hand + k hand_slot,
   // G_t(S) bf16 [chains][nt][M][64], then g_t(z), the row statistics, the dq
-  // part's dOmega partials and the tile images at the given offsets; its two
-  // flag arrays (gflag, kvread) are hflag + (2k, 2k+1) * chains * nt * FLAG_STRIDE
+  // part's dOmega partials and the tile images at the given offsets; its flag
+  // array (kvread) is hflag + k * chains * nt * FLAG_STRIDE
   uint8_t* hand;
   size_t hand_slot, off_gz, off_rs, off_dq, off_img;
   int ring;
@@ -1741,17 +1723,12 @@ struct BwdJob {
   int *sums_done, *r1done;  // slice-0 tiles done, final stage-1 CTAs done
 };
 
-// EARLY (stages of at least EARLY_STAGE items): the dOmega-sum flag a tile
-// waits on was set long before it starts, so the dk/dv part polls it up
-// front.  With shorter stages, tiles of neighbouring slices run at the same
-// time, and it is polled just before the adds, so that no tile waits for
-// another one to finish.
-template <int MF, int FEAT, bool EARLY>
+template <int MF, int FEAT>
 __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJob J) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t mbar[2 * NBAR];  // the dq part's, then the dk/dv part's
   __shared__ uint32_t tmem_base;
-  __shared__ int abort_;
+  __shared__ int abort_, done_;
   __shared__ int ticket;
   if (threadIdx.x == 0) ticket = atomicAdd(J.ticket, 1);
   __syncthreads();
@@ -1763,7 +1740,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
     const size_t tiles = (size_t)J.s.chains * J.s.nt;
     const int slot = n % J.ring;
     uint8_t* hs = J.hand + slot * J.hand_slot;
-    int* hf = J.hflag + (size_t)(2 * slot) * tiles * FLAG_STRIDE;
+    int* hf = J.hflag + (size_t)slot * tiles * FLAG_STRIDE;
     BwdQJob q = J.q;
     q.a = a;
     q.b = b;
@@ -1774,8 +1751,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
     q.rowstat = reinterpret_cast<float*>(hs + J.off_rs);
     q.domq = reinterpret_cast<float*>(hs + J.off_dq);
     q.img = hs + J.off_img;
-    q.gflag = hf;
-    q.kvread = hf + tiles * FLAG_STRIDE;
+    q.kvread = hf;
     q.ring = J.ring;
     q.nRtiles = n + J.ring < N ? (n + J.ring == N - 1 ? J.s.ntl : J.s.nt) : 0;
     BwdKVJob kv = J.kv;
@@ -1788,24 +1764,23 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
     kv.rowstat = q.rowstat;
     kv.domq = q.domq;
     kv.img = q.img;
-    kv.gflag = hf;
-    kv.kvread = hf + tiles * FLAG_STRIDE;
+    kv.kvread = hf;
     kv.acc = J.acc;
     kv.accflag = J.accflag;
     kv.n1tiles = n1;
     kv.sums_done = n == 0 ? J.sums_done : nullptr;
     // one TMEM allocation (all 512 columns) serves both parts of the tile
+    if (threadIdx.x == 0) done_ = 0;
     if (threadIdx.x < 32) tmem_alloc(smem_u32(&tmem_base), 512);
-    role_bwd_q<MF, FEAT>(q, it.idx, smem_raw, mbar, tmem_base, abort_);
+    role_bwd_q<MF, FEAT>(q, it.idx, smem_raw, mbar, tmem_base, abort_, done_);
     __syncthreads();
-    // a wait of the dq part that gave up (or saw another CTA's failure) has set
-    // the error word: the dk/dv part would only wait on what never comes
-    const bool failed = *reinterpret_cast<volatile int*>(J.q.err) != 0;
-    if (!failed) {
+    // the dk/dv part runs only after a complete dq part (a wait that gave up
+    // has left the error word set; the part would wait on what never comes)
+    if (done_) {
       tc_fence_after();
       // the dq part's order: last tile first, chains inside a position
-      role_bwd_kv<MF, FEAT, EARLY>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains,
-                                   smem_raw, mbar + NBAR, tmem_base, abort_);
+      role_bwd_kv<MF, FEAT>(kv, ntn - 1 - it.idx / J.s.chains, it.idx % J.s.chains, smem_raw,
+                            mbar + NBAR, tmem_base, abort_);
     }
     tc_fence_before();
     __syncthreads();
@@ -1873,7 +1848,6 @@ Geo geometry(const Problem& p) {
 // once at the end.
 constexpr int KV_LEAD = 320;  // about two waves of tile CTAs
 constexpr int MAX_RING = 16;
-constexpr int EARLY_STAGE = 128;  // see k_tc_bwd
 int handoff_ring(const Geo& g) {
   const int stage = g.chains * g.nt;  // items of a full stage
   const int r = 1 + (KV_LEAD + stage - 1) / stage;
@@ -1884,7 +1858,7 @@ struct Ws {
   int* flags;  // every flag and counter of the call, zeroed together
   int nflags;
   int *flag1, *flag2;         // [chains][nt] chain flags, FLAG_STRIDE ints each
-  int* hflag;                 // [ring][2][chains][nt] hand-off flags (backward)
+  int* hflag;                 // [ring][chains][nt] hand-off flags (backward)
   int* accflag;               // [chains][nt]: dOmega sums (backward)
   int *sums_done, *r1done;    // final reduction counters (backward)
   int* ticket;
@@ -1905,7 +1879,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   const size_t C = g.chains, tiles = C * g.nt, FS = FLAG_STRIDE;
   w.err = cv.take<int>(64);
   w.ring = bwd ? handoff_ring(g) : 0;
-  w.nflags = (int)((bwd ? (3 + 2 * (size_t)w.ring) * tiles + 2 : 2 * tiles) * FS + FS);
+  w.nflags = (int)((bwd ? (3 + (size_t)w.ring) * tiles + 2 : 2 * tiles) * FS + FS);
   w.flags = cv.take<int>(w.nflags);
   int* f = w.flags;
   w.flag1 = f;
@@ -1913,7 +1887,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   f += 2 * tiles * FS;
   if (bwd) {
     w.hflag = f;
-    f += 2 * (size_t)w.ring * tiles * FS;
+    f += (size_t)w.ring * tiles * FS;
     w.accflag = f;
     f += tiles * FS;
     w.sums_done = f;
@@ -1962,10 +1936,7 @@ cudaError_t configure() {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem_fwd<MF>());
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem_bwd<MF>());
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(k_tc_bwd<MF, FEAT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem_bwd<MF>());
   if (e != cudaSuccess) return e;
   *done = true;
@@ -2075,9 +2046,9 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
   J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
                 w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
-                nullptr, 0, 0, dq, w.err, gio};
+                0, 0, dq, w.err, gio};
   J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
-                  nullptr, p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
+                  p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
   J.red = RedJob{w.acc, g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
   J.L = p.L;
   J.Cs = g.Cs;
@@ -2099,12 +2070,7 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
   const long long items = sched_items(J.s);
   prof::Scope ps(prof::K_TC_BWD, s, rows * 22.0 * MD, rows * D * 2.0 * 12);
-  if (g.chains * g.nt >= EARLY_STAGE)
-    TC_TRY(launch_dep(k_tc_bwd<MF, FEAT, true>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(), s,
-                      J));
-  else
-    TC_TRY(launch_dep(k_tc_bwd<MF, FEAT, false>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(),
-                      s, J));
+  TC_TRY(launch_dep(k_tc_bwd<MF, FEAT>, dim3((unsigned)items), dim3(NTHR), smem_bwd<MF>(), s, J));
   return SLIM_OK;
 }
 
