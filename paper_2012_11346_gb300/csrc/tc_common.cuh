@@ -17,6 +17,7 @@
 //             distance between 64-column blocks, SBO = 1024 B (8 K rows).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -113,6 +114,30 @@ __device__ __forceinline__ uint64_t l2_evict_first() {
   asm("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// ------------------------------------------------------------------ TMA tile loads
+// Tensor-map loads into 128-byte-swizzled row tiles (the layout above): the
+// map's box is {64 bf16, R rows[, 1]} with CU_TENSOR_MAP_SWIZZLE_128B, the
+// shared destination is 1024-byte aligned, and the innermost coordinate is 0
+// (16-byte aligned).  Elements outside the tensor read as zero.  The map is a
+// __grid_constant__ kernel parameter (param space); completion is counted on
+// mbar like a bulk copy.
+__device__ __forceinline__ void tma_load_3d(uint32_t sdst, const CUtensorMap* map, int y, int z,
+                                            uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(sdst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(y), "r"(z), "r"(mbar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t sdst, const CUtensorMap* map, int y,
+                                            uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3}], [%4];" ::"r"(sdst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(y), "r"(mbar)
+      : "memory");
+}
+
 // Brings `bytes` (a multiple of 16, 16-byte aligned) of global memory into L2
 // ahead of a later load.
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {

@@ -165,7 +165,9 @@ struct Sync {
     return ok;
   }
 };
-constexpr int NBAR = 9;  // mbarriers per tile CTA
+constexpr int NBAR = 12;  // mbarriers per tile CTA (and per part of a backward tile)
+// the ones for tensor-map loads: the row tiles, Omega, and a later reload
+constexpr int MB_TILES = 9, MB_OMEGA = 10, MB_RELOAD = 11;
 
 // Make generic-proxy smem writes visible to the tensor core and order them
 // with the thread that issues the next MMAs.
@@ -340,6 +342,9 @@ __device__ __forceinline__ void fill_ones(uint8_t* tile, int tid) {
 
 // ================================================================== forward
 struct FwdJob {
+  // tensor maps of q, k, v ([chains][L][64] bf16, box {64, 128, 1}) and of
+  // Omega's bf16 hi/lo rows ([2 M][64], box {64, M})
+  CUtensorMap tq, tk, tv, tom;
   const __nv_bfloat16 *Q, *K, *V, *om16;
   int L, Cs, N, nt, P, chains;  // slice length, slices, tiles of a full slice, tile positions
   float* slot;                  // [chains][nt][E] inclusive prefixes
@@ -473,20 +478,32 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 512);
-  load_rows64(sQ, T, J.Q + g0, valid, tid, NTHR);
-  load_rows64(sK, T, J.K + g0, valid, tid, NTHR);
-  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
-  fill_ones(sOnes, tid);
-  if (tid < 2) gfail[tid] = 0;
-  grid_dependency_wait();  // Omega (bf16) and the slots belong to earlier kernels
-  load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
   // Omega lo in the upper half of the phiQ tile: that half is written only
   // by the g(Q) epilogue, after the Q projection (the last reader) is done,
   // while the phiK tile is overwritten as soon as the K projection is done
   uint8_t* sOl = sPhiQ + C::OMB;
-  load_rows64(sOl, MF, J.om16 + MF * D, MF, tid, NTHR);
-  cp_async_wait_all();
-  __syncthreads();  // rows were copied by other threads
+  if (tid == 0) {
+    // the three row tiles by TMA (rows past the chain's end read as zero)
+    const uint32_t bar = smem_u32(&mb[MB_TILES]);
+    mbar_expect_tx(bar, 3 * ROWT);
+    tma_load_3d(smem_u32(sQ), &J.tq, row0, c, bar);
+    tma_load_3d(smem_u32(sK), &J.tk, row0, c, bar);
+    tma_load_3d(smem_u32(sV), &J.tv, row0, c, bar);
+  }
+  fill_ones(sOnes, tid);
+  if (tid < 2) gfail[tid] = 0;
+  grid_dependency_wait();  // Omega (bf16) and the slots belong to earlier kernels
+  if (tid == 0) {
+    const uint32_t bar = smem_u32(&mb[MB_OMEGA]);
+    mbar_expect_tx(bar, 2 * C::OMB);
+    tma_load_2d(smem_u32(sOm), &J.tom, 0, bar);   // hi: rows [0, M)
+    tma_load_2d(smem_u32(sOl), &J.tom, MF, bar);  // lo: rows [M, 2M)
+  }
+  __syncthreads();  // the barriers' initialisation is seen by every thread
+  if (!mbar_wait(smem_u32(&mb[MB_TILES]), 0, J.err)) abort_ = 1;
+  if (!mbar_wait(smem_u32(&mb[MB_OMEGA]), 0, J.err)) abort_ = 1;
+  __syncthreads();
+  if (abort_) goto teardown;
   {
     const bool rv = row < valid;
     float* redN = reinterpret_cast<float*>(sPhiQ);  // 4 KB scratch below Omega lo
@@ -707,6 +724,8 @@ __device__ __forceinline__ void role_fwd(const FwdJob& J, int pos, int c, uint8_
 
 // ================================================================== backward, dq side
 struct BwdQJob {
+  // tensor maps (in the launch's parameters) of q, k, v, dout and Omega hi/lo
+  const CUtensorMap *tq, *tk, *tv, *tdo, *tom;
   const __nv_bfloat16 *Q, *K, *V, *Out, *dOut, *om16;
   StateIn fin;            // B^(N), the state the forward returned
   int L, a, b, ntn, n, N, nt, chains;  // slice n = rows [a, a+b), ntn tiles; nt: full slice
@@ -819,12 +838,20 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     const bool ok = flag_poll2(t < J.nRtiles ? J.kvread + tf * FLAG_STRIDE : nullptr,
                                n + J.ring + 1, nullptr, 0, J.err);
     gfail[1] = ok ? 0 : 1;
-  } else if (tid < LDT) {
-    load_rows64(sQ, T, J.Q + g0, valid, tid, LDT);
-    load_rows64(sK, T, J.K + g0, valid, tid, LDT);
-    load_rows64(sV, T, J.V + g0, valid, tid, LDT);
-    load_rows64(sDo, T, J.dOut + g0, valid, tid, LDT);
+  } else if (tid == 0) {
+    // the four row tiles by TMA (rows past the chain's end read as zero)
+    const uint32_t bar = smem_u32(&mb[MB_TILES]);
+    mbar_expect_tx(bar, 4 * ROWT);
+    tma_load_3d(smem_u32(sQ), J.tq, row0, c, bar);
+    tma_load_3d(smem_u32(sK), J.tk, row0, c, bar);
+    tma_load_3d(smem_u32(sV), J.tv, row0, c, bar);
+    tma_load_3d(smem_u32(sDo), J.tdo, row0, c, bar);
   }
+  // The rollback chain's flag is usually set before this tile starts: read it
+  // now, so that its round trip overlaps the loads (an acquire fence follows
+  // when it is used); the chain polls only if it was not set yet.
+  int early1 = 0, early2 = 0;
+  if (tid == GRP && linked) early1 = ld_relaxed_gpu(f1);
   // this thread's 16 columns of its out row, fetched while the tiles stream in
   uint4 orow[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
   if (row < valid) {
@@ -834,12 +861,17 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   }
   if (tid == 0) gfail[0] = 0;
   grid_dependency_wait();  // Omega (bf16), slots and buffers belong to earlier kernels
-  if (tid < LDT) {
-    load_rows64(sOm, MF, J.om16, MF, tid, LDT);
-    load_rows64(sOl, MF, J.om16 + MF * D, MF, tid, LDT);
+  if (tid == 0) {
+    const uint32_t bar = smem_u32(&mb[MB_OMEGA]);
+    mbar_expect_tx(bar, 2 * C::OMB);
+    tma_load_2d(smem_u32(sOm), J.tom, 0, bar);
+    tma_load_2d(smem_u32(sOl), J.tom, MF, bar);
   }
-  cp_async_wait_all();
-  __syncthreads();  // rows were copied by other threads
+  __syncthreads();  // the barriers' initialisation is seen by every thread
+  if (!mbar_wait(smem_u32(&mb[MB_TILES]), 0, J.err)) abort_ = 1;
+  if (!mbar_wait(smem_u32(&mb[MB_OMEGA]), 0, J.err)) abort_ = 1;
+  __syncthreads();
+  if (abort_) goto teardown;
   {
     const bool rv = row < valid;
     float* redN = reinterpret_cast<float*>(sPhiQ);  // 6 KB scratch below Omega lo
@@ -948,11 +980,14 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       redA[cg * T + row] = rs;  // V is no longer read: its tile holds the partials
     } else {
       // ---- chain group, rollback (eq. 17 per tile): the state before this
-      // tile is the state after it minus Delta_t
-      if (!mbar_wait(smem_u32(&mb[2]), 0, J.err)) gfail[1] = 1;
-      if (C::MH > 1 && !mbar_wait(smem_u32(&mb[6]), 0, J.err)) gfail[1] = 1;
-      tc_fence_after();
-      if (linked && gl == 0 && !gfail[1] && !flag_poll(f1, wnext, J.err)) gfail[1] = 1;
+      // tile is the state after it minus Delta_t.  The prefix after this tile
+      // is acquired and loaded while the Delta_t products run.
+      if (linked && gl == 0 && !gfail[1]) {
+        if (early1 == wnext)
+          fence_acq_rel_gpu();
+        else if (!flag_poll(f1, wnext, J.err))
+          gfail[1] = 1;
+      }
       group_bar(2);
       if (gfail[1]) goto join1;
       // every load of the prefix after this tile before any store: one L2 trip
@@ -984,6 +1019,11 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
 #pragma unroll
         for (int h = 0; h < C::MH; ++h) sz[h] += __ldcg(s1.z_lo + 128 * h + row);
       }
+      if (!mbar_wait(smem_u32(&mb[2]), 0, J.err)) gfail[1] = 1;
+      if (C::MH > 1 && !mbar_wait(smem_u32(&mb[6]), 0, J.err)) gfail[1] = 1;
+      tc_fence_after();
+      group_bar(2);
+      if (gfail[1]) goto join1;
 #pragma unroll
       for (int h = 0; h < C::MH; ++h) {
         const int m = 128 * h + row;
@@ -1018,6 +1058,8 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
   join1:
     __syncthreads();
     if (gfail[0] | gfail[1]) goto teardown;
+    // the state-gradient chain's flag, read ahead of its use (see early1)
+    if (tid == GRP && linked) early2 = ld_relaxed_gpu(f2);
     // phiK's tile image, while the MMAs of the next phases run (the tile is
     // overwritten by u once the copy has read it); Q, read again after them,
     // back into L2
@@ -1110,8 +1152,12 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     if (warp < 8) {
       // ---- compute group: Q and Omega again (dq = u Omega - q sum(u),
       // dOmega += u^T q), u = (dphiQ + dden z_t) (.) g'(Q), then the products
-      load_rows64(sQ, T, J.Q + g0, valid, tid, GRP);
-      load_rows64(sOm, MF, J.om16, MF, tid, GRP);
+      if (tid == 0) {
+        const uint32_t bar = smem_u32(&mb[MB_RELOAD]);
+        mbar_expect_tx(bar, ROWT + C::OMB);
+        tma_load_3d(smem_u32(sQ), J.tq, row0, c, bar);
+        tma_load_2d(smem_u32(sOm), J.tom, 0, bar);
+      }
       float usum = 0.f;
       const float rscale = rsqrtf((float)MF);
 #pragma unroll 1
@@ -1146,7 +1192,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
           st_chunk(sU, T, row, c0 + 8 * q, make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]));
       }
       redU[cg * T + row] = usum;
-      cp_async_wait_all();
+      if (!mbar_wait(smem_u32(&mb[MB_RELOAD]), 0, J.err)) gfail[0] = 1;
       group_publish(1);
       // dq and the dOmega partial go to the columns dphiQ held, so Gd stays
       // readable for the chain group; one issuing thread each
@@ -1166,7 +1212,12 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
     } else {
       // ---- chain group, state gradient (eq. 18): G_t = the prefix after this
       // tile (zero at the end of the sequence); G_t + Gd_t goes on to tile t-1
-      if (linked && gl == 0 && !flag_poll(f2, wnext, J.err)) gfail[1] = 1;
+      if (linked && gl == 0) {
+        if (early2 == wnext)
+          fence_acq_rel_gpu();
+        else if (!flag_poll(f2, wnext, J.err))
+          gfail[1] = 1;
+      }
       group_bar(2);
       if (gfail[1]) goto join2;
       float gs[C::MH][2][16], gzs[C::MH];
@@ -1227,7 +1278,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
       if (!mbar_wait(smem_u32(&mb[8]), 0, J.err)) abort_ = 1;
       tc_fence_after();
       __syncthreads();
-      if (abort_ | gfail[1]) goto teardown;
+      if (abort_ | gfail[0] | gfail[1]) goto teardown;
       // the partial joins the key side's in the dk/dv part (through L2)
       float* dqp = J.domq + tf * (size_t)(MF * 64);
       float v[16];
@@ -1253,6 +1304,7 @@ __device__ __forceinline__ void role_bwd_q(const BwdQJob& J, int b, uint8_t* sme
 
 // ================================================================== backward, dk/dv side
 struct BwdKVJob {
+  const CUtensorMap *tk, *tv, *tom;  // tensor maps (in the launch's parameters)
   const __nv_bfloat16 *Q, *K, *V, *dOut, *om16;
   // from the dq part of the same tile, indexed by (chain, tile) of a full slice
   const __nv_bfloat16* gS;   // [chains][ntf][MF][64] G_t(S)
@@ -1315,10 +1367,11 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     mbar_init(bar, 1);
     mbar_fence_init();
     fence_proxy_async_global();
-    mbar_expect_tx(bar, C::FEATB);
+    mbar_expect_tx(bar, C::FEATB + ROWT);
     bulk_load(smem_u32(sPhiK), img, C::FEATB, bar);
+    tma_load_3d(smem_u32(sV), J.tv, row0, c, bar);  // and the V tile
   }
-  // every other load at once: V, dout, G_t (lane-major -> its tile), tril(A)
+  // every other load at once: G_t (lane-major -> its tile), tril(A)
   // (lane-major -> its tile), the row statistics and g_t(z)
   if (row < valid) {
     const float* rsr = J.rowstat + (tf * T + row) * 2;
@@ -1326,7 +1379,6 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     dden = __ldcg(rsr + 1);
   }
   // (dnum = dout / den is still in its tile: the dq part left it there)
-  load_rows64(sV, T, J.V + g0, valid, tid, NTHR);
   load_lm_bf16(sG, MF, J.gS + tf * MF * 64, tid);
   {
     const uint8_t* imgA = img + C::FEATB;
@@ -1343,7 +1395,7 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     Sync sy{mb, 0, J.err};
     const bool live = rv && den != 0.f;
     if (!live) dden = 0.f;
-    if (!mbar_wait(smem_u32(&mb_img), 0, J.err)) abort_ = 1;  // phiK's tile
+    if (!mbar_wait(smem_u32(&mb_img), 0, J.err)) abort_ = 1;  // phiK's and V's tiles
     publish();
     if (abort_) goto teardown;
     // every thread has what it needs of the hand-off but the dOmega partial
@@ -1403,8 +1455,12 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
     }
     TC_WAIT(sy);
     // K and Omega again (dk = u Omega - k sum(u), dOmega += u^T k), overlapping the epilogue
-    load_rows64(sKr, T, J.K + g0, valid, tid, NTHR);
-    load_rows64(sOm, MF, J.om16, MF, tid, NTHR);
+    if (tid == 0) {
+      const uint32_t bar = smem_u32(&mb[MB_RELOAD]);
+      mbar_expect_tx(bar, ROWT + C::OMB);
+      tma_load_3d(smem_u32(sKr), J.tk, row0, c, bar);
+      tma_load_2d(smem_u32(sOm), J.tom, 0, bar);
+    }
     {
       // dphiK (+ g_z) -> u (into the phiQ tile), this thread's columns
       constexpr int W = MF / NG;
@@ -1443,8 +1499,9 @@ __device__ __forceinline__ void role_bwd_kv(const BwdKVJob& J, int t, int c, uin
       }
       redU[cg * T + row] = usum;
     }
-    cp_async_wait_all();
+    if (!mbar_wait(smem_u32(&mb[MB_RELOAD]), 0, J.err)) abort_ = 1;
     publish();
+    if (abort_) goto teardown;
     if (tid == 0) {
       const uint32_t aU = smem_u32(sU), aOm = smem_u32(sOm);
       for (int k0 = 0; k0 < MF; k0 += 16)
@@ -1704,6 +1761,7 @@ __host__ __device__ inline BwdItem sched_locate(const BwdSched& s, int x) {
 }
 
 struct BwdJob {
+  CUtensorMap tq, tk, tv, tdo, tom;  // see FwdJob; the parts point at these
   BwdSched s;
   BwdQJob q;   // slice fields set per item
   BwdKVJob kv;
@@ -1742,6 +1800,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
     uint8_t* hs = J.hand + slot * J.hand_slot;
     int* hf = J.hflag + (size_t)slot * tiles * FLAG_STRIDE;
     BwdQJob q = J.q;
+    q.tq = &J.tq;
+    q.tk = &J.tk;
+    q.tv = &J.tv;
+    q.tdo = &J.tdo;
+    q.tom = &J.tom;
     q.a = a;
     q.b = b;
     q.ntn = ntn;
@@ -1755,6 +1818,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_tc_bwd(const __grid_constant__ BwdJ
     q.ring = J.ring;
     q.nRtiles = n + J.ring < N ? (n + J.ring == N - 1 ? J.s.ntl : J.s.nt) : 0;
     BwdKVJob kv = J.kv;
+    kv.tk = &J.tk;
+    kv.tv = &J.tv;
+    kv.tom = &J.tom;
     kv.a = a;
     kv.b = b;
     kv.ntn = ntn;
@@ -1943,6 +2009,51 @@ cudaError_t configure() {
   return cudaSuccess;
 }
 
+// cuTensorMapEncodeTiled from the driver (through the runtime's entry-point
+// query, so the library needs no link against libcuda).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled() {
+  static const EncodeTiledFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      p = nullptr;
+    cudaGetLastError();
+    return reinterpret_cast<EncodeTiledFn>(p);
+  }();
+  return fn;
+}
+// [chains][L][64] bf16 rows, 128 bytes each: box {64, 128, 1} (one row tile),
+// 128-byte swizzle; rows at or past L read as zero.
+bool rows_map(CUtensorMap* m, const void* base, int chains, int L) {
+  const EncodeTiledFn fn = encode_tiled();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)L, (cuuint64_t)chains};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)L * D * 2};
+  const cuuint32_t box[3] = {(cuuint32_t)D, (cuuint32_t)T, 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+// Omega's bf16 hi rows then lo rows, [2 M][64]: box {64, M}.
+bool omega_map(CUtensorMap* m, const void* om16, int MF) {
+  const EncodeTiledFn fn = encode_tiled();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)2 * MF};
+  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)D, (cuuint32_t)MF};
+  const cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(om16), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 #define TC_TRY(x)                                  \
   do {                                             \
     cudaError_t e_ = (x);                          \
@@ -2001,12 +2112,16 @@ slim_status fwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   const Geo g = geometry(p);
   Carver cv(workspace);
   const Ws w = carve(cv, g, false);
-  TC_TRY(prepare(w, g, omega, rep, s));
   // every tile of every slice in one launch, in sequence order, chains inside
   // a tile position.  Algorithmic work per row: 8dM (phiQ, phiK, Delta, readout).
   const int P = (g.N - 1) * g.nt + slice_of(p, g, g.N - 1).nt;
-  const FwdJob J{q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flag1, w.ticket,
-                 out, st, init, w.err};
+  FwdJob J{{}, {}, {}, {}, q, k, v, w.om16, p.L, g.Cs, g.N, g.nt, P, g.chains, w.slot1, w.flag1,
+           w.ticket, out, st, init, w.err};
+  // the tensor maps first: a failure leaves nothing launched
+  if (!rows_map(&J.tq, q, g.chains, p.L) || !rows_map(&J.tk, k, g.chains, p.L) ||
+      !rows_map(&J.tv, v, g.chains, p.L) || !omega_map(&J.tom, w.om16, MF))
+    return SLIM_ERR_CUDA;
+  TC_TRY(prepare(w, g, omega, rep, s));
   const double rows = (double)g.chains * p.L, MD = (double)MF * D;
   prof::Scope ps(prof::K_TC_FWD, s, rows * 8.0 * MD, rows * D * 2.0 * 4);
   TC_TRY(launch_dep(k_tc_fwd<MF, FEAT>, dim3(P * g.chains), dim3(NTHR), smem_fwd<MF>(), s, J));
@@ -2034,8 +2149,13 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   Carver cv(workspace);
   const Ws w = carve(cv, g, true);
   const int N = g.N;
-  TC_TRY(prepare(w, g, omega, rep, s));
   BwdJob J{};
+  // the tensor maps first: a failure leaves nothing launched
+  if (!rows_map(&J.tq, q, g.chains, p.L) || !rows_map(&J.tk, k, g.chains, p.L) ||
+      !rows_map(&J.tv, v, g.chains, p.L) || !rows_map(&J.tdo, dout, g.chains, p.L) ||
+      !omega_map(&J.tom, w.om16, MF))
+    return SLIM_ERR_CUDA;
+  TC_TRY(prepare(w, g, omega, rep, s));
   J.s.N = N;
   J.s.chains = g.chains;
   J.s.nt = g.nt;
@@ -2044,10 +2164,10 @@ slim_status bwd_impl(const Problem& p, const __nv_bfloat16* q, const __nv_bfloat
   // slice 0 (C rows, or all L rows) has a tile at every position, so its
   // tiles close every dOmega sum
   // slice fields (a, b, ntn, n and the per-slice buffers) are set per item
-  J.q = BwdQJob{q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
+  J.q = BwdQJob{nullptr, nullptr, nullptr, nullptr, nullptr, q, k, v, out, dout, w.om16, st, p.L, 0, 0, 0, 0, N, g.nt, g.chains, w.slot1,
                 w.slot2, w.flag1, w.flag2, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                 0, 0, dq, w.err, gio};
-  J.kv = BwdKVJob{q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
+  J.kv = BwdKVJob{nullptr, nullptr, nullptr, q, k, v, dout, w.om16, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                   p.L, 0, 0, 0, g.nt, 0, dk, dv, nullptr, nullptr, 0, nullptr, w.err};
   J.red = RedJob{w.acc, g.chains * g.nt, w.rsums, J.s.r1n, J.s.r2n, domega, MF * D};
   J.L = p.L;
