@@ -12,6 +12,7 @@ Modules
   iterative  -- the token-by-token recurrence of App. B (C = 1)
   fd         -- central finite differences of <dY, Y>
   bidir      -- the non-causal form (no mask, one global state), two sweeps
+  stack      -- s residual layers, Algorithm 1 with one state per layer
 
 Library-facing wrappers below use the layout of the C ABI: q, k, v, dout are
 [B, H, L, d]; omega is [M, d]; the state is S_state = R^T ([B, H, M, d], the
@@ -25,7 +26,7 @@ function here is "parity unpinned".
 """
 import numpy as np
 
-from . import bidir, brute, features, fd, iterative, sliced  # noqa: F401
+from . import bidir, brute, features, fd, iterative, sliced, stack  # noqa: F401
 
 
 def _chains(x):
@@ -105,6 +106,32 @@ def oracle_bidir_bwd(q, k, v, omega, dout, S_state, z_state, C, feature):
     S = np.asarray(z_state, np.float64).reshape(B * H, M)
     dQ, dK, dV, dOmega, _ = bidir.backward(Q, K, V, Omega, dY, C, feature, R, S)
     return (dQ.reshape(B, H, L, d), dK.reshape(B, H, L, d), dV.reshape(B, H, L, d), dOmega)
+
+
+def oracle_stack_fwd(x, omegas, C, feature):
+    """Stack forward: x [B,H,L,d], omegas [s][M,d].  Returns y [B,H,L,d] and the
+    final states S_state [s][B,H,M,d], z_state [s][B,H,M]."""
+    X, (B, H) = _chains(x)
+    Oms = [np.asarray(o, dtype=np.float64) for o in omegas]
+    L, d = X.shape[1], X.shape[2]
+    Y, states = stack.forward(X, Oms, C, feature)
+    S = np.stack([np.swapaxes(R, 1, 2).reshape(B, H, Om.shape[0], d) for (R, _), Om in zip(states, Oms)])
+    z = np.stack([Sz.reshape(B, H, Om.shape[0]) for (_, Sz), Om in zip(states, Oms)])
+    return Y.reshape(B, H, L, d), S, z
+
+
+def oracle_stack_bwd(x, omegas, dy, S_state, z_state, C, feature):
+    """Stack backward from the final states.  Returns dx [B,H,L,d] and
+    domegas [s][M,d]."""
+    X, (B, H) = _chains(x)
+    dY, _ = _chains(dy)
+    Oms = [np.asarray(o, dtype=np.float64) for o in omegas]
+    L, d = X.shape[1], X.shape[2]
+    states = [(np.swapaxes(np.asarray(S_state[r], np.float64).reshape(B * H, Om.shape[0], d), 1, 2),
+               np.asarray(z_state[r], np.float64).reshape(B * H, Om.shape[0]))
+              for r, Om in enumerate(Oms)]
+    dX, dOm, _ = stack.backward(X, Oms, dY, C, feature, states)
+    return dX.reshape(B, H, L, d), np.stack(dOm)
 
 
 def rel_l2(a, b):

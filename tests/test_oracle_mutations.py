@@ -98,6 +98,16 @@ def _bidir_backward_drop_key_normaliser(Q, K, V, Omega, dY, C, feature, R, S):
 from oracle import bidir as _bidir  # noqa: E402
 _BIDIR_BACKWARD = _bidir.backward
 
+from oracle import stack as _stack  # noqa: E402
+_STACK_LAYER_BWD = _stack.layer_backward
+
+
+def _stack_layer_bwd_drops_residual(Q, K, V, Omega, dY, C, feature, R, S, G_R, G_S):
+    # mistake: the layer's gradient replaces dX instead of adding to it (the
+    # residual path dropped); planted as a layer backward that cancels dY
+    dq, dk, dv, dO, B0, G = _STACK_LAYER_BWD(Q, K, V, Omega, dY, C, feature, R, S, G_R, G_S)
+    return dq - dY, dk, dv, dO, B0, G
+
 MUTATIONS = {
     "exclusive_mask": (lambda mp: mp.setattr(sliced, "_forward_rows", _exclusive_forward_rows),
                        lambda: P.pin_brute_vs_sliced("exp"), 1e-6),
@@ -121,6 +131,9 @@ MUTATIONS = {
         lambda: P.pin_finite_differences("square"), 1e-3),
     "square_map_is_abs": (lambda mp: mp.setattr(features, "g_square", _g_abs),
                           lambda: P.pin_golden(), 1e-6),
+    "stack_residual_dropped": (
+        lambda mp: mp.setattr(_stack, "layer_backward", _stack_layer_bwd_drops_residual),
+        lambda: P.pin_stack_finite_differences("exp"), 1e-3),
     "bidir_key_grad_missing_normaliser": (
         lambda mp: mp.setattr(_bidir, "backward", _bidir_backward_drop_key_normaliser),
         lambda: P.pin_bidir_finite_differences("exp"), 1e-3),

@@ -461,3 +461,88 @@ def test_bidir_finite_differences(feature):
 
 def test_bidir_last_row_is_causal():
     assert pin_bidir_last_row_is_causal() < 1e-12
+
+
+# ----------------------------------------------------------------------------- the layer stack
+
+from oracle import stack  # noqa: E402
+
+
+def _stack_case(seed, s=3, chains=2, L=30, d=4, M=6, feature="exp"):
+    rng = np.random.default_rng(seed)
+    if feature == "square":
+        M = d
+    X = rng.standard_normal((chains, L, d)) * (0.5 if feature != "relu" else 1.0)
+    Oms = [rng.standard_normal((M, d)) for _ in range(s)]
+    dY = rng.standard_normal((chains, L, d))
+    return X, Oms, dY
+
+
+def pin_stack_quadratic_vs_sliced(feature, Cs=(1, 4, 7, 30, 64)):
+    """The stack layer by layer with the row-by-row definition of eq. 2 against
+    Algorithm 1's slice-outer, layer-inner sweep (one state per layer)."""
+    X, Oms, _ = _stack_case(24, feature=feature)
+    Yq = stack.quadratic(X, Oms, feature)
+    return max(rel(stack.forward(X, Oms, C, feature)[0], Yq) for C in Cs)
+
+
+def pin_stack_finite_differences(feature, C=3):
+    """Central differences of <dY, X^(s)> (the layer-by-layer definition) with
+    respect to X^(0) and every Omega_r, against the stack's backward sweep."""
+    X, Oms, dY = _stack_case(25, s=2, chains=1, L=6, d=3, M=4, feature=feature)
+    Y, states = stack.forward(X, Oms, C, feature)
+    dX, dOm, B0 = stack.backward(X, Oms, dY, C, feature, states)
+
+    def f():
+        return float(np.sum(dY * stack.quadratic(X, Oms, feature)))
+
+    h, worst = 1e-6, 0.0
+    for arr, got in [(X, dX)] + list(zip(Oms, dOm)):
+        fd = np.zeros_like(arr)
+        it = np.nditer(arr, flags=["multi_index"])
+        for _ in it:
+            i = it.multi_index
+            keep = arr[i]
+            arr[i] = keep + h
+            fp = f()
+            arr[i] = keep - h
+            fm = f()
+            arr[i] = keep
+            fd[i] = (fp - fm) / (2 * h)
+        worst = max(worst, rel(got, fd))
+    return worst
+
+
+def pin_stack_rollback_closes():
+    """After the reverse sweep every layer's state is rolled back to zero."""
+    X, Oms, dY = _stack_case(26)
+    _, states = stack.forward(X, Oms, 7, "exp")
+    _, _, B0 = stack.backward(X, Oms, dY, 7, "exp", states)
+    return max(max(np.abs(R).max() / np.abs(Rn).max(), np.abs(S).max() / np.abs(Sn).max())
+               for (R, S), (Rn, Sn) in zip(B0, states))
+
+
+def pin_stack_one_layer():
+    """s = 1 is one layer plus the residual: X^(1) = X + Att(X)."""
+    X, Oms, _ = _stack_case(27, s=1)
+    Y, _ = stack.forward(X, Oms, 5, "relu")
+    Yl, _, _ = sliced.forward(X, X, X, Oms[0], 5, "relu")
+    return rel(Y, X + Yl)
+
+
+@pytest.mark.parametrize("feature", ["exp", "relu", "square"])
+def test_stack_quadratic_vs_sliced(feature):
+    assert pin_stack_quadratic_vs_sliced(feature) < 1e-12
+
+
+@pytest.mark.parametrize("feature", ["exp", "square"])
+def test_stack_finite_differences(feature):
+    assert pin_stack_finite_differences(feature) < 1e-6
+
+
+def test_stack_rollback_closes():
+    assert pin_stack_rollback_closes() < 1e-11
+
+
+def test_stack_one_layer():
+    assert pin_stack_one_layer() < 1e-14
