@@ -75,8 +75,9 @@ def parse():
     ap.add_argument("--no-mem-curve", action="store_true")
     # what one step runs: the causal sweeps (default), the non-causal form, or
     # the causal sweeps over --segments chained calls (streaming)
-    ap.add_argument("--mode", choices=["causal", "bidir", "segments"], default="causal")
+    ap.add_argument("--mode", choices=["causal", "bidir", "segments", "stack"], default="causal")
     ap.add_argument("--segments", type=int, default=4)
+    ap.add_argument("--layers", type=int, default=3)
     return ap.parse_args()
 
 
@@ -279,7 +280,7 @@ def step_ceilings(w, B, H, L, ms_per_step):
 def _oracle_chain(args):
     """One chain's fp64 oracle fwd+bwd (runs in a spawned worker); the
     non-causal form for mode bidir, the causal sweeps otherwise."""
-    name, overrides, b, h, mode = args
+    name, overrides, b, h, mode, layers = args
     os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
     os.environ.setdefault("OMP_NUM_THREADS", "1")
     import oracle
@@ -287,6 +288,15 @@ def _oracle_chain(args):
     w = W.WORKLOADS[name].with_(**overrides)
     x = W.make_inputs(w)
     c = {n: W.as_float64_numpy(t[b:b + 1, h:h + 1] if t.dim() == 4 else t) for n, t in x.items()}
+    if mode == "stack":
+        xs = W.make_stack_inputs(w, layers)
+        sx = W.as_float64_numpy(xs["x"][b:b + 1, h:h + 1])
+        sdy = W.as_float64_numpy(xs["dy"][b:b + 1, h:h + 1])
+        oms = list(W.as_float64_numpy(xs["omegas"]))
+        t0 = time.perf_counter()
+        y, S, z = oracle.oracle_stack_fwd(sx, oms, w.C, w.feature)
+        oracle.oracle_stack_bwd(sx, oms, sdy, S, z, w.C, w.feature)
+        return time.perf_counter() - t0
     t0 = time.perf_counter()
     if mode == "bidir":
         o, S, z = oracle.oracle_bidir_fwd(c["q"], c["k"], c["v"], c["omega"], w.C, w.feature)
@@ -322,10 +332,10 @@ def start_oracle_pool(n):
     return pool
 
 
-def oracle_sample(w, overrides, pool, nchains, mode="causal"):
+def oracle_sample(w, overrides, pool, nchains, mode="causal", layers=3):
     """Runs nchains chains of the workload through the oracle in parallel;
     returns (tokens, wall seconds)."""
-    jobs = [(w.name, overrides, (i // w.H) % w.B, i % w.H, mode) for i in range(nchains)]
+    jobs = [(w.name, overrides, (i // w.H) % w.B, i % w.H, mode, layers) for i in range(nchains)]
     secs = pool.map(_oracle_chain, jobs)
     # the chains run side by side; input generation is outside each worker's clock
     return nchains * w.L, max(secs)
@@ -339,7 +349,7 @@ class StepSet:
     forwards chained through slim_fwd_from and the backwards, last segment
     first, through slim_bwd_from (each hands G^(0) to the one before)."""
 
-    def __init__(self, w, dev, mode, segments, x=None):
+    def __init__(self, w, dev, mode, segments, x=None, layers=3):
         import torch
         from paper_2012_11346_gb300 import slim
         from paper_2012_11346_gb300 import workloads as W
@@ -349,6 +359,24 @@ class StepSet:
         q = self.x["q"]
         f32 = torch.float32
         self.om = None if w.feature == "square" else self.x["omega"]
+        if mode == "stack":
+            # s residual layers by Algorithm 1: x, per-layer Omegas, dy
+            self.layers = layers
+            self.sx = W.make_stack_inputs(w, layers, device=dev)
+            self.soms = None if w.feature == "square" else self.sx["omegas"]
+            B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
+            self.y = torch.empty_like(self.sx["x"])
+            self.dx = torch.empty_like(self.sx["x"])
+            self.sS = torch.empty(layers, B, H, M, d, dtype=f32, device=dev)
+            self.sz = torch.empty(layers, B, H, M, dtype=f32, device=dev)
+            self.sSl, self.szl = torch.empty_like(self.sS), torch.empty_like(self.sz)
+            self.sdom = torch.empty(layers, M, d, dtype=f32, device=dev)
+            size = slim.stack_workspace_size
+            self.ws_f = self._ws(size(B, H, L, d, M, w.C, layers, q.dtype, w.feature, False), dev)
+            self.ws_b = self._ws(size(B, H, L, d, M, w.C, layers, q.dtype, w.feature, True), dev)
+            self.outputs = [self.y, self.dx, self.sdom]
+            self.inputs = [self.sx["x"], self.sx["dy"], self.sx["omegas"]]
+            return
         if mode == "segments":
             cuts = [round(i * L / segments) for i in range(segments + 1)]
             self.segs = []
@@ -411,6 +439,24 @@ class StepSet:
             sl.backward_bidir_into(x["q"], x["k"], x["v"], om, self.out, x["dout"], self.S,
                                    self.z, C, f, self.dq, self.dk, self.dv, self.dom, self.ws_b,
                                    stream)
+        elif self.mode == "stack":
+            lib, ls, sx = sl.library(), self.layers, self.sx
+            dt, ft = sl.DTYPES[sx["x"].dtype], sl.FEATURES[f]
+            B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
+            h = sl._stream_handle(stream)
+            sl._check(lib.slim_stack_fwd(sx["x"].data_ptr(), sl._ptr(self.soms), B, H, L, d, M, C,
+                                         ls, dt, ft, self.y.data_ptr(), self.sS.data_ptr(),
+                                         self.sz.data_ptr(), self.sSl.data_ptr(),
+                                         self.szl.data_ptr(), self.ws_f.data_ptr(),
+                                         self.ws_f.numel(), h), "slim_stack_fwd")
+            sl._check(lib.slim_stack_bwd(sx["x"].data_ptr(), sl._ptr(self.soms),
+                                         sx["dy"].data_ptr(), self.sS.data_ptr(),
+                                         self.sz.data_ptr(), self.sSl.data_ptr(),
+                                         self.szl.data_ptr(), B, H, L, d, M, C, ls, dt, ft,
+                                         self.dx.data_ptr(),
+                                         sl._ptr(self.sdom if self.soms is not None else None),
+                                         self.ws_b.data_ptr(), self.ws_b.numel(), h),
+                      "slim_stack_bwd")
         else:
             prev = None
             for sg in self.segs:
@@ -558,7 +604,7 @@ def run_ours(args, rank, ws, local):
     if args.H:
         w = w.with_(H=args.H)
     B, H, L, d, M = w.B, w.H, w.L, w.d, w.M
-    main = StepSet(w, dev, args.mode, args.segments)
+    main = StepSet(w, dev, args.mode, args.segments, layers=args.layers)
     step = main.run
 
     for _ in range(args.warmup):
@@ -611,7 +657,7 @@ def run_ours(args, rank, ws, local):
 
     # end to end through the public API: pinned host inputs in, results out,
     # copies overlapped with the neighbouring steps' compute (two buffer sets)
-    second = StepSet(w, dev, args.mode, args.segments, x=None)
+    second = StepSet(w, dev, args.mode, args.segments, x=None, layers=args.layers)
     sets = [main, second]
     host_in = [[t.cpu().pin_memory() for t in st.inputs] for st in sets]
     host_out = [[torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in st.outputs]
@@ -647,6 +693,7 @@ def run_ours(args, rank, ws, local):
         "config": {"workload": w.name, "B": B, "H": H, "L": L, "d": d, "M": M, "C": w.C,
                    "feature": w.feature, "input_dtype": w.dtype, "mode": args.mode,
                    **({"segments": args.segments} if args.mode == "segments" else {}),
+                   **({"layers": args.layers} if args.mode == "stack" else {}),
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
                    "l2": "no flush; per-step working set (q,k,v,dout,out,dq,dk,dv) "
                          f"{8 * main.x['q'].numel() * main.x['q'].element_size() / 2**20:.0f} MiB "
@@ -676,7 +723,7 @@ def run_ours(args, rank, ws, local):
         # inherit the parent's CUDA context.
         n = oracle_pool_size()
         pool = start_oracle_pool(n)
-        tok, sec = oracle_sample(w, {"C": w.C}, pool, n, args.mode)
+        tok, sec = oracle_sample(w, {"C": w.C}, pool, n, args.mode, args.layers)
         line["cpu_baseline"] = {"value": round(tok / sec, 2), "unit": "tokens/s", "cores": n,
                                 "kind": "oracle",
                                 "sample": f"{n} chains x L={L} of this workload, fp64 NumPy, "
@@ -709,10 +756,10 @@ def run_reference(args, rank, ws):
     n = oracle_pool_size()
     with mp.get_context("spawn").Pool(n) as pool:
         for _ in range(args.warmup):
-            oracle_sample(w, {"C": w.C}, pool, n, args.mode)
+            oracle_sample(w, {"C": w.C}, pool, n, args.mode, args.layers)
         tok, sec = 0, 0.0
         for _ in range(args.steps):
-            t, s = oracle_sample(w, {"C": w.C}, pool, n, args.mode)
+            t, s = oracle_sample(w, {"C": w.C}, pool, n, args.mode, args.layers)
             tok += t
             sec += s
     value = tok / sec

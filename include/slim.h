@@ -55,6 +55,8 @@
  *     first kernel stores the counter's address in the workspace, so the
  *     report adds no copy and no launch.  slim_check_device_error reads the
  *     same failure by blocking instead.
+ *   - A workspace's first 4 bytes are its device error word.  Every call
+ *     clears it when it starts; a bounded wait that gives up sets it.
  *   - 1 <= C; C > L behaves as C = L.  L % C != 0 gives a shorter last slice.
  *   - Outputs are written in `dtype` rounded to nearest even.  The state
  *     carried between slices depends on the kernels serving the problem (see
@@ -245,6 +247,53 @@ slim_status slim_bwd_bidir(const void* q, const void* k, const void* v, const fl
                            int B, int H, int L, int d, int M, int C,
                            slim_dtype dtype, slim_feature feature,
                            void* dq, void* dk, void* dv, float* domega,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * A stack of `layers` (s) causal linear-attention layers with residual
+ * connections, run the memory-efficient way of Algorithm 1 (Sec. 3.2-3.3):
+ * the slices in the outer loop, the layers in the inner loop, one carried
+ * state per layer (B is s x D1), and the reverse sweep of Algorithm 2 with a
+ * rollback (eq. 17) and a state gradient (eq. 18) per layer.  Layer r maps
+ * each row x of its input to q = k = v = u(x) = d^(-1/4) x / sqrt(mean(x^2)
+ * + 1e-6) -- a parameter-free row normalisation standing in for the layer
+ * norm of the paper's model (Sec. 2.2, eqs. 5-6), keeping every layer's features at the scale of
+ * one layer's inputs -- runs attention with its own random-feature matrix
+ * Omega_r (the F of Sec. 3.1) and adds its output back (the G):
+ *     X^(r) = X^(r-1) + Att_r(u, u, u),   r = 1..s,   out: X^(s).
+ * Each (slice, layer) step runs as one slim_fwd_from / slim_bwd_from call on
+ * the slice's rows, gathered into the workspace.  Memory beyond inputs and
+ * outputs: one slice's activations per layer, the per-layer states and state
+ * gradients, and one segment call's workspace (O(C * s), not O(L)).
+ *   x          [B,H,L,d] dtype: X^(0).  y: [B,H,L,d] dtype, written: X^(s).
+ *   omegas     [layers][M][d] fp32 (may be NULL for the quadratic map).
+ *   S_state, z_state  [layers][B,H,M,d], [layers][B,H,M] fp32: written by
+ *              slim_stack_fwd (each layer's final state), read by
+ *              slim_stack_bwd; S_state_lo / z_state_lo the residuals (both or
+ *              neither), as for slim_fwd.
+ *   dy         [B,H,L,d] dtype: the upstream gradient of X^(s).
+ *   dx         [B,H,L,d] dtype, written: the gradient of <dy, X^(s)> w.r.t. x.
+ *   domegas    [layers][M][d] fp32, written (NULL allowed for the quadratic map).
+ *   layers     1 .. 64.  Workspace: slim_stack_workspace_size (backward != 0
+ *              for slim_stack_bwd), 256-byte aligned; its first word is the
+ *              device error word, as for slim_fwd.
+ * Errors as for slim_fwd / slim_bwd.
+ */
+slim_status slim_stack_workspace_size(int B, int H, int L, int d, int M, int C, int layers,
+                                      slim_dtype dtype, slim_feature feature, int backward,
+                                      size_t* bytes);
+slim_status slim_stack_fwd(const void* x, const float* omegas,
+                           int B, int H, int L, int d, int M, int C, int layers,
+                           slim_dtype dtype, slim_feature feature,
+                           void* y, float* S_state, float* z_state,
+                           float* S_state_lo, float* z_state_lo,
+                           void* workspace, size_t workspace_bytes, void* stream);
+slim_status slim_stack_bwd(const void* x, const float* omegas, const void* dy,
+                           const float* S_state, const float* z_state,
+                           const float* S_state_lo, const float* z_state_lo,
+                           int B, int H, int L, int d, int M, int C, int layers,
+                           slim_dtype dtype, slim_feature feature,
+                           void* dx, float* domegas,
                            void* workspace, size_t workspace_bytes, void* stream);
 
 /*

@@ -3,12 +3,18 @@ way of Algorithm 1, fp64.
 
 ORACLE -- test infrastructure only; see oracle/__init__.py.
 
-Layer r (r = 1..s) maps the rows of its input X^(r-1) row-wise to a query, a
-key and a value -- here all three are X^(r-1) itself, with the layer's own
-random-feature matrix Omega_r -- runs the causal linear attention of eq. 2 on
-them, and adds the result back (a residual connection):
+Layer r (r = 1..s) maps each row of its input X^(r-1) to a query, a key and a
+value -- all three the row normalised to a fixed root-mean-square,
 
-    X^(r) = X^(r-1) + Att_r(X^(r-1), X^(r-1), X^(r-1)),     r = 1..s.
+    u = d^(-1/4) x / sqrt(mean_i x_i^2 + eps),       q = k = v = u,
+
+a parameter-free stand-in for the row-wise layer normalisation of the paper's
+model (Sec. 2.2, eqs. 5-6) that keeps every layer's features at the scale of the
+single-layer inputs -- runs the causal linear attention of eq. 2 on them with
+its own random-feature matrix Omega_r, and adds the result back (a residual
+connection):
+
+    X^(r) = X^(r-1) + Att_r(u(X^(r-1)), u(X^(r-1)), u(X^(r-1))),   r = 1..s.
 
 That is the F / prefix sum / G split of Sec. 3.1 (eqs. 11-13) with F^(r)
 computing T = (V g(K)^T, g(K)) and Gamma = g(Q) from the row, and G^(r) the
@@ -27,7 +33,8 @@ loop (Algorithm 2):
       and recompute layer r's output;
       then for r = s..1: the slice's gradients of layer r from its saved input,
       its final state B_r^(n) and G_r; G_r := the gradient with respect to
-      B_r^(n-1); dX^(r-1) = dX^(r) + dq + dk + dv (the residual, and q = k = v).
+      B_r^(n-1); dX^(r-1) = dX^(r) + u'(X^(r-1))^T (dq + dk + dv) (the residual,
+      and q = k = v = u(X^(r-1))).
 Only the s states, their gradients and one slice's activations are kept:
 O(C) memory besides the input (Sec. 3.4).
 
@@ -40,13 +47,31 @@ from .sliced import backward as layer_backward
 from .sliced import forward as layer_forward
 from .sliced import slices
 
+EPS = 1e-6
+
+
+def row_norm(X):
+    """u = d^(-1/4) x / sqrt(mean(x^2) + eps), row by row."""
+    d = X.shape[-1]
+    r = np.sqrt(np.mean(X * X, axis=-1, keepdims=True) + EPS)
+    return d ** -0.25 * X / r
+
+
+def row_norm_vjp(X, g):
+    """Cotangent g of u = row_norm(x) pulled back to x:
+    dx = (s / r) (g - x mean(g x) / r^2), s = d^(-1/4)."""
+    d = X.shape[-1]
+    r = np.sqrt(np.mean(X * X, axis=-1, keepdims=True) + EPS)
+    return d ** -0.25 / r * (g - X * np.mean(g * X, axis=-1, keepdims=True) / (r * r))
+
 
 def quadratic(X0, Omegas, feature):
     """The stack layer by layer over the whole sequence, each layer by the
     row-by-row definition of eq. 2 (tiny inputs)."""
     X = np.array(X0, dtype=np.float64)
     for Om in Omegas:
-        X = X + brute.att_lin_quadratic(X, X, X, Om, feature)
+        U = row_norm(X)
+        X = X + brute.att_lin_quadratic(U, U, U, Om, feature)
     return X
 
 
@@ -60,7 +85,8 @@ def forward(X0, Omegas, C, feature):
         X = np.array(X0[:, a:e], dtype=np.float64)
         for r, Om in enumerate(Omegas):
             R, S = states[r]
-            out, R, S = layer_forward(X, X, X, Om, e - a, feature, R, S)
+            U = row_norm(X)
+            out, R, S = layer_forward(U, U, U, Om, e - a, feature, R, S)
             states[r] = (R, S)
             X = X + out
         Y[:, a:e] = X
@@ -83,20 +109,22 @@ def backward(X0, Omegas, dY, C, feature, states):
         X = np.array(X0[:, a:e], dtype=np.float64)
         for r, Om in enumerate(Omegas):
             R_end, S_end = B[r]
+            U = row_norm(X)
             # the slice's own contribution, sum of T_l over its rows
-            _, dR, dS = layer_forward(X, X, X, Om, e - a, feature)
+            _, dR, dS = layer_forward(U, U, U, Om, e - a, feature)
             B[r] = (R_end - dR, S_end - dS)
-            out, _, _ = layer_forward(X, X, X, Om, e - a, feature, B[r][0], B[r][1])
+            out, _, _ = layer_forward(U, U, U, Om, e - a, feature, B[r][0], B[r][1])
             ins.append(X)
             ends.append((R_end, S_end))
             X = X + out
-        # back through the layers: the residual passes dX on, q = k = v = X
+        # back through the layers: the residual passes dX on; q = k = v = u(X)
         dX = np.array(dY[:, a:e], dtype=np.float64)
         for r in reversed(range(s)):
             Xr = ins[r]
-            dq, dk, dv, dO, _, G[r] = layer_backward(Xr, Xr, Xr, Omegas[r], dX, e - a, feature,
+            U = row_norm(Xr)
+            dq, dk, dv, dO, _, G[r] = layer_backward(U, U, U, Omegas[r], dX, e - a, feature,
                                                      ends[r][0], ends[r][1], G[r][0], G[r][1])
             dOm[r] += dO
-            dX = dX + dq + dk + dv
+            dX = dX + row_norm_vjp(Xr, dq + dk + dv)
         dX0[:, a:e] = dX
     return dX0, dOm, B

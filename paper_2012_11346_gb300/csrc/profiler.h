@@ -25,6 +25,7 @@ enum Kid {
   K_TC_REDUCE,
   K_TC_SELFTEST,
   K_TC_PREP,
+  K_STACK,
   K_COUNT
 };
 

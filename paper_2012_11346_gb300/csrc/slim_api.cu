@@ -7,6 +7,7 @@
 #include "common.cuh"
 #include "report.h"
 #include "simt_path.h"
+#include "stack.h"
 #include "tc_path.h"
 
 using slim::Problem;
@@ -328,6 +329,82 @@ slim_status slim_bwd_bidir(const void* q, const void* k, const void* v, const fl
   return slim::simt::bwd_bidir(p, q, k, v, omega, out, dout,
                                slim::StateIn{S_state, z_state, nullptr, nullptr}, dq, dk, dv,
                                domega, workspace, s);
+}
+
+slim_status slim_stack_workspace_size(int B, int H, int L, int d, int M, int C, int layers,
+                                      slim_dtype dtype, slim_feature feature, int backward,
+                                      size_t* bytes) {
+  if (!bytes || layers < 1 || layers > 64) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  *bytes = L == 0 ? 0 : slim::stack::workspace_bytes(p, layers, backward != 0);
+  return SLIM_OK;
+}
+
+slim_status slim_stack_fwd(const void* x, const float* omegas, int B, int H, int L, int d,
+                           int M, int C, int layers, slim_dtype dtype, slim_feature feature,
+                           void* y, float* S_state, float* z_state, float* S_state_lo,
+                           float* z_state_lo, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  if (layers < 1 || layers > 64) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  const void* seq[] = {x, y};
+  const void* fixed[] = {S_state, z_state};
+  const void* opt[] = {S_state_lo, z_state_lo, omegas};
+  if (!pointers_ok(seq, 2, L == 0) || !pointers_ok(fixed, 2, false) || !pointers_ok(opt, 3, true))
+    return SLIM_ERR_INVALID_ARG;
+  if (omegas == nullptr && feature != SLIM_FEAT_SQUARE) return SLIM_ERR_INVALID_ARG;
+  if (!pair_ok(S_state_lo, z_state_lo)) return SLIM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n = (size_t)layers * p.chains() * M;
+  if (L == 0) {
+    if (cudaMemsetAsync(S_state, 0, n * d * 4, s) != cudaSuccess ||
+        cudaMemsetAsync(z_state, 0, n * 4, s) != cudaSuccess ||
+        (S_state_lo && cudaMemsetAsync(S_state_lo, 0, n * d * 4, s) != cudaSuccess) ||
+        (z_state_lo && cudaMemsetAsync(z_state_lo, 0, n * 4, s) != cudaSuccess))
+      return SLIM_ERR_CUDA;
+    return SLIM_OK;
+  }
+  const size_t need = slim::stack::workspace_bytes(p, layers, false);
+  if (workspace == nullptr || workspace_bytes < need) return SLIM_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SLIM_ERR_INVALID_ARG;
+  return slim::stack::fwd(p, layers, x, omegas, y, S_state, z_state, S_state_lo, z_state_lo,
+                          workspace, s);
+}
+
+slim_status slim_stack_bwd(const void* x, const float* omegas, const void* dy,
+                           const float* S_state, const float* z_state, const float* S_state_lo,
+                           const float* z_state_lo, int B, int H, int L, int d, int M, int C,
+                           int layers, slim_dtype dtype, slim_feature feature, void* dx,
+                           float* domegas, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  if (layers < 1 || layers > 64) return SLIM_ERR_INVALID_ARG;
+  Problem p;
+  slim_status st = check_problem(B, H, L, d, M, C, dtype, feature, &p);
+  if (st != SLIM_OK) return st;
+  const void* seq[] = {x, dy, dx};
+  const void* fixed[] = {S_state, z_state};
+  const void* opt[] = {S_state_lo, z_state_lo, omegas, domegas};
+  if (!pointers_ok(seq, 3, L == 0) || !pointers_ok(fixed, 2, false) || !pointers_ok(opt, 4, true))
+    return SLIM_ERR_INVALID_ARG;
+  if ((omegas == nullptr || domegas == nullptr) && feature != SLIM_FEAT_SQUARE)
+    return SLIM_ERR_INVALID_ARG;
+  if (!pair_ok(S_state_lo, z_state_lo)) return SLIM_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (L == 0) {
+    if (domegas &&
+        cudaMemsetAsync(domegas, 0, (size_t)layers * M * d * 4, s) != cudaSuccess)
+      return SLIM_ERR_CUDA;
+    return SLIM_OK;
+  }
+  const size_t need = slim::stack::workspace_bytes(p, layers, true);
+  if (workspace == nullptr || workspace_bytes < need) return SLIM_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SLIM_ERR_INVALID_ARG;
+  return slim::stack::bwd(p, layers, x, omegas, dy, S_state, z_state, S_state_lo, z_state_lo, dx,
+                          domegas, workspace, s);
 }
 
 slim_status slim_path_for(int B, int H, int L, int d, int M, int C, slim_dtype dtype,

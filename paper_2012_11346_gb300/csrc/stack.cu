@@ -1,0 +1,403 @@
+// A stack of s residual causal linear-attention layers run the memory-efficient
+// way of Algorithm 1: slices in the outer loop, layers in the inner loop, one
+// carried state per layer (the s rows of B in Sec. 3.2), and the reverse sweep
+// of Algorithm 2 with a per-layer rollback (eq. 17) and state gradient (eq. 18).
+//
+// Layer r maps each row of its input X^(r-1) to q = k = v = u, the row scaled
+// to a root-mean-square of d^(-1/4) (u = d^(-1/4) x / sqrt(mean(x^2) + eps), a
+// parameter-free row normalisation in place of the layer norm of the paper's
+// model, Sec. 2.2 eqs. 5-6), runs attention with its own Omega_r and adds the output
+// back: X^(r) = X^(r-1) + Att_r(u, u, u).
+// Each (slice, layer) step is one call of the segment entry points
+// (slim_fwd_from / slim_bwd_from) on the slice's rows, gathered into a
+// contiguous buffer, so the work runs in the same kernels as a single layer.
+// Memory beyond inputs and outputs: one slice's activations per layer, the
+// per-layer states and state gradients, and one call's workspace -- O(C), not
+// O(L) (Sec. 3.4).
+#include <stdint.h>
+#include <string.h>
+
+#include "common.cuh"
+#include "profiler.h"
+#include "stack.h"
+
+namespace slim {
+namespace stack {
+namespace {
+
+// rows [a, a+b) of every chain of a [chains][L][d] tensor <-> [chains][b][d]
+template <typename T>
+__global__ void k_gather(const T* src, T* dst, int L, int d, int a, int b, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const long long per = (long long)b * d;
+  const long long c = i / per, r = i % per;
+  dst[i] = src[((size_t)c * L + a) * d + r];
+}
+template <typename T>
+__global__ void k_scatter(const T* src, T* dst, int L, int d, int a, int b, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const long long per = (long long)b * d;
+  const long long c = i / per, r = i % per;
+  dst[((size_t)c * L + a) * d + r] = src[i];
+}
+// out = x + y (the residual connection), in fp32, rounded to the dtype
+template <typename T>
+__global__ void k_residual(const T* x, const T* y, T* out, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) Io<T>::store(out, i, Io<T>::load(x, i) + Io<T>::load(y, i));
+}
+// (hi, lo) -= (dhi, dlo): the rollback of eq. 17 on an fp32 value/error pair
+__global__ void k_pair_sub(float* hi, float* lo, const float* dhi, const float* dlo, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  float h = hi[i], l = lo[i];
+  pair_add(h, l, -dhi[i]);
+  pair_add(h, l, -dlo[i]);
+  hi[i] = h;
+  lo[i] = l;
+}
+constexpr float kNormEps = 1e-6f;
+constexpr int kRowsPerBlock = 8;  // one warp per row
+
+__device__ float warp_sum(float v) {
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// u = scale * x / sqrt(mean(x^2) + eps) row by row, scale = d^(-1/4)
+template <typename T>
+__global__ void k_rownorm(const T* x, T* u, int d, float scale, long long rows) {
+  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const T* xr = x + row * d;
+  float ss = 0.f;
+  for (int j = lane; j < d; j += 32) {
+    const float v = Io<T>::load(xr, j);
+    ss += v * v;
+  }
+  const float inv = scale / sqrtf(warp_sum(ss) / d + kNormEps);
+  for (int j = lane; j < d; j += 32) Io<T>::store(u + row * d, j, Io<T>::load(xr, j) * inv);
+}
+
+// dX (fp32) += u'(x)^T g with g = dq + dk + dv (q = k = v = u(x)):
+//   dx += (scale / r) (g - x mean(g x) / r^2),  r = sqrt(mean(x^2) + eps),
+// and the next layer down's upstream gradient (the new dX) as the dtype
+template <typename T>
+__global__ void k_dx_accum(float* dx, const T* x, const T* dq, const T* dk, const T* dv, T* dout,
+                           int d, float scale, long long rows) {
+  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const size_t o = (size_t)row * d;
+  float ss = 0.f, gx = 0.f;
+  for (int j = lane; j < d; j += 32) {
+    const float xv = Io<T>::load(x, o + j);
+    const float g = Io<T>::load(dq, o + j) + Io<T>::load(dk, o + j) + Io<T>::load(dv, o + j);
+    ss += xv * xv;
+    gx += g * xv;
+  }
+  const float r2 = warp_sum(ss) / d + kNormEps;
+  const float m = warp_sum(gx) / d / r2;
+  const float f = scale / sqrtf(r2);
+  for (int j = lane; j < d; j += 32) {
+    const float xv = Io<T>::load(x, o + j);
+    const float g = Io<T>::load(dq, o + j) + Io<T>::load(dk, o + j) + Io<T>::load(dv, o + j);
+    const float v = dx[o + j] + f * (g - xv * m);
+    dx[o + j] = v;
+    Io<T>::store(dout, o + j, v);
+  }
+}
+// the slice's dY into the fp32 accumulator and the top layer's dout
+template <typename T>
+__global__ void k_dy_in(const T* dy, float* dx, T* dout, int L, int d, int a, int b, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const long long per = (long long)b * d;
+  const long long c = i / per, r = i % per;
+  const T v = dy[((size_t)c * L + a) * d + r];
+  dx[i] = Io<T>::load(&v, 0);
+  dout[i] = v;
+}
+// accumulated fp32 dX back to the dtype, rows [a, a+b) of every chain
+template <typename T>
+__global__ void k_dx_out(const float* dx, T* dst, int L, int d, int a, int b, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const long long per = (long long)b * d;
+  const long long c = i / per, r = i % per;
+  Io<T>::store(dst, ((size_t)c * L + a) * d + r, dx[i]);
+}
+__global__ void k_add(float* acc, const float* x, long long n) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) acc[i] += x[i];
+}
+
+unsigned nb(long long n) { return (unsigned)((n + 255) / 256); }
+unsigned nrb(long long rows) { return (unsigned)((rows + kRowsPerBlock - 1) / kRowsPerBlock); }
+// every launch of this file is counted (and timed when the profiler is on)
+#define STACK_LAUNCH(...)                           \
+  do {                                              \
+    prof::Scope ps_(prof::K_STACK, s);              \
+    __VA_ARGS__;                                    \
+  } while (0)
+
+struct Geo {
+  int chains, Cs, N, s;
+  size_t rows;   // chains * Cs: elements of a slice buffer / d
+  size_t st;     // chains * M * d, state elements
+  size_t zt;     // chains * M
+  size_t esz;    // dtype bytes
+  size_t inner;  // workspace of one segment call
+};
+
+struct Ws {
+  uint8_t** xin;  // [s + 1] slice inputs of each layer, then the top's output
+  uint8_t** yout; // [s] layer outputs on the slice
+  float *Sb, *zb, *Slb, *zlb;   // [s] running states (backward), value/error pairs
+  float *Se, *ze, *Sle, *zle;   // [s] states at the slice's end (backward)
+  float *dS, *dz, *dSl, *dzl;   // one slice's own contribution (rollback)
+  float *G, *gz, *G2, *gz2;     // [s] state gradients, double-buffered
+  float *dx;                    // fp32 dX of the slice
+  uint8_t *dout, *dq, *dk, *dv, *scratch_y;
+  uint8_t* u;                   // the normalised rows of one layer's slice input
+  float* dom;                   // one call's dOmega
+  float *Ssc, *zsc;             // a recompute's end state, not needed
+  void* inner;
+};
+
+size_t inner_bytes(const Problem& p, int Cs) {
+  size_t f = 0, b = 0;
+  slim_fwd_workspace_size(p.B, p.H, Cs, p.d, p.M, Cs, p.dtype, p.feature, &f);
+  slim_bwd_workspace_size(p.B, p.H, Cs, p.d, p.M, Cs, p.dtype, p.feature, &b);
+  return f > b ? f : b;
+}
+
+Ws carve(Carver& cv, const Problem& p, const Geo& g, bool bwd, uint8_t** xin_ptrs,
+         uint8_t** y_ptrs) {
+  Ws w{};
+  const size_t sb = g.rows * p.d * g.esz;
+  // the segment calls' workspace first: its error word is then the stack
+  // workspace's first word, where slim_check_device_error reads it
+  w.inner = cv.take<uint8_t>(g.inner);
+  w.xin = xin_ptrs;
+  w.yout = y_ptrs;
+  for (int r = 0; r <= (bwd ? g.s : 1); ++r) xin_ptrs[r] = cv.take<uint8_t>(sb);
+  if (bwd) {
+    for (int r = 0; r < g.s; ++r) y_ptrs[r] = cv.take<uint8_t>(sb);
+    const size_t S = g.s * g.st, Z = g.s * g.zt;
+    w.Sb = cv.take<float>(S); w.zb = cv.take<float>(Z);
+    w.Slb = cv.take<float>(S); w.zlb = cv.take<float>(Z);
+    w.Se = cv.take<float>(S); w.ze = cv.take<float>(Z);
+    w.Sle = cv.take<float>(S); w.zle = cv.take<float>(Z);
+    w.dS = cv.take<float>(g.st); w.dz = cv.take<float>(g.zt);
+    w.dSl = cv.take<float>(g.st); w.dzl = cv.take<float>(g.zt);
+    w.G = cv.take<float>(S); w.gz = cv.take<float>(Z);
+    w.G2 = cv.take<float>(S); w.gz2 = cv.take<float>(Z);
+    w.dx = cv.take<float>(g.rows * p.d);
+    w.dout = cv.take<uint8_t>(sb);
+    w.dq = cv.take<uint8_t>(sb);
+    w.dk = cv.take<uint8_t>(sb);
+    w.dv = cv.take<uint8_t>(sb);
+    w.scratch_y = cv.take<uint8_t>(sb);
+    w.dom = cv.take<float>((size_t)p.M * p.d);
+    w.Ssc = cv.take<float>(g.st);
+    w.zsc = cv.take<float>(g.zt);
+  } else {
+    y_ptrs[0] = cv.take<uint8_t>(sb);
+  }
+  w.u = cv.take<uint8_t>(sb);
+  return w;
+}
+
+Geo geometry(const Problem& p, int layers) {
+  Geo g;
+  g.chains = p.chains();
+  g.Cs = p.slice_len();
+  g.N = p.num_slices();
+  g.s = layers;
+  g.rows = (size_t)g.chains * g.Cs;
+  g.st = (size_t)g.chains * p.M * p.d;
+  g.zt = (size_t)g.chains * p.M;
+  g.esz = p.dtype == SLIM_BF16 ? 2 : 4;
+  g.inner = inner_bytes(p, g.Cs);
+  return g;
+}
+
+#define ST_TRY(x)                                \
+  do {                                           \
+    cudaError_t e_ = (x);                        \
+    if (e_ != cudaSuccess) return SLIM_ERR_CUDA; \
+  } while (0)
+#define ST_CALL(x)                               \
+  do {                                           \
+    slim_status s_ = (x);                        \
+    if (s_ != SLIM_OK) return s_;                \
+  } while (0)
+
+template <typename T>
+slim_status fwd_impl(const Problem& p, int layers, const T* x, const float* omegas, T* y,
+                     float* S_state, float* z_state, float* S_lo, float* z_lo, void* workspace,
+                     cudaStream_t s) {
+  const Geo g = geometry(p, layers);
+  Carver cv(workspace);
+  uint8_t* xin[65];
+  uint8_t* yo[64];
+  const Ws w = carve(cv, p, g, false, xin, yo);
+  const int d = p.d, M = p.M;
+  const float scale = powf((float)d, -0.25f);
+  T* U = reinterpret_cast<T*>(w.u);
+  for (int n = 0; n < g.N; ++n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    const long long cnt = (long long)g.chains * b * d, rows = (long long)g.chains * b;
+    T* X = reinterpret_cast<T*>(w.xin[0]);
+    T* X2 = reinterpret_cast<T*>(w.xin[1]);
+    T* Y = reinterpret_cast<T*>(w.yout[0]);
+    STACK_LAUNCH(k_gather<T><<<nb(cnt), 256, 0, s>>>(x, X, p.L, d, a, b, cnt));
+    ST_TRY(cudaGetLastError());
+    for (int r = 0; r < layers; ++r) {
+      float* Sr = S_state + (size_t)r * g.st;
+      float* zr = z_state + (size_t)r * g.zt;
+      float* Slr = S_lo ? S_lo + (size_t)r * g.st : nullptr;
+      float* zlr = z_lo ? z_lo + (size_t)r * g.zt : nullptr;
+      const float* om = omegas ? omegas + (size_t)r * M * d : nullptr;
+      STACK_LAUNCH(k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
+      ST_TRY(cudaGetLastError());
+      // layer r on the slice, from its state after the previous slice (in place)
+      ST_CALL(slim_fwd_from(U, U, U, om, p.B, p.H, b, d, M, b, p.dtype, p.feature,
+                            n ? Sr : nullptr, n ? zr : nullptr, n ? Slr : nullptr,
+                            n ? zlr : nullptr, Y, Sr, zr, Slr, zlr, w.inner, g.inner, s));
+      STACK_LAUNCH(k_residual<T><<<nb(cnt), 256, 0, s>>>(X, Y, X2, cnt));
+      ST_TRY(cudaGetLastError());
+      T* t = X;
+      X = X2;
+      X2 = t;
+    }
+    STACK_LAUNCH(k_scatter<T><<<nb(cnt), 256, 0, s>>>(X, y, p.L, d, a, b, cnt));
+    ST_TRY(cudaGetLastError());
+  }
+  return SLIM_OK;
+}
+
+template <typename T>
+slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omegas, const T* dy,
+                     const float* S_state, const float* z_state, const float* S_lo,
+                     const float* z_lo, T* dx, float* domegas, void* workspace, cudaStream_t s) {
+  const Geo g = geometry(p, layers);
+  Carver cv(workspace);
+  uint8_t* xin[65];
+  uint8_t* yo[64];
+  const Ws w = carve(cv, p, g, true, xin, yo);
+  const int d = p.d, M = p.M;
+  const size_t S = (size_t)layers * g.st, Z = (size_t)layers * g.zt;
+  // running states start at the final states B^(N) (value/error pairs)
+  ST_TRY(cudaMemcpyAsync(w.Sb, S_state, S * 4, cudaMemcpyDeviceToDevice, s));
+  ST_TRY(cudaMemcpyAsync(w.zb, z_state, Z * 4, cudaMemcpyDeviceToDevice, s));
+  if (S_lo) ST_TRY(cudaMemcpyAsync(w.Slb, S_lo, S * 4, cudaMemcpyDeviceToDevice, s));
+  else ST_TRY(cudaMemsetAsync(w.Slb, 0, S * 4, s));
+  if (z_lo) ST_TRY(cudaMemcpyAsync(w.zlb, z_lo, Z * 4, cudaMemcpyDeviceToDevice, s));
+  else ST_TRY(cudaMemsetAsync(w.zlb, 0, Z * 4, s));
+  if (domegas) ST_TRY(cudaMemsetAsync(domegas, 0, (size_t)layers * M * d * 4, s));
+  float *G = w.G, *gz = w.gz, *G2 = w.G2, *gz2 = w.gz2;
+  const float scale = powf((float)d, -0.25f);
+  T* U = reinterpret_cast<T*>(w.u);
+  for (int n = g.N - 1; n >= 0; --n) {
+    const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
+    const long long cnt = (long long)g.chains * b * d, rows = (long long)g.chains * b;
+    STACK_LAUNCH(k_gather<T><<<nb(cnt), 256, 0, s>>>(x, reinterpret_cast<T*>(w.xin[0]), p.L, d, a, b, cnt));
+    ST_TRY(cudaGetLastError());
+    // recompute the slice layer by layer, rolling each layer's state back
+    for (int r = 0; r < layers; ++r) {
+      const T* X = reinterpret_cast<const T*>(w.xin[r]);
+      const float* om = omegas ? omegas + (size_t)r * M * d : nullptr;
+      float* Sb = w.Sb + r * g.st;
+      float* zb = w.zb + r * g.zt;
+      float* Slb = w.Slb + r * g.st;
+      float* zlb = w.zlb + r * g.zt;
+      // the state at the slice's end, for the layer's backward
+      ST_TRY(cudaMemcpyAsync(w.Se + r * g.st, Sb, g.st * 4, cudaMemcpyDeviceToDevice, s));
+      ST_TRY(cudaMemcpyAsync(w.ze + r * g.zt, zb, g.zt * 4, cudaMemcpyDeviceToDevice, s));
+      ST_TRY(cudaMemcpyAsync(w.Sle + r * g.st, Slb, g.st * 4, cudaMemcpyDeviceToDevice, s));
+      ST_TRY(cudaMemcpyAsync(w.zle + r * g.zt, zlb, g.zt * 4, cudaMemcpyDeviceToDevice, s));
+      STACK_LAUNCH(k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
+      ST_TRY(cudaGetLastError());
+      // eq. 17: B_r -= the slice's sum of T_l (its own contribution, from zero)
+      ST_CALL(slim_fwd_from(U, U, U, om, p.B, p.H, b, d, M, b, p.dtype, p.feature, nullptr,
+                            nullptr, nullptr, nullptr, w.scratch_y, w.dS, w.dz, w.dSl, w.dzl,
+                            w.inner, g.inner, s));
+      STACK_LAUNCH(k_pair_sub<<<nb(g.st), 256, 0, s>>>(Sb, Slb, w.dS, w.dSl, (long long)g.st));
+      STACK_LAUNCH(k_pair_sub<<<nb(g.zt), 256, 0, s>>>(zb, zlb, w.dz, w.dzl, (long long)g.zt));
+      ST_TRY(cudaGetLastError());
+      // the layer's output on the slice from the rolled-back state
+      T* Y = reinterpret_cast<T*>(w.yout[r]);
+      ST_CALL(slim_fwd_from(U, U, U, om, p.B, p.H, b, d, M, b, p.dtype, p.feature, Sb, zb, Slb,
+                            zlb, Y, w.Ssc, w.zsc, nullptr, nullptr, w.inner, g.inner, s));
+      STACK_LAUNCH(k_residual<T><<<nb(cnt), 256, 0, s>>>(X, Y, reinterpret_cast<T*>(w.xin[r + 1]), cnt));
+      ST_TRY(cudaGetLastError());
+    }
+    // back through the layers: dX^(r-1) = dX^(r) + u'(X^(r-1))^T (dq + dk + dv)
+    STACK_LAUNCH(k_dy_in<T><<<nb(cnt), 256, 0, s>>>(dy, w.dx, reinterpret_cast<T*>(w.dout), p.L, d, a, b, cnt));
+    ST_TRY(cudaGetLastError());
+    for (int r = layers - 1; r >= 0; --r) {
+      const T* X = reinterpret_cast<const T*>(w.xin[r]);
+      const float* om = omegas ? omegas + (size_t)r * M * d : nullptr;
+      STACK_LAUNCH(k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
+      ST_TRY(cudaGetLastError());
+      ST_CALL(slim_bwd_from(U, U, U, om, w.yout[r], w.dout, w.Se + r * g.st, w.ze + r * g.zt,
+                            w.Sle + r * g.st, w.zle + r * g.zt, n + 1 < g.N ? G + r * g.st : nullptr,
+                            n + 1 < g.N ? gz + r * g.zt : nullptr, p.B, p.H, b, d, M, b, p.dtype,
+                            p.feature, w.dq, w.dk, w.dv, domegas ? w.dom : nullptr,
+                            G2 + r * g.st, gz2 + r * g.zt, w.inner, g.inner, s));
+      if (domegas) {
+        STACK_LAUNCH(k_add<<<nb((long long)M * d), 256, 0, s>>>(domegas + (size_t)r * M * d, w.dom, (long long)M * d));
+        ST_TRY(cudaGetLastError());
+      }
+      STACK_LAUNCH(k_dx_accum<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+          w.dx, X, reinterpret_cast<const T*>(w.dq), reinterpret_cast<const T*>(w.dk),
+          reinterpret_cast<const T*>(w.dv), reinterpret_cast<T*>(w.dout), d, scale, rows));
+      ST_TRY(cudaGetLastError());
+    }
+    STACK_LAUNCH(k_dx_out<T><<<nb(cnt), 256, 0, s>>>(w.dx, dx, p.L, d, a, b, cnt));
+    ST_TRY(cudaGetLastError());
+    float* t = G; G = G2; G2 = t;
+    t = gz; gz = gz2; gz2 = t;
+  }
+  return SLIM_OK;
+}
+
+}  // namespace
+
+size_t workspace_bytes(const Problem& p, int layers, bool bwd) {
+  const Geo g = geometry(p, layers);
+  Carver cv(nullptr);
+  uint8_t* xin[65];
+  uint8_t* yo[64];
+  carve(cv, p, g, bwd, xin, yo);
+  return cv.bytes();
+}
+
+slim_status fwd(const Problem& p, int layers, const void* x, const float* omegas, void* y,
+                float* S_state, float* z_state, float* S_lo, float* z_lo, void* workspace,
+                cudaStream_t s) {
+  if (p.dtype == SLIM_BF16)
+    return fwd_impl<__nv_bfloat16>(p, layers, (const __nv_bfloat16*)x, omegas, (__nv_bfloat16*)y,
+                                   S_state, z_state, S_lo, z_lo, workspace, s);
+  return fwd_impl<float>(p, layers, (const float*)x, omegas, (float*)y, S_state, z_state, S_lo,
+                         z_lo, workspace, s);
+}
+
+slim_status bwd(const Problem& p, int layers, const void* x, const float* omegas, const void* dy,
+                const float* S_state, const float* z_state, const float* S_lo,
+                const float* z_lo, void* dx, float* domegas, void* workspace, cudaStream_t s) {
+  if (p.dtype == SLIM_BF16)
+    return bwd_impl<__nv_bfloat16>(p, layers, (const __nv_bfloat16*)x, omegas,
+                                   (const __nv_bfloat16*)dy, S_state, z_state, S_lo, z_lo,
+                                   (__nv_bfloat16*)dx, domegas, workspace, s);
+  return bwd_impl<float>(p, layers, (const float*)x, omegas, (const float*)dy, S_state, z_state,
+                         S_lo, z_lo, (float*)dx, domegas, workspace, s);
+}
+
+}  // namespace stack
+}  // namespace slim

@@ -34,6 +34,9 @@ SIGNATURES = {
     "slim_bidir_workspace_size": ([_i] * 6 + [_i, _i, _i, ctypes.POINTER(_sz)], _i),
     "slim_fwd_bidir": ([_p] * 4 + [_i] * 6 + [_i, _i] + [_p] * 3 + [_p, _sz, _p], _i),
     "slim_bwd_bidir": ([_p] * 8 + [_i] * 6 + [_i, _i] + [_p] * 4 + [_p, _sz, _p], _i),
+    "slim_stack_workspace_size": ([_i] * 7 + [_i, _i, _i, ctypes.POINTER(_sz)], _i),
+    "slim_stack_fwd": ([_p] * 2 + [_i] * 7 + [_i, _i] + [_p] * 5 + [_p, _sz, _p], _i),
+    "slim_stack_bwd": ([_p] * 7 + [_i] * 7 + [_i, _i] + [_p] * 2 + [_p, _sz, _p], _i),
     "slim_check_device_error": ([_p, _p], _i),
     "slim_launch_count": ([], ctypes.c_ulonglong),
     "slim_profiler_enable": ([_i], None),
@@ -259,6 +262,58 @@ def backward_bidir(q, k, v, omega, out, dout, S_state, z_state, C, feature="exp"
                                     dv.data_ptr(), _ptr(domega), ws.data_ptr(), ws.numel(),
                                     _stream_handle(stream)), "slim_bwd_bidir")
     return dq, dk, dv, domega
+
+
+def stack_workspace_size(B, H, L, d, M, C, layers, dtype, feature, backward):
+    n = _sz(0)
+    _check(library().slim_stack_workspace_size(B, H, L, d, M, C, layers, DTYPES[dtype],
+                                               FEATURES[feature], 1 if backward else 0,
+                                               ctypes.byref(n)), "slim_stack_workspace_size")
+    return n.value
+
+
+def stack_forward(x, omegas, C, feature="exp", layers=None, workspace=None, stream=None,
+                  residuals=True):
+    """slim_stack_fwd: x [B,H,L,d]; omegas [layers, M, d] fp32 (None for the
+    quadratic map, then give `layers`).  Returns (y, S_state, z_state[, S_lo,
+    z_lo]) with per-layer states [layers, B, H, M, d] and [layers, B, H, M]."""
+    _require_cuda(x)
+    B, H, L, d = x.shape
+    layers = omegas.shape[0] if omegas is not None else layers
+    M = omegas.shape[1] if omegas is not None else d
+    y = torch.empty_like(x)
+    S = torch.empty(layers, B, H, M, d, dtype=torch.float32, device=x.device)
+    z = torch.empty(layers, B, H, M, dtype=torch.float32, device=x.device)
+    S_lo = torch.empty_like(S) if residuals else None
+    z_lo = torch.empty_like(z) if residuals else None
+    ws = workspace if workspace is not None else _workspace(
+        stack_workspace_size(B, H, L, d, M, C, layers, x.dtype, feature, False), x.device)
+    _check(library().slim_stack_fwd(x.data_ptr(), _opt_ptr(omegas), B, H, L, d, M, C, layers,
+                                    DTYPES[x.dtype], FEATURES[feature], y.data_ptr(),
+                                    S.data_ptr(), z.data_ptr(), _ptr(S_lo), _ptr(z_lo),
+                                    ws.data_ptr(), ws.numel(), _stream_handle(stream)),
+           "slim_stack_fwd")
+    return (y, S, z, S_lo, z_lo) if residuals else (y, S, z)
+
+
+def stack_backward(x, omegas, dy, S_state, z_state, C, feature="exp", S_lo=None, z_lo=None,
+                   workspace=None, stream=None):
+    """slim_stack_bwd: returns (dx, domegas) (domegas None without omegas)."""
+    _require_cuda(x, dy, S_state, z_state)
+    B, H, L, d = x.shape
+    layers = S_state.shape[0]
+    M = S_state.shape[3]
+    dx = torch.empty_like(x)
+    dom = (torch.empty(layers, M, d, dtype=torch.float32, device=x.device)
+           if omegas is not None else None)
+    ws = workspace if workspace is not None else _workspace(
+        stack_workspace_size(B, H, L, d, M, C, layers, x.dtype, feature, True), x.device)
+    _check(library().slim_stack_bwd(x.data_ptr(), _opt_ptr(omegas), dy.data_ptr(),
+                                    S_state.data_ptr(), z_state.data_ptr(), _ptr(S_lo),
+                                    _ptr(z_lo), B, H, L, d, M, C, layers, DTYPES[x.dtype],
+                                    FEATURES[feature], dx.data_ptr(), _ptr(dom), ws.data_ptr(),
+                                    ws.numel(), _stream_handle(stream)), "slim_stack_bwd")
+    return dx, dom
 
 
 def forward_into(q, k, v, omega, C, feature, out, S_state, z_state, workspace, stream=None,

@@ -114,3 +114,28 @@ def make_inputs(w: Workload, device="cpu"):
 def as_float64_numpy(t):
     """Exact upcast of a (possibly bf16) tensor to a float64 NumPy array."""
     return t.detach().to("cpu", torch.float64).numpy()
+
+
+def make_stack_inputs(w: Workload, layers, device="cpu"):
+    """Inputs of a stack of `layers` residual layers on workload w's shape:
+    dict(x [B,H,L,d], omegas [layers, M, d] fp32, dy [B,H,L,d]).  One generator
+    seeded once draws x, then each layer's Omega, then dy, with the workload's
+    distributions (x like q)."""
+    gen = torch.Generator(device="cpu").manual_seed(w.seed)
+    shape = (w.B, w.H, w.L, w.d)
+    if w.qkv_dist == "normal":
+        x = torch.randn(shape, generator=gen, dtype=torch.float32) / (w.d ** 0.25)
+    elif w.qkv_dist == "uniform":
+        x = torch.rand(shape, generator=gen, dtype=torch.float32) * 2.0 - 1.0
+    else:
+        raise ValueError(w.qkv_dist)
+    oms = []
+    for _ in range(layers):
+        if w.omega_dist == "iid":
+            oms.append(torch.randn(w.M, w.d, generator=gen, dtype=torch.float32))
+        else:
+            oms.append(orthogonal_gaussian(w.M, w.d, gen))
+    dy = torch.randn(shape, generator=gen, dtype=torch.float32)
+    dt = TORCH_DTYPE[w.dtype]
+    out = {"x": x.to(dt), "omegas": torch.stack(oms).contiguous(), "dy": dy.to(dt)}
+    return {n: t.to(device) for n, t in out.items()}

@@ -213,3 +213,50 @@ def test_streaming_arguments_rejected_before_launch(lib):
     assert bwd_from_call(lib, (None, None), (None, FAKE)) == INVALID
     assert bwd_from_call(lib, (FAKE, FAKE), (FAKE + 8, FAKE)) == INVALID
     assert bwd_from_call(lib, (FAKE, FAKE), (FAKE, FAKE), wsb=nb - 1) == WORKSPACE
+
+
+def stack_ws(B, H, L, d, M, C, layers, bwd):
+    n = ctypes.c_size_t(0)
+    st = slim.library().slim_stack_workspace_size(B, H, L, d, M, C, layers, 0, 0, 1 if bwd else 0,
+                                                   ctypes.byref(n))
+    return st, n.value
+
+
+def test_stack_workspace_scales_with_C_and_layers_not_L(lib):
+    for bwd in (False, True):
+        st, a = stack_ws(2, 2, 4096, 64, 128, 256, 3, bwd)
+        assert st == OK and a > 0
+        assert stack_ws(2, 2, 65536, 64, 128, 256, 3, bwd) == (OK, a)      # O(C), not O(L)
+        _, b = stack_ws(2, 2, 4096, 64, 128, 512, 3, bwd)
+        assert b > a
+        _, c = stack_ws(2, 2, 4096, 64, 128, 256, 6, bwd)
+        # the forward keeps one slice's rows (states are outputs); the backward
+        # keeps every layer's slice input and output and its states
+        assert c > a if bwd else c == a
+    assert stack_ws(2, 2, 4096, 64, 128, 256, 0, False)[0] == INVALID
+    assert stack_ws(2, 2, 4096, 64, 128, 256, 65, True)[0] == INVALID
+    assert stack_ws(2, 2, 4096, 64, 128, 256, 64, True)[0] == OK
+
+
+def test_stack_rejects_before_launch(lib):
+    dims = (1, 1, 8, 16, 32, 4)
+    _, nf = stack_ws(*dims, 2, False)
+    _, nb = stack_ws(*dims, 2, True)
+
+    def fwd(layers=2, om=FAKE, lo=(None, None), S=FAKE, wsb=nf, wsp=FAKE):
+        return lib.slim_stack_fwd(FAKE, om, *dims, layers, 0, 0, FAKE, S, FAKE, lo[0], lo[1],
+                                  wsp, wsb, None)
+
+    def bwd(layers=2, om=FAKE, dom=FAKE, wsb=nb, wsp=FAKE):
+        return lib.slim_stack_bwd(FAKE, om, FAKE, FAKE, FAKE, None, None, *dims, layers, 0, 0,
+                                  FAKE, dom, wsp, wsb, None)
+
+    assert fwd(layers=0) == INVALID and fwd(layers=65) == INVALID
+    assert fwd(om=None) == INVALID                  # Omega needed for exp features
+    assert fwd(lo=(FAKE, None)) == INVALID          # residuals both or neither
+    assert fwd(S=FAKE + 4) == INVALID               # misaligned state
+    assert fwd(wsb=nf - 1) == WORKSPACE
+    assert fwd(wsp=FAKE + 16) == INVALID            # workspace not 256-byte aligned
+    assert bwd(layers=65) == INVALID
+    assert bwd(dom=None) == INVALID
+    assert bwd(wsb=nb - 1) == WORKSPACE

@@ -523,11 +523,46 @@ def pin_stack_rollback_closes():
 
 
 def pin_stack_one_layer():
-    """s = 1 is one layer plus the residual: X^(1) = X + Att(X)."""
+    """s = 1 is one layer plus the residual: X^(1) = X + Att(u, u, u) with u
+    the normalised rows."""
     X, Oms, _ = _stack_case(27, s=1)
     Y, _ = stack.forward(X, Oms, 5, "relu")
-    Yl, _, _ = sliced.forward(X, X, X, Oms[0], 5, "relu")
+    U = stack.row_norm(X)
+    Yl, _, _ = sliced.forward(U, U, U, Oms[0], 5, "relu")
     return rel(Y, X + Yl)
+
+
+def pin_row_norm():
+    """The row normalisation: every row of u has root-mean-square d^(-1/4)
+    (up to eps), u is invariant to scaling the row, and its VJP against
+    central differences."""
+    rng = np.random.default_rng(28)
+    X = rng.standard_normal((2, 5, 8)) * 3.0
+    U = stack.row_norm(X)
+    d = X.shape[-1]
+    err = float(np.abs(np.sqrt(np.mean(U * U, axis=-1)) - d ** -0.25).max())
+    err = max(err, rel(stack.row_norm(7.0 * X), U))
+    g = rng.standard_normal(X.shape)
+    got = stack.row_norm_vjp(X, g)
+    fd = np.zeros_like(X)
+    h = 1e-6
+    it = np.nditer(X, flags=["multi_index"])
+    for _ in it:
+        i = it.multi_index
+        keep = X[i]
+        X[i] = keep + h
+        fp = float(np.sum(g * stack.row_norm(X)))
+        X[i] = keep - h
+        fm = float(np.sum(g * stack.row_norm(X)))
+        X[i] = keep
+        fd[i] = (fp - fm) / (2 * h)
+    # eps = 1e-6 moves the root-mean-square and the scale invariance by
+    # about eps / mean(x^2), well under 1e-5 for rows of scale 3
+    return max(err / 1e-5, rel(got, fd) / 1e-6)
+
+
+def test_row_norm():
+    assert pin_row_norm() < 1.0
 
 
 @pytest.mark.parametrize("feature", ["exp", "relu", "square"])
