@@ -25,29 +25,6 @@ namespace slim {
 namespace stack {
 namespace {
 
-// rows [a, a+b) of every chain of a [chains][L][d] tensor <-> [chains][b][d]
-template <typename T>
-__global__ void k_gather(const T* src, T* dst, int L, int d, int a, int b, long long n) {
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const long long per = (long long)b * d;
-  const long long c = i / per, r = i % per;
-  dst[i] = src[((size_t)c * L + a) * d + r];
-}
-template <typename T>
-__global__ void k_scatter(const T* src, T* dst, int L, int d, int a, int b, long long n) {
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const long long per = (long long)b * d;
-  const long long c = i / per, r = i % per;
-  dst[((size_t)c * L + a) * d + r] = src[i];
-}
-// out = x + y (the residual connection), in fp32, rounded to the dtype
-template <typename T>
-__global__ void k_residual(const T* x, const T* y, T* out, long long n) {
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < n) Io<T>::store(out, i, Io<T>::load(x, i) + Io<T>::load(y, i));
-}
 // (hi, lo) -= (dhi, dlo): the rollback of eq. 17 on an fp32 value/error pair
 __global__ void k_pair_sub(float* hi, float* lo, const float* dhi, const float* dlo, long long n) {
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -66,28 +43,48 @@ __device__ float warp_sum(float v) {
   return v;
 }
 
-// u = scale * x / sqrt(mean(x^2) + eps) row by row, scale = d^(-1/4)
+// u = scale * x / sqrt(mean(x^2) + eps) for one row, one warp per row
 template <typename T>
-__global__ void k_rownorm(const T* x, T* u, int d, float scale, long long rows) {
-  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= rows) return;
-  const T* xr = x + row * d;
+__device__ void norm_row(const T* xr, T* ur, int d, float scale, int lane) {
   float ss = 0.f;
   for (int j = lane; j < d; j += 32) {
     const float v = Io<T>::load(xr, j);
     ss += v * v;
   }
   const float inv = scale / sqrtf(warp_sum(ss) / d + kNormEps);
-  for (int j = lane; j < d; j += 32) Io<T>::store(u + row * d, j, Io<T>::load(xr, j) * inv);
+  for (int j = lane; j < d; j += 32) Io<T>::store(ur, j, Io<T>::load(xr, j) * inv);
+}
+
+// the first layer's u from the slice's rows
+template <typename T>
+__global__ void k_rownorm(const T* x, T* u, int d, float scale, long long rows) {
+  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (row >= rows) return;
+  norm_row(x + row * d, u + row * d, d, scale, threadIdx.x & 31);
+}
+
+// the residual connection out = x + y (fp32 sum rounded to the dtype), then,
+// when u is given, the next layer's u from the rounded out (the value the next
+// layer's recompute reads back)
+template <typename T>
+__global__ void k_residual_norm(const T* x, const T* y, T* out, T* u, int d, float scale,
+                                long long rows) {
+  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const size_t o = (size_t)row * d;
+  for (int j = lane; j < d; j += 32) Io<T>::store(out, o + j, Io<T>::load(x, o + j) + Io<T>::load(y, o + j));
+  __syncwarp();
+  if (u) norm_row(out + o, u + o, d, scale, lane);
 }
 
 // dX (fp32) += u'(x)^T g with g = dq + dk + dv (q = k = v = u(x)):
 //   dx += (scale / r) (g - x mean(g x) / r^2),  r = sqrt(mean(x^2) + eps),
-// and the next layer down's upstream gradient (the new dX) as the dtype
+// and the next layer down's upstream gradient (the new dX) as the dtype into
+// dout.  For the top layer (first) the old dX is dout itself: the slice's dy.
 template <typename T>
 __global__ void k_dx_accum(float* dx, const T* x, const T* dq, const T* dk, const T* dv, T* dout,
-                           int d, float scale, long long rows) {
+                           int d, float scale, long long rows, int first) {
   const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -105,44 +102,15 @@ __global__ void k_dx_accum(float* dx, const T* x, const T* dq, const T* dk, cons
   for (int j = lane; j < d; j += 32) {
     const float xv = Io<T>::load(x, o + j);
     const float g = Io<T>::load(dq, o + j) + Io<T>::load(dk, o + j) + Io<T>::load(dv, o + j);
-    const float v = dx[o + j] + f * (g - xv * m);
+    const float v = (first ? Io<T>::load(dout, o + j) : dx[o + j]) + f * (g - xv * m);
     dx[o + j] = v;
     Io<T>::store(dout, o + j, v);
   }
-}
-// the slice's dY into the fp32 accumulator and the top layer's dout
-template <typename T>
-__global__ void k_dy_in(const T* dy, float* dx, T* dout, int L, int d, int a, int b, long long n) {
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const long long per = (long long)b * d;
-  const long long c = i / per, r = i % per;
-  const T v = dy[((size_t)c * L + a) * d + r];
-  dx[i] = Io<T>::load(&v, 0);
-  dout[i] = v;
-}
-// accumulated fp32 dX back to the dtype, rows [a, a+b) of every chain
-template <typename T>
-__global__ void k_dx_out(const float* dx, T* dst, int L, int d, int a, int b, long long n) {
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const long long per = (long long)b * d;
-  const long long c = i / per, r = i % per;
-  Io<T>::store(dst, ((size_t)c * L + a) * d + r, dx[i]);
 }
 __global__ void k_add(float* acc, const float* x, long long n) {
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) acc[i] += x[i];
 }
-
-unsigned nb(long long n) { return (unsigned)((n + 255) / 256); }
-unsigned nrb(long long rows) { return (unsigned)((rows + kRowsPerBlock - 1) / kRowsPerBlock); }
-// every launch of this file is counted (and timed when the profiler is on)
-#define STACK_LAUNCH(...)                           \
-  do {                                              \
-    prof::Scope ps_(prof::K_STACK, s);              \
-    __VA_ARGS__;                                    \
-  } while (0)
 
 struct Geo {
   int chains, Cs, N, s;
@@ -153,8 +121,33 @@ struct Geo {
   size_t inner;  // workspace of one segment call
 };
 
+unsigned nb(long long n) { return (unsigned)((n + 255) / 256); }
+unsigned nrb(long long rows) { return (unsigned)((rows + kRowsPerBlock - 1) / kRowsPerBlock); }
+// every launch of this file is counted (and timed when the profiler is on),
+// with the bytes it must move
+#define STACK_LAUNCH(bytes, ...)                          \
+  do {                                                    \
+    prof::Scope ps_(prof::K_STACK, s, 0.0, (double)(bytes)); \
+    __VA_ARGS__;                                          \
+  } while (0)
+
+// rows [a, a+b) of every chain: [chains][L][d] <-> [chains][b][d], one
+// strided copy
+cudaError_t gather(const void* src, void* dst, const Geo& g, int L, int d, int a, int b,
+                   cudaStream_t s) {
+  const size_t row = (size_t)d * g.esz;
+  return cudaMemcpy2DAsync(dst, b * row, static_cast<const char*>(src) + a * row, L * row,
+                           b * row, g.chains, cudaMemcpyDeviceToDevice, s);
+}
+cudaError_t scatter(const void* src, void* dst, const Geo& g, int L, int d, int a, int b,
+                    cudaStream_t s) {
+  const size_t row = (size_t)d * g.esz;
+  return cudaMemcpy2DAsync(static_cast<char*>(dst) + a * row, L * row, src, b * row, b * row,
+                           g.chains, cudaMemcpyDeviceToDevice, s);
+}
+
 struct Ws {
-  uint8_t** xin;  // [s + 1] slice inputs of each layer, then the top's output
+  uint8_t** xin;  // backward: [s] each layer's slice input; forward: two, ping-pong
   uint8_t** yout; // [s] layer outputs on the slice
   float *Sb, *zb, *Slb, *zlb;   // [s] running states (backward), value/error pairs
   float *Se, *ze, *Sle, *zle;   // [s] states at the slice's end (backward)
@@ -184,7 +177,7 @@ Ws carve(Carver& cv, const Problem& p, const Geo& g, bool bwd, uint8_t** xin_ptr
   w.inner = cv.take<uint8_t>(g.inner);
   w.xin = xin_ptrs;
   w.yout = y_ptrs;
-  for (int r = 0; r <= (bwd ? g.s : 1); ++r) xin_ptrs[r] = cv.take<uint8_t>(sb);
+  for (int r = 0; r < (bwd ? g.s : 2); ++r) xin_ptrs[r] = cv.take<uint8_t>(sb);
   if (bwd) {
     for (int r = 0; r < g.s; ++r) y_ptrs[r] = cv.take<uint8_t>(sb);
     const size_t S = g.s * g.st, Z = g.s * g.zt;
@@ -251,11 +244,13 @@ slim_status fwd_impl(const Problem& p, int layers, const T* x, const float* omeg
   T* U = reinterpret_cast<T*>(w.u);
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    const long long cnt = (long long)g.chains * b * d, rows = (long long)g.chains * b;
+    const long long rows = (long long)g.chains * b;
+    const double sb = (double)rows * d * g.esz;  // bytes of one slice tensor
     T* X = reinterpret_cast<T*>(w.xin[0]);
     T* X2 = reinterpret_cast<T*>(w.xin[1]);
     T* Y = reinterpret_cast<T*>(w.yout[0]);
-    STACK_LAUNCH(k_gather<T><<<nb(cnt), 256, 0, s>>>(x, X, p.L, d, a, b, cnt));
+    ST_TRY(gather(x, X, g, p.L, d, a, b, s));
+    STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
     ST_TRY(cudaGetLastError());
     for (int r = 0; r < layers; ++r) {
       float* Sr = S_state + (size_t)r * g.st;
@@ -263,20 +258,19 @@ slim_status fwd_impl(const Problem& p, int layers, const T* x, const float* omeg
       float* Slr = S_lo ? S_lo + (size_t)r * g.st : nullptr;
       float* zlr = z_lo ? z_lo + (size_t)r * g.zt : nullptr;
       const float* om = omegas ? omegas + (size_t)r * M * d : nullptr;
-      STACK_LAUNCH(k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
-      ST_TRY(cudaGetLastError());
       // layer r on the slice, from its state after the previous slice (in place)
       ST_CALL(slim_fwd_from(U, U, U, om, p.B, p.H, b, d, M, b, p.dtype, p.feature,
                             n ? Sr : nullptr, n ? zr : nullptr, n ? Slr : nullptr,
                             n ? zlr : nullptr, Y, Sr, zr, Slr, zlr, w.inner, g.inner, s));
-      STACK_LAUNCH(k_residual<T><<<nb(cnt), 256, 0, s>>>(X, Y, X2, cnt));
+      const bool next = r + 1 < layers;
+      STACK_LAUNCH((next ? 4 : 3) * sb, k_residual_norm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+                                            X, Y, X2, next ? U : nullptr, d, scale, rows));
       ST_TRY(cudaGetLastError());
       T* t = X;
       X = X2;
       X2 = t;
     }
-    STACK_LAUNCH(k_scatter<T><<<nb(cnt), 256, 0, s>>>(X, y, p.L, d, a, b, cnt));
-    ST_TRY(cudaGetLastError());
+    ST_TRY(scatter(X, y, g, p.L, d, a, b, s));
   }
   return SLIM_OK;
 }
@@ -305,8 +299,11 @@ slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omeg
   T* U = reinterpret_cast<T*>(w.u);
   for (int n = g.N - 1; n >= 0; --n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    const long long cnt = (long long)g.chains * b * d, rows = (long long)g.chains * b;
-    STACK_LAUNCH(k_gather<T><<<nb(cnt), 256, 0, s>>>(x, reinterpret_cast<T*>(w.xin[0]), p.L, d, a, b, cnt));
+    const long long rows = (long long)g.chains * b;
+    const double sb = (double)rows * d * g.esz;
+    ST_TRY(gather(x, w.xin[0], g, p.L, d, a, b, s));
+    STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+                             reinterpret_cast<const T*>(w.xin[0]), U, d, scale, rows));
     ST_TRY(cudaGetLastError());
     // recompute the slice layer by layer, rolling each layer's state back
     for (int r = 0; r < layers; ++r) {
@@ -321,46 +318,54 @@ slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omeg
       ST_TRY(cudaMemcpyAsync(w.ze + r * g.zt, zb, g.zt * 4, cudaMemcpyDeviceToDevice, s));
       ST_TRY(cudaMemcpyAsync(w.Sle + r * g.st, Slb, g.st * 4, cudaMemcpyDeviceToDevice, s));
       ST_TRY(cudaMemcpyAsync(w.zle + r * g.zt, zlb, g.zt * 4, cudaMemcpyDeviceToDevice, s));
-      STACK_LAUNCH(k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
-      ST_TRY(cudaGetLastError());
       // eq. 17: B_r -= the slice's sum of T_l (its own contribution, from zero)
       ST_CALL(slim_fwd_from(U, U, U, om, p.B, p.H, b, d, M, b, p.dtype, p.feature, nullptr,
                             nullptr, nullptr, nullptr, w.scratch_y, w.dS, w.dz, w.dSl, w.dzl,
                             w.inner, g.inner, s));
-      STACK_LAUNCH(k_pair_sub<<<nb(g.st), 256, 0, s>>>(Sb, Slb, w.dS, w.dSl, (long long)g.st));
-      STACK_LAUNCH(k_pair_sub<<<nb(g.zt), 256, 0, s>>>(zb, zlb, w.dz, w.dzl, (long long)g.zt));
+      STACK_LAUNCH(24.0 * g.st, k_pair_sub<<<nb(g.st), 256, 0, s>>>(Sb, Slb, w.dS, w.dSl, (long long)g.st));
+      STACK_LAUNCH(24.0 * g.zt, k_pair_sub<<<nb(g.zt), 256, 0, s>>>(zb, zlb, w.dz, w.dzl, (long long)g.zt));
       ST_TRY(cudaGetLastError());
       // the layer's output on the slice from the rolled-back state
       T* Y = reinterpret_cast<T*>(w.yout[r]);
       ST_CALL(slim_fwd_from(U, U, U, om, p.B, p.H, b, d, M, b, p.dtype, p.feature, Sb, zb, Slb,
                             zlb, Y, w.Ssc, w.zsc, nullptr, nullptr, w.inner, g.inner, s));
-      STACK_LAUNCH(k_residual<T><<<nb(cnt), 256, 0, s>>>(X, Y, reinterpret_cast<T*>(w.xin[r + 1]), cnt));
-      ST_TRY(cudaGetLastError());
+      // the next layer's input and its u; the top layer's output is not needed
+      if (r + 1 < layers) {
+        STACK_LAUNCH(4 * sb, k_residual_norm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+                                 X, Y, reinterpret_cast<T*>(w.xin[r + 1]), U, d, scale, rows));
+        ST_TRY(cudaGetLastError());
+      }
     }
-    // back through the layers: dX^(r-1) = dX^(r) + u'(X^(r-1))^T (dq + dk + dv)
-    STACK_LAUNCH(k_dy_in<T><<<nb(cnt), 256, 0, s>>>(dy, w.dx, reinterpret_cast<T*>(w.dout), p.L, d, a, b, cnt));
-    ST_TRY(cudaGetLastError());
+    // back through the layers: dX^(r-1) = dX^(r) + u'(X^(r-1))^T (dq + dk + dv);
+    // the top layer's upstream gradient is the slice's dy
+    ST_TRY(gather(dy, w.dout, g, p.L, d, a, b, s));
     for (int r = layers - 1; r >= 0; --r) {
       const T* X = reinterpret_cast<const T*>(w.xin[r]);
       const float* om = omegas ? omegas + (size_t)r * M * d : nullptr;
-      STACK_LAUNCH(k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
-      ST_TRY(cudaGetLastError());
+      if (r + 1 < layers) {  // the top layer's u is still in place from the recompute
+        STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
+        ST_TRY(cudaGetLastError());
+      }
       ST_CALL(slim_bwd_from(U, U, U, om, w.yout[r], w.dout, w.Se + r * g.st, w.ze + r * g.zt,
                             w.Sle + r * g.st, w.zle + r * g.zt, n + 1 < g.N ? G + r * g.st : nullptr,
                             n + 1 < g.N ? gz + r * g.zt : nullptr, p.B, p.H, b, d, M, b, p.dtype,
                             p.feature, w.dq, w.dk, w.dv, domegas ? w.dom : nullptr,
                             G2 + r * g.st, gz2 + r * g.zt, w.inner, g.inner, s));
       if (domegas) {
-        STACK_LAUNCH(k_add<<<nb((long long)M * d), 256, 0, s>>>(domegas + (size_t)r * M * d, w.dom, (long long)M * d));
+        STACK_LAUNCH(12.0 * M * d, k_add<<<nb((long long)M * d), 256, 0, s>>>(
+                                       domegas + (size_t)r * M * d, w.dom, (long long)M * d));
         ST_TRY(cudaGetLastError());
       }
-      STACK_LAUNCH(k_dx_accum<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
-          w.dx, X, reinterpret_cast<const T*>(w.dq), reinterpret_cast<const T*>(w.dk),
-          reinterpret_cast<const T*>(w.dv), reinterpret_cast<T*>(w.dout), d, scale, rows));
+      const bool first = r == layers - 1;
+      STACK_LAUNCH((double)rows * d * (6.0 * g.esz + (first ? 4 : 8)),
+                   k_dx_accum<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+                       w.dx, X, reinterpret_cast<const T*>(w.dq), reinterpret_cast<const T*>(w.dk),
+                       reinterpret_cast<const T*>(w.dv), reinterpret_cast<T*>(w.dout), d, scale,
+                       rows, first ? 1 : 0));
       ST_TRY(cudaGetLastError());
     }
-    STACK_LAUNCH(k_dx_out<T><<<nb(cnt), 256, 0, s>>>(w.dx, dx, p.L, d, a, b, cnt));
-    ST_TRY(cudaGetLastError());
+    // dout now holds dX^(0) of the slice, rounded to the dtype
+    ST_TRY(scatter(w.dout, dx, g, p.L, d, a, b, s));
     float* t = G; G = G2; G2 = t;
     t = gz; gz = gz2; gz2 = t;
   }

@@ -108,6 +108,17 @@ def _stack_layer_bwd_drops_residual(Q, K, V, Omega, dY, C, feature, R, S, G_R, G
     dq, dk, dv, dO, B0, G = _STACK_LAYER_BWD(Q, K, V, Omega, dY, C, feature, R, S, G_R, G_S)
     return dq - dY, dk, dv, dO, B0, G
 
+_ROW_NORM_VJP = _stack.row_norm_vjp
+
+
+def _row_norm_vjp_no_projection(X, g):
+    # mistake: the normalisation's VJP as a plain rescale, without removing
+    # the component along x
+    d = X.shape[-1]
+    r = np.sqrt(np.mean(X * X, axis=-1, keepdims=True) + _stack.EPS)
+    return d ** -0.25 / r * g
+
+
 MUTATIONS = {
     "exclusive_mask": (lambda mp: mp.setattr(sliced, "_forward_rows", _exclusive_forward_rows),
                        lambda: P.pin_brute_vs_sliced("exp"), 1e-6),
@@ -133,6 +144,9 @@ MUTATIONS = {
                           lambda: P.pin_golden(), 1e-6),
     "stack_residual_dropped": (
         lambda mp: mp.setattr(_stack, "layer_backward", _stack_layer_bwd_drops_residual),
+        lambda: P.pin_stack_finite_differences("exp"), 1e-3),
+    "stack_norm_vjp_no_projection": (
+        lambda mp: mp.setattr(_stack, "row_norm_vjp", _row_norm_vjp_no_projection),
         lambda: P.pin_stack_finite_differences("exp"), 1e-3),
     "bidir_key_grad_missing_normaliser": (
         lambda mp: mp.setattr(_bidir, "backward", _bidir_backward_drop_key_normaliser),
