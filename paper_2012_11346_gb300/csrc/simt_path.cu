@@ -70,54 +70,84 @@ struct GemmP {
 // in twice the working precision and rounded once.  The backward pass needs
 // it: its contractions cancel (signed feature gradients summed against
 // Omega), which multiplies plain fp32 rounding error by 10-30.
-template <bool PRECISE>
+// RM rows per thread: a CTA computes a (16 RM) x 64 tile of C (RM = 4 for
+// most products, 1 or 2 when m is 16 or 32 -- the tiles of short slices).
+template <bool PRECISE, int RM>
 __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
-  __shared__ __align__(16) float As[GK][GT + 4];
-  __shared__ __align__(16) float Bs[GK][GT + 4];
+  // two stages: chunk k0 + GK is read from global memory into registers while
+  // chunk k0 is multiplied out of shared memory, one barrier per chunk
+  constexpr int TM = 16 * RM;
+  __shared__ __align__(16) float As[2][GK][TM + 4];
+  __shared__ __align__(16) float Bs[2][GK][GT + 4];
+  constexpr int PA = TM * GK / 256, PB = GT * GK / 256;  // elements a thread stages
   const int z = blockIdx.z + P.zoff;
   const int z0 = z / P.nb1, z1 = z % P.nb1;
   const float* A = P.a.p + z0 * P.a.b0 + z1 * P.a.b1;
   const float* Bm = P.b.p + z0 * P.b.b0 + z1 * P.b.b1;
-  const int i0 = blockIdx.y * GT, j0 = blockIdx.x * GT;
+  const int i0 = blockIdx.y * TM, j0 = blockIdx.x * GT;
   const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
-  float acc[4][4], err[4][4];
+  const bool a_kc = P.a.cs == 1, b_nc = P.b.cs == 1;
+  float acc[RM][4], err[RM][4];
 #pragma unroll
-  for (int r = 0; r < 4; ++r)
+  for (int r = 0; r < RM; ++r)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[r][c] = err[r][c] = 0.f;
 
+  // element e of a chunk: (kk, row) of A and (kk, col) of B, laid out so that
+  // consecutive threads read consecutive addresses of the contiguous dimension
+  float ra[PA], rb[PB];
+  auto fetch = [&](int k0) {
+#pragma unroll
+    for (int i = 0; i < PA; ++i) {
+      const int e = tid + i * 256;
+      const int kk = a_kc ? e % GK : e / TM, r = a_kc ? e / GK : e % TM;
+      const int gi = i0 + r, gk = k0 + kk;
+      ra[i] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < PB; ++i) {
+      const int e = tid + i * 256;
+      const int kb = b_nc ? e / GT : e % GK, cb = b_nc ? e % GT : e / GK;
+      const int gkb = k0 + kb, gj = j0 + cb;
+      rb[i] = (gkb < P.k && gj < P.n) ? Bm[gkb * P.b.rs + gj * P.b.cs] : 0.f;
+    }
+  };
+  auto stage = [&](int buf) {
+#pragma unroll
+    for (int i = 0; i < PA; ++i) {
+      const int e = tid + i * 256;
+      As[buf][a_kc ? e % GK : e / TM][a_kc ? e / GK : e % TM] = ra[i];
+    }
+#pragma unroll
+    for (int i = 0; i < PB; ++i) {
+      const int e = tid + i * 256;
+      Bs[buf][b_nc ? e / GT : e % GK][b_nc ? e % GT : e / GK] = rb[i];
+    }
+  };
+
+  fetch(0);
+  stage(0);
+  __syncthreads();
+  int buf = 0;
   for (int k0 = 0; k0 < P.k; k0 += GK) {
-    if (P.a.cs == 1) {  // k contiguous
-      for (int e = tid; e < GT * GK; e += 256) {
-        int r = e / GK, kk = e % GK, gi = i0 + r, gk = k0 + kk;
-        As[kk][r] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk] : 0.f;
-      }
-    } else {            // rows contiguous
-      for (int e = tid; e < GT * GK; e += 256) {
-        int kk = e / GT, r = e % GT, gi = i0 + r, gk = k0 + kk;
-        As[kk][r] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
-      }
-    }
-    if (P.b.cs == 1) {  // columns contiguous
-      for (int e = tid; e < GT * GK; e += 256) {
-        int kk = e / GT, c = e % GT, gk = k0 + kk, gj = j0 + c;
-        Bs[kk][c] = (gk < P.k && gj < P.n) ? Bm[gk * P.b.rs + gj] : 0.f;
-      }
-    } else {            // k contiguous
-      for (int e = tid; e < GT * GK; e += 256) {
-        int c = e / GK, kk = e % GK, gk = k0 + kk, gj = j0 + c;
-        Bs[kk][c] = (gk < P.k && gj < P.n) ? Bm[gk * P.b.rs + gj * P.b.cs] : 0.f;
-      }
-    }
-    __syncthreads();
+    const bool more = k0 + GK < P.k;
+    if (more) fetch(k0 + GK);
 #pragma unroll
     for (int kk = 0; kk < GK; ++kk) {
-      float4 a4 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
-      float4 b4 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
-      float a[4] = {a4.x, a4.y, a4.z, a4.w};
+      float a[RM];
+      if constexpr (RM == 4) {
+        const float4 a4 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
+        a[0] = a4.x; a[1] = a4.y; a[2] = a4.z; a[3] = a4.w;
+      } else if constexpr (RM == 2) {
+        const float2 a2 = *reinterpret_cast<const float2*>(&As[buf][kk][ty * 2]);
+        a[0] = a2.x; a[1] = a2.y;
+      } else {
+        a[0] = As[buf][kk][ty];
+      }
+      float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
       float b[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int r = 0; r < RM; ++r)
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           if (PRECISE) {
@@ -132,13 +162,16 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
           }
         }
     }
+    // the other buffer was last read before the previous barrier
+    if (more) stage(buf ^ 1);
     __syncthreads();
+    buf ^= 1;
   }
 
   float* Cm = P.c.p + z0 * P.c.b0 + z1 * P.c.b1;
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const int i = i0 + ty * 4 + r;
+  for (int r = 0; r < RM; ++r) {
+    const int i = i0 + ty * RM + r;
     if (i >= P.m) continue;
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
@@ -158,6 +191,9 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
 // Loads rows [a, a+b) of every chain, converts to fp32, applies the feature
 // map.  Rows b..Cp-1 of the padded tile are zero everywhere (including the
 // ones column of [V | 1]), so they add nothing to any contraction.
+constexpr int kPrepFeat = 128;    // features per projection chunk
+constexpr int kPrepStride = 130;  // omT row stride in floats (8-byte rows, 2-way bank spread)
+
 template <typename T>
 __global__ void __launch_bounds__(256) k_prep(
     const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
@@ -168,8 +204,8 @@ __global__ void __launch_bounds__(256) k_prep(
   constexpr int R = 16;            // rows per CTA (q and k -> 32 vectors)
   float* xs = sm;                  // [32][d]
   float* xn2 = xs + 32 * d;        // [32]
-  float* omT = xn2 + 32;           // [d][64]
-  float* omn = omT + d * 64;       // [64]
+  float* omT = xn2 + 32;           // [d][kPrepStride]: a chunk of Omega, transposed
+  float* omn = omT + d * kPrepStride;  // [kPrepFeat]
   const int c = blockIdx.y, r0 = blockIdx.x * R, tid = threadIdx.x;
   const int dp = d + 1;
   const size_t rowbase = (size_t)c * L + a;
@@ -228,26 +264,55 @@ __global__ void __launch_bounds__(256) k_prep(
   }
   // error bound of an fp32 dot product of length d, times a safety factor 2
   const float gamma = 2.f * (float)(d + 2) * 5.9604645e-08f;
-  for (int m0 = 0; m0 < M; m0 += 64) {
+  // The projections x . omega_m, PF features at a time: thread (f, grp) owns
+  // features m0 + 2f and m0 + 2f + 1 of vectors 8 grp .. 8 grp + 7, reading
+  // four x values per vector as one float4 and two Omega values as one float2
+  // (64 FMAs per 12 shared-memory loads).  Each dot product is summed in j
+  // order, one fmaf per term.
+  const int f = tid % 64, grp = tid / 64;
+  for (int m0 = 0; m0 < M; m0 += kPrepFeat) {
     __syncthreads();
-    for (int e = tid; e < 64 * d; e += 256) {
+    for (int e = tid; e < kPrepFeat * d; e += 256) {
       int mm = e / d, j = e % d;
-      omT[j * 64 + mm] = (m0 + mm < M) ? omega[(size_t)(m0 + mm) * d + j] : 0.f;
+      omT[j * kPrepStride + mm] = (m0 + mm < M) ? omega[(size_t)(m0 + mm) * d + j] : 0.f;
     }
     __syncthreads();
-    if (tid < 64) {
+    if (tid < kPrepFeat) {
       float s = 0.f;
-      for (int j = 0; j < d; ++j) s = fmaf(omT[j * 64 + tid], omT[j * 64 + tid], s);
+      for (int j = 0; j < d; ++j) s = fmaf(omT[j * kPrepStride + tid], omT[j * kPrepStride + tid], s);
       omn[tid] = sqrtf(s);
     }
     __syncthreads();
-    const int mm = tid % 64, grp = tid / 64, m = m0 + mm;
-    if (m < M) {
+    float acc[8][2];
+#pragma unroll
+    for (int vv = 0; vv < 8; ++vv) acc[vv][0] = acc[vv][1] = 0.f;
+    for (int j = 0; j < d; j += 4) {
+      float2 o[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t)
+        o[t] = *reinterpret_cast<const float2*>(&omT[(j + t) * kPrepStride + 2 * f]);
+#pragma unroll
+      for (int vv = 0; vv < 8; ++vv) {
+        const float4 x = *reinterpret_cast<const float4*>(&xs[(grp * 8 + vv) * d + j]);
+        acc[vv][0] = fmaf(x.x, o[0].x, acc[vv][0]);
+        acc[vv][1] = fmaf(x.x, o[0].y, acc[vv][1]);
+        acc[vv][0] = fmaf(x.y, o[1].x, acc[vv][0]);
+        acc[vv][1] = fmaf(x.y, o[1].y, acc[vv][1]);
+        acc[vv][0] = fmaf(x.z, o[2].x, acc[vv][0]);
+        acc[vv][1] = fmaf(x.z, o[2].y, acc[vv][1]);
+        acc[vv][0] = fmaf(x.w, o[3].x, acc[vv][0]);
+        acc[vv][1] = fmaf(x.w, o[3].y, acc[vv][1]);
+      }
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int mm = 2 * f + h, m = m0 + mm;
+      if (m >= M) continue;
+#pragma unroll
       for (int vv = 0; vv < 8; ++vv) {
         const int vec = grp * 8 + vv;
         const int rr = vec % R, r = r0 + rr;
-        float dot = 0.f;
-        for (int j = 0; j < d; ++j) dot = fmaf(xs[vec * d + j], omT[j * 64 + mm], dot);
+        const float dot = acc[vv][h];
         float phi = 0.f;
         if (r < b) {
           if (feature == SLIM_FEAT_EXP) {
@@ -256,10 +321,10 @@ __global__ void __launch_bounds__(256) k_prep(
             // The sign of omega.x decides ReLU's branch; near zero it is
             // recomputed in fp64 so the decision is the exact one.
             if (fabsf(dot) <= gamma * omn[mm] * sqrtf(xn2[vec])) {
-              double acc = 0.0;
+              double a64 = 0.0;
               for (int j = 0; j < d; ++j)
-                acc += (double)omega[(size_t)m * d + j] * (double)xs[vec * d + j];
-              phi = acc > 0.0 ? (float)acc * inv_sqrt_m : 0.f;
+                a64 += (double)omega[(size_t)m * d + j] * (double)xs[vec * d + j];
+              phi = a64 > 0.0 ? (float)a64 * inv_sqrt_m : 0.f;
             } else {
               phi = dot > 0.f ? dot * inv_sqrt_m : 0.f;
             }
@@ -333,13 +398,20 @@ __global__ void k_store(const float* stage, T* dst, int L, int d, int a, int b, 
   Io<T>::store(dst, ((size_t)c * L + a + r) * d + j, stage[((size_t)c * Cp + r) * d + j]);
 }
 
-// dOmega += sum over chains of the slice's per-chain partials, fixed order.
-__global__ void k_reduce_domega(const float* part, float* domega, int chains, int MD) {
+// dOmega += the sum of a launch's partials (per chain and row split), in a
+// fixed order, compensated (TwoSum) so that the number of partials does not
+// show in the fp32 result.
+__global__ void k_reduce_domega(const float* part, float* domega, int parts, int MD) {
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= MD) return;
-  float s = 0.f;
-  for (int c = 0; c < chains; ++c) s += part[(size_t)c * MD + e];
-  domega[e] += s;
+  float s = domega[e], c = 0.f;
+  for (int i = 0; i < parts; ++i) {
+    float t, err;
+    two_sum(s, part[(size_t)i * MD + e], t, err);
+    s = t;
+    c += err;
+  }
+  domega[e] = s + c;
 }
 
 // The pair is kept normalised (|lo| <= ulp(hi)/2), so hi is the rounded state
@@ -378,8 +450,12 @@ __global__ void k_state_in(StateIn st, float* hi, float* lo, int chains, int M, 
 // ------------------------------------------------------------------ host side
 namespace {
 
+constexpr int kGroupRows = 1024;  // rows per launch when short slices are grouped
+constexpr int kSplitCtas = 304;   // dOmega contractions: about two waves of 152 SMs
+
 struct Geo {
-  int chains, d, dp, M, Cs, T, nt, Cp, N;
+  int chains, d, dp, M, Cs, T, nt, Cp, N;  // Cs: rows per launch sequence (a slice or a group)
+  int ks;        // row splits of the dOmega contractions (divides nt)
   bool precise;  // fp32 problems: compensated contractions
 };
 
@@ -390,11 +466,31 @@ Geo geometry(const Problem& p) {
   g.dp = p.d + 1;
   g.M = p.M;
   g.Cs = p.slice_len();
-  g.T = g.Cs >= 64 ? 64 : ((g.Cs + 15) / 16) * 16;
-  if (g.T < 16) g.T = 16;
+  if (g.Cs < 64 && g.Cs % 16 == 0 && p.L > g.Cs) {
+    // Short slices (16, 32 or 48 rows): one tile per slice (T = C) and
+    // kGroupRows / C consecutive slices per launch.  The scan over a launch's
+    // tiles forms the state at every slice boundary (eq. 16) and the backward's
+    // reverse scan every rolled-back state (eq. 17), so each slice is evaluated
+    // as on its own; grouping trades workspace (kGroupRows rows, not C) for a
+    // launch sequence per group instead of per slice.
+    g.T = g.Cs;
+    const long long whole = ((long long)p.L + g.T - 1) / g.T * g.T;  // L in whole slices
+    const long long rows = (long long)(kGroupRows / g.T) * g.T;
+    g.Cs = (int)(rows < whole ? rows : whole);
+  } else {
+    g.T = g.Cs >= 64 ? 64 : ((g.Cs + 15) / 16) * 16;
+    if (g.T < 16) g.T = 16;
+  }
   g.nt = (g.Cs + g.T - 1) / g.T;
   g.Cp = g.nt * g.T;
-  g.N = p.num_slices();
+  g.N = p.L == 0 ? 0 : (p.L + g.Cs - 1) / g.Cs;
+  // dOmega = sum over rows of u^T x is M x d per chain: few CTAs with a long
+  // reduction.  Split the rows into ks runs of whole tiles, one partial each.
+  const int mn = ((g.M + GT - 1) / GT) * ((g.d + GT - 1) / GT);
+  const int want = (kSplitCtas + g.chains * mn - 1) / (g.chains * mn);
+  g.ks = 1;
+  for (int k = 2; k <= g.nt && k <= want; ++k)
+    if (g.nt % k == 0) g.ks = k;
   g.precise = p.dtype == SLIM_F32;
   return g;
 }
@@ -433,7 +529,7 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
     w.usum_q = cv.take<float>(C * g.Cp);
     w.usum_k = cv.take<float>(C * g.Cp);
     w.stage = cv.take<float>(C * g.Cp * g.d);
-    w.pOm = cv.take<float>(C * g.M * g.d);
+    w.pOm = cv.take<float>(C * g.ks * g.M * g.d);
   }
   return w;
 }
@@ -453,12 +549,19 @@ cudaError_t gemm(cudaStream_t s, bool precise, int m, int n, int k, Mat a, Mat b
   for (int z = 0; z < nz; z += 65535) {
     GemmP P{m, n, k, a, b, c, nb1, z, beta, causal, sx, sx_b0, sx_rs, ss, ss_b0};
     const int zc = (nz - z < 65535) ? nz - z : 65535;
-    dim3 grid((n + GT - 1) / GT, (m + GT - 1) / GT, zc);
+    // rows per CTA tile: 16 or 32 for the short tiles of grouped slices
+    const int rm = m <= 16 ? 1 : (m <= 32 ? 2 : 4), tm = 16 * rm;
+    dim3 grid((n + GT - 1) / GT, (m + tm - 1) / tm, zc);
     prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
-    if (precise)
-      k_gemm<true><<<grid, 256, 0, s>>>(P);
-    else
-      k_gemm<false><<<grid, 256, 0, s>>>(P);
+    if (precise) {
+      if (rm == 1) k_gemm<true, 1><<<grid, 256, 0, s>>>(P);
+      else if (rm == 2) k_gemm<true, 2><<<grid, 256, 0, s>>>(P);
+      else k_gemm<true, 4><<<grid, 256, 0, s>>>(P);
+    } else {
+      if (rm == 1) k_gemm<false, 1><<<grid, 256, 0, s>>>(P);
+      else if (rm == 2) k_gemm<false, 2><<<grid, 256, 0, s>>>(P);
+      else k_gemm<false, 4><<<grid, 256, 0, s>>>(P);
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -477,13 +580,13 @@ template <typename T>
 cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w,
                         const void* q, const void* k, const void* v, const void* dout,
                         const void* out, const float* omega, int a, int b, bool bwd) {
-  const size_t smem = (32 * g.d + 32 + g.d * 64 + 64) * sizeof(float);
+  const size_t smem = (32 * g.d + 32 + g.d * kPrepStride + kPrepFeat) * sizeof(float);
   static bool attr_set[kMaxDevices] = {};  // per dtype instantiation and device
   bool* set = device_flag(attr_set);
   if (set == nullptr) return cudaErrorInvalidDevice;
   if (!*set) {
     cudaError_t e = cudaFuncSetAttribute(k_prep<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         64 * 1024);
+                                         96 * 1024);
     if (e != cudaSuccess) return e;
     *set = true;
   }
@@ -684,13 +787,16 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dk, p.L, g.d,
                                                                       a, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
-    // dOmega partial per chain: u_q^T x_q + u_k^T x_k
-    SLIM_TRY(gemm(s, g.precise, g.M, g.d, g.Cp, mat(w.dphiQ, Cp * M, 0, 1, M), mat(w.Xq, Cp * d, 0, d, 1),
-                  omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.M, g.d, g.Cp, mat(w.dphiK, Cp * M, 0, 1, M), mat(w.Xk, Cp * d, 0, d, 1),
-                  omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 1.f, 0));
+    // dOmega partials per chain and row split: u_q^T x_q + u_k^T x_k
+    const long long kc = (long long)(g.nt / g.ks) * T, ks = g.ks;
+    SLIM_TRY(gemm(s, g.precise, g.M, g.d, (int)kc, mat(w.dphiQ, Cp * M, kc * M, 1, M),
+                  mat(w.Xq, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains,
+                  g.ks, 0.f, 0));
+    SLIM_TRY(gemm(s, g.precise, g.M, g.d, (int)kc, mat(w.dphiK, Cp * M, kc * M, 1, M),
+                  mat(w.Xk, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains,
+                  g.ks, 1.f, 0));
     { prof::Scope ps(prof::K_REDUCE, s);
-    k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains,
+    k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains * g.ks,
                                                              (int)(M * d)); }
     SLIM_TRY(cudaGetLastError());
   }
@@ -736,11 +842,13 @@ cudaError_t side_vjp(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w
              omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? X : nullptr, Cp * d, d,
              usum, Cp);
     if (e != cudaSuccess) return e;
-    e = gemm(s, g.precise, g.M, g.d, g.Cp, mat(dphi, Cp * M, 0, 1, M), mat(X, Cp * d, 0, d, 1),
-             omat(w.pOm, M * d, 0, d, 1), g.chains, 1, 0.f, 0);
+    const long long kc = (long long)(g.nt / g.ks) * g.T, ks = g.ks;
+    e = gemm(s, g.precise, g.M, g.d, (int)kc, mat(dphi, Cp * M, kc * M, 1, M),
+             mat(X, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains, g.ks,
+             0.f, 0);
     if (e != cudaSuccess) return e;
     { prof::Scope ps(prof::K_REDUCE, s);
-    k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains,
+    k_reduce_domega<<<blocks((long long)M * d), 256, 0, s>>>(w.pOm, domega, g.chains * g.ks,
                                                              (int)(M * d)); }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

@@ -79,6 +79,10 @@ EDGE = [
     (64, 16, 130, 1000, "f32", "exp"),
     (64, 128, 200, 33, "bf16", "relu"),
     (128, 256, 70, 16, "f32", "exp"),
+    # short slices grouped 1024 rows per launch: several groups, ragged ends
+    (64, 128, 2100, 16, "f32", "relu"),
+    (32, 64, 1500, 48, "bf16", "exp"),
+    (128, 256, 1100, 32, "bf16", "exp"),
     (128, 64, 129, 128, "bf16", "exp"),
     (32, 32, 150, 40, "f32", "square"),
     (128, 128, 90, 64, "f32", "square"),
