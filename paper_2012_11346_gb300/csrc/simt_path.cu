@@ -92,11 +92,22 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
   for (int r = 0; r < RM; ++r)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[r][c] = err[r][c] = 0.f;
+  // A last column tile of 65 columns (n = d + 1: the [V | 1] operands) takes
+  // its 65th column itself, computed by the threads with tx = 0, instead of
+  // leaving it to a CTA of its own.
+  const bool ext = P.n - j0 == GT + 1;
+  float acc_e[RM], err_e[RM];
+#pragma unroll
+  for (int r = 0; r < RM; ++r) acc_e[r] = err_e[r] = 0.f;
 
   // element e of a chunk: (kk, row) of A and (kk, col) of B, laid out so that
   // consecutive threads read consecutive addresses of the contiguous dimension
-  float ra[PA], rb[PB];
+  float ra[PA], rb[PB], rx = 0.f;
   auto fetch = [&](int k0) {
+    if (ext && tid < GK) {
+      const int gk = k0 + tid;
+      rx = gk < P.k ? Bm[gk * P.b.rs + (j0 + GT) * P.b.cs] : 0.f;
+    }
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
       const int e = tid + i * 256;
@@ -113,6 +124,7 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
     }
   };
   auto stage = [&](int buf) {
+    if (ext && tid < GK) Bs[buf][tid][GT] = rx;
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
       const int e = tid + i * 256;
@@ -161,6 +173,22 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
             acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
           }
         }
+      if (ext && tx == 0) {
+        const float be = Bs[buf][kk][GT];
+#pragma unroll
+        for (int r = 0; r < RM; ++r) {
+          if (PRECISE) {
+            const float p = __fmul_rn(a[r], be);
+            const float ep = __fmaf_rn(a[r], be, -p);
+            float sum, es;
+            two_sum(acc_e[r], p, sum, es);
+            acc_e[r] = sum;
+            err_e[r] = __fadd_rn(err_e[r], __fadd_rn(es, ep));
+          } else {
+            acc_e[r] = fmaf(a[r], be, acc_e[r]);
+          }
+        }
+      }
     }
     // the other buffer was last read before the previous barrier
     if (more) stage(buf ^ 1);
@@ -169,6 +197,13 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
   }
 
   float* Cm = P.c.p + z0 * P.c.b0 + z1 * P.c.b1;
+  auto put = [&](int i, int j, float v) {
+    if (P.causal && j > i) v = 0.f;
+    if (P.sx) v -= P.sx[z0 * P.sx_b0 + i * P.sx_rs + j] * P.ss[z0 * P.ss_b0 + i];
+    float* dst = Cm + i * P.c.rs + j * P.c.cs;
+    if (P.beta != 0.f) v += P.beta * *dst;
+    *dst = v;
+  };
 #pragma unroll
   for (int r = 0; r < RM; ++r) {
     const int i = i0 + ty * RM + r;
@@ -177,13 +212,9 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
     for (int c = 0; c < 4; ++c) {
       const int j = j0 + tx * 4 + c;
       if (j >= P.n) continue;
-      float v = PRECISE ? __fadd_rn(acc[r][c], err[r][c]) : acc[r][c];
-      if (P.causal && j > i) v = 0.f;
-      if (P.sx) v -= P.sx[z0 * P.sx_b0 + i * P.sx_rs + j] * P.ss[z0 * P.ss_b0 + i];
-      float* dst = Cm + i * P.c.rs + j * P.c.cs;
-      if (P.beta != 0.f) v += P.beta * *dst;
-      *dst = v;
+      put(i, j, PRECISE ? __fadd_rn(acc[r][c], err[r][c]) : acc[r][c]);
     }
+    if (ext && tx == 0) put(i, j0 + GT, PRECISE ? __fadd_rn(acc_e[r], err_e[r]) : acc_e[r]);
   }
 }
 
@@ -551,7 +582,10 @@ cudaError_t gemm(cudaStream_t s, bool precise, int m, int n, int k, Mat a, Mat b
     const int zc = (nz - z < 65535) ? nz - z : 65535;
     // rows per CTA tile: 16 or 32 for the short tiles of grouped slices
     const int rm = m <= 16 ? 1 : (m <= 32 ? 2 : 4), tm = 16 * rm;
-    dim3 grid((n + GT - 1) / GT, (m + tm - 1) / tm, zc);
+    // n = 64 q + 1 (the [V | 1] operands): the last 64-column tile takes the
+    // extra column
+    const int nx = (n > GT && n % GT == 1) ? n / GT : (n + GT - 1) / GT;
+    dim3 grid(nx, (m + tm - 1) / tm, zc);
     prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
     if (precise) {
       if (rm == 1) k_gemm<true, 1><<<grid, 256, 0, s>>>(P);
