@@ -71,3 +71,32 @@ def test_bidir_last_row_matches_causal(cuda_device):
     torch.cuda.synchronize()
     assert oracle.rel_l2(to64(ob[:, :, -1]), to64(oc[:, :, -1])) < TOL["bf16"]
     assert oracle.rel_l2(to64(Sb), to64(Sc)) < TOL["bf16"]
+
+
+@pytest.mark.slow
+def test_bidir_full_size_sampled_chains(cuda_device):
+    """The bench workload's shape (B8 H8 L4096 d64 M256 C1024 bf16) in the
+    non-causal form, in the launch configuration the benchmark times: the
+    oracle recomputes two chains (the chains are independent; Omega is shared).
+    dOmega, a sum over all chains, is checked on a second backward whose dout is
+    zero outside the sampled chains."""
+    w = W.WORKLOADS["L4096_bf16"]
+    x = W.make_inputs(w, device=cuda_device)
+    g = gpu_bidir(x, w.C, w.feature)
+    xc = cpu_inputs(x)
+    keep = [(0, 0), (w.B - 1, w.H - 1)]
+    refs = []
+    for b, h in keep:
+        sub_in = {n: (a[b:b + 1, h:h + 1] if a.ndim == 4 else a) for n, a in xc.items()}
+        ref = oracle_bidir(sub_in, w.C, w.feature)
+        refs.append(ref)
+        sub = {n: g[n][b:b + 1, h:h + 1] for n in ("out", "S_state", "z_state", "dq", "dk", "dv")}
+        compare(sub, ref, TOL[w.dtype], names=tuple(sub), where=f"bidir full chain ({b},{h})")
+    m = torch.zeros_like(x["dout"])
+    for b, h in keep:
+        m[b, h] = x["dout"][b, h]
+    om = x["omega"]
+    _, _, _, dom = slim.backward_bidir(x["q"], x["k"], x["v"], om, g["out"], m, g["S_state"],
+                                       g["z_state"], w.C, w.feature)
+    torch.cuda.synchronize()
+    assert oracle.rel_l2(to64(dom), sum(r["domega"] for r in refs)) <= TOL[w.dtype]

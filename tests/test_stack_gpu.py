@@ -80,3 +80,37 @@ def test_empty_sequence(cuda_device):
     torch.cuda.synchronize()
     assert y.numel() == 0 and dx.numel() == 0
     assert not S.any() and not z.any() and not dom.any()
+
+
+@pytest.mark.slow
+def test_stack_full_size_sampled_chains(cuda_device):
+    """Three layers on the bench workload's shape (B8 H8 L4096 d64 M256 C1024
+    bf16), as `bench.py --mode stack --layers 3` runs them: the oracle
+    recomputes two chains (chains are independent through every layer; the
+    Omegas are shared).  dOmega is checked on a second backward whose dy is
+    zero outside the sampled chains (the backward is linear in dy)."""
+    w = W.WORKLOADS["L4096_bf16"]
+    layers = 3
+    x = W.make_stack_inputs(w, layers, device=cuda_device)
+    y, S, z, Sl, zl = slim.stack_forward(x["x"], x["omegas"], w.C, w.feature)
+    dx, _ = slim.stack_backward(x["x"], x["omegas"], x["dy"], S, z, w.C, w.feature, S_lo=Sl,
+                                z_lo=zl)
+    keep = [(0, 0), (w.B - 1, w.H - 1)]
+    m = torch.zeros_like(x["dy"])
+    for b, h in keep:
+        m[b, h] = x["dy"][b, h]
+    _, dom = slim.stack_backward(x["x"], x["omegas"], m, S, z, w.C, w.feature, S_lo=Sl, z_lo=zl)
+    torch.cuda.synchronize()
+    omc = list(to64(x["omegas"]))
+    ref_dom = 0.0
+    for b, h in keep:
+        xc = to64(x["x"][b:b + 1, h:h + 1])
+        ry, rS, rz = oracle.oracle_stack_fwd(xc, omc, w.C, w.feature)
+        rdx, rdom = oracle.oracle_stack_bwd(xc, omc, to64(x["dy"][b:b + 1, h:h + 1]), rS, rz, w.C,
+                                            w.feature)
+        ref_dom = ref_dom + rdom
+        got = {"out": y[b:b + 1, h:h + 1], "S_state": S[:, b:b + 1, h:h + 1],
+               "z_state": z[:, b:b + 1, h:h + 1], "dq": dx[b:b + 1, h:h + 1]}
+        ref = {"out": ry, "S_state": rS, "z_state": rz, "dq": rdx}
+        compare(got, ref, TOL[w.dtype], names=tuple(got), where=f"stack full chain ({b},{h})")
+    assert oracle.rel_l2(to64(dom), ref_dom) <= TOL[w.dtype]
