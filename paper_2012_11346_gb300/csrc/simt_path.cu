@@ -62,138 +62,204 @@ struct GemmP {
   long long ss_b0;
 };
 
-// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z.  256 threads,
-// 64 x 64 outputs per CTA, 4 x 4 per thread.  PRECISE = false: fp32 FMA.
-// PRECISE = true (fp32 problems): every product and sum is error-free
-// transformed (FMA-based TwoProduct, Knuth TwoSum) and the errors are
-// accumulated beside the sum, so the result is as accurate as a sum computed
-// in twice the working precision and rounded once.  The backward pass needs
-// it: its contractions cancel (signed feature gradients summed against
-// Omega), which multiplies plain fp32 rounding error by 10-30.
-// RM rows per thread: a CTA computes a (16 RM) x 64 tile of C (RM = 4 for
-// most products, 1 or 2 when m is 16 or 32 -- the tiles of short slices).
-template <bool PRECISE, int RM>
-__global__ void __launch_bounds__(256) k_gemm(GemmP P) {
-  // two stages: chunk k0 + GK is read from global memory into registers while
-  // chunk k0 is multiplied out of shared memory, one barrier per chunk
-  constexpr int TM = 16 * RM;
-  __shared__ __align__(16) float As[2][GK][TM + 4];
-  __shared__ __align__(16) float Bs[2][GK][GT + 4];
-  constexpr int PA = TM * GK / 256, PB = GT * GK / 256;  // elements a thread stages
+// Multiply-add of a * b into (acc, err): plain FMA, or error-free (FMA-based
+// TwoProduct, Knuth TwoSum) with the errors accumulated beside the sum.
+template <bool PRECISE>
+__device__ __forceinline__ void mac(float a, float b, float& acc, float& err) {
+  if (PRECISE) {
+    const float p = __fmul_rn(a, b);
+    const float ep = __fmaf_rn(a, b, -p);
+    float sum, es;
+    two_sum(acc, p, sum, es);
+    acc = sum;
+    err = __fadd_rn(err, __fadd_rn(es, ep));
+  } else {
+    acc = fmaf(a, b, acc);
+  }
+}
+
+// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z.  A CTA
+// computes a TM x TN tile of C.  Its threads form KS groups of
+// (TM/4)(TN/4); group g takes the reduction chunks g, g + KS, ... and each of
+// its threads keeps 4 x 4 outputs, so a step of the reduction costs a thread
+// two 16-byte shared-memory loads for 16 multiply-adds.  The groups' partial
+// tiles are summed in group order at the end (a fixed order: the result does
+// not depend on scheduling).  Small tiles of long reductions -- the products
+// of 16- and 32-row tiles of short slices -- get several groups, so that a
+// launch has enough threads to fill the SMs.
+// PRECISE = false: fp32 FMA.  PRECISE = true (fp32 problems): every product
+// and sum is error-free transformed and the errors are accumulated beside the
+// sum, so the result is as accurate as a sum computed in twice the working
+// precision and rounded once.  The backward pass needs it: its contractions
+// cancel (signed feature gradients summed against Omega), which multiplies
+// plain fp32 rounding error by 10-30.
+template <bool PRECISE, int TM, int TN, int KS>
+__global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
+  // two stages per group: its next chunk is read from global memory into
+  // registers while its current chunk is multiplied out of shared memory, one
+  // barrier per step
+  constexpr int NT = (TM / 4) * (TN / 4);  // threads per group
+  constexpr int ASZ = 2 * GK * (TM + 4), BSZ = 2 * GK * (TN + 4);
+  constexpr int RED = PRECISE ? 2 * 17 : 17;  // floats a thread hands to group 0
+  constexpr int SMF = KS * (ASZ + BSZ);
+  static_assert(KS == 1 || (KS - 1) * NT * RED <= SMF, "reduction scratch");
+  __shared__ __align__(16) float sm[SMF];
+  const int tid = threadIdx.x, grp = tid / NT, lt = tid % NT;
+  float (*As)[GK][TM + 4] = reinterpret_cast<float (*)[GK][TM + 4]>(sm + grp * (ASZ + BSZ));
+  float (*Bs)[GK][TN + 4] = reinterpret_cast<float (*)[GK][TN + 4]>(sm + grp * (ASZ + BSZ) + ASZ);
+  constexpr int PA = TM * GK / NT, PB = TN * GK / NT;  // elements a thread stages
   const int z = blockIdx.z + P.zoff;
   const int z0 = z / P.nb1, z1 = z % P.nb1;
   const float* A = P.a.p + z0 * P.a.b0 + z1 * P.a.b1;
   const float* Bm = P.b.p + z0 * P.b.b0 + z1 * P.b.b1;
-  const int i0 = blockIdx.y * TM, j0 = blockIdx.x * GT;
-  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  const int i0 = blockIdx.y * TM, j0 = blockIdx.x * TN;
+  const int tx = lt % (TN / 4), ty = lt / (TN / 4);
   const bool a_kc = P.a.cs == 1, b_nc = P.b.cs == 1;
-  float acc[RM][4], err[RM][4];
+  float acc[4][4], err[4][4];
 #pragma unroll
-  for (int r = 0; r < RM; ++r)
+  for (int r = 0; r < 4; ++r)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[r][c] = err[r][c] = 0.f;
   // A last column tile of 65 columns (n = d + 1: the [V | 1] operands) takes
   // its 65th column itself, computed by the threads with tx = 0, instead of
   // leaving it to a CTA of its own.
-  const bool ext = P.n - j0 == GT + 1;
-  float acc_e[RM], err_e[RM];
+  const bool ext = TN == GT && P.n - j0 == GT + 1;
+  float acc_e[4], err_e[4];
 #pragma unroll
-  for (int r = 0; r < RM; ++r) acc_e[r] = err_e[r] = 0.f;
+  for (int r = 0; r < 4; ++r) acc_e[r] = err_e[r] = 0.f;
 
   // element e of a chunk: (kk, row) of A and (kk, col) of B, laid out so that
   // consecutive threads read consecutive addresses of the contiguous dimension
   float ra[PA], rb[PB], rx = 0.f;
   auto fetch = [&](int k0) {
-    if (ext && tid < GK) {
-      const int gk = k0 + tid;
+    if (ext && lt < GK) {
+      const int gk = k0 + lt;
       rx = gk < P.k ? Bm[gk * P.b.rs + (j0 + GT) * P.b.cs] : 0.f;
     }
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
-      const int e = tid + i * 256;
+      const int e = lt + i * NT;
       const int kk = a_kc ? e % GK : e / TM, r = a_kc ? e / GK : e % TM;
       const int gi = i0 + r, gk = k0 + kk;
       ra[i] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
     }
 #pragma unroll
     for (int i = 0; i < PB; ++i) {
-      const int e = tid + i * 256;
-      const int kb = b_nc ? e / GT : e % GK, cb = b_nc ? e % GT : e / GK;
+      const int e = lt + i * NT;
+      const int kb = b_nc ? e / TN : e % GK, cb = b_nc ? e % TN : e / GK;
       const int gkb = k0 + kb, gj = j0 + cb;
       rb[i] = (gkb < P.k && gj < P.n) ? Bm[gkb * P.b.rs + gj * P.b.cs] : 0.f;
     }
   };
   auto stage = [&](int buf) {
-    if (ext && tid < GK) Bs[buf][tid][GT] = rx;
+    if (ext && lt < GK) Bs[buf][lt][GT] = rx;
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
-      const int e = tid + i * 256;
+      const int e = lt + i * NT;
       As[buf][a_kc ? e % GK : e / TM][a_kc ? e / GK : e % TM] = ra[i];
     }
 #pragma unroll
     for (int i = 0; i < PB; ++i) {
-      const int e = tid + i * 256;
-      Bs[buf][b_nc ? e / GT : e % GK][b_nc ? e % GT : e / GK] = rb[i];
+      const int e = lt + i * NT;
+      Bs[buf][b_nc ? e / TN : e % GK][b_nc ? e % TN : e / GK] = rb[i];
     }
   };
 
-  fetch(0);
+  // group grp takes chunks grp, grp + KS, ...; every group runs the same
+  // number of steps (chunks past the end read as zeros)
+  const int steps = (P.k + GK * KS - 1) / (GK * KS);
+  fetch(grp * GK);
   stage(0);
   __syncthreads();
   int buf = 0;
-  for (int k0 = 0; k0 < P.k; k0 += GK) {
-    const bool more = k0 + GK < P.k;
-    if (more) fetch(k0 + GK);
+  for (int st = 0; st < steps; ++st) {
+    const bool more = st + 1 < steps;
+    if (more) fetch((grp + (st + 1) * KS) * GK);
 #pragma unroll
     for (int kk = 0; kk < GK; ++kk) {
-      float a[RM];
-      if constexpr (RM == 4) {
-        const float4 a4 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
-        a[0] = a4.x; a[1] = a4.y; a[2] = a4.z; a[3] = a4.w;
-      } else if constexpr (RM == 2) {
-        const float2 a2 = *reinterpret_cast<const float2*>(&As[buf][kk][ty * 2]);
-        a[0] = a2.x; a[1] = a2.y;
-      } else {
-        a[0] = As[buf][kk][ty];
-      }
-      float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
-      float b[4] = {b4.x, b4.y, b4.z, b4.w};
+      const float4 a4 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
+      const float a[4] = {a4.x, a4.y, a4.z, a4.w};
+      const float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
+      const float b[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
-      for (int r = 0; r < RM; ++r)
+      for (int r = 0; r < 4; ++r)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          if (PRECISE) {
-            const float p = __fmul_rn(a[r], b[c]);
-            const float ep = __fmaf_rn(a[r], b[c], -p);
-            float sum, es;
-            two_sum(acc[r][c], p, sum, es);
-            acc[r][c] = sum;
-            err[r][c] = __fadd_rn(err[r][c], __fadd_rn(es, ep));
-          } else {
-            acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
-          }
-        }
+        for (int c = 0; c < 4; ++c) mac<PRECISE>(a[r], b[c], acc[r][c], err[r][c]);
       if (ext && tx == 0) {
         const float be = Bs[buf][kk][GT];
 #pragma unroll
-        for (int r = 0; r < RM; ++r) {
-          if (PRECISE) {
-            const float p = __fmul_rn(a[r], be);
-            const float ep = __fmaf_rn(a[r], be, -p);
-            float sum, es;
-            two_sum(acc_e[r], p, sum, es);
-            acc_e[r] = sum;
-            err_e[r] = __fadd_rn(err_e[r], __fadd_rn(es, ep));
-          } else {
-            acc_e[r] = fmaf(a[r], be, acc_e[r]);
-          }
-        }
+        for (int r = 0; r < 4; ++r) mac<PRECISE>(a[r], be, acc_e[r], err_e[r]);
       }
     }
     // the other buffer was last read before the previous barrier
     if (more) stage(buf ^ 1);
     __syncthreads();
     buf ^= 1;
+  }
+
+  if (KS > 1) {
+    // groups 1..KS-1 hand their partial tiles to group 0 through shared
+    // memory (free after the loop's last barrier); element v of thread lt of
+    // group g at red[((g - 1) * RED + v) * NT + lt]
+    if (grp > 0) {
+      float* red = sm + (grp - 1) * RED * NT + lt;
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          red[(4 * r + c) * NT] = acc[r][c];
+          if (PRECISE) red[(17 + 4 * r + c) * NT] = err[r][c];
+        }
+    }
+    __syncthreads();
+    if (grp == 0) {
+#pragma unroll 1
+      for (int g = 1; g < KS; ++g) {
+        const float* red = sm + (g - 1) * RED * NT + lt;
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const float v = red[(4 * r + c) * NT];
+            if (PRECISE) {
+              float sum, es;
+              two_sum(acc[r][c], v, sum, es);
+              acc[r][c] = sum;
+              err[r][c] = __fadd_rn(err[r][c], __fadd_rn(es, red[(17 + 4 * r + c) * NT]));
+            } else {
+              acc[r][c] += v;
+            }
+          }
+      }
+    }
+    if (ext) {
+      // the extra column, row by row through slot 16 (and 33)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        __syncthreads();
+        if (grp > 0 && tx == 0) {
+          float* red = sm + (grp - 1) * RED * NT + lt;
+          red[16 * NT] = acc_e[r];
+          if (PRECISE) red[33 * NT] = err_e[r];
+        }
+        __syncthreads();
+        if (grp == 0 && tx == 0) {
+#pragma unroll 1
+          for (int g = 1; g < KS; ++g) {
+            const float* red = sm + (g - 1) * RED * NT + lt;
+            if (PRECISE) {
+              float sum, es;
+              two_sum(acc_e[r], red[16 * NT], sum, es);
+              acc_e[r] = sum;
+              err_e[r] = __fadd_rn(err_e[r], __fadd_rn(es, red[33 * NT]));
+            } else {
+              acc_e[r] += red[16 * NT];
+            }
+          }
+        }
+      }
+    }
+    if (grp > 0) return;
   }
 
   float* Cm = P.c.p + z0 * P.c.b0 + z1 * P.c.b1;
@@ -205,8 +271,8 @@ __global__ void __launch_bounds__(256) k_gemm(GemmP P) {
     *dst = v;
   };
 #pragma unroll
-  for (int r = 0; r < RM; ++r) {
-    const int i = i0 + ty * RM + r;
+  for (int r = 0; r < 4; ++r) {
+    const int i = i0 + ty * 4 + r;
     if (i >= P.m) continue;
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
@@ -580,22 +646,39 @@ cudaError_t gemm(cudaStream_t s, bool precise, int m, int n, int k, Mat a, Mat b
   for (int z = 0; z < nz; z += 65535) {
     GemmP P{m, n, k, a, b, c, nb1, z, beta, causal, sx, sx_b0, sx_rs, ss, ss_b0};
     const int zc = (nz - z < 65535) ? nz - z : 65535;
-    // rows per CTA tile: 16 or 32 for the short tiles of grouped slices
-    const int rm = m <= 16 ? 1 : (m <= 32 ? 2 : 4), tm = 16 * rm;
+    // rows per CTA tile: 16 or 32 for the short tiles of grouped slices;
+    // columns: 16 for products only that wide
+    const int tn = n <= 16 ? 16 : GT;
+    const int tm = (m <= 16 || tn == 16) ? 16 : (m <= 32 ? 32 : 64);
+    // reduction groups per CTA for the small tiles, when the reduction has
+    // at least two chunks per group
+    const int want = tn == 16 ? 8 : (tm == 16 ? 4 : (tm == 32 ? 2 : 1));
+    const int ks = (k >= 2 * GK * want) ? want : 1;
     // n = 64 q + 1 (the [V | 1] operands): the last 64-column tile takes the
     // extra column
-    const int nx = (n > GT && n % GT == 1) ? n / GT : (n + GT - 1) / GT;
+    const int nx = (tn == GT && n > GT && n % GT == 1) ? n / GT : (n + tn - 1) / tn;
     dim3 grid(nx, (m + tm - 1) / tm, zc);
     prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
-    if (precise) {
-      if (rm == 1) k_gemm<true, 1><<<grid, 256, 0, s>>>(P);
-      else if (rm == 2) k_gemm<true, 2><<<grid, 256, 0, s>>>(P);
-      else k_gemm<true, 4><<<grid, 256, 0, s>>>(P);
-    } else {
-      if (rm == 1) k_gemm<false, 1><<<grid, 256, 0, s>>>(P);
-      else if (rm == 2) k_gemm<false, 2><<<grid, 256, 0, s>>>(P);
-      else k_gemm<false, 4><<<grid, 256, 0, s>>>(P);
+    const int nthr = (tm / 4) * (tn / 4) * ks;
+#define SLIM_GEMM_LAUNCH(PR)                                                          \
+    if (tn == 16) {                                                                   \
+      if (ks > 1) k_gemm<PR, 16, 16, 8><<<grid, nthr, 0, s>>>(P);                     \
+      else k_gemm<PR, 16, 16, 1><<<grid, nthr, 0, s>>>(P);                            \
+    } else if (tm == 16) {                                                            \
+      if (ks > 1) k_gemm<PR, 16, GT, 4><<<grid, nthr, 0, s>>>(P);                     \
+      else k_gemm<PR, 16, GT, 1><<<grid, nthr, 0, s>>>(P);                            \
+    } else if (tm == 32) {                                                            \
+      if (ks > 1) k_gemm<PR, 32, GT, 2><<<grid, nthr, 0, s>>>(P);                     \
+      else k_gemm<PR, 32, GT, 1><<<grid, nthr, 0, s>>>(P);                            \
+    } else {                                                                          \
+      k_gemm<PR, 64, GT, 1><<<grid, nthr, 0, s>>>(P);                                 \
     }
+    if (precise) {
+      SLIM_GEMM_LAUNCH(true)
+    } else {
+      SLIM_GEMM_LAUNCH(false)
+    }
+#undef SLIM_GEMM_LAUNCH
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -644,19 +727,23 @@ cudaError_t tile_deltas(cudaStream_t s, const Geo& g, const Ws& w) {
               omat(w.delta, nt * M * dp, M * dp, dp, 1), g.chains, g.nt, 0.f, 0);
 }
 
-// A_t = tril(phiQ_t phiK_t^T); [num | den] = phiQ_t P_t + A_t [V_t | 1]
-cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w) {
+// A_t = tril(phiQ_t phiK_t^T); [num | den] = phiQ_t P_t + A_t [V_t | 1].
+// den_only: the backward, which has the forward's output, needs only the
+// denominator column (phiQ_t z_t + rowsum A_t), not num.
+cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w, bool den_only) {
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
+  const long long c0 = den_only ? g.d : 0;  // first column computed
+  const int nc = den_only ? 1 : g.dp;
   cudaError_t e = gemm(s, g.precise, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                        mat(w.phiK, Cp * M, T * M, 1, M), omat(w.A, nt * T * T, T * T, T, 1),
                        g.chains, g.nt, 0.f, 1);
   if (e != cudaSuccess) return e;
-  e = gemm(s, g.precise, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
-           mat(w.delta, nt * M * dp, M * dp, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
-           g.chains, g.nt, 0.f, 0);
+  e = gemm(s, g.precise, g.T, nc, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+           mat(w.delta + c0, nt * M * dp, M * dp, dp, 1),
+           omat(w.numden + c0, Cp * dp, T * dp, dp, 1), g.chains, g.nt, 0.f, 0);
   if (e != cudaSuccess) return e;
-  return gemm(s, g.precise, g.T, g.dp, g.T, mat(w.A, nt * T * T, T * T, T, 1),
-              mat(w.Vx, Cp * dp, T * dp, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
+  return gemm(s, g.precise, g.T, nc, g.T, mat(w.A, nt * T * T, T * T, T, 1),
+              mat(w.Vx + c0, Cp * dp, T * dp, dp, 1), omat(w.numden + c0, Cp * dp, T * dp, dp, 1),
               g.chains, g.nt, 1.f, 0);
 }
 
@@ -688,7 +775,7 @@ slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
     SLIM_TRY(tile_deltas(s, g, w));
     SLIM_TRY(scan(s, g, w.delta, w.st_hi, w.st_lo, SCAN_FWD));
-    SLIM_TRY(scores_and_readout(s, g, w));
+    SLIM_TRY(scores_and_readout(s, g, w, false));
     { prof::Scope ps(prof::K_FINALIZE, s, 0.0, (double)g.chains * b * g.d * sizeof(T));
     k_finalize_out<T><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(
         w.numden, (T*)out, p.L, g.d, a, b, g.Cp, g.chains); }
@@ -737,7 +824,7 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
     SLIM_TRY(tile_deltas(s, g, w));
     SLIM_TRY(scan(s, g, w.delta, w.st_hi, w.st_lo, SCAN_ROLLBACK));
-    SLIM_TRY(scores_and_readout(s, g, w));
+    SLIM_TRY(scores_and_readout(s, g, w, true));
     { prof::Scope ps(prof::K_DSTAT, s);
     k_dstat<<<blocks((long long)g.chains * Cp * dp), 256, 0, s>>>(w.numden, w.dout32, w.rowdot, w.W,
                                                                g.d, b, g.Cp, g.chains); }
@@ -950,8 +1037,9 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
-                  mat(w.st_hi, M * dp, 0, dp, 1), omat(w.numden, Cp * dp, T * dp, dp, 1),
+    // den = g(Q) z: the only column of [num | den] the gradients need
+    SLIM_TRY(gemm(s, g.precise, g.T, 1, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+                  mat(w.st_hi + d, M * dp, 0, dp, 1), omat(w.numden + d, Cp * dp, T * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_DSTAT, s);
     k_dstat<<<blocks((long long)g.chains * Cp * dp), 256, 0, s>>>(w.numden, w.dout32, w.rowdot,
