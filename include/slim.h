@@ -61,9 +61,9 @@
  *   - Outputs are written in `dtype` rounded to nearest even.  The state
  *     carried between slices depends on the kernels serving the problem (see
  *     slim_path_for).  The fp32-compute kernels carry it as an fp32
- *     value/error pair (TwoSum) and accumulate every contraction of fp32
- *     problems in compensated fp32 (error-free products and sums); their
- *     residual outputs (S_state_lo, z_state_lo) hold the pair's low part.
+ *     value/error pair (TwoSum) and accumulate the contractions in fp32
+ *     FMA; their residual outputs (S_state_lo, z_state_lo) hold the pair's
+ *     low part.
  *     The tensor-core kernels (bf16) chain plain fp32 prefixes from tile to
  *     tile, accumulate in fp32, and write zero residuals.
  *   - Supported: d in {16, 32, 64, 128}; M a multiple of 16 in [16, 256];

@@ -62,24 +62,8 @@ struct GemmP {
   long long ss_b0;
 };
 
-// Multiply-add of a * b into (acc, err): plain FMA, or error-free (FMA-based
-// TwoProduct, Knuth TwoSum) with the errors accumulated beside the sum.
-template <bool PRECISE>
-__device__ __forceinline__ void mac(float a, float b, float& acc, float& err) {
-  if (PRECISE) {
-    const float p = __fmul_rn(a, b);
-    const float ep = __fmaf_rn(a, b, -p);
-    float sum, es;
-    two_sum(acc, p, sum, es);
-    acc = sum;
-    err = __fadd_rn(err, __fadd_rn(es, ep));
-  } else {
-    acc = fmaf(a, b, acc);
-  }
-}
-
-// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z.  A CTA
-// computes a TM x TN tile of C.  Its threads form KS groups of
+// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z, in fp32 FMA.
+// A CTA computes a TM x TN tile of C.  Its threads form KS groups of
 // (TM/4)(TN/4); group g takes the reduction chunks g, g + KS, ... and each of
 // its threads keeps 4 x 4 outputs, so a step of the reduction costs a thread
 // two 16-byte shared-memory loads for 16 multiply-adds.  The groups' partial
@@ -87,20 +71,17 @@ __device__ __forceinline__ void mac(float a, float b, float& acc, float& err) {
 // not depend on scheduling).  Small tiles of long reductions -- the products
 // of 16- and 32-row tiles of short slices -- get several groups, so that a
 // launch has enough threads to fill the SMs.
-// PRECISE = false: fp32 FMA.  PRECISE = true (fp32 problems): every product
-// and sum is error-free transformed and the errors are accumulated beside the
-// sum, so the result is as accurate as a sum computed in twice the working
-// precision and rounded once.  The backward pass needs it: its contractions
-// cancel (signed feature gradients summed against Omega), which multiplies
-// plain fp32 rounding error by 10-30.
-template <bool PRECISE, int TM, int TN, int KS>
+// Plain fp32 accumulation holds the fp32 problems' 1e-5 bound: on the L=8192
+// ReLU workload dq is within 3.5e-7 of the fp64 oracle (error-free
+// TwoProduct/TwoSum accumulation gave 1.8e-7 at 2.7x the time).
+template <int TM, int TN, int KS>
 __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
   // two stages per group: its next chunk is read from global memory into
   // registers while its current chunk is multiplied out of shared memory, one
   // barrier per step
   constexpr int NT = (TM / 4) * (TN / 4);  // threads per group
   constexpr int ASZ = 2 * GK * (TM + 4), BSZ = 2 * GK * (TN + 4);
-  constexpr int RED = PRECISE ? 2 * 17 : 17;  // floats a thread hands to group 0
+  constexpr int RED = 17;  // floats a thread hands to group 0
   constexpr int SMF = KS * (ASZ + BSZ);
   static_assert(KS == 1 || (KS - 1) * NT * RED <= SMF, "reduction scratch");
   __shared__ __align__(16) float sm[SMF];
@@ -115,18 +96,18 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
   const int i0 = blockIdx.y * TM, j0 = blockIdx.x * TN;
   const int tx = lt % (TN / 4), ty = lt / (TN / 4);
   const bool a_kc = P.a.cs == 1, b_nc = P.b.cs == 1;
-  float acc[4][4], err[4][4];
+  float acc[4][4];
 #pragma unroll
   for (int r = 0; r < 4; ++r)
 #pragma unroll
-    for (int c = 0; c < 4; ++c) acc[r][c] = err[r][c] = 0.f;
+    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
   // A last column tile of 65 columns (n = d + 1: the [V | 1] operands) takes
   // its 65th column itself, computed by the threads with tx = 0, instead of
   // leaving it to a CTA of its own.
   const bool ext = TN == GT && P.n - j0 == GT + 1;
-  float acc_e[4], err_e[4];
+  float acc_e[4];
 #pragma unroll
-  for (int r = 0; r < 4; ++r) acc_e[r] = err_e[r] = 0.f;
+  for (int r = 0; r < 4; ++r) acc_e[r] = 0.f;
 
   // element e of a chunk: (kk, row) of A and (kk, col) of B, laid out so that
   // consecutive threads read consecutive addresses of the contiguous dimension
@@ -184,11 +165,11 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
 #pragma unroll
       for (int r = 0; r < 4; ++r)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) mac<PRECISE>(a[r], b[c], acc[r][c], err[r][c]);
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
       if (ext && tx == 0) {
         const float be = Bs[buf][kk][GT];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) mac<PRECISE>(a[r], be, acc_e[r], err_e[r]);
+        for (int r = 0; r < 4; ++r) acc_e[r] = fmaf(a[r], be, acc_e[r]);
       }
     }
     // the other buffer was last read before the previous barrier
@@ -206,10 +187,7 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
 #pragma unroll
       for (int r = 0; r < 4; ++r)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          red[(4 * r + c) * NT] = acc[r][c];
-          if (PRECISE) red[(17 + 4 * r + c) * NT] = err[r][c];
-        }
+        for (int c = 0; c < 4; ++c) red[(4 * r + c) * NT] = acc[r][c];
     }
     __syncthreads();
     if (grp == 0) {
@@ -219,43 +197,19 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
 #pragma unroll
         for (int r = 0; r < 4; ++r)
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const float v = red[(4 * r + c) * NT];
-            if (PRECISE) {
-              float sum, es;
-              two_sum(acc[r][c], v, sum, es);
-              acc[r][c] = sum;
-              err[r][c] = __fadd_rn(err[r][c], __fadd_rn(es, red[(17 + 4 * r + c) * NT]));
-            } else {
-              acc[r][c] += v;
-            }
-          }
+          for (int c = 0; c < 4; ++c) acc[r][c] += red[(4 * r + c) * NT];
       }
     }
     if (ext) {
-      // the extra column, row by row through slot 16 (and 33)
+      // the extra column, row by row through slot 16
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
         __syncthreads();
-        if (grp > 0 && tx == 0) {
-          float* red = sm + (grp - 1) * RED * NT + lt;
-          red[16 * NT] = acc_e[r];
-          if (PRECISE) red[33 * NT] = err_e[r];
-        }
+        if (grp > 0 && tx == 0) sm[(grp - 1) * RED * NT + 16 * NT + lt] = acc_e[r];
         __syncthreads();
         if (grp == 0 && tx == 0) {
 #pragma unroll 1
-          for (int g = 1; g < KS; ++g) {
-            const float* red = sm + (g - 1) * RED * NT + lt;
-            if (PRECISE) {
-              float sum, es;
-              two_sum(acc_e[r], red[16 * NT], sum, es);
-              acc_e[r] = sum;
-              err_e[r] = __fadd_rn(err_e[r], __fadd_rn(es, red[33 * NT]));
-            } else {
-              acc_e[r] += red[16 * NT];
-            }
-          }
+          for (int g = 1; g < KS; ++g) acc_e[r] += sm[(g - 1) * RED * NT + 16 * NT + lt];
         }
       }
     }
@@ -278,9 +232,9 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
     for (int c = 0; c < 4; ++c) {
       const int j = j0 + tx * 4 + c;
       if (j >= P.n) continue;
-      put(i, j, PRECISE ? __fadd_rn(acc[r][c], err[r][c]) : acc[r][c]);
+      put(i, j, acc[r][c]);
     }
-    if (ext && tx == 0) put(i, j0 + GT, PRECISE ? __fadd_rn(acc_e[r], err_e[r]) : acc_e[r]);
+    if (ext && tx == 0) put(i, j0 + GT, acc_e[r]);
   }
 }
 
@@ -553,7 +507,6 @@ constexpr int kSplitCtas = 304;   // dOmega contractions: about two waves of 152
 struct Geo {
   int chains, d, dp, M, Cs, T, nt, Cp, N;  // Cs: rows per launch sequence (a slice or a group)
   int ks;        // row splits of the dOmega contractions (divides nt)
-  bool precise;  // fp32 problems: compensated contractions
 };
 
 Geo geometry(const Problem& p) {
@@ -588,7 +541,6 @@ Geo geometry(const Problem& p) {
   g.ks = 1;
   for (int k = 2; k <= g.nt && k <= want; ++k)
     if (g.nt % k == 0) g.ks = k;
-  g.precise = p.dtype == SLIM_F32;
   return g;
 }
 
@@ -638,7 +590,7 @@ OutMat omat(float* p, long long b0, long long b1, long long rs, long long cs) {
   return OutMat{p, b0, b1, rs, cs};
 }
 
-cudaError_t gemm(cudaStream_t s, bool precise, int m, int n, int k, Mat a, Mat b, OutMat c,
+cudaError_t gemm(cudaStream_t s, int m, int n, int k, Mat a, Mat b, OutMat c,
                  int nb0, int nb1,
                  float beta, int causal, const float* sx = nullptr, long long sx_b0 = 0,
                  long long sx_rs = 0, const float* ss = nullptr, long long ss_b0 = 0) {
@@ -660,25 +612,18 @@ cudaError_t gemm(cudaStream_t s, bool precise, int m, int n, int k, Mat a, Mat b
     dim3 grid(nx, (m + tm - 1) / tm, zc);
     prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
     const int nthr = (tm / 4) * (tn / 4) * ks;
-#define SLIM_GEMM_LAUNCH(PR)                                                          \
-    if (tn == 16) {                                                                   \
-      if (ks > 1) k_gemm<PR, 16, 16, 8><<<grid, nthr, 0, s>>>(P);                     \
-      else k_gemm<PR, 16, 16, 1><<<grid, nthr, 0, s>>>(P);                            \
-    } else if (tm == 16) {                                                            \
-      if (ks > 1) k_gemm<PR, 16, GT, 4><<<grid, nthr, 0, s>>>(P);                     \
-      else k_gemm<PR, 16, GT, 1><<<grid, nthr, 0, s>>>(P);                            \
-    } else if (tm == 32) {                                                            \
-      if (ks > 1) k_gemm<PR, 32, GT, 2><<<grid, nthr, 0, s>>>(P);                     \
-      else k_gemm<PR, 32, GT, 1><<<grid, nthr, 0, s>>>(P);                            \
-    } else {                                                                          \
-      k_gemm<PR, 64, GT, 1><<<grid, nthr, 0, s>>>(P);                                 \
-    }
-    if (precise) {
-      SLIM_GEMM_LAUNCH(true)
+    if (tn == 16) {
+      if (ks > 1) k_gemm<16, 16, 8><<<grid, nthr, 0, s>>>(P);
+      else k_gemm<16, 16, 1><<<grid, nthr, 0, s>>>(P);
+    } else if (tm == 16) {
+      if (ks > 1) k_gemm<16, GT, 4><<<grid, nthr, 0, s>>>(P);
+      else k_gemm<16, GT, 1><<<grid, nthr, 0, s>>>(P);
+    } else if (tm == 32) {
+      if (ks > 1) k_gemm<32, GT, 2><<<grid, nthr, 0, s>>>(P);
+      else k_gemm<32, GT, 1><<<grid, nthr, 0, s>>>(P);
     } else {
-      SLIM_GEMM_LAUNCH(false)
+      k_gemm<64, GT, 1><<<grid, nthr, 0, s>>>(P);
     }
-#undef SLIM_GEMM_LAUNCH
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -723,7 +668,7 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
 // Delta_t = phiK_t^T [V_t | 1]  (M x dp per tile)
 cudaError_t tile_deltas(cudaStream_t s, const Geo& g, const Ws& w) {
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
-  return gemm(s, g.precise, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
+  return gemm(s, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
               omat(w.delta, nt * M * dp, M * dp, dp, 1), g.chains, g.nt, 0.f, 0);
 }
 
@@ -734,15 +679,15 @@ cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w, bool d
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
   const long long c0 = den_only ? g.d : 0;  // first column computed
   const int nc = den_only ? 1 : g.dp;
-  cudaError_t e = gemm(s, g.precise, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+  cudaError_t e = gemm(s, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                        mat(w.phiK, Cp * M, T * M, 1, M), omat(w.A, nt * T * T, T * T, T, 1),
                        g.chains, g.nt, 0.f, 1);
   if (e != cudaSuccess) return e;
-  e = gemm(s, g.precise, g.T, nc, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+  e = gemm(s, g.T, nc, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
            mat(w.delta + c0, nt * M * dp, M * dp, dp, 1),
            omat(w.numden + c0, Cp * dp, T * dp, dp, 1), g.chains, g.nt, 0.f, 0);
   if (e != cudaSuccess) return e;
-  return gemm(s, g.precise, g.T, nc, g.T, mat(w.A, nt * T * T, T * T, T, 1),
+  return gemm(s, g.T, nc, g.T, mat(w.A, nt * T * T, T * T, T, 1),
               mat(w.Vx + c0, Cp * dp, T * dp, dp, 1), omat(w.numden + c0, Cp * dp, T * dp, dp, 1),
               g.chains, g.nt, 1.f, 0);
 }
@@ -830,33 +775,33 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
                                                                g.d, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
     // dA_t = tril(W_t [V_t | 1]^T)
-    SLIM_TRY(gemm(s, g.precise, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.Vx, Cp * dp, T * dp, 1, dp), omat(w.dA, nt * T * T, T * T, T, 1),
                   g.chains, g.nt, 0.f, 1));
     // dphiQ = W_t P_t^T + dA_t phiK_t
-    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.delta, nt * M * dp, M * dp, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
+    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
                   mat(w.phiK, Cp * M, T * M, M, 1), omat(w.dphiQ, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 1.f, 0));
     // Gd_t = phiQ_t^T W_t, then G_t = G + sum_{t' > t} Gd_t'
-    SLIM_TRY(gemm(s, g.precise, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+    SLIM_TRY(gemm(s, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
     // dphiK = dA_t^T phiQ_t + [V_t | 1] G_t^T
-    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
+    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
                   mat(w.phiQ, Cp * M, T * M, M, 1), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
                   mat(w.gdelta, nt * M * dp, M * dp, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 1.f, 0));
     // dV = A_t^T dnum + phiK_t G_t(S)
-    SLIM_TRY(gemm(s, g.precise, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
+    SLIM_TRY(gemm(s, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
                   mat(w.gdelta, nt * M * dp, M * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1),
                   g.chains, g.nt, 1.f, 0));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
@@ -894,14 +839,14 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(cudaGetLastError());
     const bool ex = p.feature == SLIM_FEAT_EXP;
     // dX = u Omega (- x sum u for the exp map)
-    SLIM_TRY(gemm(s, g.precise, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
                   omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xq : nullptr,
                   Cp * d, d, w.usum_q, Cp));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
     k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dq, p.L, g.d,
                                                                       a, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
-    SLIM_TRY(gemm(s, g.precise, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
                   omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xk : nullptr,
                   Cp * d, d, w.usum_k, Cp));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
@@ -910,10 +855,10 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(cudaGetLastError());
     // dOmega partials per chain and row split: u_q^T x_q + u_k^T x_k
     const long long kc = (long long)(g.nt / g.ks) * T, ks = g.ks;
-    SLIM_TRY(gemm(s, g.precise, g.M, g.d, (int)kc, mat(w.dphiQ, Cp * M, kc * M, 1, M),
+    SLIM_TRY(gemm(s, g.M, g.d, (int)kc, mat(w.dphiQ, Cp * M, kc * M, 1, M),
                   mat(w.Xq, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains,
                   g.ks, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.M, g.d, (int)kc, mat(w.dphiK, Cp * M, kc * M, 1, M),
+    SLIM_TRY(gemm(s, g.M, g.d, (int)kc, mat(w.dphiK, Cp * M, kc * M, 1, M),
                   mat(w.Xk, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains,
                   g.ks, 1.f, 0));
     { prof::Scope ps(prof::K_REDUCE, s);
@@ -959,12 +904,12 @@ cudaError_t side_vjp(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w
                                                             (float)(1.0 / sqrt((double)g.M))); }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const bool ex = p.feature == SLIM_FEAT_EXP;
-    e = gemm(s, g.precise, g.Cp, g.d, g.M, mat(dphi, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    e = gemm(s, g.Cp, g.d, g.M, mat(dphi, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
              omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? X : nullptr, Cp * d, d,
              usum, Cp);
     if (e != cudaSuccess) return e;
     const long long kc = (long long)(g.nt / g.ks) * g.T, ks = g.ks;
-    e = gemm(s, g.precise, g.M, g.d, (int)kc, mat(dphi, Cp * M, kc * M, 1, M),
+    e = gemm(s, g.M, g.d, (int)kc, mat(dphi, Cp * M, kc * M, 1, M),
              mat(X, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains, g.ks,
              0.f, 0);
     if (e != cudaSuccess) return e;
@@ -1005,7 +950,7 @@ slim_status fwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, TT * M, M, 1),
+    SLIM_TRY(gemm(s, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, TT * M, M, 1),
                   mat(w.st_hi, M * dp, 0, dp, 1), omat(w.numden, Cp * dp, TT * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_FINALIZE, s, 0.0, (double)g.chains * b * g.d * sizeof(T));
@@ -1038,17 +983,17 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
     // den = g(Q) z: the only column of [num | den] the gradients need
-    SLIM_TRY(gemm(s, g.precise, g.T, 1, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.T, 1, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                   mat(w.st_hi + d, M * dp, 0, dp, 1), omat(w.numden + d, Cp * dp, T * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_DSTAT, s);
     k_dstat<<<blocks((long long)g.chains * Cp * dp), 256, 0, s>>>(w.numden, w.dout32, w.rowdot,
                                                                   w.W, g.d, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
-    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.st_hi, M * dp, 0, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+    SLIM_TRY(gemm(s, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
@@ -1058,10 +1003,10 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
                   mat(w.g_hi, M * dp, 0, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.precise, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
                   mat(w.g_hi, M * dp, 0, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
                   g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
