@@ -242,27 +242,52 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
 // Loads rows [a, a+b) of every chain, converts to fp32, applies the feature
 // map.  Rows b..Cp-1 of the padded tile are zero everywhere (including the
 // ones column of [V | 1]), so they add nothing to any contraction.
-constexpr int kPrepFeat = 128;    // features per projection chunk
-constexpr int kPrepStride = 130;  // omT row stride in floats (8-byte rows, 2-way bank spread)
+constexpr int kPrepFeat = 128;  // features per projection chunk
+
+// Omega in the layout the projections read, built once per call: chunk c of
+// kPrepFeat features is a [d][kPrepFeat] block (feature index contiguous,
+// zero past M), and omn[m] = |omega_m|.
+__global__ void k_omega_prep(const float* __restrict__ omega, int M, int d, float* omT,
+                             float* omn) {
+  const int nch = (M + kPrepFeat - 1) / kPrepFeat;
+  const long long n = (long long)nch * d * kPrepFeat;
+  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int mm = (int)(e % kPrepFeat);
+    const long long cj = e / kPrepFeat;
+    const int j = (int)(cj % d), c = (int)(cj / d);
+    const int m = c * kPrepFeat + mm;
+    omT[e] = m < M ? omega[(size_t)m * d + j] : 0.f;
+  }
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) / 32, lane = threadIdx.x % 32;
+  const int nw = gridDim.x * blockDim.x / 32;
+  for (int m = warp; m < M; m += nw) {
+    float t = 0.f;
+    for (int j = lane; j < d; j += 32) t = fmaf(omega[(size_t)m * d + j], omega[(size_t)m * d + j], t);
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) omn[m] = sqrtf(t);
+  }
+}
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_prep(
     const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
     const T* __restrict__ dout, const T* __restrict__ out, const float* __restrict__ omega,
-    int L, int d, int M, int a, int b, int Cp, int feature, float inv_sqrt_m,
+    const float* __restrict__ omT_g, const float* __restrict__ omn_g,
+    int L, int ld, int M, int a, int b, int Cp, int feature, float inv_sqrt_m,
     float* Xq, float* Xk, float* Vx, float* phiQ, float* phiK, float* dout32, float* rowdot) {
   extern __shared__ __align__(16) float sm[];
   constexpr int R = 16;            // rows per CTA (q and k -> 32 vectors)
-  float* xs = sm;                  // [32][d]
+  const int d = 1 << ld;           // d is a power of two (16 .. 128)
+  float* omT = sm;                 // [d][kPrepFeat]: a chunk of Omega, transposed
+  float* xs = omT + d * kPrepFeat; // [32][d]
   float* xn2 = xs + 32 * d;        // [32]
-  float* omT = xn2 + 32;           // [d][kPrepStride]: a chunk of Omega, transposed
-  float* omn = omT + d * kPrepStride;  // [kPrepFeat]
   const int c = blockIdx.y, r0 = blockIdx.x * R, tid = threadIdx.x;
   const int dp = d + 1;
   const size_t rowbase = (size_t)c * L + a;
 
   for (int e = tid; e < R * d; e += 256) {
-    int rr = e / d, j = e % d, r = r0 + rr;
+    const int rr = e >> ld, j = e & (d - 1), r = r0 + rr;
     float xq = 0.f, xk = 0.f, xv = 0.f;
     if (r < b) {
       size_t g = (rowbase + r) * d + j;
@@ -305,8 +330,9 @@ __global__ void __launch_bounds__(256) k_prep(
 
   if (feature == SLIM_FEAT_SQUARE) {
     // elementwise quadratic map g(x)_i = x_i^2, M = d (Sec. 4): no Omega
+    __syncthreads();
     for (int e = tid; e < 2 * R * d; e += 256) {
-      const int vec = e / d, m = e % d, r = r0 + vec % R;
+      const int vec = e >> ld, m = e & (d - 1), r = r0 + vec % R;
       const float x = xs[vec * d + m];
       float* dst = (vec < R) ? phiQ : phiK;
       dst[((size_t)c * Cp + r) * M + m] = (r < b) ? x * x : 0.f;
@@ -323,15 +349,10 @@ __global__ void __launch_bounds__(256) k_prep(
   const int f = tid % 64, grp = tid / 64;
   for (int m0 = 0; m0 < M; m0 += kPrepFeat) {
     __syncthreads();
-    for (int e = tid; e < kPrepFeat * d; e += 256) {
-      int mm = e / d, j = e % d;
-      omT[j * kPrepStride + mm] = (m0 + mm < M) ? omega[(size_t)(m0 + mm) * d + j] : 0.f;
-    }
-    __syncthreads();
-    if (tid < kPrepFeat) {
-      float s = 0.f;
-      for (int j = 0; j < d; ++j) s = fmaf(omT[j * kPrepStride + tid], omT[j * kPrepStride + tid], s);
-      omn[tid] = sqrtf(s);
+    {
+      const float4* src = reinterpret_cast<const float4*>(omT_g + (size_t)(m0 / kPrepFeat) * d * kPrepFeat);
+      float4* dst = reinterpret_cast<float4*>(omT);
+      for (int e = tid; e < d * kPrepFeat / 4; e += 256) dst[e] = src[e];
     }
     __syncthreads();
     float acc[8][2];
@@ -341,7 +362,7 @@ __global__ void __launch_bounds__(256) k_prep(
       float2 o[4];
 #pragma unroll
       for (int t = 0; t < 4; ++t)
-        o[t] = *reinterpret_cast<const float2*>(&omT[(j + t) * kPrepStride + 2 * f]);
+        o[t] = *reinterpret_cast<const float2*>(&omT[(j + t) * kPrepFeat + 2 * f]);
 #pragma unroll
       for (int vv = 0; vv < 8; ++vv) {
         const float4 x = *reinterpret_cast<const float4*>(&xs[(grp * 8 + vv) * d + j]);
@@ -355,34 +376,34 @@ __global__ void __launch_bounds__(256) k_prep(
         acc[vv][1] = fmaf(x.w, o[3].y, acc[vv][1]);
       }
     }
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int mm = 2 * f + h, m = m0 + mm;
-      if (m >= M) continue;
+    // features m0 + 2f and m0 + 2f + 1 (M is even: both exist or neither)
+    const int m = m0 + 2 * f;
+    if (m < M) {
 #pragma unroll
       for (int vv = 0; vv < 8; ++vv) {
         const int vec = grp * 8 + vv;
         const int rr = vec % R, r = r0 + rr;
-        const float dot = acc[vv][h];
-        float phi = 0.f;
+        float phi[2] = {0.f, 0.f};
         if (r < b) {
-          if (feature == SLIM_FEAT_EXP) {
-            phi = expf(dot - 0.5f * xn2[vec]) * inv_sqrt_m;
-          } else {
-            // The sign of omega.x decides ReLU's branch; near zero it is
-            // recomputed in fp64 so the decision is the exact one.
-            if (fabsf(dot) <= gamma * omn[mm] * sqrtf(xn2[vec])) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const float dot = acc[vv][h];
+            if (feature == SLIM_FEAT_EXP) {
+              phi[h] = expf(dot - 0.5f * xn2[vec]) * inv_sqrt_m;
+            } else if (fabsf(dot) <= gamma * omn_g[m + h] * sqrtf(xn2[vec])) {
+              // The sign of omega.x decides ReLU's branch; near zero it is
+              // recomputed in fp64 so the decision is the exact one.
               double a64 = 0.0;
               for (int j = 0; j < d; ++j)
-                a64 += (double)omega[(size_t)m * d + j] * (double)xs[vec * d + j];
-              phi = a64 > 0.0 ? (float)a64 * inv_sqrt_m : 0.f;
+                a64 += (double)omega[(size_t)(m + h) * d + j] * (double)xs[vec * d + j];
+              phi[h] = a64 > 0.0 ? (float)a64 * inv_sqrt_m : 0.f;
             } else {
-              phi = dot > 0.f ? dot * inv_sqrt_m : 0.f;
+              phi[h] = dot > 0.f ? dot * inv_sqrt_m : 0.f;
             }
           }
         }
         float* dst = (vec < R) ? phiQ : phiK;
-        dst[((size_t)c * Cp + r) * M + m] = phi;
+        *reinterpret_cast<float2*>(&dst[((size_t)c * Cp + r) * M + m]) = make_float2(phi[0], phi[1]);
       }
     }
   }
@@ -547,7 +568,7 @@ Geo geometry(const Problem& p) {
 struct Ws {
   int* err;
   float *st_hi, *st_lo, *g_hi, *g_lo;
-  float *Xq, *Xk, *Vx, *phiQ, *phiK, *delta, *A, *numden;
+  float *Xq, *Xk, *Vx, *phiQ, *phiK, *delta, *A, *numden, *omT, *omn;
   float *dout32, *rowdot, *W, *dA, *dphiQ, *dphiK, *gdelta, *usum_q, *usum_k, *stage, *pOm;
 };
 
@@ -565,6 +586,8 @@ Ws carve(Carver& cv, const Geo& g, bool bwd) {
   w.delta = cv.take<float>(C * g.nt * g.M * g.dp);
   w.A = cv.take<float>(C * g.nt * g.T * g.T);
   w.numden = cv.take<float>(C * g.Cp * g.dp);
+  w.omT = cv.take<float>((size_t)((g.M + kPrepFeat - 1) / kPrepFeat) * kPrepFeat * g.d);
+  w.omn = cv.take<float>(g.M);
   if (bwd) {
     w.g_hi = cv.take<float>(C * g.M * g.dp);
     w.g_lo = cv.take<float>(C * g.M * g.dp);
@@ -642,7 +665,7 @@ template <typename T>
 cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w,
                         const void* q, const void* k, const void* v, const void* dout,
                         const void* out, const float* omega, int a, int b, bool bwd) {
-  const size_t smem = (32 * g.d + 32 + g.d * kPrepStride + kPrepFeat) * sizeof(float);
+  const size_t smem = (g.d * kPrepFeat + 32 * g.d + 32) * sizeof(float);
   static bool attr_set[kMaxDevices] = {};  // per dtype instantiation and device
   bool* set = device_flag(attr_set);
   if (set == nullptr) return cudaErrorInvalidDevice;
@@ -655,13 +678,25 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
   dim3 grid(g.Cp / 16, g.chains);
   const float inv_sqrt_m = (float)(1.0 / sqrt((double)g.M));
   const double rows = (double)g.chains * b;
+  int ld = 0;
+  while ((1 << ld) < g.d) ++ld;
   prof::Scope ps(prof::K_PREP, s, 4.0 * rows * g.d * g.M,
                  rows * g.d * sizeof(T) * (bwd ? 5.0 : 3.0));
   k_prep<T><<<grid, 256, smem, s>>>(
       (const T*)q, (const T*)k, (const T*)v, bwd ? (const T*)dout : nullptr,
-      bwd ? (const T*)out : nullptr, omega, p.L, g.d, g.M, a, b, g.Cp, (int)p.feature,
-      inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
+      bwd ? (const T*)out : nullptr, omega, w.omT, w.omn, p.L, ld, g.M, a, b, g.Cp,
+      (int)p.feature, inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
       bwd ? w.rowdot : nullptr);
+  return cudaGetLastError();
+}
+
+// Omega's projection layout and row norms, once per call (no Omega for the
+// quadratic map).
+cudaError_t omega_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w,
+                       const float* omega) {
+  if (p.feature == SLIM_FEAT_SQUARE || p.L == 0 || omega == nullptr) return cudaSuccess;
+  prof::Scope ps(prof::K_PREP, s);
+  k_omega_prep<<<64, 256, 0, s>>>(omega, g.M, g.d, w.omT, w.omn);
   return cudaGetLastError();
 }
 
@@ -705,6 +740,7 @@ slim_status fwd_impl(const Problem& p, const void* q, const void* k, const void*
   const Ws w = carve(cv, g, false);
   const size_t E = (size_t)g.chains * g.M * g.dp;
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(omega_prep(s, p, g, w, omega));
   if (init.S) {
     // B^(0) from an earlier segment (eq. 16 with n - 1 = 0 carried in)
     prof::Scope ps(prof::K_STATE, s);
@@ -746,6 +782,7 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
   const long long T = g.T, M = g.M, d = g.d, dp = g.dp, Cp = g.Cp, nt = g.nt;
   const size_t E = (size_t)g.chains * g.M * g.dp;
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(omega_prep(s, p, g, w, omega));
   if (domega) SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
   const bool square = p.feature == SLIM_FEAT_SQUARE;
   { prof::Scope ps(prof::K_STATE, s);
@@ -934,6 +971,7 @@ slim_status fwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   const long long TT = g.T, M = g.M, dp = g.dp, Cp = g.Cp;
   const size_t E = (size_t)g.chains * g.M * g.dp;
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(omega_prep(s, p, g, w, omega));
   SLIM_TRY(cudaMemsetAsync(w.st_hi, 0, E * sizeof(float), s));
   SLIM_TRY(cudaMemsetAsync(w.st_lo, 0, E * sizeof(float), s));
   // sweep 1: B = sum over every tile of every slice of g(K)^T [V | 1]
@@ -972,6 +1010,7 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   const long long T = g.T, M = g.M, d = g.d, dp = g.dp, Cp = g.Cp, nt = g.nt;
   const size_t E = (size_t)g.chains * g.M * g.dp;
   SLIM_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), s));
+  SLIM_TRY(omega_prep(s, p, g, w, omega));
   if (domega) SLIM_TRY(cudaMemsetAsync(domega, 0, (size_t)g.M * g.d * sizeof(float), s));
   { prof::Scope ps(prof::K_STATE, s);
   k_state_in<<<blocks((long long)E), 256, 0, s>>>(st, w.st_hi, w.st_lo, g.chains, g.M, g.d); }
