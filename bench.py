@@ -49,7 +49,7 @@ MUFU_EX2_PER_S = 9.5e12
 
 # roofline bound of each kernel: (bound, which algorithmic quantity)
 KERNEL_BOUND = {
-    "simt_gemm": ("alu", "flops"),
+    "mma_gemm": ("tensor", "flops"),
     "simt_prep": ("alu", "flops"),
     "tc_fwd": ("tensor", "flops"),
     "tc_bwd": ("tensor", "flops"),
@@ -253,8 +253,8 @@ def roofline(stats, steps):
 
 def step_ceilings(w, B, H, L, ms_per_step):
     """The three floors of one fwd+bwd step from its algorithmic work per
-    token-head: 30dM FLOPs (on the tensor pipe for bf16, the FP32 FMA pipe
-    otherwise), 12ds HBM bytes (s = element size) and 4M exponentials (exp
+    token-head: 30dM FLOPs (on the tensor pipe for bf16; for fp32 as six
+    products of bf16 pieces on the tensor pipe), 12ds HBM bytes (s = element size) and 4M exponentials (exp
     features; none for ReLU), against the measured peaks."""
     peaks, which = measured_peaks()
     th = B * H * L
@@ -265,7 +265,11 @@ def step_ceilings(w, B, H, L, ms_per_step):
     if w.dtype == "bf16":
         compute_us, compute = flops / (peaks["bf16_tflops"] * 1e12) * 1e6, "tensor"
     else:
-        compute_us, compute = flops / (FP32_ALU_TFLOPS * 1e12) * 1e6, "fp32 alu"
+        # fp32 products on the tensor pipe as 6 products of bf16 pieces (24-bit
+        # operands), the faster of that and the FP32 FMA pipe
+        compute_us, compute = min(
+            (flops * 6 / (peaks["bf16_tflops"] * 1e12) * 1e6, "tensor x6"),
+            (flops / (FP32_ALU_TFLOPS * 1e12) * 1e6, "fp32 alu"))
     floors = {compute: compute_us, "hbm": hbm_bytes / (peaks["hbm_gbs"] * 1e9) * 1e6,
               "mufu": exps / MUFU_EX2_PER_S * 1e6}
     bound = max(floors, key=floors.get)

@@ -12,7 +12,7 @@ namespace prof {
 namespace {
 
 const char* kNames[K_COUNT] = {
-    "simt_gemm",   "simt_prep",     "simt_scan",      "simt_finalize", "simt_dstat",
+    "mma_gemm",    "simt_prep",     "simt_scan",      "simt_finalize", "simt_dstat",
     "simt_vjp",    "simt_store",    "simt_reduce",    "simt_state",    "tc_fwd",
     "tc_bwd",      "tc_delta",      "tc_scan",        "tc_bwd_q",      "tc_bwd_kv",
     "tc_reduce",   "tc_selftest",   "tc_prep",        "stack_rows"};

@@ -62,158 +62,217 @@ struct GemmP {
   long long ss_b0;
 };
 
-// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z, in fp32 FMA.
-// A CTA computes a TM x TN tile of C.  Its threads form KS groups of
-// (TM/4)(TN/4); group g takes the reduction chunks g, g + KS, ... and each of
-// its threads keeps 4 x 4 outputs, so a step of the reduction costs a thread
-// two 16-byte shared-memory loads for 16 multiply-adds.  The groups' partial
-// tiles are summed in group order at the end (a fixed order: the result does
-// not depend on scheduling).  Small tiles of long reductions -- the products
-// of 16- and 32-row tiles of short slices -- get several groups, so that a
-// launch has enough threads to fill the SMs.
-// Plain fp32 accumulation holds the fp32 problems' 1e-5 bound: on the L=8192
-// ReLU workload dq is within 3.5e-7 of the fp64 oracle (error-free
-// TwoProduct/TwoSum accumulation gave 1.8e-7 at 2.7x the time).
-template <int TM, int TN, int KS>
-__global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
-  // two stages per group: its next chunk is read from global memory into
-  // registers while its current chunk is multiplied out of shared memory, one
-  // barrier per step
-  constexpr int NT = (TM / 4) * (TN / 4);  // threads per group
-  constexpr int ASZ = 2 * GK * (TM + 4), BSZ = 2 * GK * (TN + 4);
-  constexpr int RED = 17;  // floats a thread hands to group 0
-  constexpr int SMF = KS * (ASZ + BSZ);
-  static_assert(KS == 1 || (KS - 1) * NT * RED <= SMF, "reduction scratch");
-  __shared__ __align__(16) float sm[SMF];
+// ------------------------------------------------------------------ tensor-core contraction
+// x = h + m + l with bf16 pieces: h = bf16(x), m = bf16(x - h), l = bf16(x - h - m)
+// (each difference is exact in fp32), 24 bits of x in NS = 3 pieces, 16 in 2.
+template <int NS>
+__device__ __forceinline__ void split_bf16(float x, float (&pc)[NS]) {
+#pragma unroll
+  for (int i = 0; i < NS; ++i) {
+    pc[i] = __bfloat162float(__float2bfloat16_rn(x));
+    x = __fsub_rn(x, pc[i]);
+  }
+}
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+// D += A B for one m16n8k16 tile: A 16 x 16 bf16 (row-major fragment), B
+// 16 x 8 bf16 (column fragment), D fp32; one warp.
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// C[m x n] = sum_k A[m x k] B[k x n], batched over blockIdx.z, on the tensor
+// cores with warp MMAs: m16 tiles fit the 16-row tiles of short slices, where
+// tcgen05's smallest M, 64, would leave three quarters of every MMA empty.  Each
+// operand element is split once, when its chunk is staged, into NS bf16
+// pieces; shared memory holds the pieces as bf16 pairs along k, so a
+// fragment register is one 32-bit load.  The pieces' products with
+// i + j < NS are summed into fp32 accumulators, smallest first: NS = 3 (6
+// products, 24-bit operands) keeps fp32 problems' products to about 2^-24,
+// NS = 2 (3 products, 16-bit operands) serves bf16 problems.  Warp (wm, wn)
+// of a group owns rows 16 wm .. 16 wm + 15 and columns WN wn .. WN wn + WN - 1
+// of the CTA tile.  A CTA's threads form KS groups; group g takes the reduction
+// chunks g, g + KS, ... and the groups' partial tiles are summed in group order
+// at the end (a fixed order: the result does not depend on scheduling), so
+// that small tiles of long reductions still fill the SMs.  The 65th
+// column of an n = 64q + 1 product is summed in fp32 FMA from the pieces by
+// the group's first TM threads.
+template <int TM, int TN, int KS, int NS>
+__global__ void __launch_bounds__(((TM / 16) * (TN >= 32 ? TN / 32 : 1) * 32) * KS) k_mma(GemmP P) {
+  constexpr int WN = TN >= 32 ? 32 : TN;          // columns per warp
+  constexpr int NB = WN / 8;                      // n8 blocks per warp
+  constexpr int NT = (TM / 16) * (TN / WN) * 32;  // threads per group
+  constexpr int K2 = GK / 2;                      // k pairs per chunk
+  constexpr int LA = TM + 8, LB = TN + 8;         // row strides (words): conflict-free fragments
+  constexpr int ASZ = 2 * NS * K2 * LA, BSZ = 2 * NS * K2 * LB;  // words, two buffers
+  constexpr int RED = 4 * NB + 1;  // floats a thread hands to group 0
+  constexpr int SMW = KS * (ASZ + BSZ);
+  static_assert(KS == 1 || (KS - 1) * NT * RED <= SMW, "reduction scratch");
+  static_assert(TM * K2 % NT == 0 && TN * K2 % NT == 0, "staging split");
+  __shared__ __align__(16) uint32_t sm[SMW];
   const int tid = threadIdx.x, grp = tid / NT, lt = tid % NT;
-  float (*As)[GK][TM + 4] = reinterpret_cast<float (*)[GK][TM + 4]>(sm + grp * (ASZ + BSZ));
-  float (*Bs)[GK][TN + 4] = reinterpret_cast<float (*)[GK][TN + 4]>(sm + grp * (ASZ + BSZ) + ASZ);
-  constexpr int PA = TM * GK / NT, PB = TN * GK / NT;  // elements a thread stages
+  // piece q of the k pair kk2 of row r (A) / column n (B) of buffer bf
+  uint32_t* Ap = sm + grp * (ASZ + BSZ);
+  uint32_t* Bp = Ap + ASZ;
+  auto aw = [&](int bf, int q, int kk2, int r) -> uint32_t& { return Ap[((bf * NS + q) * K2 + kk2) * LA + r]; };
+  auto bw = [&](int bf, int q, int kk2, int n) -> uint32_t& { return Bp[((bf * NS + q) * K2 + kk2) * LB + n]; };
+  constexpr int PA = TM * K2 / NT, PB = TN * K2 / NT;  // k pairs a thread stages
   const int z = blockIdx.z + P.zoff;
   const int z0 = z / P.nb1, z1 = z % P.nb1;
   const float* A = P.a.p + z0 * P.a.b0 + z1 * P.a.b1;
   const float* Bm = P.b.p + z0 * P.b.b0 + z1 * P.b.b1;
   const int i0 = blockIdx.y * TM, j0 = blockIdx.x * TN;
-  const int tx = lt % (TN / 4), ty = lt / (TN / 4);
+  const int warp = lt / 32, lane = lt % 32, g = lane >> 2, t = lane & 3;
+  const int wm = warp / (TN / WN), wn = warp % (TN / WN);
   const bool a_kc = P.a.cs == 1, b_nc = P.b.cs == 1;
-  float acc[4][4];
+  float acc[NB][4];
 #pragma unroll
-  for (int r = 0; r < 4; ++r)
+  for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
-  // A last column tile of 65 columns (n = d + 1: the [V | 1] operands) takes
-  // its 65th column itself, computed by the threads with tx = 0, instead of
-  // leaving it to a CTA of its own.
+    for (int c = 0; c < 4; ++c) acc[nb][c] = 0.f;
   const bool ext = TN == GT && P.n - j0 == GT + 1;
-  float acc_e[4];
-#pragma unroll
-  for (int r = 0; r < 4; ++r) acc_e[r] = 0.f;
+  float acc_e = 0.f;
 
-  // element e of a chunk: (kk, row) of A and (kk, col) of B, laid out so that
+  // pair e of a chunk: (kk2, row) of A and (kk2, col) of B, laid out so that
   // consecutive threads read consecutive addresses of the contiguous dimension
-  float ra[PA], rb[PB], rx = 0.f;
+  float ra[PA][2], rb[PB][2], rx[2] = {0.f, 0.f};
   auto fetch = [&](int k0) {
-    if (ext && lt < GK) {
-      const int gk = k0 + lt;
-      rx = gk < P.k ? Bm[gk * P.b.rs + (j0 + GT) * P.b.cs] : 0.f;
+    if (ext && lt < K2) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int gk = k0 + 2 * lt + h;
+        rx[h] = gk < P.k ? Bm[gk * P.b.rs + (j0 + GT) * P.b.cs] : 0.f;
+      }
     }
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
       const int e = lt + i * NT;
-      const int kk = a_kc ? e % GK : e / TM, r = a_kc ? e / GK : e % TM;
-      const int gi = i0 + r, gk = k0 + kk;
-      ra[i] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
+      const int kk2 = a_kc ? e % K2 : e / TM, r = a_kc ? e / K2 : e % TM;
+      const int gi = i0 + r;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int gk = k0 + 2 * kk2 + h;
+        ra[i][h] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
+      }
     }
 #pragma unroll
     for (int i = 0; i < PB; ++i) {
       const int e = lt + i * NT;
-      const int kb = b_nc ? e / TN : e % GK, cb = b_nc ? e % TN : e / GK;
-      const int gkb = k0 + kb, gj = j0 + cb;
-      rb[i] = (gkb < P.k && gj < P.n) ? Bm[gkb * P.b.rs + gj * P.b.cs] : 0.f;
+      const int kb2 = b_nc ? e / TN : e % K2, cb = b_nc ? e % TN : e / K2;
+      const int gj = j0 + cb;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int gk = k0 + 2 * kb2 + h;
+        rb[i][h] = (gk < P.k && gj < P.n) ? Bm[gk * P.b.rs + gj * P.b.cs] : 0.f;
+      }
     }
   };
-  auto stage = [&](int buf) {
-    if (ext && lt < GK) Bs[buf][lt][GT] = rx;
+  auto put_pieces = [&](uint32_t* w0, int stride, const float (&x)[2]) {
+    float p0[NS], p1[NS];
+    split_bf16<NS>(x[0], p0);
+    split_bf16<NS>(x[1], p1);
+#pragma unroll
+    for (int q = 0; q < NS; ++q) w0[q * stride] = pack2(p0[q], p1[q]);
+  };
+  auto stage = [&](int bf) {
+    if (ext && lt < K2) put_pieces(&bw(bf, 0, lt, GT), K2 * LB, rx);
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
       const int e = lt + i * NT;
-      As[buf][a_kc ? e % GK : e / TM][a_kc ? e / GK : e % TM] = ra[i];
+      const int kk2 = a_kc ? e % K2 : e / TM, r = a_kc ? e / K2 : e % TM;
+      put_pieces(&aw(bf, 0, kk2, r), K2 * LA, ra[i]);
     }
 #pragma unroll
     for (int i = 0; i < PB; ++i) {
       const int e = lt + i * NT;
-      Bs[buf][b_nc ? e / TN : e % GK][b_nc ? e % TN : e / GK] = rb[i];
+      const int kb2 = b_nc ? e / TN : e % K2, cb = b_nc ? e % TN : e / K2;
+      put_pieces(&bw(bf, 0, kb2, cb), K2 * LB, rb[i]);
+    }
+  };
+  // the fp32 value (to the pieces' precision) of a staged element pair
+  auto unpieces = [&](const uint32_t* w0, int stride, float& lo, float& hi) {
+    lo = hi = 0.f;
+#pragma unroll
+    for (int q = NS - 1; q >= 0; --q) {
+      __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(&w0[q * stride]);
+      lo += __low2float(v);
+      hi += __high2float(v);
     }
   };
 
-  // group grp takes chunks grp, grp + KS, ...; every group runs the same
-  // number of steps (chunks past the end read as zeros)
   const int steps = (P.k + GK * KS - 1) / (GK * KS);
   fetch(grp * GK);
   stage(0);
   __syncthreads();
   int buf = 0;
+  const int ar = 16 * wm + g;  // this thread's fragment rows ar and ar + 8
   for (int st = 0; st < steps; ++st) {
     const bool more = st + 1 < steps;
     if (more) fetch((grp + (st + 1) * KS) * GK);
+    // register i of the A fragment: k pair t + 4 (i / 2) of row ar + 8 (i % 2)
+    uint32_t af[NS][4];
 #pragma unroll
-    for (int kk = 0; kk < GK; ++kk) {
-      const float4 a4 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
-      const float a[4] = {a4.x, a4.y, a4.z, a4.w};
-      const float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
-      const float b[4] = {b4.x, b4.y, b4.z, b4.w};
+    for (int q = 0; q < NS; ++q)
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int i = 0; i < 4; ++i) af[q][i] = aw(buf, q, t + 4 * (i >> 1), ar + 8 * (i & 1));
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(a[r], b[c], acc[r][c]);
-      if (ext && tx == 0) {
-        const float be = Bs[buf][kk][GT];
+    for (int nb = 0; nb < NB; ++nb) {
+      const int col = WN * wn + 8 * nb + g;
+      uint32_t bfr[NS][2];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) acc_e[r] = fmaf(a[r], be, acc_e[r]);
+      for (int q = 0; q < NS; ++q)
+#pragma unroll
+        for (int i = 0; i < 2; ++i) bfr[q][i] = bw(buf, q, t + 4 * i, col);
+      // products of pieces (i, j) with i + j < NS, smallest first
+#pragma unroll
+      for (int o = NS - 1; o >= 0; --o)
+#pragma unroll
+        for (int i = 0; i <= o; ++i) mma16816(acc[nb], af[i], bfr[o - i]);
+    }
+    if (ext && lt < TM) {
+#pragma unroll
+      for (int kk2 = 0; kk2 < K2; ++kk2) {
+        float a0, a1, b0, b1;
+        unpieces(&aw(buf, 0, kk2, lt), K2 * LA, a0, a1);
+        unpieces(&bw(buf, 0, kk2, GT), K2 * LB, b0, b1);
+        acc_e = fmaf(a1, b1, fmaf(a0, b0, acc_e));
       }
     }
-    // the other buffer was last read before the previous barrier
     if (more) stage(buf ^ 1);
     __syncthreads();
     buf ^= 1;
   }
 
   if (KS > 1) {
-    // groups 1..KS-1 hand their partial tiles to group 0 through shared
-    // memory (free after the loop's last barrier); element v of thread lt of
-    // group g at red[((g - 1) * RED + v) * NT + lt]
+    // groups 1..KS-1 hand their partial tiles to group 0 (element v of
+    // thread lt of group g at red[((g - 1) RED + v) NT + lt]), summed in
+    // group order
+    float* smf = reinterpret_cast<float*>(sm);
     if (grp > 0) {
-      float* red = sm + (grp - 1) * RED * NT + lt;
+      float* red = smf + (grp - 1) * RED * NT + lt;
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) red[(4 * r + c) * NT] = acc[r][c];
+        for (int c = 0; c < 4; ++c) red[(4 * nb + c) * NT] = acc[nb][c];
+      red[4 * NB * NT] = acc_e;
     }
     __syncthreads();
-    if (grp == 0) {
-#pragma unroll 1
-      for (int g = 1; g < KS; ++g) {
-        const float* red = sm + (g - 1) * RED * NT + lt;
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[r][c] += red[(4 * r + c) * NT];
-      }
-    }
-    if (ext) {
-      // the extra column, row by row through slot 16
-#pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        __syncthreads();
-        if (grp > 0 && tx == 0) sm[(grp - 1) * RED * NT + 16 * NT + lt] = acc_e[r];
-        __syncthreads();
-        if (grp == 0 && tx == 0) {
-#pragma unroll 1
-          for (int g = 1; g < KS; ++g) acc_e[r] += sm[(g - 1) * RED * NT + 16 * NT + lt];
-        }
-      }
-    }
     if (grp > 0) return;
+#pragma unroll 1
+    for (int gg = 1; gg < KS; ++gg) {
+      const float* red = smf + (gg - 1) * RED * NT + lt;
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[nb][c] += red[(4 * nb + c) * NT];
+      acc_e += red[4 * NB * NT];
+    }
   }
 
   float* Cm = P.c.p + z0 * P.c.b0 + z1 * P.c.b1;
@@ -225,17 +284,13 @@ __global__ void __launch_bounds__((TM / 4) * (TN / 4) * KS) k_gemm(GemmP P) {
     *dst = v;
   };
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const int i = i0 + ty * 4 + r;
-    if (i >= P.m) continue;
+  for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-      const int j = j0 + tx * 4 + c;
-      if (j >= P.n) continue;
-      put(i, j, acc[r][c]);
+      const int i = i0 + ar + 8 * (c >> 1), j = j0 + WN * wn + 8 * nb + 2 * t + (c & 1);
+      if (i < P.m && j < P.n) put(i, j, acc[nb][c]);
     }
-    if (ext && tx == 0) put(i, j0 + GT, acc_e[r]);
-  }
+  if (ext && lt < TM && i0 + lt < P.m) put(i0 + lt, j0 + GT, acc_e);
 }
 
 // ------------------------------------------------------------------ per-slice staging
@@ -528,6 +583,7 @@ constexpr int kSplitCtas = 304;   // dOmega contractions: about two waves of 152
 struct Geo {
   int chains, d, dp, M, Cs, T, nt, Cp, N;  // Cs: rows per launch sequence (a slice or a group)
   int ks;        // row splits of the dOmega contractions (divides nt)
+  int ns;        // bf16 pieces per operand element in the tensor-core contractions
 };
 
 Geo geometry(const Problem& p) {
@@ -562,6 +618,8 @@ Geo geometry(const Problem& p) {
   g.ks = 1;
   for (int k = 2; k <= g.nt && k <= want; ++k)
     if (g.nt % k == 0) g.ks = k;
+  // fp32 problems: 3 pieces (24 bits); bf16 problems: 2 (16 bits)
+  g.ns = p.dtype == SLIM_F32 ? 3 : 2;
   return g;
 }
 
@@ -613,7 +671,7 @@ OutMat omat(float* p, long long b0, long long b1, long long rs, long long cs) {
   return OutMat{p, b0, b1, rs, cs};
 }
 
-cudaError_t gemm(cudaStream_t s, int m, int n, int k, Mat a, Mat b, OutMat c,
+cudaError_t gemm(cudaStream_t s, int ns, int m, int n, int k, Mat a, Mat b, OutMat c,
                  int nb0, int nb1,
                  float beta, int causal, const float* sx = nullptr, long long sx_b0 = 0,
                  long long sx_rs = 0, const float* ss = nullptr, long long ss_b0 = 0) {
@@ -626,27 +684,35 @@ cudaError_t gemm(cudaStream_t s, int m, int n, int k, Mat a, Mat b, OutMat c,
     const int tn = n <= 16 ? 16 : GT;
     const int tm = (m <= 16 || tn == 16) ? 16 : (m <= 32 ? 32 : 64);
     // reduction groups per CTA for the small tiles, when the reduction has
-    // at least two chunks per group
-    const int want = tn == 16 ? 8 : (tm == 16 ? 4 : (tm == 32 ? 2 : 1));
+    // at least two chunks per group (fewer with 3 pieces: shared memory)
+    const int want = tn == 16 ? (ns == 2 ? 8 : 4)
+                              : (tm == 16 ? (ns == 2 ? 4 : 2) : (tm == 32 ? 2 : 1));
     const int ks = (k >= 2 * GK * want) ? want : 1;
     // n = 64 q + 1 (the [V | 1] operands): the last 64-column tile takes the
     // extra column
     const int nx = (tn == GT && n > GT && n % GT == 1) ? n / GT : (n + tn - 1) / tn;
     dim3 grid(nx, (m + tm - 1) / tm, zc);
     prof::Scope ps(prof::K_GEMM, s, 2.0 * m * n * k * zc);
-    const int nthr = (tm / 4) * (tn / 4) * ks;
-    if (tn == 16) {
-      if (ks > 1) k_gemm<16, 16, 8><<<grid, nthr, 0, s>>>(P);
-      else k_gemm<16, 16, 1><<<grid, nthr, 0, s>>>(P);
-    } else if (tm == 16) {
-      if (ks > 1) k_gemm<16, GT, 4><<<grid, nthr, 0, s>>>(P);
-      else k_gemm<16, GT, 1><<<grid, nthr, 0, s>>>(P);
-    } else if (tm == 32) {
-      if (ks > 1) k_gemm<32, GT, 2><<<grid, nthr, 0, s>>>(P);
-      else k_gemm<32, GT, 1><<<grid, nthr, 0, s>>>(P);
-    } else {
-      k_gemm<64, GT, 1><<<grid, nthr, 0, s>>>(P);
+    const int nthr = (tm / 16) * (tn >= 32 ? tn / 32 : 1) * 32 * ks;
+#define SLIM_MMA_LAUNCH(NS, K16, K64)                                                 \
+    if (tn == 16) {                                                                   \
+      if (ks > 1) k_mma<16, 16, K16, NS><<<grid, nthr, 0, s>>>(P);                    \
+      else k_mma<16, 16, 1, NS><<<grid, nthr, 0, s>>>(P);                             \
+    } else if (tm == 16) {                                                            \
+      if (ks > 1) k_mma<16, GT, K64, NS><<<grid, nthr, 0, s>>>(P);                    \
+      else k_mma<16, GT, 1, NS><<<grid, nthr, 0, s>>>(P);                             \
+    } else if (tm == 32) {                                                            \
+      if (ks > 1) k_mma<32, GT, 2, NS><<<grid, nthr, 0, s>>>(P);                      \
+      else k_mma<32, GT, 1, NS><<<grid, nthr, 0, s>>>(P);                             \
+    } else {                                                                          \
+      k_mma<64, GT, 1, NS><<<grid, nthr, 0, s>>>(P);                                  \
     }
+    if (ns == 2) {
+      SLIM_MMA_LAUNCH(2, 8, 4)
+    } else {
+      SLIM_MMA_LAUNCH(3, 4, 2)
+    }
+#undef SLIM_MMA_LAUNCH
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -703,7 +769,7 @@ cudaError_t omega_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws&
 // Delta_t = phiK_t^T [V_t | 1]  (M x dp per tile)
 cudaError_t tile_deltas(cudaStream_t s, const Geo& g, const Ws& w) {
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
-  return gemm(s, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
+  return gemm(s, g.ns, g.M, g.dp, g.T, mat(w.phiK, Cp * M, T * M, 1, M), mat(w.Vx, Cp * dp, T * dp, dp, 1),
               omat(w.delta, nt * M * dp, M * dp, dp, 1), g.chains, g.nt, 0.f, 0);
 }
 
@@ -714,15 +780,15 @@ cudaError_t scores_and_readout(cudaStream_t s, const Geo& g, const Ws& w, bool d
   const long long T = g.T, M = g.M, dp = g.dp, Cp = g.Cp, nt = g.nt;
   const long long c0 = den_only ? g.d : 0;  // first column computed
   const int nc = den_only ? 1 : g.dp;
-  cudaError_t e = gemm(s, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+  cudaError_t e = gemm(s, g.ns, g.T, g.T, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                        mat(w.phiK, Cp * M, T * M, 1, M), omat(w.A, nt * T * T, T * T, T, 1),
                        g.chains, g.nt, 0.f, 1);
   if (e != cudaSuccess) return e;
-  e = gemm(s, g.T, nc, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+  e = gemm(s, g.ns, g.T, nc, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
            mat(w.delta + c0, nt * M * dp, M * dp, dp, 1),
            omat(w.numden + c0, Cp * dp, T * dp, dp, 1), g.chains, g.nt, 0.f, 0);
   if (e != cudaSuccess) return e;
-  return gemm(s, g.T, nc, g.T, mat(w.A, nt * T * T, T * T, T, 1),
+  return gemm(s, g.ns, g.T, nc, g.T, mat(w.A, nt * T * T, T * T, T, 1),
               mat(w.Vx + c0, Cp * dp, T * dp, dp, 1), omat(w.numden + c0, Cp * dp, T * dp, dp, 1),
               g.chains, g.nt, 1.f, 0);
 }
@@ -812,33 +878,33 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
                                                                g.d, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
     // dA_t = tril(W_t [V_t | 1]^T)
-    SLIM_TRY(gemm(s, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.T, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.Vx, Cp * dp, T * dp, 1, dp), omat(w.dA, nt * T * T, T * T, T, 1),
                   g.chains, g.nt, 0.f, 1));
     // dphiQ = W_t P_t^T + dA_t phiK_t
-    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.delta, nt * M * dp, M * dp, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, T, 1),
                   mat(w.phiK, Cp * M, T * M, M, 1), omat(w.dphiQ, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 1.f, 0));
     // Gd_t = phiQ_t^T W_t, then G_t = G + sum_{t' > t} Gd_t'
-    SLIM_TRY(gemm(s, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+    SLIM_TRY(gemm(s, g.ns, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
     // dphiK = dA_t^T phiQ_t + [V_t | 1] G_t^T
-    SLIM_TRY(gemm(s, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.T, mat(w.dA, nt * T * T, T * T, 1, T),
                   mat(w.phiQ, Cp * M, T * M, M, 1), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
                   mat(w.gdelta, nt * M * dp, M * dp, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 1.f, 0));
     // dV = A_t^T dnum + phiK_t G_t(S)
-    SLIM_TRY(gemm(s, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.d, g.T, mat(w.A, nt * T * T, T * T, 1, T),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
                   mat(w.gdelta, nt * M * dp, M * dp, dp, 1), omat(w.stage, Cp * d, T * d, d, 1),
                   g.chains, g.nt, 1.f, 0));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
@@ -876,14 +942,14 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(cudaGetLastError());
     const bool ex = p.feature == SLIM_FEAT_EXP;
     // dX = u Omega (- x sum u for the exp map)
-    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    SLIM_TRY(gemm(s, g.ns, g.Cp, g.d, g.M, mat(w.dphiQ, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
                   omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xq : nullptr,
                   Cp * d, d, w.usum_q, Cp));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
     k_store<IO><<<blocks((long long)g.chains * b * g.d), 256, 0, s>>>(w.stage, (IO*)dq, p.L, g.d,
                                                                       a, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
-    SLIM_TRY(gemm(s, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    SLIM_TRY(gemm(s, g.ns, g.Cp, g.d, g.M, mat(w.dphiK, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
                   omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? w.Xk : nullptr,
                   Cp * d, d, w.usum_k, Cp));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));
@@ -892,10 +958,10 @@ slim_status bwd_impl(const Problem& p, const void* q, const void* k, const void*
     SLIM_TRY(cudaGetLastError());
     // dOmega partials per chain and row split: u_q^T x_q + u_k^T x_k
     const long long kc = (long long)(g.nt / g.ks) * T, ks = g.ks;
-    SLIM_TRY(gemm(s, g.M, g.d, (int)kc, mat(w.dphiQ, Cp * M, kc * M, 1, M),
+    SLIM_TRY(gemm(s, g.ns, g.M, g.d, (int)kc, mat(w.dphiQ, Cp * M, kc * M, 1, M),
                   mat(w.Xq, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains,
                   g.ks, 0.f, 0));
-    SLIM_TRY(gemm(s, g.M, g.d, (int)kc, mat(w.dphiK, Cp * M, kc * M, 1, M),
+    SLIM_TRY(gemm(s, g.ns, g.M, g.d, (int)kc, mat(w.dphiK, Cp * M, kc * M, 1, M),
                   mat(w.Xk, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains,
                   g.ks, 1.f, 0));
     { prof::Scope ps(prof::K_REDUCE, s);
@@ -941,12 +1007,12 @@ cudaError_t side_vjp(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w
                                                             (float)(1.0 / sqrt((double)g.M))); }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const bool ex = p.feature == SLIM_FEAT_EXP;
-    e = gemm(s, g.Cp, g.d, g.M, mat(dphi, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
+    e = gemm(s, g.ns, g.Cp, g.d, g.M, mat(dphi, Cp * M, 0, M, 1), mat(omega, 0, 0, d, 1),
              omat(w.stage, Cp * d, 0, d, 1), g.chains, 1, 0.f, 0, ex ? X : nullptr, Cp * d, d,
              usum, Cp);
     if (e != cudaSuccess) return e;
     const long long kc = (long long)(g.nt / g.ks) * g.T, ks = g.ks;
-    e = gemm(s, g.M, g.d, (int)kc, mat(dphi, Cp * M, kc * M, 1, M),
+    e = gemm(s, g.ns, g.M, g.d, (int)kc, mat(dphi, Cp * M, kc * M, 1, M),
              mat(X, Cp * d, kc * d, d, 1), omat(w.pOm, ks * M * d, M * d, d, 1), g.chains, g.ks,
              0.f, 0);
     if (e != cudaSuccess) return e;
@@ -988,7 +1054,7 @@ slim_status fwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
-    SLIM_TRY(gemm(s, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, TT * M, M, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, TT * M, M, 1),
                   mat(w.st_hi, M * dp, 0, dp, 1), omat(w.numden, Cp * dp, TT * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_FINALIZE, s, 0.0, (double)g.chains * b * g.d * sizeof(T));
@@ -1022,17 +1088,17 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
     // den = g(Q) z: the only column of [num | den] the gradients need
-    SLIM_TRY(gemm(s, g.T, 1, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, 1, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                   mat(w.st_hi + d, M * dp, 0, dp, 1), omat(w.numden + d, Cp * dp, T * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_DSTAT, s);
     k_dstat<<<blocks((long long)g.chains * Cp * dp), 256, 0, s>>>(w.numden, w.dout32, w.rowdot,
                                                                   w.W, g.d, b, g.Cp, g.chains); }
     SLIM_TRY(cudaGetLastError());
-    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.dp, mat(w.W, Cp * dp, T * dp, dp, 1),
                   mat(w.st_hi, M * dp, 0, 1, dp), omat(w.dphiQ, Cp * M, T * M, M, 1),
                   g.chains, g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
+    SLIM_TRY(gemm(s, g.ns, g.M, g.dp, g.T, mat(w.phiQ, Cp * M, T * M, 1, M),
                   mat(w.W, Cp * dp, T * dp, dp, 1), omat(w.gdelta, nt * M * dp, M * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
     SLIM_TRY(scan(s, g, w.gdelta, w.g_hi, w.g_lo, SCAN_GREV));
@@ -1042,10 +1108,10 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
     SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
-    SLIM_TRY(gemm(s, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
                   mat(w.g_hi, M * dp, 0, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 0.f, 0));
-    SLIM_TRY(gemm(s, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
+    SLIM_TRY(gemm(s, g.ns, g.T, g.d, g.M, mat(w.phiK, Cp * M, T * M, M, 1),
                   mat(w.g_hi, M * dp, 0, dp, 1), omat(w.stage, Cp * d, T * d, d, 1), g.chains,
                   g.nt, 0.f, 0));
     { prof::Scope ps(prof::K_STORE, s, 0.0, (double)g.chains * b * g.d * sizeof(IO));

@@ -26,5 +26,8 @@ def test_relu_fp32_floors():
     w = W.WORKLOADS["L8192_relu_f32"]
     c = bench.step_ceilings(w, w.B, w.H, w.L, 46.0)
     assert c["exps"] == 0 and c["floors_us"]["mufu"] == 0
-    assert "fp32 alu" in c["floors_us"] and "tensor" not in c["floors_us"]
+    # fp32 products as six bf16-piece products on the tensor pipe
+    peaks, _ = bench.measured_peaks()
+    assert "tensor x6" in c["floors_us"] and "tensor" not in c["floors_us"]
+    assert abs(c["floors_us"]["tensor x6"] - 6 * c["flops"] / (peaks["bf16_tflops"] * 1e6)) < 0.01
     assert c["hbm_bytes"] == 12 * 64 * 4 * w.B * w.H * w.L
