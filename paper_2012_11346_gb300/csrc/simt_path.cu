@@ -329,7 +329,7 @@ __global__ void __launch_bounds__(256) k_prep(
     const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
     const T* __restrict__ dout, const T* __restrict__ out, const float* __restrict__ omega,
     const float* __restrict__ omT_g, const float* __restrict__ omn_g,
-    int L, int ld, int M, int a, int b, int Cp, int feature, float inv_sqrt_m,
+    int L, int ld, int M, int a, int b, int Cp, int feature, int sides, float inv_sqrt_m,
     float* Xq, float* Xk, float* Vx, float* phiQ, float* phiK, float* dout32, float* rowdot) {
   extern __shared__ __align__(16) float sm[];
   constexpr int R = 16;            // rows per CTA (q and k -> 32 vectors)
@@ -410,6 +410,9 @@ __global__ void __launch_bounds__(256) k_prep(
       for (int e = tid; e < d * kPrepFeat / 4; e += 256) dst[e] = src[e];
     }
     __syncthreads();
+    // sides: bit 0 the query features, bit 1 the key features (the
+    // non-causal sweeps need one side each); vectors 0..R-1 are queries
+    if (!(sides & (grp < 2 ? 1 : 2))) continue;
     float acc[8][2];
 #pragma unroll
     for (int vv = 0; vv < 8; ++vv) acc[vv][0] = acc[vv][1] = 0.f;
@@ -730,7 +733,8 @@ unsigned blocks(long long n, int t = 256) { return (unsigned)((n + t - 1) / t); 
 template <typename T>
 cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws& w,
                         const void* q, const void* k, const void* v, const void* dout,
-                        const void* out, const float* omega, int a, int b, bool bwd) {
+                        const void* out, const float* omega, int a, int b, bool bwd,
+                        int sides = 3) {
   const size_t smem = (g.d * kPrepFeat + 32 * g.d + 32) * sizeof(float);
   static bool attr_set[kMaxDevices] = {};  // per dtype instantiation and device
   bool* set = device_flag(attr_set);
@@ -746,12 +750,12 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
   const double rows = (double)g.chains * b;
   int ld = 0;
   while ((1 << ld) < g.d) ++ld;
-  prof::Scope ps(prof::K_PREP, s, 4.0 * rows * g.d * g.M,
+  prof::Scope ps(prof::K_PREP, s, (sides == 3 ? 4.0 : 2.0) * rows * g.d * g.M,
                  rows * g.d * sizeof(T) * (bwd ? 5.0 : 3.0));
   k_prep<T><<<grid, 256, smem, s>>>(
       (const T*)q, (const T*)k, (const T*)v, bwd ? (const T*)dout : nullptr,
       bwd ? (const T*)out : nullptr, omega, w.omT, w.omn, p.L, ld, g.M, a, b, g.Cp,
-      (int)p.feature, inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
+      (int)p.feature, sides, inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
       bwd ? w.rowdot : nullptr);
   return cudaGetLastError();
 }
@@ -1043,7 +1047,7 @@ slim_status fwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   // sweep 1: B = sum over every tile of every slice of g(K)^T [V | 1]
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false, 2));
     SLIM_TRY(tile_deltas(s, g, w));
     SLIM_TRY(scan(s, g, w.delta, w.st_hi, w.st_lo, SCAN_FWD));
   }
@@ -1053,7 +1057,7 @@ slim_status fwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   // sweep 2: [num | den] = g(Q) B, out = num / den
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(launch_prep<T>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false, 1));
     SLIM_TRY(gemm(s, g.ns, g.T, g.dp, g.M, mat(w.phiQ, Cp * M, TT * M, M, 1),
                   mat(w.st_hi, M * dp, 0, dp, 1), omat(w.numden, Cp * dp, TT * dp, dp, 1),
                   g.chains, g.nt, 0.f, 0));
@@ -1086,7 +1090,7 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   // sweep 1, query side: W = [dnum | dden], dphiQ = W B^T, G += g(Q)^T W
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true));
+    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, dout, out, omega, a, b, true, 1));
     // den = g(Q) z: the only column of [num | den] the gradients need
     SLIM_TRY(gemm(s, g.ns, g.T, 1, g.M, mat(w.phiQ, Cp * M, T * M, M, 1),
                   mat(w.st_hi + d, M * dp, 0, dp, 1), omat(w.numden + d, Cp * dp, T * dp, dp, 1),
@@ -1107,7 +1111,7 @@ slim_status bwd_bidir_impl(const Problem& p, const void* q, const void* k, const
   // sweep 2, key/value side: dphiK = [V | 1] G^T, dV = g(K) G_S
   for (int n = 0; n < g.N; ++n) {
     const int a = n * g.Cs, b = (p.L - a < g.Cs) ? p.L - a : g.Cs;
-    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false));
+    SLIM_TRY(launch_prep<IO>(s, p, g, w, q, k, v, nullptr, nullptr, omega, a, b, false, 2));
     SLIM_TRY(gemm(s, g.ns, g.T, g.M, g.dp, mat(w.Vx, Cp * dp, T * dp, dp, 1),
                   mat(w.g_hi, M * dp, 0, 1, dp), omat(w.dphiK, Cp * M, T * M, M, 1), g.chains,
                   g.nt, 0.f, 0));
