@@ -142,6 +142,31 @@ __global__ void __launch_bounds__(((TM / 16) * (TN >= 32 ? TN / 32 : 1) * 32) * 
   // pair e of a chunk: (kk2, row) of A and (kk2, col) of B, laid out so that
   // consecutive threads read consecutive addresses of the contiguous dimension
   float ra[PA][2], rb[PB][2], rx[2] = {0.f, 0.f};
+  // Each thread stages the same (pair, row) slots of every chunk: its element
+  // addresses are fixed bases plus k0 times the operand's k stride.
+  const float* pa[PA];
+  int ka[PA];
+  bool oka[PA];
+#pragma unroll
+  for (int i = 0; i < PA; ++i) {
+    const int e = lt + i * NT;
+    const int kk2 = a_kc ? e % K2 : e / TM, r = a_kc ? e / K2 : e % TM;
+    oka[i] = i0 + r < P.m;
+    ka[i] = 2 * kk2;
+    pa[i] = A + (oka[i] ? (long long)(i0 + r) * P.a.rs + 2LL * kk2 * P.a.cs : 0);
+  }
+  const float* pb[PB];
+  int kb[PB];
+  bool okb[PB];
+#pragma unroll
+  for (int i = 0; i < PB; ++i) {
+    const int e = lt + i * NT;
+    const int kb2 = b_nc ? e / TN : e % K2, cb = b_nc ? e % TN : e / K2;
+    okb[i] = j0 + cb < P.n;
+    kb[i] = 2 * kb2;
+    pb[i] = Bm + (okb[i] ? 2LL * kb2 * P.b.rs + (long long)(j0 + cb) * P.b.cs : 0);
+  }
+  const long long ak = P.a.cs, bk = P.b.rs;  // k strides
   auto fetch = [&](int k0) {
     if (ext && lt < K2) {
 #pragma unroll
@@ -152,25 +177,17 @@ __global__ void __launch_bounds__(((TM / 16) * (TN >= 32 ? TN / 32 : 1) * 32) * 
     }
 #pragma unroll
     for (int i = 0; i < PA; ++i) {
-      const int e = lt + i * NT;
-      const int kk2 = a_kc ? e % K2 : e / TM, r = a_kc ? e / K2 : e % TM;
-      const int gi = i0 + r;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int gk = k0 + 2 * kk2 + h;
-        ra[i][h] = (gi < P.m && gk < P.k) ? A[gi * P.a.rs + gk * P.a.cs] : 0.f;
-      }
+      const float* src = pa[i] + k0 * ak;
+      const int gk = k0 + ka[i];
+      ra[i][0] = (oka[i] && gk < P.k) ? src[0] : 0.f;
+      ra[i][1] = (oka[i] && gk + 1 < P.k) ? src[ak] : 0.f;
     }
 #pragma unroll
     for (int i = 0; i < PB; ++i) {
-      const int e = lt + i * NT;
-      const int kb2 = b_nc ? e / TN : e % K2, cb = b_nc ? e % TN : e / K2;
-      const int gj = j0 + cb;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int gk = k0 + 2 * kb2 + h;
-        rb[i][h] = (gk < P.k && gj < P.n) ? Bm[gk * P.b.rs + gj * P.b.cs] : 0.f;
-      }
+      const float* src = pb[i] + k0 * bk;
+      const int gk = k0 + kb[i];
+      rb[i][0] = (okb[i] && gk < P.k) ? src[0] : 0.f;
+      rb[i][1] = (okb[i] && gk + 1 < P.k) ? src[bk] : 0.f;
     }
   };
   auto put_pieces = [&](uint32_t* w0, int stride, const float (&x)[2]) {
