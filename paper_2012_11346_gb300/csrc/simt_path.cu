@@ -344,7 +344,7 @@ __global__ void k_omega_prep(const float* __restrict__ omega, int M, int d, floa
 template <typename T>
 __global__ void __launch_bounds__(256) k_prep(
     const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
-    const T* __restrict__ dout, const T* __restrict__ out, const float* __restrict__ omega,
+    const T* __restrict__ dout, const T* __restrict__ out,
     const float* __restrict__ omT_g, const float* __restrict__ omn_g,
     int L, int ld, int M, int a, int b, int Cp, int feature, int sides, float inv_sqrt_m,
     float* Xq, float* Xk, float* Vx, float* phiQ, float* phiK, float* dout32, float* rowdot) {
@@ -467,11 +467,20 @@ __global__ void __launch_bounds__(256) k_prep(
               phi[h] = expf(dot - 0.5f * xn2[vec]) * inv_sqrt_m;
             } else if (fabsf(dot) <= gamma * omn_g[m + h] * sqrtf(xn2[vec])) {
               // The sign of omega.x decides ReLU's branch; near zero it is
-              // recomputed in fp64 so the decision is the exact one.
-              double a64 = 0.0;
-              for (int j = 0; j < d; ++j)
-                a64 += (double)omega[(size_t)(m + h) * d + j] * (double)xs[vec * d + j];
-              phi[h] = a64 > 0.0 ? (float)a64 * inv_sqrt_m : 0.f;
+              // recomputed as a compensated dot product (FMA TwoProduct and
+              // TwoSum, about 48 bits, Ogita-Rump-Oishi Dot2) so that the
+              // decision is the exact one.
+              float sh = 0.f, sl = 0.f;
+              for (int j = 0; j < d; ++j) {
+                const float xw = xs[vec * d + j], ow = omT[j * kPrepFeat + 2 * f + h];
+                const float p = __fmul_rn(xw, ow), ep = __fmaf_rn(xw, ow, -p);
+                float t, e;
+                two_sum(sh, p, t, e);
+                sh = t;
+                sl = __fadd_rn(sl, __fadd_rn(e, ep));
+              }
+              const float a32 = __fadd_rn(sh, sl);
+              phi[h] = a32 > 0.f ? a32 * inv_sqrt_m : 0.f;
             } else {
               phi[h] = dot > 0.f ? dot * inv_sqrt_m : 0.f;
             }
@@ -771,7 +780,7 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
                  rows * g.d * sizeof(T) * (bwd ? 5.0 : 3.0));
   k_prep<T><<<grid, 256, smem, s>>>(
       (const T*)q, (const T*)k, (const T*)v, bwd ? (const T*)dout : nullptr,
-      bwd ? (const T*)out : nullptr, omega, w.omT, w.omn, p.L, ld, g.M, a, b, g.Cp,
+      bwd ? (const T*)out : nullptr, w.omT, w.omn, p.L, ld, g.M, a, b, g.Cp,
       (int)p.feature, sides, inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
       bwd ? w.rowdot : nullptr);
   return cudaGetLastError();
