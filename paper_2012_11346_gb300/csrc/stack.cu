@@ -36,46 +36,104 @@ __global__ void k_pair_sub(float* hi, float* lo, const float* dhi, const float* 
   lo[i] = l;
 }
 constexpr float kNormEps = 1e-6f;
-constexpr int kRowsPerBlock = 8;  // one warp per row
+constexpr int kRowThreads = 256;  // threads per block of the row kernels
 
-__device__ float warp_sum(float v) {
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+// Row kernels: thread `sub` of a row's d/8 lanes owns elements 8 sub .. 8 sub + 7
+// and moves them as one 16-byte (bf16) or two 16-byte (fp32) accesses; the
+// slice buffers are workspace rows of d contiguous elements, 16-byte aligned.
+// A block serves kRowThreads / (d/8) rows.
+__device__ __forceinline__ void ld8(const float* p, float* v) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0], b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void st8(float* p, const float* v) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+__device__ __forceinline__ void ld8(const __nv_bfloat16* p, float* v) {
+  const uint4 r = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const __nv_bfloat162 h = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+    v[2 * i] = __low2float(h);
+    v[2 * i + 1] = __high2float(h);
+  }
+}
+__device__ __forceinline__ void st8(__nv_bfloat16* p, const float* v) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    w[i] = *reinterpret_cast<const uint32_t*>(&h);
+  }
+  *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+// the value a store of x in the dtype reads back as
+__device__ __forceinline__ float as_dtype(float x, const float*) { return x; }
+__device__ __forceinline__ float as_dtype(float x, const __nv_bfloat16*) {
+  return __bfloat162float(__float2bfloat16_rn(x));
+}
+// sum over the lpr lanes of a row (aligned groups of a power of two)
+__device__ __forceinline__ float row_sum(float v, int lpr) {
+  for (int o = lpr >> 1; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-// u = scale * x / sqrt(mean(x^2) + eps) for one row, one warp per row
+// This thread's row and first element.  Threads past the last row stay to the
+// end (their lanes take part in the row sums' shuffles) and touch no memory.
+struct RowPos {
+  bool ok;  // the row exists
+  size_t o; // element offset of this thread's 8 (0 when !ok)
+};
+__device__ __forceinline__ RowPos row_pos(int d, long long rows) {
+  const int lpr = d >> 3;
+  const long long row = (long long)blockIdx.x * (kRowThreads / lpr) + threadIdx.x / lpr;
+  const bool ok = row < rows;
+  return RowPos{ok, ok ? (size_t)row * d + (threadIdx.x % lpr) * 8 : 0};
+}
+
+// u = scale * x / sqrt(mean(x^2) + eps) for one row, from this thread's 8
+// values v; the lanes of a row meet in row_sum, so every lane takes part
 template <typename T>
-__device__ void norm_row(const T* xr, T* ur, int d, float scale, int lane) {
+__device__ __forceinline__ void norm8(const float* v, T* ur, int d, float scale, bool ok) {
   float ss = 0.f;
-  for (int j = lane; j < d; j += 32) {
-    const float v = Io<T>::load(xr, j);
-    ss += v * v;
-  }
-  const float inv = scale / sqrtf(warp_sum(ss) / d + kNormEps);
-  for (int j = lane; j < d; j += 32) Io<T>::store(ur, j, Io<T>::load(xr, j) * inv);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
+  const float inv = scale / sqrtf(row_sum(ss, d >> 3) / d + kNormEps);
+  float u[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) u[i] = v[i] * inv;
+  if (ok) st8(ur, u);
 }
 
 // the first layer's u from the slice's rows
 template <typename T>
-__global__ void k_rownorm(const T* x, T* u, int d, float scale, long long rows) {
-  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
-  if (row >= rows) return;
-  norm_row(x + row * d, u + row * d, d, scale, threadIdx.x & 31);
+__global__ void __launch_bounds__(kRowThreads) k_rownorm(const T* x, T* u, int d, float scale,
+                                                         long long rows) {
+  const RowPos rp = row_pos(d, rows);
+  float v[8] = {};
+  if (rp.ok) ld8(x + rp.o, v);
+  norm8(v, u + rp.o, d, scale, rp.ok);
 }
 
 // the residual connection out = x + y (fp32 sum rounded to the dtype), then,
 // when u is given, the next layer's u from the rounded out (the value the next
 // layer's recompute reads back)
 template <typename T>
-__global__ void k_residual_norm(const T* x, const T* y, T* out, T* u, int d, float scale,
-                                long long rows) {
-  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= rows) return;
-  const size_t o = (size_t)row * d;
-  for (int j = lane; j < d; j += 32) Io<T>::store(out, o + j, Io<T>::load(x, o + j) + Io<T>::load(y, o + j));
-  __syncwarp();
-  if (u) norm_row(out + o, u + o, d, scale, lane);
+__global__ void __launch_bounds__(kRowThreads) k_residual_norm(const T* x, const T* y, T* out,
+                                                               T* u, int d, float scale,
+                                                               long long rows) {
+  const RowPos rp = row_pos(d, rows);
+  float a[8] = {}, b[8] = {};
+  if (rp.ok) {
+    ld8(x + rp.o, a);
+    ld8(y + rp.o, b);
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) a[i] = as_dtype(a[i] + b[i], x);
+  if (rp.ok) st8(out + rp.o, a);
+  if (u) norm8(a, u + rp.o, d, scale, rp.ok);
 }
 
 // dX (fp32) += u'(x)^T g with g = dq + dk + dv (q = k = v = u(x)):
@@ -83,29 +141,41 @@ __global__ void k_residual_norm(const T* x, const T* y, T* out, T* u, int d, flo
 // and the next layer down's upstream gradient (the new dX) as the dtype into
 // dout.  For the top layer (first) the old dX is dout itself: the slice's dy.
 template <typename T>
-__global__ void k_dx_accum(float* dx, const T* x, const T* dq, const T* dk, const T* dv, T* dout,
-                           int d, float scale, long long rows, int first) {
-  const long long row = (long long)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= rows) return;
-  const size_t o = (size_t)row * d;
+__global__ void __launch_bounds__(kRowThreads) k_dx_accum(float* dx, const T* x, const T* dq,
+                                                          const T* dk, const T* dv, T* dout,
+                                                          int d, float scale, long long rows,
+                                                          int first) {
+  const RowPos rp = row_pos(d, rows);
+  const size_t o = rp.o;
+  float xv[8] = {}, g[8] = {}, t[8] = {};
+  if (rp.ok) {
+    ld8(x + o, xv);
+    ld8(dq + o, g);
+    ld8(dk + o, t);
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) g[i] += t[i];
+  if (rp.ok) ld8(dv + o, t);
   float ss = 0.f, gx = 0.f;
-  for (int j = lane; j < d; j += 32) {
-    const float xv = Io<T>::load(x, o + j);
-    const float g = Io<T>::load(dq, o + j) + Io<T>::load(dk, o + j) + Io<T>::load(dv, o + j);
-    ss += xv * xv;
-    gx += g * xv;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    g[i] += t[i];
+    ss = fmaf(xv[i], xv[i], ss);
+    gx = fmaf(g[i], xv[i], gx);
   }
-  const float r2 = warp_sum(ss) / d + kNormEps;
-  const float m = warp_sum(gx) / d / r2;
+  const int lpr = d >> 3;
+  const float r2 = row_sum(ss, lpr) / d + kNormEps;
+  const float m = row_sum(gx, lpr) / d / r2;
   const float f = scale / sqrtf(r2);
-  for (int j = lane; j < d; j += 32) {
-    const float xv = Io<T>::load(x, o + j);
-    const float g = Io<T>::load(dq, o + j) + Io<T>::load(dk, o + j) + Io<T>::load(dv, o + j);
-    const float v = (first ? Io<T>::load(dout, o + j) : dx[o + j]) + f * (g - xv * m);
-    dx[o + j] = v;
-    Io<T>::store(dout, o + j, v);
-  }
+  if (!rp.ok) return;  // after the last shuffle
+  if (first)
+    ld8(dout + o, t);
+  else
+    ld8(dx + o, t);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) t[i] += f * (g[i] - xv[i] * m);
+  st8(dx + o, t);
+  st8(dout + o, t);
 }
 __global__ void k_add(float* acc, const float* x, long long n) {
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -122,7 +192,11 @@ struct Geo {
 };
 
 unsigned nb(long long n) { return (unsigned)((n + 255) / 256); }
-unsigned nrb(long long rows) { return (unsigned)((rows + kRowsPerBlock - 1) / kRowsPerBlock); }
+// blocks of the row kernels for `rows` rows of d elements
+unsigned nrb(long long rows, int d) {
+  const long long per = kRowThreads / (d / 8);
+  return (unsigned)((rows + per - 1) / per);
+}
 // every launch of this file is counted (and timed when the profiler is on),
 // with the bytes it must move
 #define STACK_LAUNCH(bytes, ...)                          \
@@ -250,7 +324,7 @@ slim_status fwd_impl(const Problem& p, int layers, const T* x, const float* omeg
     T* X2 = reinterpret_cast<T*>(w.xin[1]);
     T* Y = reinterpret_cast<T*>(w.yout[0]);
     ST_TRY(gather(x, X, g, p.L, d, a, b, s));
-    STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
+    STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows, d), kRowThreads, 0, s>>>(X, U, d, scale, rows));
     ST_TRY(cudaGetLastError());
     for (int r = 0; r < layers; ++r) {
       float* Sr = S_state + (size_t)r * g.st;
@@ -263,7 +337,7 @@ slim_status fwd_impl(const Problem& p, int layers, const T* x, const float* omeg
                             n ? Sr : nullptr, n ? zr : nullptr, n ? Slr : nullptr,
                             n ? zlr : nullptr, Y, Sr, zr, Slr, zlr, w.inner, g.inner, s));
       const bool next = r + 1 < layers;
-      STACK_LAUNCH((next ? 4 : 3) * sb, k_residual_norm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+      STACK_LAUNCH((next ? 4 : 3) * sb, k_residual_norm<T><<<nrb(rows, d), kRowThreads, 0, s>>>(
                                             X, Y, X2, next ? U : nullptr, d, scale, rows));
       ST_TRY(cudaGetLastError());
       T* t = X;
@@ -302,7 +376,7 @@ slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omeg
     const long long rows = (long long)g.chains * b;
     const double sb = (double)rows * d * g.esz;
     ST_TRY(gather(x, w.xin[0], g, p.L, d, a, b, s));
-    STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+    STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows, d), kRowThreads, 0, s>>>(
                              reinterpret_cast<const T*>(w.xin[0]), U, d, scale, rows));
     ST_TRY(cudaGetLastError());
     // recompute the slice layer by layer, rolling each layer's state back
@@ -331,7 +405,7 @@ slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omeg
                             zlb, Y, w.Ssc, w.zsc, nullptr, nullptr, w.inner, g.inner, s));
       // the next layer's input and its u; the top layer's output is not needed
       if (r + 1 < layers) {
-        STACK_LAUNCH(4 * sb, k_residual_norm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+        STACK_LAUNCH(4 * sb, k_residual_norm<T><<<nrb(rows, d), kRowThreads, 0, s>>>(
                                  X, Y, reinterpret_cast<T*>(w.xin[r + 1]), U, d, scale, rows));
         ST_TRY(cudaGetLastError());
       }
@@ -343,7 +417,7 @@ slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omeg
       const T* X = reinterpret_cast<const T*>(w.xin[r]);
       const float* om = omegas ? omegas + (size_t)r * M * d : nullptr;
       if (r + 1 < layers) {  // the top layer's u is still in place from the recompute
-        STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(X, U, d, scale, rows));
+        STACK_LAUNCH(2 * sb, k_rownorm<T><<<nrb(rows, d), kRowThreads, 0, s>>>(X, U, d, scale, rows));
         ST_TRY(cudaGetLastError());
       }
       ST_CALL(slim_bwd_from(U, U, U, om, w.yout[r], w.dout, w.Se + r * g.st, w.ze + r * g.zt,
@@ -358,7 +432,7 @@ slim_status bwd_impl(const Problem& p, int layers, const T* x, const float* omeg
       }
       const bool first = r == layers - 1;
       STACK_LAUNCH((double)rows * d * (6.0 * g.esz + (first ? 4 : 8)),
-                   k_dx_accum<T><<<nrb(rows), 32 * kRowsPerBlock, 0, s>>>(
+                   k_dx_accum<T><<<nrb(rows, d), kRowThreads, 0, s>>>(
                        w.dx, X, reinterpret_cast<const T*>(w.dq), reinterpret_cast<const T*>(w.dk),
                        reinterpret_cast<const T*>(w.dv), reinterpret_cast<T*>(w.dout), d, scale,
                        rows, first ? 1 : 0));
