@@ -1,4 +1,7 @@
-// fp32-compute (SIMT) path of libslim: every supported (d, M, dtype, feature).
+// fp32-compute path of libslim: every supported (d, M, dtype, feature) that the
+// tcgen05 tile kernels do not take.  Operands and intermediates are fp32; the
+// contractions run as warp MMAs on bf16 pieces of them (k_mma), the feature
+// map and the scans on the FP32 pipe.
 //
 // One slice of Algorithm 1 at a time.  Inside a slice the rows are cut into
 // tiles of T rows and every step is a small batched contraction over
@@ -34,8 +37,8 @@
 namespace slim {
 namespace simt {
 
-constexpr int GT = 64;  // output tile of the contraction kernel
-constexpr int GK = 16;  // reduction chunk
+constexpr int GT = 64;  // output tile width of the contraction kernel
+constexpr int GK = 16;  // reduction chunk (one k16 MMA step)
 
 struct Mat {
   const float* p;

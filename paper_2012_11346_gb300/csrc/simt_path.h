@@ -1,4 +1,4 @@
-// fp32-compute (SIMT) path of libslim; see simt_path.cu.
+// fp32-compute path of libslim (fp32 operands, warp-MMA contractions); see simt_path.cu.
 #pragma once
 #include "common.cuh"
 
