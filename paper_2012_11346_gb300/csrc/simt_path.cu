@@ -344,7 +344,10 @@ __global__ void k_omega_prep(const float* __restrict__ omega, int M, int d, floa
   }
 }
 
-template <typename T>
+// R rows per CTA (2R vectors: R queries, then R keys).  One staged chunk of
+// Omega serves all of them, in blocks of 32 vectors; R = 64 when the rows fit
+// (d <= 64), so that the chunk is staged once per 128 vectors, not 32.
+template <typename T, int R>
 __global__ void __launch_bounds__(256) k_prep(
     const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
     const T* __restrict__ dout, const T* __restrict__ out,
@@ -352,11 +355,11 @@ __global__ void __launch_bounds__(256) k_prep(
     int L, int ld, int M, int a, int b, int Cp, int feature, int sides, float inv_sqrt_m,
     float* Xq, float* Xk, float* Vx, float* phiQ, float* phiK, float* dout32, float* rowdot) {
   extern __shared__ __align__(16) float sm[];
-  constexpr int R = 16;            // rows per CTA (q and k -> 32 vectors)
+  static_assert(R % 16 == 0, "vector blocks");
   const int d = 1 << ld;           // d is a power of two (16 .. 128)
   float* omT = sm;                 // [d][kPrepFeat]: a chunk of Omega, transposed
-  float* xs = omT + d * kPrepFeat; // [32][d]
-  float* xn2 = xs + 32 * d;        // [32]
+  float* xs = omT + d * kPrepFeat; // [2R][d]
+  float* xn2 = xs + 2 * R * d;     // [2R]
   const int c = blockIdx.y, r0 = blockIdx.x * R, tid = threadIdx.x;
   const int dp = d + 1;
   const size_t rowbase = (size_t)c * L + a;
@@ -416,8 +419,8 @@ __global__ void __launch_bounds__(256) k_prep(
   }
   // error bound of an fp32 dot product of length d, times a safety factor 2
   const float gamma = 2.f * (float)(d + 2) * 5.9604645e-08f;
-  // The projections x . omega_m, PF features at a time: thread (f, grp) owns
-  // features m0 + 2f and m0 + 2f + 1 of vectors 8 grp .. 8 grp + 7, reading
+  // The projections x . omega_m, 128 features at a time: thread (f, grp) owns
+  // features m0 + 2f and m0 + 2f + 1 of vectors vbase .. vbase + 7, reading
   // four x values per vector as one float4 and two Omega values as one float2
   // (64 FMAs per 12 shared-memory loads).  Each dot product is summed in j
   // order, one fmaf per term.
@@ -430,9 +433,11 @@ __global__ void __launch_bounds__(256) k_prep(
       for (int e = tid; e < d * kPrepFeat / 4; e += 256) dst[e] = src[e];
     }
     __syncthreads();
+    for (int vb = 0; vb < 2 * R / 32; ++vb) {
+    const int vbase = vb * 32 + grp * 8;  // this thread's vectors vbase .. vbase + 7
     // sides: bit 0 the query features, bit 1 the key features (the
     // non-causal sweeps need one side each); vectors 0..R-1 are queries
-    if (!(sides & (grp < 2 ? 1 : 2))) continue;
+    if (!(sides & (vbase < R ? 1 : 2))) continue;
     float acc[8][2];
 #pragma unroll
     for (int vv = 0; vv < 8; ++vv) acc[vv][0] = acc[vv][1] = 0.f;
@@ -443,7 +448,7 @@ __global__ void __launch_bounds__(256) k_prep(
         o[t] = *reinterpret_cast<const float2*>(&omT[(j + t) * kPrepFeat + 2 * f]);
 #pragma unroll
       for (int vv = 0; vv < 8; ++vv) {
-        const float4 x = *reinterpret_cast<const float4*>(&xs[(grp * 8 + vv) * d + j]);
+        const float4 x = *reinterpret_cast<const float4*>(&xs[(vbase + vv) * d + j]);
         acc[vv][0] = fmaf(x.x, o[0].x, acc[vv][0]);
         acc[vv][1] = fmaf(x.x, o[0].y, acc[vv][1]);
         acc[vv][0] = fmaf(x.y, o[1].x, acc[vv][0]);
@@ -459,7 +464,7 @@ __global__ void __launch_bounds__(256) k_prep(
     if (m < M) {
 #pragma unroll
       for (int vv = 0; vv < 8; ++vv) {
-        const int vec = grp * 8 + vv;
+        const int vec = vbase + vv;
         const int rr = vec % R, r = r0 + rr;
         float phi[2] = {0.f, 0.f};
         if (r < b) {
@@ -492,6 +497,7 @@ __global__ void __launch_bounds__(256) k_prep(
         float* dst = (vec < R) ? phiQ : phiK;
         *reinterpret_cast<float2*>(&dst[((size_t)c * Cp + r) * M + m]) = make_float2(phi[0], phi[1]);
       }
+    }
     }
   }
 }
@@ -764,24 +770,30 @@ cudaError_t launch_prep(cudaStream_t s, const Problem& p, const Geo& g, const Ws
                         const void* q, const void* k, const void* v, const void* dout,
                         const void* out, const float* omega, int a, int b, bool bwd,
                         int sides = 3) {
-  const size_t smem = (g.d * kPrepFeat + 32 * g.d + 32) * sizeof(float);
+  // 64 rows per CTA where they fit (d <= 64, whole blocks of the slice buffer)
+  const bool wide = g.d <= 64 && g.Cp % 64 == 0;
+  const int R = wide ? 64 : 16;
+  const size_t smem = (g.d * kPrepFeat + 2 * R * g.d + 2 * R) * sizeof(float);
   static bool attr_set[kMaxDevices] = {};  // per dtype instantiation and device
   bool* set = device_flag(attr_set);
   if (set == nullptr) return cudaErrorInvalidDevice;
   if (!*set) {
-    cudaError_t e = cudaFuncSetAttribute(k_prep<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_prep<T, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          96 * 1024);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k_prep<T, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
     if (e != cudaSuccess) return e;
     *set = true;
   }
-  dim3 grid(g.Cp / 16, g.chains);
+  dim3 grid(g.Cp / R, g.chains);
   const float inv_sqrt_m = (float)(1.0 / sqrt((double)g.M));
   const double rows = (double)g.chains * b;
   int ld = 0;
   while ((1 << ld) < g.d) ++ld;
   prof::Scope ps(prof::K_PREP, s, (sides == 3 ? 4.0 : 2.0) * rows * g.d * g.M,
                  rows * g.d * sizeof(T) * (bwd ? 5.0 : 3.0));
-  k_prep<T><<<grid, 256, smem, s>>>(
+  auto kern = wide ? k_prep<T, 64> : k_prep<T, 16>;
+  kern<<<grid, 256, smem, s>>>(
       (const T*)q, (const T*)k, (const T*)v, bwd ? (const T*)dout : nullptr,
       bwd ? (const T*)out : nullptr, w.omT, w.omn, p.L, ld, g.M, a, b, g.Cp,
       (int)p.feature, sides, inv_sqrt_m, w.Xq, w.Xk, w.Vx, w.phiQ, w.phiK, bwd ? w.dout32 : nullptr,
